@@ -1,0 +1,191 @@
+"""fp64 CPU oracle of the ResBM boundary bottleneck -- TEST INFRASTRUCTURE.
+
+Only tests/, __graft_entry__.smoke() and bench.py's CPU-baseline / reference leg import this
+package. The product path never does; it shares no code with it.
+
+Each function converts its inputs to C-contiguous float64 (exact for bf16 and fp32 values),
+calls the plain C implementation in resbm_oracle.c and returns float64 numpy arrays.
+Citations (sections and equations of the ResBM paper):
+  pid / rect_identity ........ Sec. 3.3, Eq. rect_identity_definition and Eq. Pid_definition
+  encode_fwd / decode_fwd .... Sec. 3.2 (two linear layers with a nonlinearity; placement
+                               across the boundary; identity path) and
+                               Eq. generalized_transformer_equation
+  decode_bwd / encode_bwd .... the chain rule of the two forward functions
+"""
+import ctypes
+import os
+
+import numpy as np
+
+from . import build as _build
+
+ACT_SILU, ACT_GELU_TANH, ACT_IDENTITY = 0, 1, 2
+ACTS = {"silu": ACT_SILU, "gelu_tanh": ACT_GELU_TANH, "identity": ACT_IDENTITY}
+
+_lib = None
+_dp = ctypes.POINTER(ctypes.c_double)
+_i64 = ctypes.c_int64
+
+
+def _load(path=None):
+    lib = ctypes.CDLL(path or _build.build())
+    lib.oracle_max_threads.restype = ctypes.c_int
+    lib.oracle_act.restype = ctypes.c_double
+    lib.oracle_act.argtypes = [ctypes.c_int, ctypes.c_double]
+    lib.oracle_dact.restype = ctypes.c_double
+    lib.oracle_dact.argtypes = [ctypes.c_int, ctypes.c_double]
+    lib.oracle_rect_identity.argtypes = [_i64, _i64, _dp]
+    lib.oracle_pid.restype = ctypes.c_int
+    lib.oracle_pid.argtypes = [_i64, _i64, _i64, _dp, _dp]
+    lib.oracle_encode_fwd.restype = ctypes.c_int
+    lib.oracle_encode_fwd.argtypes = [_i64] * 4 + [ctypes.c_int] + [_dp] * 6
+    lib.oracle_decode_fwd.restype = ctypes.c_int
+    lib.oracle_decode_fwd.argtypes = [_i64] * 4 + [ctypes.c_int] * 2 + [_dp] * 4
+    lib.oracle_decode_bwd.restype = ctypes.c_int
+    lib.oracle_decode_bwd.argtypes = [_i64] * 4 + [ctypes.c_int] * 2 + [_dp] * 7
+    lib.oracle_encode_bwd.restype = ctypes.c_int
+    lib.oracle_encode_bwd.argtypes = [_i64] * 4 + [ctypes.c_int] + [_dp] * 8
+    return lib
+
+
+def lib():
+    global _lib
+    if _lib is None:
+        _lib = _load()
+    return _lib
+
+
+class Oracle:
+    """The oracle bound to one compiled library (the default one, or a test variant)."""
+
+    def __init__(self, path=None):
+        self._l = _load(path) if path else lib()
+
+    # -- helpers ---------------------------------------------------------------------------
+    @staticmethod
+    def _in(a, shape):
+        a = np.ascontiguousarray(np.asarray(a, dtype=np.float64))
+        if a.shape != tuple(shape):
+            raise ValueError("expected shape %s, got %s" % (tuple(shape), a.shape))
+        return a
+
+    @staticmethod
+    def _p(a):
+        return None if a is None else a.ctypes.data_as(_dp)
+
+    @staticmethod
+    def _act(act):
+        return ACTS[act] if isinstance(act, str) else int(act)
+
+    def max_threads(self):
+        return int(self._l.oracle_max_threads())
+
+    # -- Sec. 3.3 ---------------------------------------------------------------------------
+    def act(self, act, x):
+        return self._l.oracle_act(self._act(act), float(x))
+
+    def dact(self, act, x):
+        return self._l.oracle_dact(self._act(act), float(x))
+
+    def rect_identity(self, c, C):
+        out = np.empty((c, C), np.float64)
+        self._l.oracle_rect_identity(c, C, self._p(out))
+        return out
+
+    def pid(self, x, C):
+        x = np.ascontiguousarray(np.asarray(x, dtype=np.float64))
+        L, c = x.shape
+        y = np.empty((L, C), np.float64)
+        if self._l.oracle_pid(L, c, C, self._p(x), self._p(y)) != 0:
+            raise MemoryError("oracle_pid")
+        return y
+
+    # -- Sec. 3.2 forward -------------------------------------------------------------------
+    def encode_fwd(self, X, F, We1, We2, act="silu"):
+        """Returns (B, P): B = X . I_{d x r} + phi(F . We1) . We2, P = F . We1."""
+        F = np.asarray(F)
+        T, d = F.shape
+        m, r = np.asarray(We2).shape
+        X = self._in(X, (T, d)); F = self._in(F, (T, d))
+        We1 = self._in(We1, (d, m)); We2 = self._in(We2, (m, r))
+        B = np.empty((T, r)); P = np.empty((T, m))
+        rc = self._l.oracle_encode_fwd(T, d, r, m, self._act(act), self._p(X), self._p(F),
+                                       self._p(We1), self._p(We2), self._p(B), self._p(P))
+        if rc != 0:
+            raise MemoryError("oracle_encode_fwd")
+        return B, P
+
+    def decode_fwd(self, B, Wd1, Wd2, act="silu", merge=1):
+        """Returns Y = [merge] B . I_{r x d} + phi(B . Wd1) . Wd2."""
+        B = np.asarray(B)
+        T, r = B.shape
+        m, d = np.asarray(Wd2).shape
+        B = self._in(B, (T, r)); Wd1 = self._in(Wd1, (r, m)); Wd2 = self._in(Wd2, (m, d))
+        Y = np.empty((T, d))
+        rc = self._l.oracle_decode_fwd(T, d, r, m, self._act(act), int(merge), self._p(B),
+                                       self._p(Wd1), self._p(Wd2), self._p(Y))
+        if rc != 0:
+            raise MemoryError("oracle_decode_fwd")
+        return Y
+
+    # -- chain rule -------------------------------------------------------------------------
+    def decode_bwd(self, dY, B, Wd1, Wd2, act="silu", merge=1):
+        """Returns (dB, dWd1, dWd2) for the upstream gradient dY of decode_fwd's Y."""
+        B = np.asarray(B)
+        T, r = B.shape
+        m, d = np.asarray(Wd2).shape
+        dY = self._in(dY, (T, d)); B = self._in(B, (T, r))
+        Wd1 = self._in(Wd1, (r, m)); Wd2 = self._in(Wd2, (m, d))
+        dB = np.empty((T, r)); dWd1 = np.empty((r, m)); dWd2 = np.empty((m, d))
+        rc = self._l.oracle_decode_bwd(T, d, r, m, self._act(act), int(merge), self._p(dY),
+                                       self._p(B), self._p(Wd1), self._p(Wd2), self._p(dB),
+                                       self._p(dWd1), self._p(dWd2))
+        if rc != 0:
+            raise MemoryError("oracle_decode_bwd")
+        return dB, dWd1, dWd2
+
+    def encode_bwd(self, dB, F, We1, We2, act="silu", want_dX=True):
+        """Returns (dF, dX, dWe1, dWe2) for the upstream gradient dB of encode_fwd's B.
+
+        dX is the full T x d gradient of X (dB in the first r columns, zeros after) or None.
+        """
+        F = np.asarray(F)
+        T, d = F.shape
+        m, r = np.asarray(We2).shape
+        dB = self._in(dB, (T, r)); F = self._in(F, (T, d))
+        We1 = self._in(We1, (d, m)); We2 = self._in(We2, (m, r))
+        dF = np.empty((T, d)); dX = np.empty((T, d)) if want_dX else None
+        dWe1 = np.empty((d, m)); dWe2 = np.empty((m, r))
+        rc = self._l.oracle_encode_bwd(T, d, r, m, self._act(act), self._p(dB), self._p(F),
+                                       self._p(We1), self._p(We2), self._p(dF), self._p(dX),
+                                       self._p(dWe1), self._p(dWe2))
+        if rc != 0:
+            raise MemoryError("oracle_encode_bwd")
+        return dF, dX, dWe1, dWe2
+
+    def boundary_step(self, X, F, dY, We1, We2, Wd1, Wd2, act="silu", merge=1):
+        """One boundary forward + backward: the four functions above chained, B handed over."""
+        B, P = self.encode_fwd(X, F, We1, We2, act)
+        Y = self.decode_fwd(B, Wd1, Wd2, act, merge)
+        dB, dWd1, dWd2 = self.decode_bwd(dY, B, Wd1, Wd2, act, merge)
+        dF, dX, dWe1, dWe2 = self.encode_bwd(dB, F, We1, We2, act)
+        return dict(B=B, P=P, Y=Y, dB=dB, dF=dF, dX=dX, dWe1=dWe1, dWe2=dWe2,
+                    dWd1=dWd1, dWd2=dWd2)
+
+
+_default = None
+
+
+def default():
+    global _default
+    if _default is None:
+        _default = Oracle()
+    return _default
+
+
+def __getattr__(name):
+    # module-level shortcuts: oracle.encode_fwd(...) etc.
+    if name in ("act", "dact", "rect_identity", "pid", "encode_fwd", "decode_fwd",
+                "decode_bwd", "encode_bwd", "boundary_step", "max_threads"):
+        return getattr(default(), name)
+    raise AttributeError(name)

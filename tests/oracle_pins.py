@@ -1,0 +1,250 @@
+"""Pins of the fp64 oracle to facts outside the oracle itself.
+
+Each pin takes an oracle instance (`oracle.Oracle`) and raises AssertionError when the oracle
+disagrees with what the ResBM paper or plain mathematics fixes. test_oracle_pins.py runs them
+on the real oracle; test_oracle_mutants.py runs them on copies of the oracle with a planted
+mistake and checks that at least one pin catches each mistake.
+"""
+import json
+import math
+import os
+
+import numpy as np
+
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+ACTS = ("silu", "gelu_tanh", "identity")
+
+
+def _rand(shape, seed, scale=1.0):
+    return np.random.default_rng(seed).standard_normal(shape) * scale
+
+
+def _weights(d, r, m, seed):
+    return dict(We1=_rand((d, m), seed + 1, 1 / math.sqrt(d)),
+                We2=_rand((m, r), seed + 2, 1 / math.sqrt(m)),
+                Wd1=_rand((r, m), seed + 3, 1 / math.sqrt(r)),
+                Wd2=_rand((m, d), seed + 4, 1 / math.sqrt(m)))
+
+
+# ---------------------------------------------------------------------------------------------
+# Sec. 3.3: rectangular identity, P^id and their composition.
+# ---------------------------------------------------------------------------------------------
+
+def pin_rect_identity_is_numpy_eye(o):
+    """Eq. rect_identity_definition equals numpy's rectangular eye for c<C, c>C, c=C."""
+    for c, C in [(3, 5), (5, 3), (4, 4), (1, 7), (7, 1)]:
+        assert np.array_equal(o.rect_identity(c, C), np.eye(c, C)), (c, C)
+
+
+def pin_pid_truncate_pad_identity(o):
+    """Eq. Pid bullets: c<C appends C-c zero columns, c>C drops the last c-C, c=C is I_c."""
+    x = _rand((4, 6), 11)
+    y = o.pid(x, 9)
+    assert y.shape == (4, 9)
+    assert np.array_equal(y[:, :6], x) and not np.any(y[:, 6:])
+    assert np.array_equal(o.pid(x, 2), x[:, :2])
+    assert np.array_equal(o.pid(x, 6), x)
+
+
+def pin_composition_rank_min(o):
+    """Sec. 3.3: a chain of rectangular identities multiplies to the c0 x cD rectangular
+    identity restricted to rank k = min(c0..cD); it is exactly I_{c0 x cD} whenever every
+    middle dimension is at least min(c0, cD) (the d -> r -> d round trip is diag(1_r, 0))."""
+    chains = [(6, 9, 7, 4), (4, 6, 8), (8, 3, 8), (5, 2, 9, 5), (3, 3, 3), (16, 4, 16, 4)]
+    for ch in chains:
+        prod = np.eye(ch[0])
+        for a, b in zip(ch[:-1], ch[1:]):
+            prod = prod @ o.rect_identity(a, b)
+        k = min(ch)
+        expect = np.zeros((ch[0], ch[-1]))
+        expect[np.arange(k), np.arange(k)] = 1.0
+        assert np.array_equal(prod, expect), ch
+        assert np.linalg.matrix_rank(prod) == k
+        if min(ch[1:-1]) >= min(ch[0], ch[-1]):
+            assert np.array_equal(prod, np.eye(ch[0], ch[-1])), ch
+
+
+# ---------------------------------------------------------------------------------------------
+# The nonlinearity.
+# ---------------------------------------------------------------------------------------------
+
+def pin_act_special_values(o):
+    """phi(0) = 0; phi(x) - phi(-x) = x for SiLU and GELU(tanh) (both are x * (an even
+    function's complement)); phi -> x for large x and -> 0 for large -x; identity is x."""
+    for act in ("silu", "gelu_tanh"):
+        assert o.act(act, 0.0) == 0.0
+        for x in (0.3, 1.7, 4.2, 9.0):
+            assert abs(o.act(act, x) - o.act(act, -x) - x) <= 1e-14 * max(1.0, x)
+        assert abs(o.act(act, 40.0) - 40.0) < 1e-12
+        assert abs(o.act(act, -40.0)) < 1e-12
+    for x in (-3.0, 0.0, 2.5):
+        assert o.act("identity", x) == x and o.dact("identity", x) == 1.0
+
+
+def pin_silu_is_x_sigmoid(o):
+    """SiLU(x) = x * sigmoid(x), sigmoid from scipy's expit."""
+    from scipy.special import expit
+    for x in np.linspace(-12, 12, 49):
+        assert abs(o.act("silu", x) - x * expit(x)) <= 1e-15 * max(1.0, abs(x))
+
+
+def pin_gelu_tanh_close_to_exact_gelu(o):
+    """The tanh form of GELU stays within 1e-3 of x * Phi(x) (Phi from math.erf)."""
+    for x in np.linspace(-8, 8, 161):
+        exact = 0.5 * x * (1.0 + math.erf(x / math.sqrt(2.0)))
+        assert abs(o.act("gelu_tanh", x) - exact) < 1e-3, x
+
+
+def pin_dact_matches_finite_difference(o):
+    h = 1e-5
+    for act in ACTS:
+        for x in np.linspace(-7, 7, 57):
+            fd = (o.act(act, x + h) - o.act(act, x - h)) / (2 * h)
+            assert abs(fd - o.dact(act, x)) <= 1e-8 * max(1.0, abs(x)), (act, x)
+
+
+# ---------------------------------------------------------------------------------------------
+# The identity path alone (learned contributions zeroed), Sec. 3.2-3.3.
+# ---------------------------------------------------------------------------------------------
+
+def pin_zero_weights_leave_identity_path(o):
+    T, d, r, m = 5, 12, 4, 3
+    X, F, dY = _rand((T, d), 21), _rand((T, d), 22), _rand((T, d), 23)
+    w = _weights(d, r, m, 30)
+    z_e2, z_d2 = np.zeros((m, r)), np.zeros((m, d))
+    for act in ACTS:
+        B, _ = o.encode_fwd(X, F, w["We1"], z_e2, act)
+        assert np.array_equal(B, X[:, :r])                        # B = X . I_{d x r}
+        Bw, _ = o.encode_fwd(X, F, w["We1"], w["We2"], act)
+        Y = o.decode_fwd(Bw, w["Wd1"], z_d2, act, merge=1)
+        assert np.array_equal(Y[:, :r], Bw) and not np.any(Y[:, r:])  # Y = B . I_{r x d}
+        assert not np.any(o.decode_fwd(Bw, w["Wd1"], z_d2, act, merge=0))
+        dB, dWd1, _ = o.decode_bwd(dY, Bw, w["Wd1"], z_d2, act, merge=1)
+        assert np.array_equal(dB, dY[:, :r]) and not np.any(dWd1)
+        dF, dX, _, dWe2 = o.encode_bwd(dB, F, w["We1"], z_e2, act)
+        assert not np.any(dF)
+        assert np.array_equal(dX[:, :r], dB) and not np.any(dX[:, r:])
+    # c = C: with no compression and zero learned weights the block is the vanilla residual
+    Xs = _rand((T, 6), 24)
+    ws = _weights(6, 6, 2, 40)
+    B, _ = o.encode_fwd(Xs, Xs, ws["We1"], np.zeros((2, 6)), "silu")
+    assert np.array_equal(o.decode_fwd(B, ws["Wd1"], np.zeros((2, 6)), "silu", 1), Xs)
+
+
+# ---------------------------------------------------------------------------------------------
+# The textbook special case: phi = identity makes encoder and decoder two plain matmuls.
+# ---------------------------------------------------------------------------------------------
+
+def pin_identity_act_is_two_matmuls(o):
+    T, d, r, m = 6, 10, 3, 4
+    X, F, dY = _rand((T, d), 51), _rand((T, d), 52), _rand((T, d), 53)
+    w = _weights(d, r, m, 60)
+    We1, We2, Wd1, Wd2 = w["We1"], w["We2"], w["Wd1"], w["Wd2"]
+    tol = dict(rtol=1e-12, atol=1e-12)
+    B, P = o.encode_fwd(X, F, We1, We2, "identity")
+    np.testing.assert_allclose(P, np.matmul(F, We1), **tol)
+    np.testing.assert_allclose(B, X[:, :r] + np.matmul(np.matmul(F, We1), We2), **tol)
+    for merge in (0, 1):
+        Y = o.decode_fwd(B, Wd1, Wd2, "identity", merge)
+        pad = np.hstack([B, np.zeros((T, d - r))]) * merge
+        np.testing.assert_allclose(Y, pad + B @ Wd1 @ Wd2, **tol)
+        dB, dWd1, dWd2 = o.decode_bwd(dY, B, Wd1, Wd2, "identity", merge)
+        np.testing.assert_allclose(dB, merge * dY[:, :r] + dY @ Wd2.T @ Wd1.T, **tol)
+        np.testing.assert_allclose(dWd2, (B @ Wd1).T @ dY, **tol)
+        np.testing.assert_allclose(dWd1, B.T @ (dY @ Wd2.T), **tol)
+    dBup = _rand((T, r), 54)
+    dF, dX, dWe1, dWe2 = o.encode_bwd(dBup, F, We1, We2, "identity")
+    np.testing.assert_allclose(dF, dBup @ We2.T @ We1.T, **tol)
+    np.testing.assert_allclose(dWe1, F.T @ (dBup @ We2.T), **tol)
+    np.testing.assert_allclose(dWe2, (F @ We1).T @ dBup, **tol)
+    np.testing.assert_allclose(dX, np.hstack([dBup, np.zeros((T, d - r))]), **tol)
+
+
+# ---------------------------------------------------------------------------------------------
+# Brute force: central finite differences of the scalar sum(dY * Y) through both sides.
+# ---------------------------------------------------------------------------------------------
+
+def _fd_check(o, T, d, r, m, act, merge, seed):
+    X, F, dY = _rand((T, d), seed), _rand((T, d), seed + 1), _rand((T, d), seed + 2)
+    w = _weights(d, r, m, seed + 10)
+    params = dict(X=X, F=F, **w)
+
+    def loss(p):
+        B, _ = o.encode_fwd(p["X"], p["F"], p["We1"], p["We2"], act)
+        return float(np.sum(dY * o.decode_fwd(B, p["Wd1"], p["Wd2"], act, merge)))
+
+    B, _ = o.encode_fwd(X, F, w["We1"], w["We2"], act)
+    dB, dWd1, dWd2 = o.decode_bwd(dY, B, w["Wd1"], w["Wd2"], act, merge)
+    dF, dX, dWe1, dWe2 = o.encode_bwd(dB, F, w["We1"], w["We2"], act)
+    grads = dict(X=dX, F=dF, We1=dWe1, We2=dWe2, Wd1=dWd1, Wd2=dWd2)
+    for name, g in grads.items():
+        assert g.shape == params[name].shape, name
+        scale = max(1.0, float(np.max(np.abs(g))))
+        for idx in np.ndindex(*g.shape):
+            p = {k: v.copy() for k, v in params.items()}
+            x0 = p[name][idx]
+            h = 1e-6 * max(1.0, abs(x0))
+            p[name][idx] = x0 + h
+            lp = loss(p)
+            p[name][idx] = x0 - h
+            lm = loss(p)
+            fd = (lp - lm) / (2 * h)
+            assert abs(fd - g[idx]) <= 1e-7 * scale, (act, merge, name, idx, fd, g[idx])
+
+
+def pin_gradients_match_finite_differences(o):
+    # distinct T, d, r, m so that a transposed operand cannot go unnoticed
+    for act in ACTS:
+        for merge in (1, 0):
+            _fd_check(o, T=3, d=7, r=2, m=3, act=act, merge=merge, seed=100)
+    _fd_check(o, T=2, d=5, r=4, m=2, act="silu", merge=1, seed=200)   # r > m
+    _fd_check(o, T=2, d=3, r=3, m=2, act="silu", merge=1, seed=300)   # r = d (c = C)
+
+
+def pin_weight_grads_sum_over_tokens(o):
+    """The weight gradients are sums over tokens: the gradient of a batch is the sum of the
+    gradients of its two halves; the per-token outputs of a row do not depend on the others."""
+    T, d, r, m = 8, 9, 2, 3
+    X, F, dY = _rand((T, d), 71), _rand((T, d), 72), _rand((T, d), 73)
+    w = _weights(d, r, m, 80)
+    B, _ = o.encode_fwd(X, F, w["We1"], w["We2"], "silu")
+    full = o.decode_bwd(dY, B, w["Wd1"], w["Wd2"], "silu", 1)
+    lo = o.decode_bwd(dY[:3], B[:3], w["Wd1"], w["Wd2"], "silu", 1)
+    hi = o.decode_bwd(dY[3:], B[3:], w["Wd1"], w["Wd2"], "silu", 1)
+    np.testing.assert_array_equal(full[0], np.vstack([lo[0], hi[0]]))
+    for k in (1, 2):
+        np.testing.assert_allclose(full[k], lo[k] + hi[k], rtol=1e-12, atol=1e-12)
+    efull = o.encode_bwd(full[0], F, w["We1"], w["We2"], "silu")
+    elo = o.encode_bwd(full[0][:5], F[:5], w["We1"], w["We2"], "silu")
+    ehi = o.encode_bwd(full[0][5:], F[5:], w["We1"], w["We2"], "silu")
+    for k in (0, 1):
+        np.testing.assert_array_equal(efull[k], np.vstack([elo[k], ehi[k]]))
+    for k in (2, 3):
+        np.testing.assert_allclose(efull[k], elo[k] + ehi[k], rtol=1e-12, atol=1e-12)
+    Bsub, _ = o.encode_fwd(X[[6, 1]], F[[6, 1]], w["We1"], w["We2"], "silu")
+    np.testing.assert_array_equal(Bsub, B[[6, 1]])
+
+
+# ---------------------------------------------------------------------------------------------
+# Appendix A.3 / Sec. 4.1: what crosses the boundary.
+# ---------------------------------------------------------------------------------------------
+
+def pin_boundary_bytes(o):
+    with open(os.path.join(GOLDEN, "appendix_a3_bytes.json")) as f:
+        g = json.load(f)["facts"]
+    T = g["microbatch"] * g["tokens_per_boundary_message"]
+    d, r, m, e = g["hidden_dim"], g["bottleneck_dim_128x"], g["bottleneck_dim_128x"], g["bytes_per_element_bf16"]
+    assert d // r == g["compression_rate"]
+    X = _rand((T, d), 91)
+    w = _weights(d, r, m, 92)
+    B, _ = o.encode_fwd(X, X, w["We1"], w["We2"], "silu")
+    assert X.size * e == g["uncompressed_boundary_bytes"]
+    assert B.shape == (T, r) and B.size * e == g["compressed_boundary_bytes"]
+    dB, _, _ = o.decode_bwd(X, B, w["Wd1"], w["Wd2"], "silu", 1)   # the gradient sent back
+    assert dB.shape == (T, r)
+    per_step = g["stage_boundaries"] * g["directions"]
+    assert per_step * X.size * e == g["uncompressed_step_bytes"]
+    assert per_step * (B.size + dB.size) // 2 * e == g["compressed_step_bytes"]
+
+
+PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_")]

@@ -1,0 +1,54 @@
+"""Planted mistakes in a copy of the oracle must each fail at least one pin (no GPU).
+
+Every mutant is a one-line textual change to a temporary copy of oracle/resbm_oracle.c (the
+committed oracle is never touched); each keeps all memory accesses in bounds.
+"""
+import os
+import tempfile
+
+import pytest
+
+import oracle
+from oracle import build as obuild
+from oracle_pins import PINS
+
+MUTANTS = {
+    "dropped_send_skip": ("B[i] = S[i] + E[i];", "B[i] = E[i];"),
+    "wrong_sign_receive_merge": ("Y[i] = merge ? R[i] + D[i] : D[i];",
+                                 "Y[i] = merge ? R[i] - D[i] : D[i];"),
+    "silu_derivative_sign": ("return s + x * s * (1.0 - s);", "return s + x * s * (1.0 + s);"),
+    "dact_at_wrong_tensor": ("dQ[i] = dG[i] * oracle_dact(act, Q[i]);",
+                             "dQ[i] = dG[i] * oracle_dact(act, G[i]);"),
+    "missing_dact_in_encoder": ("dP[i] = dA[i] * oracle_dact(act, P[i]);", "dP[i] = dA[i];"),
+    "dropped_skip_gradient": ("        if (merge) {\n            rc = pid_backward",
+                              "        if (0) {\n            rc = pid_backward"),
+    "identity_on_antidiagonal": ("I[i * C + j] = (i == j) ? 1.0 : 0.0;",
+                                 "I[i * C + j] = (i == C - 1 - j) ? 1.0 : 0.0;"),
+    "gelu_constant": ("kGeluC = 0.044715;", "kGeluC = 0.44715;"),
+    "dropped_first_token_in_reduction": (
+        "        for (int64_t k = 0; k < K; ++k) {\n            const double a = A[k * M + i];",
+        "        for (int64_t k = 1; k < K; ++k) {\n            const double a = A[k * M + i];"),
+    "transposed_operand_in_nt_product": ("acc += A[i * K + k] * B[j * K + k];",
+                                         "acc += A[i * K + k] * B[k * N + j];"),
+    "encoder_reads_decoder_order": ("mm_nn(T, r, m, A, We2, E);", "mm_nn(T, r, m, P, We2, E);"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_planted_mistake_is_caught(name):
+    find, repl = MUTANTS[name]
+    src = open(obuild.SRC).read()
+    assert src.count(find) == 1, "mutation anchor not unique: %s" % name
+    with tempfile.TemporaryDirectory() as tmp:
+        path = os.path.join(tmp, "mutant.c")
+        with open(path, "w") as f:
+            f.write(src.replace(find, repl))
+        lib = obuild.build(src=path, out=os.path.join(tmp, "libmutant.so"))
+        o = oracle.Oracle(lib)
+        caught = []
+        for pin in PINS:
+            try:
+                pin(o)
+            except AssertionError:
+                caught.append(pin.__name__)
+        assert caught, "no pin caught the planted mistake %s" % name
