@@ -1,0 +1,176 @@
+/*
+ * resbm.h -- C ABI of the ResBM boundary bottleneck on one GB300 (sm_103a).
+ *
+ * ResBM (Residual Bottleneck Models, arXiv 2604.11947) places an autoencoder across every
+ * pipeline-stage boundary (Sec. 3.2): the encoder E at the end of block l compresses the
+ * feed-forward output z_l (T x d) to the boundary tensor b_l (T x r, r < d), which is the only
+ * tensor that crosses the boundary; the decoder D at the start of block l+1 expands it back
+ * to T x d. Both are "two linear layers with a non-linearity applied between them" (Sec. 3.2).
+ * The identity path survives the change of width through the fixed projection
+ * P^id(x) = x . I_{c x C} (Eq. rect_identity_definition, Eq. Pid_definition): truncation to
+ * the first r columns on the sending side, zero padding on the receiving side, merged by the
+ * generalized residual update x_{l+1} = x_l P^id + F(x_l) (Eq. generalized_transformer_equation).
+ *
+ * Notation (paper -> this header): L*batch -> T tokens, H -> d, h -> r, x_l^Attn -> X,
+ * z_l -> F, b_l -> B; m is the hidden width between the two linear layers (the paper does not
+ * fix it; m = r in the shipped workloads). All matrices are dense, row-major, in the paper's
+ * "x . W" orientation:
+ *     X, F, Y, dY, dF, dX : T x d        B, dB : T x r        P : T x m (fp32)
+ *     We1 : d x m    We2 : m x r    Wd1 : r x m    Wd2 : m x d
+ *
+ * Computed (phi = the activation chosen in the descriptor):
+ *   encode fwd   B  = X . I_{d x r} + phi(F . We1) . We2             P = F . We1 (saved, fp32)
+ *   decode fwd   Y  = [merge] B . I_{r x d} + phi(B . Wd1) . Wd2
+ *   decode bwd   dB = [merge] dY . I_{r x d}^T + ((dY . Wd2^T) * phi'(Q)) . Wd1^T,  Q = B . Wd1
+ *                dWd2 = phi(Q)^T . dY        dWd1 = B^T . ((dY . Wd2^T) * phi'(Q))
+ *   encode bwd   dP = (dB . We2^T) * phi'(P);  dF = dP . We1^T;  dX[:, :r] += dB
+ *                dWe1 = F^T . dP            dWe2 = phi(P)^T . dB
+ *
+ * Conventions shared by every entry point:
+ *   - Every tensor pointer is DEVICE memory owned by the caller (for example a torch tensor's
+ *     storage). The library allocates nothing, frees nothing and never synchronizes: work is
+ *     enqueued on `stream` (a cudaStream_t; NULL is the legacy default stream) and the call
+ *     returns. Inputs must stay alive and unmodified until the enqueued work has finished.
+ *   - I/O tensors and weights have the descriptor's dtype (fp32 or bf16); P and every weight
+ *     gradient are fp32. Arithmetic accumulates in fp32. For bf16 the intermediates that feed a
+ *     tensor-core product are rounded to bf16; outputs are rounded once, to nearest even.
+ *   - Weight gradients are OVERWRITTEN (they are complete sums over the T tokens). dX is
+ *     ACCUMULATED: dB is added into its first r columns and its other columns are not touched.
+ *   - Arguments are validated before anything is enqueued; a failure returns a status code and
+ *     enqueues nothing. The library never aborts or exits. A CUDA error at launch time returns
+ *     RESBM_ERR_CUDA (resbm_last_cuda_error() gives the cudaError_t value).
+ *   - Outputs must not overlap inputs (X may alias F: both are only read).
+ *   - Results are deterministic: the same inputs, descriptor and device give the same bits.
+ *   - T = 0 is valid: nothing is read, weight gradients are set to zero.
+ *   - The scratch memory `ws` (device, >= resbm_workspace_bytes(...) bytes, 256-byte aligned)
+ *     belongs to the call until its work finishes; its contents on entry do not matter.
+ */
+#ifndef RESBM_H
+#define RESBM_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define RESBM_API __attribute__((visibility("default")))
+#else
+#define RESBM_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    RESBM_OK = 0,
+    RESBM_ERR_INVALID_ARG = 1,   /* null/misaligned pointer, bad size or enum, overlap */
+    RESBM_ERR_UNSUPPORTED = 2,   /* valid request this build cannot run */
+    RESBM_ERR_WORKSPACE = 3,     /* ws is NULL or smaller than resbm_workspace_bytes() */
+    RESBM_ERR_CUDA = 4           /* a CUDA runtime call or launch failed */
+} resbm_status;
+
+typedef enum { RESBM_F32 = 0, RESBM_BF16 = 1 } resbm_dtype;
+
+/* phi of Sec. 3.2 (the paper does not name it): SiLU x*sigmoid(x) (default),
+ * GELU tanh form 0.5x(1+tanh(sqrt(2/pi)(x+0.044715x^3))), or identity. */
+typedef enum { RESBM_ACT_SILU = 0, RESBM_ACT_GELU_TANH = 1, RESBM_ACT_IDENTITY = 2 } resbm_act;
+
+typedef enum {
+    RESBM_OP_ENCODE_FWD = 0,
+    RESBM_OP_DECODE_FWD = 1,
+    RESBM_OP_DECODE_BWD = 2,
+    RESBM_OP_ENCODE_BWD = 3,
+    RESBM_OP_BOUNDARY_STEP = 4
+} resbm_op;
+
+/* desc.flags bits */
+#define RESBM_FLAG_GENERIC 1u   /* force the portable CUDA-core kernels (no tensor cores) */
+
+typedef struct {
+    int64_t T;               /* tokens (batch * sequence), >= 0                              */
+    int64_t d;               /* residual width H, >= 1                                       */
+    int64_t r;               /* bottleneck width h, 1 <= r <= d (compression d / r)          */
+    int64_t m;               /* hidden width of the two-layer encoder / decoder, >= 1        */
+    int32_t dtype;           /* resbm_dtype of X, F, B, Y, dY, dB, dF, dX and the weights    */
+    int32_t act;             /* resbm_act                                                     */
+    int32_t merge_identity;  /* 1: Y = B . I_{r x d} + D(B);  0: Y = D(B) (the caller adds the
+                                padded skip itself, e.g. after attention)                     */
+    uint32_t flags;          /* RESBM_FLAG_* bits, 0 for the default kernels                 */
+} resbm_desc;
+
+/* Pointers for resbm_boundary_step (all device memory, layouts as above). */
+typedef struct {
+    const void *X, *F, *dY;                 /* inputs, T x d                                  */
+    const void *We1, *We2, *Wd1, *Wd2;      /* weights                                        */
+    void *B;                                /* out: T x r boundary tensor                     */
+    float *P;                               /* out: T x m fp32 F.We1, or NULL (kept in ws)    */
+    void *Y;                                /* out: T x d decoder output                      */
+    void *dB;                               /* out: T x r gradient sent back                  */
+    void *dF;                               /* out: T x d                                     */
+    void *dX;                               /* in/out: T x d, first r columns += dB; or NULL  */
+    float *dWe1, *dWe2, *dWd1, *dWd2;       /* out: fp32 weight gradients                     */
+} resbm_step_args;
+
+/* Library version string, e.g. "resbm 0.1.0 sm_103a". */
+RESBM_API const char *resbm_version(void);
+
+/* Human-readable name of a status code (static storage). */
+RESBM_API const char *resbm_status_string(resbm_status status);
+
+/* The cudaError_t value behind the last RESBM_ERR_CUDA returned on this host thread (0 if none). */
+RESBM_API int resbm_last_cuda_error(void);
+
+/* Number of kernels this library has enqueued in this process so far (all devices, all host
+ * threads): lets a caller account for the GPU work behind a sequence of calls. */
+RESBM_API uint64_t resbm_kernel_launches(void);
+
+/* Scratch bytes that `op` (a resbm_op) needs for `desc`, written to *bytes.
+ * Returns RESBM_ERR_INVALID_ARG for a bad descriptor or op. Does not touch the GPU. */
+RESBM_API resbm_status resbm_workspace_bytes(const resbm_desc *desc, int op, size_t *bytes);
+
+/* Send side, Sec. 3.2 (encoder at the end of block l) with the truncating identity path of
+ * Eq. Pid (c = d > C = r): B = X[:, :r] + phi(F . We1) . We2.
+ *   X   : T x d, only its first r columns are read (x_l^Attn, the skip source)
+ *   F   : T x d (z_l, the feed-forward output); may be the same pointer as X
+ *   B   : T x r out. P_save: T x m fp32 out (F . We1, reused by resbm_encode_bwd) or NULL. */
+RESBM_API resbm_status resbm_encode_fwd(const resbm_desc *desc, const void *X, const void *F,
+                              const void *We1, const void *We2, void *B, float *P_save,
+                              void *ws, size_t ws_bytes, void *stream);
+
+/* Receive side, Sec. 3.2 (decoder at the start of block l+1) with the zero-padding identity
+ * path of Eq. Pid (c = r < C = d): Y = [merge] B . I_{r x d} + phi(B . Wd1) . Wd2.
+ *   B : T x r in.  Y : T x d out. */
+RESBM_API resbm_status resbm_decode_fwd(const resbm_desc *desc, const void *B, const void *Wd1,
+                              const void *Wd2, void *Y, void *ws, size_t ws_bytes,
+                              void *stream);
+
+/* Backward of resbm_decode_fwd for the upstream gradient dY (the compressed gradient dB is
+ * what crosses the boundary backwards, Appendix A.3).
+ *   dY : T x d in.  B : T x r in (the forward input).  dB : T x r out.
+ *   dWd1 : r x m fp32 out.  dWd2 : m x d fp32 out. */
+RESBM_API resbm_status resbm_decode_bwd(const resbm_desc *desc, const void *dY, const void *B,
+                              const void *Wd1, const void *Wd2, void *dB, float *dWd1,
+                              float *dWd2, void *ws, size_t ws_bytes, void *stream);
+
+/* Backward of resbm_encode_fwd for the upstream gradient dB.
+ *   dB : T x r in.  F : T x d in.  P_save : T x m fp32 from resbm_encode_fwd, or NULL
+ *   (then F . We1 is recomputed, which reads F twice).
+ *   dF : T x d out.  dX : T x d in/out, dX[:, :r] += dB (gradient of the truncating identity
+ *   path), or NULL to skip.  dWe1 : d x m fp32 out.  dWe2 : m x r fp32 out. */
+RESBM_API resbm_status resbm_encode_bwd(const resbm_desc *desc, const void *dB, const void *F,
+                              const float *P_save, const void *We1, const void *We2,
+                              void *dF, void *dX, float *dWe1, float *dWe2,
+                              void *ws, size_t ws_bytes, void *stream);
+
+/* One boundary forward and backward on one GPU, the pipeline handoff kept in device memory:
+ * encode_fwd -> decode_fwd -> decode_bwd -> encode_bwd, in that order on `stream`. B produced
+ * by the encoder is what the decoder reads; dB produced by the decoder backward is what the
+ * encoder backward reads. */
+RESBM_API resbm_status resbm_boundary_step(const resbm_desc *desc, const resbm_step_args *args,
+                                 void *ws, size_t ws_bytes, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* RESBM_H */

@@ -1,0 +1,377 @@
+// generic.cu -- the portable CUDA-core path of the ResBM boundary bottleneck.
+//
+// Every product of Sec. 3.2 (and of its chain-rule backward) runs through one tiled FFMA
+// kernel whose operand loaders and epilogue are small functors: the nonlinearity, its
+// derivative, the identity-path add of Eq. generalized_transformer_equation and the rounding
+// to the I/O dtype are folded into loads and stores. It handles every shape and both dtypes
+// and is the fp32 path (fp32 products at full fp32 precision). Weight gradients are split
+// over tokens into fp32 partials that a second kernel sums in a fixed order (deterministic).
+#include "common.cuh"
+#include "internal.h"
+
+namespace resbm {
+namespace {
+
+constexpr int BM = 64, BN = 64, BK = 16, NT = 256;
+
+// ---- operand loaders: element (row, col) of a logical matrix as fp32 -----------------------
+template <typename T> struct LdRM {  // M[row][col] = p[row * ld + col]
+    const T *p; int64_t ld;
+    __device__ float operator()(int64_t i, int64_t k) const { return to_f32(p[i * ld + k]); }
+};
+template <typename T> struct LdT {   // M[row][col] = p[col * ld + row] (transposed view)
+    const T *p; int64_t ld;
+    __device__ float operator()(int64_t i, int64_t k) const { return to_f32(p[k * ld + i]); }
+};
+struct LdAct {                       // phi(p[row][col])
+    const float *p; int64_t ld; int act;
+    __device__ float operator()(int64_t i, int64_t k) const { return act_f(act, p[i * ld + k]); }
+};
+struct LdActT {                      // phi(p[col][row])
+    const float *p; int64_t ld; int act;
+    __device__ float operator()(int64_t i, int64_t k) const { return act_f(act, p[k * ld + i]); }
+};
+struct LdDact {                      // g[row][col] * phi'(x[row][col])
+    const float *g; const float *x; int64_t ld; int act;
+    __device__ float operator()(int64_t i, int64_t k) const
+    {
+        return g[i * ld + k] * dact_f(act, x[i * ld + k]);
+    }
+};
+
+// ---- epilogues: ep(row, col, split, acc) ----------------------------------------------------
+struct EpF32 {
+    float *out; int64_t ld; int64_t zstride;
+    __device__ void operator()(int64_t i, int64_t n, int z, float acc) const
+    {
+        out[z * zstride + i * ld + n] = acc;
+    }
+};
+template <typename T> struct EpStore {
+    T *out; int64_t ld;
+    __device__ void operator()(int64_t i, int64_t n, int, float acc) const
+    {
+        out[i * ld + n] = from_f32<T>(acc);
+    }
+};
+template <typename T> struct EpEncB {   // B = X . I_{d x r} + E
+    T *B; const T *X; int64_t r, d;
+    __device__ void operator()(int64_t i, int64_t n, int, float acc) const
+    {
+        B[i * r + n] = from_f32<T>(to_f32(X[i * d + n]) + acc);
+    }
+};
+template <typename T> struct EpDecY {   // Y = [merge] B . I_{r x d} + D
+    T *Y; const T *B; int64_t d, r; int merge;
+    __device__ void operator()(int64_t i, int64_t n, int, float acc) const
+    {
+        const float skip = (merge && n < r) ? to_f32(B[i * r + n]) : 0.0f;
+        Y[i * d + n] = from_f32<T>(skip + acc);
+    }
+};
+template <typename T> struct EpDecDB {  // dB = [merge] dY . I_{r x d}^T + dQ . Wd1^T
+    T *dB; const T *dY; int64_t r, d; int merge;
+    __device__ void operator()(int64_t i, int64_t n, int, float acc) const
+    {
+        const float skip = merge ? to_f32(dY[i * d + n]) : 0.0f;
+        dB[i * r + n] = from_f32<T>(skip + acc);
+    }
+};
+
+// C[M x N] = A[M x K] . B[K x N]; blockIdx.z selects a K range of length kchunk.
+template <class LA, class LB, class EP>
+__global__ void __launch_bounds__(NT) k_gemm(int64_t M, int64_t N, int64_t K, int64_t kchunk,
+                                             LA la, LB lb, EP ep)
+{
+    __shared__ float As[BK][BM + 1];
+    __shared__ float Bs[BK][BN + 1];
+    const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+    const int64_t m0 = (int64_t)blockIdx.x * BM, n0 = (int64_t)blockIdx.y * BN;
+    const int64_t kb0 = (int64_t)blockIdx.z * kchunk;
+    const int64_t kb1 = min(K, kb0 + kchunk);
+    float acc[4][4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] = 0.0f;
+
+    for (int64_t k0 = kb0; k0 < kb1; k0 += BK) {
+        for (int e = tid; e < BM * BK; e += NT) {
+            const int kk = e % BK, mm = e / BK;
+            const int64_t gm = m0 + mm, gk = k0 + kk;
+            As[kk][mm] = (gm < M && gk < kb1) ? la(gm, gk) : 0.0f;
+        }
+        for (int e = tid; e < BN * BK; e += NT) {
+            const int nn = e % BN, kk = e / BN;
+            const int64_t gn = n0 + nn, gk = k0 + kk;
+            Bs[kk][nn] = (gn < N && gk < kb1) ? lb(gk, gn) : 0.0f;
+        }
+        __syncthreads();
+#pragma unroll
+        for (int kk = 0; kk < BK; ++kk) {
+            float a[4], b[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) a[i] = As[kk][ty + 16 * i];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) b[j] = Bs[kk][tx + 16 * j];
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
+        }
+        __syncthreads();
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int64_t gm = m0 + ty + 16 * i, gn = n0 + tx + 16 * j;
+            if (gm < M && gn < N) ep(gm, gn, (int)blockIdx.z, acc[i][j]);
+        }
+}
+
+template <class LA, class LB, class EP>
+cudaError_t gemm(int64_t M, int64_t N, int64_t K, int splits, LA la, LB lb, EP ep,
+                 cudaStream_t s)
+{
+    if (M <= 0 || N <= 0) return cudaSuccess;
+    int64_t kchunk = K;
+    if (splits > 1) kchunk = ((K + splits - 1) / splits + BK - 1) / BK * BK;
+    if (kchunk <= 0) kchunk = BK;
+    const int64_t nz = (K + kchunk - 1) / kchunk;
+    dim3 grid((unsigned)((M + BM - 1) / BM), (unsigned)((N + BN - 1) / BN),
+              (unsigned)(nz > 0 ? nz : 1));
+    k_gemm<<<grid, NT, 0, s>>>(M, N, K, kchunk, la, lb, ep);
+    count_launches(1);
+    return cudaGetLastError();
+}
+
+// out[e] = sum over s = 0, 1, ..., S-1 of part[s * n + e]   (fixed order)
+__global__ void k_reduce_splits(const float *__restrict__ part, int64_t n, int S,
+                                float *__restrict__ out)
+{
+    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n;
+         e += (int64_t)gridDim.x * blockDim.x) {
+        float acc = 0.0f;
+        for (int s = 0; s < S; ++s) acc += part[s * n + e];
+        out[e] = acc;
+    }
+}
+
+// dX[:, :r] += dB  (the gradient of the truncating identity projection)
+template <typename T>
+__global__ void k_dx_accumulate(T *dX, const T *__restrict__ dB, int64_t Tn, int64_t d, int64_t r)
+{
+    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < Tn * r;
+         e += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t t = e / r, j = e - t * r;
+        dX[t * d + j] = from_f32<T>(to_f32(dX[t * d + j]) + to_f32(dB[e]));
+    }
+}
+
+int grid_for(int64_t n, const Ctx &c)
+{
+    int64_t g = (n + 255) / 256;
+    const int64_t cap = (int64_t)c.sm_count * 8;
+    if (g > cap) g = cap;
+    return (int)(g < 1 ? 1 : g);
+}
+
+// Token splits of the weight-gradient reductions.
+int token_splits(int64_t T)
+{
+    int64_t s = (T + 1023) / 1024;
+    if (s < 1) s = 1;
+    if (s > 32) s = 32;
+    return (int)s;
+}
+
+// A weight gradient over tokens: partials (if split) then a fixed-order sum.
+template <class LA, class LB>
+cudaError_t weight_grad(int64_t M, int64_t N, int64_t T, LA la, LB lb, float *out, float *part,
+                        const Ctx &c)
+{
+    const int S = token_splits(T);
+    if (S == 1) return gemm(M, N, T, 1, la, lb, EpF32{out, N, 0}, c.stream);
+    cudaError_t e = gemm(M, N, T, S, la, lb, EpF32{part, N, M * N}, c.stream);
+    if (e != cudaSuccess) return e;
+    // the number of splits actually launched (the last ones may be empty)
+    int64_t kchunk = ((T + S - 1) / S + BK - 1) / BK * BK;
+    const int nz = (int)((T + kchunk - 1) / kchunk);
+    k_reduce_splits<<<grid_for(M * N, c), 256, 0, c.stream>>>(part, M * N, nz, out);
+    count_launches(1);
+    return cudaGetLastError();
+}
+
+struct GenericWs {
+    float *P, *Q, *dG, *dA, *part1, *part2;
+};
+
+GenericWs carve(const resbm_desc &d, int op, void *base, size_t *bytes)
+{
+    WsCarver w(base);
+    GenericWs g{};
+    const int64_t T = d.T, S = token_splits(d.T);
+    switch (op) {
+    case RESBM_OP_ENCODE_FWD:
+        g.P = w.take<float>(T * d.m);
+        break;
+    case RESBM_OP_DECODE_FWD:
+        g.Q = w.take<float>(T * d.m);
+        break;
+    case RESBM_OP_DECODE_BWD:
+        g.Q = w.take<float>(T * d.m);
+        g.dG = w.take<float>(T * d.m);
+        g.part1 = w.take<float>(S * d.m * d.d);
+        g.part2 = w.take<float>(S * d.r * d.m);
+        break;
+    case RESBM_OP_ENCODE_BWD:
+        g.P = w.take<float>(T * d.m);
+        g.dA = w.take<float>(T * d.m);
+        g.part1 = w.take<float>(S * d.d * d.m);
+        g.part2 = w.take<float>(S * d.m * d.r);
+        break;
+    default:
+        break;
+    }
+    if (bytes) *bytes = w.used;
+    return g;
+}
+
+template <typename T>
+cudaError_t enc_fwd_t(const resbm_desc &d, const T *X, const T *F, const T *We1, const T *We2,
+                      T *B, float *P_save, void *ws, const Ctx &c)
+{
+    GenericWs g = carve(d, RESBM_OP_ENCODE_FWD, ws, nullptr);
+    float *P = P_save ? P_save : g.P;
+    cudaError_t e = gemm(d.T, d.m, d.d, 1, LdRM<T>{F, d.d}, LdRM<T>{We1, d.m},
+                         EpF32{P, d.m, 0}, c.stream);                       // P = F . We1
+    if (e != cudaSuccess) return e;
+    return gemm(d.T, d.r, d.m, 1, LdAct{P, d.m, d.act}, LdRM<T>{We2, d.r},
+                EpEncB<T>{B, X, d.r, d.d}, c.stream);                       // B = X I + phi(P) We2
+}
+
+template <typename T>
+cudaError_t dec_fwd_t(const resbm_desc &d, const T *B, const T *Wd1, const T *Wd2, T *Y,
+                      void *ws, const Ctx &c)
+{
+    GenericWs g = carve(d, RESBM_OP_DECODE_FWD, ws, nullptr);
+    cudaError_t e = gemm(d.T, d.m, d.r, 1, LdRM<T>{B, d.r}, LdRM<T>{Wd1, d.m},
+                         EpF32{g.Q, d.m, 0}, c.stream);                     // Q = B . Wd1
+    if (e != cudaSuccess) return e;
+    return gemm(d.T, d.d, d.m, 1, LdAct{g.Q, d.m, d.act}, LdRM<T>{Wd2, d.d},
+                EpDecY<T>{Y, B, d.d, d.r, d.merge_identity}, c.stream);     // Y = [B I] + phi(Q) Wd2
+}
+
+template <typename T>
+cudaError_t dec_bwd_t(const resbm_desc &d, const T *dY, const T *B, const T *Wd1, const T *Wd2,
+                      T *dB, float *dWd1, float *dWd2, void *ws, const Ctx &c)
+{
+    GenericWs g = carve(d, RESBM_OP_DECODE_BWD, ws, nullptr);
+    cudaError_t e = gemm(d.T, d.m, d.r, 1, LdRM<T>{B, d.r}, LdRM<T>{Wd1, d.m},
+                         EpF32{g.Q, d.m, 0}, c.stream);                     // Q = B . Wd1
+    if (e != cudaSuccess) return e;
+    e = gemm(d.T, d.m, d.d, 1, LdRM<T>{dY, d.d}, LdT<T>{Wd2, d.d}, EpF32{g.dG, d.m, 0},
+             c.stream);                                                     // dG = dY . Wd2^T
+    if (e != cudaSuccess) return e;
+    const LdDact dQ{g.dG, g.Q, d.m, d.act};                                 // dQ = dG * phi'(Q)
+    e = gemm(d.T, d.r, d.m, 1, dQ, LdT<T>{Wd1, d.m},
+             EpDecDB<T>{dB, dY, d.r, d.d, d.merge_identity}, c.stream);     // dB
+    if (e != cudaSuccess) return e;
+    e = weight_grad(d.m, d.d, d.T, LdActT{g.Q, d.m, d.act}, LdRM<T>{dY, d.d}, dWd2, g.part1,
+                    c);                                                     // dWd2 = phi(Q)^T dY
+    if (e != cudaSuccess) return e;
+    return weight_grad(d.r, d.m, d.T, LdT<T>{B, d.r}, dQ, dWd1, g.part2, c); // dWd1 = B^T dQ
+}
+
+template <typename T>
+cudaError_t enc_bwd_t(const resbm_desc &d, const T *dB, const T *F, const float *P_save,
+                      const T *We1, const T *We2, T *dF, T *dX, float *dWe1, float *dWe2,
+                      void *ws, const Ctx &c)
+{
+    GenericWs g = carve(d, RESBM_OP_ENCODE_BWD, ws, nullptr);
+    cudaError_t e = cudaSuccess;
+    const float *P = P_save;
+    if (!P) {
+        e = gemm(d.T, d.m, d.d, 1, LdRM<T>{F, d.d}, LdRM<T>{We1, d.m}, EpF32{g.P, d.m, 0},
+                 c.stream);                                                 // P = F . We1
+        if (e != cudaSuccess) return e;
+        P = g.P;
+    }
+    e = gemm(d.T, d.m, d.r, 1, LdRM<T>{dB, d.r}, LdT<T>{We2, d.r}, EpF32{g.dA, d.m, 0},
+             c.stream);                                                     // dA = dB . We2^T
+    if (e != cudaSuccess) return e;
+    const LdDact dP{g.dA, P, d.m, d.act};                                   // dP = dA * phi'(P)
+    e = gemm(d.T, d.d, d.m, 1, dP, LdT<T>{We1, d.m}, EpStore<T>{dF, d.d}, c.stream); // dF
+    if (e != cudaSuccess) return e;
+    e = weight_grad(d.d, d.m, d.T, LdT<T>{F, d.d}, dP, dWe1, g.part1, c);   // dWe1 = F^T dP
+    if (e != cudaSuccess) return e;
+    e = weight_grad(d.m, d.r, d.T, LdActT{P, d.m, d.act}, LdRM<T>{dB, d.r}, dWe2, g.part2,
+                    c);                                                     // dWe2 = phi(P)^T dB
+    if (e != cudaSuccess) return e;
+    if (dX) {
+        k_dx_accumulate<T><<<grid_for(d.T * d.r, c), 256, 0, c.stream>>>(dX, dB, d.T, d.d, d.r);
+        count_launches(1);
+        e = cudaGetLastError();
+    }
+    return e;
+}
+
+}  // namespace
+
+size_t generic_ws_bytes(const resbm_desc &d, int op)
+{
+    size_t b = 0;
+    carve(d, op, nullptr, &b);
+    return b;
+}
+
+#define RESBM_DISPATCH(dt, F32CALL, BF16CALL) \
+    ((dt) == RESBM_F32 ? (F32CALL) : (BF16CALL))
+
+cudaError_t generic_encode_fwd(const resbm_desc &d, const void *X, const void *F, const void *We1,
+                               const void *We2, void *B, float *P_save, void *ws, const Ctx &c)
+{
+    using bf = __nv_bfloat16;
+    return RESBM_DISPATCH(d.dtype,
+        enc_fwd_t<float>(d, (const float *)X, (const float *)F, (const float *)We1,
+                         (const float *)We2, (float *)B, P_save, ws, c),
+        enc_fwd_t<bf>(d, (const bf *)X, (const bf *)F, (const bf *)We1, (const bf *)We2,
+                      (bf *)B, P_save, ws, c));
+}
+
+cudaError_t generic_decode_fwd(const resbm_desc &d, const void *B, const void *Wd1,
+                               const void *Wd2, void *Y, void *ws, const Ctx &c)
+{
+    using bf = __nv_bfloat16;
+    return RESBM_DISPATCH(d.dtype,
+        dec_fwd_t<float>(d, (const float *)B, (const float *)Wd1, (const float *)Wd2,
+                         (float *)Y, ws, c),
+        dec_fwd_t<bf>(d, (const bf *)B, (const bf *)Wd1, (const bf *)Wd2, (bf *)Y, ws, c));
+}
+
+cudaError_t generic_decode_bwd(const resbm_desc &d, const void *dY, const void *B,
+                               const void *Wd1, const void *Wd2, void *dB, float *dWd1,
+                               float *dWd2, void *ws, const Ctx &c)
+{
+    using bf = __nv_bfloat16;
+    return RESBM_DISPATCH(d.dtype,
+        dec_bwd_t<float>(d, (const float *)dY, (const float *)B, (const float *)Wd1,
+                         (const float *)Wd2, (float *)dB, dWd1, dWd2, ws, c),
+        dec_bwd_t<bf>(d, (const bf *)dY, (const bf *)B, (const bf *)Wd1, (const bf *)Wd2,
+                      (bf *)dB, dWd1, dWd2, ws, c));
+}
+
+cudaError_t generic_encode_bwd(const resbm_desc &d, const void *dB, const void *F,
+                               const float *P_save, const void *We1, const void *We2, void *dF,
+                               void *dX, float *dWe1, float *dWe2, void *ws, const Ctx &c)
+{
+    using bf = __nv_bfloat16;
+    return RESBM_DISPATCH(d.dtype,
+        enc_bwd_t<float>(d, (const float *)dB, (const float *)F, P_save, (const float *)We1,
+                         (const float *)We2, (float *)dF, (float *)dX, dWe1, dWe2, ws, c),
+        enc_bwd_t<bf>(d, (const bf *)dB, (const bf *)F, P_save, (const bf *)We1,
+                      (const bf *)We2, (bf *)dF, (bf *)dX, dWe1, dWe2, ws, c));
+}
+
+}  // namespace resbm

@@ -1,0 +1,378 @@
+// resbm_abi.cu -- the C ABI of include/resbm.h: argument validation, scratch sizing and the
+// choice between the tensor-core kernels and the portable CUDA-core kernels.
+#include <cuda_runtime.h>
+#include <stdint.h>
+#include <string.h>
+
+#include <atomic>
+
+#include "internal.h"
+#include "resbm.h"
+#include "tc.h"
+
+using namespace resbm;
+
+namespace resbm {
+static std::atomic<uint64_t> g_launches{0};
+void count_launches(uint64_t n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
+}  // namespace resbm
+
+namespace {
+
+thread_local int g_last_cuda_error = 0;
+
+resbm_status cuda_fail(cudaError_t e)
+{
+    g_last_cuda_error = (int)e;
+    return RESBM_ERR_CUDA;
+}
+
+constexpr int kMaxDevices = 64;
+std::atomic<int> g_sm_count[kMaxDevices];
+
+resbm_status make_ctx(void *stream, Ctx *c)
+{
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e);
+    int sms = (dev >= 0 && dev < kMaxDevices) ? g_sm_count[dev].load(std::memory_order_relaxed) : 0;
+    if (sms <= 0) {
+        e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        if (e != cudaSuccess) return cuda_fail(e);
+        if (dev >= 0 && dev < kMaxDevices) g_sm_count[dev].store(sms, std::memory_order_relaxed);
+    }
+    c->stream = static_cast<cudaStream_t>(stream);
+    c->device = dev;
+    c->sm_count = sms;
+    return RESBM_OK;
+}
+
+size_t elem_size(const resbm_desc &d) { return d.dtype == RESBM_BF16 ? 2 : 4; }
+
+bool mul_ok(int64_t a, int64_t b) { return a >= 0 && b >= 0 && (a == 0 || b <= INT64_MAX / a); }
+
+resbm_status check_desc(const resbm_desc *d)
+{
+    if (!d) return RESBM_ERR_INVALID_ARG;
+    if (d->T < 0 || d->d < 1 || d->r < 1 || d->m < 1 || d->r > d->d) return RESBM_ERR_INVALID_ARG;
+    if (d->dtype != RESBM_F32 && d->dtype != RESBM_BF16) return RESBM_ERR_INVALID_ARG;
+    if (d->act != RESBM_ACT_SILU && d->act != RESBM_ACT_GELU_TANH && d->act != RESBM_ACT_IDENTITY)
+        return RESBM_ERR_INVALID_ARG;
+    if (d->merge_identity != 0 && d->merge_identity != 1) return RESBM_ERR_INVALID_ARG;
+    if (d->flags & ~RESBM_FLAG_GENERIC) return RESBM_ERR_INVALID_ARG;
+    // every element count (and the byte counts derived from it) must fit in int64
+    const int64_t big = INT64_MAX / 64;
+    if (!mul_ok(d->T, d->d) || d->T * d->d > big || !mul_ok(d->T, d->m) || d->T * d->m > big ||
+        !mul_ok(d->d, d->m) || d->d * d->m > big || !mul_ok(d->m, d->r) || d->m * d->r > big)
+        return RESBM_ERR_INVALID_ARG;
+    return RESBM_OK;
+}
+
+// A tensor argument: required non-null when it has elements, aligned to its element size.
+bool ptr_ok(const void *p, size_t align, bool required)
+{
+    if (!p) return !required;
+    return (reinterpret_cast<uintptr_t>(p) % align) == 0;
+}
+
+struct Range {
+    uintptr_t lo, hi;
+};
+Range rng(const void *p, int64_t n, size_t es)
+{
+    uintptr_t a = reinterpret_cast<uintptr_t>(p);
+    return Range{a, a + (uintptr_t)n * es};
+}
+bool overlaps(Range a, Range b)
+{
+    if (!a.lo || !b.lo || a.lo == a.hi || b.lo == b.hi) return false;
+    return a.lo < b.hi && b.lo < a.hi;
+}
+template <size_t N> bool any_overlap(const Range (&outs)[N], const Range *ins, size_t nin)
+{
+    for (size_t i = 0; i < N; ++i) {
+        for (size_t j = 0; j < nin; ++j)
+            if (overlaps(outs[i], ins[j])) return true;
+        for (size_t j = i + 1; j < N; ++j)
+            if (overlaps(outs[i], outs[j])) return true;
+    }
+    return false;
+}
+
+bool use_tc(const resbm_desc &d, int op) { return !(d.flags & RESBM_FLAG_GENERIC) && tc_supported(d, op); }
+
+size_t ws_for(const resbm_desc &d, int op)
+{
+    size_t g = generic_ws_bytes(d, op);
+    size_t t = tc_supported(d, op) ? tc_ws_bytes(d, op) : 0;
+    return g > t ? g : t;
+}
+
+size_t step_ws_bytes(const resbm_desc &d)
+{
+    WsCarver w(nullptr);
+    w.take<float>(d.T * d.m);  // P when the caller passes none
+    size_t inner = 0;
+    for (int op = RESBM_OP_ENCODE_FWD; op <= RESBM_OP_ENCODE_BWD; ++op) {
+        size_t b = ws_for(d, op);
+        if (b > inner) inner = b;
+    }
+    w.take<char>(inner);
+    return w.used;
+}
+
+resbm_status check_ws(const resbm_desc &d, int op, void *ws, size_t ws_bytes)
+{
+    size_t need = op == RESBM_OP_BOUNDARY_STEP ? step_ws_bytes(d) : ws_for(d, op);
+    if (need == 0) return RESBM_OK;
+    if (!ws || ws_bytes < need) return RESBM_ERR_WORKSPACE;
+    if (reinterpret_cast<uintptr_t>(ws) % 256) return RESBM_ERR_INVALID_ARG;
+    return RESBM_OK;
+}
+
+resbm_status zero_f32(float *p, int64_t n, cudaStream_t s)
+{
+    if (!p || n <= 0) return RESBM_OK;
+    cudaError_t e = cudaMemsetAsync(p, 0, (size_t)n * sizeof(float), s);
+    return e == cudaSuccess ? RESBM_OK : cuda_fail(e);
+}
+
+resbm_status finish(cudaError_t e) { return e == cudaSuccess ? RESBM_OK : cuda_fail(e); }
+
+// ---- per-op validation (no GPU work) ---------------------------------------------------------
+resbm_status validate_encode_fwd(const resbm_desc &d, const void *X, const void *F,
+                                 const void *We1, const void *We2, const void *B,
+                                 const float *P)
+{
+    const size_t es = elem_size(d);
+    const bool t = d.T > 0;
+    if (!ptr_ok(X, es, t) || !ptr_ok(F, es, t) || !ptr_ok(We1, es, true) ||
+        !ptr_ok(We2, es, true) || !ptr_ok(B, es, t) || !ptr_ok(P, 4, false))
+        return RESBM_ERR_INVALID_ARG;
+    const Range outs[] = {rng(B, d.T * d.r, es), rng(P, d.T * d.m, 4)};
+    const Range ins[] = {rng(X, d.T * d.d, es), rng(F, d.T * d.d, es), rng(We1, d.d * d.m, es),
+                         rng(We2, d.m * d.r, es)};
+    return any_overlap(outs, ins, 4) ? RESBM_ERR_INVALID_ARG : RESBM_OK;
+}
+
+resbm_status validate_decode_fwd(const resbm_desc &d, const void *B, const void *Wd1,
+                                 const void *Wd2, const void *Y)
+{
+    const size_t es = elem_size(d);
+    const bool t = d.T > 0;
+    if (!ptr_ok(B, es, t) || !ptr_ok(Wd1, es, true) || !ptr_ok(Wd2, es, true) ||
+        !ptr_ok(Y, es, t))
+        return RESBM_ERR_INVALID_ARG;
+    const Range outs[] = {rng(Y, d.T * d.d, es)};
+    const Range ins[] = {rng(B, d.T * d.r, es), rng(Wd1, d.r * d.m, es), rng(Wd2, d.m * d.d, es)};
+    return any_overlap(outs, ins, 3) ? RESBM_ERR_INVALID_ARG : RESBM_OK;
+}
+
+resbm_status validate_decode_bwd(const resbm_desc &d, const void *dY, const void *B,
+                                 const void *Wd1, const void *Wd2, const void *dB,
+                                 const float *dWd1, const float *dWd2)
+{
+    const size_t es = elem_size(d);
+    const bool t = d.T > 0;
+    if (!ptr_ok(dY, es, t) || !ptr_ok(B, es, t) || !ptr_ok(Wd1, es, true) ||
+        !ptr_ok(Wd2, es, true) || !ptr_ok(dB, es, t) || !ptr_ok(dWd1, 4, true) ||
+        !ptr_ok(dWd2, 4, true))
+        return RESBM_ERR_INVALID_ARG;
+    const Range outs[] = {rng(dB, d.T * d.r, es), rng(dWd1, d.r * d.m, 4), rng(dWd2, d.m * d.d, 4)};
+    const Range ins[] = {rng(dY, d.T * d.d, es), rng(B, d.T * d.r, es), rng(Wd1, d.r * d.m, es),
+                         rng(Wd2, d.m * d.d, es)};
+    return any_overlap(outs, ins, 4) ? RESBM_ERR_INVALID_ARG : RESBM_OK;
+}
+
+resbm_status validate_encode_bwd(const resbm_desc &d, const void *dB, const void *F,
+                                 const float *P, const void *We1, const void *We2,
+                                 const void *dF, const void *dX, const float *dWe1,
+                                 const float *dWe2)
+{
+    const size_t es = elem_size(d);
+    const bool t = d.T > 0;
+    if (!ptr_ok(dB, es, t) || !ptr_ok(F, es, t) || !ptr_ok(P, 4, false) ||
+        !ptr_ok(We1, es, true) || !ptr_ok(We2, es, true) || !ptr_ok(dF, es, t) ||
+        !ptr_ok(dX, es, false) || !ptr_ok(dWe1, 4, true) || !ptr_ok(dWe2, 4, true))
+        return RESBM_ERR_INVALID_ARG;
+    const Range outs[] = {rng(dF, d.T * d.d, es), rng(dX, d.T * d.d, es), rng(dWe1, d.d * d.m, 4),
+                          rng(dWe2, d.m * d.r, 4)};
+    const Range ins[] = {rng(dB, d.T * d.r, es), rng(F, d.T * d.d, es), rng(P, d.T * d.m, 4),
+                         rng(We1, d.d * d.m, es), rng(We2, d.m * d.r, es)};
+    return any_overlap(outs, ins, 5) ? RESBM_ERR_INVALID_ARG : RESBM_OK;
+}
+
+// ---- per-op execution (after validation) -----------------------------------------------------
+resbm_status run_encode_fwd(const resbm_desc &d, const void *X, const void *F, const void *We1,
+                            const void *We2, void *B, float *P, void *ws, const Ctx &c)
+{
+    if (d.T == 0) return RESBM_OK;
+    if (use_tc(d, RESBM_OP_ENCODE_FWD)) return finish(tc_encode_fwd(d, X, F, We1, We2, B, P, ws, c));
+    return finish(generic_encode_fwd(d, X, F, We1, We2, B, P, ws, c));
+}
+
+resbm_status run_decode_fwd(const resbm_desc &d, const void *B, const void *Wd1, const void *Wd2,
+                            void *Y, void *ws, const Ctx &c)
+{
+    if (d.T == 0) return RESBM_OK;
+    if (use_tc(d, RESBM_OP_DECODE_FWD)) return finish(tc_decode_fwd(d, B, Wd1, Wd2, Y, ws, c));
+    return finish(generic_decode_fwd(d, B, Wd1, Wd2, Y, ws, c));
+}
+
+resbm_status run_decode_bwd(const resbm_desc &d, const void *dY, const void *B, const void *Wd1,
+                            const void *Wd2, void *dB, float *dWd1, float *dWd2, void *ws,
+                            const Ctx &c)
+{
+    if (d.T == 0) {
+        resbm_status s = zero_f32(dWd1, d.r * d.m, c.stream);
+        return s != RESBM_OK ? s : zero_f32(dWd2, d.m * d.d, c.stream);
+    }
+    if (use_tc(d, RESBM_OP_DECODE_BWD))
+        return finish(tc_decode_bwd(d, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, c));
+    return finish(generic_decode_bwd(d, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, c));
+}
+
+resbm_status run_encode_bwd(const resbm_desc &d, const void *dB, const void *F, const float *P,
+                            const void *We1, const void *We2, void *dF, void *dX, float *dWe1,
+                            float *dWe2, void *ws, const Ctx &c)
+{
+    if (d.T == 0) {
+        resbm_status s = zero_f32(dWe1, d.d * d.m, c.stream);
+        return s != RESBM_OK ? s : zero_f32(dWe2, d.m * d.r, c.stream);
+    }
+    if (use_tc(d, RESBM_OP_ENCODE_BWD))
+        return finish(tc_encode_bwd(d, dB, F, P, We1, We2, dF, dX, dWe1, dWe2, ws, c));
+    return finish(generic_encode_bwd(d, dB, F, P, We1, We2, dF, dX, dWe1, dWe2, ws, c));
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *resbm_version(void) { return "resbm 0.1.0 sm_103a"; }
+
+const char *resbm_status_string(resbm_status s)
+{
+    switch (s) {
+    case RESBM_OK: return "RESBM_OK";
+    case RESBM_ERR_INVALID_ARG: return "RESBM_ERR_INVALID_ARG";
+    case RESBM_ERR_UNSUPPORTED: return "RESBM_ERR_UNSUPPORTED";
+    case RESBM_ERR_WORKSPACE: return "RESBM_ERR_WORKSPACE";
+    case RESBM_ERR_CUDA: return "RESBM_ERR_CUDA";
+    }
+    return "RESBM_ERR_UNKNOWN";
+}
+
+int resbm_last_cuda_error(void) { return g_last_cuda_error; }
+
+uint64_t resbm_kernel_launches(void) { return g_launches.load(std::memory_order_relaxed); }
+
+resbm_status resbm_workspace_bytes(const resbm_desc *desc, int op, size_t *bytes)
+{
+    resbm_status s = check_desc(desc);
+    if (s != RESBM_OK) return s;
+    if (!bytes || op < RESBM_OP_ENCODE_FWD || op > RESBM_OP_BOUNDARY_STEP)
+        return RESBM_ERR_INVALID_ARG;
+    *bytes = op == RESBM_OP_BOUNDARY_STEP ? step_ws_bytes(*desc) : ws_for(*desc, op);
+    return RESBM_OK;
+}
+
+resbm_status resbm_encode_fwd(const resbm_desc *desc, const void *X, const void *F,
+                              const void *We1, const void *We2, void *B, float *P_save,
+                              void *ws, size_t ws_bytes, void *stream)
+{
+    resbm_status s = check_desc(desc);
+    if (s == RESBM_OK) s = validate_encode_fwd(*desc, X, F, We1, We2, B, P_save);
+    if (s == RESBM_OK) s = check_ws(*desc, RESBM_OP_ENCODE_FWD, ws, ws_bytes);
+    Ctx c;
+    if (s == RESBM_OK) s = make_ctx(stream, &c);
+    if (s == RESBM_OK) s = run_encode_fwd(*desc, X, F, We1, We2, B, P_save, ws, c);
+    return s;
+}
+
+resbm_status resbm_decode_fwd(const resbm_desc *desc, const void *B, const void *Wd1,
+                              const void *Wd2, void *Y, void *ws, size_t ws_bytes, void *stream)
+{
+    resbm_status s = check_desc(desc);
+    if (s == RESBM_OK) s = validate_decode_fwd(*desc, B, Wd1, Wd2, Y);
+    if (s == RESBM_OK) s = check_ws(*desc, RESBM_OP_DECODE_FWD, ws, ws_bytes);
+    Ctx c;
+    if (s == RESBM_OK) s = make_ctx(stream, &c);
+    if (s == RESBM_OK) s = run_decode_fwd(*desc, B, Wd1, Wd2, Y, ws, c);
+    return s;
+}
+
+resbm_status resbm_decode_bwd(const resbm_desc *desc, const void *dY, const void *B,
+                              const void *Wd1, const void *Wd2, void *dB, float *dWd1,
+                              float *dWd2, void *ws, size_t ws_bytes, void *stream)
+{
+    resbm_status s = check_desc(desc);
+    if (s == RESBM_OK) s = validate_decode_bwd(*desc, dY, B, Wd1, Wd2, dB, dWd1, dWd2);
+    if (s == RESBM_OK) s = check_ws(*desc, RESBM_OP_DECODE_BWD, ws, ws_bytes);
+    Ctx c;
+    if (s == RESBM_OK) s = make_ctx(stream, &c);
+    if (s == RESBM_OK) s = run_decode_bwd(*desc, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, c);
+    return s;
+}
+
+resbm_status resbm_encode_bwd(const resbm_desc *desc, const void *dB, const void *F,
+                              const float *P_save, const void *We1, const void *We2, void *dF,
+                              void *dX, float *dWe1, float *dWe2, void *ws, size_t ws_bytes,
+                              void *stream)
+{
+    resbm_status s = check_desc(desc);
+    if (s == RESBM_OK)
+        s = validate_encode_bwd(*desc, dB, F, P_save, We1, We2, dF, dX, dWe1, dWe2);
+    if (s == RESBM_OK) s = check_ws(*desc, RESBM_OP_ENCODE_BWD, ws, ws_bytes);
+    Ctx c;
+    if (s == RESBM_OK) s = make_ctx(stream, &c);
+    if (s == RESBM_OK)
+        s = run_encode_bwd(*desc, dB, F, P_save, We1, We2, dF, dX, dWe1, dWe2, ws, c);
+    return s;
+}
+
+resbm_status resbm_boundary_step(const resbm_desc *desc, const resbm_step_args *a, void *ws,
+                                 size_t ws_bytes, void *stream)
+{
+    resbm_status s = check_desc(desc);
+    if (s != RESBM_OK) return s;
+    if (!a) return RESBM_ERR_INVALID_ARG;
+    const resbm_desc &d = *desc;
+    s = check_ws(d, RESBM_OP_BOUNDARY_STEP, ws, ws_bytes);
+    if (s != RESBM_OK) return s;
+    WsCarver w(ws);
+    float *P = a->P ? a->P : w.take<float>(d.T * d.m);
+    void *inner = w.take<char>(0);
+    // validate all four stages before enqueueing anything
+    s = validate_encode_fwd(d, a->X, a->F, a->We1, a->We2, a->B, a->P);
+    if (s == RESBM_OK) s = validate_decode_fwd(d, a->B, a->Wd1, a->Wd2, a->Y);
+    if (s == RESBM_OK)
+        s = validate_decode_bwd(d, a->dY, a->B, a->Wd1, a->Wd2, a->dB, a->dWd1, a->dWd2);
+    if (s == RESBM_OK)
+        s = validate_encode_bwd(d, a->dB, a->F, a->P, a->We1, a->We2, a->dF, a->dX, a->dWe1,
+                                a->dWe2);
+    if (s == RESBM_OK) {
+        // outputs of different stages must not overlap each other or the step's inputs
+        const size_t es = elem_size(d);
+        const Range outs[] = {rng(a->B, d.T * d.r, es), rng(a->P, d.T * d.m, 4),
+                              rng(a->Y, d.T * d.d, es), rng(a->dB, d.T * d.r, es),
+                              rng(a->dF, d.T * d.d, es), rng(a->dX, d.T * d.d, es),
+                              rng(a->dWe1, d.d * d.m, 4), rng(a->dWe2, d.m * d.r, 4),
+                              rng(a->dWd1, d.r * d.m, 4), rng(a->dWd2, d.m * d.d, 4)};
+        const Range ins[] = {rng(a->X, d.T * d.d, es), rng(a->F, d.T * d.d, es),
+                             rng(a->dY, d.T * d.d, es)};
+        if (any_overlap(outs, ins, 3)) s = RESBM_ERR_INVALID_ARG;
+    }
+    Ctx c;
+    if (s == RESBM_OK) s = make_ctx(stream, &c);
+    if (s == RESBM_OK) s = run_encode_fwd(d, a->X, a->F, a->We1, a->We2, a->B, P, inner, c);
+    if (s == RESBM_OK) s = run_decode_fwd(d, a->B, a->Wd1, a->Wd2, a->Y, inner, c);
+    if (s == RESBM_OK)
+        s = run_decode_bwd(d, a->dY, a->B, a->Wd1, a->Wd2, a->dB, a->dWd1, a->dWd2, inner, c);
+    if (s == RESBM_OK)
+        s = run_encode_bwd(d, a->dB, a->F, P, a->We1, a->We2, a->dF, a->dX, a->dWe1, a->dWe2,
+                           inner, c);
+    return s;
+}
+
+}  // extern "C"

@@ -1,0 +1,24 @@
+// tc.h -- host-side interface of the sm_103a tensor-core (tcgen05 + TMA) kernels.
+#pragma once
+
+#include "internal.h"
+
+namespace resbm {
+
+// Whether the tensor-core kernels handle this descriptor for `op` (bf16 I/O, shapes that fit
+// their tiles); otherwise the portable kernels run.
+bool tc_supported(const resbm_desc &d, int op);
+size_t tc_ws_bytes(const resbm_desc &d, int op);
+
+cudaError_t tc_encode_fwd(const resbm_desc &d, const void *X, const void *F, const void *We1,
+                          const void *We2, void *B, float *P_save, void *ws, const Ctx &c);
+cudaError_t tc_decode_fwd(const resbm_desc &d, const void *B, const void *Wd1, const void *Wd2,
+                          void *Y, void *ws, const Ctx &c);
+cudaError_t tc_decode_bwd(const resbm_desc &d, const void *dY, const void *B, const void *Wd1,
+                          const void *Wd2, void *dB, float *dWd1, float *dWd2, void *ws,
+                          const Ctx &c);
+cudaError_t tc_encode_bwd(const resbm_desc &d, const void *dB, const void *F, const float *P_save,
+                          const void *We1, const void *We2, void *dF, void *dX, float *dWe1,
+                          float *dWe2, void *ws, const Ctx &c);
+
+}  // namespace resbm

@@ -182,15 +182,18 @@ def rows_at(cfg: BoundaryConfig, name: str, idx) -> np.ndarray:
 
 
 def tensor(cfg: BoundaryConfig, name: str, threads: int | None = None,
-           chunk_elems: int = 1 << 18) -> np.ndarray:
-    """A whole tensor, drawn in row chunks on a thread pool (numpy releases the GIL)."""
-    nrows, ncols = shapes(cfg)[name]
+           chunk_elems: int = 1 << 18, nrows: int | None = None) -> np.ndarray:
+    """A whole tensor (or its first nrows rows), drawn in row chunks on a thread pool (numpy
+    releases the GIL)."""
+    full_rows, ncols = shapes(cfg)[name]
+    nrows = full_rows if nrows is None else min(nrows, full_rows)
     step = max(1, chunk_elems // max(1, ncols))
     out = np.empty((nrows, ncols), np.float32)
     starts = list(range(0, nrows, step))
 
     def work(t0):
-        out[t0:min(t0 + step, nrows)] = rows(cfg, name, t0, t0 + step)
+        t1 = min(t0 + step, nrows)
+        out[t0:t1] = rows(cfg, name, t0, t1)
 
     if len(starts) == 1:
         work(0)

@@ -1,0 +1,137 @@
+"""The C ABI on the host, without a GPU: the library loads, exports every declared symbol, and
+rejects bad arguments with status codes before touching the device."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2604_11947_gb300 import build, resbm
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return resbm.load()
+
+
+def declared_functions():
+    src = open(os.path.join(ROOT, "include", "resbm.h")).read()
+    return sorted(set(re.findall(r"RESBM_API\s+[\w\s\*]*?\b(resbm_\w+)\s*\(", src)))
+
+
+def test_exports_every_declared_symbol(lib):
+    names = declared_functions()
+    assert len(names) == 10, names
+    assert sorted(resbm.EXPORTS) == names
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_version_and_status_strings(lib):
+    assert "sm_103a" in resbm.resbm_version()
+    assert resbm.status_string(resbm.RESBM_OK) == "RESBM_OK"
+    assert resbm.status_string(resbm.RESBM_ERR_WORKSPACE) == "RESBM_ERR_WORKSPACE"
+    assert resbm.status_string(99) == "RESBM_ERR_UNKNOWN"
+    assert lib.resbm_last_cuda_error() == 0
+    assert resbm.resbm_kernel_launches() == 0   # nothing launched on a host without a GPU
+
+
+def test_struct_layout_matches_header():
+    assert ctypes.sizeof(resbm.resbm_desc) == 4 * 8 + 4 * 4
+    assert ctypes.sizeof(resbm.resbm_step_args) == 17 * ctypes.sizeof(ctypes.c_void_p)
+
+
+@pytest.mark.parametrize("op", range(5))
+def test_workspace_query(lib, op):
+    d = resbm.make_desc(65536, 4096, 32, 32)
+    n = resbm.resbm_workspace_bytes(d, op)
+    assert n >= 0
+    if op in (resbm.RESBM_OP_DECODE_BWD, resbm.RESBM_OP_ENCODE_BWD, resbm.RESBM_OP_BOUNDARY_STEP):
+        assert n > 0
+    d0 = resbm.make_desc(0, 4096, 32, 32)
+    assert resbm.resbm_workspace_bytes(d0, op) >= 0
+
+
+@pytest.mark.parametrize("bad", [
+    dict(T=-1), dict(d=0), dict(r=0), dict(m=0), dict(r=5000, d=4096), dict(dtype=7),
+    dict(act=9), dict(merge_identity=2), dict(flags=8), dict(T=1 << 40, d=1 << 30),
+])
+def test_bad_descriptor_rejected(lib, bad):
+    kw = dict(T=16, d=64, r=8, m=8, dtype=1, act=0, merge_identity=1, flags=0)
+    kw.update(bad)
+    d = resbm.resbm_desc(kw["T"], kw["d"], kw["r"], kw["m"], kw["dtype"], kw["act"],
+                         kw["merge_identity"], kw["flags"])
+    out = ctypes.c_size_t(0)
+    assert lib.resbm_workspace_bytes(ctypes.byref(d), 0, ctypes.byref(out)) == resbm.RESBM_ERR_INVALID_ARG
+    st = lib.resbm_decode_fwd(ctypes.byref(d), 4096, 4096, 4096, 1 << 20, None, 0, None)
+    assert st == resbm.RESBM_ERR_INVALID_ARG
+
+
+def test_bad_op_and_null_desc(lib):
+    d = resbm.make_desc(16, 64, 8, 8)
+    out = ctypes.c_size_t(0)
+    assert lib.resbm_workspace_bytes(ctypes.byref(d), 5, ctypes.byref(out)) == resbm.RESBM_ERR_INVALID_ARG
+    assert lib.resbm_workspace_bytes(None, 0, ctypes.byref(out)) == resbm.RESBM_ERR_INVALID_ARG
+    assert lib.resbm_workspace_bytes(ctypes.byref(d), 0, None) == resbm.RESBM_ERR_INVALID_ARG
+    assert lib.resbm_encode_fwd(None, 1, 1, 1, 1, 1, None, None, 0, None) == resbm.RESBM_ERR_INVALID_ARG
+
+
+# Fake, never-dereferenced device addresses: validation must fail before any GPU work.
+A = 1 << 32
+
+
+def test_null_and_misaligned_pointers(lib):
+    d = resbm.make_desc(16, 64, 8, 8, dtype="bf16")
+    ws = 1 << 36
+    big = 1 << 30
+    enc = lib.resbm_encode_fwd
+    assert enc(ctypes.byref(d), None, A, A + big, A + 2 * big, A + 3 * big, None, ws, big, None) == resbm.RESBM_ERR_INVALID_ARG
+    assert enc(ctypes.byref(d), A + 1, A, A + big, A + 2 * big, A + 3 * big, None, ws, big, None) == resbm.RESBM_ERR_INVALID_ARG
+    # fp32 P must be 4-byte aligned
+    assert enc(ctypes.byref(d), A, A, A + big, A + 2 * big, A + 3 * big, A + 4 * big + 2, ws, big, None) == resbm.RESBM_ERR_INVALID_ARG
+    # weights are required even for T = 0
+    d0 = resbm.make_desc(0, 64, 8, 8)
+    assert lib.resbm_decode_fwd(ctypes.byref(d0), None, None, A, None, None, 0, None) == resbm.RESBM_ERR_INVALID_ARG
+
+
+def test_overlapping_output_rejected(lib):
+    d = resbm.make_desc(16, 64, 8, 8, dtype="bf16")
+    big = 1 << 30
+    # Y (16 x 64 bf16 = 2 KiB) starting inside B's range
+    st = lib.resbm_decode_fwd(ctypes.byref(d), A, A + big, A + 2 * big, A + 64, 1 << 36, big, None)
+    assert st == resbm.RESBM_ERR_INVALID_ARG
+    # decode bwd: dWd2 overlapping dY
+    st = lib.resbm_decode_bwd(ctypes.byref(d), A, A + big, A + 2 * big, A + 3 * big, A + 4 * big,
+                              A + 5 * big, A + 16, 1 << 36, big, None)
+    assert st == resbm.RESBM_ERR_INVALID_ARG
+
+
+def test_workspace_too_small(lib):
+    d = resbm.make_desc(4096, 512, 16, 16, dtype="bf16")
+    need = resbm.resbm_workspace_bytes(d, resbm.RESBM_OP_DECODE_BWD)
+    big = 1 << 30
+    args = [A, A + big, A + 2 * big, A + 3 * big, A + 4 * big, A + 5 * big, A + 6 * big]
+    st = lib.resbm_decode_bwd(ctypes.byref(d), *args, A + 8 * big, need - 1, None)
+    assert st == resbm.RESBM_ERR_WORKSPACE
+    st = lib.resbm_decode_bwd(ctypes.byref(d), *args, None, need, None)
+    assert st == resbm.RESBM_ERR_WORKSPACE
+    # misaligned workspace
+    st = lib.resbm_decode_bwd(ctypes.byref(d), *args, A + 8 * big + 16, need, None)
+    assert st == resbm.RESBM_ERR_INVALID_ARG
+
+
+def test_step_rejects_output_aliasing_input(lib):
+    d = resbm.make_desc(16, 64, 8, 8, dtype="bf16")
+    big = 1 << 30
+    ptrs = {n: A + i * big for i, n in enumerate(
+        ["X", "F", "dY", "We1", "We2", "Wd1", "Wd2", "B", "P", "Y", "dB", "dF", "dX",
+         "dWe1", "dWe2", "dWd1", "dWd2"])}
+    ptrs["dF"] = ptrs["X"]
+    args = resbm.resbm_step_args(**ptrs)
+    need = resbm.resbm_workspace_bytes(d, resbm.RESBM_OP_BOUNDARY_STEP)
+    st = lib.resbm_boundary_step(ctypes.byref(d), ctypes.byref(args), 1 << 40, need, None)
+    assert st == resbm.RESBM_ERR_INVALID_ARG
+    assert lib.resbm_boundary_step(ctypes.byref(d), None, 1 << 40, need, None) == resbm.RESBM_ERR_INVALID_ARG

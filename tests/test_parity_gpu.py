@@ -1,0 +1,269 @@
+"""The CUDA path (through the C ABI) against the fp64 oracle on the same seeded inputs."""
+import numpy as np
+import pytest
+import torch
+
+from gpu_helpers import INPUTS, gpu_step, host_inputs, oracle_step, sample_tokens, to_dev, to_host
+from metrics import TOL, check
+from paper_2604_11947_gb300 import resbm, synth
+
+import oracle
+
+pytestmark = pytest.mark.gpu
+
+PATHS = {"default": 0, "generic": resbm.RESBM_FLAG_GENERIC}
+OUTS = ("B", "Y", "dB", "dF", "dX", "dWe1", "dWe2", "dWd1", "dWd2")
+
+SMALL = {
+    # name: config (ragged token counts, several 128-token tiles, r and m around the tiles)
+    "tiny_f32": synth.CONFIGS["tiny_f32"],
+    "ragged_bf16_r32": synth.BoundaryConfig("ragged_bf16_r32", T=1000, d=512, r=32, m=32),
+    "ragged_bf16_r16": synth.BoundaryConfig("ragged_bf16_r16", T=777, d=384, r=16, m=16),
+    "bf16_r64": synth.BoundaryConfig("bf16_r64", T=300, d=256, r=64, m=64),
+    "bf16_m_ne_r": synth.BoundaryConfig("bf16_m_ne_r", T=515, d=320, r=16, m=48),
+    "bf16_r128": synth.BoundaryConfig("bf16_r128", T=260, d=512, r=128, m=128),
+    "f32_ragged": synth.BoundaryConfig("f32_ragged", T=333, d=200, r=8, m=5, dtype="f32"),
+    "bf16_odd_d": synth.BoundaryConfig("bf16_odd_d", T=129, d=100, r=3, m=7),
+    "bf16_no_compression": synth.BoundaryConfig("bf16_no_compression", T=200, d=64, r=64, m=16),
+    "bf16_r1": synth.BoundaryConfig("bf16_r1", T=64, d=128, r=1, m=1),
+}
+
+
+def _compare_all(cfg, got, want):
+    errs = {}
+    for k in OUTS:
+        errs[k] = check(k, to_host(got[k]), want[k], cfg.dtype)
+    return errs
+
+
+@pytest.mark.parametrize("path", PATHS)
+@pytest.mark.parametrize("name", SMALL)
+def test_small_configs_match_oracle(name, path):
+    cfg = SMALL[name]
+    h = host_inputs(cfg)
+    dev = {k: to_dev(v, cfg) for k, v in h.items()}
+    got = gpu_step(cfg, dev, flags=PATHS[path])
+    want = oracle_step(cfg, h)
+    _compare_all(cfg, got, want)
+    # the saved pre-activation P = F . We1 is an fp32 output: fp32 accumulation error only
+    check("P", to_host(got["P"]), want["P"], "f32", tol=1e-4)
+
+
+@pytest.mark.parametrize("act", ["gelu_tanh", "identity"])
+@pytest.mark.parametrize("merge", [0, 1])
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_activation_and_merge_variants(act, merge, dtype):
+    cfg = synth.BoundaryConfig("v", T=400, d=256, r=16, m=24, dtype=dtype, act=act, merge=merge)
+    h = host_inputs(cfg)
+    dev = {k: to_dev(v, cfg) for k, v in h.items()}
+    for flags in PATHS.values():
+        _compare_all(cfg, gpu_step(cfg, dev, flags=flags), oracle_step(cfg, h))
+
+
+def test_single_bf16_config_full():
+    """T = 16384, d = 2048, r = 16 (batch 8 x seq 2048, 128x): every element of every output."""
+    cfg = synth.CONFIGS["single_bf16"]
+    h = host_inputs(cfg)
+    dev = {k: to_dev(v, cfg) for k, v in h.items()}
+    got = gpu_step(cfg, dev)
+    want = oracle_step(cfg, h)
+    _compare_all(cfg, got, want)
+
+
+def _sampled_full_size(cfg, n_tokens=96, flags=0):
+    """Full-size launch (the benchmarked shapes) checked on a token sample S:
+    run 1 with the full dY: per-token outputs of S against the oracle on S;
+    run 2 with dY zero outside S: the weight gradients (sums over tokens) are exactly the
+    oracle's over S, and the backward per-token outputs vanish outside S."""
+    S = sample_tokens(cfg.T, n_tokens)
+    dev = {}
+    for k in INPUTS:
+        dev[k] = to_dev(synth.tensor(cfg, k), cfg)
+    hS = {k: synth.rows_at(cfg, k, S) for k in ("X", "F", "dY")}
+    for k in ("We1", "We2", "Wd1", "Wd2"):
+        hS[k] = to_host(dev[k])
+    want = oracle_step(cfg, hS)
+    Sg = torch.from_numpy(S).cuda()
+    got = gpu_step(cfg, dev, flags=flags)
+    for k in ("B", "Y", "dB", "dF", "dX"):
+        check(k, to_host(got[k][Sg]), want[k], cfg.dtype)
+    del got
+    dY_masked = torch.zeros_like(dev["dY"])
+    dY_masked[Sg] = dev["dY"][Sg]
+    dev["dY"] = dY_masked
+    got = gpu_step(cfg, dev, flags=flags)
+    for k in ("dWe1", "dWe2", "dWd1", "dWd2"):
+        check(k, to_host(got[k]), want[k], cfg.dtype)
+    for k in ("dB", "dF", "dX"):
+        check(k, to_host(got[k][Sg]), want[k], cfg.dtype)
+    outside = torch.ones(cfg.T, dtype=torch.bool, device="cuda")
+    outside[Sg] = False
+    for k in ("dB", "dF", "dX"):
+        assert not torch.any(got[k][outside]), k
+
+
+@pytest.mark.slow
+def test_large_bf16_full_size():
+    """T = 65536, d = 4096, r = 32 (batch 32 x seq 2048, 128x): the headline workload."""
+    _sampled_full_size(synth.CONFIGS["large_bf16"])
+
+
+@pytest.mark.slow
+@pytest.mark.parametrize("name", ["sweep_r512", "sweep_r128", "sweep_r64", "sweep_r32"])
+def test_sweep_full_size(name):
+    """d = 8192, T = 32768, r in {512, 128, 64, 32} (16x .. 256x compression)."""
+    _sampled_full_size(synth.CONFIGS[name], n_tokens=48)
+
+
+# ---------------------------------------------------------------------------------------------
+# The single ops, their optional arguments, and edge cases.
+# ---------------------------------------------------------------------------------------------
+
+def _ws(desc, op):
+    return resbm.workspace(desc, op)
+
+
+@pytest.mark.parametrize("path", PATHS)
+def test_single_ops_and_optional_arguments(path):
+    cfg = synth.BoundaryConfig("ops", T=700, d=384, r=32, m=32)
+    flags = PATHS[path]
+    h = host_inputs(cfg, INPUTS + ("dB", "dX0"))
+    dev = {k: to_dev(v, cfg) for k, v in h.items()}
+    desc = resbm.desc_from_config(cfg, flags)
+    T, d, r, m = cfg.T, cfg.d, cfg.r, cfg.m
+    bf = torch.bfloat16
+    B = torch.empty(T, r, dtype=bf, device="cuda")
+    P = torch.empty(T, m, dtype=torch.float32, device="cuda")
+    resbm.resbm_encode_fwd(desc, dev["X"], dev["F"], dev["We1"], dev["We2"], B, None,
+                           _ws(desc, resbm.RESBM_OP_ENCODE_FWD))
+    wantB, wantP = oracle.encode_fwd(h["X"], h["F"], h["We1"], h["We2"], cfg.act)
+    check("B", to_host(B), wantB, "bf16")
+    B2 = torch.empty_like(B)
+    resbm.resbm_encode_fwd(desc, dev["X"], dev["F"], dev["We1"], dev["We2"], B2, P,
+                           _ws(desc, resbm.RESBM_OP_ENCODE_FWD))
+    torch.cuda.synchronize()
+    assert torch.equal(B, B2)
+    check("P", to_host(P), wantP, "f32", tol=1e-4)
+    # X aliasing F (single-input variant)
+    resbm.resbm_encode_fwd(desc, dev["F"], dev["F"], dev["We1"], dev["We2"], B2, None,
+                           _ws(desc, resbm.RESBM_OP_ENCODE_FWD))
+    check("B", to_host(B2), oracle.encode_fwd(h["F"], h["F"], h["We1"], h["We2"], cfg.act)[0], "bf16")
+    # encode bwd with a given dB, with and without P_save, with and without dX
+    dF = torch.empty(T, d, dtype=bf, device="cuda")
+    dX = dev["dX0"].clone()
+    dWe1 = torch.empty(d, m, device="cuda")
+    dWe2 = torch.empty(m, r, device="cuda")
+    wdF, wdX, wdWe1, wdWe2 = oracle.encode_bwd(h["dB"], h["F"], h["We1"], h["We2"], cfg.act)
+    for Psave in (P, None):
+        dX.copy_(dev["dX0"])
+        resbm.resbm_encode_bwd(desc, dev["dB"], dev["F"], Psave, dev["We1"], dev["We2"], dF, dX,
+                               dWe1, dWe2, _ws(desc, resbm.RESBM_OP_ENCODE_BWD))
+        check("dF", to_host(dF), wdF, "bf16")
+        check("dWe1", to_host(dWe1), wdWe1, "bf16")
+        check("dWe2", to_host(dWe2), wdWe2, "bf16")
+        # dX[:, :r] += dB in bf16, other columns untouched
+        expect = h["dX0"].astype(np.float64) + wdX
+        check("dX", to_host(dX), expect, "bf16")
+        assert torch.equal(dX[:, r:], dev["dX0"][:, r:])
+    dF2 = torch.empty_like(dF)
+    resbm.resbm_encode_bwd(desc, dev["dB"], dev["F"], P, dev["We1"], dev["We2"], dF2, None,
+                           dWe1, dWe2, _ws(desc, resbm.RESBM_OP_ENCODE_BWD))
+    torch.cuda.synchronize()
+    assert torch.equal(dF, dF2)
+    # decode fwd / bwd alone
+    Y = torch.empty(T, d, dtype=bf, device="cuda")
+    resbm.resbm_decode_fwd(desc, dev["dB"], dev["Wd1"], dev["Wd2"], Y, _ws(desc, resbm.RESBM_OP_DECODE_FWD))
+    check("Y", to_host(Y), oracle.decode_fwd(h["dB"], h["Wd1"], h["Wd2"], cfg.act, cfg.merge), "bf16")
+    dB = torch.empty(T, r, dtype=bf, device="cuda")
+    dWd1 = torch.empty(r, m, device="cuda")
+    dWd2 = torch.empty(m, d, device="cuda")
+    resbm.resbm_decode_bwd(desc, dev["dY"], dev["dB"], dev["Wd1"], dev["Wd2"], dB, dWd1, dWd2,
+                           _ws(desc, resbm.RESBM_OP_DECODE_BWD))
+    wdB, wdWd1, wdWd2 = oracle.decode_bwd(h["dY"], h["dB"], h["Wd1"], h["Wd2"], cfg.act, cfg.merge)
+    check("dB", to_host(dB), wdB, "bf16")
+    check("dWd1", to_host(dWd1), wdWd1, "bf16")
+    check("dWd2", to_host(dWd2), wdWd2, "bf16")
+
+
+@pytest.mark.parametrize("path", PATHS)
+def test_zero_learned_weights_give_identity_path_bitwise(path):
+    """The identity path alone (Sec. 3.3): with zero second-layer weights B = X[:, :r] and
+    Y = pad(B) exactly; backward gives dB = dY[:, :r], dF = 0 exactly."""
+    cfg = synth.BoundaryConfig("zero", T=300, d=256, r=16, m=16)
+    h = host_inputs(cfg)
+    h["We2"] = np.zeros_like(h["We2"])
+    h["Wd2"] = np.zeros_like(h["Wd2"])
+    dev = {k: to_dev(v, cfg) for k, v in h.items()}
+    got = gpu_step(cfg, dev, flags=PATHS[path])
+    r = cfg.r
+    assert torch.equal(got["B"], dev["X"][:, :r])
+    assert torch.equal(got["Y"][:, :r], got["B"]) and not torch.any(got["Y"][:, r:])
+    assert torch.equal(got["dB"], dev["dY"][:, :r])
+    assert not torch.any(got["dF"])
+    assert torch.equal(got["dX"][:, :r], dev["dY"][:, :r]) and not torch.any(got["dX"][:, r:])
+
+
+def test_no_compression_zero_weights_is_vanilla_residual():
+    """r = d (c = C, Sec. 3.3) with zero learned weights: Y == X bit for bit."""
+    cfg = synth.BoundaryConfig("vanilla", T=256, d=64, r=64, m=16)
+    h = host_inputs(cfg)
+    h["We2"] = np.zeros_like(h["We2"])
+    h["Wd2"] = np.zeros_like(h["Wd2"])
+    dev = {k: to_dev(v, cfg) for k, v in h.items()}
+    for flags in PATHS.values():
+        got = gpu_step(cfg, dev, flags=flags)
+        assert torch.equal(got["Y"], dev["X"])
+
+
+@pytest.mark.parametrize("path", PATHS)
+def test_empty_batch_zeroes_weight_grads(path):
+    cfg = synth.BoundaryConfig("empty", T=0, d=128, r=8, m=8)
+    desc = resbm.desc_from_config(cfg, PATHS[path])
+    w = {k: to_dev(synth.tensor(cfg, k), cfg) for k in ("We1", "We2", "Wd1", "Wd2")}
+    empty = torch.empty(0, cfg.d, dtype=torch.bfloat16, device="cuda")
+    out = resbm.step_outputs(desc)
+    for k in ("dWe1", "dWe2", "dWd1", "dWd2"):
+        out[k].fill_(7.0)
+    ws = resbm.workspace(desc, resbm.RESBM_OP_BOUNDARY_STEP)
+    resbm.resbm_boundary_step(desc, ws, X=empty, F=empty, dY=empty, **w, **out)
+    torch.cuda.synchronize()
+    for k in ("dWe1", "dWe2", "dWd1", "dWd2"):
+        assert not torch.any(out[k]), k
+
+
+@pytest.mark.parametrize("path", PATHS)
+def test_deterministic(path):
+    cfg = synth.BoundaryConfig("det", T=2048, d=512, r=32, m=32)
+    h = host_inputs(cfg)
+    dev = {k: to_dev(v, cfg) for k, v in h.items()}
+    a = gpu_step(cfg, dev, flags=PATHS[path])
+    b = gpu_step(cfg, dev, flags=PATHS[path])
+    for k in OUTS + ("P",):
+        assert torch.equal(a[k], b[k]), k
+
+
+def test_workspace_too_small_is_reported_on_device():
+    cfg = synth.BoundaryConfig("ws", T=256, d=256, r=16, m=16)
+    desc = resbm.desc_from_config(cfg)
+    h = host_inputs(cfg)
+    dev = {k: to_dev(v, cfg) for k, v in h.items()}
+    out = resbm.step_outputs(desc)
+    need = resbm.resbm_workspace_bytes(desc, resbm.RESBM_OP_BOUNDARY_STEP)
+    ws = torch.empty(max(need - 256, 1), dtype=torch.uint8, device="cuda")
+    with pytest.raises(resbm.ResbmError) as e:
+        resbm.resbm_boundary_step(desc, ws, **dev, **out)
+    assert e.value.status == resbm.RESBM_ERR_WORKSPACE
+
+
+def test_runs_on_a_side_stream():
+    cfg = synth.BoundaryConfig("stream", T=512, d=256, r=16, m=16)
+    h = host_inputs(cfg)
+    dev = {k: to_dev(v, cfg) for k, v in h.items()}
+    ref = gpu_step(cfg, dev)
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        got = gpu_step(cfg, dev)
+    torch.cuda.synchronize()
+    for k in OUTS:
+        assert torch.equal(ref[k], got[k]), k
