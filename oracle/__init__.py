@@ -35,6 +35,11 @@ def _load(path=None):
     lib.oracle_dact.restype = ctypes.c_double
     lib.oracle_dact.argtypes = [ctypes.c_int, ctypes.c_double]
     lib.oracle_rect_identity.argtypes = [_i64, _i64, _dp]
+    lib.oracle_round_bf16.restype = ctypes.c_double
+    lib.oracle_round_bf16.argtypes = [ctypes.c_double]
+    lib.oracle_round_f32.restype = ctypes.c_double
+    lib.oracle_round_f32.argtypes = [ctypes.c_double]
+    lib.oracle_round_array.argtypes = [ctypes.c_int, _i64, _dp]
     lib.oracle_pid.restype = ctypes.c_int
     lib.oracle_pid.argtypes = [_i64, _i64, _i64, _dp, _dp]
     lib.oracle_encode_fwd.restype = ctypes.c_int
@@ -79,6 +84,15 @@ class Oracle:
 
     def max_threads(self):
         return int(self._l.oracle_max_threads())
+
+    # -- transfer rounding (Appendix A.3: the boundary tensors travel in bf16) ----------------
+    _BITS = {"bf16": 8, "f32": 24}
+
+    def round_to(self, x, dtype):
+        """x rounded to the transfer dtype ("bf16" or "f32"), nearest-even, from fp64."""
+        y = np.array(x, dtype=np.float64, copy=True, order="C")
+        self._l.oracle_round_array(self._BITS[dtype], y.size, self._p(y))
+        return y
 
     # -- Sec. 3.3 ---------------------------------------------------------------------------
     def act(self, act, x):
@@ -163,11 +177,18 @@ class Oracle:
             raise MemoryError("oracle_encode_bwd")
         return dF, dX, dWe1, dWe2
 
-    def boundary_step(self, X, F, dY, We1, We2, Wd1, Wd2, act="silu", merge=1):
-        """One boundary forward + backward: the four functions above chained, B handed over."""
+    def boundary_step(self, X, F, dY, We1, We2, Wd1, Wd2, act="silu", merge=1, transfer=None):
+        """One boundary forward + backward: the four functions above chained. B is handed to
+        the decoder and dB back to the encoder; with transfer = "bf16" / "f32" they are first
+        rounded to that dtype, as they are when sent across the boundary (Appendix A.3). The
+        returned B and dB are the values that crossed."""
         B, P = self.encode_fwd(X, F, We1, We2, act)
+        if transfer:
+            B = self.round_to(B, transfer)
         Y = self.decode_fwd(B, Wd1, Wd2, act, merge)
         dB, dWd1, dWd2 = self.decode_bwd(dY, B, Wd1, Wd2, act, merge)
+        if transfer:
+            dB = self.round_to(dB, transfer)
         dF, dX, dWe1, dWe2 = self.encode_bwd(dB, F, We1, We2, act)
         return dict(B=B, P=P, Y=Y, dB=dB, dF=dF, dX=dX, dWe1=dWe1, dWe2=dWe2,
                     dWd1=dWd1, dWd2=dWd2)
@@ -185,7 +206,7 @@ def default():
 
 def __getattr__(name):
     # module-level shortcuts: oracle.encode_fwd(...) etc.
-    if name in ("act", "dact", "rect_identity", "pid", "encode_fwd", "decode_fwd",
+    if name in ("act", "dact", "rect_identity", "pid", "encode_fwd", "decode_fwd", "round_to",
                 "decode_bwd", "encode_bwd", "boundary_step", "max_threads"):
         return getattr(default(), name)
     raise AttributeError(name)

@@ -19,6 +19,9 @@
  *                                                                 padded skip after attention)
  *   Backward               the chain rule of the above for the scalar  sum(dY * Y)  (decoder) and
  *                          sum(dB * B) (encoder); a gradient through y = x . M is dx = dy . M^T.
+ *   Transfer rounding      B and dB cross the boundary in the transfer dtype (Appendix A.3 counts
+ *                          them in bf16): oracle_round_array rounds them, nearest-even, before
+ *                          the receiving side uses them.
  *
  * Readings where the paper is silent (listed with the same numbers in the design notes):
  *   - hidden width m of the two-layer encoder/decoder is a free argument (Sec. 3.2 does not fix it);
@@ -138,6 +141,32 @@ static void mm_tn(int64_t M, int64_t N, int64_t K, const double *A, const double
             for (int64_t j = 0; j < N; ++j) z[j] += a * b[j];
         }
     }
+}
+
+/* ------------------------------------------------------------------------------------------ */
+/* Rounding of the tensors that cross the boundary. Appendix A.3 counts the forward activation  */
+/* b_l and the backward gradient d b_l in bf16: what the receiving side consumes is the value   */
+/* rounded to the transfer dtype. Both roundings are to nearest, ties to even, taken directly    */
+/* from the fp64 value (no intermediate fp32 rounding).                                         */
+/* ------------------------------------------------------------------------------------------ */
+
+/* Round x to `bits` significant bits (bf16: 8, fp32: 24), nearest-even; normal range only. */
+static double round_significand(double x, int bits)
+{
+    if (x == 0.0 || !isfinite(x)) return x;
+    int e;
+    double f = frexp(x, &e);                 /* x = f * 2^e, 0.5 <= |f| < 1 */
+    double scaled = ldexp(f, bits);          /* exact: |scaled| in [2^(bits-1), 2^bits) */
+    double r = nearbyint(scaled);            /* default rounding mode: to nearest, ties to even */
+    return ldexp(r, e - bits);
+}
+
+double oracle_round_bf16(double x) { return round_significand(x, 8); }
+double oracle_round_f32(double x) { return round_significand(x, 24); }
+
+void oracle_round_array(int dtype_bits, int64_t n, double *x)
+{
+    for (int64_t i = 0; i < n; ++i) x[i] = round_significand(x[i], dtype_bits);
 }
 
 static double *alloc_d(int64_t n)

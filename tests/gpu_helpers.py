@@ -40,8 +40,21 @@ def gpu_step(cfg, dev, flags=0, with_dX=True, with_P=True, dX0=None):
 
 
 def oracle_step(cfg, h):
+    """The oracle's boundary step; B and dB cross the boundary rounded to the I/O dtype."""
     return oracle.boundary_step(h["X"], h["F"], h["dY"], h["We1"], h["We2"], h["Wd1"], h["Wd2"],
-                                act=cfg.act, merge=cfg.merge)
+                                act=cfg.act, merge=cfg.merge, transfer=cfg.dtype)
+
+
+def check_output(name, got, want, cfg, dX0=None):
+    """Compare one step output (torch tensor) with the oracle's (numpy). dX is compared on its
+    first r columns (the identity-path gradient); its other columns must be untouched."""
+    from metrics import check
+    g = to_host(got)
+    if name == "dX":
+        base = np.zeros_like(g) if dX0 is None else np.asarray(dX0, np.float64)
+        assert np.array_equal(g[:, cfg.r:], base[:, cfg.r:]), "dX columns >= r were modified"
+        return check(name, g[:, :cfg.r], base[:, :cfg.r] + want[:, :cfg.r], cfg.dtype)
+    return check(name, g, want, cfg.dtype)
 
 
 def sample_tokens(T, n, seed=0, tile=128):

@@ -226,6 +226,52 @@ def pin_weight_grads_sum_over_tokens(o):
 
 
 # ---------------------------------------------------------------------------------------------
+# Transfer rounding of B and dB (they cross the boundary in bf16, Appendix A.3).
+# ---------------------------------------------------------------------------------------------
+
+def pin_transfer_rounding_nearest_even(o):
+    """bf16 keeps 8 significant bits: between 1 and 2 the spacing is 2^-7. Ties go to the even
+    neighbour, values past a tie go up even when fp32 could not hold them, and rounding to
+    fp32 keeps 24 bits."""
+    r = lambda v: float(o.round_to(np.array([v]), "bf16")[0])  # noqa: E731
+    assert r(1.0 + 2 ** -8) == 1.0                       # tie -> even (1.0)
+    assert r(1.0 + 3 * 2 ** -8) == 1.0 + 2 ** -6         # tie -> even (1 + 2^-6)
+    assert r(-(1.0 + 3 * 2 ** -8)) == -(1.0 + 2 ** -6)
+    assert r(1.0 + 2 ** -8 + 2 ** -40) == 1.0 + 2 ** -7  # just above the tie: up
+    assert r(1.0 + 2 ** -8 - 2 ** -40) == 1.0            # just below: down
+    assert r(3.0 * 2 ** 70) == 3.0 * 2 ** 70 and r(0.0) == 0.0
+    assert r(255.5) == 256.0 and r(254.5) == 254.0       # 8 bits: 254 and 256 are neighbours
+    f = lambda v: float(o.round_to(np.array([v]), "f32")[0])  # noqa: E731
+    assert f(1.0 + 2 ** -24) == 1.0 and f(1.0 + 3 * 2 ** -24) == 1.0 + 2 ** -22
+    assert f(1.0 + 2 ** -23) == 1.0 + 2 ** -23
+
+
+def pin_transfer_rounding_matches_torch_on_fp32_values(o):
+    import torch
+    x = (np.random.default_rng(7).standard_normal(20000) * 30).astype(np.float32)
+    want = torch.from_numpy(x).to(torch.bfloat16).double().numpy()
+    np.testing.assert_array_equal(o.round_to(x.astype(np.float64), "bf16"), want)
+    y = np.random.default_rng(8).standard_normal(20000) * 1e3
+    np.testing.assert_array_equal(o.round_to(y, "f32"), y.astype(np.float32).astype(np.float64))
+
+
+def pin_step_hands_over_rounded_tensors(o):
+    """With bf16 transfer, the decoder sees the bf16 value of B and the encoder backward the
+    bf16 value of dB: the step equals the single ops chained on the rounded tensors."""
+    T, d, r, m = 5, 16, 4, 3
+    X, F, dY = _rand((T, d), 111), _rand((T, d), 112), _rand((T, d), 113)
+    w = _weights(d, r, m, 114)
+    s = o.boundary_step(X, F, dY, w["We1"], w["We2"], w["Wd1"], w["Wd2"], transfer="bf16")
+    B, _ = o.encode_fwd(X, F, w["We1"], w["We2"])
+    Bq = o.round_to(B, "bf16")
+    assert np.array_equal(s["B"], Bq) and not np.array_equal(Bq, B)
+    np.testing.assert_array_equal(s["Y"], o.decode_fwd(Bq, w["Wd1"], w["Wd2"]))
+    dB, _, _ = o.decode_bwd(dY, Bq, w["Wd1"], w["Wd2"])
+    np.testing.assert_array_equal(s["dB"], o.round_to(dB, "bf16"))
+    np.testing.assert_array_equal(s["dF"], o.encode_bwd(o.round_to(dB, "bf16"), F, w["We1"], w["We2"])[0])
+
+
+# ---------------------------------------------------------------------------------------------
 # Appendix A.3 / Sec. 4.1: what crosses the boundary.
 # ---------------------------------------------------------------------------------------------
 

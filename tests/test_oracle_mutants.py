@@ -31,6 +31,9 @@ MUTANTS = {
     "transposed_operand_in_nt_product": ("acc += A[i * K + k] * B[j * K + k];",
                                          "acc += A[i * K + k] * B[k * N + j];"),
     "encoder_reads_decoder_order": ("mm_nn(T, r, m, A, We2, E);", "mm_nn(T, r, m, P, We2, E);"),
+    "rounding_ties_away_from_zero": ("double r = nearbyint(scaled);", "double r = round(scaled);"),
+    "rounding_keeps_one_bit_less": ("double scaled = ldexp(f, bits);",
+                                    "double scaled = ldexp(f, bits - 1);"),
 }
 
 

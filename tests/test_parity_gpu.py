@@ -3,7 +3,8 @@ import numpy as np
 import pytest
 import torch
 
-from gpu_helpers import INPUTS, gpu_step, host_inputs, oracle_step, sample_tokens, to_dev, to_host
+from gpu_helpers import (INPUTS, check_output, gpu_step, host_inputs, oracle_step, sample_tokens,
+                         to_dev, to_host)
 from metrics import TOL, check
 from paper_2604_11947_gb300 import resbm, synth
 
@@ -30,10 +31,7 @@ SMALL = {
 
 
 def _compare_all(cfg, got, want):
-    errs = {}
-    for k in OUTS:
-        errs[k] = check(k, to_host(got[k]), want[k], cfg.dtype)
-    return errs
+    return {k: check_output(k, got[k], want[k], cfg) for k in OUTS}
 
 
 @pytest.mark.parametrize("path", PATHS)
@@ -86,7 +84,7 @@ def _sampled_full_size(cfg, n_tokens=96, flags=0):
     Sg = torch.from_numpy(S).cuda()
     got = gpu_step(cfg, dev, flags=flags)
     for k in ("B", "Y", "dB", "dF", "dX"):
-        check(k, to_host(got[k][Sg]), want[k], cfg.dtype)
+        check_output(k, got[k][Sg], want[k], cfg)
     del got
     dY_masked = torch.zeros_like(dev["dY"])
     dY_masked[Sg] = dev["dY"][Sg]
@@ -95,7 +93,7 @@ def _sampled_full_size(cfg, n_tokens=96, flags=0):
     for k in ("dWe1", "dWe2", "dWd1", "dWd2"):
         check(k, to_host(got[k]), want[k], cfg.dtype)
     for k in ("dB", "dF", "dX"):
-        check(k, to_host(got[k][Sg]), want[k], cfg.dtype)
+        check_output(k, got[k][Sg], want[k], cfg)
     outside = torch.ones(cfg.T, dtype=torch.bool, device="cuda")
     outside[Sg] = False
     for k in ("dB", "dF", "dX"):
