@@ -14,8 +14,9 @@
 namespace resbm {
 namespace tc {
 
-// Error word written by kernels (0 = no error); read by resbm_device_error().
-extern __device__ unsigned int g_resbm_device_error;
+// Error word written by the kernels of the one translation unit that includes this header
+// (0 = no error); the host reads it with cudaMemcpyFromSymbol from that unit.
+static __device__ unsigned int g_resbm_device_error = 0;
 
 enum : unsigned {
     kErrWaitTimeout = 1u,   // an mbarrier wait exceeded kWaitNs
