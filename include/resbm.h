@@ -124,6 +124,13 @@ RESBM_API int resbm_last_cuda_error(void);
  * threads): lets a caller account for the GPU work behind a sequence of calls. */
 RESBM_API uint64_t resbm_kernel_launches(void);
 
+/* Error word of the tensor-core kernels on the current device (0: none). Every wait inside
+ * those kernels gives up after a bounded time instead of spinning forever; a kernel that gave
+ * up sets a bit here (1: a wait timed out) and returns, leaving its outputs undefined.
+ * Reading the word synchronizes with the device (it is a device-to-host copy). With clear != 0
+ * a non-zero word is reset to 0. */
+RESBM_API resbm_status resbm_device_error(unsigned int *code, int clear);
+
 /* Scratch bytes that `op` (a resbm_op) needs for `desc`, written to *bytes.
  * Returns RESBM_ERR_INVALID_ARG for a bad descriptor or op. Does not touch the GPU. */
 RESBM_API resbm_status resbm_workspace_bytes(const resbm_desc *desc, int op, size_t *bytes);

@@ -47,6 +47,26 @@ resbm_status make_ctx(void *stream, Ctx *c)
     return RESBM_OK;
 }
 
+// SM count that sizes the scratch memory: the current device's, or kDefaultSms when no device
+// can be queried (the tensor-core backward kernels keep one partial slot per CTA).
+constexpr int kDefaultSms = 160;
+int sizing_sms()
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        cudaGetLastError();
+        return kDefaultSms;
+    }
+    int sms = (dev >= 0 && dev < kMaxDevices) ? g_sm_count[dev].load(std::memory_order_relaxed) : 0;
+    if (sms > 0) return sms;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0) {
+        cudaGetLastError();
+        return kDefaultSms;
+    }
+    if (dev >= 0 && dev < kMaxDevices) g_sm_count[dev].store(sms, std::memory_order_relaxed);
+    return sms;
+}
+
 size_t elem_size(const resbm_desc &d) { return d.dtype == RESBM_BF16 ? 2 : 4; }
 
 bool mul_ok(int64_t a, int64_t b) { return a >= 0 && b >= 0 && (a == 0 || b <= INT64_MAX / a); }
@@ -104,7 +124,7 @@ bool use_tc(const resbm_desc &d, int op) { return !(d.flags & RESBM_FLAG_GENERIC
 size_t ws_for(const resbm_desc &d, int op)
 {
     size_t g = generic_ws_bytes(d, op);
-    size_t t = tc_supported(d, op) ? tc_ws_bytes(d, op) : 0;
+    size_t t = tc_supported(d, op) ? tc_ws_bytes(d, op, sizing_sms()) : 0;
     return g > t ? g : t;
 }
 
@@ -203,11 +223,16 @@ resbm_status validate_encode_bwd(const resbm_desc &d, const void *dB, const void
 }
 
 // ---- per-op execution (after validation) -----------------------------------------------------
+// A tensor-core launcher answers cudaErrorNotSupported (before launching anything) when it
+// cannot take the call, e.g. for pointers that are not 16-byte aligned; the portable kernels run.
 resbm_status run_encode_fwd(const resbm_desc &d, const void *X, const void *F, const void *We1,
                             const void *We2, void *B, float *P, void *ws, const Ctx &c)
 {
     if (d.T == 0) return RESBM_OK;
-    if (use_tc(d, RESBM_OP_ENCODE_FWD)) return finish(tc_encode_fwd(d, X, F, We1, We2, B, P, ws, c));
+    if (use_tc(d, RESBM_OP_ENCODE_FWD)) {
+        cudaError_t e = tc_encode_fwd(d, X, F, We1, We2, B, P, ws, c);
+        if (e != cudaErrorNotSupported) return finish(e);
+    }
     return finish(generic_encode_fwd(d, X, F, We1, We2, B, P, ws, c));
 }
 
@@ -215,7 +240,10 @@ resbm_status run_decode_fwd(const resbm_desc &d, const void *B, const void *Wd1,
                             void *Y, void *ws, const Ctx &c)
 {
     if (d.T == 0) return RESBM_OK;
-    if (use_tc(d, RESBM_OP_DECODE_FWD)) return finish(tc_decode_fwd(d, B, Wd1, Wd2, Y, ws, c));
+    if (use_tc(d, RESBM_OP_DECODE_FWD)) {
+        cudaError_t e = tc_decode_fwd(d, B, Wd1, Wd2, Y, ws, c);
+        if (e != cudaErrorNotSupported) return finish(e);
+    }
     return finish(generic_decode_fwd(d, B, Wd1, Wd2, Y, ws, c));
 }
 
@@ -227,8 +255,10 @@ resbm_status run_decode_bwd(const resbm_desc &d, const void *dY, const void *B, 
         resbm_status s = zero_f32(dWd1, d.r * d.m, c.stream);
         return s != RESBM_OK ? s : zero_f32(dWd2, d.m * d.d, c.stream);
     }
-    if (use_tc(d, RESBM_OP_DECODE_BWD))
-        return finish(tc_decode_bwd(d, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, c));
+    if (use_tc(d, RESBM_OP_DECODE_BWD)) {
+        cudaError_t e = tc_decode_bwd(d, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, c);
+        if (e != cudaErrorNotSupported) return finish(e);
+    }
     return finish(generic_decode_bwd(d, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, c));
 }
 
@@ -240,8 +270,10 @@ resbm_status run_encode_bwd(const resbm_desc &d, const void *dB, const void *F, 
         resbm_status s = zero_f32(dWe1, d.d * d.m, c.stream);
         return s != RESBM_OK ? s : zero_f32(dWe2, d.m * d.r, c.stream);
     }
-    if (use_tc(d, RESBM_OP_ENCODE_BWD))
-        return finish(tc_encode_bwd(d, dB, F, P, We1, We2, dF, dX, dWe1, dWe2, ws, c));
+    if (use_tc(d, RESBM_OP_ENCODE_BWD)) {
+        cudaError_t e = tc_encode_bwd(d, dB, F, P, We1, We2, dF, dX, dWe1, dWe2, ws, c);
+        if (e != cudaErrorNotSupported) return finish(e);
+    }
     return finish(generic_encode_bwd(d, dB, F, P, We1, We2, dF, dX, dWe1, dWe2, ws, c));
 }
 
@@ -266,6 +298,14 @@ const char *resbm_status_string(resbm_status s)
 int resbm_last_cuda_error(void) { return g_last_cuda_error; }
 
 uint64_t resbm_kernel_launches(void) { return g_launches.load(std::memory_order_relaxed); }
+
+resbm_status resbm_device_error(unsigned int *code, int clear)
+{
+    if (!code) return RESBM_ERR_INVALID_ARG;
+    *code = 0;
+    cudaError_t e = tc_device_error(code, clear != 0);
+    return e == cudaSuccess ? RESBM_OK : cuda_fail(e);
+}
 
 resbm_status resbm_workspace_bytes(const resbm_desc *desc, int op, size_t *bytes)
 {

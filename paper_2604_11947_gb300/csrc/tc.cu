@@ -1,31 +1,258 @@
-// tc.cu -- sm_103a tensor-core kernels of the ResBM boundary bottleneck.
+// tc.cu -- host side of the sm_103a tensor-core kernels (tcgen05 + TMA) of the ResBM boundary.
+//
+// All tensor-core kernels are compiled in this one translation unit (they share the device
+// error word of tc_common.cuh). Tensor maps are encoded per call through the driver entry point
+// cuTensorMapEncodeTiled (no link-time dependency on libcuda).
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_runtime.h>
+
+#include <atomic>
+#include <mutex>
+
 #include "tc.h"
+#include "tc_common.cuh"
+#include "tc_dec_fwd.cuh"
+#include "tc_enc_fwd.cuh"
+#include "tc_dec_bwd.cuh"
 
 namespace resbm {
 
-bool tc_supported(const resbm_desc &, int) { return false; }
-size_t tc_ws_bytes(const resbm_desc &, int) { return 0; }
+namespace {
 
-cudaError_t tc_encode_fwd(const resbm_desc &, const void *, const void *, const void *,
-                          const void *, void *, float *, void *, const Ctx &)
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
+{
+    static std::once_flag once;
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    });
+    return fn;
+}
+
+// 2D bf16 tensor map over a row-major matrix (outer rows x inner columns, row pitch in bytes).
+bool make_map(CUtensorMap *m, const void *ptr, uint64_t inner, uint64_t outer, uint64_t pitch_bytes,
+              uint32_t box_inner, uint32_t box_outer, CUtensorMapSwizzle swz)
+{
+    auto fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[2] = {inner, outer};
+    cuuint64_t strides[1] = {pitch_bytes};
+    cuuint32_t box[2] = {box_inner, box_outer};
+    cuuint32_t es[2] = {1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), dims, strides, box, es,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool al16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Dynamic shared memory attribute, set once per (kernel, device): `done` is the calling
+// launcher's own per-device flag array (one per kernel instantiation).
+constexpr int kMaxDev = 64;
+template <typename K>
+cudaError_t ensure_smem(K kernel, uint32_t bytes, int dev, std::atomic<uint8_t> (&done)[kMaxDev])
+{
+    if (dev >= 0 && dev < kMaxDev && done[dev].load(std::memory_order_acquire)) return cudaSuccess;
+    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+    if (e == cudaSuccess && dev >= 0 && dev < kMaxDev) done[dev].store(1, std::memory_order_release);
+    return e;
+}
+
+bool tc_width_ok(int64_t m) { return m == 16 || m == 32 || m == 64 || m == 128; }
+
+int grid_tokens(const Ctx &c, int64_t T)
+{
+    int64_t g = (T + 15) / 16;
+    if (g > c.sm_count) g = c.sm_count;
+    return (int)(g < 1 ? 1 : g);
+}
+
+template <int M>
+cudaError_t launch_dec_fwd(const resbm_desc &d, const void *B, const void *Wd1, const void *Wd2, void *Y,
+                           const Ctx &c)
+{
+    using Cfg = tc::DecFwdCfg<M>;
+    CUtensorMap m_wd2, m_y128, m_y16;
+    if (!make_map(&m_wd2, Wd2, d.d, d.m, d.d * 2, 64, M, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&m_y128, Y, d.d, d.T, d.d * 2, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&m_y16, Y, d.d, d.T, d.d * 2, 64, 16, CU_TENSOR_MAP_SWIZZLE_128B))
+        return cudaErrorInvalidValue;
+    static std::atomic<uint8_t> smem_set[kMaxDev];
+    cudaError_t e = ensure_smem(tc::k_dec_fwd<M>, Cfg::SMEM_BYTES, c.device, smem_set);
+    if (e != cudaSuccess) return e;
+    tc::DecFwdArgs a{static_cast<const __nv_bfloat16 *>(B), static_cast<const __nv_bfloat16 *>(Wd1), d.T, d.d,
+                     d.act, d.merge_identity};
+    tc::k_dec_fwd<M><<<grid_tokens(c, d.T), Cfg::THREADS, Cfg::SMEM_BYTES, c.stream>>>(m_wd2, m_y128, m_y16, a);
+    count_launches(1);
+    return cudaGetLastError();
+}
+
+template <int M>
+cudaError_t launch_enc_fwd(const resbm_desc &d, const void *X, const void *F, const void *We1, const void *We2,
+                           void *B, float *P, const Ctx &c)
+{
+    using Cfg = tc::EncFwdCfg<M>;
+    const CUtensorMapSwizzle wswz = Cfg::WSW == 128  ? CU_TENSOR_MAP_SWIZZLE_128B
+                                    : Cfg::WSW == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                                     : CU_TENSOR_MAP_SWIZZLE_32B;
+    CUtensorMap m_f128, m_f16, m_we1;
+    if (!make_map(&m_f128, F, d.d, d.T, d.d * 2, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&m_f16, F, d.d, d.T, d.d * 2, 64, 16, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&m_we1, We1, d.m, d.d, d.m * 2, Cfg::WSW / 2, 64, wswz))
+        return cudaErrorInvalidValue;
+    static std::atomic<uint8_t> smem_set[kMaxDev];
+    cudaError_t e = ensure_smem(tc::k_enc_fwd<M>, Cfg::SMEM_BYTES, c.device, smem_set);
+    if (e != cudaSuccess) return e;
+    tc::EncFwdArgs a{static_cast<const __nv_bfloat16 *>(X), static_cast<const __nv_bfloat16 *>(We2),
+                     static_cast<__nv_bfloat16 *>(B), P, d.T, d.d, d.act};
+    tc::k_enc_fwd<M><<<grid_tokens(c, d.T), Cfg::THREADS, Cfg::SMEM_BYTES, c.stream>>>(m_f128, m_f16, m_we1, a);
+    count_launches(1);
+    return cudaGetLastError();
+}
+
+// Partial-slot layout of the backward kernels: one slot per (CTA, group of NT tiles).
+struct BwdPlan {
+    int grid = 1, max_groups = 1;
+    int64_t slots = 1;
+    float *part_big = nullptr;    // slots x d x m
+    float *part_small = nullptr;  // slots x small_elems
+    size_t bytes = 0;
+};
+
+BwdPlan bwd_plan(const resbm_desc &d, int sms, int nt, int64_t small_elems, void *ws)
+{
+    BwdPlan p;
+    int64_t g = (d.T + 15) / 16;
+    if (g > sms) g = sms;
+    p.grid = (int)(g < 1 ? 1 : g);
+    const int64_t U = (d.T + 15) / 16;
+    const int64_t max_tokens = 16 * ((U + p.grid - 1) / p.grid);
+    const int64_t max_tiles = (max_tokens + 127) / 128;
+    p.max_groups = (int)((max_tiles + nt - 1) / nt);
+    if (p.max_groups < 1) p.max_groups = 1;
+    p.slots = (int64_t)p.grid * p.max_groups;
+    WsCarver w(ws);
+    p.part_big = w.take<float>(p.slots * d.d * d.m);
+    p.part_small = w.take<float>(p.slots * small_elems);
+    p.bytes = w.used;
+    return p;
+}
+
+int reduce_grid(int64_t n, const Ctx &c)
+{
+    int64_t g = (n + 255) / 256;
+    const int64_t cap = (int64_t)c.sm_count * 4;
+    if (g > cap) g = cap;
+    return (int)(g < 1 ? 1 : g);
+}
+
+template <int M>
+cudaError_t launch_dec_bwd(const resbm_desc &d, const void *dY, const void *B, const void *Wd1, const void *Wd2,
+                           void *dB, float *dWd1, float *dWd2, void *ws, const Ctx &c)
+{
+    using Cfg = tc::DecBwdCfg<M>;
+    const BwdPlan p = bwd_plan(d, c.sm_count, Cfg::NT, d.r * d.m, ws);
+    CUtensorMap m_dy128, m_dy16, m_wd2;
+    if (!make_map(&m_dy128, dY, d.d, d.T, d.d * 2, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&m_dy16, dY, d.d, d.T, d.d * 2, 64, 16, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&m_wd2, Wd2, d.d, d.m, d.d * 2, 64, M, CU_TENSOR_MAP_SWIZZLE_128B))
+        return cudaErrorInvalidValue;
+    static std::atomic<uint8_t> smem_set[kMaxDev];
+    cudaError_t e = ensure_smem(tc::k_dec_bwd<M>, Cfg::SMEM_BYTES, c.device, smem_set);
+    if (e != cudaSuccess) return e;
+    tc::DecBwdArgs a{static_cast<const __nv_bfloat16 *>(B), static_cast<const __nv_bfloat16 *>(Wd1),
+                     static_cast<const __nv_bfloat16 *>(dY), static_cast<__nv_bfloat16 *>(dB), p.part_big,
+                     p.part_small, d.T, d.d, d.act, d.merge_identity, p.max_groups};
+    tc::k_dec_bwd<M><<<p.grid, Cfg::THREADS, Cfg::SMEM_BYTES, c.stream>>>(m_dy128, m_dy16, m_wd2, a);
+    count_launches(1);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    // dWd2 (m x d) = sum of the d x m slices, transposed; dWd1 (r x m) = sum of the slices
+    tc::k_reduce_slots<<<reduce_grid(d.d * d.m, c), 256, 0, c.stream>>>(p.part_big, p.slots, d.d, d.m, dWd2, 1);
+    tc::k_reduce_slots<<<reduce_grid(d.r * d.m, c), 256, 0, c.stream>>>(p.part_small, p.slots, d.r, d.m, dWd1, 0);
+    count_launches(2);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+bool tc_supported(const resbm_desc &d, int op)
+{
+    if (d.dtype != RESBM_BF16 || d.m != d.r || !tc_width_ok(d.m)) return false;
+    if (d.T > INT32_MAX || encode_fn() == nullptr) return false;
+    if (op == RESBM_OP_DECODE_FWD) {
+        const int64_t nch = d.m <= 32 ? 256 : 128;
+        return d.d % nch == 0;
+    }
+    if (op == RESBM_OP_ENCODE_FWD) return d.d % 64 == 0;
+    if (op == RESBM_OP_DECODE_BWD) return d.m <= 64 && d.d % 128 == 0;
+    return false;
+}
+
+size_t tc_ws_bytes(const resbm_desc &d, int op, int sms)
+{
+    if (op == RESBM_OP_DECODE_BWD) return bwd_plan(d, sms, 4, d.r * d.m, nullptr).bytes;
+    return 0;
+}
+
+cudaError_t tc_encode_fwd(const resbm_desc &d, const void *X, const void *F, const void *We1, const void *We2,
+                          void *B, float *P, void *, const Ctx &c)
+{
+    if (!al16(X) || !al16(F) || !al16(We1) || !al16(We2) || !al16(B) || (P && !al16(P)))
+        return cudaErrorNotSupported;
+    switch (d.m) {
+    case 16: return launch_enc_fwd<16>(d, X, F, We1, We2, B, P, c);
+    case 32: return launch_enc_fwd<32>(d, X, F, We1, We2, B, P, c);
+    case 64: return launch_enc_fwd<64>(d, X, F, We1, We2, B, P, c);
+    case 128: return launch_enc_fwd<128>(d, X, F, We1, We2, B, P, c);
+    }
+    return cudaErrorNotSupported;
+}
+
+cudaError_t tc_decode_fwd(const resbm_desc &d, const void *B, const void *Wd1, const void *Wd2, void *Y, void *,
+                          const Ctx &c)
+{
+    if (!al16(B) || !al16(Wd1) || !al16(Wd2) || !al16(Y)) return cudaErrorNotSupported;
+    switch (d.m) {
+    case 16: return launch_dec_fwd<16>(d, B, Wd1, Wd2, Y, c);
+    case 32: return launch_dec_fwd<32>(d, B, Wd1, Wd2, Y, c);
+    case 64: return launch_dec_fwd<64>(d, B, Wd1, Wd2, Y, c);
+    case 128: return launch_dec_fwd<128>(d, B, Wd1, Wd2, Y, c);
+    }
+    return cudaErrorNotSupported;
+}
+
+cudaError_t tc_decode_bwd(const resbm_desc &d, const void *dY, const void *B, const void *Wd1, const void *Wd2,
+                          void *dB, float *dWd1, float *dWd2, void *ws, const Ctx &c)
+{
+    if (!al16(dY) || !al16(B) || !al16(Wd1) || !al16(Wd2) || !al16(dB)) return cudaErrorNotSupported;
+    switch (d.m) {
+    case 16: return launch_dec_bwd<16>(d, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, c);
+    case 32: return launch_dec_bwd<32>(d, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, c);
+    case 64: return launch_dec_bwd<64>(d, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, c);
+    }
+    return cudaErrorNotSupported;
+}
+
+cudaError_t tc_encode_bwd(const resbm_desc &, const void *, const void *, const float *, const void *,
+                          const void *, void *, void *, float *, float *, void *, const Ctx &)
 {
     return cudaErrorNotSupported;
 }
-cudaError_t tc_decode_fwd(const resbm_desc &, const void *, const void *, const void *, void *,
-                          void *, const Ctx &)
+
+cudaError_t tc_device_error(unsigned int *code, bool clear)
 {
-    return cudaErrorNotSupported;
-}
-cudaError_t tc_decode_bwd(const resbm_desc &, const void *, const void *, const void *,
-                          const void *, void *, float *, float *, void *, const Ctx &)
-{
-    return cudaErrorNotSupported;
-}
-cudaError_t tc_encode_bwd(const resbm_desc &, const void *, const void *, const float *,
-                          const void *, const void *, void *, void *, float *, float *, void *,
-                          const Ctx &)
-{
-    return cudaErrorNotSupported;
+    cudaError_t e = cudaMemcpyFromSymbol(code, tc::g_resbm_device_error, sizeof(unsigned int));
+    if (e == cudaSuccess && clear && *code) {
+        const unsigned int zero = 0;
+        e = cudaMemcpyToSymbol(tc::g_resbm_device_error, &zero, sizeof(zero));
+    }
+    return e;
 }
 
 }  // namespace resbm

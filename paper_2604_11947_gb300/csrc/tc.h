@@ -8,7 +8,11 @@ namespace resbm {
 // Whether the tensor-core kernels handle this descriptor for `op` (bf16 I/O, shapes that fit
 // their tiles); otherwise the portable kernels run.
 bool tc_supported(const resbm_desc &d, int op);
-size_t tc_ws_bytes(const resbm_desc &d, int op);
+
+// Reads (and optionally clears) the error word of the tensor-core kernels; synchronizing.
+cudaError_t tc_device_error(unsigned int *code, bool clear);
+// Scratch bytes of the tensor-core kernels for `op` on a device with `sms` SMs.
+size_t tc_ws_bytes(const resbm_desc &d, int op, int sms);
 
 cudaError_t tc_encode_fwd(const resbm_desc &d, const void *X, const void *F, const void *We1,
                           const void *We2, void *B, float *P_save, void *ws, const Ctx &c);

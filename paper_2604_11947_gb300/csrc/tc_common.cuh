@@ -42,6 +42,54 @@ __device__ __forceinline__ void flag_error(unsigned code)
     atomicOr(&g_resbm_device_error, code);
 }
 
+// Token range [start, end) of CTA b out of G over T tokens: T is cut into 16-token units and
+// every CTA gets a contiguous run of floor or ceil(units / G) of them (balanced to 16 tokens).
+__device__ __forceinline__ void token_range(int64_t T, int b, int G, int64_t &start, int64_t &end)
+{
+    const int64_t U = (T + 15) / 16;
+    start = 16 * ((U * b) / G);
+    end = 16 * ((U * (b + 1)) / G);
+    if (end > T) end = T;
+    if (start > T) start = T;
+}
+
+// ---- small per-token products on CUDA cores (fp32 accumulate) ---------------------------------
+// acc[0..16) = sum over k of x[k] * W[k][n0 .. n0 + 16), W a K x N row-major bf16 matrix in
+// shared memory (rows 16-byte aligned); k runs in order 0, 1, ..., K-1.
+template <int K, int N>
+__device__ __forceinline__ void vecmat16(const float (&x)[K], const __nv_bfloat16 *W, int n0, float (&acc)[16])
+{
+#pragma unroll
+    for (int i = 0; i < 16; ++i) acc[i] = 0.0f;
+#pragma unroll
+    for (int k = 0; k < K; ++k) {
+        const uint4 *w = reinterpret_cast<const uint4 *>(W + k * N + n0);
+        const uint4 w0 = w[0], w1 = w[1];
+        const uint32_t wv[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            acc[2 * j] = fmaf(x[k], __uint_as_float(wv[j] << 16), acc[2 * j]);
+            acc[2 * j + 1] = fmaf(x[k], __uint_as_float(wv[j] & 0xFFFF0000u), acc[2 * j + 1]);
+        }
+    }
+}
+
+// A row of N bf16 values (16-byte aligned, N % 8 == 0) as fp32.
+template <int N> __device__ __forceinline__ void load_bf16_row(const __nv_bfloat16 *src, float (&x)[N])
+{
+    const uint4 *s = reinterpret_cast<const uint4 *>(src);
+#pragma unroll
+    for (int v = 0; v < N / 8; ++v) {
+        const uint4 u = s[v];
+        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            x[8 * v + 2 * e] = __uint_as_float(w[e] << 16);
+            x[8 * v + 2 * e + 1] = __uint_as_float(w[e] & 0xFFFF0000u);
+        }
+    }
+}
+
 // ---- mbarrier ---------------------------------------------------------------------------------
 __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count)
 {

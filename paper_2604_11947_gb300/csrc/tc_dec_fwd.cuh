@@ -21,7 +21,7 @@ namespace tc {
 template <int M_> struct DecFwdCfg {
     static constexpr int M = M_;                       // hidden width m (= r on this path)
     static constexpr int R = M_;                       // bottleneck width r
-    static constexpr int NCH = M_ <= 64 ? 256 : 128;   // Y columns per MMA chunk
+    static constexpr int NCH = M_ <= 32 ? 256 : 128;   // Y columns per MMA chunk
     static constexpr int NSTAGE = M_ <= 64 ? 3 : 2;    // Wd2 chunk ring depth
     static constexpr int KBLK = (M_ + 63) / 64;        // 64-wide K blocks of G
     static constexpr uint32_t W_STAGE_BYTES = M_ * NCH * 2;
@@ -44,16 +44,6 @@ struct DecFwdArgs {
     int64_t T, d;
     int act, merge;
 };
-
-// Token range [start, end) of CTA b out of G over T tokens, in 16-token units.
-__device__ __forceinline__ void token_range(int64_t T, int b, int G, int64_t &start, int64_t &end)
-{
-    const int64_t U = (T + 15) / 16;
-    start = 16 * ((U * b) / G);
-    end = 16 * ((U * (b + 1)) / G);
-    if (end > T) end = T;
-    if (start > T) start = T;
-}
 
 template <int M_>
 __global__ void __launch_bounds__(192, 1)
@@ -104,13 +94,17 @@ __global__ void __launch_bounds__(192, 1)
             uint32_t it = 0;
             bool ok = true;
             for (int64_t t0 = start; t0 < end && ok; t0 += 128) {
-                for (int c = 0; c < nchunks && ok; ++c, ++it) {
+                for (int c = 0; c < nchunks; ++c) {
                     const uint32_t s = it % C::NSTAGE, ph = (it / C::NSTAGE) & 1;
-                    ok = mbar_wait(smem_u32(&w_empty[s]), ph ^ 1);
+                    if (!mbar_wait(smem_u32(&w_empty[s]), ph ^ 1)) {
+                        ok = false;
+                        break;
+                    }
                     const uint32_t dst = smem_u32(smem + C::OFF_W + s * C::W_STAGE_BYTES);
                     mbar_expect_tx(smem_u32(&w_full[s]), C::W_STAGE_BYTES);
                     for (int b = 0; b < C::NCH / 64; ++b)
                         tma_load_2d(dst + b * (C::M * 128), &tm_wd2, c * C::NCH + 64 * b, 0, smem_u32(&w_full[s]));
+                    ++it;
                 }
             }
             // drain: every issued load has landed before the CTA can exit
@@ -187,7 +181,7 @@ __global__ void __launch_bounds__(192, 1)
                 float accq[16];
 #pragma unroll
                 for (int j = 0; j < 16; ++j) accq[j] = 0.0f;
-#pragma unroll 4
+#pragma unroll
                 for (int k = 0; k < C::R; ++k) {
                     const uint32_t bb = brow[k >> 1];
                     const float bk = __uint_as_float((k & 1) ? (bb & 0xFFFF0000u) : (bb << 16));
@@ -228,18 +222,21 @@ __global__ void __launch_bounds__(192, 1)
                 if (et == 0) bulk_wait_read<1>();  // staging buffer sb is free again
                 named_barrier(1, 128);
                 uint8_t *stg = smem + C::OFF_STG + sb * C::STG_BYTES;
-                const int ncols = (int)min<int64_t>(C::NCH, a.d - (int64_t)c * C::NCH);
-                for (int g = 0; g < ncols / 32; ++g) {
+                const int64_t left = a.d - (int64_t)c * C::NCH;
+                const int ncols = left < C::NCH ? (int)left : C::NCH;
+#pragma unroll
+                for (int g = 0; g < C::NCH / 32; ++g) {
+                    if (g * 32 >= ncols) break;
                     float v[32];
                     tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + ab * C::NCH + g * 32, v);
                     tmem_ld_wait();
-                    const int col0 = c * C::NCH + g * 32;
-                    if (a.merge && col0 < C::R) {
+                    // identity path: the first r columns of Y get B (only chunk 0 holds them)
+                    if (g * 32 < C::R && a.merge && c == 0) {
 #pragma unroll
                         for (int i = 0; i < 32; ++i) {
-                            if (col0 + i < C::R) {
-                                const uint32_t bb = brow[(col0 + i) >> 1];
-                                v[i] += __uint_as_float(((col0 + i) & 1) ? (bb & 0xFFFF0000u) : (bb << 16));
+                            if (g * 32 + i < C::R) {
+                                const uint32_t bb = brow[(g * 32 + i) >> 1];
+                                v[i] += __uint_as_float(((g * 32 + i) & 1) ? (bb & 0xFFFF0000u) : (bb << 16));
                             }
                         }
                     }

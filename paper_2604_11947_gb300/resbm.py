@@ -26,6 +26,7 @@ DTYPES = {"f32": RESBM_F32, "bf16": RESBM_BF16}
 TORCH_DTYPES = {RESBM_F32: torch.float32, RESBM_BF16: torch.bfloat16}
 
 EXPORTS = ("resbm_version", "resbm_status_string", "resbm_last_cuda_error", "resbm_kernel_launches",
+           "resbm_device_error",
            "resbm_workspace_bytes", "resbm_encode_fwd", "resbm_decode_fwd", "resbm_decode_bwd",
            "resbm_encode_bwd", "resbm_boundary_step")
 
@@ -75,6 +76,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.resbm_status_string.argtypes = [i32]
     lib.resbm_last_cuda_error.restype = i32
     lib.resbm_kernel_launches.restype = ctypes.c_uint64
+    lib.resbm_device_error.restype = i32
+    lib.resbm_device_error.argtypes = [ctypes.POINTER(ctypes.c_uint), i32]
     lib.resbm_workspace_bytes.restype = i32
     lib.resbm_workspace_bytes.argtypes = [D, i32, ctypes.POINTER(sz)]
     lib.resbm_encode_fwd.restype = i32
@@ -102,6 +105,13 @@ def resbm_version() -> str:
 
 def resbm_kernel_launches() -> int:
     return int(load().resbm_kernel_launches())
+
+
+def resbm_device_error(clear=False) -> int:
+    """The tensor-core kernels' error word (synchronizes with the device)."""
+    out = ctypes.c_uint(0)
+    _check("resbm_device_error", load().resbm_device_error(ctypes.byref(out), int(bool(clear))))
+    return int(out.value)
 
 
 def make_desc(T, d, r, m, dtype="bf16", act="silu", merge_identity=1, flags=0) -> resbm_desc:
