@@ -15,6 +15,7 @@
 #include "tc_dec_fwd.cuh"
 #include "tc_enc_fwd.cuh"
 #include "tc_dec_bwd.cuh"
+#include "tc_enc_bwd.cuh"
 
 namespace resbm {
 
@@ -179,6 +180,62 @@ cudaError_t launch_dec_bwd(const resbm_desc &d, const void *dY, const void *B, c
     return cudaGetLastError();
 }
 
+// Scratch of the encoder backward: P (T x m fp32, used when the caller has none) and the slots.
+struct EncBwdWs {
+    float *P;
+    BwdPlan plan;
+    size_t bytes;
+};
+
+EncBwdWs enc_bwd_ws(const resbm_desc &d, int sms, void *ws)
+{
+    EncBwdWs w{};
+    WsCarver c(ws);
+    w.P = c.take<float>(d.T * d.m);
+    char *rest = c.take<char>(0);
+    const int nt = d.m <= 32 ? 4 : 2;
+    w.plan = bwd_plan(d, sms, nt, d.m * d.r, ws ? rest : nullptr);
+    w.bytes = c.used + w.plan.bytes;
+    return w;
+}
+
+template <int M>
+cudaError_t launch_enc_bwd(const resbm_desc &d, const void *dB, const void *F, const float *P, const void *We1,
+                           const void *We2, void *dF, void *dX, float *dWe1, float *dWe2, void *ws, const Ctx &c)
+{
+    using Cfg = tc::EncBwdCfg<M>;
+    const EncBwdWs w = enc_bwd_ws(d, c.sm_count, ws);
+    const BwdPlan &p = w.plan;
+    const CUtensorMapSwizzle dswz = Cfg::DSW == 128  ? CU_TENSOR_MAP_SWIZZLE_128B
+                                    : Cfg::DSW == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                                     : CU_TENSOR_MAP_SWIZZLE_32B;
+    CUtensorMap m_f128, m_f16, m_we1, m_df128, m_df16;
+    if (!make_map(&m_f128, F, d.d, d.T, d.d * 2, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&m_f16, F, d.d, d.T, d.d * 2, 64, 16, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&m_we1, We1, d.m, d.d, d.m * 2, M, 128, dswz) ||
+        !make_map(&m_df128, dF, d.d, d.T, d.d * 2, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&m_df16, dF, d.d, d.T, d.d * 2, 64, 16, CU_TENSOR_MAP_SWIZZLE_128B))
+        return cudaErrorInvalidValue;
+    cudaError_t e;
+    if (!P) {  // P = F . We1 with the forward kernel (no B), so it matches a saved P bit for bit
+        e = launch_enc_fwd<M>(d, nullptr, F, We1, We2, nullptr, w.P, c);
+        if (e != cudaSuccess) return e;
+        P = w.P;
+    }
+    static std::atomic<uint8_t> smem_set[kMaxDev];
+    e = ensure_smem(tc::k_enc_bwd<M>, Cfg::SMEM_BYTES, c.device, smem_set);
+    if (e != cudaSuccess) return e;
+    tc::EncBwdArgs a{static_cast<const __nv_bfloat16 *>(dB), P, static_cast<const __nv_bfloat16 *>(We2),
+                     static_cast<__nv_bfloat16 *>(dX), p.part_big, p.part_small, d.T, d.d, d.act, p.max_groups};
+    tc::k_enc_bwd<M><<<p.grid, Cfg::THREADS, Cfg::SMEM_BYTES, c.stream>>>(m_f128, m_f16, m_we1, m_df128, m_df16, a);
+    count_launches(1);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    tc::k_reduce_slots<<<reduce_grid(d.d * d.m, c), 256, 0, c.stream>>>(p.part_big, p.slots, d.d, d.m, dWe1, 0);
+    tc::k_reduce_slots<<<reduce_grid(d.m * d.r, c), 256, 0, c.stream>>>(p.part_small, p.slots, d.m, d.r, dWe2, 0);
+    count_launches(2);
+    return cudaGetLastError();
+}
+
 }  // namespace
 
 bool tc_supported(const resbm_desc &d, int op)
@@ -190,13 +247,14 @@ bool tc_supported(const resbm_desc &d, int op)
         return d.d % nch == 0;
     }
     if (op == RESBM_OP_ENCODE_FWD) return d.d % 64 == 0;
-    if (op == RESBM_OP_DECODE_BWD) return d.m <= 64 && d.d % 128 == 0;
+    if (op == RESBM_OP_DECODE_BWD || op == RESBM_OP_ENCODE_BWD) return d.m <= 64 && d.d % 128 == 0;
     return false;
 }
 
 size_t tc_ws_bytes(const resbm_desc &d, int op, int sms)
 {
     if (op == RESBM_OP_DECODE_BWD) return bwd_plan(d, sms, 4, d.r * d.m, nullptr).bytes;
+    if (op == RESBM_OP_ENCODE_BWD) return enc_bwd_ws(d, sms, nullptr).bytes;
     return 0;
 }
 
@@ -239,9 +297,16 @@ cudaError_t tc_decode_bwd(const resbm_desc &d, const void *dY, const void *B, co
     return cudaErrorNotSupported;
 }
 
-cudaError_t tc_encode_bwd(const resbm_desc &, const void *, const void *, const float *, const void *,
-                          const void *, void *, void *, float *, float *, void *, const Ctx &)
+cudaError_t tc_encode_bwd(const resbm_desc &d, const void *dB, const void *F, const float *P, const void *We1,
+                          const void *We2, void *dF, void *dX, float *dWe1, float *dWe2, void *ws, const Ctx &c)
 {
+    if (!al16(dB) || !al16(F) || (P && !al16(P)) || !al16(We1) || !al16(We2) || !al16(dF) || (dX && !al16(dX)))
+        return cudaErrorNotSupported;
+    switch (d.m) {
+    case 16: return launch_enc_bwd<16>(d, dB, F, P, We1, We2, dF, dX, dWe1, dWe2, ws, c);
+    case 32: return launch_enc_bwd<32>(d, dB, F, P, We1, We2, dF, dX, dWe1, dWe2, ws, c);
+    case 64: return launch_enc_bwd<64>(d, dB, F, P, We1, We2, dF, dX, dWe1, dWe2, ws, c);
+    }
     return cudaErrorNotSupported;
 }
 

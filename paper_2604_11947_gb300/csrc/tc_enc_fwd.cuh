@@ -175,7 +175,7 @@ __global__ void __launch_bounds__(192, 1)
             }
             tc_fence_before();
             mbar_arrive(smem_u32(&acc_empty[ab]));
-            if (row < valid) {
+            if (row < valid) {  // (with a.B == null only P is wanted: P = F . We1 for the backward)
                 const int64_t tok = t0 + row;
                 if (a.P) {
                     float4 *dst = reinterpret_cast<float4 *>(a.P + tok * C::M);
@@ -189,6 +189,7 @@ __global__ void __launch_bounds__(192, 1)
                 uint4 *bd = reinterpret_cast<uint4 *>(a.B + tok * C::R);
 #pragma unroll
                 for (int jb = 0; jb < C::R; jb += 8) {
+                    if (a.B == nullptr) break;
                     // E[jb .. jb+8) = sum_j A[j] We2[j][jb .. jb+8), fp32
                     float e[8];
 #pragma unroll
