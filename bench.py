@@ -39,6 +39,8 @@ def parse():
     p.add_argument("--steps", type=int, default=200)
     p.add_argument("--warmup", type=int, default=10)
     p.add_argument("--config", default="large_bf16", choices=sorted(synth.CONFIGS))
+    p.add_argument("--tokens", type=int, default=None,
+                   help="override T (smaller cases for profiler captures; not a bench line)")
     p.add_argument("--impl", default="resbm", choices=("resbm", "reference"))
     p.add_argument("--generic", action="store_true", help="force the CUDA-core kernels")
     p.add_argument("--no-e2e", action="store_true")
@@ -245,6 +247,8 @@ def run_reference(args, cfg, rank):
 def main():
     args = parse()
     cfg = synth.CONFIGS[args.config]
+    if args.tokens:
+        cfg = cfg.with_(name="%s_T%d" % (cfg.name, args.tokens), T=args.tokens)
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))

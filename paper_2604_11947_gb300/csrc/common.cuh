@@ -52,6 +52,40 @@ __device__ __forceinline__ float dact_f(int act, float x)
     return 1.0f;
 }
 
+// The same functions with CUDA's fast intrinsics (__expf, __fdividef, __tanhf-free tanh via
+// __expf): used where the result feeds a bf16 tensor-core operand (rounded to 8 significant bits,
+// far coarser than the intrinsics' error).
+__device__ __forceinline__ float fast_tanh(float u)
+{
+    // tanh(u) = 1 - 2 / (exp(2u) + 1), saturating cleanly for large |u|
+    return 1.0f - __fdividef(2.0f, __expf(2.0f * u) + 1.0f);
+}
+
+__device__ __forceinline__ float act_fast(int act, float x)
+{
+    if (act == RESBM_ACT_SILU) return __fdividef(x, 1.0f + __expf(-x));
+    if (act == RESBM_ACT_GELU_TANH) {
+        const float u = kSqrt2OverPi * fmaf(kGeluC * x, x * x, x);
+        return 0.5f * x * (1.0f + fast_tanh(u));
+    }
+    return x;
+}
+
+__device__ __forceinline__ float dact_fast(int act, float x)
+{
+    if (act == RESBM_ACT_SILU) {
+        const float s = __fdividef(1.0f, 1.0f + __expf(-x));
+        return s * fmaf(x, 1.0f - s, 1.0f);
+    }
+    if (act == RESBM_ACT_GELU_TANH) {
+        const float u = kSqrt2OverPi * fmaf(kGeluC * x, x * x, x);
+        const float th = fast_tanh(u);
+        const float du = kSqrt2OverPi * fmaf(3.0f * kGeluC * x, x, 1.0f);
+        return 0.5f * (1.0f + th) + 0.5f * x * (1.0f - th * th) * du;
+    }
+    return 1.0f;
+}
+
 // act and its derivative at the same point (one exp / tanh)
 __device__ __forceinline__ void act_and_dact(int act, float x, float &a, float &da)
 {

@@ -117,12 +117,13 @@ cudaError_t launch_enc_fwd(const resbm_desc &d, const void *X, const void *F, co
     return cudaGetLastError();
 }
 
-// Partial-slot layout of the backward kernels: one slot per (CTA, group of NT tiles).
+// Scratch layout of the backward kernels: the d x m weight gradient has one fp32 slot per CTA
+// (tc_wgrad.cuh); the small one has one slot per (CTA, tile group).
 struct BwdPlan {
-    int grid = 1, max_groups = 1;
-    int64_t slots = 1;
-    float *part_big = nullptr;    // slots x d x m
-    float *part_small = nullptr;  // slots x small_elems
+    int grid = 1, max_groups = 1, nch = 1;
+    int64_t slots = 1;              // small partial slots
+    float *part_big = nullptr;      // grid x d x m
+    float *part_small = nullptr;    // slots x small_elems
     size_t bytes = 0;
 };
 
@@ -138,8 +139,9 @@ BwdPlan bwd_plan(const resbm_desc &d, int sms, int nt, int64_t small_elems, void
     p.max_groups = (int)((max_tiles + nt - 1) / nt);
     if (p.max_groups < 1) p.max_groups = 1;
     p.slots = (int64_t)p.grid * p.max_groups;
+    p.nch = (int)(d.d / 128);
     WsCarver w(ws);
-    p.part_big = w.take<float>(p.slots * d.d * d.m);
+    p.part_big = w.take<float>((int64_t)p.grid * d.d * d.m);
     p.part_small = w.take<float>(p.slots * small_elems);
     p.bytes = w.used;
     return p;
@@ -167,15 +169,19 @@ cudaError_t launch_dec_bwd(const resbm_desc &d, const void *dY, const void *B, c
     static std::atomic<uint8_t> smem_set[kMaxDev];
     cudaError_t e = ensure_smem(tc::k_dec_bwd<M>, Cfg::SMEM_BYTES, c.device, smem_set);
     if (e != cudaSuccess) return e;
-    tc::DecBwdArgs a{static_cast<const __nv_bfloat16 *>(B), static_cast<const __nv_bfloat16 *>(Wd1),
-                     static_cast<const __nv_bfloat16 *>(dY), static_cast<__nv_bfloat16 *>(dB), p.part_big,
+    tc::DecBwdArgs a{static_cast<const __nv_bfloat16 *>(B),
+                     static_cast<const __nv_bfloat16 *>(Wd1),
+                     static_cast<const __nv_bfloat16 *>(dY),
+                     static_cast<__nv_bfloat16 *>(dB),
+                     tc::WgradArgs{p.part_big, p.nch},
                      p.part_small, d.T, d.d, d.act, d.merge_identity, p.max_groups};
     tc::k_dec_bwd<M><<<p.grid, Cfg::THREADS, Cfg::SMEM_BYTES, c.stream>>>(m_dy128, m_dy16, m_wd2, a);
     count_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    // dWd2 (m x d) = sum of the d x m slices, transposed; dWd1 (r x m) = sum of the slices
-    tc::k_reduce_slots<<<reduce_grid(d.d * d.m, c), 256, 0, c.stream>>>(p.part_big, p.slots, d.d, d.m, dWd2, 1);
-    tc::k_reduce_slots<<<reduce_grid(d.r * d.m, c), 256, 0, c.stream>>>(p.part_small, p.slots, d.r, d.m, dWd1, 0);
+    // dWd2 (m x d) = sum of the per-CTA slots (d x m), transposed; dWd1 (r x m) = sum of the slices
+    tc::k_reduce_slots<<<reduce_grid(d.d * d.m / 4, c), 256, 0, c.stream>>>(p.part_big, p.grid, d.d, d.m, dWd2, 1, 0);
+    tc::k_reduce_slots<<<reduce_grid(d.r * d.m / 4, c), 256, 0, c.stream>>>(p.part_small, p.slots, d.r, d.m, dWd1, 0,
+                                                                              al16(dWd1));
     count_launches(2);
     return cudaGetLastError();
 }
@@ -226,12 +232,15 @@ cudaError_t launch_enc_bwd(const resbm_desc &d, const void *dB, const void *F, c
     e = ensure_smem(tc::k_enc_bwd<M>, Cfg::SMEM_BYTES, c.device, smem_set);
     if (e != cudaSuccess) return e;
     tc::EncBwdArgs a{static_cast<const __nv_bfloat16 *>(dB), P, static_cast<const __nv_bfloat16 *>(We2),
-                     static_cast<__nv_bfloat16 *>(dX), p.part_big, p.part_small, d.T, d.d, d.act, p.max_groups};
+                     static_cast<__nv_bfloat16 *>(dX), tc::WgradArgs{p.part_big, p.nch},
+                     p.part_small, d.T, d.d, d.act, p.max_groups};
     tc::k_enc_bwd<M><<<p.grid, Cfg::THREADS, Cfg::SMEM_BYTES, c.stream>>>(m_f128, m_f16, m_we1, m_df128, m_df16, a);
     count_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    tc::k_reduce_slots<<<reduce_grid(d.d * d.m, c), 256, 0, c.stream>>>(p.part_big, p.slots, d.d, d.m, dWe1, 0);
-    tc::k_reduce_slots<<<reduce_grid(d.m * d.r, c), 256, 0, c.stream>>>(p.part_small, p.slots, d.m, d.r, dWe2, 0);
+    tc::k_reduce_slots<<<reduce_grid(d.d * d.m / 4, c), 256, 0, c.stream>>>(p.part_big, p.grid, d.d, d.m, dWe1, 0,
+                                                                            al16(dWe1));
+    tc::k_reduce_slots<<<reduce_grid(d.m * d.r / 4, c), 256, 0, c.stream>>>(p.part_small, p.slots, d.m, d.r, dWe2, 0,
+                                                                              al16(dWe2));
     count_launches(2);
     return cudaGetLastError();
 }

@@ -22,6 +22,7 @@
 
 #include "common.cuh"
 #include "tc_common.cuh"
+#include "tc_wgrad.cuh"
 
 namespace resbm {
 namespace tc {
@@ -38,7 +39,8 @@ template <int M_> struct DecBwdCfg {
     static constexpr uint32_t WD1_BYTES = R * M_ * 2;
     static constexpr uint32_t OFF_Y = 0;
     static constexpr uint32_t OFF_W = OFF_Y + NSY * Y_STAGE;
-    static constexpr uint32_t OFF_GT = OFF_W + 2 * W_STAGE;
+    static constexpr int NW = M_ <= 32 ? 4 : 3;               // Wd2 slice ring depth
+    static constexpr uint32_t OFF_GT = OFF_W + NW * W_STAGE;
     static constexpr uint32_t OFF_WD1 = OFF_GT + NT * GT_TILE;
     static constexpr uint32_t OFF_WD1T = OFF_WD1 + WD1_BYTES;
     static constexpr uint32_t SMEM_BYTES = OFF_WD1T + WD1_BYTES + 1024;
@@ -54,7 +56,7 @@ struct DecBwdArgs {
     const __nv_bfloat16 *Wd1;  // r x m
     const __nv_bfloat16 *dY;   // T x d (first r columns re-read for the identity path)
     __nv_bfloat16 *dB;         // T x r
-    float *part2;              // slots x d x m   (dWd2^T partials)
+    WgradArgs wg;              // dWd2^T chunks (d x m), reduced across CTAs
     float *part1;              // slots x r x m   (dWd1 partials)
     int64_t T, d;
     int act, merge, max_groups;
@@ -68,8 +70,8 @@ __global__ void __launch_bounds__(192, 1)
     using C = DecBwdCfg<M_>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    __shared__ uint64_t y_full[C::NSY], y_empty[C::NSY], w_full[2], w_empty[2];
-    __shared__ uint64_t gt_full, gt_empty, wt_full[2], wt_empty[2], dg_full, dg_empty, p2_done, done_bar;
+    __shared__ uint64_t y_full[C::NSY], y_empty[C::NSY], w_full[C::NW], w_empty[C::NW];
+    __shared__ uint64_t gt_full[C::NT], gt_empty, wt_full[2], wt_empty[2], dg_full, dg_empty, p2_done, done_bar;
     __shared__ uint32_t tmem_base_sh;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -84,13 +86,15 @@ __global__ void __launch_bounds__(192, 1)
             mbar_init(smem_u32(&y_full[s]), 1);
             mbar_init(smem_u32(&y_empty[s]), 1);
         }
-        for (int i = 0; i < 2; ++i) {
+        for (int i = 0; i < C::NW; ++i) {
             mbar_init(smem_u32(&w_full[i]), 1);
             mbar_init(smem_u32(&w_empty[i]), 1);
+        }
+        for (int i = 0; i < 2; ++i) {
             mbar_init(smem_u32(&wt_full[i]), 1);
             mbar_init(smem_u32(&wt_empty[i]), 128);
         }
-        mbar_init(smem_u32(&gt_full), 1);
+        for (int i = 0; i < C::NT; ++i) mbar_init(smem_u32(&gt_full[i]), 1);
         mbar_init(smem_u32(&gt_empty), 1);
         mbar_init(smem_u32(&dg_full), 1);
         mbar_init(smem_u32(&dg_empty), 128);
@@ -125,16 +129,20 @@ __global__ void __launch_bounds__(192, 1)
                 if (g > 0) ok = mbar_wait(smem_u32(&p2_done), (g - 1) & 1);  // the ring was scratch
                 const int tb = g * C::NT, te = min(ntiles, tb + C::NT);
                 for (int c = 0; c < nch && ok; ++c) {
-                    {
-                        const uint32_t s = wit & 1, ph = (wit >> 1) & 1;
-                        if (!mbar_wait(smem_u32(&w_empty[s]), ph ^ 1)) { ok = false; break; }
-                        const uint32_t dst = smem_u32(smem + C::OFF_W + s * C::W_STAGE);
-                        mbar_expect_tx(smem_u32(&w_full[s]), C::W_STAGE);
-                        for (int h = 0; h < 2; ++h)
-                            tma_load_2d(dst + h * (C::M * 128), &tm_wd2, c * 128 + 64 * h, 0, smem_u32(&w_full[s]));
-                        ++wit;
-                    }
+                    // order: dY tile 0 of the chunk, the chunk's Wd2 slice, the other dY tiles.
+                    // The MMA needs the slice before any tile of the chunk, so it must not queue
+                    // behind tiles that wait for ring slots (that would deadlock), and it must not
+                    // delay the first tile (that would stall the stream on the small weight ring).
                     for (int i = tb; i < te; ++i) {
+                        if (i == tb + 1) {
+                            const uint32_t s = wit % C::NW, ph = (wit / C::NW) & 1;
+                            if (!mbar_wait(smem_u32(&w_empty[s]), ph ^ 1)) { ok = false; break; }
+                            const uint32_t dst = smem_u32(smem + C::OFF_W + s * C::W_STAGE);
+                            mbar_expect_tx(smem_u32(&w_full[s]), C::W_STAGE);
+                            for (int h = 0; h < 2; ++h)
+                                tma_load_2d(dst + h * (C::M * 128), &tm_wd2, c * 128 + 64 * h, 0, smem_u32(&w_full[s]));
+                            ++wit;
+                        }
                         const int64_t t0 = start + 128 * (int64_t)i;
                         const int valid = (int)((end - t0) < 128 ? (end - t0) : 128);
                         const int nb = (valid + 15) / 16;
@@ -154,6 +162,16 @@ __global__ void __launch_bounds__(192, 1)
                         }
                         ++yit;
                     }
+                    if (!ok) break;
+                    if (te - tb == 1) {  // a one-tile group: the slice after its only tile
+                        const uint32_t s = wit % C::NW, ph = (wit / C::NW) & 1;
+                        if (!mbar_wait(smem_u32(&w_empty[s]), ph ^ 1)) { ok = false; break; }
+                        const uint32_t dst = smem_u32(smem + C::OFF_W + s * C::W_STAGE);
+                        mbar_expect_tx(smem_u32(&w_full[s]), C::W_STAGE);
+                        for (int h = 0; h < 2; ++h)
+                            tma_load_2d(dst + h * (C::M * 128), &tm_wd2, c * 128 + 64 * h, 0, smem_u32(&w_full[s]));
+                        ++wit;
+                    }
                 }
             }
             // drain the loads still in flight
@@ -161,9 +179,9 @@ __global__ void __launch_bounds__(192, 1)
                 const uint32_t j = yit - 1 - k;
                 mbar_wait(smem_u32(&y_full[j % C::NSY]), (j / C::NSY) & 1);
             }
-            for (uint32_t k = 0; k < (wit < 2u ? wit : 2u); ++k) {
+            for (uint32_t k = 0; k < (wit < (uint32_t)C::NW ? wit : (uint32_t)C::NW); ++k) {
                 const uint32_t j = wit - 1 - k;
-                mbar_wait(smem_u32(&w_full[j & 1]), (j >> 1) & 1);
+                mbar_wait(smem_u32(&w_full[j % C::NW]), (j / C::NW) & 1);
             }
         }
     } else if (warp == 1) {
@@ -175,13 +193,12 @@ __global__ void __launch_bounds__(192, 1)
             bool ok = true;
             for (int g = 0; g < ngroups && ok; ++g) {
                 const int tb = g * C::NT, te = min(ntiles, tb + C::NT);
-                ok = mbar_wait(smem_u32(&gt_full), g & 1);
-                if (g > 0) ok = ok && mbar_wait(smem_u32(&dg_empty), (g - 1) & 1);
+                if (g > 0) ok = mbar_wait(smem_u32(&dg_empty), (g - 1) & 1);
                 tc_fence_after();
                 for (int c = 0; c < nch && ok; ++c, ++cit) {
-                    const uint32_t sw = wit & 1;
+                    const uint32_t sw = wit % C::NW;
                     const uint32_t ab = cit & 1;
-                    ok = mbar_wait(smem_u32(&w_full[sw]), (wit >> 1) & 1) &&
+                    ok = mbar_wait(smem_u32(&w_full[sw]), (wit / C::NW) & 1) &&
                          mbar_wait(smem_u32(&wt_empty[ab]), ((cit >> 1) & 1) ^ 1);
                     tc_fence_after();
                     const uint32_t waddr = smem_u32(smem + C::OFF_W + sw * C::W_STAGE);
@@ -199,6 +216,10 @@ __global__ void __launch_bounds__(192, 1)
                             const uint64_t bd = smem_desc(waddr + (k >> 2) * (C::M * 128) + (k & 3) * 32, 16, 1024, kSwz128);
                             mma_bf16(tmem_dg + (i - tb) * C::MS, ad, bd, id_dg, (c | k) != 0);
                         }
+                        // the dWd2 product needs the tile's G^T (published per tile in phase 0;
+                        // the dG products above did not wait for it)
+                        ok = ok && mbar_wait(smem_u32(&gt_full[i - tb]), g & 1);
+                        tc_fence_after();
                         const int nks = (valid + 15) / 16;
                         for (int k = 0; k < nks; ++k) {
                             const uint64_t ad = smem_desc(yaddr + k * 2048, 16384, 1024, kSwz128);
@@ -250,32 +271,33 @@ __global__ void __launch_bounds__(192, 1)
                     vecmat16<C::R, C::M>(bq, wd1, jb, acc);   // Q = B . Wd1
 #pragma unroll
                     for (int e = 0; e < 16; ++e) {
-                        const float gv = active ? act_f(a.act, acc[e]) : 0.0f;
+                        const float gv = active ? act_fast(a.act, acc[e]) : 0.0f;
                         *reinterpret_cast<__nv_bfloat16 *>(gt + swz_offset(jb + e, byte, 128)) = __float2bfloat16_rn(gv);
                     }
                 }
+                // publish this tile's G^T so its first dWd2 product can start
+                fence_async_smem();
+                named_barrier(1, 128);
+                if (et == 0) mbar_arrive(smem_u32(&gt_full[i - tb]));
             }
-            fence_async_smem();
-            named_barrier(1, 128);
-            if (et == 0) mbar_arrive(smem_u32(&gt_full));
 
             // ---- phase 1: drain each chunk's dWd2^T partial ----
             for (int c = 0; c < nch && ok; ++c, ++cit) {
                 const uint32_t ab = cit & 1;
                 ok = mbar_wait(smem_u32(&wt_full[ab]), (cit >> 1) & 1);
                 tc_fence_after();
-                float4 *dst = reinterpret_cast<float4 *>(a.part2 + (slot * a.d + (int64_t)c * 128 + row) * C::M);
+                float v[C::M];
 #pragma unroll
                 for (int j = 0; j < C::M; j += 16) {
                     float t16[16];
                     tmem_ld16(tmem_wt + ((uint32_t)(q * 32) << 16) + ab * C::MS + j, t16);
                     tmem_ld_wait();
 #pragma unroll
-                    for (int e = 0; e < 4; ++e)
-                        dst[j / 4 + e] = make_float4(t16[4 * e], t16[4 * e + 1], t16[4 * e + 2], t16[4 * e + 3]);
+                    for (int e = 0; e < 16; ++e) v[j + e] = t16[e];
                 }
                 tc_fence_before();
-                mbar_arrive(smem_u32(&wt_empty[ab]));
+                mbar_arrive(smem_u32(&wt_empty[ab]));   // the accumulator is free again
+                wgrad_chunk<C::M>(a.wg, v, c, row, g == 0);
             }
 
             // ---- phase 2: dQ, dB, dWd1 partial ----
@@ -314,7 +336,7 @@ __global__ void __launch_bounds__(192, 1)
                     float acc[16];
                     vecmat16<C::R, C::M>(bq, wd1, jb, acc);
 #pragma unroll
-                    for (int e = 0; e < 16; ++e) dq[jb + e] = active ? dq[jb + e] * dact_f(a.act, acc[e]) : 0.0f;
+                    for (int e = 0; e < 16; ++e) dq[jb + e] = active ? dq[jb + e] * dact_fast(a.act, acc[e]) : 0.0f;
                 }
                 if (active) {
                     // dB = [merge] dY[:, :r] + dQ . Wd1^T
@@ -346,31 +368,31 @@ __global__ void __launch_bounds__(192, 1)
 #pragma unroll
                 for (int j = 0; j < C::M; ++j) sQ[row * (C::M + 1) + j] = dq[j];
                 named_barrier(1, 128);
+                // output o = et + 128 kk is (ki, j) = (o / M, o % M); 128 is a multiple of M, so j
+                // is the same for all of this thread's outputs. Each output sums over t in order;
+                // the outputs' chains interleave so their latencies overlap.
+                {
+                    static_assert((C::R * C::M) % 128 == 0 && 128 % C::M == 0, "dWd1 output split");
+                    const int j = et % C::M, ki0 = et / C::M;
+#pragma unroll 2
+                    for (int t = 0; t < valid; ++t) {
+                        const float qv = sQ[t * (C::M + 1) + j];
+                        const float *bt = sB + t * (C::R + 1) + ki0;
 #pragma unroll
-                for (int kk = 0; kk < NOUT; ++kk) {
-                    const int o = et + 128 * kk;
-                    if (o < C::R * C::M) {
-                        const int ki = o / C::M, j = o % C::M;
-                        float s = acc1[kk];
-                        for (int t = 0; t < valid; ++t) s = fmaf(sB[t * (C::R + 1) + ki], sQ[t * (C::M + 1) + j], s);
-                        acc1[kk] = s;
+                        for (int kk = 0; kk < NOUT; ++kk) acc1[kk] = fmaf(bt[kk * (128 / C::M)], qv, acc1[kk]);
                     }
                 }
             }
             tc_fence_before();
             mbar_arrive(smem_u32(&dg_empty));
 #pragma unroll
-            for (int kk = 0; kk < NOUT; ++kk) {
-                const int o = et + 128 * kk;
-                if (o < C::R * C::M) a.part1[slot * (C::R * C::M) + o] = acc1[kk];
-            }
+            for (int kk = 0; kk < NOUT; ++kk) a.part1[slot * (C::R * C::M) + et + 128 * kk] = acc1[kk];
             named_barrier(1, 128);   // scratch reads done before the ring is reused
             if (et == 0) mbar_arrive(smem_u32(&p2_done));
         }
         // slots of groups this CTA does not have: zeros
         for (int g = ngroups; g < a.max_groups; ++g) {
             const int64_t slot = (int64_t)blockIdx.x * a.max_groups + g;
-            for (int64_t e = et; e < a.d * C::M; e += 128) a.part2[slot * a.d * C::M + e] = 0.0f;
             for (int e = et; e < C::R * C::M; e += 128) a.part1[slot * (C::R * C::M) + e] = 0.0f;
         }
     }
@@ -382,20 +404,43 @@ __global__ void __launch_bounds__(192, 1)
     }
 }
 
-// out = sum over slots s = 0, 1, ... of part[s] (rows x cols each), fixed order. With transpose
-// the result is written cols x rows (part slices are d x m, the weight gradient is m x d).
-__global__ void k_reduce_slots(const float *__restrict__ part, int64_t slots, int64_t rows, int64_t cols,
-                               float *__restrict__ out, int transpose)
+// out = sum over slots s = 0, 1, ... of part[s] (rows x cols each, rows * cols % 4 == 0), each
+// element summed in slot order. Four consecutive elements per thread (16-byte loads) and eight
+// slots loaded ahead keep enough reads in flight. With transpose the result is written
+// cols x rows (part slices are d x m, the weight gradient is m x d); out4 says out is 16-byte
+// aligned (untransposed only).
+__device__ __forceinline__ void add4(float4 &a, const float4 &b)
 {
-    const int64_t n = rows * cols;
-    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n; e += (int64_t)gridDim.x * blockDim.x) {
-        float s = 0.0f;
-        for (int64_t k = 0; k < slots; ++k) s += part[k * n + e];
+    a.x += b.x; a.y += b.y; a.z += b.z; a.w += b.w;
+}
+
+__global__ void k_reduce_slots(const float *__restrict__ part, int64_t slots, int64_t rows, int64_t cols,
+                               float *__restrict__ out, int transpose, int out4)
+{
+    const int64_t n4 = rows * cols / 4;
+    const float4 *p4 = reinterpret_cast<const float4 *>(part);
+    for (int64_t e4 = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e4 < n4; e4 += (int64_t)gridDim.x * blockDim.x) {
+        float4 acc = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+        int64_t s = 0;
+        for (; s + 8 <= slots; s += 8) {
+            float4 v[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) v[u] = p4[(s + u) * n4 + e4];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) add4(acc, v[u]);
+        }
+        for (; s < slots; ++s) add4(acc, p4[s * n4 + e4]);
+        const int64_t e = 4 * e4;
         if (transpose) {
             const int64_t rr = e / cols, cc = e - rr * cols;
-            out[cc * rows + rr] = s;
+            out[(cc + 0) * rows + rr] = acc.x;
+            out[(cc + 1) * rows + rr] = acc.y;
+            out[(cc + 2) * rows + rr] = acc.z;
+            out[(cc + 3) * rows + rr] = acc.w;
+        } else if (out4) {
+            reinterpret_cast<float4 *>(out)[e4] = acc;
         } else {
-            out[e] = s;
+            out[e] = acc.x; out[e + 1] = acc.y; out[e + 2] = acc.z; out[e + 3] = acc.w;
         }
     }
 }

@@ -176,8 +176,11 @@ __global__ void __launch_bounds__(192, 1)
             const uint32_t gb = tile_i & 1;
             ok = mbar_wait(smem_u32(&g_empty[gb]), ((tile_i >> 1) & 1) ^ 1);
             uint8_t *gbuf = smem + C::OFF_G + gb * C::G_BYTES;
+            // rows past the valid tokens only feed output rows that are never stored
+            const int jend = (q * 32 < valid) ? C::M : 0;
 #pragma unroll
             for (int jb = 0; jb < C::M; jb += 16) {
+                if (jb >= jend) break;
                 float accq[16];
 #pragma unroll
                 for (int j = 0; j < 16; ++j) accq[j] = 0.0f;
@@ -224,9 +227,11 @@ __global__ void __launch_bounds__(192, 1)
                 uint8_t *stg = smem + C::OFF_STG + sb * C::STG_BYTES;
                 const int64_t left = a.d - (int64_t)c * C::NCH;
                 const int ncols = left < C::NCH ? (int)left : C::NCH;
+                // a warp whose 32 rows all lie past the tile's valid tokens has nothing to store
+                const int gend = (q * 32 < valid) ? ncols : 0;
 #pragma unroll
                 for (int g = 0; g < C::NCH / 32; ++g) {
-                    if (g * 32 >= ncols) break;
+                    if (g * 32 >= gend) break;
                     float v[32];
                     tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + ab * C::NCH + g * 32, v);
                     tmem_ld_wait();

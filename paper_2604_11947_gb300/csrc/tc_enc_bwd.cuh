@@ -21,6 +21,7 @@
 
 #include "common.cuh"
 #include "tc_common.cuh"
+#include "tc_wgrad.cuh"
 
 namespace resbm {
 namespace tc {
@@ -41,7 +42,8 @@ template <int M_> struct EncBwdCfg {
     static constexpr uint32_t OFF_F = 0;
     static constexpr uint32_t OFF_STG = OFF_F + NSF * F_STAGE;
     static constexpr uint32_t OFF_W = OFF_STG + 2 * STG_HALF;
-    static constexpr uint32_t OFF_DPA = OFF_W + 2 * W_STAGE;
+    static constexpr int NW = M_ <= 16 ? 4 : 3;                  // We1 slice ring depth
+    static constexpr uint32_t OFF_DPA = OFF_W + NW * W_STAGE;
     static constexpr uint32_t OFF_DPT = OFF_DPA + NT * DPA_TILE;
     static constexpr uint32_t OFF_WE2T = OFF_DPT + NT * DPT_TILE;
     static constexpr uint32_t SMEM_BYTES = OFF_WE2T + WE2T_BYTES + 1024;
@@ -56,7 +58,7 @@ struct EncBwdArgs {
     const float *P;            // T x m
     const __nv_bfloat16 *We2;  // m x r
     __nv_bfloat16 *dX;         // T x d or null
-    float *part1;              // slots x d x m  (dWe1 partials)
+    WgradArgs wg;              // dWe1 chunks (d x m), reduced across CTAs
     float *part2;              // slots x m x r  (dWe2 partials)
     int64_t T, d;
     int act, max_groups;
@@ -71,8 +73,8 @@ __global__ void __launch_bounds__(192, 1)
     using C = EncBwdCfg<M_>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    __shared__ uint64_t f_full[C::NSF], f_empty[C::NSF], w_full[2], w_empty[2];
-    __shared__ uint64_t dp_full, dp_empty, df_full[2], df_empty[2], we_full[2], we_empty[2], p3_done, done_bar;
+    __shared__ uint64_t f_full[C::NSF], f_empty[C::NSF], w_full[C::NW], w_empty[C::NW];
+    __shared__ uint64_t dp_full[C::NT], dp_empty, df_full[2], df_empty[2], we_full[2], we_empty[2], p3_done, done_bar;
     __shared__ uint32_t tmem_base_sh;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -87,15 +89,17 @@ __global__ void __launch_bounds__(192, 1)
             mbar_init(smem_u32(&f_full[s]), 1);
             mbar_init(smem_u32(&f_empty[s]), 1);
         }
-        for (int i = 0; i < 2; ++i) {
+        for (int i = 0; i < C::NW; ++i) {
             mbar_init(smem_u32(&w_full[i]), 1);
             mbar_init(smem_u32(&w_empty[i]), 1);
+        }
+        for (int i = 0; i < 2; ++i) {
             mbar_init(smem_u32(&df_full[i]), 1);
             mbar_init(smem_u32(&df_empty[i]), 128);
             mbar_init(smem_u32(&we_full[i]), 1);
             mbar_init(smem_u32(&we_empty[i]), 128);
         }
-        mbar_init(smem_u32(&dp_full), 1);
+        for (int i = 0; i < C::NT; ++i) mbar_init(smem_u32(&dp_full[i]), 1);
         mbar_init(smem_u32(&dp_empty), 1);
         mbar_init(smem_u32(&p3_done), 1);
         mbar_init(smem_u32(&done_bar), 1);
@@ -125,15 +129,19 @@ __global__ void __launch_bounds__(192, 1)
                 if (g > 0) ok = mbar_wait(smem_u32(&p3_done), (g - 1) & 1);  // the ring was scratch
                 const int tb = g * C::NT, te = min(ntiles, tb + C::NT);
                 for (int c = 0; c < nch && ok; ++c) {
-                    {
-                        const uint32_t s = wit & 1;
-                        if (!mbar_wait(smem_u32(&w_empty[s]), ((wit >> 1) & 1) ^ 1)) { ok = false; break; }
-                        mbar_expect_tx(smem_u32(&w_full[s]), C::W_STAGE);
-                        tma_load_2d(smem_u32(smem + C::OFF_W + s * C::W_STAGE), &tm_we1, 0, c * 128,
-                                    smem_u32(&w_full[s]));
-                        ++wit;
-                    }
+                    // order: F tile 0 of the chunk, the chunk's We1 slice, the other F tiles.
+                    // The MMA needs the slice before any tile of the chunk, so it must not queue
+                    // behind tiles that wait for ring slots (that would deadlock), and it must not
+                    // delay the first tile (that would stall the stream on the small weight ring).
                     for (int i = tb; i < te; ++i) {
+                        if (i == tb + 1) {
+                            const uint32_t s = wit % C::NW;
+                            if (!mbar_wait(smem_u32(&w_empty[s]), ((wit / C::NW) & 1) ^ 1)) { ok = false; break; }
+                            mbar_expect_tx(smem_u32(&w_full[s]), C::W_STAGE);
+                            tma_load_2d(smem_u32(smem + C::OFF_W + s * C::W_STAGE), &tm_we1, 0, c * 128,
+                                        smem_u32(&w_full[s]));
+                            ++wit;
+                        }
                         const int64_t t0 = start + 128 * (int64_t)i;
                         const int valid = (int)((end - t0) < 128 ? (end - t0) : 128);
                         const int nb = (valid + 15) / 16;
@@ -153,15 +161,24 @@ __global__ void __launch_bounds__(192, 1)
                         }
                         ++fit;
                     }
+                    if (!ok) break;
+                    if (te - tb == 1) {  // a one-tile group: the slice after its only tile
+                        const uint32_t s = wit % C::NW;
+                        if (!mbar_wait(smem_u32(&w_empty[s]), ((wit / C::NW) & 1) ^ 1)) { ok = false; break; }
+                        mbar_expect_tx(smem_u32(&w_full[s]), C::W_STAGE);
+                        tma_load_2d(smem_u32(smem + C::OFF_W + s * C::W_STAGE), &tm_we1, 0, c * 128,
+                                    smem_u32(&w_full[s]));
+                        ++wit;
+                    }
                 }
             }
             for (uint32_t k = 0; k < (fit < (uint32_t)C::NSF ? fit : (uint32_t)C::NSF); ++k) {
                 const uint32_t j = fit - 1 - k;
                 mbar_wait(smem_u32(&f_full[j % C::NSF]), (j / C::NSF) & 1);
             }
-            for (uint32_t k = 0; k < (wit < 2u ? wit : 2u); ++k) {
+            for (uint32_t k = 0; k < (wit < (uint32_t)C::NW ? wit : (uint32_t)C::NW); ++k) {
                 const uint32_t j = wit - 1 - k;
-                mbar_wait(smem_u32(&w_full[j & 1]), (j >> 1) & 1);
+                mbar_wait(smem_u32(&w_full[j % C::NW]), (j / C::NW) & 1);
             }
         }
     } else if (warp == 1) {
@@ -174,11 +191,9 @@ __global__ void __launch_bounds__(192, 1)
             bool ok = true;
             for (int g = 0; g < ngroups && ok; ++g) {
                 const int tb = g * C::NT, te = min(ntiles, tb + C::NT);
-                ok = mbar_wait(smem_u32(&dp_full), g & 1);
-                tc_fence_after();
                 for (int c = 0; c < nch && ok; ++c, ++cit, ++wit) {
-                    const uint32_t sw = wit & 1, ae = cit & 1;
-                    ok = mbar_wait(smem_u32(&w_full[sw]), (wit >> 1) & 1) &&
+                    const uint32_t sw = wit % C::NW, ae = cit & 1;
+                    ok = mbar_wait(smem_u32(&w_full[sw]), (wit / C::NW) & 1) &&
                          mbar_wait(smem_u32(&we_empty[ae]), ((cit >> 1) & 1) ^ 1);
                     tc_fence_after();
                     const uint32_t waddr = smem_u32(smem + C::OFF_W + sw * C::W_STAGE);
@@ -186,7 +201,9 @@ __global__ void __launch_bounds__(192, 1)
                         const int64_t t0 = start + 128 * (int64_t)i;
                         const int valid = (int)((end - t0) < 128 ? (end - t0) : 128);
                         const uint32_t s = fit % C::NSF, ad_buf = dfit & 1;
-                        ok = mbar_wait(smem_u32(&f_full[s]), (fit / C::NSF) & 1) &&
+                        // dP of the tile (phase 0, published per tile), its F tile, a free dF buffer
+                        ok = mbar_wait(smem_u32(&dp_full[i - tb]), g & 1) &&
+                             mbar_wait(smem_u32(&f_full[s]), (fit / C::NSF) & 1) &&
                              mbar_wait(smem_u32(&df_empty[ad_buf]), ((dfit >> 1) & 1) ^ 1);
                         tc_fence_after();
                         const uint32_t faddr = smem_u32(smem + C::OFF_F + s * C::F_STAGE);
@@ -256,7 +273,7 @@ __global__ void __launch_bounds__(192, 1)
                     float acc[16];
                     vecmat16<C::R, C::M>(db, we2t, jb, acc);   // dA = dB . We2^T
 #pragma unroll
-                    for (int e = 0; e < 16; ++e) dp[jb + e] = active ? acc[e] * dact_f(a.act, dp[jb + e]) : 0.0f;
+                    for (int e = 0; e < 16; ++e) dp[jb + e] = active ? acc[e] * dact_fast(a.act, dp[jb + e]) : 0.0f;
                 }
                 // dP rows = tokens (K-major over m, DSW-byte rows)
                 uint8_t *pa = smem + C::OFF_DPA + (i - tb) * C::DPA_TILE;
@@ -276,6 +293,10 @@ __global__ void __launch_bounds__(192, 1)
 #pragma unroll
                 for (int j = 0; j < C::M; ++j)
                     *reinterpret_cast<__nv_bfloat16 *>(pt + swz_offset(j, byte, 128)) = __float2bfloat16_rn(dp[j]);
+                // publish this tile's dP so its products can start
+                fence_async_smem();
+                named_barrier(1, 128);
+                if (et == 0) mbar_arrive(smem_u32(&dp_full[i - tb]));
                 // identity path: dX[:, :r] += dB
                 if (active && a.dX) {
                     uint4 *xp = reinterpret_cast<uint4 *>(a.dX + tok * a.d);
@@ -294,9 +315,6 @@ __global__ void __launch_bounds__(192, 1)
                     }
                 }
             }
-            fence_async_smem();
-            named_barrier(1, 128);
-            if (et == 0) mbar_arrive(smem_u32(&dp_full));
 
             // ---- phase 1: dF tiles out by TMA; dWe1 chunks to the partial slot ----
             for (int c = 0; c < nch && ok; ++c, ++cit) {
@@ -312,8 +330,11 @@ __global__ void __launch_bounds__(192, 1)
                         if (et == 0) bulk_wait_read<1>();   // staging half sb is free again
                         named_barrier(1, 128);
                         uint8_t *stg = smem + C::OFF_STG + sb * C::STG_HALF;
+                        // a warp whose rows all lie past the valid tokens has nothing to store
+                        const int gqend = (q * 32 < valid) ? 2 : 0;
 #pragma unroll
                         for (int gq = 0; gq < 2; ++gq) {
+                            if (gq >= gqend) break;
                             float v[32];
                             tmem_ld32(tmem_df + ((uint32_t)(q * 32) << 16) + ad_buf * 128 + h * 64 + gq * 32, v);
                             tmem_ld_wait();
@@ -346,22 +367,22 @@ __global__ void __launch_bounds__(192, 1)
                         }
                     }
                 }
-                // the chunk's dWe1 rows (lane = d column) -> partial slot
+                // the chunk's dWe1 rows (lane = d column) -> cross-CTA reduction
                 const uint32_t ae = cit & 1;
                 ok = ok && mbar_wait(smem_u32(&we_full[ae]), (cit >> 1) & 1);
                 tc_fence_after();
-                float4 *dst = reinterpret_cast<float4 *>(a.part1 + (slot * a.d + (int64_t)c * 128 + row) * C::M);
+                float v[C::M];
 #pragma unroll
                 for (int j = 0; j < C::M; j += 16) {
                     float t16[16];
                     tmem_ld16(tmem_we + ((uint32_t)(q * 32) << 16) + ae * C::MS + j, t16);
                     tmem_ld_wait();
 #pragma unroll
-                    for (int e = 0; e < 4; ++e)
-                        dst[j / 4 + e] = make_float4(t16[4 * e], t16[4 * e + 1], t16[4 * e + 2], t16[4 * e + 3]);
+                    for (int e = 0; e < 16; ++e) v[j + e] = t16[e];
                 }
                 tc_fence_before();
-                mbar_arrive(smem_u32(&we_empty[ae]));
+                mbar_arrive(smem_u32(&we_empty[ae]));   // the accumulator is free again
+                wgrad_chunk<C::M>(a.wg, v, c, row, g == 0);
             }
 
             // ---- phase 3: dWe2 partial = sum over tokens of phi(P)^T dB ----
@@ -383,8 +404,8 @@ __global__ void __launch_bounds__(192, 1)
 #pragma unroll
                     for (int j = 0; j < C::M / 4; ++j) {
                         const float4 v = ps[j];
-                        av[4 * j] = act_f(a.act, v.x); av[4 * j + 1] = act_f(a.act, v.y);
-                        av[4 * j + 2] = act_f(a.act, v.z); av[4 * j + 3] = act_f(a.act, v.w);
+                        av[4 * j] = act_fast(a.act, v.x); av[4 * j + 1] = act_fast(a.act, v.y);
+                        av[4 * j + 2] = act_fast(a.act, v.z); av[4 * j + 3] = act_fast(a.act, v.w);
                     }
                     load_bf16_row<C::R>(a.dB + tok * C::R, db);
                 } else {
@@ -399,28 +420,28 @@ __global__ void __launch_bounds__(192, 1)
 #pragma unroll
                 for (int k = 0; k < C::R; ++k) sD[row * (C::R + 1) + k] = db[k];
                 named_barrier(1, 128);
+                // output o = et + 128 kk is (j, k) = (o / R, o % R); 128 is a multiple of R, so k
+                // is the same for all of this thread's outputs. Each output sums over t in order;
+                // the outputs' chains interleave so their latencies overlap.
+                {
+                    static_assert((C::M * C::R) % 128 == 0 && 128 % C::R == 0, "dWe2 output split");
+                    const int k = et % C::R, j0 = et / C::R;
+#pragma unroll 2
+                    for (int t = 0; t < valid; ++t) {
+                        const float dv = sD[t * (C::R + 1) + k];
+                        const float *at = sA + t * (C::M + 1) + j0;
 #pragma unroll
-                for (int kk = 0; kk < NOUT; ++kk) {
-                    const int o = et + 128 * kk;
-                    if (o < C::M * C::R) {
-                        const int j = o / C::R, k = o % C::R;
-                        float s = acc2[kk];
-                        for (int t = 0; t < valid; ++t) s = fmaf(sA[t * (C::M + 1) + j], sD[t * (C::R + 1) + k], s);
-                        acc2[kk] = s;
+                        for (int kk = 0; kk < NOUT; ++kk) acc2[kk] = fmaf(at[kk * (128 / C::R)], dv, acc2[kk]);
                     }
                 }
             }
 #pragma unroll
-            for (int kk = 0; kk < NOUT; ++kk) {
-                const int o = et + 128 * kk;
-                if (o < C::M * C::R) a.part2[slot * (C::M * C::R) + o] = acc2[kk];
-            }
+            for (int kk = 0; kk < NOUT; ++kk) a.part2[slot * (C::M * C::R) + et + 128 * kk] = acc2[kk];
             named_barrier(1, 128);
             if (et == 0) mbar_arrive(smem_u32(&p3_done));
         }
         for (int g = ngroups; g < a.max_groups; ++g) {
             const int64_t slot = (int64_t)blockIdx.x * a.max_groups + g;
-            for (int64_t e = et; e < a.d * C::M; e += 128) a.part1[slot * a.d * C::M + e] = 0.0f;
             for (int e = et; e < C::M * C::R; e += 128) a.part2[slot * (C::M * C::R) + e] = 0.0f;
         }
         if (et == 0) bulk_wait<0>();
