@@ -169,6 +169,35 @@ RESBM_API resbm_status resbm_encode_bwd(const resbm_desc *desc, const void *dB, 
                               void *dF, void *dX, float *dWe1, float *dWe2,
                               void *ws, size_t ws_bytes, void *stream);
 
+/* Size of the library's fixed device scratch array used by resbm_decode_bwd_noalloc (32 MiB
+ * per device). */
+#define RESBM_STATIC_SCRATCH_BYTES ((size_t)32 << 20)
+
+/* resbm_decode_bwd without a workspace argument: the same computation, kernels and results,
+ * with its scratch taken from a fixed array that the library holds in device memory
+ * (RESBM_STATIC_SCRATCH_BYTES, reserved when the library's device code is loaded) instead of
+ * from the caller. The paper has no counterpart: this entry point is a library convenience.
+ *
+ * It is meant for callers that cannot hand over device memory for scratch: a C or C++ program
+ * that links this library without a device allocator of its own, or a runtime that fixes its
+ * device memory at start-up and may not allocate (or free) during a training step. Nothing is
+ * allocated or freed by the call, on the device or on the host.
+ *   - Arguments and results are those of resbm_decode_bwd. The scratch needed is the
+ *     resbm_workspace_bytes(desc, RESBM_OP_DECODE_BWD) figure; a call that needs more than
+ *     RESBM_STATIC_SCRATCH_BYTES returns RESBM_ERR_WORKSPACE and enqueues nothing. With the
+ *     tensor-core kernels on 152 SMs this admits d * m up to about 55,000: d = 1024 with
+ *     m = 32 fits, d = 4096 with m = 32 does not.
+ *   - Nothing in the array has to start at zero: every call writes the scratch it reads.
+ *   - The first call on each device looks up the array's device address (cudaGetSymbolAddress)
+ *     and keeps it; make that first call on a device before starting any stream capture on it.
+ *   - There is ONE array per device, shared by every call on that device. Calls enqueued on one
+ *     stream run one after the other and are safe; calls whose work can overlap in time (on
+ *     different streams, or from different host threads without ordering) race on the array
+ *     and give undefined results. Use resbm_decode_bwd with separate workspaces for those. */
+RESBM_API resbm_status resbm_decode_bwd_noalloc(const resbm_desc *desc, const void *dY,
+                                      const void *B, const void *Wd1, const void *Wd2,
+                                      void *dB, float *dWd1, float *dWd2, void *stream);
+
 /* One boundary forward and backward on one GPU, the pipeline handoff kept in device memory:
  * encode_fwd -> decode_fwd -> decode_bwd -> encode_bwd, in that order on `stream`. B produced
  * by the encoder is what the decoder reads; dB produced by the decoder backward is what the

@@ -277,6 +277,25 @@ resbm_status run_encode_bwd(const resbm_desc &d, const void *dB, const void *F, 
     return finish(generic_encode_bwd(d, dB, F, P, We1, We2, dF, dX, dWe1, dWe2, ws, c));
 }
 
+// ---- fixed scratch of resbm_decode_bwd_noalloc -----------------------------------------------
+// One array per device, reserved with the library's device code; its address is looked up on
+// the first call on each device and kept (all host threads share the cached value).
+static __device__ __align__(256) unsigned char g_static_scratch[RESBM_STATIC_SCRATCH_BYTES];
+std::atomic<void *> g_static_scratch_ptr[kMaxDevices];
+
+resbm_status static_scratch(int dev, void **out)
+{
+    if (dev < 0 || dev >= kMaxDevices) return RESBM_ERR_UNSUPPORTED;
+    void *p = g_static_scratch_ptr[dev].load(std::memory_order_acquire);
+    if (!p) {
+        cudaError_t e = cudaGetSymbolAddress(&p, g_static_scratch);
+        if (e != cudaSuccess) return cuda_fail(e);
+        g_static_scratch_ptr[dev].store(p, std::memory_order_release);
+    }
+    *out = p;
+    return RESBM_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -351,6 +370,22 @@ resbm_status resbm_decode_bwd(const resbm_desc *desc, const void *dY, const void
     if (s == RESBM_OK) s = check_ws(*desc, RESBM_OP_DECODE_BWD, ws, ws_bytes);
     Ctx c;
     if (s == RESBM_OK) s = make_ctx(stream, &c);
+    if (s == RESBM_OK) s = run_decode_bwd(*desc, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, c);
+    return s;
+}
+
+resbm_status resbm_decode_bwd_noalloc(const resbm_desc *desc, const void *dY, const void *B,
+                                      const void *Wd1, const void *Wd2, void *dB, float *dWd1,
+                                      float *dWd2, void *stream)
+{
+    resbm_status s = check_desc(desc);
+    if (s == RESBM_OK) s = validate_decode_bwd(*desc, dY, B, Wd1, Wd2, dB, dWd1, dWd2);
+    if (s == RESBM_OK && ws_for(*desc, RESBM_OP_DECODE_BWD) > RESBM_STATIC_SCRATCH_BYTES)
+        s = RESBM_ERR_WORKSPACE;
+    Ctx c;
+    if (s == RESBM_OK) s = make_ctx(stream, &c);
+    void *ws = nullptr;
+    if (s == RESBM_OK) s = static_scratch(c.device, &ws);
     if (s == RESBM_OK) s = run_decode_bwd(*desc, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, c);
     return s;
 }

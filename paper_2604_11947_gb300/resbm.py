@@ -20,6 +20,7 @@ RESBM_ACT_SILU, RESBM_ACT_GELU_TANH, RESBM_ACT_IDENTITY = 0, 1, 2
 (RESBM_OP_ENCODE_FWD, RESBM_OP_DECODE_FWD, RESBM_OP_DECODE_BWD, RESBM_OP_ENCODE_BWD,
  RESBM_OP_BOUNDARY_STEP) = range(5)
 RESBM_FLAG_GENERIC = 1
+RESBM_STATIC_SCRATCH_BYTES = 32 << 20
 
 ACTS = {"silu": RESBM_ACT_SILU, "gelu_tanh": RESBM_ACT_GELU_TANH, "identity": RESBM_ACT_IDENTITY}
 DTYPES = {"f32": RESBM_F32, "bf16": RESBM_BF16}
@@ -28,7 +29,7 @@ TORCH_DTYPES = {RESBM_F32: torch.float32, RESBM_BF16: torch.bfloat16}
 EXPORTS = ("resbm_version", "resbm_status_string", "resbm_last_cuda_error", "resbm_kernel_launches",
            "resbm_device_error",
            "resbm_workspace_bytes", "resbm_encode_fwd", "resbm_decode_fwd", "resbm_decode_bwd",
-           "resbm_encode_bwd", "resbm_boundary_step")
+           "resbm_encode_bwd", "resbm_boundary_step", "resbm_decode_bwd_noalloc")
 
 
 class resbm_desc(ctypes.Structure):
@@ -89,6 +90,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.resbm_encode_bwd.restype = i32
     lib.resbm_encode_bwd.argtypes = [D] + [vp] * 9 + [vp, sz, vp]
     lib.resbm_boundary_step.restype = i32
+    lib.resbm_decode_bwd_noalloc.restype = i32
+    lib.resbm_decode_bwd_noalloc.argtypes = [D] + [vp] * 7 + [vp]
     lib.resbm_boundary_step.argtypes = [D, ctypes.POINTER(resbm_step_args), vp, sz, vp]
     if path is None:
         _lib = lib
@@ -177,6 +180,13 @@ def resbm_decode_bwd(desc, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, stream=None):
     st = load().resbm_decode_bwd(ctypes.byref(desc), _p(dY), _p(B), _p(Wd1), _p(Wd2), _p(dB),
                                  _p(dWd1), _p(dWd2), _p(ws), _nbytes(ws), _stream(stream))
     _check("resbm_decode_bwd", st)
+
+
+def resbm_decode_bwd_noalloc(desc, dY, B, Wd1, Wd2, dB, dWd1, dWd2, stream=None):
+    """resbm_decode_bwd with the library's fixed device scratch instead of a workspace."""
+    st = load().resbm_decode_bwd_noalloc(ctypes.byref(desc), _p(dY), _p(B), _p(Wd1), _p(Wd2),
+                                         _p(dB), _p(dWd1), _p(dWd2), _stream(stream))
+    _check("resbm_decode_bwd_noalloc", st)
 
 
 def resbm_encode_bwd(desc, dB, F, P_save, We1, We2, dF, dX, dWe1, dWe2, ws, stream=None):
