@@ -147,10 +147,13 @@ BwdPlan bwd_plan(const resbm_desc &d, int sms, int nt, int64_t small_elems, void
     return p;
 }
 
-int reduce_grid(int64_t n, const Ctx &c)
+// Launch shape of k_reduce_slots: one block per 32 float4 columns (capped at 8 blocks per SM,
+// the blocks then stride over the rest).
+const dim3 kReduceBlock(32, tc::kSlotGroups);
+int reduce_grid(int64_t n4, const Ctx &c)
 {
-    int64_t g = (n + 255) / 256;
-    const int64_t cap = (int64_t)c.sm_count * 4;
+    int64_t g = (n4 + 31) / 32;
+    const int64_t cap = (int64_t)c.sm_count * 8;
     if (g > cap) g = cap;
     return (int)(g < 1 ? 1 : g);
 }
@@ -179,8 +182,8 @@ cudaError_t launch_dec_bwd(const resbm_desc &d, const void *dY, const void *B, c
     count_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     // dWd2 (m x d) = sum of the per-CTA slots (d x m), transposed; dWd1 (r x m) = sum of the slices
-    tc::k_reduce_slots<<<reduce_grid(d.d * d.m / 4, c), 256, 0, c.stream>>>(p.part_big, p.grid, d.d, d.m, dWd2, 1, 0);
-    tc::k_reduce_slots<<<reduce_grid(d.r * d.m / 4, c), 256, 0, c.stream>>>(p.part_small, p.slots, d.r, d.m, dWd1, 0,
+    tc::k_reduce_slots<<<reduce_grid(d.d * d.m / 4, c), kReduceBlock, 0, c.stream>>>(p.part_big, p.grid, d.d, d.m, dWd2, 1, 0);
+    tc::k_reduce_slots<<<reduce_grid(d.r * d.m / 4, c), kReduceBlock, 0, c.stream>>>(p.part_small, p.slots, d.r, d.m, dWd1, 0,
                                                                               al16(dWd1));
     count_launches(2);
     return cudaGetLastError();
@@ -237,9 +240,9 @@ cudaError_t launch_enc_bwd(const resbm_desc &d, const void *dB, const void *F, c
     tc::k_enc_bwd<M><<<p.grid, Cfg::THREADS, Cfg::SMEM_BYTES, c.stream>>>(m_f128, m_f16, m_we1, m_df128, m_df16, a);
     count_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    tc::k_reduce_slots<<<reduce_grid(d.d * d.m / 4, c), 256, 0, c.stream>>>(p.part_big, p.grid, d.d, d.m, dWe1, 0,
+    tc::k_reduce_slots<<<reduce_grid(d.d * d.m / 4, c), kReduceBlock, 0, c.stream>>>(p.part_big, p.grid, d.d, d.m, dWe1, 0,
                                                                             al16(dWe1));
-    tc::k_reduce_slots<<<reduce_grid(d.m * d.r / 4, c), 256, 0, c.stream>>>(p.part_small, p.slots, d.m, d.r, dWe2, 0,
+    tc::k_reduce_slots<<<reduce_grid(d.m * d.r / 4, c), kReduceBlock, 0, c.stream>>>(p.part_small, p.slots, d.m, d.r, dWe2, 0,
                                                                               al16(dWe2));
     count_launches(2);
     return cudaGetLastError();

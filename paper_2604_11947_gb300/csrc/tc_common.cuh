@@ -296,6 +296,13 @@ __device__ __forceinline__ uint64_t smem_desc(uint32_t addr, uint32_t lbo, uint3
     return d;
 }
 
+// Descriptor increment (bytes >> 4) of K step k (16 bf16 elements) inside a K-major operand of
+// 128-byte swizzled 64-column blocks: 4 steps of 32 bytes per block, blocks `block_bytes` apart.
+__host__ __device__ constexpr uint64_t kmaj_off(int k, uint32_t block_bytes)
+{
+    return (uint64_t)(((uint32_t)(k >> 2) * block_bytes + (uint32_t)(k & 3) * 32u) >> 4);
+}
+
 // Instruction descriptor for kind::f16 with bf16 A and B, fp32 D, dense, M x N.
 // a_mn / b_mn: operand stored MN-major (transposed) instead of K-major.
 __host__ __device__ constexpr uint32_t idesc_bf16(uint32_t M, uint32_t N, bool a_mn, bool b_mn)

@@ -189,6 +189,12 @@ __global__ void __launch_bounds__(192, 1)
         if (elect_one()) {
             constexpr uint32_t id_dg = idesc_bf16(128, C::M, false, false);  // dY (K-major) . Wd2 (K-major)
             constexpr uint32_t id_wt = idesc_bf16(128, C::M, true, false);   // dY^T (MN-major) . G^T (K-major)
+            // shared-memory descriptors of ring slot 0, advanced per slot and K step by adding the
+            // byte offset >> 4 to the start-address field (no carry: shared addresses < 256 KB)
+            const uint64_t yk0 = smem_desc(smem_u32(smem + C::OFF_Y), 16, 1024, kSwz128);     // dY, K-major
+            const uint64_t ym0 = smem_desc(smem_u32(smem + C::OFF_Y), 16384, 1024, kSwz128);  // dY, MN-major
+            const uint64_t wk0 = smem_desc(smem_u32(smem + C::OFF_W), 16, 1024, kSwz128);     // Wd2 slice
+            const uint64_t gk0 = smem_desc(smem_u32(smem + C::OFF_GT), 16, 1024, kSwz128);    // G^T tiles
             uint32_t yit = 0, wit = 0, cit = 0;
             bool ok = true;
             for (int g = 0; g < ngroups && ok; ++g) {
@@ -201,30 +207,40 @@ __global__ void __launch_bounds__(192, 1)
                     ok = mbar_wait(smem_u32(&w_full[sw]), (wit / C::NW) & 1) &&
                          mbar_wait(smem_u32(&wt_empty[ab]), ((cit >> 1) & 1) ^ 1);
                     tc_fence_after();
-                    const uint32_t waddr = smem_u32(smem + C::OFF_W + sw * C::W_STAGE);
+                    const uint64_t wk = wk0 + ((sw * C::W_STAGE) >> 4);
+                    const uint32_t d_wt = tmem_wt + ab * C::MS;
                     for (int i = tb; i < te && ok; ++i, ++yit) {
                         const int64_t t0 = start + 128 * (int64_t)i;
                         const int valid = (int)((end - t0) < 128 ? (end - t0) : 128);
                         const uint32_t s = yit % C::NSY;
                         ok = mbar_wait(smem_u32(&y_full[s]), (yit / C::NSY) & 1);
                         tc_fence_after();
-                        const uint32_t yaddr = smem_u32(smem + C::OFF_Y + s * C::Y_STAGE);
-                        const uint32_t gaddr = smem_u32(smem + C::OFF_GT + (i - tb) * C::GT_TILE);
+                        const uint64_t yk = yk0 + ((s * C::Y_STAGE) >> 4);
+                        const uint64_t ym = ym0 + ((s * C::Y_STAGE) >> 4);
+                        const uint64_t gk = gk0 + (((i - tb) * C::GT_TILE) >> 4);
+                        const uint32_t d_dg = tmem_dg + (i - tb) * C::MS;
+                        // dG_tile += dY_tile . Wd2_chunk^T: K = 128 columns in 8 steps of 16
+                        mma_bf16(d_dg, yk, wk, id_dg, c != 0);
 #pragma unroll
-                        for (int k = 0; k < 8; ++k) {
-                            const uint64_t ad = smem_desc(yaddr + (k >> 2) * 16384 + (k & 3) * 32, 16, 1024, kSwz128);
-                            const uint64_t bd = smem_desc(waddr + (k >> 2) * (C::M * 128) + (k & 3) * 32, 16, 1024, kSwz128);
-                            mma_bf16(tmem_dg + (i - tb) * C::MS, ad, bd, id_dg, (c | k) != 0);
+                        for (int k = 1; k < 8; ++k)
+                            mma_bf16(d_dg, yk + kmaj_off(k, 16384), wk + kmaj_off(k, C::M * 128), id_dg, true);
+                        // the dWd2 product needs the tile's G^T (published per tile in phase 0,
+                        // once per group; the dG products above did not wait for it)
+                        if (c == 0) {
+                            ok = ok && mbar_wait(smem_u32(&gt_full[i - tb]), g & 1);
+                            tc_fence_after();
                         }
-                        // the dWd2 product needs the tile's G^T (published per tile in phase 0;
-                        // the dG products above did not wait for it)
-                        ok = ok && mbar_wait(smem_u32(&gt_full[i - tb]), g & 1);
-                        tc_fence_after();
-                        const int nks = (valid + 15) / 16;
-                        for (int k = 0; k < nks; ++k) {
-                            const uint64_t ad = smem_desc(yaddr + k * 2048, 16384, 1024, kSwz128);
-                            const uint64_t bd = smem_desc(gaddr + (k >> 2) * (C::M * 128) + (k & 3) * 32, 16, 1024, kSwz128);
-                            mma_bf16(tmem_wt + ab * C::MS, ad, bd, id_wt, (i > tb) || (k > 0));
+                        // dWd2T_chunk += dY_tile^T . G_tile: K = the tile's tokens in steps of 16
+                        if (valid == 128) {
+#pragma unroll
+                            for (int k = 0; k < 8; ++k)
+                                mma_bf16(d_wt, ym + ((k * 2048) >> 4), gk + kmaj_off(k, C::M * 128), id_wt,
+                                         (i > tb) || (k > 0));
+                        } else {
+                            const int nks = (valid + 15) / 16;
+                            for (int k = 0; k < nks; ++k)
+                                mma_bf16(d_wt, ym + ((k * 2048) >> 4), gk + kmaj_off(k, C::M * 128), id_wt,
+                                         (i > tb) || (k > 0));
                         }
                         mma_commit(smem_u32(&y_empty[s]));
                     }
@@ -414,34 +430,57 @@ __device__ __forceinline__ void add4(float4 &a, const float4 &b)
     a.x += b.x; a.y += b.y; a.z += b.z; a.w += b.w;
 }
 
-__global__ void k_reduce_slots(const float *__restrict__ part, int64_t slots, int64_t rows, int64_t cols,
-                               float *__restrict__ out, int transpose, int out4)
+// Fixed-order sum of `slots` partial fp32 matrices (rows x cols, cols % 4 == 0) into `out`
+// (transposed to cols x rows if `transpose`; `out4`: out is 16-byte aligned). A block of
+// 32 x kSlotGroups threads owns 32 consecutive float4 columns of the flattened matrix; thread
+// row g sums the g-th contiguous range of slots in slot order, and the groups' sums are then
+// added in group order: the same order for every launch, so results are bitwise reproducible.
+constexpr int kSlotGroups = 16;
+
+__global__ void __launch_bounds__(32 * kSlotGroups) k_reduce_slots(const float *__restrict__ part, int64_t slots,
+                                                                   int64_t rows, int64_t cols,
+                                                                   float *__restrict__ out, int transpose, int out4)
 {
+    __shared__ float4 grp[kSlotGroups][32];
     const int64_t n4 = rows * cols / 4;
     const float4 *p4 = reinterpret_cast<const float4 *>(part);
-    for (int64_t e4 = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e4 < n4; e4 += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t per = (slots + kSlotGroups - 1) / kSlotGroups;
+    const int64_t s0 = threadIdx.y * per;
+    const int64_t s1 = s0 + per < slots ? s0 + per : slots;
+    for (int64_t base = (int64_t)blockIdx.x * 32; base < n4; base += (int64_t)gridDim.x * 32) {
+        const int64_t e4 = base + threadIdx.x;
         float4 acc = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
-        int64_t s = 0;
-        for (; s + 8 <= slots; s += 8) {
-            float4 v[8];
+        if (e4 < n4) {
+            int64_t s = s0;
+            for (; s + 4 <= s1; s += 4) {
+                float4 v[4];
 #pragma unroll
-            for (int u = 0; u < 8; ++u) v[u] = p4[(s + u) * n4 + e4];
+                for (int u = 0; u < 4; ++u) v[u] = __ldcs(&p4[(s + u) * n4 + e4]);
 #pragma unroll
-            for (int u = 0; u < 8; ++u) add4(acc, v[u]);
+                for (int u = 0; u < 4; ++u) add4(acc, v[u]);
+            }
+            for (; s < s1; ++s) add4(acc, __ldcs(&p4[s * n4 + e4]));
         }
-        for (; s < slots; ++s) add4(acc, p4[s * n4 + e4]);
-        const int64_t e = 4 * e4;
-        if (transpose) {
-            const int64_t rr = e / cols, cc = e - rr * cols;
-            out[(cc + 0) * rows + rr] = acc.x;
-            out[(cc + 1) * rows + rr] = acc.y;
-            out[(cc + 2) * rows + rr] = acc.z;
-            out[(cc + 3) * rows + rr] = acc.w;
-        } else if (out4) {
-            reinterpret_cast<float4 *>(out)[e4] = acc;
-        } else {
-            out[e] = acc.x; out[e + 1] = acc.y; out[e + 2] = acc.z; out[e + 3] = acc.w;
+        grp[threadIdx.y][threadIdx.x] = acc;
+        __syncthreads();
+        if (threadIdx.y == 0 && e4 < n4) {
+            float4 t = grp[0][threadIdx.x];
+#pragma unroll
+            for (int g = 1; g < kSlotGroups; ++g) add4(t, grp[g][threadIdx.x]);
+            const int64_t e = 4 * e4;
+            if (transpose) {
+                const int64_t rr = e / cols, cc = e - rr * cols;
+                out[(cc + 0) * rows + rr] = t.x;
+                out[(cc + 1) * rows + rr] = t.y;
+                out[(cc + 2) * rows + rr] = t.z;
+                out[(cc + 3) * rows + rr] = t.w;
+            } else if (out4) {
+                reinterpret_cast<float4 *>(out)[e4] = t;
+            } else {
+                out[e] = t.x; out[e + 1] = t.y; out[e + 2] = t.z; out[e + 3] = t.w;
+            }
         }
+        __syncthreads();
     }
 }
 

@@ -187,6 +187,12 @@ __global__ void __launch_bounds__(192, 1)
             constexpr Swz dswz = C::DSW == 128 ? kSwz128 : C::DSW == 64 ? kSwz64 : kSwz32;
             constexpr uint32_t id_df = idesc_bf16(128, 128, false, false);   // dP (K-major) . We1 (K-major)
             constexpr uint32_t id_we = idesc_bf16(128, C::M, true, false);   // F^T (MN-major) . dP^T (K-major)
+            // shared-memory descriptors of slot / tile 0, advanced by adding byte offset >> 4 to
+            // the start-address field (no carry: shared addresses < 256 KB)
+            const uint64_t fm0 = smem_desc(smem_u32(smem + C::OFF_F), 16384, 1024, kSwz128);   // F, MN-major
+            const uint64_t wd0 = smem_desc(smem_u32(smem + C::OFF_W), 16, 8 * C::DSW, dswz);   // We1 slice
+            const uint64_t pa0 = smem_desc(smem_u32(smem + C::OFF_DPA), 16, 8 * C::DSW, dswz); // dP
+            const uint64_t pt0 = smem_desc(smem_u32(smem + C::OFF_DPT), 16, 1024, kSwz128);    // dP^T
             uint32_t fit = 0, wit = 0, cit = 0, dfit = 0;
             bool ok = true;
             for (int g = 0; g < ngroups && ok; ++g) {
@@ -196,33 +202,37 @@ __global__ void __launch_bounds__(192, 1)
                     ok = mbar_wait(smem_u32(&w_full[sw]), (wit / C::NW) & 1) &&
                          mbar_wait(smem_u32(&we_empty[ae]), ((cit >> 1) & 1) ^ 1);
                     tc_fence_after();
-                    const uint32_t waddr = smem_u32(smem + C::OFF_W + sw * C::W_STAGE);
+                    const uint64_t wd = wd0 + ((sw * C::W_STAGE) >> 4);
+                    const uint32_t d_we = tmem_we + ae * C::MS;
                     for (int i = tb; i < te && ok; ++i, ++fit, ++dfit) {
                         const int64_t t0 = start + 128 * (int64_t)i;
                         const int valid = (int)((end - t0) < 128 ? (end - t0) : 128);
                         const uint32_t s = fit % C::NSF, ad_buf = dfit & 1;
-                        // dP of the tile (phase 0, published per tile), its F tile, a free dF buffer
-                        ok = mbar_wait(smem_u32(&dp_full[i - tb]), g & 1) &&
-                             mbar_wait(smem_u32(&f_full[s]), (fit / C::NSF) & 1) &&
+                        // dP of the tile (phase 0, published per tile once per group), its F
+                        // tile, a free dF buffer
+                        if (c == 0) ok = mbar_wait(smem_u32(&dp_full[i - tb]), g & 1);
+                        ok = ok && mbar_wait(smem_u32(&f_full[s]), (fit / C::NSF) & 1) &&
                              mbar_wait(smem_u32(&df_empty[ad_buf]), ((dfit >> 1) & 1) ^ 1);
                         tc_fence_after();
-                        const uint32_t faddr = smem_u32(smem + C::OFF_F + s * C::F_STAGE);
-                        const uint32_t pa = smem_u32(smem + C::OFF_DPA + (i - tb) * C::DPA_TILE);
-                        const uint32_t pt = smem_u32(smem + C::OFF_DPT + (i - tb) * C::DPT_TILE);
-                        // dF = dP . We1_chunk^T (K = m)
+                        const uint64_t fm = fm0 + ((s * C::F_STAGE) >> 4);
+                        const uint64_t pa = pa0 + (((i - tb) * C::DPA_TILE) >> 4);
+                        const uint64_t pt = pt0 + (((i - tb) * C::DPT_TILE) >> 4);
+                        const uint32_t d_df = tmem_df + ad_buf * 128;
+                        // dF = dP . We1_chunk^T (K = m in steps of 16 = 32 bytes of a swizzled row)
 #pragma unroll
-                        for (int k = 0; k < C::M / 16; ++k) {
-                            const uint64_t ad = smem_desc(pa + k * 32, 16, 8 * C::DSW, dswz);
-                            const uint64_t bd = smem_desc(waddr + k * 32, 16, 8 * C::DSW, dswz);
-                            mma_bf16(tmem_df + ad_buf * 128, ad, bd, id_df, k > 0);
-                        }
+                        for (int k = 0; k < C::M / 16; ++k) mma_bf16(d_df, pa + 2 * k, wd + 2 * k, id_df, k > 0);
                         mma_commit(smem_u32(&df_full[ad_buf]));
-                        // dWe1^T_chunk += F^T . dP  (K = tokens)
-                        const int nks = (valid + 15) / 16;
-                        for (int k = 0; k < nks; ++k) {
-                            const uint64_t ad = smem_desc(faddr + k * 2048, 16384, 1024, kSwz128);
-                            const uint64_t bd = smem_desc(pt + (k >> 2) * (C::M * 128) + (k & 3) * 32, 16, 1024, kSwz128);
-                            mma_bf16(tmem_we + ae * C::MS, ad, bd, id_we, (i > tb) || (k > 0));
+                        // dWe1^T_chunk += F^T . dP  (K = the tile's tokens in steps of 16)
+                        if (valid == 128) {
+#pragma unroll
+                            for (int k = 0; k < 8; ++k)
+                                mma_bf16(d_we, fm + ((k * 2048) >> 4), pt + kmaj_off(k, C::M * 128), id_we,
+                                         (i > tb) || (k > 0));
+                        } else {
+                            const int nks = (valid + 15) / 16;
+                            for (int k = 0; k < nks; ++k)
+                                mma_bf16(d_we, fm + ((k * 2048) >> 4), pt + kmaj_off(k, C::M * 128), id_we,
+                                         (i > tb) || (k > 0));
                         }
                         mma_commit(smem_u32(&f_empty[s]));
                     }
