@@ -158,27 +158,34 @@ int reduce_grid(int64_t n4, const Ctx &c)
     return (int)(g < 1 ? 1 : g);
 }
 
+CUtensorMapSwizzle swizzle_for(uint32_t row_bytes)
+{
+    return row_bytes == 128 ? CU_TENSOR_MAP_SWIZZLE_128B
+           : row_bytes == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
+                             : CU_TENSOR_MAP_SWIZZLE_32B;
+}
+
 template <int M>
 cudaError_t launch_dec_bwd(const resbm_desc &d, const void *dY, const void *B, const void *Wd1, const void *Wd2,
                            void *dB, float *dWd1, float *dWd2, void *ws, const Ctx &c)
 {
     using Cfg = tc::DecBwdCfg<M>;
     const BwdPlan p = bwd_plan(d, c.sm_count, Cfg::NT, d.r * d.m, ws);
-    CUtensorMap m_dy128, m_dy16, m_wd2;
+    CUtensorMap m_dy128, m_dy16, m_wd2, m_b, m_yr;
     if (!make_map(&m_dy128, dY, d.d, d.T, d.d * 2, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B) ||
         !make_map(&m_dy16, dY, d.d, d.T, d.d * 2, 64, 16, CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !make_map(&m_wd2, Wd2, d.d, d.m, d.d * 2, 64, M, CU_TENSOR_MAP_SWIZZLE_128B))
+        !make_map(&m_wd2, Wd2, d.d, d.m, d.d * 2, 64, M, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&m_b, B, d.r, d.T, d.r * 2, M, 128, swizzle_for(Cfg::RB)) ||
+        !make_map(&m_yr, dY, d.d, d.T, d.d * 2, M, 128, swizzle_for(Cfg::RB)))
         return cudaErrorInvalidValue;
     static std::atomic<uint8_t> smem_set[kMaxDev];
     cudaError_t e = ensure_smem(tc::k_dec_bwd<M>, Cfg::SMEM_BYTES, c.device, smem_set);
     if (e != cudaSuccess) return e;
-    tc::DecBwdArgs a{static_cast<const __nv_bfloat16 *>(B),
-                     static_cast<const __nv_bfloat16 *>(Wd1),
-                     static_cast<const __nv_bfloat16 *>(dY),
+    tc::DecBwdArgs a{static_cast<const __nv_bfloat16 *>(Wd1),
                      static_cast<__nv_bfloat16 *>(dB),
                      tc::WgradArgs{p.part_big, p.nch},
                      p.part_small, d.T, d.d, d.act, d.merge_identity, p.max_groups};
-    tc::k_dec_bwd<M><<<p.grid, Cfg::THREADS, Cfg::SMEM_BYTES, c.stream>>>(m_dy128, m_dy16, m_wd2, a);
+    tc::k_dec_bwd<M><<<p.grid, Cfg::THREADS, Cfg::SMEM_BYTES, c.stream>>>(m_dy128, m_dy16, m_wd2, m_b, m_yr, a);
     count_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     // dWd2 (m x d) = sum of the per-CTA slots (d x m), transposed; dWd1 (r x m) = sum of the slices
@@ -187,6 +194,11 @@ cudaError_t launch_dec_bwd(const resbm_desc &d, const void *dY, const void *B, c
                                                                               al16(dWd1));
     count_launches(2);
     return cudaGetLastError();
+}
+
+int dec_bwd_nt(int64_t m)
+{
+    return m <= 16 ? tc::DecBwdCfg<16>::NT : m <= 32 ? tc::DecBwdCfg<32>::NT : tc::DecBwdCfg<64>::NT;
 }
 
 // Scratch of the encoder backward: P (T x m fp32, used when the caller has none) and the slots.
@@ -202,7 +214,7 @@ EncBwdWs enc_bwd_ws(const resbm_desc &d, int sms, void *ws)
     WsCarver c(ws);
     w.P = c.take<float>(d.T * d.m);
     char *rest = c.take<char>(0);
-    const int nt = d.m <= 32 ? 4 : 2;
+    const int nt = d.m <= 16 ? tc::EncBwdCfg<16>::NT : d.m <= 32 ? tc::EncBwdCfg<32>::NT : tc::EncBwdCfg<64>::NT;
     w.plan = bwd_plan(d, sms, nt, d.m * d.r, ws ? rest : nullptr);
     w.bytes = c.used + w.plan.bytes;
     return w;
@@ -215,15 +227,13 @@ cudaError_t launch_enc_bwd(const resbm_desc &d, const void *dB, const void *F, c
     using Cfg = tc::EncBwdCfg<M>;
     const EncBwdWs w = enc_bwd_ws(d, c.sm_count, ws);
     const BwdPlan &p = w.plan;
-    const CUtensorMapSwizzle dswz = Cfg::DSW == 128  ? CU_TENSOR_MAP_SWIZZLE_128B
-                                    : Cfg::DSW == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
-                                                     : CU_TENSOR_MAP_SWIZZLE_32B;
-    CUtensorMap m_f128, m_f16, m_we1, m_df128, m_df16;
+    CUtensorMap m_f128, m_f16, m_we1, m_df128, m_df16, m_db;
     if (!make_map(&m_f128, F, d.d, d.T, d.d * 2, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B) ||
         !make_map(&m_f16, F, d.d, d.T, d.d * 2, 64, 16, CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !make_map(&m_we1, We1, d.m, d.d, d.m * 2, M, 128, dswz) ||
+        !make_map(&m_we1, We1, d.m, d.d, d.m * 2, M, 128, swizzle_for(Cfg::RB)) ||
         !make_map(&m_df128, dF, d.d, d.T, d.d * 2, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !make_map(&m_df16, dF, d.d, d.T, d.d * 2, 64, 16, CU_TENSOR_MAP_SWIZZLE_128B))
+        !make_map(&m_df16, dF, d.d, d.T, d.d * 2, 64, 16, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&m_db, dB, d.r, d.T, d.r * 2, M, 128, swizzle_for(Cfg::RB)))
         return cudaErrorInvalidValue;
     cudaError_t e;
     if (!P) {  // P = F . We1 with the forward kernel (no B), so it matches a saved P bit for bit
@@ -234,10 +244,10 @@ cudaError_t launch_enc_bwd(const resbm_desc &d, const void *dB, const void *F, c
     static std::atomic<uint8_t> smem_set[kMaxDev];
     e = ensure_smem(tc::k_enc_bwd<M>, Cfg::SMEM_BYTES, c.device, smem_set);
     if (e != cudaSuccess) return e;
-    tc::EncBwdArgs a{static_cast<const __nv_bfloat16 *>(dB), P, static_cast<const __nv_bfloat16 *>(We2),
-                     static_cast<__nv_bfloat16 *>(dX), tc::WgradArgs{p.part_big, p.nch},
-                     p.part_small, d.T, d.d, d.act, p.max_groups};
-    tc::k_enc_bwd<M><<<p.grid, Cfg::THREADS, Cfg::SMEM_BYTES, c.stream>>>(m_f128, m_f16, m_we1, m_df128, m_df16, a);
+    tc::EncBwdArgs a{P, static_cast<const __nv_bfloat16 *>(We2), static_cast<__nv_bfloat16 *>(dX),
+                     tc::WgradArgs{p.part_big, p.nch}, p.part_small, d.T, d.d, d.act, p.max_groups};
+    tc::k_enc_bwd<M><<<p.grid, Cfg::THREADS, Cfg::SMEM_BYTES, c.stream>>>(m_f128, m_f16, m_we1, m_df128, m_df16,
+                                                                          m_db, a);
     count_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     tc::k_reduce_slots<<<reduce_grid(d.d * d.m / 4, c), kReduceBlock, 0, c.stream>>>(p.part_big, p.grid, d.d, d.m, dWe1, 0,
@@ -265,7 +275,7 @@ bool tc_supported(const resbm_desc &d, int op)
 
 size_t tc_ws_bytes(const resbm_desc &d, int op, int sms)
 {
-    if (op == RESBM_OP_DECODE_BWD) return bwd_plan(d, sms, 4, d.r * d.m, nullptr).bytes;
+    if (op == RESBM_OP_DECODE_BWD) return bwd_plan(d, sms, dec_bwd_nt(d.m), d.r * d.m, nullptr).bytes;
     if (op == RESBM_OP_ENCODE_BWD) return enc_bwd_ws(d, sms, nullptr).bytes;
     return 0;
 }

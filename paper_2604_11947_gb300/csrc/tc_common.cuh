@@ -325,5 +325,54 @@ __device__ __forceinline__ uint32_t swz_offset(uint32_t row, uint32_t byte_in_ro
     return row * row_bytes + (((chunk ^ sel) & mask) << 4) + (byte_in_row & 15u);
 }
 
+// The N (a multiple of 16) fp32 TMEM columns at taddr of this thread's lane (warp-collective).
+template <int N> __device__ __forceinline__ void tmem_ld_row(uint32_t taddr, float (&v)[N])
+{
+#pragma unroll
+    for (int j = 0; j < N; j += 16) {
+        float t[16];
+        tmem_ld16(taddr + j, t);
+        tmem_ld_wait();
+#pragma unroll
+        for (int e = 0; e < 16; ++e) v[j + e] = t[e];
+    }
+}
+
+// Row `row` of a swizzled bf16 tile whose rows are N elements (2N bytes, the swizzle width):
+// store N fp32 values rounded to bf16, or load them back as fp32 (16-byte accesses).
+template <int N> __device__ __forceinline__ void store_bf16_swz_row(uint8_t *tile, int row, const float (&v)[N])
+{
+#pragma unroll
+    for (int cc = 0; cc < N / 8; ++cc) {
+        uint32_t pk[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            __nv_bfloat162 h = __floats2bfloat162_rn(v[8 * cc + 2 * e], v[8 * cc + 2 * e + 1]);
+            pk[e] = *reinterpret_cast<uint32_t *>(&h);
+        }
+        *reinterpret_cast<uint4 *>(tile + swz_offset(row, 16 * cc, 2 * N)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+    }
+}
+
+template <int N> __device__ __forceinline__ void load_bf16_swz_row(const uint8_t *tile, int row, float (&v)[N])
+{
+#pragma unroll
+    for (int cc = 0; cc < N / 8; ++cc) {
+        const uint4 u = *reinterpret_cast<const uint4 *>(tile + swz_offset(row, 16 * cc, 2 * N));
+        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            v[8 * cc + 2 * e] = __uint_as_float(w[e] << 16);
+            v[8 * cc + 2 * e + 1] = __uint_as_float(w[e] & 0xFFFF0000u);
+        }
+    }
+}
+
+// Swizzle mode of a K-major or MN-major operand whose rows are `row_bytes` (32, 64 or 128).
+__host__ __device__ constexpr Swz swz_for(uint32_t row_bytes)
+{
+    return row_bytes == 128 ? kSwz128 : row_bytes == 64 ? kSwz64 : kSwz32;
+}
+
 }  // namespace tc
 }  // namespace resbm

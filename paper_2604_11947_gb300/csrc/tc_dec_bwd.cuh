@@ -1,22 +1,28 @@
 // tc_dec_bwd.cuh -- backward of the receive side on tensor cores (chain rule of Sec. 3.2's
 // decoder with the zero-padding identity path of Eq. Pid):
-//   G = phi(Q), Q = B . Wd1;  dG = dY . Wd2^T;  dQ = dG * phi'(Q);
+//   Q = B . Wd1, G = phi(Q);  dG = dY . Wd2^T;  dQ = dG * phi'(Q);
 //   dB = [merge] dY[:, :r] + dQ . Wd1^T;  dWd2 = G^T . dY;  dWd1 = B^T . dQ.
 //
 // Persistent CTAs over contiguous 16-token-aligned token ranges, processed in groups of up to
-// NT tiles of 128 tokens. For each group:
-//   phase 0 (epilogue warps): Q, G on CUDA cores; G^T (m rows x 128 tokens per tile, K-major
-//            over tokens, 128B swizzle) into shared memory.
-//   phase 1 (producer + MMA): d in chunks of 128 columns; per chunk one Wd2 slice (K-major) and,
-//            per tile, one dY tile (128 tokens x 128 columns) feeding two MMAs:
+// NT tiles of 128 tokens. Every product runs on tcgen05; the CUDA cores only apply phi and phi'
+// and convert. For each group:
+//   phase 0: the group's B tiles (TMA) -> Q_tile = B . Wd1 in TMEM (kept for phase 2) -> the
+//            epilogue writes G = phi(Q) as bf16 rows [token][m] to shared memory.
+//   phase 1: d in chunks of 128 columns; per chunk one Wd2 slice and, per tile, one dY tile
+//            (128 tokens x 128 columns) feeding two MMAs:
 //              dG_tile   (128 tokens x m, TMEM, kept over all chunks) += dY . Wd2_chunk^T
 //              dWd2T_chk (128 columns x m, TMEM, double-buffered)     += dY^T . G_tile
-//            (the second MMA reads the same shared-memory tile as an MN-major operand).
-//            The epilogue warps drain each finished dWd2T chunk to the fp32 partial slot.
-//   phase 2 (epilogue warps): dQ, dB, and the dWd1 partial (B^T . dQ summed over the group's
-//            tokens in a fixed order, via the then idle dY ring as scratch).
+//            (the same dY stage read K-major and MN-major; G read MN-major). The epilogue
+//            drains each finished dWd2T chunk to the CTA's fp32 partial slot.
+//   phase 2: the epilogue writes dQ = dG * phi'(Q) as two bf16 tiles hi + lo (rows [token][m],
+//            in the idle dY ring; hi = dQ rounded to bf16, lo = the rounded remainder, so the
+//            products see dQ to about 16 significant bits: dB crosses the boundary and is
+//            rounded again there) -> dB_tile = dQ . Wd1^T (into the tile's dG columns) and
+//            dWd1 += B^T . dQ over the group's tokens (the B tile read MN-major as a 128-row
+//            operand whose rows >= r are never read back) -> the epilogue adds [merge]
+//            dY[:, :r] (a TMA tile) and stores dB as bf16; the group's dWd1 goes to its slot.
 // A second kernel sums the partial slots in a fixed order (deterministic).
-// HBM traffic per token: read dY (2d), B (2r), dY[:, :r] again (2r, L2), write dB (2r);
+// HBM traffic per token: read dY (2d), B (2r), dY[:, :r] again (2r, mostly L2), write dB (2r);
 // per slot: d x m + r x m fp32 partials.
 #pragma once
 
@@ -31,30 +37,38 @@ template <int M_> struct DecBwdCfg {
     static constexpr int M = M_;
     static constexpr int R = M_;
     static constexpr int MS = M_ < 32 ? 32 : M_;              // TMEM columns per accumulator
-    static constexpr int NT = 4;                              // tiles per group
+    static constexpr int NT = M_ <= 32 ? 4 : 2;               // tiles per group
     static constexpr int NSY = M_ <= 32 ? 4 : 3;              // dY ring depth
+    static constexpr int NW = M_ <= 16 ? 4 : 3;               // Wd2 slice ring depth
+    static constexpr uint32_t RB = M_ * 2;                    // row bytes (= swizzle) of the r / m wide tiles
     static constexpr uint32_t Y_STAGE = 128 * 128 * 2;        // 128 tokens x 128 columns
     static constexpr uint32_t W_STAGE = M_ * 128 * 2;         // m rows x 128 columns
-    static constexpr uint32_t GT_TILE = M_ * 128 * 2;         // m rows x 128 tokens
+    static constexpr uint32_t TILE = 128 * RB;                // 128 tokens x r (or m) columns
     static constexpr uint32_t WD1_BYTES = R * M_ * 2;
     static constexpr uint32_t OFF_Y = 0;
     static constexpr uint32_t OFF_W = OFF_Y + NSY * Y_STAGE;
-    static constexpr int NW = M_ <= 32 ? 4 : 3;               // Wd2 slice ring depth
-    static constexpr uint32_t OFF_GT = OFF_W + NW * W_STAGE;
-    static constexpr uint32_t OFF_WD1 = OFF_GT + NT * GT_TILE;
-    static constexpr uint32_t OFF_WD1T = OFF_WD1 + WD1_BYTES;
+    static constexpr uint32_t OFF_G = OFF_W + NW * W_STAGE;   // G tiles [token][m]
+    static constexpr uint32_t OFF_B = OFF_G + NT * TILE;      // B tiles [token][r] (TMA)
+    static constexpr uint32_t OFF_WD1 = OFF_B + NT * TILE;    // Wd1 [r][m]: K-major B operand of dQ . Wd1^T
+    static constexpr uint32_t OFF_WD1T = OFF_WD1 + WD1_BYTES; // Wd1^T [m][r]: K-major B operand of B . Wd1
     static constexpr uint32_t SMEM_BYTES = OFF_WD1T + WD1_BYTES + 1024;
-    static constexpr uint32_t TMEM_NEED = (NT + 2) * MS;
+    // phase-2 scratch in the idle dY ring: dQ hi tiles (slot 0), dY[:, :r] tiles (slot 1),
+    // dQ lo tiles (slot 2)
+    static constexpr uint32_t OFF_DQ = OFF_Y;
+    static constexpr uint32_t OFF_YR = OFF_Y + Y_STAGE;
+    static constexpr uint32_t OFF_DQLO = OFF_Y + 2 * Y_STAGE;
+    static_assert(NT * TILE <= Y_STAGE && NSY >= 3, "phase-2 scratch must fit in three ring slots");
+    static_assert(SMEM_BYTES <= 232448 - 512, "shared memory budget");
+    // TMEM columns: dG (later dB) NT x MS | Q NT x MS | dWd2T 2 x MS | dWd1 MS
+    static constexpr uint32_t TM_DG = 0, TM_Q = NT * MS, TM_WT = 2 * NT * MS, TM_W1 = TM_WT + 2 * MS;
+    static constexpr uint32_t TMEM_NEED = TM_W1 + MS;
+    static_assert(TMEM_NEED <= 512, "TMEM budget");
     static constexpr uint32_t TMEM_COLS = TMEM_NEED <= 128 ? 128 : TMEM_NEED <= 256 ? 256 : 512;
-    static constexpr uint32_t SCRATCH_BYTES = 128 * (R + M_ + 2) * 4;   // phase 2, inside the dY ring
-    static_assert(SCRATCH_BYTES <= NSY * Y_STAGE, "phase-2 scratch must fit in the dY ring");
     static constexpr int THREADS = 192;
 };
 
 struct DecBwdArgs {
-    const __nv_bfloat16 *B;    // T x r
     const __nv_bfloat16 *Wd1;  // r x m
-    const __nv_bfloat16 *dY;   // T x d (first r columns re-read for the identity path)
     __nv_bfloat16 *dB;         // T x r
     WgradArgs wg;              // dWd2^T chunks (d x m), reduced across CTAs
     float *part1;              // slots x r x m   (dWd1 partials)
@@ -65,13 +79,15 @@ struct DecBwdArgs {
 template <int M_>
 __global__ void __launch_bounds__(192, 1)
     k_dec_bwd(const __grid_constant__ CUtensorMap tm_dy128, const __grid_constant__ CUtensorMap tm_dy16,
-              const __grid_constant__ CUtensorMap tm_wd2, const DecBwdArgs a)
+              const __grid_constant__ CUtensorMap tm_wd2, const __grid_constant__ CUtensorMap tm_b,
+              const __grid_constant__ CUtensorMap tm_yr, const DecBwdArgs a)
 {
     using C = DecBwdCfg<M_>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     __shared__ uint64_t y_full[C::NSY], y_empty[C::NSY], w_full[C::NW], w_empty[C::NW];
-    __shared__ uint64_t gt_full[C::NT], gt_empty, wt_full[2], wt_empty[2], dg_full, dg_empty, p2_done, done_bar;
+    __shared__ uint64_t b_full, q_full, g_full[C::NT], g_empty, wt_full[2], wt_empty[2], dg_full, dg_empty;
+    __shared__ uint64_t yr_full, dq_full[C::NT], db_full[C::NT], w1_full, p2_done, done_bar;
     __shared__ uint32_t tmem_base_sh;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -94,28 +110,37 @@ __global__ void __launch_bounds__(192, 1)
             mbar_init(smem_u32(&wt_full[i]), 1);
             mbar_init(smem_u32(&wt_empty[i]), 128);
         }
-        for (int i = 0; i < C::NT; ++i) mbar_init(smem_u32(&gt_full[i]), 1);
-        mbar_init(smem_u32(&gt_empty), 1);
+        for (int i = 0; i < C::NT; ++i) {
+            mbar_init(smem_u32(&g_full[i]), 1);
+            mbar_init(smem_u32(&dq_full[i]), 1);
+            mbar_init(smem_u32(&db_full[i]), 1);
+        }
+        mbar_init(smem_u32(&b_full), 1);
+        mbar_init(smem_u32(&q_full), 1);
+        mbar_init(smem_u32(&g_empty), 1);
         mbar_init(smem_u32(&dg_full), 1);
         mbar_init(smem_u32(&dg_empty), 128);
+        mbar_init(smem_u32(&yr_full), 1);
+        mbar_init(smem_u32(&w1_full), 1);
         mbar_init(smem_u32(&p2_done), 1);
         mbar_init(smem_u32(&done_bar), 1);
         fence_mbar_init();
     }
     if (warp == 1) tmem_alloc(smem_u32(&tmem_base_sh), C::TMEM_COLS);
-    if (warp >= 2) {  // Wd1 (r x m) and its transpose (m x r), bf16, into shared memory
-        const uint4 *src = reinterpret_cast<const uint4 *>(a.Wd1);
-        uint4 *dst = reinterpret_cast<uint4 *>(smem + C::OFF_WD1);
-        for (int i = threadIdx.x - 64; i < (int)(C::WD1_BYTES / 16); i += 128) dst[i] = src[i];
-        __nv_bfloat16 *dt = reinterpret_cast<__nv_bfloat16 *>(smem + C::OFF_WD1T);
-        for (int e = threadIdx.x - 64; e < C::R * C::M; e += 128) dt[(e % C::M) * C::R + e / C::M] = a.Wd1[e];
+    if (warp >= 2) {  // Wd1 (r x m) and Wd1^T (m x r) as swizzled K-major operands
+        const int et = threadIdx.x - 64;
+        for (int e = et; e < C::R * C::M; e += 128) {
+            const int i = e / C::M, j = e % C::M;
+            const __nv_bfloat16 v = a.Wd1[e];
+            *reinterpret_cast<__nv_bfloat16 *>(smem + C::OFF_WD1 + swz_offset(i, 2 * j, C::RB)) = v;
+            *reinterpret_cast<__nv_bfloat16 *>(smem + C::OFF_WD1T + swz_offset(j, 2 * i, C::RB)) = v;
+        }
+        fence_async_smem();
     }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = tmem_base_sh;
-    const uint32_t tmem_dg = tmem;                     // NT accumulators of MS columns
-    const uint32_t tmem_wt = tmem + C::NT * C::MS;     // 2 accumulators of MS columns
 
     if (warp == 0) {
         // ---------------- producer ----------------
@@ -123,11 +148,23 @@ __global__ void __launch_bounds__(192, 1)
             tma_prefetch_desc(&tm_dy128);
             tma_prefetch_desc(&tm_dy16);
             tma_prefetch_desc(&tm_wd2);
+            tma_prefetch_desc(&tm_b);
+            tma_prefetch_desc(&tm_yr);
             uint32_t yit = 0, wit = 0;
+            int b_issued = 0, yr_issued = 0;
             bool ok = true;
             for (int g = 0; g < ngroups && ok; ++g) {
-                if (g > 0) ok = mbar_wait(smem_u32(&p2_done), (g - 1) & 1);  // the ring was scratch
+                // the ring, the B tiles and the phase-2 scratch of the previous group are free
+                if (g > 0) ok = mbar_wait(smem_u32(&p2_done), (g - 1) & 1);
+                if (!ok) break;
                 const int tb = g * C::NT, te = min(ntiles, tb + C::NT);
+                // the group's B tiles (128-row boxes: rows past T read as zeros, rows past this
+                // CTA's range are loaded but never used)
+                mbar_expect_tx(smem_u32(&b_full), (uint32_t)(te - tb) * C::TILE);
+                for (int i = tb; i < te; ++i)
+                    tma_load_2d(smem_u32(smem + C::OFF_B + (i - tb) * C::TILE), &tm_b, 0,
+                                (int32_t)(start + 128 * (int64_t)i), smem_u32(&b_full));
+                ++b_issued;
                 for (int c = 0; c < nch && ok; ++c) {
                     // order: dY tile 0 of the chunk, the chunk's Wd2 slice, the other dY tiles.
                     // The MMA needs the slice before any tile of the chunk, so it must not queue
@@ -173,6 +210,15 @@ __global__ void __launch_bounds__(192, 1)
                         ++wit;
                     }
                 }
+                if (!ok) break;
+                // dY[:, :r] tiles for phase 2, into ring slot 1 once the group's MMAs are done
+                // with the ring
+                if (!mbar_wait(smem_u32(&dg_full), g & 1)) { ok = false; break; }
+                mbar_expect_tx(smem_u32(&yr_full), (uint32_t)(te - tb) * C::TILE);
+                for (int i = tb; i < te; ++i)
+                    tma_load_2d(smem_u32(smem + C::OFF_YR + (i - tb) * C::TILE), &tm_yr, 0,
+                                (int32_t)(start + 128 * (int64_t)i), smem_u32(&yr_full));
+                ++yr_issued;
             }
             // drain the loads still in flight
             for (uint32_t k = 0; k < (yit < (uint32_t)C::NSY ? yit : (uint32_t)C::NSY); ++k) {
@@ -183,24 +229,52 @@ __global__ void __launch_bounds__(192, 1)
                 const uint32_t j = wit - 1 - k;
                 mbar_wait(smem_u32(&w_full[j % C::NW]), (j / C::NW) & 1);
             }
+            if (b_issued > 0) mbar_wait(smem_u32(&b_full), (b_issued - 1) & 1);
+            if (yr_issued > 0) mbar_wait(smem_u32(&yr_full), (yr_issued - 1) & 1);
         }
     } else if (warp == 1) {
         // ---------------- MMA issuer ----------------
         if (elect_one()) {
+            constexpr Swz rsw = swz_for(C::RB);
+            constexpr uint32_t id_q = idesc_bf16(128, C::M, false, false);   // B (K-major) . Wd1 (Wd1^T rows, K-major)
             constexpr uint32_t id_dg = idesc_bf16(128, C::M, false, false);  // dY (K-major) . Wd2 (K-major)
-            constexpr uint32_t id_wt = idesc_bf16(128, C::M, true, false);   // dY^T (MN-major) . G^T (K-major)
-            // shared-memory descriptors of ring slot 0, advanced per slot and K step by adding the
-            // byte offset >> 4 to the start-address field (no carry: shared addresses < 256 KB)
+            constexpr uint32_t id_wt = idesc_bf16(128, C::M, true, true);    // dY^T (MN-major) . G (MN-major)
+            constexpr uint32_t id_db = idesc_bf16(128, C::R, false, false);  // dQ (K-major) . Wd1^T (Wd1 rows, K-major)
+            constexpr uint32_t id_w1 = idesc_bf16(128, C::M, true, true);    // B^T (MN-major) . dQ (MN-major)
+            // shared-memory descriptors of slot / tile 0, advanced by adding the byte offset >> 4
+            // to the start-address field (no carry: shared addresses < 256 KB). The 128-row B^T
+            // operand has one real block of r rows: its block stride (LBO) is 0, so every block
+            // reads the same r rows and the extra output rows are duplicates.
             const uint64_t yk0 = smem_desc(smem_u32(smem + C::OFF_Y), 16, 1024, kSwz128);     // dY, K-major
             const uint64_t ym0 = smem_desc(smem_u32(smem + C::OFF_Y), 16384, 1024, kSwz128);  // dY, MN-major
             const uint64_t wk0 = smem_desc(smem_u32(smem + C::OFF_W), 16, 1024, kSwz128);     // Wd2 slice
-            const uint64_t gk0 = smem_desc(smem_u32(smem + C::OFF_GT), 16, 1024, kSwz128);    // G^T tiles
+            const uint64_t gm0 = smem_desc(smem_u32(smem + C::OFF_G), 0, 8 * C::RB, rsw);     // G, MN-major
+            const uint64_t bk0 = smem_desc(smem_u32(smem + C::OFF_B), 16, 8 * C::RB, rsw);    // B, K-major
+            const uint64_t bm0 = smem_desc(smem_u32(smem + C::OFF_B), 0, 8 * C::RB, rsw);     // B^T, MN-major
+            const uint64_t qk0 = smem_desc(smem_u32(smem + C::OFF_DQ), 16, 8 * C::RB, rsw);   // dQ, K-major
+            const uint64_t qm0 = smem_desc(smem_u32(smem + C::OFF_DQ), 0, 8 * C::RB, rsw);    // dQ, MN-major
+            const uint64_t w1k = smem_desc(smem_u32(smem + C::OFF_WD1), 16, 8 * C::RB, rsw);  // Wd1 rows
+            const uint64_t w1t = smem_desc(smem_u32(smem + C::OFF_WD1T), 16, 8 * C::RB, rsw); // Wd1^T rows
+            constexpr uint64_t TILE16 = C::TILE >> 4;
+            constexpr uint64_t KROWS16 = (16 * C::RB) >> 4;                 // 16 token rows of an r / m wide tile
+            constexpr uint64_t LO16 = (C::OFF_DQLO - C::OFF_DQ) >> 4;       // dQ hi tile -> lo tile
             uint32_t yit = 0, wit = 0, cit = 0;
             bool ok = true;
             for (int g = 0; g < ngroups && ok; ++g) {
                 const int tb = g * C::NT, te = min(ntiles, tb + C::NT);
+                // TMEM of the previous group (dG / dB, Q, dWd1) has been read out
                 if (g > 0) ok = mbar_wait(smem_u32(&dg_empty), (g - 1) & 1);
+                ok = ok && mbar_wait(smem_u32(&b_full), g & 1);
                 tc_fence_after();
+                // ---- phase 0: Q_tile = B_tile . Wd1 (K = r) ----
+                for (int i = tb; i < te && ok; ++i) {
+                    const uint64_t bk = bk0 + (i - tb) * TILE16;
+#pragma unroll
+                    for (int k = 0; k < C::R / 16; ++k)
+                        mma_bf16(tmem + C::TM_Q + (i - tb) * C::MS, bk + 2 * k, w1t + 2 * k, id_q, k > 0);
+                }
+                mma_commit(smem_u32(&q_full));
+                // ---- phase 1: the dY stream ----
                 for (int c = 0; c < nch && ok; ++c, ++cit) {
                     const uint32_t sw = wit % C::NW;
                     const uint32_t ab = cit & 1;
@@ -208,7 +282,7 @@ __global__ void __launch_bounds__(192, 1)
                          mbar_wait(smem_u32(&wt_empty[ab]), ((cit >> 1) & 1) ^ 1);
                     tc_fence_after();
                     const uint64_t wk = wk0 + ((sw * C::W_STAGE) >> 4);
-                    const uint32_t d_wt = tmem_wt + ab * C::MS;
+                    const uint32_t d_wt = tmem + C::TM_WT + ab * C::MS;
                     for (int i = tb; i < te && ok; ++i, ++yit) {
                         const int64_t t0 = start + 128 * (int64_t)i;
                         const int valid = (int)((end - t0) < 128 ? (end - t0) : 128);
@@ -217,30 +291,28 @@ __global__ void __launch_bounds__(192, 1)
                         tc_fence_after();
                         const uint64_t yk = yk0 + ((s * C::Y_STAGE) >> 4);
                         const uint64_t ym = ym0 + ((s * C::Y_STAGE) >> 4);
-                        const uint64_t gk = gk0 + (((i - tb) * C::GT_TILE) >> 4);
-                        const uint32_t d_dg = tmem_dg + (i - tb) * C::MS;
+                        const uint64_t gm = gm0 + (i - tb) * TILE16;
+                        const uint32_t d_dg = tmem + C::TM_DG + (i - tb) * C::MS;
                         // dG_tile += dY_tile . Wd2_chunk^T: K = 128 columns in 8 steps of 16
                         mma_bf16(d_dg, yk, wk, id_dg, c != 0);
 #pragma unroll
                         for (int k = 1; k < 8; ++k)
                             mma_bf16(d_dg, yk + kmaj_off(k, 16384), wk + kmaj_off(k, C::M * 128), id_dg, true);
-                        // the dWd2 product needs the tile's G^T (published per tile in phase 0,
+                        // the dWd2 product needs the tile's G (published per tile in phase 0,
                         // once per group; the dG products above did not wait for it)
                         if (c == 0) {
-                            ok = ok && mbar_wait(smem_u32(&gt_full[i - tb]), g & 1);
+                            ok = ok && mbar_wait(smem_u32(&g_full[i - tb]), g & 1);
                             tc_fence_after();
                         }
                         // dWd2T_chunk += dY_tile^T . G_tile: K = the tile's tokens in steps of 16
                         if (valid == 128) {
 #pragma unroll
                             for (int k = 0; k < 8; ++k)
-                                mma_bf16(d_wt, ym + ((k * 2048) >> 4), gk + kmaj_off(k, C::M * 128), id_wt,
-                                         (i > tb) || (k > 0));
+                                mma_bf16(d_wt, ym + ((k * 2048) >> 4), gm + k * KROWS16, id_wt, (i > tb) || (k > 0));
                         } else {
                             const int nks = (valid + 15) / 16;
                             for (int k = 0; k < nks; ++k)
-                                mma_bf16(d_wt, ym + ((k * 2048) >> 4), gk + kmaj_off(k, C::M * 128), id_wt,
-                                         (i > tb) || (k > 0));
+                                mma_bf16(d_wt, ym + ((k * 2048) >> 4), gm + k * KROWS16, id_wt, (i > tb) || (k > 0));
                         }
                         mma_commit(smem_u32(&y_empty[s]));
                     }
@@ -248,8 +320,31 @@ __global__ void __launch_bounds__(192, 1)
                     mma_commit(smem_u32(&wt_full[ab]));
                     ++wit;
                 }
-                mma_commit(smem_u32(&gt_empty));
+                mma_commit(smem_u32(&g_empty));
                 mma_commit(smem_u32(&dg_full));
+                // ---- phase 2: dB_tile = (dQ_hi + dQ_lo) . Wd1^T (K = m);
+                //      dWd1 += B^T . (dQ_hi + dQ_lo) (K = tokens) ----
+                for (int i = tb; i < te && ok; ++i) {
+                    const int64_t t0 = start + 128 * (int64_t)i;
+                    const int valid = (int)((end - t0) < 128 ? (end - t0) : 128);
+                    ok = mbar_wait(smem_u32(&dq_full[i - tb]), g & 1);
+                    tc_fence_after();
+                    const uint64_t qk = qk0 + (i - tb) * TILE16;
+                    const uint64_t qm = qm0 + (i - tb) * TILE16;
+                    const uint64_t bm = bm0 + (i - tb) * TILE16;
+                    const uint32_t d_db = tmem + C::TM_DG + (i - tb) * C::MS;
+#pragma unroll
+                    for (int k = 0; k < C::M / 16; ++k) mma_bf16(d_db, qk + 2 * k, w1k + 2 * k, id_db, k > 0);
+#pragma unroll
+                    for (int k = 0; k < C::M / 16; ++k) mma_bf16(d_db, qk + LO16 + 2 * k, w1k + 2 * k, id_db, true);
+                    const int nks = (valid + 15) / 16;
+                    for (int k = 0; k < nks; ++k) {
+                        mma_bf16(tmem + C::TM_W1, bm + k * KROWS16, qm + k * KROWS16, id_w1, (i > tb) || (k > 0));
+                        mma_bf16(tmem + C::TM_W1, bm + k * KROWS16, qm + LO16 + k * KROWS16, id_w1, true);
+                    }
+                    mma_commit(smem_u32(&db_full[i - tb]));
+                }
+                mma_commit(smem_u32(&w1_full));
             }
             mma_commit(smem_u32(&done_bar));
             mbar_wait(smem_u32(&done_bar), 0);
@@ -259,42 +354,27 @@ __global__ void __launch_bounds__(192, 1)
         const int q = warp & 3;
         const int row = q * 32 + lane;  // token row (phases 0, 2) or d-column row (phase 1)
         const int et = threadIdx.x - 64;
-        const __nv_bfloat16 *wd1 = reinterpret_cast<const __nv_bfloat16 *>(smem + C::OFF_WD1);    // r x m
-        const __nv_bfloat16 *wd1t = reinterpret_cast<const __nv_bfloat16 *>(smem + C::OFF_WD1T);  // m x r
-        constexpr int NOUT = (C::R * C::M + 127) / 128;  // dWd1 outputs per thread
+        const uint32_t lane_base = (uint32_t)(q * 32) << 16;
         uint32_t cit = 0;
         bool ok = true;
         for (int g = 0; g < ngroups && ok; ++g) {
             const int tb = g * C::NT, te = min(ntiles, tb + C::NT);
             const int64_t slot = (int64_t)blockIdx.x * a.max_groups + g;
-            // ---- phase 0: G^T of every tile of the group ----
-            ok = mbar_wait(smem_u32(&gt_empty), (g & 1) ^ 1);
+            // ---- phase 0: G = phi(Q) of every tile of the group ----
+            ok = mbar_wait(smem_u32(&g_empty), (g & 1) ^ 1) && mbar_wait(smem_u32(&q_full), g & 1);
+            tc_fence_after();
             for (int i = tb; i < te; ++i) {
                 const int64_t t0 = start + 128 * (int64_t)i;
                 const bool active = t0 + row < end;
-                float bq[C::R];
-                if (active) {
-                    load_bf16_row<C::R>(a.B + (t0 + row) * C::R, bq);
-                } else {
+                float v[C::M];
+                tmem_ld_row<C::M>(tmem + lane_base + C::TM_Q + (i - tb) * C::MS, v);
 #pragma unroll
-                    for (int k = 0; k < C::R; ++k) bq[k] = 0.0f;
-                }
-                uint8_t *gt = smem + C::OFF_GT + (i - tb) * C::GT_TILE + (row >> 6) * (C::M * 128);
-                const uint32_t byte = (row & 63) * 2;
-#pragma unroll
-                for (int jb = 0; jb < C::M; jb += 16) {
-                    float acc[16];
-                    vecmat16<C::R, C::M>(bq, wd1, jb, acc);   // Q = B . Wd1
-#pragma unroll
-                    for (int e = 0; e < 16; ++e) {
-                        const float gv = active ? act_fast(a.act, acc[e]) : 0.0f;
-                        *reinterpret_cast<__nv_bfloat16 *>(gt + swz_offset(jb + e, byte, 128)) = __float2bfloat16_rn(gv);
-                    }
-                }
-                // publish this tile's G^T so its first dWd2 product can start
+                for (int j = 0; j < C::M; ++j) v[j] = active ? act_fast(a.act, v[j]) : 0.0f;
+                store_bf16_swz_row<C::M>(smem + C::OFF_G + (i - tb) * C::TILE, row, v);
+                // publish this tile's G so its first dWd2 product can start
                 fence_async_smem();
                 named_barrier(1, 128);
-                if (et == 0) mbar_arrive(smem_u32(&gt_full[i - tb]));
+                if (et == 0) mbar_arrive(smem_u32(&g_full[i - tb]));
             }
 
             // ---- phase 1: drain each chunk's dWd2^T partial ----
@@ -303,107 +383,79 @@ __global__ void __launch_bounds__(192, 1)
                 ok = mbar_wait(smem_u32(&wt_full[ab]), (cit >> 1) & 1);
                 tc_fence_after();
                 float v[C::M];
-#pragma unroll
-                for (int j = 0; j < C::M; j += 16) {
-                    float t16[16];
-                    tmem_ld16(tmem_wt + ((uint32_t)(q * 32) << 16) + ab * C::MS + j, t16);
-                    tmem_ld_wait();
-#pragma unroll
-                    for (int e = 0; e < 16; ++e) v[j + e] = t16[e];
-                }
+                tmem_ld_row<C::M>(tmem + lane_base + C::TM_WT + ab * C::MS, v);
                 tc_fence_before();
                 mbar_arrive(smem_u32(&wt_empty[ab]));   // the accumulator is free again
                 wgrad_chunk<C::M>(a.wg, v, c, row, g == 0);
             }
 
-            // ---- phase 2: dQ, dB, dWd1 partial ----
+            // ---- phase 2: dQ (hi + lo), then dB and the dWd1 partial ----
             ok = ok && mbar_wait(smem_u32(&dg_full), g & 1);
             tc_fence_after();
-            // scratch rows padded by one float so that a warp's row-wise stores hit distinct banks
-            float *sB = reinterpret_cast<float *>(smem + C::OFF_Y);   // [128][R + 1]
-            float *sQ = sB + 128 * (C::R + 1);                          // [128][M + 1]
-            float acc1[NOUT];
-#pragma unroll
-            for (int k = 0; k < NOUT; ++k) acc1[k] = 0.0f;
             for (int i = tb; i < te; ++i) {
                 const int64_t t0 = start + 128 * (int64_t)i;
-                const int valid = (int)((end - t0) < 128 ? (end - t0) : 128);
-                const bool active = row < valid;
-                const int64_t tok = t0 + row;
-                float dq[C::M];
+                const bool active = t0 + row < end;
+                float hi[C::M], lo[C::M];
+                tmem_ld_row<C::M>(tmem + lane_base + C::TM_DG + (i - tb) * C::MS, hi);
+                tmem_ld_row<C::M>(tmem + lane_base + C::TM_Q + (i - tb) * C::MS, lo);
 #pragma unroll
-                for (int j = 0; j < C::M; j += 16) {
-                    float t16[16];
-                    tmem_ld16(tmem_dg + ((uint32_t)(q * 32) << 16) + (i - tb) * C::MS + j, t16);
-                    tmem_ld_wait();
-#pragma unroll
-                    for (int e = 0; e < 16; ++e) dq[j + e] = t16[e];
+                for (int j = 0; j < C::M; ++j) {
+                    const float x = active ? hi[j] * dact_f(a.act, lo[j]) : 0.0f;
+                    hi[j] = __bfloat162float(__float2bfloat16_rn(x));
+                    lo[j] = x - hi[j];
                 }
-                float bq[C::R];
-                if (active) {
-                    load_bf16_row<C::R>(a.B + tok * C::R, bq);
-                } else {
-#pragma unroll
-                    for (int k = 0; k < C::R; ++k) bq[k] = 0.0f;
-                }
-                // dQ = dG * phi'(Q), Q recomputed from B
-#pragma unroll
-                for (int jb = 0; jb < C::M; jb += 16) {
-                    float acc[16];
-                    vecmat16<C::R, C::M>(bq, wd1, jb, acc);
-#pragma unroll
-                    for (int e = 0; e < 16; ++e) dq[jb + e] = active ? dq[jb + e] * dact_fast(a.act, acc[e]) : 0.0f;
-                }
+                store_bf16_swz_row<C::M>(smem + C::OFF_DQ + (i - tb) * C::TILE, row, hi);
+                store_bf16_swz_row<C::M>(smem + C::OFF_DQLO + (i - tb) * C::TILE, row, lo);
+                // dG of the tile is read (its columns receive dB next) and dQ is published
+                tc_fence_before();
+                fence_async_smem();
+                named_barrier(1, 128);
+                if (et == 0) mbar_arrive(smem_u32(&dq_full[i - tb]));
+            }
+            ok = ok && mbar_wait(smem_u32(&yr_full), g & 1);
+            for (int i = tb; i < te && ok; ++i) {
+                const int64_t t0 = start + 128 * (int64_t)i;
+                const bool active = t0 + row < end;
+                ok = mbar_wait(smem_u32(&db_full[i - tb]), g & 1);
+                tc_fence_after();
+                float o[C::R];
+                tmem_ld_row<C::R>(tmem + lane_base + C::TM_DG + (i - tb) * C::MS, o);
                 if (active) {
                     // dB = [merge] dY[:, :r] + dQ . Wd1^T
-                    uint4 *dbo = reinterpret_cast<uint4 *>(a.dB + tok * C::R);
+                    if (a.merge) {
+                        float y[C::R];
+                        load_bf16_swz_row<C::R>(smem + C::OFF_YR + (i - tb) * C::TILE, row, y);
 #pragma unroll
-                    for (int ib = 0; ib < C::R; ib += 16) {
-                        float o[16];
-                        vecmat16<C::M, C::R>(dq, wd1t, ib, o);
-                        if (a.merge) {
-                            float y[16];
-                            load_bf16_row<16>(a.dY + tok * a.d + ib, y);
+                        for (int e = 0; e < C::R; ++e) o[e] = y[e] + o[e];
+                    }
+                    uint4 *dbo = reinterpret_cast<uint4 *>(a.dB + (t0 + row) * C::R);
 #pragma unroll
-                            for (int e = 0; e < 16; ++e) o[e] = y[e] + o[e];
-                        }
-                        uint32_t pk[8];
+                    for (int v8 = 0; v8 < C::R / 8; ++v8) {
+                        uint32_t pk[4];
 #pragma unroll
-                        for (int e = 0; e < 8; ++e) {
-                            __nv_bfloat162 hh = __floats2bfloat162_rn(o[2 * e], o[2 * e + 1]);
+                        for (int e = 0; e < 4; ++e) {
+                            __nv_bfloat162 hh = __floats2bfloat162_rn(o[8 * v8 + 2 * e], o[8 * v8 + 2 * e + 1]);
                             pk[e] = *reinterpret_cast<uint32_t *>(&hh);
                         }
-                        dbo[ib / 8] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-                        dbo[ib / 8 + 1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+                        dbo[v8] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
                     }
                 }
-                // dWd1 partial: sum over the tile's tokens of B[t][k] dQ[t][j], in token order
-                named_barrier(1, 128);   // the previous tile's scratch reads are done
+            }
+            // the group's dWd1 (rows = r, lanes 0 .. r-1) to its partial slot
+            ok = ok && mbar_wait(smem_u32(&w1_full), g & 1);
+            tc_fence_after();
+            if (q * 32 < C::R) {
+                float w[C::M];
+                tmem_ld_row<C::M>(tmem + lane_base + C::TM_W1, w);
+                if (row < C::R) {
+                    float4 *dst = reinterpret_cast<float4 *>(a.part1 + (slot * C::R + row) * C::M);
 #pragma unroll
-                for (int k = 0; k < C::R; ++k) sB[row * (C::R + 1) + k] = bq[k];
-#pragma unroll
-                for (int j = 0; j < C::M; ++j) sQ[row * (C::M + 1) + j] = dq[j];
-                named_barrier(1, 128);
-                // output o = et + 128 kk is (ki, j) = (o / M, o % M); 128 is a multiple of M, so j
-                // is the same for all of this thread's outputs. Each output sums over t in order;
-                // the outputs' chains interleave so their latencies overlap.
-                {
-                    static_assert((C::R * C::M) % 128 == 0 && 128 % C::M == 0, "dWd1 output split");
-                    const int j = et % C::M, ki0 = et / C::M;
-#pragma unroll 2
-                    for (int t = 0; t < valid; ++t) {
-                        const float qv = sQ[t * (C::M + 1) + j];
-                        const float *bt = sB + t * (C::R + 1) + ki0;
-#pragma unroll
-                        for (int kk = 0; kk < NOUT; ++kk) acc1[kk] = fmaf(bt[kk * (128 / C::M)], qv, acc1[kk]);
-                    }
+                    for (int e = 0; e < C::M / 4; ++e) dst[e] = make_float4(w[4 * e], w[4 * e + 1], w[4 * e + 2], w[4 * e + 3]);
                 }
             }
             tc_fence_before();
             mbar_arrive(smem_u32(&dg_empty));
-#pragma unroll
-            for (int kk = 0; kk < NOUT; ++kk) a.part1[slot * (C::R * C::M) + et + 128 * kk] = acc1[kk];
-            named_barrier(1, 128);   // scratch reads done before the ring is reused
+            named_barrier(1, 128);   // phase-2 scratch reads done before the ring is reused
             if (et == 0) mbar_arrive(smem_u32(&p2_done));
         }
         // slots of groups this CTA does not have: zeros

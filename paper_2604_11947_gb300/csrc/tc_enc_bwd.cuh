@@ -1,22 +1,28 @@
 // tc_enc_bwd.cuh -- backward of the send side on tensor cores (chain rule of Sec. 3.2's encoder
 // with the truncating identity path of Eq. Pid):
-//   dP = (dB . We2^T) * phi'(P);  dF = dP . We1^T;  dX[:, :r] += dB;
+//   dA = dB . We2^T;  dP = dA * phi'(P);  dF = dP . We1^T;  dX[:, :r] += dB;
 //   dWe1 = F^T . dP;  dWe2 = phi(P)^T . dB.
 //
-// Persistent CTAs over contiguous 16-token-aligned token ranges, in groups of up to NT tiles.
-//   phase 0 (epilogue warps): dP per token on CUDA cores (P from the forward pass), stored as
-//            bf16 twice: rows = tokens (K-major over m; A operand of the dF product) and rows = m
-//            (K-major over tokens; B operand of the dWe1 product). dX[:, :r] += dB.
-//   phase 1 (producer + MMA): d in chunks of 128 columns; per chunk one We1 slice (128 x m,
-//            K-major) and per tile one F tile (128 tokens x 128 columns) feeding
+// Persistent CTAs over contiguous 16-token-aligned token ranges, in groups of up to NT tiles of
+// 128 tokens. Every product runs on tcgen05; the CUDA cores apply phi and phi', convert, and
+// do the identity-path update. For each group:
+//   phase 0: the group's dB tiles (TMA) -> dA_tile = dB . We2^T in TMEM -> the epilogue reads P
+//            (fp32, from the forward pass) and writes dP = dA * phi'(P) and A = phi(P) as bf16
+//            rows [token][m] to shared memory (for m <= 32 dP also as hi + lo, hi = dP rounded
+//            to bf16 and lo = the rounded remainder, so dF sees dP to about 16 significant
+//            bits), and applies dX[:, :r] += dB -> dWe2 += A^T . dB over the group's tokens (the
+//            A tile read MN-major as a 128-row operand whose rows >= m are never read back).
+//            dB and A tiles live in F-ring slots 1 and 2, which the producer fills with F only
+//            after phase 0.
+//   phase 1: d in chunks of 128 columns; per chunk one We1 slice (128 x m, K-major) and per tile
+//            one F tile (128 tokens x 128 columns) feeding
 //              dF_tile_chunk (128 x 128 fp32, TMEM, double-buffered) = dP . We1_chunk^T
 //              dWe1_chunk    (128 columns x m, TMEM, double-buffered) += F^T . dP
-//            (F read as an MN-major operand). The epilogue converts dF to bf16 and stores it by
-//            TMA, and drains each finished dWe1 chunk to the group's fp32 partial slot.
-//   phase 3 (epilogue warps): the dWe2 partial (phi(P)^T . dB over the group's tokens, fixed
-//            order) with the then idle F ring as scratch.
-// HBM traffic per token: read F (2d), P (4m), dB (2r), dX[:, :r] (2r); write dF (2d), dX[:, :r]
-// (2r); P and dB are read again in phase 3 (L2). Per slot: d x m + m x r fp32 partials.
+//            (F read MN-major, dP read K-major and MN-major). The epilogue converts dF to bf16
+//            and stores it by TMA, and drains each finished dWe1 chunk to the CTA's fp32
+//            partial slot; the group's dWe2 goes to its own partial slot.
+// HBM traffic per token: read F (2d), P (4m), dB (2r), dX[:, :r] (2r); write dF (2d),
+// dX[:, :r] (2r). Per slot: d x m + m x r fp32 partials.
 #pragma once
 
 #include "common.cuh"
@@ -29,32 +35,38 @@ namespace tc {
 template <int M_> struct EncBwdCfg {
     static constexpr int M = M_;
     static constexpr int R = M_;
-    static constexpr int MS = M_ < 32 ? 32 : M_;                 // TMEM columns per dWe1 accumulator
+    static constexpr int MS = M_ < 32 ? 32 : M_;                 // TMEM columns per m-wide accumulator
     static constexpr int NT = M_ <= 32 ? 4 : 2;                  // tiles per group
-    static constexpr int NSF = M_ <= 32 ? 3 : 2;                 // F ring depth
-    static constexpr uint32_t DSW = M_ * 2 >= 128 ? 128 : M_ * 2;  // row bytes (= swizzle) of dP_A, We1
+    static constexpr int NSF = 3;                                // F ring depth
+    static constexpr int NW = M_ <= 16 ? 4 : 3;                  // We1 slice ring depth
+    static constexpr int NDA = M_ <= 32 ? NT : 1;                // dA TMEM regions (a ring)
+    static constexpr bool DPLO = M_ <= 32;                       // dP kept as bf16 hi + lo for dF
+    static constexpr uint32_t RB = M_ * 2;                       // row bytes (= swizzle) of r / m wide tiles
     static constexpr uint32_t F_STAGE = 128 * 128 * 2;
     static constexpr uint32_t STG_HALF = 128 * 64 * 2;           // dF staging: 128 rows x 64 columns
-    static constexpr uint32_t W_STAGE = 128 * DSW;               // We1 slice: 128 rows x m
-    static constexpr uint32_t DPA_TILE = 128 * DSW;              // dP, rows = tokens
-    static constexpr uint32_t DPT_TILE = M_ * 256;               // dP^T, rows = m, 128 tokens
-    static constexpr uint32_t WE2T_BYTES = R * M_ * 2;
+    static constexpr uint32_t W_STAGE = 128 * RB;                // We1 slice: 128 rows x m
+    static constexpr uint32_t TILE = 128 * RB;                   // 128 tokens x r (or m) columns
+    static constexpr uint32_t WE2_BYTES = M_ * R * 2;
     static constexpr uint32_t OFF_F = 0;
     static constexpr uint32_t OFF_STG = OFF_F + NSF * F_STAGE;
     static constexpr uint32_t OFF_W = OFF_STG + 2 * STG_HALF;
-    static constexpr int NW = M_ <= 16 ? 4 : 3;                  // We1 slice ring depth
-    static constexpr uint32_t OFF_DPA = OFF_W + NW * W_STAGE;
-    static constexpr uint32_t OFF_DPT = OFF_DPA + NT * DPA_TILE;
-    static constexpr uint32_t OFF_WE2T = OFF_DPT + NT * DPT_TILE;
-    static constexpr uint32_t SMEM_BYTES = OFF_WE2T + WE2T_BYTES + 1024;
-    static constexpr uint32_t SCRATCH_BYTES = 128 * (M_ + 1 + R + 1) * 4;  // phase 3: F ring + staging
-    static_assert(SCRATCH_BYTES <= OFF_W, "phase-3 scratch must fit in the F ring and staging");
-    static constexpr uint32_t TMEM_COLS = 512;                   // dF 2 x 128, dWe1 2 x MS
+    static constexpr uint32_t OFF_DP = OFF_W + NW * W_STAGE;     // dP (hi) tiles [token][m]
+    static constexpr uint32_t OFF_DPLO = OFF_DP + NT * TILE;     // dP lo tiles (if DPLO)
+    static constexpr uint32_t OFF_WE2 = OFF_DPLO + (DPLO ? NT * TILE : 0);  // We2 [m][r], K-major
+    static constexpr uint32_t SMEM_BYTES = OFF_WE2 + WE2_BYTES + 1024;
+    // phase-0 scratch in F-ring slots 1 and 2
+    static constexpr uint32_t OFF_DB = OFF_F + (NSF - 2) * F_STAGE;   // dB tiles [token][r] (TMA)
+    static constexpr uint32_t OFF_A = OFF_F + (NSF - 1) * F_STAGE;    // A = phi(P) tiles [token][m]
+    static_assert(NT * TILE <= F_STAGE && NSF >= 3, "phase-0 scratch must fit in two ring slots");
+    static_assert(SMEM_BYTES <= 232448 - 512, "shared memory budget");
+    // TMEM columns: dF 2 x 128 | dWe1 2 x MS | dA NDA x MS | dWe2 MS
+    static constexpr uint32_t TM_DF = 0, TM_WE = 256, TM_DA = 256 + 2 * MS, TM_W2 = TM_DA + NDA * MS;
+    static_assert(TM_W2 + MS <= 512, "TMEM budget");
+    static constexpr uint32_t TMEM_COLS = 512;
     static constexpr int THREADS = 192;
 };
 
 struct EncBwdArgs {
-    const __nv_bfloat16 *dB;   // T x r
     const float *P;            // T x m
     const __nv_bfloat16 *We2;  // m x r
     __nv_bfloat16 *dX;         // T x d or null
@@ -68,13 +80,15 @@ template <int M_>
 __global__ void __launch_bounds__(192, 1)
     k_enc_bwd(const __grid_constant__ CUtensorMap tm_f128, const __grid_constant__ CUtensorMap tm_f16,
               const __grid_constant__ CUtensorMap tm_we1, const __grid_constant__ CUtensorMap tm_df128,
-              const __grid_constant__ CUtensorMap tm_df16, const EncBwdArgs a)
+              const __grid_constant__ CUtensorMap tm_df16, const __grid_constant__ CUtensorMap tm_db,
+              const EncBwdArgs a)
 {
     using C = EncBwdCfg<M_>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     __shared__ uint64_t f_full[C::NSF], f_empty[C::NSF], w_full[C::NW], w_empty[C::NW];
-    __shared__ uint64_t dp_full[C::NT], dp_empty, df_full[2], df_empty[2], we_full[2], we_empty[2], p3_done, done_bar;
+    __shared__ uint64_t df_full[2], df_empty[2], we_full[2], we_empty[2];
+    __shared__ uint64_t db_full, da_full[C::NDA], da_empty[C::NDA], dp_full[C::NT], p0_done, w2_full, st_done, done_bar;
     __shared__ uint32_t tmem_base_sh;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -99,23 +113,28 @@ __global__ void __launch_bounds__(192, 1)
             mbar_init(smem_u32(&we_full[i]), 1);
             mbar_init(smem_u32(&we_empty[i]), 128);
         }
+        for (int i = 0; i < C::NDA; ++i) {
+            mbar_init(smem_u32(&da_full[i]), 1);
+            mbar_init(smem_u32(&da_empty[i]), 128);
+        }
         for (int i = 0; i < C::NT; ++i) mbar_init(smem_u32(&dp_full[i]), 1);
-        mbar_init(smem_u32(&dp_empty), 1);
-        mbar_init(smem_u32(&p3_done), 1);
+        mbar_init(smem_u32(&db_full), 1);
+        mbar_init(smem_u32(&p0_done), 2);   // the dWe2 MMAs' commit + the epilogue's dB reads
+        mbar_init(smem_u32(&w2_full), 1);
+        mbar_init(smem_u32(&st_done), 1);
         mbar_init(smem_u32(&done_bar), 1);
         fence_mbar_init();
     }
     if (warp == 1) tmem_alloc(smem_u32(&tmem_base_sh), C::TMEM_COLS);
-    if (warp >= 2) {  // We2^T (r x m bf16) into shared memory
-        __nv_bfloat16 *dt = reinterpret_cast<__nv_bfloat16 *>(smem + C::OFF_WE2T);
-        for (int e = threadIdx.x - 64; e < C::M * C::R; e += 128) dt[(e % C::R) * C::M + e / C::R] = a.We2[e];
+    if (warp >= 2) {  // We2 (m x r) as a swizzled K-major operand
+        for (int e = threadIdx.x - 64; e < C::M * C::R; e += 128)
+            *reinterpret_cast<__nv_bfloat16 *>(smem + C::OFF_WE2 + swz_offset(e / C::R, 2 * (e % C::R), C::RB)) = a.We2[e];
+        fence_async_smem();
     }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = tmem_base_sh;
-    const uint32_t tmem_df = tmem;            // 2 x 128 columns
-    const uint32_t tmem_we = tmem + 256;      // 2 x MS columns
 
     if (warp == 0) {
         // ---------------- producer ----------------
@@ -123,11 +142,24 @@ __global__ void __launch_bounds__(192, 1)
             tma_prefetch_desc(&tm_f128);
             tma_prefetch_desc(&tm_f16);
             tma_prefetch_desc(&tm_we1);
-            uint32_t fit = 0, wit = 0;
+            tma_prefetch_desc(&tm_db);
+            // F stages use slots 0, 1, ... from the start of every group (so that slots 1 and 2
+            // can hold the phase-0 scratch); bit s of fpar is the fill count of slot s, mod 2
+            uint32_t fpar = 0, filled = 0, wit = 0;
+            int db_issued = 0;
             bool ok = true;
             for (int g = 0; g < ngroups && ok; ++g) {
-                if (g > 0) ok = mbar_wait(smem_u32(&p3_done), (g - 1) & 1);  // the ring was scratch
+                // the previous group's MMAs are done with the whole ring
+                if (g > 0) ok = mbar_wait(smem_u32(&st_done), (g - 1) & 1);
+                if (!ok) break;
                 const int tb = g * C::NT, te = min(ntiles, tb + C::NT);
+                mbar_expect_tx(smem_u32(&db_full), (uint32_t)(te - tb) * C::TILE);
+                for (int i = tb; i < te; ++i)
+                    tma_load_2d(smem_u32(smem + C::OFF_DB + (i - tb) * C::TILE), &tm_db, 0,
+                                (int32_t)(start + 128 * (int64_t)i), smem_u32(&db_full));
+                ++db_issued;
+                bool p0_seen = false;
+                uint32_t j = 0;   // F stage of this group
                 for (int c = 0; c < nch && ok; ++c) {
                     // order: F tile 0 of the chunk, the chunk's We1 slice, the other F tiles.
                     // The MMA needs the slice before any tile of the chunk, so it must not queue
@@ -145,8 +177,14 @@ __global__ void __launch_bounds__(192, 1)
                         const int64_t t0 = start + 128 * (int64_t)i;
                         const int valid = (int)((end - t0) < 128 ? (end - t0) : 128);
                         const int nb = (valid + 15) / 16;
-                        const uint32_t s = fit % C::NSF;
-                        if (!mbar_wait(smem_u32(&f_empty[s]), ((fit / C::NSF) & 1) ^ 1)) { ok = false; break; }
+                        const uint32_t s = j % C::NSF;
+                        if (s >= (uint32_t)(C::NSF - 2) && !p0_seen) {   // phase-0 scratch released
+                            if (!mbar_wait(smem_u32(&p0_done), g & 1)) { ok = false; break; }
+                            p0_seen = true;
+                        }
+                        if (!mbar_wait(smem_u32(&f_empty[s]), ((fpar >> s) & 1) ^ 1)) { ok = false; break; }
+                        fpar ^= 1u << s;
+                        filled |= 1u << s;
                         const uint32_t dst = smem_u32(smem + C::OFF_F + s * C::F_STAGE);
                         const uint32_t bar = smem_u32(&f_full[s]);
                         mbar_expect_tx(bar, valid == 128 ? C::F_STAGE : (uint32_t)nb * 2u * 2048u);
@@ -159,7 +197,7 @@ __global__ void __launch_bounds__(192, 1)
                                                 (int32_t)(t0 + 16 * rg), bar);
                             }
                         }
-                        ++fit;
+                        ++j;
                     }
                     if (!ok) break;
                     if (te - tb == 1) {  // a one-tile group: the slice after its only tile
@@ -172,74 +210,116 @@ __global__ void __launch_bounds__(192, 1)
                     }
                 }
             }
-            for (uint32_t k = 0; k < (fit < (uint32_t)C::NSF ? fit : (uint32_t)C::NSF); ++k) {
-                const uint32_t j = fit - 1 - k;
-                mbar_wait(smem_u32(&f_full[j % C::NSF]), (j / C::NSF) & 1);
-            }
+            // drain the loads still in flight
+            for (int s = 0; s < C::NSF; ++s)
+                if ((filled >> s) & 1) mbar_wait(smem_u32(&f_full[s]), ((fpar >> s) & 1) ^ 1);
             for (uint32_t k = 0; k < (wit < (uint32_t)C::NW ? wit : (uint32_t)C::NW); ++k) {
-                const uint32_t j = wit - 1 - k;
-                mbar_wait(smem_u32(&w_full[j % C::NW]), (j / C::NW) & 1);
+                const uint32_t jj = wit - 1 - k;
+                mbar_wait(smem_u32(&w_full[jj % C::NW]), (jj / C::NW) & 1);
             }
+            if (db_issued > 0) mbar_wait(smem_u32(&db_full), (db_issued - 1) & 1);
         }
     } else if (warp == 1) {
         // ---------------- MMA issuer ----------------
         if (elect_one()) {
-            constexpr Swz dswz = C::DSW == 128 ? kSwz128 : C::DSW == 64 ? kSwz64 : kSwz32;
-            constexpr uint32_t id_df = idesc_bf16(128, 128, false, false);   // dP (K-major) . We1 (K-major)
-            constexpr uint32_t id_we = idesc_bf16(128, C::M, true, false);   // F^T (MN-major) . dP^T (K-major)
-            // shared-memory descriptors of slot / tile 0, advanced by adding byte offset >> 4 to
-            // the start-address field (no carry: shared addresses < 256 KB)
+            constexpr Swz rsw = swz_for(C::RB);
+            constexpr uint32_t id_da = idesc_bf16(128, C::M, false, false);   // dB (K-major) . We2 rows (K-major)
+            constexpr uint32_t id_w2 = idesc_bf16(128, C::R, true, true);     // A^T (MN-major) . dB (MN-major)
+            constexpr uint32_t id_df = idesc_bf16(128, 128, false, false);    // dP (K-major) . We1 (K-major)
+            constexpr uint32_t id_we = idesc_bf16(128, C::M, true, true);     // F^T (MN-major) . dP (MN-major)
+            // shared-memory descriptors of slot / tile 0, advanced by adding the byte offset >> 4
+            // to the start-address field (no carry: shared addresses < 256 KB). The 128-row A^T
+            // operand has one real block of m rows: its block stride (LBO) is 0, so every block
+            // reads the same m rows and the extra output rows are duplicates.
             const uint64_t fm0 = smem_desc(smem_u32(smem + C::OFF_F), 16384, 1024, kSwz128);   // F, MN-major
-            const uint64_t wd0 = smem_desc(smem_u32(smem + C::OFF_W), 16, 8 * C::DSW, dswz);   // We1 slice
-            const uint64_t pa0 = smem_desc(smem_u32(smem + C::OFF_DPA), 16, 8 * C::DSW, dswz); // dP
-            const uint64_t pt0 = smem_desc(smem_u32(smem + C::OFF_DPT), 16, 1024, kSwz128);    // dP^T
-            uint32_t fit = 0, wit = 0, cit = 0, dfit = 0;
+            const uint64_t wd0 = smem_desc(smem_u32(smem + C::OFF_W), 16, 8 * C::RB, rsw);     // We1 slice
+            const uint64_t pk0 = smem_desc(smem_u32(smem + C::OFF_DP), 16, 8 * C::RB, rsw);    // dP, K-major
+            const uint64_t pm0 = smem_desc(smem_u32(smem + C::OFF_DP), 0, 8 * C::RB, rsw);     // dP, MN-major
+            const uint64_t dbk0 = smem_desc(smem_u32(smem + C::OFF_DB), 16, 8 * C::RB, rsw);   // dB, K-major
+            const uint64_t dbm0 = smem_desc(smem_u32(smem + C::OFF_DB), 0, 8 * C::RB, rsw);    // dB, MN-major
+            const uint64_t am0 = smem_desc(smem_u32(smem + C::OFF_A), 0, 8 * C::RB, rsw);      // A^T, MN-major
+            const uint64_t we2k = smem_desc(smem_u32(smem + C::OFF_WE2), 16, 8 * C::RB, rsw);  // We2 rows
+            constexpr uint64_t TILE16 = C::TILE >> 4;
+            constexpr uint64_t KROWS16 = (16 * C::RB) >> 4;              // 16 token rows of an r / m wide tile
+            constexpr uint64_t LO16 = (C::OFF_DPLO - C::OFF_DP) >> 4;    // dP hi tile -> lo tile
+            uint32_t fpar = 0, wit = 0, cit = 0, dfit = 0, u = 0;
             bool ok = true;
             for (int g = 0; g < ngroups && ok; ++g) {
                 const int tb = g * C::NT, te = min(ntiles, tb + C::NT);
+                ok = mbar_wait(smem_u32(&db_full), g & 1);
+                tc_fence_after();
+                // ---- phase 0: dA_tile = dB_tile . We2^T (K = r), a ring of NDA TMEM regions ----
+                for (int i = tb; i < te && ok; ++i, ++u) {
+                    const uint32_t rg = u % C::NDA;
+                    if (u >= (uint32_t)C::NDA) {
+                        ok = mbar_wait(smem_u32(&da_empty[rg]), ((u / C::NDA) - 1) & 1);
+                        tc_fence_after();
+                    }
+                    const uint64_t dbk = dbk0 + (i - tb) * TILE16;
+#pragma unroll
+                    for (int k = 0; k < C::R / 16; ++k)
+                        mma_bf16(tmem + C::TM_DA + rg * C::MS, dbk + 2 * k, we2k + 2 * k, id_da, k > 0);
+                    mma_commit(smem_u32(&da_full[rg]));
+                }
+                // dWe2 += A_tile^T . dB_tile (K = the tile's tokens), once the tile's A is written
+                for (int i = tb; i < te && ok; ++i) {
+                    const int64_t t0 = start + 128 * (int64_t)i;
+                    const int valid = (int)((end - t0) < 128 ? (end - t0) : 128);
+                    ok = mbar_wait(smem_u32(&dp_full[i - tb]), g & 1);
+                    tc_fence_after();
+                    const uint64_t am = am0 + (i - tb) * TILE16;
+                    const uint64_t dbm = dbm0 + (i - tb) * TILE16;
+                    const int nks = (valid + 15) / 16;
+                    for (int k = 0; k < nks; ++k)
+                        mma_bf16(tmem + C::TM_W2, am + k * KROWS16, dbm + k * KROWS16, id_w2, (i > tb) || (k > 0));
+                }
+                mma_commit(smem_u32(&p0_done));   // dB and A tiles are no longer read
+                mma_commit(smem_u32(&w2_full));
+                // ---- phase 1: the F stream ----
+                uint32_t j = 0;
                 for (int c = 0; c < nch && ok; ++c, ++cit, ++wit) {
                     const uint32_t sw = wit % C::NW, ae = cit & 1;
                     ok = mbar_wait(smem_u32(&w_full[sw]), (wit / C::NW) & 1) &&
                          mbar_wait(smem_u32(&we_empty[ae]), ((cit >> 1) & 1) ^ 1);
                     tc_fence_after();
                     const uint64_t wd = wd0 + ((sw * C::W_STAGE) >> 4);
-                    const uint32_t d_we = tmem_we + ae * C::MS;
-                    for (int i = tb; i < te && ok; ++i, ++fit, ++dfit) {
+                    const uint32_t d_we = tmem + C::TM_WE + ae * C::MS;
+                    for (int i = tb; i < te && ok; ++i, ++dfit, ++j) {
                         const int64_t t0 = start + 128 * (int64_t)i;
                         const int valid = (int)((end - t0) < 128 ? (end - t0) : 128);
-                        const uint32_t s = fit % C::NSF, ad_buf = dfit & 1;
-                        // dP of the tile (phase 0, published per tile once per group), its F
-                        // tile, a free dF buffer
-                        if (c == 0) ok = mbar_wait(smem_u32(&dp_full[i - tb]), g & 1);
-                        ok = ok && mbar_wait(smem_u32(&f_full[s]), (fit / C::NSF) & 1) &&
+                        const uint32_t s = j % C::NSF, ad_buf = dfit & 1;
+                        ok = mbar_wait(smem_u32(&f_full[s]), (fpar >> s) & 1) &&
                              mbar_wait(smem_u32(&df_empty[ad_buf]), ((dfit >> 1) & 1) ^ 1);
+                        fpar ^= 1u << s;
                         tc_fence_after();
                         const uint64_t fm = fm0 + ((s * C::F_STAGE) >> 4);
-                        const uint64_t pa = pa0 + (((i - tb) * C::DPA_TILE) >> 4);
-                        const uint64_t pt = pt0 + (((i - tb) * C::DPT_TILE) >> 4);
-                        const uint32_t d_df = tmem_df + ad_buf * 128;
+                        const uint64_t pk = pk0 + (i - tb) * TILE16;
+                        const uint64_t pm = pm0 + (i - tb) * TILE16;
+                        const uint32_t d_df = tmem + C::TM_DF + ad_buf * 128;
                         // dF = dP . We1_chunk^T (K = m in steps of 16 = 32 bytes of a swizzled row)
 #pragma unroll
-                        for (int k = 0; k < C::M / 16; ++k) mma_bf16(d_df, pa + 2 * k, wd + 2 * k, id_df, k > 0);
+                        for (int k = 0; k < C::M / 16; ++k) mma_bf16(d_df, pk + 2 * k, wd + 2 * k, id_df, k > 0);
+                        if (C::DPLO) {
+#pragma unroll
+                            for (int k = 0; k < C::M / 16; ++k) mma_bf16(d_df, pk + LO16 + 2 * k, wd + 2 * k, id_df, true);
+                        }
                         mma_commit(smem_u32(&df_full[ad_buf]));
                         // dWe1^T_chunk += F^T . dP  (K = the tile's tokens in steps of 16)
                         if (valid == 128) {
 #pragma unroll
                             for (int k = 0; k < 8; ++k)
-                                mma_bf16(d_we, fm + ((k * 2048) >> 4), pt + kmaj_off(k, C::M * 128), id_we,
-                                         (i > tb) || (k > 0));
+                                mma_bf16(d_we, fm + ((k * 2048) >> 4), pm + k * KROWS16, id_we, (i > tb) || (k > 0));
                         } else {
                             const int nks = (valid + 15) / 16;
                             for (int k = 0; k < nks; ++k)
-                                mma_bf16(d_we, fm + ((k * 2048) >> 4), pt + kmaj_off(k, C::M * 128), id_we,
-                                         (i > tb) || (k > 0));
+                                mma_bf16(d_we, fm + ((k * 2048) >> 4), pm + k * KROWS16, id_we, (i > tb) || (k > 0));
                         }
                         mma_commit(smem_u32(&f_empty[s]));
                     }
                     mma_commit(smem_u32(&w_empty[sw]));
                     mma_commit(smem_u32(&we_full[ae]));
                 }
-                mma_commit(smem_u32(&dp_empty));
+                mma_commit(smem_u32(&st_done));
             }
             mma_commit(smem_u32(&done_bar));
             mbar_wait(smem_u32(&done_bar), 0);
@@ -249,80 +329,78 @@ __global__ void __launch_bounds__(192, 1)
         const int q = warp & 3;
         const int row = q * 32 + lane;
         const int et = threadIdx.x - 64;
-        const __nv_bfloat16 *we2t = reinterpret_cast<const __nv_bfloat16 *>(smem + C::OFF_WE2T);  // r x m
-        constexpr int NOUT = (C::M * C::R + 127) / 128;
-        uint32_t cit = 0, dfit = 0, sit = 0;
+        const uint32_t lane_base = (uint32_t)(q * 32) << 16;
+        uint32_t cit = 0, dfit = 0, sit = 0, u = 0;
         bool ok = true;
         for (int g = 0; g < ngroups && ok; ++g) {
             const int tb = g * C::NT, te = min(ntiles, tb + C::NT);
             const int64_t slot = (int64_t)blockIdx.x * a.max_groups + g;
-            // ---- phase 0: dP (two layouts), dX ----
-            ok = mbar_wait(smem_u32(&dp_empty), (g & 1) ^ 1);
-            for (int i = tb; i < te; ++i) {
+            // ---- phase 0: dP and A = phi(P) of every tile, dX[:, :r] += dB ----
+            ok = mbar_wait(smem_u32(&db_full), g & 1);
+            for (int i = tb; i < te; ++i, ++u) {
                 const int64_t t0 = start + 128 * (int64_t)i;
                 const bool active = t0 + row < end;
                 const int64_t tok = t0 + row;
-                float db[C::R];
-                float dp[C::M];
+                // this token's P row and dX[:, :r] row, fetched before waiting for dA
+                float pv[C::M];
+                float xv[C::R];
+#pragma unroll
+                for (int jj = 0; jj < C::M; ++jj) pv[jj] = 0.0f;
+#pragma unroll
+                for (int jj = 0; jj < C::R; ++jj) xv[jj] = 0.0f;
                 if (active) {
-                    load_bf16_row<C::R>(a.dB + tok * C::R, db);
                     const float4 *ps = reinterpret_cast<const float4 *>(a.P + tok * C::M);
 #pragma unroll
-                    for (int j = 0; j < C::M / 4; ++j) {
-                        const float4 v = ps[j];
-                        dp[4 * j] = v.x; dp[4 * j + 1] = v.y; dp[4 * j + 2] = v.z; dp[4 * j + 3] = v.w;
+                    for (int jj = 0; jj < C::M / 4; ++jj) {
+                        const float4 v = ps[jj];
+                        pv[4 * jj] = v.x; pv[4 * jj + 1] = v.y; pv[4 * jj + 2] = v.z; pv[4 * jj + 3] = v.w;
                     }
-                } else {
-#pragma unroll
-                    for (int k = 0; k < C::R; ++k) db[k] = 0.0f;
-#pragma unroll
-                    for (int j = 0; j < C::M; ++j) dp[j] = 0.0f;
+                    if (a.dX) load_bf16_row<C::R>(a.dX + tok * a.d, xv);
                 }
+                const uint32_t rg = u % C::NDA;
+                ok = ok && mbar_wait(smem_u32(&da_full[rg]), (u / C::NDA) & 1);
+                tc_fence_after();
+                float da[C::M];
+                tmem_ld_row<C::M>(tmem + lane_base + C::TM_DA + rg * C::MS, da);
+                tc_fence_before();
+                mbar_arrive(smem_u32(&da_empty[rg]));   // the dA region is free again
+                float av[C::M];
 #pragma unroll
-                for (int jb = 0; jb < C::M; jb += 16) {
-                    float acc[16];
-                    vecmat16<C::R, C::M>(db, we2t, jb, acc);   // dA = dB . We2^T
-#pragma unroll
-                    for (int e = 0; e < 16; ++e) dp[jb + e] = active ? acc[e] * dact_fast(a.act, dp[jb + e]) : 0.0f;
+                for (int jj = 0; jj < C::M; ++jj) {
+                    float ph = 0.0f, dph = 0.0f;
+                    act_and_dact(a.act, pv[jj], ph, dph);
+                    const float x = active ? da[jj] * dph : 0.0f;
+                    da[jj] = __bfloat162float(__float2bfloat16_rn(x));   // hi
+                    pv[jj] = x - da[jj];                                 // lo
+                    av[jj] = active ? ph : 0.0f;
                 }
-                // dP rows = tokens (K-major over m, DSW-byte rows)
-                uint8_t *pa = smem + C::OFF_DPA + (i - tb) * C::DPA_TILE;
-#pragma unroll
-                for (int cc = 0; cc < C::M / 8; ++cc) {
-                    uint32_t pk[4];
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        __nv_bfloat162 h = __floats2bfloat162_rn(dp[8 * cc + 2 * e], dp[8 * cc + 2 * e + 1]);
-                        pk[e] = *reinterpret_cast<uint32_t *>(&h);
-                    }
-                    *reinterpret_cast<uint4 *>(pa + swz_offset(row, 16 * cc, C::DSW)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-                }
-                // dP^T rows = m (K-major over the tile's tokens, 128B rows, two 64-token blocks)
-                uint8_t *pt = smem + C::OFF_DPT + (i - tb) * C::DPT_TILE + (row >> 6) * (C::M * 128);
-                const uint32_t byte = (row & 63) * 2;
-#pragma unroll
-                for (int j = 0; j < C::M; ++j)
-                    *reinterpret_cast<__nv_bfloat16 *>(pt + swz_offset(j, byte, 128)) = __float2bfloat16_rn(dp[j]);
-                // publish this tile's dP so its products can start
-                fence_async_smem();
-                named_barrier(1, 128);
-                if (et == 0) mbar_arrive(smem_u32(&dp_full[i - tb]));
+                store_bf16_swz_row<C::M>(smem + C::OFF_DP + (i - tb) * C::TILE, row, da);
+                if (C::DPLO) store_bf16_swz_row<C::M>(smem + C::OFF_DPLO + (i - tb) * C::TILE, row, pv);
+                store_bf16_swz_row<C::M>(smem + C::OFF_A + (i - tb) * C::TILE, row, av);
                 // identity path: dX[:, :r] += dB
                 if (active && a.dX) {
+                    float db[C::R];
+                    load_bf16_swz_row<C::R>(smem + C::OFF_DB + (i - tb) * C::TILE, row, db);
                     uint4 *xp = reinterpret_cast<uint4 *>(a.dX + tok * a.d);
 #pragma unroll
-                    for (int v = 0; v < C::R / 8; ++v) {
-                        float xv[8];
-                        load_bf16_row<8>(a.dX + tok * a.d + 8 * v, xv);
+                    for (int v8 = 0; v8 < C::R / 8; ++v8) {
                         uint32_t pk[4];
 #pragma unroll
                         for (int e = 0; e < 4; ++e) {
-                            __nv_bfloat162 h = __floats2bfloat162_rn(xv[2 * e] + db[8 * v + 2 * e],
-                                                                     xv[2 * e + 1] + db[8 * v + 2 * e + 1]);
+                            __nv_bfloat162 h = __floats2bfloat162_rn(xv[8 * v8 + 2 * e] + db[8 * v8 + 2 * e],
+                                                                     xv[8 * v8 + 2 * e + 1] + db[8 * v8 + 2 * e + 1]);
                             pk[e] = *reinterpret_cast<uint32_t *>(&h);
                         }
-                        xp[v] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+                        xp[v8] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
                     }
+                }
+                // publish this tile's dP and A; after the last tile every thread's dB reads are
+                // done (p0_done before the last dp_full, so the stream cannot overtake it)
+                fence_async_smem();
+                named_barrier(1, 128);
+                if (et == 0) {
+                    if (i == te - 1) mbar_arrive(smem_u32(&p0_done));
+                    mbar_arrive(smem_u32(&dp_full[i - tb]));
                 }
             }
 
@@ -346,7 +424,7 @@ __global__ void __launch_bounds__(192, 1)
                         for (int gq = 0; gq < 2; ++gq) {
                             if (gq >= gqend) break;
                             float v[32];
-                            tmem_ld32(tmem_df + ((uint32_t)(q * 32) << 16) + ad_buf * 128 + h * 64 + gq * 32, v);
+                            tmem_ld32(tmem + lane_base + C::TM_DF + ad_buf * 128 + h * 64 + gq * 32, v);
                             tmem_ld_wait();
                             uint32_t p[16];
 #pragma unroll
@@ -370,85 +448,37 @@ __global__ void __launch_bounds__(192, 1)
                             if (valid == 128) {
                                 tma_store_2d(&tm_df128, x, (int32_t)t0, smem_u32(stg));
                             } else {
-                                for (int rg = 0; rg * 16 < valid; ++rg)
-                                    tma_store_2d(&tm_df16, x, (int32_t)(t0 + 16 * rg), smem_u32(stg) + rg * 2048);
+                                for (int rgi = 0; rgi * 16 < valid; ++rgi)
+                                    tma_store_2d(&tm_df16, x, (int32_t)(t0 + 16 * rgi), smem_u32(stg) + rgi * 2048);
                             }
                             bulk_commit();
                         }
                     }
                 }
-                // the chunk's dWe1 rows (lane = d column) -> cross-CTA reduction
+                // the chunk's dWe1 rows (lane = d column) -> the CTA's partial slot
                 const uint32_t ae = cit & 1;
                 ok = ok && mbar_wait(smem_u32(&we_full[ae]), (cit >> 1) & 1);
                 tc_fence_after();
                 float v[C::M];
-#pragma unroll
-                for (int j = 0; j < C::M; j += 16) {
-                    float t16[16];
-                    tmem_ld16(tmem_we + ((uint32_t)(q * 32) << 16) + ae * C::MS + j, t16);
-                    tmem_ld_wait();
-#pragma unroll
-                    for (int e = 0; e < 16; ++e) v[j + e] = t16[e];
-                }
+                tmem_ld_row<C::M>(tmem + lane_base + C::TM_WE + ae * C::MS, v);
                 tc_fence_before();
                 mbar_arrive(smem_u32(&we_empty[ae]));   // the accumulator is free again
                 wgrad_chunk<C::M>(a.wg, v, c, row, g == 0);
             }
 
-            // ---- phase 3: dWe2 partial = sum over tokens of phi(P)^T dB ----
-            if (et == 0) bulk_wait_read<0>();   // staging no longer read by TMA stores
-            named_barrier(1, 128);
-            float *sA = reinterpret_cast<float *>(smem + C::OFF_F);   // [128][M + 1]
-            float *sD = sA + 128 * (C::M + 1);                          // [128][R + 1]
-            float acc2[NOUT];
+            // ---- the group's dWe2 (rows = m, lanes 0 .. m-1) to its partial slot ----
+            ok = ok && mbar_wait(smem_u32(&w2_full), g & 1);
+            tc_fence_after();
+            if (q * 32 < C::M) {
+                float w[C::R];
+                tmem_ld_row<C::R>(tmem + lane_base + C::TM_W2, w);
+                if (row < C::M) {
+                    float4 *dst = reinterpret_cast<float4 *>(a.part2 + (slot * C::M + row) * C::R);
 #pragma unroll
-            for (int k = 0; k < NOUT; ++k) acc2[k] = 0.0f;
-            for (int i = tb; i < te; ++i) {
-                const int64_t t0 = start + 128 * (int64_t)i;
-                const int valid = (int)((end - t0) < 128 ? (end - t0) : 128);
-                const bool active = row < valid;
-                const int64_t tok = t0 + row;
-                float av[C::M], db[C::R];
-                if (active) {
-                    const float4 *ps = reinterpret_cast<const float4 *>(a.P + tok * C::M);
-#pragma unroll
-                    for (int j = 0; j < C::M / 4; ++j) {
-                        const float4 v = ps[j];
-                        av[4 * j] = act_fast(a.act, v.x); av[4 * j + 1] = act_fast(a.act, v.y);
-                        av[4 * j + 2] = act_fast(a.act, v.z); av[4 * j + 3] = act_fast(a.act, v.w);
-                    }
-                    load_bf16_row<C::R>(a.dB + tok * C::R, db);
-                } else {
-#pragma unroll
-                    for (int j = 0; j < C::M; ++j) av[j] = 0.0f;
-#pragma unroll
-                    for (int k = 0; k < C::R; ++k) db[k] = 0.0f;
-                }
-                named_barrier(1, 128);
-#pragma unroll
-                for (int j = 0; j < C::M; ++j) sA[row * (C::M + 1) + j] = av[j];
-#pragma unroll
-                for (int k = 0; k < C::R; ++k) sD[row * (C::R + 1) + k] = db[k];
-                named_barrier(1, 128);
-                // output o = et + 128 kk is (j, k) = (o / R, o % R); 128 is a multiple of R, so k
-                // is the same for all of this thread's outputs. Each output sums over t in order;
-                // the outputs' chains interleave so their latencies overlap.
-                {
-                    static_assert((C::M * C::R) % 128 == 0 && 128 % C::R == 0, "dWe2 output split");
-                    const int k = et % C::R, j0 = et / C::R;
-#pragma unroll 2
-                    for (int t = 0; t < valid; ++t) {
-                        const float dv = sD[t * (C::R + 1) + k];
-                        const float *at = sA + t * (C::M + 1) + j0;
-#pragma unroll
-                        for (int kk = 0; kk < NOUT; ++kk) acc2[kk] = fmaf(at[kk * (128 / C::R)], dv, acc2[kk]);
-                    }
+                    for (int e = 0; e < C::R / 4; ++e) dst[e] = make_float4(w[4 * e], w[4 * e + 1], w[4 * e + 2], w[4 * e + 3]);
                 }
             }
-#pragma unroll
-            for (int kk = 0; kk < NOUT; ++kk) a.part2[slot * (C::M * C::R) + et + 128 * kk] = acc2[kk];
-            named_barrier(1, 128);
-            if (et == 0) mbar_arrive(smem_u32(&p3_done));
+            tc_fence_before();
         }
         for (int g = ngroups; g < a.max_groups; ++g) {
             const int64_t slot = (int64_t)blockIdx.x * a.max_groups + g;

@@ -3,8 +3,8 @@ import numpy as np
 import pytest
 import torch
 
-from gpu_helpers import (INPUTS, check_output, gpu_step, host_inputs, oracle_step, sample_tokens,
-                         to_dev, to_host)
+from gpu_helpers import (INPUTS, assert_step_is_its_stages, check_output, gpu_stages, gpu_step,
+                         host_inputs, oracle_step, sample_tokens, to_dev, to_host)
 from metrics import TOL, check
 from paper_2604_11947_gb300 import resbm, synth
 
@@ -32,8 +32,17 @@ SMALL = {
 }
 
 
-def _compare_all(cfg, got, want):
-    return {k: check_output(k, got[k], want[k], cfg) for k in OUTS}
+def _compare_all(cfg, got, want, dev, flags=0):
+    """The step's boundary tensors (B and dB, after the transfer rounding) against the oracle's;
+    every later output against the oracle with the stage that produces it run on the oracle's
+    transferred tensor (gpu_stages); and the step against its own stages, bit for bit."""
+    errs = {k: check_output(k, got[k], want[k], cfg) for k in ("B", "dB")}
+    stages = gpu_stages(cfg, dev, want, flags)
+    for k in OUTS:
+        if k not in ("B",):
+            errs["stage_" + k] = check_output(k, stages[k], want[k], cfg)
+    assert_step_is_its_stages(cfg, dev, got, flags)
+    return errs
 
 
 @pytest.mark.parametrize("path", PATHS)
@@ -44,7 +53,7 @@ def test_small_configs_match_oracle(name, path):
     dev = {k: to_dev(v, cfg) for k, v in h.items()}
     got = gpu_step(cfg, dev, flags=PATHS[path])
     want = oracle_step(cfg, h)
-    _compare_all(cfg, got, want)
+    _compare_all(cfg, got, want, dev, PATHS[path])
     # the saved pre-activation P = F . We1 is an fp32 output: fp32 accumulation error only
     check("P", to_host(got["P"]), want["P"], "f32", tol=1e-4)
 
@@ -56,8 +65,9 @@ def test_activation_and_merge_variants(act, merge, dtype):
     cfg = synth.BoundaryConfig("v", T=400, d=256, r=16, m=24, dtype=dtype, act=act, merge=merge)
     h = host_inputs(cfg)
     dev = {k: to_dev(v, cfg) for k, v in h.items()}
+    want = oracle_step(cfg, h)
     for flags in PATHS.values():
-        _compare_all(cfg, gpu_step(cfg, dev, flags=flags), oracle_step(cfg, h))
+        _compare_all(cfg, gpu_step(cfg, dev, flags=flags), want, dev, flags)
 
 
 def test_single_bf16_config_full():
@@ -67,7 +77,7 @@ def test_single_bf16_config_full():
     dev = {k: to_dev(v, cfg) for k, v in h.items()}
     got = gpu_step(cfg, dev)
     want = oracle_step(cfg, h)
-    _compare_all(cfg, got, want)
+    _compare_all(cfg, got, want, dev)
 
 
 def _sampled_full_size(cfg, n_tokens=96, flags=0):
