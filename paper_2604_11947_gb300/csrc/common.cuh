@@ -105,4 +105,41 @@ __device__ __forceinline__ void act_and_dact(int act, float x, float &a, float &
     }
 }
 
+// ---- the same functions over a row of N values -----------------------------------------------
+// The branch on the activation is taken once, outside the element loop, so that the N
+// independent evaluations interleave instead of running one after the other.
+#define RESBM_ACT_ROW_LOOP(ACT, BODY)                                                 \
+    do {                                                                              \
+        if ((ACT) == RESBM_ACT_SILU) {                                                \
+            constexpr int kAct = RESBM_ACT_SILU;                                      \
+            _Pragma("unroll") for (int j = 0; j < N; ++j) { BODY; }                   \
+        } else if ((ACT) == RESBM_ACT_GELU_TANH) {                                    \
+            constexpr int kAct = RESBM_ACT_GELU_TANH;                                 \
+            _Pragma("unroll") for (int j = 0; j < N; ++j) { BODY; }                   \
+        } else {                                                                      \
+            constexpr int kAct = RESBM_ACT_IDENTITY;                                  \
+            _Pragma("unroll") for (int j = 0; j < N; ++j) { BODY; }                   \
+        }                                                                             \
+    } while (0)
+
+// v = phi(v), precise or fast
+template <int N> __device__ __forceinline__ void act_row(int act, float (&v)[N])
+{
+    RESBM_ACT_ROW_LOOP(act, v[j] = act_f(kAct, v[j]));
+}
+template <int N> __device__ __forceinline__ void act_fast_row(int act, float (&v)[N])
+{
+    RESBM_ACT_ROW_LOOP(act, v[j] = act_fast(kAct, v[j]));
+}
+// d = phi'(x), fast (d may alias x)
+template <int N> __device__ __forceinline__ void dact_fast_row(int act, const float (&x)[N], float (&d)[N])
+{
+    RESBM_ACT_ROW_LOOP(act, d[j] = dact_fast(kAct, x[j]));
+}
+// a = phi(x), d = phi'(x), precise
+template <int N> __device__ __forceinline__ void act_dact_row(int act, const float (&x)[N], float (&a)[N], float (&d)[N])
+{
+    RESBM_ACT_ROW_LOOP(act, act_and_dact(kAct, x[j], a[j], d[j]));
+}
+
 }  // namespace resbm

@@ -147,15 +147,25 @@ BwdPlan bwd_plan(const resbm_desc &d, int sms, int nt, int64_t small_elems, void
     return p;
 }
 
-// Launch shape of k_reduce_slots: one block per 32 float4 columns (capped at 8 blocks per SM,
-// the blocks then stride over the rest).
+// The two weight-gradient reductions of a backward op in one launch: the small (r x m) job
+// first, on its own blocks, the large (d x m) one on the rest; one block per 32 float4 columns,
+// the whole grid resident at once (8 blocks of 256 threads per SM).
 const dim3 kReduceBlock(32, tc::kSlotGroups);
-int reduce_grid(int64_t n4, const Ctx &c)
+tc::ReduceJob reduce_job(const float *part, int64_t slots, int64_t rows, int64_t cols, float *out, int transpose,
+                         int out4, int64_t cap)
 {
-    int64_t g = (n4 + 31) / 32;
-    const int64_t cap = (int64_t)c.sm_count * 8;
+    int64_t g = (rows * cols / 4 + 31) / 32;
     if (g > cap) g = cap;
-    return (int)(g < 1 ? 1 : g);
+    return tc::ReduceJob{part, slots, rows, cols, out, transpose, out4, (int)(g < 1 ? 1 : g)};
+}
+cudaError_t launch_reduce(const tc::ReduceJob &small, tc::ReduceJob big, const Ctx &c)
+{
+    const int64_t resident = (int64_t)c.sm_count * 8;
+    const int64_t left = resident - small.blocks;
+    if (big.blocks > left && left >= 1) big.blocks = (int)left;
+    tc::k_reduce_slots<<<small.blocks + big.blocks, kReduceBlock, 0, c.stream>>>(small, big);
+    count_launches(1);
+    return cudaGetLastError();
 }
 
 CUtensorMapSwizzle swizzle_for(uint32_t row_bytes)
@@ -189,11 +199,9 @@ cudaError_t launch_dec_bwd(const resbm_desc &d, const void *dY, const void *B, c
     count_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     // dWd2 (m x d) = sum of the per-CTA slots (d x m), transposed; dWd1 (r x m) = sum of the slices
-    tc::k_reduce_slots<<<reduce_grid(d.d * d.m / 4, c), kReduceBlock, 0, c.stream>>>(p.part_big, p.grid, d.d, d.m, dWd2, 1, 0);
-    tc::k_reduce_slots<<<reduce_grid(d.r * d.m / 4, c), kReduceBlock, 0, c.stream>>>(p.part_small, p.slots, d.r, d.m, dWd1, 0,
-                                                                              al16(dWd1));
-    count_launches(2);
-    return cudaGetLastError();
+    const int64_t cap = (int64_t)c.sm_count * 8;
+    return launch_reduce(reduce_job(p.part_small, p.slots, d.r, d.m, dWd1, 0, al16(dWd1), cap),
+                         reduce_job(p.part_big, p.grid, d.d, d.m, dWd2, 1, 0, cap), c);
 }
 
 int dec_bwd_nt(int64_t m)
@@ -250,12 +258,9 @@ cudaError_t launch_enc_bwd(const resbm_desc &d, const void *dB, const void *F, c
                                                                           m_db, a);
     count_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    tc::k_reduce_slots<<<reduce_grid(d.d * d.m / 4, c), kReduceBlock, 0, c.stream>>>(p.part_big, p.grid, d.d, d.m, dWe1, 0,
-                                                                            al16(dWe1));
-    tc::k_reduce_slots<<<reduce_grid(d.m * d.r / 4, c), kReduceBlock, 0, c.stream>>>(p.part_small, p.slots, d.m, d.r, dWe2, 0,
-                                                                              al16(dWe2));
-    count_launches(2);
-    return cudaGetLastError();
+    const int64_t cap = (int64_t)c.sm_count * 8;
+    return launch_reduce(reduce_job(p.part_small, p.slots, d.m, d.r, dWe2, 0, al16(dWe2), cap),
+                         reduce_job(p.part_big, p.grid, d.d, d.m, dWe1, 0, al16(dWe1), cap), c);
 }
 
 }  // namespace

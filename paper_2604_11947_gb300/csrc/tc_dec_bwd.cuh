@@ -368,8 +368,9 @@ __global__ void __launch_bounds__(192, 1)
                 const bool active = t0 + row < end;
                 float v[C::M];
                 tmem_ld_row<C::M>(tmem + lane_base + C::TM_Q + (i - tb) * C::MS, v);
+                act_fast_row<C::M>(a.act, v);
 #pragma unroll
-                for (int j = 0; j < C::M; ++j) v[j] = active ? act_fast(a.act, v[j]) : 0.0f;
+                for (int j = 0; j < C::M; ++j) v[j] = active ? v[j] : 0.0f;
                 store_bf16_swz_row<C::M>(smem + C::OFF_G + (i - tb) * C::TILE, row, v);
                 // publish this tile's G so its first dWd2 product can start
                 fence_async_smem();
@@ -398,9 +399,10 @@ __global__ void __launch_bounds__(192, 1)
                 float hi[C::M], lo[C::M];
                 tmem_ld_row<C::M>(tmem + lane_base + C::TM_DG + (i - tb) * C::MS, hi);
                 tmem_ld_row<C::M>(tmem + lane_base + C::TM_Q + (i - tb) * C::MS, lo);
+                dact_fast_row<C::M>(a.act, lo, lo);   // phi'(Q)
 #pragma unroll
                 for (int j = 0; j < C::M; ++j) {
-                    const float x = active ? hi[j] * dact_f(a.act, lo[j]) : 0.0f;
+                    const float x = active ? hi[j] * lo[j] : 0.0f;
                     hi[j] = __bfloat162float(__float2bfloat16_rn(x));
                     lo[j] = x - hi[j];
                 }
@@ -482,34 +484,41 @@ __device__ __forceinline__ void add4(float4 &a, const float4 &b)
     a.x += b.x; a.y += b.y; a.z += b.z; a.w += b.w;
 }
 
-// Fixed-order sum of `slots` partial fp32 matrices (rows x cols, cols % 4 == 0) into `out`
-// (transposed to cols x rows if `transpose`; `out4`: out is 16-byte aligned). A block of
-// 32 x kSlotGroups threads owns 32 consecutive float4 columns of the flattened matrix; thread
-// row g sums the g-th contiguous range of slots in slot order, and the groups' sums are then
-// added in group order: the same order for every launch, so results are bitwise reproducible.
-constexpr int kSlotGroups = 16;
+// Fixed-order sums of per-CTA partial fp32 matrices. A job sums `slots` matrices of rows x cols
+// (rows * cols % 4 == 0) into `out` (transposed to cols x rows if `transpose`; `out4`: out is
+// 16-byte aligned). A block of 32 x kSlotGroups threads owns 32 consecutive float4 columns of
+// the flattened matrix; thread row g sums the g-th contiguous range of slots in slot order, and
+// the groups' sums are then added in group order: the same order for every launch, so results
+// are bitwise reproducible. One launch runs two jobs (the two weight gradients of a backward
+// op): blocks [0, first.blocks) take the first, the rest the second.
+constexpr int kSlotGroups = 8;
 
-__global__ void __launch_bounds__(32 * kSlotGroups) k_reduce_slots(const float *__restrict__ part, int64_t slots,
-                                                                   int64_t rows, int64_t cols,
-                                                                   float *__restrict__ out, int transpose, int out4)
+struct ReduceJob {
+    const float *part;
+    int64_t slots, rows, cols;
+    float *out;
+    int transpose, out4;
+    int blocks;
+};
+
+__device__ __forceinline__ void reduce_job(const ReduceJob &j, int64_t block, int64_t nblocks, float4 (&grp)[kSlotGroups][32])
 {
-    __shared__ float4 grp[kSlotGroups][32];
-    const int64_t n4 = rows * cols / 4;
-    const float4 *p4 = reinterpret_cast<const float4 *>(part);
-    const int64_t per = (slots + kSlotGroups - 1) / kSlotGroups;
+    const int64_t n4 = j.rows * j.cols / 4;
+    const float4 *p4 = reinterpret_cast<const float4 *>(j.part);
+    const int64_t per = (j.slots + kSlotGroups - 1) / kSlotGroups;
     const int64_t s0 = threadIdx.y * per;
-    const int64_t s1 = s0 + per < slots ? s0 + per : slots;
-    for (int64_t base = (int64_t)blockIdx.x * 32; base < n4; base += (int64_t)gridDim.x * 32) {
+    const int64_t s1 = s0 + per < j.slots ? s0 + per : j.slots;
+    for (int64_t base = block * 32; base < n4; base += nblocks * 32) {
         const int64_t e4 = base + threadIdx.x;
         float4 acc = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
         if (e4 < n4) {
             int64_t s = s0;
-            for (; s + 4 <= s1; s += 4) {
-                float4 v[4];
+            for (; s + 8 <= s1; s += 8) {
+                float4 v[8];
 #pragma unroll
-                for (int u = 0; u < 4; ++u) v[u] = __ldcs(&p4[(s + u) * n4 + e4]);
+                for (int u = 0; u < 8; ++u) v[u] = __ldcs(&p4[(s + u) * n4 + e4]);
 #pragma unroll
-                for (int u = 0; u < 4; ++u) add4(acc, v[u]);
+                for (int u = 0; u < 8; ++u) add4(acc, v[u]);
             }
             for (; s < s1; ++s) add4(acc, __ldcs(&p4[s * n4 + e4]));
         }
@@ -520,20 +529,29 @@ __global__ void __launch_bounds__(32 * kSlotGroups) k_reduce_slots(const float *
 #pragma unroll
             for (int g = 1; g < kSlotGroups; ++g) add4(t, grp[g][threadIdx.x]);
             const int64_t e = 4 * e4;
-            if (transpose) {
-                const int64_t rr = e / cols, cc = e - rr * cols;
-                out[(cc + 0) * rows + rr] = t.x;
-                out[(cc + 1) * rows + rr] = t.y;
-                out[(cc + 2) * rows + rr] = t.z;
-                out[(cc + 3) * rows + rr] = t.w;
-            } else if (out4) {
-                reinterpret_cast<float4 *>(out)[e4] = t;
+            if (j.transpose) {
+                const int64_t rr = e / j.cols, cc = e - rr * j.cols;
+                j.out[(cc + 0) * j.rows + rr] = t.x;
+                j.out[(cc + 1) * j.rows + rr] = t.y;
+                j.out[(cc + 2) * j.rows + rr] = t.z;
+                j.out[(cc + 3) * j.rows + rr] = t.w;
+            } else if (j.out4) {
+                reinterpret_cast<float4 *>(j.out)[e4] = t;
             } else {
-                out[e] = t.x; out[e + 1] = t.y; out[e + 2] = t.z; out[e + 3] = t.w;
+                j.out[e] = t.x; j.out[e + 1] = t.y; j.out[e + 2] = t.z; j.out[e + 3] = t.w;
             }
         }
         __syncthreads();
     }
+}
+
+__global__ void __launch_bounds__(32 * kSlotGroups) k_reduce_slots(const ReduceJob first, const ReduceJob second)
+{
+    __shared__ float4 grp[kSlotGroups][32];
+    if ((int)blockIdx.x < first.blocks)
+        reduce_job(first, blockIdx.x, first.blocks, grp);
+    else
+        reduce_job(second, blockIdx.x - first.blocks, gridDim.x - first.blocks, grp);
 }
 
 }  // namespace tc

@@ -197,11 +197,12 @@ __global__ void __launch_bounds__(192, 1)
                         accq[2 * j + 1] = fmaf(bk, __uint_as_float(wv[j] & 0xFFFF0000u), accq[2 * j + 1]);
                     }
                 }
+                act_fast_row<16>(a.act, accq);
                 uint32_t packed[8];
 #pragma unroll
                 for (int j = 0; j < 8; ++j) {
-                    const float g0 = active ? act_f(a.act, accq[2 * j]) : 0.0f;
-                    const float g1 = active ? act_f(a.act, accq[2 * j + 1]) : 0.0f;
+                    const float g0 = active ? accq[2 * j] : 0.0f;
+                    const float g1 = active ? accq[2 * j + 1] : 0.0f;
                     __nv_bfloat162 h = __floats2bfloat162_rn(g0, g1);
                     packed[j] = *reinterpret_cast<uint32_t *>(&h);
                 }

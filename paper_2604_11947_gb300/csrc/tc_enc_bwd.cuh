@@ -364,15 +364,14 @@ __global__ void __launch_bounds__(192, 1)
                 tmem_ld_row<C::M>(tmem + lane_base + C::TM_DA + rg * C::MS, da);
                 tc_fence_before();
                 mbar_arrive(smem_u32(&da_empty[rg]));   // the dA region is free again
-                float av[C::M];
+                float av[C::M], dph[C::M];
+                act_dact_row<C::M>(a.act, pv, av, dph);
 #pragma unroll
                 for (int jj = 0; jj < C::M; ++jj) {
-                    float ph = 0.0f, dph = 0.0f;
-                    act_and_dact(a.act, pv[jj], ph, dph);
-                    const float x = active ? da[jj] * dph : 0.0f;
+                    const float x = active ? da[jj] * dph[jj] : 0.0f;
                     da[jj] = __bfloat162float(__float2bfloat16_rn(x));   // hi
                     pv[jj] = x - da[jj];                                 // lo
-                    av[jj] = active ? ph : 0.0f;
+                    av[jj] = active ? av[jj] : 0.0f;
                 }
                 store_bf16_swz_row<C::M>(smem + C::OFF_DP + (i - tb) * C::TILE, row, da);
                 if (C::DPLO) store_bf16_swz_row<C::M>(smem + C::OFF_DPLO + (i - tb) * C::TILE, row, pv);

@@ -183,8 +183,7 @@ __global__ void __launch_bounds__(192, 1)
                     for (int j = 0; j < C::M / 4; ++j)
                         dst[j] = make_float4(p[4 * j], p[4 * j + 1], p[4 * j + 2], p[4 * j + 3]);
                 }
-#pragma unroll
-                for (int j = 0; j < C::M; ++j) p[j] = act_f(a.act, p[j]);
+                act_row<C::M>(a.act, p);
                 const uint4 *xs = reinterpret_cast<const uint4 *>(a.X + tok * a.d);
                 uint4 *bd = reinterpret_cast<uint4 *>(a.B + tok * C::R);
 #pragma unroll
