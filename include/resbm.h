@@ -85,6 +85,11 @@ typedef enum {
 
 /* desc.flags bits */
 #define RESBM_FLAG_GENERIC 1u   /* force the portable CUDA-core kernels (no tensor cores) */
+/* One linear layer on each side instead of two (the single-matrix special case of Sec. 3.2's
+ * encoder / decoder): E(F) = F . We1 with We1 d x r, D(B) = B . Wd2 with Wd2 r x d. Requires
+ * m == r; act is not used; We2 and Wd1 are not read and dWe2 and dWd1 not written (all may be
+ * NULL). Everything else, the identity path included, is as in the two-layer form. */
+#define RESBM_FLAG_LINEAR 2u
 
 typedef struct {
     int64_t T;               /* tokens (batch * sequence), >= 0                              */

@@ -50,6 +50,14 @@ def _load(path=None):
     lib.oracle_decode_bwd.argtypes = [_i64] * 4 + [ctypes.c_int] * 2 + [_dp] * 7
     lib.oracle_encode_bwd.restype = ctypes.c_int
     lib.oracle_encode_bwd.argtypes = [_i64] * 4 + [ctypes.c_int] + [_dp] * 8
+    lib.oracle_linear_encode_fwd.restype = ctypes.c_int
+    lib.oracle_linear_encode_fwd.argtypes = [_i64] * 3 + [_dp] * 4
+    lib.oracle_linear_decode_fwd.restype = ctypes.c_int
+    lib.oracle_linear_decode_fwd.argtypes = [_i64] * 3 + [ctypes.c_int] + [_dp] * 3
+    lib.oracle_linear_decode_bwd.restype = ctypes.c_int
+    lib.oracle_linear_decode_bwd.argtypes = [_i64] * 3 + [ctypes.c_int] + [_dp] * 5
+    lib.oracle_linear_encode_bwd.restype = ctypes.c_int
+    lib.oracle_linear_encode_bwd.argtypes = [_i64] * 3 + [_dp] * 6
     return lib
 
 
@@ -177,6 +185,65 @@ class Oracle:
             raise MemoryError("oracle_encode_bwd")
         return dF, dX, dWe1, dWe2
 
+    # -- one linear layer per side (no nonlinearity) ------------------------------------------
+    def linear_encode_fwd(self, X, F, We):
+        """Returns B = X . I_{d x r} + F . We (We: d x r)."""
+        F = np.asarray(F)
+        T, d = F.shape
+        r = np.asarray(We).shape[1]
+        X = self._in(X, (T, d)); F = self._in(F, (T, d)); We = self._in(We, (d, r))
+        B = np.empty((T, r))
+        if self._l.oracle_linear_encode_fwd(T, d, r, self._p(X), self._p(F), self._p(We), self._p(B)) != 0:
+            raise MemoryError("oracle_linear_encode_fwd")
+        return B
+
+    def linear_decode_fwd(self, B, Wd, merge=1):
+        """Returns Y = [merge] B . I_{r x d} + B . Wd (Wd: r x d)."""
+        B = np.asarray(B)
+        T, r = B.shape
+        d = np.asarray(Wd).shape[1]
+        B = self._in(B, (T, r)); Wd = self._in(Wd, (r, d))
+        Y = np.empty((T, d))
+        if self._l.oracle_linear_decode_fwd(T, d, r, int(merge), self._p(B), self._p(Wd), self._p(Y)) != 0:
+            raise MemoryError("oracle_linear_decode_fwd")
+        return Y
+
+    def linear_decode_bwd(self, dY, B, Wd, merge=1):
+        """Returns (dB, dWd) for the upstream gradient dY of linear_decode_fwd's Y."""
+        B = np.asarray(B)
+        T, r = B.shape
+        d = np.asarray(Wd).shape[1]
+        dY = self._in(dY, (T, d)); B = self._in(B, (T, r)); Wd = self._in(Wd, (r, d))
+        dB = np.empty((T, r)); dWd = np.empty((r, d))
+        if self._l.oracle_linear_decode_bwd(T, d, r, int(merge), self._p(dY), self._p(B), self._p(Wd),
+                                            self._p(dB), self._p(dWd)) != 0:
+            raise MemoryError("oracle_linear_decode_bwd")
+        return dB, dWd
+
+    def linear_encode_bwd(self, dB, F, We, want_dX=True):
+        """Returns (dF, dX, dWe) for the upstream gradient dB of linear_encode_fwd's B."""
+        F = np.asarray(F)
+        T, d = F.shape
+        r = np.asarray(We).shape[1]
+        dB = self._in(dB, (T, r)); F = self._in(F, (T, d)); We = self._in(We, (d, r))
+        dF = np.empty((T, d)); dX = np.empty((T, d)) if want_dX else None; dWe = np.empty((d, r))
+        if self._l.oracle_linear_encode_bwd(T, d, r, self._p(dB), self._p(F), self._p(We), self._p(dF),
+                                            self._p(dX), self._p(dWe)) != 0:
+            raise MemoryError("oracle_linear_encode_bwd")
+        return dF, dX, dWe
+
+    def linear_boundary_step(self, X, F, dY, We, Wd, merge=1, transfer=None):
+        """The one-linear-layer boundary forward + backward, chained like boundary_step."""
+        B = self.linear_encode_fwd(X, F, We)
+        if transfer:
+            B = self.round_to(B, transfer)
+        Y = self.linear_decode_fwd(B, Wd, merge)
+        dB, dWd = self.linear_decode_bwd(dY, B, Wd, merge)
+        if transfer:
+            dB = self.round_to(dB, transfer)
+        dF, dX, dWe = self.linear_encode_bwd(dB, F, We)
+        return dict(B=B, Y=Y, dB=dB, dF=dF, dX=dX, dWe1=dWe, dWd2=dWd)
+
     def boundary_step(self, X, F, dY, We1, We2, Wd1, Wd2, act="silu", merge=1, transfer=None):
         """One boundary forward + backward: the four functions above chained. B is handed to
         the decoder and dB back to the encoder; with transfer = "bf16" / "f32" they are first
@@ -207,6 +274,8 @@ def default():
 def __getattr__(name):
     # module-level shortcuts: oracle.encode_fwd(...) etc.
     if name in ("act", "dact", "rect_identity", "pid", "encode_fwd", "decode_fwd", "round_to",
-                "decode_bwd", "encode_bwd", "boundary_step", "max_threads"):
+                "decode_bwd", "encode_bwd", "boundary_step", "max_threads", "linear_encode_fwd",
+                "linear_decode_fwd", "linear_decode_bwd", "linear_encode_bwd",
+                "linear_boundary_step"):
         return getattr(default(), name)
     raise AttributeError(name)

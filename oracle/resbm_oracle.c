@@ -316,3 +316,66 @@ int oracle_encode_bwd(int64_t T, int64_t d, int64_t r, int64_t m, int act,
     free(P); free(A); free(dA); free(dP);
     return rc;
 }
+
+/* ------------------------------------------------------------------------------------------ */
+/* One linear layer per side (the single-matrix special case of the Sec. 3.2 encoder and       */
+/* decoder; no nonlinearity):                                                                   */
+/*   send:     B = X . I_{d x r} + F . We          We: d x r                                    */
+/*   receive:  Y = merge ? B . I_{r x d} + B . Wd : B . Wd          Wd: r x d                   */
+/*   backward: dB = B-gradient of sum(dY * Y) = merge * dY . I_{r x d}^T + dY . Wd^T;           */
+/*             dWd = B^T . dY;  dF = dB . We^T;  dWe = F^T . dB;  dX = dB . I_{d x r}^T.          */
+/* ------------------------------------------------------------------------------------------ */
+int oracle_linear_encode_fwd(int64_t T, int64_t d, int64_t r, const double *X, const double *F,
+                             const double *We, double *B)
+{
+    double *S = alloc_d(T * r), *L = alloc_d(T * r);
+    int rc = (S && L) ? 0 : -1;
+    if (rc == 0) rc = oracle_pid(T, d, r, X, S);
+    if (rc == 0) {
+        mm_nn(T, r, d, F, We, L);                /* L = F . We             */
+        for (int64_t i = 0; i < T * r; ++i) B[i] = S[i] + L[i];
+    }
+    free(S); free(L);
+    return rc;
+}
+
+int oracle_linear_decode_fwd(int64_t T, int64_t d, int64_t r, int merge, const double *B,
+                             const double *Wd, double *Y)
+{
+    double *L = alloc_d(T * d), *Pad = merge ? alloc_d(T * d) : NULL;
+    int rc = (L && (!merge || Pad)) ? 0 : -1;
+    if (rc == 0) {
+        mm_nn(T, d, r, B, Wd, L);                /* L = B . Wd             */
+        if (merge) rc = oracle_pid(T, r, d, B, Pad);
+    }
+    if (rc == 0)
+        for (int64_t i = 0; i < T * d; ++i) Y[i] = merge ? Pad[i] + L[i] : L[i];
+    free(L); free(Pad);
+    return rc;
+}
+
+int oracle_linear_decode_bwd(int64_t T, int64_t d, int64_t r, int merge, const double *dY,
+                             const double *B, const double *Wd, double *dB, double *dWd)
+{
+    double *dBskip = alloc_d(T * r);
+    int rc = dBskip ? 0 : -1;
+    if (rc == 0) {
+        mm_tn(r, d, T, B, dY, dWd);              /* dWd = B^T . dY          */
+        mm_nt(T, r, d, dY, Wd, dB);              /* dB  = dY . Wd^T         */
+        if (merge == 1) {                        /* + dY . I_{r x d}^T      */
+            rc = pid_backward(T, r, d, dY, dBskip);
+            if (rc == 0)
+                for (int64_t i = 0; i < T * r; ++i) dB[i] += dBskip[i];
+        }
+    }
+    free(dBskip);
+    return rc;
+}
+
+int oracle_linear_encode_bwd(int64_t T, int64_t d, int64_t r, const double *dB, const double *F,
+                             const double *We, double *dF, double *dX, double *dWe)
+{
+    mm_tn(d, r, T, F, dB, dWe);                  /* dWe = F^T . dB          */
+    mm_nt(T, d, r, dB, We, dF);                  /* dF  = dB . We^T         */
+    return dX ? pid_backward(T, d, r, dB, dX) : 0;
+}

@@ -169,6 +169,13 @@ __global__ void k_dx_accumulate(T *dX, const T *__restrict__ dB, int64_t Tn, int
     }
 }
 
+// out = the n x n identity matrix
+template <typename T> __global__ void k_identity(T *out, int64_t n)
+{
+    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n * n; e += (int64_t)gridDim.x * blockDim.x)
+        out[e] = from_f32<T>(e / n == e % n ? 1.0f : 0.0f);
+}
+
 int grid_for(int64_t n, const Ctx &c)
 {
     int64_t g = (n + 255) / 256;
@@ -372,6 +379,17 @@ cudaError_t generic_encode_bwd(const resbm_desc &d, const void *dB, const void *
                          (const float *)We2, (float *)dF, (float *)dX, dWe1, dWe2, ws, c),
         enc_bwd_t<bf>(d, (const bf *)dB, (const bf *)F, P_save, (const bf *)We1,
                       (const bf *)We2, (bf *)dF, (bf *)dX, dWe1, dWe2, ws, c));
+}
+
+cudaError_t fill_identity(const resbm_desc &d, void *out, const Ctx &c)
+{
+    const int64_t n = d.r;
+    if (d.dtype == RESBM_F32)
+        k_identity<float><<<grid_for(n * n, c), 256, 0, c.stream>>>(static_cast<float *>(out), n);
+    else
+        k_identity<__nv_bfloat16><<<grid_for(n * n, c), 256, 0, c.stream>>>(static_cast<__nv_bfloat16 *>(out), n);
+    count_launches(1);
+    return cudaGetLastError();
 }
 
 }  // namespace resbm

@@ -35,6 +35,8 @@ struct WsCarver {
 
 // ---- generic CUDA-core path (any shape, fp32 or bf16) ------------------------------------
 size_t generic_ws_bytes(const resbm_desc &d, int op);
+// out (r x r, the descriptor's dtype) = the identity matrix
+cudaError_t fill_identity(const resbm_desc &d, void *out, const Ctx &c);
 cudaError_t generic_encode_fwd(const resbm_desc &d, const void *X, const void *F, const void *We1,
                                const void *We2, void *B, float *P_save, void *ws, const Ctx &c);
 cudaError_t generic_decode_fwd(const resbm_desc &d, const void *B, const void *Wd1,

@@ -79,7 +79,8 @@ resbm_status check_desc(const resbm_desc *d)
     if (d->act != RESBM_ACT_SILU && d->act != RESBM_ACT_GELU_TANH && d->act != RESBM_ACT_IDENTITY)
         return RESBM_ERR_INVALID_ARG;
     if (d->merge_identity != 0 && d->merge_identity != 1) return RESBM_ERR_INVALID_ARG;
-    if (d->flags & ~RESBM_FLAG_GENERIC) return RESBM_ERR_INVALID_ARG;
+    if (d->flags & ~(RESBM_FLAG_GENERIC | RESBM_FLAG_LINEAR)) return RESBM_ERR_INVALID_ARG;
+    if ((d->flags & RESBM_FLAG_LINEAR) && d->m != d->r) return RESBM_ERR_INVALID_ARG;
     // every element count (and the byte counts derived from it) must fit in int64
     const int64_t big = INT64_MAX / 64;
     if (!mul_ok(d->T, d->d) || d->T * d->d > big || !mul_ok(d->T, d->m) || d->T * d->m > big ||
@@ -121,11 +122,48 @@ template <size_t N> bool any_overlap(const Range (&outs)[N], const Range *ins, s
 
 bool use_tc(const resbm_desc &d, int op) { return !(d.flags & RESBM_FLAG_GENERIC) && tc_supported(d, op); }
 
-size_t ws_for(const resbm_desc &d, int op)
+// ---- RESBM_FLAG_LINEAR ---------------------------------------------------------------------
+// One linear layer per side runs as the two-layer path with identity second layers
+// (We2 = Wd1 = I_r, phi = identity): exact, since multiplying by I_r and applying the identity
+// function change no value. The identity matrix and two r x r gradient outputs nobody reads
+// sit at the front of the workspace.
+bool is_linear(const resbm_desc &d) { return (d.flags & RESBM_FLAG_LINEAR) != 0; }
+
+resbm_desc two_layer(const resbm_desc &d)
 {
+    resbm_desc e = d;
+    if (is_linear(d)) {
+        e.act = RESBM_ACT_IDENTITY;
+        e.flags &= ~RESBM_FLAG_LINEAR;
+    }
+    return e;
+}
+
+struct LinearWs {
+    void *I;
+    float *dW2, *dW1;
+    void *inner;
+    size_t bytes;
+};
+LinearWs carve_linear(const resbm_desc &d, void *ws)
+{
+    WsCarver w(ws);
+    LinearWs l;
+    l.I = w.take<char>((size_t)(d.r * d.r) * elem_size(d));
+    l.dW2 = w.take<float>(d.r * d.r);
+    l.dW1 = w.take<float>(d.r * d.r);
+    l.inner = w.take<char>(0);
+    l.bytes = w.used;
+    return l;
+}
+
+size_t ws_for(const resbm_desc &d0, int op)
+{
+    const resbm_desc d = two_layer(d0);
     size_t g = generic_ws_bytes(d, op);
     size_t t = tc_supported(d, op) ? tc_ws_bytes(d, op, sizing_sms()) : 0;
-    return g > t ? g : t;
+    const size_t inner = g > t ? g : t;
+    return is_linear(d0) ? carve_linear(d0, nullptr).bytes + inner : inner;
 }
 
 size_t step_ws_bytes(const resbm_desc &d)
@@ -167,7 +205,7 @@ resbm_status validate_encode_fwd(const resbm_desc &d, const void *X, const void 
     const size_t es = elem_size(d);
     const bool t = d.T > 0;
     if (!ptr_ok(X, es, t) || !ptr_ok(F, es, t) || !ptr_ok(We1, es, true) ||
-        !ptr_ok(We2, es, true) || !ptr_ok(B, es, t) || !ptr_ok(P, 4, false))
+        !ptr_ok(We2, es, !is_linear(d)) || !ptr_ok(B, es, t) || !ptr_ok(P, 4, false))
         return RESBM_ERR_INVALID_ARG;
     const Range outs[] = {rng(B, d.T * d.r, es), rng(P, d.T * d.m, 4)};
     const Range ins[] = {rng(X, d.T * d.d, es), rng(F, d.T * d.d, es), rng(We1, d.d * d.m, es),
@@ -180,7 +218,7 @@ resbm_status validate_decode_fwd(const resbm_desc &d, const void *B, const void 
 {
     const size_t es = elem_size(d);
     const bool t = d.T > 0;
-    if (!ptr_ok(B, es, t) || !ptr_ok(Wd1, es, true) || !ptr_ok(Wd2, es, true) ||
+    if (!ptr_ok(B, es, t) || !ptr_ok(Wd1, es, !is_linear(d)) || !ptr_ok(Wd2, es, true) ||
         !ptr_ok(Y, es, t))
         return RESBM_ERR_INVALID_ARG;
     const Range outs[] = {rng(Y, d.T * d.d, es)};
@@ -194,8 +232,8 @@ resbm_status validate_decode_bwd(const resbm_desc &d, const void *dY, const void
 {
     const size_t es = elem_size(d);
     const bool t = d.T > 0;
-    if (!ptr_ok(dY, es, t) || !ptr_ok(B, es, t) || !ptr_ok(Wd1, es, true) ||
-        !ptr_ok(Wd2, es, true) || !ptr_ok(dB, es, t) || !ptr_ok(dWd1, 4, true) ||
+    if (!ptr_ok(dY, es, t) || !ptr_ok(B, es, t) || !ptr_ok(Wd1, es, !is_linear(d)) ||
+        !ptr_ok(Wd2, es, true) || !ptr_ok(dB, es, t) || !ptr_ok(dWd1, 4, !is_linear(d)) ||
         !ptr_ok(dWd2, 4, true))
         return RESBM_ERR_INVALID_ARG;
     const Range outs[] = {rng(dB, d.T * d.r, es), rng(dWd1, d.r * d.m, 4), rng(dWd2, d.m * d.d, 4)};
@@ -212,8 +250,8 @@ resbm_status validate_encode_bwd(const resbm_desc &d, const void *dB, const void
     const size_t es = elem_size(d);
     const bool t = d.T > 0;
     if (!ptr_ok(dB, es, t) || !ptr_ok(F, es, t) || !ptr_ok(P, 4, false) ||
-        !ptr_ok(We1, es, true) || !ptr_ok(We2, es, true) || !ptr_ok(dF, es, t) ||
-        !ptr_ok(dX, es, false) || !ptr_ok(dWe1, 4, true) || !ptr_ok(dWe2, 4, true))
+        !ptr_ok(We1, es, true) || !ptr_ok(We2, es, !is_linear(d)) || !ptr_ok(dF, es, t) ||
+        !ptr_ok(dX, es, false) || !ptr_ok(dWe1, 4, true) || !ptr_ok(dWe2, 4, !is_linear(d)))
         return RESBM_ERR_INVALID_ARG;
     const Range outs[] = {rng(dF, d.T * d.d, es), rng(dX, d.T * d.d, es), rng(dWe1, d.d * d.m, 4),
                           rng(dWe2, d.m * d.r, 4)};
@@ -275,6 +313,48 @@ resbm_status run_encode_bwd(const resbm_desc &d, const void *dB, const void *F, 
         if (e != cudaErrorNotSupported) return finish(e);
     }
     return finish(generic_encode_bwd(d, dB, F, P, We1, We2, dF, dX, dWe1, dWe2, ws, c));
+}
+
+// ---- the four ops on either form (after validation) -----------------------------------------
+resbm_status exec_encode_fwd(const resbm_desc &d, const void *X, const void *F, const void *We1,
+                             const void *We2, void *B, float *P, void *ws, const Ctx &c)
+{
+    if (!is_linear(d)) return run_encode_fwd(d, X, F, We1, We2, B, P, ws, c);
+    const LinearWs l = carve_linear(d, ws);
+    resbm_status s = finish(fill_identity(d, l.I, c));
+    return s != RESBM_OK ? s : run_encode_fwd(two_layer(d), X, F, We1, l.I, B, P, l.inner, c);
+}
+
+resbm_status exec_decode_fwd(const resbm_desc &d, const void *B, const void *Wd1, const void *Wd2,
+                             void *Y, void *ws, const Ctx &c)
+{
+    if (!is_linear(d)) return run_decode_fwd(d, B, Wd1, Wd2, Y, ws, c);
+    const LinearWs l = carve_linear(d, ws);
+    resbm_status s = finish(fill_identity(d, l.I, c));
+    return s != RESBM_OK ? s : run_decode_fwd(two_layer(d), B, l.I, Wd2, Y, l.inner, c);
+}
+
+resbm_status exec_decode_bwd(const resbm_desc &d, const void *dY, const void *B, const void *Wd1,
+                             const void *Wd2, void *dB, float *dWd1, float *dWd2, void *ws,
+                             const Ctx &c)
+{
+    if (!is_linear(d)) return run_decode_bwd(d, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, c);
+    const LinearWs l = carve_linear(d, ws);
+    resbm_status s = finish(fill_identity(d, l.I, c));
+    return s != RESBM_OK ? s
+                         : run_decode_bwd(two_layer(d), dY, B, l.I, Wd2, dB, l.dW1, dWd2, l.inner, c);
+}
+
+resbm_status exec_encode_bwd(const resbm_desc &d, const void *dB, const void *F, const float *P,
+                             const void *We1, const void *We2, void *dF, void *dX, float *dWe1,
+                             float *dWe2, void *ws, const Ctx &c)
+{
+    if (!is_linear(d)) return run_encode_bwd(d, dB, F, P, We1, We2, dF, dX, dWe1, dWe2, ws, c);
+    const LinearWs l = carve_linear(d, ws);
+    resbm_status s = finish(fill_identity(d, l.I, c));
+    return s != RESBM_OK ? s
+                         : run_encode_bwd(two_layer(d), dB, F, P, We1, l.I, dF, dX, dWe1, l.dW2,
+                                          l.inner, c);
 }
 
 // ---- fixed scratch of resbm_decode_bwd_noalloc -----------------------------------------------
@@ -345,7 +425,7 @@ resbm_status resbm_encode_fwd(const resbm_desc *desc, const void *X, const void 
     if (s == RESBM_OK) s = check_ws(*desc, RESBM_OP_ENCODE_FWD, ws, ws_bytes);
     Ctx c;
     if (s == RESBM_OK) s = make_ctx(stream, &c);
-    if (s == RESBM_OK) s = run_encode_fwd(*desc, X, F, We1, We2, B, P_save, ws, c);
+    if (s == RESBM_OK) s = exec_encode_fwd(*desc, X, F, We1, We2, B, P_save, ws, c);
     return s;
 }
 
@@ -357,7 +437,7 @@ resbm_status resbm_decode_fwd(const resbm_desc *desc, const void *B, const void 
     if (s == RESBM_OK) s = check_ws(*desc, RESBM_OP_DECODE_FWD, ws, ws_bytes);
     Ctx c;
     if (s == RESBM_OK) s = make_ctx(stream, &c);
-    if (s == RESBM_OK) s = run_decode_fwd(*desc, B, Wd1, Wd2, Y, ws, c);
+    if (s == RESBM_OK) s = exec_decode_fwd(*desc, B, Wd1, Wd2, Y, ws, c);
     return s;
 }
 
@@ -370,7 +450,7 @@ resbm_status resbm_decode_bwd(const resbm_desc *desc, const void *dY, const void
     if (s == RESBM_OK) s = check_ws(*desc, RESBM_OP_DECODE_BWD, ws, ws_bytes);
     Ctx c;
     if (s == RESBM_OK) s = make_ctx(stream, &c);
-    if (s == RESBM_OK) s = run_decode_bwd(*desc, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, c);
+    if (s == RESBM_OK) s = exec_decode_bwd(*desc, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, c);
     return s;
 }
 
@@ -386,7 +466,7 @@ resbm_status resbm_decode_bwd_noalloc(const resbm_desc *desc, const void *dY, co
     if (s == RESBM_OK) s = make_ctx(stream, &c);
     void *ws = nullptr;
     if (s == RESBM_OK) s = static_scratch(c.device, &ws);
-    if (s == RESBM_OK) s = run_decode_bwd(*desc, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, c);
+    if (s == RESBM_OK) s = exec_decode_bwd(*desc, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, c);
     return s;
 }
 
@@ -402,7 +482,7 @@ resbm_status resbm_encode_bwd(const resbm_desc *desc, const void *dB, const void
     Ctx c;
     if (s == RESBM_OK) s = make_ctx(stream, &c);
     if (s == RESBM_OK)
-        s = run_encode_bwd(*desc, dB, F, P_save, We1, We2, dF, dX, dWe1, dWe2, ws, c);
+        s = exec_encode_bwd(*desc, dB, F, P_save, We1, We2, dF, dX, dWe1, dWe2, ws, c);
     return s;
 }
 
@@ -440,13 +520,23 @@ resbm_status resbm_boundary_step(const resbm_desc *desc, const resbm_step_args *
     }
     Ctx c;
     if (s == RESBM_OK) s = make_ctx(stream, &c);
-    if (s == RESBM_OK) s = run_encode_fwd(d, a->X, a->F, a->We1, a->We2, a->B, P, inner, c);
-    if (s == RESBM_OK) s = run_decode_fwd(d, a->B, a->Wd1, a->Wd2, a->Y, inner, c);
+    const void *We2 = a->We2, *Wd1 = a->Wd1;
+    float *dWe2 = a->dWe2, *dWd1 = a->dWd1;
+    const resbm_desc e = two_layer(d);
+    if (s == RESBM_OK && is_linear(d)) {
+        const LinearWs l = carve_linear(d, inner);
+        s = finish(fill_identity(d, l.I, c));
+        We2 = Wd1 = l.I;
+        dWe2 = l.dW2;
+        dWd1 = l.dW1;
+        inner = l.inner;
+    }
+    if (s == RESBM_OK) s = run_encode_fwd(e, a->X, a->F, a->We1, We2, a->B, P, inner, c);
+    if (s == RESBM_OK) s = run_decode_fwd(e, a->B, Wd1, a->Wd2, a->Y, inner, c);
     if (s == RESBM_OK)
-        s = run_decode_bwd(d, a->dY, a->B, a->Wd1, a->Wd2, a->dB, a->dWd1, a->dWd2, inner, c);
+        s = run_decode_bwd(e, a->dY, a->B, Wd1, a->Wd2, a->dB, dWd1, a->dWd2, inner, c);
     if (s == RESBM_OK)
-        s = run_encode_bwd(d, a->dB, a->F, P, a->We1, a->We2, a->dF, a->dX, a->dWe1, a->dWe2,
-                           inner, c);
+        s = run_encode_bwd(e, a->dB, a->F, P, a->We1, We2, a->dF, a->dX, a->dWe1, dWe2, inner, c);
     return s;
 }
 

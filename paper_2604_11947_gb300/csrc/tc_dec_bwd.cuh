@@ -92,6 +92,9 @@ __global__ void __launch_bounds__(192, 1)
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nch = (int)(a.d / 128);
+    // every CTA walks the d chunks in the same cyclic order but from its own starting chunk,
+    // so that at any moment the CTAs read different column ranges of their rows
+    const int c_first = (int)(blockIdx.x % (unsigned)nch);
     int64_t start, end;
     token_range(a.T, blockIdx.x, gridDim.x, start, end);
     const int ntiles = (int)((end - start + 127) / 128);
@@ -166,6 +169,7 @@ __global__ void __launch_bounds__(192, 1)
                                 (int32_t)(start + 128 * (int64_t)i), smem_u32(&b_full));
                 ++b_issued;
                 for (int c = 0; c < nch && ok; ++c) {
+                    const int cc = c + c_first < nch ? c + c_first : c + c_first - nch;
                     // order: dY tile 0 of the chunk, the chunk's Wd2 slice, the other dY tiles.
                     // The MMA needs the slice before any tile of the chunk, so it must not queue
                     // behind tiles that wait for ring slots (that would deadlock), and it must not
@@ -177,7 +181,7 @@ __global__ void __launch_bounds__(192, 1)
                             const uint32_t dst = smem_u32(smem + C::OFF_W + s * C::W_STAGE);
                             mbar_expect_tx(smem_u32(&w_full[s]), C::W_STAGE);
                             for (int h = 0; h < 2; ++h)
-                                tma_load_2d(dst + h * (C::M * 128), &tm_wd2, c * 128 + 64 * h, 0, smem_u32(&w_full[s]));
+                                tma_load_2d(dst + h * (C::M * 128), &tm_wd2, cc * 128 + 64 * h, 0, smem_u32(&w_full[s]));
                             ++wit;
                         }
                         const int64_t t0 = start + 128 * (int64_t)i;
@@ -190,10 +194,10 @@ __global__ void __launch_bounds__(192, 1)
                         mbar_expect_tx(bar, valid == 128 ? C::Y_STAGE : (uint32_t)nb * 2u * 2048u);
                         for (int h = 0; h < 2; ++h) {
                             if (valid == 128) {
-                                tma_load_2d(dst + h * 16384, &tm_dy128, c * 128 + 64 * h, (int32_t)t0, bar);
+                                tma_load_2d(dst + h * 16384, &tm_dy128, cc * 128 + 64 * h, (int32_t)t0, bar);
                             } else {
                                 for (int rg = 0; rg < nb; ++rg)
-                                    tma_load_2d(dst + h * 16384 + rg * 2048, &tm_dy16, c * 128 + 64 * h,
+                                    tma_load_2d(dst + h * 16384 + rg * 2048, &tm_dy16, cc * 128 + 64 * h,
                                                 (int32_t)(t0 + 16 * rg), bar);
                             }
                         }
@@ -206,7 +210,7 @@ __global__ void __launch_bounds__(192, 1)
                         const uint32_t dst = smem_u32(smem + C::OFF_W + s * C::W_STAGE);
                         mbar_expect_tx(smem_u32(&w_full[s]), C::W_STAGE);
                         for (int h = 0; h < 2; ++h)
-                            tma_load_2d(dst + h * (C::M * 128), &tm_wd2, c * 128 + 64 * h, 0, smem_u32(&w_full[s]));
+                            tma_load_2d(dst + h * (C::M * 128), &tm_wd2, cc * 128 + 64 * h, 0, smem_u32(&w_full[s]));
                         ++wit;
                     }
                 }
@@ -380,6 +384,7 @@ __global__ void __launch_bounds__(192, 1)
 
             // ---- phase 1: drain each chunk's dWd2^T partial ----
             for (int c = 0; c < nch && ok; ++c, ++cit) {
+                const int cc = c + c_first < nch ? c + c_first : c + c_first - nch;
                 const uint32_t ab = cit & 1;
                 ok = mbar_wait(smem_u32(&wt_full[ab]), (cit >> 1) & 1);
                 tc_fence_after();
@@ -387,7 +392,7 @@ __global__ void __launch_bounds__(192, 1)
                 tmem_ld_row<C::M>(tmem + lane_base + C::TM_WT + ab * C::MS, v);
                 tc_fence_before();
                 mbar_arrive(smem_u32(&wt_empty[ab]));   // the accumulator is free again
-                wgrad_chunk<C::M>(a.wg, v, c, row, g == 0);
+                wgrad_chunk<C::M>(a.wg, v, cc, row, g == 0);
             }
 
             // ---- phase 2: dQ (hi + lo), then dB and the dWd1 partial ----

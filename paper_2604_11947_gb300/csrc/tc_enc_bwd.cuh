@@ -93,6 +93,9 @@ __global__ void __launch_bounds__(192, 1)
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nch = (int)(a.d / 128);
+    // every CTA walks the d chunks in the same cyclic order but from its own starting chunk,
+    // so that at any moment the CTAs read different column ranges of their rows
+    const int c_first = (int)(blockIdx.x % (unsigned)nch);
     int64_t start, end;
     token_range(a.T, blockIdx.x, gridDim.x, start, end);
     const int ntiles = (int)((end - start + 127) / 128);
@@ -161,6 +164,7 @@ __global__ void __launch_bounds__(192, 1)
                 bool p0_seen = false;
                 uint32_t j = 0;   // F stage of this group
                 for (int c = 0; c < nch && ok; ++c) {
+                    const int cc = c + c_first < nch ? c + c_first : c + c_first - nch;
                     // order: F tile 0 of the chunk, the chunk's We1 slice, the other F tiles.
                     // The MMA needs the slice before any tile of the chunk, so it must not queue
                     // behind tiles that wait for ring slots (that would deadlock), and it must not
@@ -170,7 +174,7 @@ __global__ void __launch_bounds__(192, 1)
                             const uint32_t s = wit % C::NW;
                             if (!mbar_wait(smem_u32(&w_empty[s]), ((wit / C::NW) & 1) ^ 1)) { ok = false; break; }
                             mbar_expect_tx(smem_u32(&w_full[s]), C::W_STAGE);
-                            tma_load_2d(smem_u32(smem + C::OFF_W + s * C::W_STAGE), &tm_we1, 0, c * 128,
+                            tma_load_2d(smem_u32(smem + C::OFF_W + s * C::W_STAGE), &tm_we1, 0, cc * 128,
                                         smem_u32(&w_full[s]));
                             ++wit;
                         }
@@ -190,10 +194,10 @@ __global__ void __launch_bounds__(192, 1)
                         mbar_expect_tx(bar, valid == 128 ? C::F_STAGE : (uint32_t)nb * 2u * 2048u);
                         for (int h = 0; h < 2; ++h) {
                             if (valid == 128) {
-                                tma_load_2d(dst + h * 16384, &tm_f128, c * 128 + 64 * h, (int32_t)t0, bar);
+                                tma_load_2d(dst + h * 16384, &tm_f128, cc * 128 + 64 * h, (int32_t)t0, bar);
                             } else {
                                 for (int rg = 0; rg < nb; ++rg)
-                                    tma_load_2d(dst + h * 16384 + rg * 2048, &tm_f16, c * 128 + 64 * h,
+                                    tma_load_2d(dst + h * 16384 + rg * 2048, &tm_f16, cc * 128 + 64 * h,
                                                 (int32_t)(t0 + 16 * rg), bar);
                             }
                         }
@@ -204,7 +208,7 @@ __global__ void __launch_bounds__(192, 1)
                         const uint32_t s = wit % C::NW;
                         if (!mbar_wait(smem_u32(&w_empty[s]), ((wit / C::NW) & 1) ^ 1)) { ok = false; break; }
                         mbar_expect_tx(smem_u32(&w_full[s]), C::W_STAGE);
-                        tma_load_2d(smem_u32(smem + C::OFF_W + s * C::W_STAGE), &tm_we1, 0, c * 128,
+                        tma_load_2d(smem_u32(smem + C::OFF_W + s * C::W_STAGE), &tm_we1, 0, cc * 128,
                                     smem_u32(&w_full[s]));
                         ++wit;
                     }
@@ -405,6 +409,7 @@ __global__ void __launch_bounds__(192, 1)
 
             // ---- phase 1: dF tiles out by TMA; dWe1 chunks to the partial slot ----
             for (int c = 0; c < nch && ok; ++c, ++cit) {
+                const int cc = c + c_first < nch ? c + c_first : c + c_first - nch;
                 for (int i = tb; i < te && ok; ++i, ++dfit) {
                     const int64_t t0 = start + 128 * (int64_t)i;
                     const int valid = (int)((end - t0) < 128 ? (end - t0) : 128);
@@ -443,7 +448,7 @@ __global__ void __launch_bounds__(192, 1)
                         fence_async_smem();
                         named_barrier(1, 128);
                         if (et == 0) {
-                            const int x = c * 128 + 64 * h;
+                            const int x = cc * 128 + 64 * h;
                             if (valid == 128) {
                                 tma_store_2d(&tm_df128, x, (int32_t)t0, smem_u32(stg));
                             } else {
@@ -462,7 +467,7 @@ __global__ void __launch_bounds__(192, 1)
                 tmem_ld_row<C::M>(tmem + lane_base + C::TM_WE + ae * C::MS, v);
                 tc_fence_before();
                 mbar_arrive(smem_u32(&we_empty[ae]));   // the accumulator is free again
-                wgrad_chunk<C::M>(a.wg, v, c, row, g == 0);
+                wgrad_chunk<C::M>(a.wg, v, cc, row, g == 0);
             }
 
             // ---- the group's dWe2 (rows = m, lanes 0 .. m-1) to its partial slot ----

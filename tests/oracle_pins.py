@@ -226,6 +226,80 @@ def pin_weight_grads_sum_over_tokens(o):
 
 
 # ---------------------------------------------------------------------------------------------
+# One linear layer per side (the single-matrix special case of the encoder / decoder).
+# ---------------------------------------------------------------------------------------------
+
+def pin_linear_is_plain_matrix_products(o):
+    """One linear layer per side against numpy's matmul, the textbook form of every output."""
+    T, d, r = 5, 9, 3
+    X, F, dY = _rand((T, d), 401), _rand((T, d), 402), _rand((T, d), 403)
+    We, Wd = _rand((d, r), 404, 0.3), _rand((r, d), 405, 0.3)
+    tol = dict(rtol=1e-12, atol=1e-12)
+    B = o.linear_encode_fwd(X, F, We)
+    np.testing.assert_allclose(B, X[:, :r] + F @ We, **tol)
+    for merge in (0, 1):
+        pad = np.hstack([B, np.zeros((T, d - r))]) * merge
+        np.testing.assert_allclose(o.linear_decode_fwd(B, Wd, merge), pad + B @ Wd, **tol)
+        dB, dWd = o.linear_decode_bwd(dY, B, Wd, merge)
+        np.testing.assert_allclose(dB, merge * dY[:, :r] + dY @ Wd.T, **tol)
+        np.testing.assert_allclose(dWd, B.T @ dY, **tol)
+    dBup = _rand((T, r), 406)
+    dF, dX, dWe = o.linear_encode_bwd(dBup, F, We)
+    np.testing.assert_allclose(dF, dBup @ We.T, **tol)
+    np.testing.assert_allclose(dWe, F.T @ dBup, **tol)
+    np.testing.assert_allclose(dX, np.hstack([dBup, np.zeros((T, d - r))]), **tol)
+
+
+def pin_linear_is_two_layer_form_with_identity_second_layers(o):
+    """The two independent code paths agree: one linear layer per side equals the two-layer
+    form with phi = identity and identity matrices as the second layers (We2 = Wd1 = I_r)."""
+    T, d, r = 6, 8, 3
+    X, F, dY = _rand((T, d), 411), _rand((T, d), 412), _rand((T, d), 413)
+    We, Wd = _rand((d, r), 414, 0.3), _rand((r, d), 415, 0.3)
+    I = np.eye(r)
+    a = o.linear_boundary_step(X, F, dY, We, Wd, merge=1)
+    b = o.boundary_step(X, F, dY, We, I, I, Wd, act="identity", merge=1)
+    for k in ("B", "Y", "dB", "dF", "dX", "dWe1", "dWd2"):
+        np.testing.assert_allclose(a[k], b[k], rtol=1e-12, atol=1e-12, err_msg=k)
+
+
+def pin_linear_gradients_match_finite_differences(o):
+    T, d, r = 3, 7, 2
+    X, F, dY = _rand((T, d), 421), _rand((T, d), 422), _rand((T, d), 423)
+    params = dict(X=X, F=F, We=_rand((d, r), 424, 0.3), Wd=_rand((r, d), 425, 0.3))
+    for merge in (1, 0):
+        def loss(p):
+            B = o.linear_encode_fwd(p["X"], p["F"], p["We"])
+            return float(np.sum(dY * o.linear_decode_fwd(B, p["Wd"], merge)))
+
+        B = o.linear_encode_fwd(X, F, params["We"])
+        dB, dWd = o.linear_decode_bwd(dY, B, params["Wd"], merge)
+        dF, dX, dWe = o.linear_encode_bwd(dB, F, params["We"])
+        grads = dict(X=dX, F=dF, We=dWe, Wd=dWd)
+        for name, g in grads.items():
+            scale = max(1.0, float(np.max(np.abs(g))))
+            for idx in np.ndindex(*g.shape):
+                p = {k: v.copy() for k, v in params.items()}
+                x0 = p[name][idx]
+                h = 1e-6 * max(1.0, abs(x0))
+                p[name][idx] = x0 + h
+                lp = loss(p)
+                p[name][idx] = x0 - h
+                lm = loss(p)
+                assert abs((lp - lm) / (2 * h) - g[idx]) <= 1e-7 * scale, (merge, name, idx)
+
+
+def pin_linear_zero_weights_leave_identity_path(o):
+    T, d, r = 4, 6, 2
+    X, F, dY = _rand((T, d), 431), _rand((T, d), 432), _rand((T, d), 433)
+    z = o.linear_boundary_step(X, F, dY, np.zeros((d, r)), np.zeros((r, d)), merge=1)
+    np.testing.assert_array_equal(z["B"], X[:, :r])
+    np.testing.assert_array_equal(z["Y"], np.hstack([X[:, :r], np.zeros((T, d - r))]))
+    np.testing.assert_array_equal(z["dB"], dY[:, :r])
+    np.testing.assert_array_equal(z["dF"], np.zeros((T, d)))
+
+
+# ---------------------------------------------------------------------------------------------
 # Transfer rounding of B and dB (they cross the boundary in bf16, Appendix A.3).
 # ---------------------------------------------------------------------------------------------
 

@@ -135,3 +135,20 @@ def test_step_rejects_output_aliasing_input(lib):
     st = lib.resbm_boundary_step(ctypes.byref(d), ctypes.byref(args), 1 << 40, need, None)
     assert st == resbm.RESBM_ERR_INVALID_ARG
     assert lib.resbm_boundary_step(ctypes.byref(d), None, 1 << 40, need, None) == resbm.RESBM_ERR_INVALID_ARG
+
+
+def test_linear_flag_rules(lib):
+    """RESBM_FLAG_LINEAR needs m == r; its second-layer tensors may be absent."""
+    big = 1 << 32
+    A = 1 << 40
+    bad = resbm.make_desc(16, 64, 8, 4, flags=resbm.RESBM_FLAG_LINEAR)
+    assert lib.resbm_decode_fwd(ctypes.byref(bad), A, None, A + big, A + 2 * big, A + 3 * big, big, None) \
+        == resbm.RESBM_ERR_INVALID_ARG
+    ok = resbm.make_desc(16, 64, 8, 8, flags=resbm.RESBM_FLAG_LINEAR)
+    # without the flag a missing Wd1 is an argument error; with it, only the workspace is missing
+    plain = resbm.make_desc(16, 64, 8, 8)
+    assert lib.resbm_decode_fwd(ctypes.byref(plain), A, None, A + big, A + 2 * big, None, 0, None) \
+        == resbm.RESBM_ERR_INVALID_ARG
+    assert lib.resbm_decode_fwd(ctypes.byref(ok), A, None, A + big, A + 2 * big, None, 0, None) \
+        == resbm.RESBM_ERR_WORKSPACE
+    assert resbm.resbm_workspace_bytes(ok, resbm.RESBM_OP_DECODE_FWD) > 0

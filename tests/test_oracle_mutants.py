@@ -34,6 +34,9 @@ MUTANTS = {
     "rounding_ties_away_from_zero": ("double r = nearbyint(scaled);", "double r = round(scaled);"),
     "rounding_keeps_one_bit_less": ("double scaled = ldexp(f, bits);",
                                     "double scaled = ldexp(f, bits - 1);"),
+    "linear_decoder_bwd_transposed": ("mm_nt(T, r, d, dY, Wd, dB);              /* dB  = dY . Wd^T         */",
+                                      "mm_nn(T, r, d, dY, Wd, dB);              /* dB  = dY . Wd^T         */"),
+    "linear_encoder_bwd_drops_dX": ("return dX ? pid_backward(T, d, r, dB, dX) : 0;", "return 0;"),
 }
 
 

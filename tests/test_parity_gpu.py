@@ -286,3 +286,85 @@ def test_runs_on_a_side_stream():
 def test_no_kernel_reported_a_timeout():
     """The tensor-core kernels' bounded waits never gave up during this test session."""
     assert resbm.resbm_device_error() == 0
+
+
+# ---------------------------------------------------------------------------------------------
+# One linear layer per side (RESBM_FLAG_LINEAR): We1 is d x r, Wd2 is r x d, no We2 / Wd1.
+# ---------------------------------------------------------------------------------------------
+
+LINEAR = {
+    "bf16_r32": synth.BoundaryConfig("lin_bf16", T=1000, d=512, r=32, m=32),
+    "bf16_r16_merge0": synth.BoundaryConfig("lin_bf16_m0", T=777, d=384, r=16, m=16, merge=0),
+    "f32_r8": synth.BoundaryConfig("lin_f32", T=333, d=200, r=8, m=8, dtype="f32"),
+}
+
+
+@pytest.mark.parametrize("path", PATHS)
+@pytest.mark.parametrize("name", LINEAR)
+def test_linear_mode_matches_oracle(name, path):
+    cfg = LINEAR[name]
+    flags = PATHS[path] | resbm.RESBM_FLAG_LINEAR
+    desc = resbm.desc_from_config(cfg, flags)
+    T, d, r = cfg.T, cfg.d, cfg.r
+    h = host_inputs(cfg, ("X", "F", "dY", "We1", "Wd2"))
+    dev = {k: to_dev(v, cfg) for k, v in h.items()}
+    io = torch.bfloat16 if cfg.dtype == "bf16" else torch.float32
+    want = oracle.linear_boundary_step(h["X"], h["F"], h["dY"], h["We1"], h["Wd2"], cfg.merge,
+                                       transfer=cfg.dtype)
+    # the whole step through the C ABI (second-layer tensors absent)
+    out = dict(B=torch.empty(T, r, dtype=io, device="cuda"), Y=torch.empty(T, d, dtype=io, device="cuda"),
+               dB=torch.empty(T, r, dtype=io, device="cuda"), dF=torch.empty(T, d, dtype=io, device="cuda"),
+               dX=torch.zeros(T, d, dtype=io, device="cuda"), dWe1=torch.empty(d, r, device="cuda"),
+               dWd2=torch.empty(r, d, device="cuda"))
+    ws = resbm.workspace(desc, resbm.RESBM_OP_BOUNDARY_STEP)
+    resbm.resbm_boundary_step(desc, ws, X=dev["X"], F=dev["F"], dY=dev["dY"], We1=dev["We1"],
+                              Wd2=dev["Wd2"], **out)
+    torch.cuda.synchronize()
+    for k in ("B", "dB"):
+        check_output(k, out[k], want[k], cfg)
+    # each later stage on the oracle's transferred tensor, against the oracle
+    B = to_dev(want["B"], cfg)
+    Y = torch.empty_like(out["Y"])
+    resbm.resbm_decode_fwd(desc, B, None, dev["Wd2"], Y, resbm.workspace(desc, resbm.RESBM_OP_DECODE_FWD))
+    dB = torch.empty_like(out["dB"])
+    dWd2 = torch.empty_like(out["dWd2"])
+    resbm.resbm_decode_bwd(desc, dev["dY"], B, None, dev["Wd2"], dB, None, dWd2,
+                           resbm.workspace(desc, resbm.RESBM_OP_DECODE_BWD))
+    dF = torch.empty_like(out["dF"])
+    dX = torch.zeros_like(out["dX"])
+    dWe1 = torch.empty_like(out["dWe1"])
+    resbm.resbm_encode_bwd(desc, to_dev(want["dB"], cfg), dev["F"], None, dev["We1"], None, dF, dX,
+                           dWe1, None, resbm.workspace(desc, resbm.RESBM_OP_ENCODE_BWD))
+    torch.cuda.synchronize()
+    for k, v in dict(Y=Y, dB=dB, dWd2=dWd2, dF=dF, dX=dX, dWe1=dWe1).items():
+        check_output(k, v, want[k], cfg)
+    # the step is its own stages, bit for bit
+    resbm.resbm_decode_fwd(desc, out["B"], None, dev["Wd2"], Y, resbm.workspace(desc, resbm.RESBM_OP_DECODE_FWD))
+    resbm.resbm_decode_bwd(desc, dev["dY"], out["B"], None, dev["Wd2"], dB, None, dWd2,
+                           resbm.workspace(desc, resbm.RESBM_OP_DECODE_BWD))
+    dX.zero_()
+    resbm.resbm_encode_bwd(desc, out["dB"], dev["F"], None, dev["We1"], None, dF, dX, dWe1, None,
+                           resbm.workspace(desc, resbm.RESBM_OP_ENCODE_BWD))
+    torch.cuda.synchronize()
+    for k, v in dict(Y=Y, dB=dB, dWd2=dWd2, dF=dF, dX=dX, dWe1=dWe1).items():
+        assert torch.equal(v, out[k]), k
+
+
+def test_linear_zero_weights_give_identity_path_bitwise():
+    cfg = synth.BoundaryConfig("lin_zero", T=300, d=256, r=16, m=16)
+    desc = resbm.desc_from_config(cfg, resbm.RESBM_FLAG_LINEAR)
+    h = host_inputs(cfg, ("X", "F", "dY"))
+    dev = {k: to_dev(v, cfg) for k, v in h.items()}
+    T, d, r = cfg.T, cfg.d, cfg.r
+    bf = torch.bfloat16
+    zero_e, zero_d = torch.zeros(d, r, dtype=bf, device="cuda"), torch.zeros(r, d, dtype=bf, device="cuda")
+    out = dict(B=torch.empty(T, r, dtype=bf, device="cuda"), Y=torch.empty(T, d, dtype=bf, device="cuda"),
+               dB=torch.empty(T, r, dtype=bf, device="cuda"), dF=torch.empty(T, d, dtype=bf, device="cuda"),
+               dWe1=torch.empty(d, r, device="cuda"), dWd2=torch.empty(r, d, device="cuda"))
+    resbm.resbm_boundary_step(desc, resbm.workspace(desc, resbm.RESBM_OP_BOUNDARY_STEP), X=dev["X"],
+                              F=dev["F"], dY=dev["dY"], We1=zero_e, Wd2=zero_d, **out)
+    torch.cuda.synchronize()
+    assert torch.equal(out["B"], dev["X"][:, :r])
+    assert torch.equal(out["Y"][:, :r], out["B"]) and not torch.any(out["Y"][:, r:])
+    assert torch.equal(out["dB"], dev["dY"][:, :r])
+    assert not torch.any(out["dF"])
