@@ -194,13 +194,22 @@ def oracle_rate(cfg, budget_s):
     return n, t
 
 
-def cpu_baseline(cfg, budget_s=15.0):
+def cpu_baseline(cfg, budget_s=15.0, one_core_budget_s=5.0):
+    """The oracle on all host cores (OpenMP) and on one core, each on a bounded token sample."""
     import oracle
+    cores = oracle.max_threads()
     n, t = oracle_rate(cfg, budget_s)
-    return {"value": n / t, "unit": "tokens/s", "cores": oracle.max_threads(), "kind": "oracle",
+    oracle.set_threads(1)
+    try:
+        n1, t1 = oracle_rate(cfg, one_core_budget_s)
+    finally:
+        oracle.set_threads(cores)
+    return {"value": n / t, "unit": "tokens/s", "cores": cores, "kind": "oracle",
             "sample": "fp64 oracle boundary step (encode fwd, decode fwd, decode bwd, encode bwd, "
                       "weight gradients over the sample) on tokens 0..%d of the %s workload, "
-                      "%.2f s" % (n - 1, cfg.name, t)}
+                      "%.2f s on %d threads" % (n - 1, cfg.name, t, cores),
+            "one_core": {"value": n1 / t1, "unit": "tokens/s", "cores": 1,
+                         "sample": "tokens 0..%d, %.2f s" % (n1 - 1, t1)}}
 
 
 def describe(cfg, extra=None):
@@ -241,6 +250,22 @@ def run_reference(args, cfg, rank):
             "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
+
+
+# ---- multi-rank host logic (one independent replica per GPU) --------------------------------
+def max_over_ranks(ms, dist, device):
+    """The slowest rank's time: every rank gets the maximum of all ranks' `ms`."""
+    if not dist:
+        return ms
+    import torch
+    t = torch.tensor([float(ms)], device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(tokens_per_rank, world, steps, ms_total):
+    """Whole-job tokens/s: the tokens all ranks processed over the slowest rank's time."""
+    return tokens_per_rank * world * steps / (ms_total / 1e3)
 
 
 # ---- the GPU arm ----------------------------------------------------------------------------
@@ -323,13 +348,9 @@ def main():
     if dist:
         dist.barrier()
     clk = clocks.stop()
-    ms_total = start.elapsed_time(end)
-    if dist:
-        t = torch.tensor([ms_total], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms_total = float(t.item())
+    ms_total = max_over_ranks(start.elapsed_time(end), dist, "cuda")
     ms_step = ms_total / max(args.steps, 1)
-    value = cfg.T * world * args.steps / (ms_total / 1e3)
+    value = job_throughput(cfg.T, world, args.steps, ms_total)
 
     op_ms = {op: statistics.mean(evs[i][j].elapsed_time(evs[i][j + 1]) for i in range(args.steps))
              for j, op in enumerate(OPS)}
@@ -421,12 +442,8 @@ def run_e2e(args, cfg, desc, dev, out, ws, resbm, torch, dist, world):
     for i in range(n):
         step(i)
     torch.cuda.synchronize()
-    ms = (time.perf_counter() - t0) * 1e3
-    if dist:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
-    return {"value": cfg.T * world * n / (ms / 1e3), "unit": "tokens/s",
+    ms = max_over_ranks((time.perf_counter() - t0) * 1e3, dist, "cuda")
+    return {"value": job_throughput(cfg.T, world, n, ms), "unit": "tokens/s",
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": n,
             "ms_per_step": ms / n,
             "pipelined": "H2D, compute and D2H on three streams, two device buffer sets; "

@@ -30,6 +30,7 @@ _i64 = ctypes.c_int64
 def _load(path=None):
     lib = ctypes.CDLL(path or _build.build())
     lib.oracle_max_threads.restype = ctypes.c_int
+    lib.oracle_set_threads.argtypes = [ctypes.c_int]
     lib.oracle_act.restype = ctypes.c_double
     lib.oracle_act.argtypes = [ctypes.c_int, ctypes.c_double]
     lib.oracle_dact.restype = ctypes.c_double
@@ -92,6 +93,10 @@ class Oracle:
 
     def max_threads(self):
         return int(self._l.oracle_max_threads())
+
+    def set_threads(self, n):
+        """OpenMP threads of later calls (the results do not depend on it)."""
+        self._l.oracle_set_threads(int(n))
 
     # -- transfer rounding (Appendix A.3: the boundary tensors travel in bf16) ----------------
     _BITS = {"bf16": 8, "f32": 24}
@@ -274,7 +279,7 @@ def default():
 def __getattr__(name):
     # module-level shortcuts: oracle.encode_fwd(...) etc.
     if name in ("act", "dact", "rect_identity", "pid", "encode_fwd", "decode_fwd", "round_to",
-                "decode_bwd", "encode_bwd", "boundary_step", "max_threads", "linear_encode_fwd",
+                "decode_bwd", "encode_bwd", "boundary_step", "max_threads", "set_threads", "linear_encode_fwd",
                 "linear_decode_fwd", "linear_decode_bwd", "linear_encode_bwd",
                 "linear_boundary_step"):
         return getattr(default(), name)

@@ -58,6 +58,16 @@ int oracle_max_threads(void)
 #endif
 }
 
+/* Number of OpenMP threads later calls use (results do not depend on it). */
+void oracle_set_threads(int n)
+{
+#ifdef _OPENMP
+    if (n > 0) omp_set_num_threads(n);
+#else
+    (void)n;
+#endif
+}
+
 /* ------------------------------------------------------------------------------------------ */
 /* Nonlinearity phi and its derivative (Sec. 3.2: "a non-linearity applied between them").      */
 /* SiLU: x * sigmoid(x).  GELU(tanh form): 0.5 x (1 + tanh(sqrt(2/pi) (x + 0.044715 x^3))).      */
