@@ -141,5 +141,10 @@ template <int N> __device__ __forceinline__ void act_dact_row(int act, const flo
 {
     RESBM_ACT_ROW_LOOP(act, act_and_dact(kAct, x[j], a[j], d[j]));
 }
+// a = phi(x), d = phi'(x), fast
+template <int N> __device__ __forceinline__ void act_dact_fast_row(int act, const float (&x)[N], float (&a)[N], float (&d)[N])
+{
+    RESBM_ACT_ROW_LOOP(act, (a[j] = act_fast(kAct, x[j]), d[j] = dact_fast(kAct, x[j])));
+}
 
 }  // namespace resbm

@@ -9,6 +9,7 @@
 
 #include <atomic>
 #include <mutex>
+#include <utility>
 
 #include "tc.h"
 #include "tc_common.cuh"
@@ -53,6 +54,27 @@ bool make_map(CUtensorMap *m, const void *ptr, uint64_t inner, uint64_t outer, u
 
 bool al16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
+// Every kernel of this file is launched with programmatic stream serialization: it may be
+// scheduled while the previous kernel of the stream is still finishing, and waits at its start
+// (griddepcontrol.wait, before touching global memory) until that kernel has completed and its
+// writes are visible. What overlaps is the launch itself and the placement of CTAs on SMs that
+// the previous kernel has already left.
+template <typename... KArgs, typename... Args>
+cudaError_t launch(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream, Args &&...args)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
 // Dynamic shared memory attribute, set once per (kernel, device): `done` is the calling
 // launcher's own per-device flag array (one per kernel instantiation).
 constexpr int kMaxDev = 64;
@@ -89,9 +111,9 @@ cudaError_t launch_dec_fwd(const resbm_desc &d, const void *B, const void *Wd1, 
     if (e != cudaSuccess) return e;
     tc::DecFwdArgs a{static_cast<const __nv_bfloat16 *>(B), static_cast<const __nv_bfloat16 *>(Wd1), d.T, d.d,
                      d.act, d.merge_identity};
-    tc::k_dec_fwd<M><<<grid_tokens(c, d.T), Cfg::THREADS, Cfg::SMEM_BYTES, c.stream>>>(m_wd2, m_y128, m_y16, a);
+    e = launch(tc::k_dec_fwd<M>, grid_tokens(c, d.T), Cfg::THREADS, Cfg::SMEM_BYTES, c.stream, m_wd2, m_y128, m_y16, a);
     count_launches(1);
-    return cudaGetLastError();
+    return e;
 }
 
 template <int M>
@@ -112,9 +134,9 @@ cudaError_t launch_enc_fwd(const resbm_desc &d, const void *X, const void *F, co
     if (e != cudaSuccess) return e;
     tc::EncFwdArgs a{static_cast<const __nv_bfloat16 *>(X), static_cast<const __nv_bfloat16 *>(We2),
                      static_cast<__nv_bfloat16 *>(B), P, d.T, d.d, d.act};
-    tc::k_enc_fwd<M><<<grid_tokens(c, d.T), Cfg::THREADS, Cfg::SMEM_BYTES, c.stream>>>(m_f128, m_f16, m_we1, a);
+    e = launch(tc::k_enc_fwd<M>, grid_tokens(c, d.T), Cfg::THREADS, Cfg::SMEM_BYTES, c.stream, m_f128, m_f16, m_we1, a);
     count_launches(1);
-    return cudaGetLastError();
+    return e;
 }
 
 // Scratch layout of the backward kernels: the d x m weight gradient has one fp32 slot per CTA
@@ -163,9 +185,9 @@ cudaError_t launch_reduce(const tc::ReduceJob &small, tc::ReduceJob big, const C
     const int64_t resident = (int64_t)c.sm_count * 8;
     const int64_t left = resident - small.blocks;
     if (big.blocks > left && left >= 1) big.blocks = (int)left;
-    tc::k_reduce_slots<<<small.blocks + big.blocks, kReduceBlock, 0, c.stream>>>(small, big);
+    const cudaError_t e = launch(tc::k_reduce_slots, small.blocks + big.blocks, kReduceBlock, 0, c.stream, small, big);
     count_launches(1);
-    return cudaGetLastError();
+    return e;
 }
 
 CUtensorMapSwizzle swizzle_for(uint32_t row_bytes)
@@ -195,9 +217,9 @@ cudaError_t launch_dec_bwd(const resbm_desc &d, const void *dY, const void *B, c
                      static_cast<__nv_bfloat16 *>(dB),
                      tc::WgradArgs{p.part_big, p.nch},
                      p.part_small, d.T, d.d, d.act, d.merge_identity, p.max_groups};
-    tc::k_dec_bwd<M><<<p.grid, Cfg::THREADS, Cfg::SMEM_BYTES, c.stream>>>(m_dy128, m_dy16, m_wd2, m_b, m_yr, a);
+    e = launch(tc::k_dec_bwd<M>, p.grid, Cfg::THREADS, Cfg::SMEM_BYTES, c.stream, m_dy128, m_dy16, m_wd2, m_b, m_yr, a);
     count_launches(1);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if (e != cudaSuccess) return e;
     // dWd2 (m x d) = sum of the per-CTA slots (d x m), transposed; dWd1 (r x m) = sum of the slices
     const int64_t cap = (int64_t)c.sm_count * 8;
     return launch_reduce(reduce_job(p.part_small, p.slots, d.r, d.m, dWd1, 0, al16(dWd1), cap),
@@ -254,10 +276,10 @@ cudaError_t launch_enc_bwd(const resbm_desc &d, const void *dB, const void *F, c
     if (e != cudaSuccess) return e;
     tc::EncBwdArgs a{P, static_cast<const __nv_bfloat16 *>(We2), static_cast<__nv_bfloat16 *>(dX),
                      tc::WgradArgs{p.part_big, p.nch}, p.part_small, d.T, d.d, d.act, p.max_groups};
-    tc::k_enc_bwd<M><<<p.grid, Cfg::THREADS, Cfg::SMEM_BYTES, c.stream>>>(m_f128, m_f16, m_we1, m_df128, m_df16,
-                                                                          m_db, a);
+    e = launch(tc::k_enc_bwd<M>, p.grid, Cfg::THREADS, Cfg::SMEM_BYTES, c.stream, m_f128, m_f16, m_we1, m_df128,
+               m_df16, m_db, a);
     count_launches(1);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if (e != cudaSuccess) return e;
     const int64_t cap = (int64_t)c.sm_count * 8;
     return launch_reduce(reduce_job(p.part_small, p.slots, d.m, d.r, dWe2, 0, al16(dWe2), cap),
                          reduce_job(p.part_big, p.grid, d.d, d.m, dWe1, 0, al16(dWe1), cap), c);

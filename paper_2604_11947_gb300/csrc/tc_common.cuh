@@ -37,6 +37,18 @@ __device__ __forceinline__ unsigned long long globaltimer()
     return t;
 }
 
+// Programmatic dependent launch: wait until the previous kernel of the stream has completed and
+// its memory is visible (a no-op when the launch had no programmatic dependency), and let the
+// next kernel be scheduled now (it waits the same way before it touches memory).
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void griddep_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+// Fetch the 128-byte line holding p into L2 (no register result, no wait).
+__device__ __forceinline__ void prefetch_l2(const void *p)
+{
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
+}
+
 __device__ __forceinline__ void flag_error(unsigned code)
 {
     atomicOr(&g_resbm_device_error, code);

@@ -83,6 +83,8 @@ __global__ void __launch_bounds__(192, 1)
               const __grid_constant__ CUtensorMap tm_yr, const DecBwdArgs a)
 {
     using C = DecBwdCfg<M_>;
+    griddep_wait();               // the previous kernel of the stream has completed
+    griddep_launch_dependents();  // the next one may be scheduled on SMs as they free up
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     __shared__ uint64_t y_full[C::NSY], y_empty[C::NSY], w_full[C::NW], w_empty[C::NW];
@@ -553,6 +555,8 @@ __device__ __forceinline__ void reduce_job(const ReduceJob &j, int64_t block, in
 __global__ void __launch_bounds__(32 * kSlotGroups) k_reduce_slots(const ReduceJob first, const ReduceJob second)
 {
     __shared__ float4 grp[kSlotGroups][32];
+    griddep_wait();
+    griddep_launch_dependents();
     if ((int)blockIdx.x < first.blocks)
         reduce_job(first, blockIdx.x, first.blocks, grp);
     else

@@ -84,6 +84,8 @@ __global__ void __launch_bounds__(192, 1)
               const EncBwdArgs a)
 {
     using C = EncBwdCfg<M_>;
+    griddep_wait();               // the previous kernel of the stream has completed
+    griddep_launch_dependents();  // the next one may be scheduled on SMs as they free up
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     __shared__ uint64_t f_full[C::NSF], f_empty[C::NSF], w_full[C::NW], w_empty[C::NW];
@@ -340,6 +342,16 @@ __global__ void __launch_bounds__(192, 1)
             const int tb = g * C::NT, te = min(ntiles, tb + C::NT);
             const int64_t slot = (int64_t)blockIdx.x * a.max_groups + g;
             // ---- phase 0: dP and A = phi(P) of every tile, dX[:, :r] += dB ----
+            // the group's P rows and dX[:, :r] rows towards L2 first, so that the per-tile loads
+            // below do not each wait for DRAM
+            for (int i = tb; i < te; ++i) {
+                const int64_t tok = start + 128 * (int64_t)i + row;
+                if (tok < end) {
+                    prefetch_l2(a.P + tok * C::M);
+                    if (C::M * 4 > 128) prefetch_l2(a.P + tok * C::M + 32);
+                    if (a.dX) prefetch_l2(a.dX + tok * a.d);
+                }
+            }
             ok = mbar_wait(smem_u32(&db_full), g & 1);
             for (int i = tb; i < te; ++i, ++u) {
                 const int64_t t0 = start + 128 * (int64_t)i;
@@ -369,7 +381,7 @@ __global__ void __launch_bounds__(192, 1)
                 tc_fence_before();
                 mbar_arrive(smem_u32(&da_empty[rg]));   // the dA region is free again
                 float av[C::M], dph[C::M];
-                act_dact_row<C::M>(a.act, pv, av, dph);
+                act_dact_fast_row<C::M>(a.act, pv, av, dph);
 #pragma unroll
                 for (int jj = 0; jj < C::M; ++jj) {
                     const float x = active ? da[jj] * dph[jj] : 0.0f;

@@ -49,6 +49,8 @@ __global__ void __launch_bounds__(192, 1)
               const __grid_constant__ CUtensorMap tm_we1, const EncFwdArgs a)
 {
     using C = EncFwdCfg<M_>;
+    griddep_wait();               // the previous kernel of the stream has completed
+    griddep_launch_dependents();  // the next one may be scheduled on SMs as they free up
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     __shared__ uint64_t full[C::NSTAGE], empty[C::NSTAGE];
