@@ -52,6 +52,13 @@ bool make_map(CUtensorMap *m, const void *ptr, uint64_t inner, uint64_t outer, u
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+CUtensorMapSwizzle swizzle_for(uint32_t row_bytes)
+{
+    return row_bytes == 128 ? CU_TENSOR_MAP_SWIZZLE_128B
+           : row_bytes == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
+                             : CU_TENSOR_MAP_SWIZZLE_32B;
+}
+
 bool al16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 // Every kernel of this file is launched with programmatic stream serialization: it may be
@@ -101,17 +108,18 @@ cudaError_t launch_dec_fwd(const resbm_desc &d, const void *B, const void *Wd1, 
                            const Ctx &c)
 {
     using Cfg = tc::DecFwdCfg<M>;
-    CUtensorMap m_wd2, m_y128, m_y16;
+    CUtensorMap m_wd2, m_y128, m_y16, m_b;
     if (!make_map(&m_wd2, Wd2, d.d, d.m, d.d * 2, 64, M, CU_TENSOR_MAP_SWIZZLE_128B) ||
         !make_map(&m_y128, Y, d.d, d.T, d.d * 2, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !make_map(&m_y16, Y, d.d, d.T, d.d * 2, 64, 16, CU_TENSOR_MAP_SWIZZLE_128B))
+        !make_map(&m_y16, Y, d.d, d.T, d.d * 2, 64, 16, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&m_b, B, d.r, d.T, d.r * 2, Cfg::GB / 2, 128, swizzle_for(Cfg::GB)))
         return cudaErrorInvalidValue;
     static std::atomic<uint8_t> smem_set[kMaxDev];
     cudaError_t e = ensure_smem(tc::k_dec_fwd<M>, Cfg::SMEM_BYTES, c.device, smem_set);
     if (e != cudaSuccess) return e;
-    tc::DecFwdArgs a{static_cast<const __nv_bfloat16 *>(B), static_cast<const __nv_bfloat16 *>(Wd1), d.T, d.d,
-                     d.act, d.merge_identity};
-    e = launch(tc::k_dec_fwd<M>, grid_tokens(c, d.T), Cfg::THREADS, Cfg::SMEM_BYTES, c.stream, m_wd2, m_y128, m_y16, a);
+    tc::DecFwdArgs a{static_cast<const __nv_bfloat16 *>(Wd1), d.T, d.d, d.act, d.merge_identity};
+    e = launch(tc::k_dec_fwd<M>, grid_tokens(c, d.T), Cfg::THREADS, Cfg::SMEM_BYTES, c.stream, m_wd2, m_y128, m_y16,
+               m_b, a);
     count_launches(1);
     return e;
 }
@@ -190,12 +198,6 @@ cudaError_t launch_reduce(const tc::ReduceJob &small, tc::ReduceJob big, const C
     return e;
 }
 
-CUtensorMapSwizzle swizzle_for(uint32_t row_bytes)
-{
-    return row_bytes == 128 ? CU_TENSOR_MAP_SWIZZLE_128B
-           : row_bytes == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
-                             : CU_TENSOR_MAP_SWIZZLE_32B;
-}
 
 template <int M>
 cudaError_t launch_dec_bwd(const resbm_desc &d, const void *dY, const void *B, const void *Wd1, const void *Wd2,

@@ -3,12 +3,12 @@
 //
 // Persistent CTAs; CTA b owns a contiguous token range (16-token aligned, balanced to within
 // 16 tokens) and walks it in tiles of up to 128 tokens. Per tile:
-//   epilogue warps : Q = B . Wd1 on CUDA cores (fp32), G = phi(Q) -> bf16 -> shared memory
-//                    (the MMA A operand, K-major, 128B swizzle)
-//   producer warp  : Wd2 column chunks (m x NCH, MN-major B operand) by TMA into a ring
-//   MMA warp       : D_chunk (128 x NCH fp32, TMEM, double-buffered) = G . Wd2_chunk
-//   epilogue warps : TMEM -> registers, + B on the first r columns, -> bf16 -> swizzled staging
-//                    -> TMA store of Y (boxes of 128 rows, or 16 rows for a partial tile)
+//   producer warp  : the tile's B rows by TMA; Wd2 column chunks (m x NCH, MN-major) into a ring
+//   MMA warp       : Q = B . Wd1 into the next free accumulator, then per chunk
+//                    D_chunk (128 x NCH fp32, TMEM, double-buffered) = G . Wd2_chunk
+//   epilogue warps : G = phi(Q) -> bf16 -> shared memory (the A operand, K-major), then per
+//                    chunk TMEM -> registers, + B on the first r columns, -> bf16 -> swizzled
+//                    staging -> TMA store of Y (boxes of 128 rows, or 16 rows for a partial tile)
 // HBM traffic per token: read B (2r bytes), write Y (2d bytes); Wd2 is re-read from L2.
 #pragma once
 
@@ -23,32 +23,40 @@ template <int M_> struct DecFwdCfg {
     static constexpr int R = M_;                       // bottleneck width r
     static constexpr int NCH = M_ <= 32 ? 256 : 128;   // Y columns per MMA chunk
     static constexpr int NSTAGE = M_ <= 64 ? 3 : 2;    // Wd2 chunk ring depth
-    static constexpr int KBLK = (M_ + 63) / 64;        // 64-wide K blocks of G
+    static constexpr uint32_t GB = M_ * 2 < 128 ? M_ * 2 : 128;   // row bytes (= swizzle) of a 128-row block
+    static constexpr int NB = M_ * 2 / GB;             // such blocks across the r (or m) columns
+    static constexpr int SPB = GB / 32;                // 16-element K steps per block
     static constexpr uint32_t W_STAGE_BYTES = M_ * NCH * 2;
-    static constexpr uint32_t G_BYTES = KBLK * 128 * 128;
+    static constexpr uint32_t TILE_BYTES = 128 * M_ * 2;   // 128 tokens x r (or m) bf16, NB blocks
     static constexpr uint32_t STG_BYTES = 128 * NCH * 2;
-    static constexpr uint32_t WD1_BYTES = R * M_ * 2;
+    static constexpr uint32_t WD1T_BYTES = R * M_ * 2;
     // shared-memory map (offsets from a 1024-aligned base)
     static constexpr uint32_t OFF_W = 0;
-    static constexpr uint32_t OFF_G = OFF_W + NSTAGE * W_STAGE_BYTES;
-    static constexpr uint32_t OFF_STG = OFF_G + 2 * G_BYTES;
-    static constexpr uint32_t OFF_WD1 = OFF_STG + 2 * STG_BYTES;
-    static constexpr uint32_t SMEM_BYTES = OFF_WD1 + WD1_BYTES + 1024;  // + alignment slack
+    static constexpr uint32_t OFF_G = OFF_W + NSTAGE * W_STAGE_BYTES;   // G tile [token][m]
+    static constexpr uint32_t OFF_B = OFF_G + TILE_BYTES;                // B tile [token][r] (TMA)
+    static constexpr uint32_t OFF_STG = OFF_B + TILE_BYTES;
+    static constexpr uint32_t OFF_WD1T = OFF_STG + 2 * STG_BYTES;       // Wd1^T [m][r], K-major
+    static constexpr uint32_t SMEM_BYTES = OFF_WD1T + WD1T_BYTES + 1024;  // + alignment slack
+    static_assert(SMEM_BYTES <= 232448 - 512, "shared memory budget");
     static constexpr uint32_t TMEM_COLS = 2 * NCH;
     static constexpr int THREADS = 192;
 };
 
 struct DecFwdArgs {
-    const __nv_bfloat16 *B;     // T x r
     const __nv_bfloat16 *Wd1;   // r x m
     int64_t T, d;
     int act, merge;
 };
 
+// Receive side. Per tile of 128 tokens: the producer loads the tile's B rows by TMA; the MMA
+// computes Q = B . Wd1 into the next free accumulator (a "chunk" of its own in the accumulator
+// sequence); the epilogue turns Q into G = phi(Q) (bf16, shared memory) and then drains the
+// tile's Y chunks (G . Wd2_chunk, + B on the first r columns), storing them by TMA.
 template <int M_>
 __global__ void __launch_bounds__(192, 1)
     k_dec_fwd(const __grid_constant__ CUtensorMap tm_wd2, const __grid_constant__ CUtensorMap tm_y128,
-              const __grid_constant__ CUtensorMap tm_y16, const DecFwdArgs a)
+              const __grid_constant__ CUtensorMap tm_y16, const __grid_constant__ CUtensorMap tm_b,
+              const DecFwdArgs a)
 {
     using C = DecFwdCfg<M_>;
     griddep_wait();               // the previous kernel of the stream has completed
@@ -56,7 +64,7 @@ __global__ void __launch_bounds__(192, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     __shared__ uint64_t w_full[C::NSTAGE], w_empty[C::NSTAGE];
-    __shared__ uint64_t g_full[2], g_empty[2], acc_full[2], acc_empty[2], done_bar;
+    __shared__ uint64_t b_full, b_empty, g_full, acc_full[2], acc_empty[2], done_bar;
     __shared__ uint32_t tmem_base_sh;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -70,19 +78,24 @@ __global__ void __launch_bounds__(192, 1)
             mbar_init(smem_u32(&w_empty[s]), 1);
         }
         for (int i = 0; i < 2; ++i) {
-            mbar_init(smem_u32(&g_full[i]), 1);
-            mbar_init(smem_u32(&g_empty[i]), 1);
             mbar_init(smem_u32(&acc_full[i]), 1);
             mbar_init(smem_u32(&acc_empty[i]), 128);
         }
+        mbar_init(smem_u32(&b_full), 1);
+        mbar_init(smem_u32(&b_empty), 1);
+        mbar_init(smem_u32(&g_full), 1);
         mbar_init(smem_u32(&done_bar), 1);
         fence_mbar_init();
     }
     if (warp == 1) tmem_alloc(smem_u32(&tmem_base_sh), C::TMEM_COLS);
-    if (warp >= 2) {  // Wd1 (r x m bf16) into shared memory, once
-        const uint4 *src = reinterpret_cast<const uint4 *>(a.Wd1);
-        uint4 *dst = reinterpret_cast<uint4 *>(smem + C::OFF_WD1);
-        for (int i = threadIdx.x - 64; i < (int)(C::WD1_BYTES / 16); i += 128) dst[i] = src[i];
+    if (warp >= 2) {  // Wd1^T (m x r) as a swizzled K-major operand: NB blocks of GB-byte rows
+        for (int e = threadIdx.x - 64; e < C::R * C::M; e += 128) {
+            const int k = e / C::M, n = e % C::M;   // Wd1[k][n]
+            const int kb = k / (C::GB / 2), kk = k % (C::GB / 2);
+            *reinterpret_cast<__nv_bfloat16 *>(smem + C::OFF_WD1T + kb * (C::M * C::GB) + swz_offset(n, 2 * kk, C::GB)) =
+                a.Wd1[e];
+        }
+        fence_async_smem();
     }
     tc_fence_before();
     __syncthreads();
@@ -90,12 +103,20 @@ __global__ void __launch_bounds__(192, 1)
     const uint32_t tmem = tmem_base_sh;
 
     if (warp == 0) {
-        // ---------------- producer: Wd2 chunks ----------------
+        // ---------------- producer: B tiles and Wd2 chunks ----------------
         if (elect_one()) {
             tma_prefetch_desc(&tm_wd2);
-            uint32_t it = 0;
+            tma_prefetch_desc(&tm_b);
+            uint32_t it = 0, tile_i = 0;
             bool ok = true;
-            for (int64_t t0 = start; t0 < end && ok; t0 += 128) {
+            for (int64_t t0 = start; t0 < end && ok; t0 += 128, ++tile_i) {
+                // the tile's B rows, once the previous tile's are no longer read (128-row boxes:
+                // rows past T read as zeros, rows past this CTA's range are loaded, never used)
+                if (!mbar_wait(smem_u32(&b_empty), (tile_i & 1) ^ 1)) break;
+                mbar_expect_tx(smem_u32(&b_full), C::TILE_BYTES);
+                for (int b = 0; b < C::NB; ++b)
+                    tma_load_2d(smem_u32(smem + C::OFF_B + b * (128 * C::GB)), &tm_b, b * (C::GB / 2), (int32_t)t0,
+                                smem_u32(&b_full));
                 for (int c = 0; c < nchunks; ++c) {
                     const uint32_t s = it % C::NSTAGE, ph = (it / C::NSTAGE) & 1;
                     if (!mbar_wait(smem_u32(&w_empty[s]), ph ^ 1)) {
@@ -115,18 +136,38 @@ __global__ void __launch_bounds__(192, 1)
                 const uint32_t j = it - 1 - k;
                 mbar_wait(smem_u32(&w_full[j % C::NSTAGE]), (j / C::NSTAGE) & 1);
             }
+            if (tile_i > 0) mbar_wait(smem_u32(&b_full), (tile_i - 1) & 1);
         }
     } else if (warp == 1) {
         // ---------------- MMA issuer ----------------
         if (elect_one()) {
-            constexpr uint32_t idesc = idesc_bf16(128, C::NCH, false, true);
+            constexpr Swz gsw = swz_for(C::GB);
+            constexpr uint32_t id_q = idesc_bf16(128, C::M, false, false);    // B (K-major) . Wd1^T rows (K-major)
+            constexpr uint32_t id_y = idesc_bf16(128, C::NCH, false, true);   // G (K-major) . Wd2 chunk (MN-major)
+            const uint64_t bk0 = smem_desc(smem_u32(smem + C::OFF_B), 16, 8 * C::GB, gsw);
+            const uint64_t gk0 = smem_desc(smem_u32(smem + C::OFF_G), 16, 8 * C::GB, gsw);
+            const uint64_t wt0 = smem_desc(smem_u32(smem + C::OFF_WD1T), 16, 8 * C::GB, gsw);
             uint32_t it = 0, acc_it = 0, tile_i = 0;
             bool ok = true;
             for (int64_t t0 = start; t0 < end && ok; t0 += 128, ++tile_i) {
-                const uint32_t gb = tile_i & 1;
-                ok = mbar_wait(smem_u32(&g_full[gb]), (tile_i >> 1) & 1);
+                // Q = B . Wd1 into the next accumulator
+                {
+                    const uint32_t ab = acc_it & 1;
+                    ok = mbar_wait(smem_u32(&b_full), tile_i & 1) &&
+                         mbar_wait(smem_u32(&acc_empty[ab]), ((acc_it >> 1) & 1) ^ 1);
+                    tc_fence_after();
+#pragma unroll
+                    for (int k = 0; k < C::R / 16; ++k) {
+                        const uint64_t off = (uint64_t)(((k / C::SPB) * (128 * C::GB) + (k % C::SPB) * 32) >> 4);
+                        const uint64_t woff = (uint64_t)(((k / C::SPB) * (C::M * C::GB) + (k % C::SPB) * 32) >> 4);
+                        mma_bf16(tmem + ab * C::NCH, bk0 + off, wt0 + woff, id_q, k > 0);
+                    }
+                    mma_commit(smem_u32(&acc_full[ab]));
+                    ++acc_it;
+                }
+                // the tile's Y chunks once its G is in shared memory
+                ok = ok && mbar_wait(smem_u32(&g_full), tile_i & 1);
                 tc_fence_after();
-                const uint32_t gaddr = smem_u32(smem + C::OFF_G + gb * C::G_BYTES);
                 for (int c = 0; c < nchunks && ok; ++c, ++it, ++acc_it) {
                     const uint32_t s = it % C::NSTAGE, ph = (it / C::NSTAGE) & 1;
                     const uint32_t ab = acc_it & 1;
@@ -136,14 +177,13 @@ __global__ void __launch_bounds__(192, 1)
                     const uint32_t waddr = smem_u32(smem + C::OFF_W + s * C::W_STAGE_BYTES);
 #pragma unroll
                     for (int k = 0; k < C::M / 16; ++k) {
-                        const uint64_t ad = smem_desc(gaddr + (k / 4) * 16384 + (k % 4) * 32, 16, 1024, kSwz128);
+                        const uint64_t off = (uint64_t)(((k / C::SPB) * (128 * C::GB) + (k % C::SPB) * 32) >> 4);
                         const uint64_t bd = smem_desc(waddr + k * 16 * 128, C::M * 128, 1024, kSwz128);
-                        mma_bf16(tmem + ab * C::NCH, ad, bd, idesc, k > 0);
+                        mma_bf16(tmem + ab * C::NCH, gk0 + off, bd, id_y, k > 0);
                     }
                     mma_commit(smem_u32(&w_empty[s]));
                     mma_commit(smem_u32(&acc_full[ab]));
                 }
-                mma_commit(smem_u32(&g_empty[gb]));
             }
             mma_commit(smem_u32(&done_bar));
             mbar_wait(smem_u32(&done_bar), 0);
@@ -153,72 +193,35 @@ __global__ void __launch_bounds__(192, 1)
         const int q = warp & 3;
         const int row = q * 32 + lane;
         const int et = threadIdx.x - 64;  // 0..127
-        const __nv_bfloat16 *wd1 = reinterpret_cast<const __nv_bfloat16 *>(smem + C::OFF_WD1);
+        const uint32_t lane_base = (uint32_t)(q * 32) << 16;
         uint32_t acc_it = 0, tile_i = 0, store_it = 0;
         bool ok = true;
         for (int64_t t0 = start; t0 < end && ok; t0 += 128, ++tile_i) {
             const int64_t t1 = (end - t0) < 128 ? end : t0 + 128;
             const int valid = (int)(t1 - t0);
             const bool active = row < valid;
-            const int64_t tok = t0 + row;
-            // B row (r bf16) in registers
-            uint32_t brow[C::R / 2];
-            if (active) {
-                const uint4 *src = reinterpret_cast<const uint4 *>(a.B + tok * C::R);
+            // ---- G = phi(Q) -> bf16 -> the G tile (K-major, NB blocks of GB-byte rows) ----
+            {
+                const uint32_t ab = acc_it & 1;
+                ok = mbar_wait(smem_u32(&acc_full[ab]), (acc_it >> 1) & 1);
+                tc_fence_after();
+                float g[C::M];
+                tmem_ld_row<C::M>(tmem + lane_base + ab * C::NCH, g);
+                tc_fence_before();
+                mbar_arrive(smem_u32(&acc_empty[ab]));
+                ++acc_it;
+                act_fast_row<C::M>(a.act, g);
 #pragma unroll
-                for (int i = 0; i < C::R / 8; ++i) {
-                    const uint4 v = src[i];
-                    brow[4 * i] = v.x; brow[4 * i + 1] = v.y; brow[4 * i + 2] = v.z; brow[4 * i + 3] = v.w;
+                for (int b = 0; b < C::NB; ++b) {
+                    float gb[C::GB / 2];
+#pragma unroll
+                    for (int j = 0; j < C::GB / 2; ++j) gb[j] = active ? g[b * (C::GB / 2) + j] : 0.0f;
+                    store_bf16_swz_row<C::GB / 2>(smem + C::OFF_G + b * (128 * C::GB), row, gb);
                 }
-            } else {
-#pragma unroll
-                for (int i = 0; i < C::R / 2; ++i) brow[i] = 0u;
+                fence_async_smem();
+                named_barrier(1, 128);
+                if (et == 0) mbar_arrive(smem_u32(&g_full));
             }
-            // G = phi(B . Wd1) -> bf16 -> G buffer (row `row`, K-major, 128B swizzle)
-            const uint32_t gb = tile_i & 1;
-            ok = mbar_wait(smem_u32(&g_empty[gb]), ((tile_i >> 1) & 1) ^ 1);
-            uint8_t *gbuf = smem + C::OFF_G + gb * C::G_BYTES;
-            // rows past the valid tokens only feed output rows that are never stored
-            const int jend = (q * 32 < valid) ? C::M : 0;
-#pragma unroll
-            for (int jb = 0; jb < C::M; jb += 16) {
-                if (jb >= jend) break;
-                float accq[16];
-#pragma unroll
-                for (int j = 0; j < 16; ++j) accq[j] = 0.0f;
-#pragma unroll
-                for (int k = 0; k < C::R; ++k) {
-                    const uint32_t bb = brow[k >> 1];
-                    const float bk = __uint_as_float((k & 1) ? (bb & 0xFFFF0000u) : (bb << 16));
-                    const uint4 *w = reinterpret_cast<const uint4 *>(wd1 + k * C::M + jb);
-                    const uint4 w0 = w[0], w1 = w[1];
-                    const uint32_t wv[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
-#pragma unroll
-                    for (int j = 0; j < 8; ++j) {
-                        accq[2 * j] = fmaf(bk, __uint_as_float(wv[j] << 16), accq[2 * j]);
-                        accq[2 * j + 1] = fmaf(bk, __uint_as_float(wv[j] & 0xFFFF0000u), accq[2 * j + 1]);
-                    }
-                }
-                act_fast_row<16>(a.act, accq);
-                uint32_t packed[8];
-#pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                    const float g0 = active ? accq[2 * j] : 0.0f;
-                    const float g1 = active ? accq[2 * j + 1] : 0.0f;
-                    __nv_bfloat162 h = __floats2bfloat162_rn(g0, g1);
-                    packed[j] = *reinterpret_cast<uint32_t *>(&h);
-                }
-                // 16 bf16 = two 16-byte chunks at K offset jb within block jb / 64
-                const uint32_t kb = jb >> 6, byte = (jb & 63) * 2;
-                uint8_t *blk = gbuf + kb * 16384;
-                *reinterpret_cast<uint4 *>(blk + swz_offset(row, byte, 128)) =
-                    make_uint4(packed[0], packed[1], packed[2], packed[3]);
-                *reinterpret_cast<uint4 *>(blk + swz_offset(row, byte + 16, 128)) =
-                    make_uint4(packed[4], packed[5], packed[6], packed[7]);
-            }
-            fence_async_smem();
-            named_barrier(1, 128);
-            if (et == 0) mbar_arrive(smem_u32(&g_full[gb]));
 
             for (int c = 0; c < nchunks && ok; ++c, ++acc_it, ++store_it) {
                 const uint32_t ab = acc_it & 1;
@@ -236,15 +239,22 @@ __global__ void __launch_bounds__(192, 1)
                 for (int g = 0; g < C::NCH / 32; ++g) {
                     if (g * 32 >= gend) break;
                     float v[32];
-                    tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + ab * C::NCH + g * 32, v);
+                    tmem_ld32(tmem + lane_base + ab * C::NCH + g * 32, v);
                     tmem_ld_wait();
                     // identity path: the first r columns of Y get B (only chunk 0 holds them)
                     if (g * 32 < C::R && a.merge && c == 0) {
+                        const uint8_t *bblk = smem + C::OFF_B + ((g * 32) / (C::GB / 2)) * (128 * C::GB);
+                        const uint32_t b0 = ((g * 32) % (C::GB / 2)) * 2;
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) {
+                        for (int i = 0; i < 32; i += 8) {
                             if (g * 32 + i < C::R) {
-                                const uint32_t bb = brow[(g * 32 + i) >> 1];
-                                v[i] += __uint_as_float(((g * 32 + i) & 1) ? (bb & 0xFFFF0000u) : (bb << 16));
+                                const uint4 u = *reinterpret_cast<const uint4 *>(bblk + swz_offset(row, b0 + 2 * i, C::GB));
+                                const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+                                for (int e = 0; e < 4; ++e) {
+                                    v[i + 2 * e] += __uint_as_float(w[e] << 16);
+                                    v[i + 2 * e + 1] += __uint_as_float(w[e] & 0xFFFF0000u);
+                                }
                             }
                         }
                     }
@@ -267,6 +277,7 @@ __global__ void __launch_bounds__(192, 1)
                 fence_async_smem();
                 named_barrier(1, 128);
                 if (et == 0) {
+                    if (c == 0) mbar_arrive(smem_u32(&b_empty));   // the B tile is no longer read
                     const uint32_t sbase = smem_u32(stg);
                     for (int b = 0; b < ncols / 64; ++b) {
                         const int x = c * C::NCH + 64 * b;
