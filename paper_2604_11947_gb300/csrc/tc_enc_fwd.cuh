@@ -5,8 +5,9 @@
 //   producer warp : for each tile, d in chunks of 64 columns: F tile chunk (128 x 64, K-major,
 //                   128B swizzle; 16-row boxes for a partial tile) + We1 rows (64 x m, MN-major)
 //   MMA warp      : P (128 x m fp32 in TMEM, double-buffered per tile) += F_chunk . We1_chunk
-//   epilogue warps: TMEM -> registers (one token per thread), store P, A = phi(P),
-//                   E = A . We2 (fp32 on CUDA cores, We2 in shared memory), B = X[:, :r] + E
+//   epilogue warps: TMEM -> registers (one token per thread), store P, A = phi(P) as a bf16
+//                   hi + lo pair in shared memory; the MMA warp then computes E = A . We2 into
+//                   TMEM (polled between the next tile's stages); B = X[:, :r] + E
 // HBM traffic per token: read F (2d), X[:, :r] (2r); write B (2r), P (4m).
 #pragma once
 
@@ -24,20 +25,28 @@ template <int M_> struct EncFwdCfg {
     static constexpr uint32_t F_BYTES = 128 * 128;                      // 128 rows x 64 bf16
     static constexpr uint32_t W_BYTES = 64 * M_ * 2;                    // 64 rows x m bf16
     static constexpr uint32_t STAGE_BYTES = F_BYTES + W_BYTES;
-    static constexpr int NSTAGE = M_ <= 32 ? 8 : (M_ == 64 ? 6 : 5);
-    static constexpr uint32_t WE2_BYTES = M_ * R * 2;
+    static constexpr int NSTAGE = M_ <= 32 ? 8 : (M_ == 64 ? 6 : 3);
+    static constexpr uint32_t GB = M_ * 2 < 128 ? M_ * 2 : 128;        // row bytes (= swizzle) of an A block
+    static constexpr int NB = M_ * 2 / GB;                              // blocks across the m columns
+    static constexpr int SPB = GB / 32;                                 // 16-element K steps per block
+    static constexpr uint32_t A_TILE = 128 * M_ * 2;                    // 128 tokens x m bf16
+    static constexpr uint32_t WE2T_BYTES = R * M_ * 2;
     static constexpr uint32_t OFF_STAGE = 0;
-    static constexpr uint32_t OFF_WE2 = NSTAGE * STAGE_BYTES;
-    static constexpr uint32_t SMEM_BYTES = OFF_WE2 + WE2_BYTES + 1024;
+    static constexpr uint32_t OFF_A = NSTAGE * STAGE_BYTES;             // A = phi(P): hi tile, then lo tile
+    static constexpr uint32_t OFF_WE2T = OFF_A + 2 * A_TILE;            // We2^T [r][m], K-major
+    static constexpr uint32_t SMEM_BYTES = OFF_WE2T + WE2T_BYTES + 1024;
+    static_assert(SMEM_BYTES <= 232448 - 512, "shared memory budget");
     static constexpr uint32_t ACC_STRIDE = M_ < 32 ? 32 : M_;          // TMEM columns per accumulator
-    static constexpr uint32_t TMEM_COLS = 2 * ACC_STRIDE;
+    static constexpr uint32_t TM_E = 2 * ACC_STRIDE;                    // E = A . We2 (r columns)
+    static constexpr uint32_t TMEM_NEED = TM_E + ACC_STRIDE;
+    static constexpr uint32_t TMEM_COLS = TMEM_NEED <= 128 ? 128 : TMEM_NEED <= 256 ? 256 : 512;
     static constexpr int THREADS = 192;
 };
 
 struct EncFwdArgs {
     const __nv_bfloat16 *X;    // T x d (first r columns read)
     const __nv_bfloat16 *We2;  // m x r
-    __nv_bfloat16 *B;          // T x r
+    __nv_bfloat16 *B;          // T x r, or null: P = F . We1 only (for the backward)
     float *P;                  // T x m or null
     int64_t T, d;
     int act;
@@ -54,11 +63,12 @@ __global__ void __launch_bounds__(192, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     __shared__ uint64_t full[C::NSTAGE], empty[C::NSTAGE];
-    __shared__ uint64_t acc_full[2], acc_empty[2], done_bar;
+    __shared__ uint64_t acc_full[2], acc_empty[2], a_full, e_full, done_bar;
     __shared__ uint32_t tmem_base_sh;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nk = (int)(a.d / 64);
+    const bool want_b = a.B != nullptr;
     int64_t start, end;
     token_range(a.T, blockIdx.x, gridDim.x, start, end);
 
@@ -71,14 +81,20 @@ __global__ void __launch_bounds__(192, 1)
             mbar_init(smem_u32(&acc_full[i]), 1);
             mbar_init(smem_u32(&acc_empty[i]), 128);
         }
+        mbar_init(smem_u32(&a_full), 1);
+        mbar_init(smem_u32(&e_full), 1);
         mbar_init(smem_u32(&done_bar), 1);
         fence_mbar_init();
     }
     if (warp == 1) tmem_alloc(smem_u32(&tmem_base_sh), C::TMEM_COLS);
-    if (warp >= 2) {  // We2 (m x r bf16) into shared memory, once
-        const uint4 *src = reinterpret_cast<const uint4 *>(a.We2);
-        uint4 *dst = reinterpret_cast<uint4 *>(smem + C::OFF_WE2);
-        for (int i = threadIdx.x - 64; i < (int)(C::WE2_BYTES / 16); i += 128) dst[i] = src[i];
+    if (warp >= 2 && want_b) {  // We2^T (r x m) as a swizzled K-major operand: NB blocks of GB-byte rows
+        for (int e = threadIdx.x - 64; e < C::M * C::R; e += 128) {
+            const int k = e / C::R, n = e % C::R;   // We2[k][n]
+            const int kb = k / (C::GB / 2), kk = k % (C::GB / 2);
+            *reinterpret_cast<__nv_bfloat16 *>(smem + C::OFF_WE2T + kb * (C::R * C::GB) + swz_offset(n, 2 * kk, C::GB)) =
+                a.We2[e];
+        }
+        fence_async_smem();
     }
     tc_fence_before();
     __syncthreads();
@@ -128,16 +144,51 @@ __global__ void __launch_bounds__(192, 1)
         // ---------------- MMA issuer ----------------
         if (elect_one()) {
             constexpr Swz wswz = C::WSW == 128 ? kSwz128 : C::WSW == 64 ? kSwz64 : kSwz32;
+            constexpr Swz gsw = swz_for(C::GB);
             constexpr uint32_t idesc = idesc_bf16(128, C::M, false, true);
+            constexpr uint32_t id_e = idesc_bf16(128, C::R, false, false);   // A (K-major) . We2^T rows (K-major)
+            const uint64_t ak0 = smem_desc(smem_u32(smem + C::OFF_A), 16, 8 * C::GB, gsw);
+            const uint64_t wt0 = smem_desc(smem_u32(smem + C::OFF_WE2T), 16, 8 * C::GB, gsw);
+            constexpr uint64_t LO16 = C::A_TILE >> 4;
+            // E = (A_hi + A_lo) . We2 of the tile whose A the epilogue has published
+            uint32_t e_issued = 0;
+            auto issue_e = [&]() {
+#pragma unroll
+                for (int k = 0; k < C::M / 16; ++k) {
+                    const uint64_t off = (uint64_t)(((k / C::SPB) * (128 * C::GB) + (k % C::SPB) * 32) >> 4);
+                    const uint64_t woff = (uint64_t)(((k / C::SPB) * (C::R * C::GB) + (k % C::SPB) * 32) >> 4);
+                    mma_bf16(tmem + C::TM_E, ak0 + off, wt0 + woff, id_e, k > 0);
+                    mma_bf16(tmem + C::TM_E, ak0 + LO16 + off, wt0 + woff, id_e, true);
+                }
+                mma_commit(smem_u32(&e_full));
+                ++e_issued;
+            };
             uint32_t it = 0, tile_i = 0;
+            // Wait for (bar, parity) while issuing, in the meantime, the E product of an earlier
+            // tile as soon as the epilogue publishes its A: the epilogue waits for that E before
+            // it frees the accumulators this thread may be waiting for, so no wait may block it.
+            auto wait_serving_e = [&](uint32_t bar, uint32_t parity) -> bool {
+                const unsigned long long t_start = globaltimer();
+                for (uint32_t i = 0;; ++i) {
+                    if (want_b && e_issued < tile_i && mbar_test_wait(smem_u32(&a_full), e_issued & 1)) {
+                        tc_fence_after();
+                        issue_e();
+                    }
+                    if (mbar_try_wait(bar, parity)) return true;
+                    if ((i & 255u) == 0 && globaltimer() - t_start > kWaitNs) {
+                        flag_error(kErrWaitTimeout);
+                        return false;
+                    }
+                }
+            };
             bool ok = true;
             for (int64_t t0 = start; t0 < end && ok; t0 += 128, ++tile_i) {
                 const uint32_t ab = tile_i & 1;
-                ok = mbar_wait(smem_u32(&acc_empty[ab]), ((tile_i >> 1) & 1) ^ 1);
+                ok = wait_serving_e(smem_u32(&acc_empty[ab]), ((tile_i >> 1) & 1) ^ 1);
                 tc_fence_after();
                 for (int kc = 0; kc < nk && ok; ++kc, ++it) {
                     const uint32_t s = it % C::NSTAGE, ph = (it / C::NSTAGE) & 1;
-                    ok = mbar_wait(smem_u32(&full[s]), ph);
+                    ok = wait_serving_e(smem_u32(&full[s]), ph);
                     tc_fence_after();
                     const uint32_t faddr = smem_u32(smem + C::OFF_STAGE + s * C::STAGE_BYTES);
                     const uint32_t waddr = faddr + C::F_BYTES;
@@ -151,6 +202,12 @@ __global__ void __launch_bounds__(192, 1)
                 }
                 mma_commit(smem_u32(&acc_full[ab]));
             }
+            // the E products not issued inside the stream (at least the last tile's)
+            while (ok && want_b && e_issued < tile_i) {
+                ok = mbar_wait(smem_u32(&a_full), e_issued & 1);
+                tc_fence_after();
+                if (ok) issue_e();
+            }
             mma_commit(smem_u32(&done_bar));
             mbar_wait(smem_u32(&done_bar), 0);
         }
@@ -158,64 +215,68 @@ __global__ void __launch_bounds__(192, 1)
         // ---------------- epilogue: one token per thread ----------------
         const int q = warp & 3;
         const int row = q * 32 + lane;
-        const __nv_bfloat16 *we2 = reinterpret_cast<const __nv_bfloat16 *>(smem + C::OFF_WE2);
+        const int et = threadIdx.x - 64;
+        const uint32_t lane_base = (uint32_t)(q * 32) << 16;
         uint32_t tile_i = 0;
         bool ok = true;
         for (int64_t t0 = start; t0 < end && ok; t0 += 128, ++tile_i) {
             const int valid = (int)((end - t0) < 128 ? (end - t0) : 128);
+            const bool active = row < valid;
+            const int64_t tok = t0 + row;
             const uint32_t ab = tile_i & 1;
             ok = mbar_wait(smem_u32(&acc_full[ab]), (tile_i >> 1) & 1);
             tc_fence_after();
             float p[C::M];
-#pragma unroll
-            for (int j = 0; j < C::M; j += 16) {
-                float v[16];
-                tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + ab * C::ACC_STRIDE + j, v);
-                tmem_ld_wait();
-#pragma unroll
-                for (int i = 0; i < 16; ++i) p[j + i] = v[i];
-            }
+            tmem_ld_row<C::M>(tmem + lane_base + ab * C::ACC_STRIDE, p);
             tc_fence_before();
             mbar_arrive(smem_u32(&acc_empty[ab]));
-            if (row < valid) {  // (with a.B == null only P is wanted: P = F . We1 for the backward)
-                const int64_t tok = t0 + row;
-                if (a.P) {
-                    float4 *dst = reinterpret_cast<float4 *>(a.P + tok * C::M);
+            if (active && a.P) {
+                float4 *dst = reinterpret_cast<float4 *>(a.P + tok * C::M);
 #pragma unroll
-                    for (int j = 0; j < C::M / 4; ++j)
-                        dst[j] = make_float4(p[4 * j], p[4 * j + 1], p[4 * j + 2], p[4 * j + 3]);
+                for (int j = 0; j < C::M / 4; ++j)
+                    dst[j] = make_float4(p[4 * j], p[4 * j + 1], p[4 * j + 2], p[4 * j + 3]);
+            }
+            if (!want_b) continue;   // P only
+            // this token's X[:, :r], fetched now and used after E
+            float xv[C::R];
+#pragma unroll
+            for (int j = 0; j < C::R; ++j) xv[j] = 0.0f;
+            if (active) load_bf16_row<C::R>(a.X + tok * a.d, xv);
+            // A = phi(P) as bf16 hi + lo (the E product then sees A to about 16 significant bits)
+            act_row<C::M>(a.act, p);
+#pragma unroll
+            for (int b = 0; b < C::NB; ++b) {
+                float hi[C::GB / 2], lo[C::GB / 2];
+#pragma unroll
+                for (int j = 0; j < C::GB / 2; ++j) {
+                    const float x = active ? p[b * (C::GB / 2) + j] : 0.0f;
+                    hi[j] = __bfloat162float(__float2bfloat16_rn(x));
+                    lo[j] = x - hi[j];
                 }
-                act_row<C::M>(a.act, p);
-                const uint4 *xs = reinterpret_cast<const uint4 *>(a.X + tok * a.d);
+                store_bf16_swz_row<C::GB / 2>(smem + C::OFF_A + b * (128 * C::GB), row, hi);
+                store_bf16_swz_row<C::GB / 2>(smem + C::OFF_A + C::A_TILE + b * (128 * C::GB), row, lo);
+            }
+            fence_async_smem();
+            named_barrier(1, 128);
+            if (et == 0) mbar_arrive(smem_u32(&a_full));
+            // B = X[:, :r] + E
+            ok = mbar_wait(smem_u32(&e_full), tile_i & 1);
+            tc_fence_after();
+            float e[C::R];
+            tmem_ld_row<C::R>(tmem + lane_base + C::TM_E, e);
+            tc_fence_before();
+            if (active) {
                 uint4 *bd = reinterpret_cast<uint4 *>(a.B + tok * C::R);
 #pragma unroll
-                for (int jb = 0; jb < C::R; jb += 8) {
-                    if (a.B == nullptr) break;
-                    // E[jb .. jb+8) = sum_j A[j] We2[j][jb .. jb+8), fp32
-                    float e[8];
-#pragma unroll
-                    for (int i = 0; i < 8; ++i) e[i] = 0.0f;
-#pragma unroll
-                    for (int j = 0; j < C::M; ++j) {
-                        const uint4 w = *reinterpret_cast<const uint4 *>(we2 + j * C::R + jb);
-                        const uint32_t wv[4] = {w.x, w.y, w.z, w.w};
-#pragma unroll
-                        for (int i = 0; i < 4; ++i) {
-                            e[2 * i] = fmaf(p[j], __uint_as_float(wv[i] << 16), e[2 * i]);
-                            e[2 * i + 1] = fmaf(p[j], __uint_as_float(wv[i] & 0xFFFF0000u), e[2 * i + 1]);
-                        }
-                    }
-                    const uint4 x = xs[jb / 8];
-                    const uint32_t xv[4] = {x.x, x.y, x.z, x.w};
+                for (int v8 = 0; v8 < C::R / 8; ++v8) {
                     uint32_t o[4];
 #pragma unroll
                     for (int i = 0; i < 4; ++i) {
-                        const float b0 = __uint_as_float(xv[i] << 16) + e[2 * i];
-                        const float b1 = __uint_as_float(xv[i] & 0xFFFF0000u) + e[2 * i + 1];
-                        __nv_bfloat162 h = __floats2bfloat162_rn(b0, b1);
+                        __nv_bfloat162 h = __floats2bfloat162_rn(xv[8 * v8 + 2 * i] + e[8 * v8 + 2 * i],
+                                                                 xv[8 * v8 + 2 * i + 1] + e[8 * v8 + 2 * i + 1]);
                         o[i] = *reinterpret_cast<uint32_t *>(&h);
                     }
-                    bd[jb / 8] = make_uint4(o[0], o[1], o[2], o[3]);
+                    bd[v8] = make_uint4(o[0], o[1], o[2], o[3]);
                 }
             }
         }
