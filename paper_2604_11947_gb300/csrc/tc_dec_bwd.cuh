@@ -150,6 +150,7 @@ __global__ void __launch_bounds__(192, 1)
     if (warp == 0) {
         // ---------------- producer ----------------
         if (elect_one()) {
+            const uint64_t stream_pol = l2_evict_first();   // read once
             tma_prefetch_desc(&tm_dy128);
             tma_prefetch_desc(&tm_dy16);
             tma_prefetch_desc(&tm_wd2);
@@ -196,11 +197,11 @@ __global__ void __launch_bounds__(192, 1)
                         mbar_expect_tx(bar, valid == 128 ? C::Y_STAGE : (uint32_t)nb * 2u * 2048u);
                         for (int h = 0; h < 2; ++h) {
                             if (valid == 128) {
-                                tma_load_2d(dst + h * 16384, &tm_dy128, cc * 128 + 64 * h, (int32_t)t0, bar);
+                                tma_load_2d_hint(dst + h * 16384, &tm_dy128, cc * 128 + 64 * h, (int32_t)t0, bar, stream_pol);
                             } else {
                                 for (int rg = 0; rg < nb; ++rg)
-                                    tma_load_2d(dst + h * 16384 + rg * 2048, &tm_dy16, cc * 128 + 64 * h,
-                                                (int32_t)(t0 + 16 * rg), bar);
+                                    tma_load_2d_hint(dst + h * 16384 + rg * 2048, &tm_dy16, cc * 128 + 64 * h,
+                                                (int32_t)(t0 + 16 * rg), bar, stream_pol);
                             }
                         }
                         ++yit;

@@ -282,10 +282,10 @@ __global__ void __launch_bounds__(192, 1)
                     for (int b = 0; b < ncols / 64; ++b) {
                         const int x = c * C::NCH + 64 * b;
                         if (valid == 128) {
-                            tma_store_2d(&tm_y128, x, (int32_t)t0, sbase + b * 16384);
+                            tma_store_2d_hint(&tm_y128, x, (int32_t)t0, sbase + b * 16384, l2_evict_first());
                         } else {
                             for (int rg = 0; rg * 16 < valid; ++rg)
-                                tma_store_2d(&tm_y16, x, (int32_t)(t0 + 16 * rg), sbase + b * 16384 + rg * 2048);
+                                tma_store_2d_hint(&tm_y16, x, (int32_t)(t0 + 16 * rg), sbase + b * 16384 + rg * 2048, l2_evict_first());
                         }
                     }
                     bulk_commit();

@@ -144,6 +144,7 @@ __global__ void __launch_bounds__(192, 1)
     if (warp == 0) {
         // ---------------- producer ----------------
         if (elect_one()) {
+            const uint64_t stream_pol = l2_evict_first();   // read once
             tma_prefetch_desc(&tm_f128);
             tma_prefetch_desc(&tm_f16);
             tma_prefetch_desc(&tm_we1);
@@ -196,11 +197,11 @@ __global__ void __launch_bounds__(192, 1)
                         mbar_expect_tx(bar, valid == 128 ? C::F_STAGE : (uint32_t)nb * 2u * 2048u);
                         for (int h = 0; h < 2; ++h) {
                             if (valid == 128) {
-                                tma_load_2d(dst + h * 16384, &tm_f128, cc * 128 + 64 * h, (int32_t)t0, bar);
+                                tma_load_2d_hint(dst + h * 16384, &tm_f128, cc * 128 + 64 * h, (int32_t)t0, bar, stream_pol);
                             } else {
                                 for (int rg = 0; rg < nb; ++rg)
-                                    tma_load_2d(dst + h * 16384 + rg * 2048, &tm_f16, cc * 128 + 64 * h,
-                                                (int32_t)(t0 + 16 * rg), bar);
+                                    tma_load_2d_hint(dst + h * 16384 + rg * 2048, &tm_f16, cc * 128 + 64 * h,
+                                                (int32_t)(t0 + 16 * rg), bar, stream_pol);
                             }
                         }
                         ++j;
@@ -462,10 +463,10 @@ __global__ void __launch_bounds__(192, 1)
                         if (et == 0) {
                             const int x = cc * 128 + 64 * h;
                             if (valid == 128) {
-                                tma_store_2d(&tm_df128, x, (int32_t)t0, smem_u32(stg));
+                                tma_store_2d_hint(&tm_df128, x, (int32_t)t0, smem_u32(stg), l2_evict_first());
                             } else {
                                 for (int rgi = 0; rgi * 16 < valid; ++rgi)
-                                    tma_store_2d(&tm_df16, x, (int32_t)(t0 + 16 * rgi), smem_u32(stg) + rgi * 2048);
+                                    tma_store_2d_hint(&tm_df16, x, (int32_t)(t0 + 16 * rgi), smem_u32(stg) + rgi * 2048, l2_evict_first());
                             }
                             bulk_commit();
                         }

@@ -104,6 +104,7 @@ __global__ void __launch_bounds__(192, 1)
     if (warp == 0) {
         // ---------------- producer ----------------
         if (elect_one()) {
+            const uint64_t stream_pol = l2_evict_first();   // read once
             tma_prefetch_desc(&tm_f128);
             tma_prefetch_desc(&tm_f16);
             tma_prefetch_desc(&tm_we1);
@@ -124,10 +125,10 @@ __global__ void __launch_bounds__(192, 1)
                     const uint32_t bar = smem_u32(&full[s]);
                     mbar_expect_tx(bar, fbytes + C::W_BYTES);
                     if (valid == 128) {
-                        tma_load_2d(fdst, &tm_f128, kc * 64, (int32_t)t0, bar);
+                        tma_load_2d_hint(fdst, &tm_f128, kc * 64, (int32_t)t0, bar, stream_pol);
                     } else {
                         for (int rg = 0; rg < nbox16; ++rg)
-                            tma_load_2d(fdst + rg * 2048, &tm_f16, kc * 64, (int32_t)(t0 + 16 * rg), bar);
+                            tma_load_2d_hint(fdst + rg * 2048, &tm_f16, kc * 64, (int32_t)(t0 + 16 * rg), bar, stream_pol);
                     }
                     for (int wb = 0; wb < C::WBOXES; ++wb)
                         tma_load_2d(wdst + wb * 64 * C::WSW, &tm_we1, wb * 64, kc * 64, bar);

@@ -30,7 +30,7 @@ __device__ __forceinline__ void wgrad_chunk(const WgradArgs &w, const float (&v)
             const float4 o = st[e];
             x.x = o.x + x.x; x.y = o.y + x.y; x.z = o.z + x.z; x.w = o.w + x.w;
         }
-        st[e] = x;
+        st_global_hint(&st[e], x, l2_evict_last());   // read back by the reduction soon
     }
 }
 
