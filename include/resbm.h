@@ -136,6 +136,13 @@ RESBM_API uint64_t resbm_kernel_launches(void);
  * a non-zero word is reset to 0. */
 RESBM_API resbm_status resbm_device_error(unsigned int *code, int clear);
 
+/* Failure-path self-test (no counterpart in the paper): enqueues on `stream` a one-CTA kernel
+ * whose only wait can never complete. Like every wait in the tensor-core kernels it gives up
+ * after its bounded time (about 2 s), sets bit 1 of the error word read by resbm_device_error()
+ * and returns; nothing faults and the context stays usable. Lets a caller (and the tests) check
+ * that a stuck wait is reported instead of hanging the device. */
+RESBM_API resbm_status resbm_selftest_wait_timeout(void *stream);
+
 /* Scratch bytes that `op` (a resbm_op) needs for `desc`, written to *bytes.
  * Returns RESBM_ERR_INVALID_ARG for a bad descriptor or op. Does not touch the GPU. */
 RESBM_API resbm_status resbm_workspace_bytes(const resbm_desc *desc, int op, size_t *bytes);

@@ -406,6 +406,13 @@ resbm_status resbm_device_error(unsigned int *code, int clear)
     return e == cudaSuccess ? RESBM_OK : cuda_fail(e);
 }
 
+resbm_status resbm_selftest_wait_timeout(void *stream)
+{
+    Ctx c;
+    resbm_status s = make_ctx(stream, &c);
+    return s != RESBM_OK ? s : finish(tc_wait_selftest(c));
+}
+
 resbm_status resbm_workspace_bytes(const resbm_desc *desc, int op, size_t *bytes)
 {
     resbm_status s = check_desc(desc);

@@ -361,6 +361,28 @@ cudaError_t tc_encode_bwd(const resbm_desc &d, const void *dB, const void *F, co
     return cudaErrorNotSupported;
 }
 
+namespace tc {
+// One thread waits on an mbarrier that nothing arrives on; mbar_wait gives up after kWaitNs,
+// sets the timeout bit of the error word and returns, and the kernel exits normally.
+__global__ void k_wait_selftest()
+{
+    __shared__ uint64_t bar;
+    if (threadIdx.x == 0) {
+        mbar_init(smem_u32(&bar), 1);
+        fence_mbar_init();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) mbar_wait(smem_u32(&bar), 0);
+}
+}  // namespace tc
+
+cudaError_t tc_wait_selftest(const Ctx &c)
+{
+    tc::k_wait_selftest<<<1, 32, 0, c.stream>>>();
+    count_launches(1);
+    return cudaGetLastError();
+}
+
 cudaError_t tc_device_error(unsigned int *code, bool clear)
 {
     cudaError_t e = cudaMemcpyFromSymbol(code, tc::g_resbm_device_error, sizeof(unsigned int));

@@ -11,6 +11,9 @@ bool tc_supported(const resbm_desc &d, int op);
 
 // Reads (and optionally clears) the error word of the tensor-core kernels; synchronizing.
 cudaError_t tc_device_error(unsigned int *code, bool clear);
+// Enqueues a one-CTA kernel whose only wait can never complete: it gives up after the bounded
+// wait time and records the timeout in the error word (a test of that path; nothing faults).
+cudaError_t tc_wait_selftest(const Ctx &c);
 // Scratch bytes of the tensor-core kernels for `op` on a device with `sms` SMs.
 size_t tc_ws_bytes(const resbm_desc &d, int op, int sms);
 

@@ -30,7 +30,8 @@ TORCH_DTYPES = {RESBM_F32: torch.float32, RESBM_BF16: torch.bfloat16}
 EXPORTS = ("resbm_version", "resbm_status_string", "resbm_last_cuda_error", "resbm_kernel_launches",
            "resbm_device_error",
            "resbm_workspace_bytes", "resbm_encode_fwd", "resbm_decode_fwd", "resbm_decode_bwd",
-           "resbm_encode_bwd", "resbm_boundary_step", "resbm_decode_bwd_noalloc")
+           "resbm_encode_bwd", "resbm_boundary_step", "resbm_decode_bwd_noalloc",
+           "resbm_selftest_wait_timeout")
 
 
 class resbm_desc(ctypes.Structure):
@@ -91,6 +92,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.resbm_encode_bwd.restype = i32
     lib.resbm_encode_bwd.argtypes = [D] + [vp] * 9 + [vp, sz, vp]
     lib.resbm_boundary_step.restype = i32
+    lib.resbm_selftest_wait_timeout.restype = i32
+    lib.resbm_selftest_wait_timeout.argtypes = [vp]
     lib.resbm_decode_bwd_noalloc.restype = i32
     lib.resbm_decode_bwd_noalloc.argtypes = [D] + [vp] * 7 + [vp]
     lib.resbm_boundary_step.argtypes = [D, ctypes.POINTER(resbm_step_args), vp, sz, vp]
@@ -116,6 +119,11 @@ def resbm_device_error(clear=False) -> int:
     out = ctypes.c_uint(0)
     _check("resbm_device_error", load().resbm_device_error(ctypes.byref(out), int(bool(clear))))
     return int(out.value)
+
+
+def resbm_selftest_wait_timeout(stream=None):
+    """Enqueue the failure-path self-test kernel (a wait that gives up after ~2 s)."""
+    _check("resbm_selftest_wait_timeout", load().resbm_selftest_wait_timeout(_stream(stream)))
 
 
 def make_desc(T, d, r, m, dtype="bf16", act="silu", merge_identity=1, flags=0) -> resbm_desc:

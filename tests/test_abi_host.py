@@ -24,7 +24,7 @@ def declared_functions():
 
 def test_exports_every_declared_symbol(lib):
     names = declared_functions()
-    assert len(names) == 12, names
+    assert len(names) == 13, names
     assert sorted(resbm.EXPORTS) == names
     for n in names:
         assert hasattr(lib, n), n
