@@ -131,7 +131,8 @@ RESBM_API uint64_t resbm_kernel_launches(void);
 
 /* Error word of the tensor-core kernels on the current device (0: none). Every wait inside
  * those kernels gives up after a bounded time instead of spinning forever; a kernel that gave
- * up sets a bit here (1: a wait timed out) and returns, leaving its outputs undefined.
+ * up sets a bit here (1: a wait timed out; 4: a CTA's token share did not fit the launch's
+ * tile-group plan, an internal error) and returns, leaving its outputs undefined.
  * Reading the word synchronizes with the device (it is a device-to-host copy). With clear != 0
  * a non-zero word is reset to 0. */
 RESBM_API resbm_status resbm_device_error(unsigned int *code, int clear);

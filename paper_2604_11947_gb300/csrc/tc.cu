@@ -66,20 +66,35 @@ bool al16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 // (griddepcontrol.wait, before touching global memory) until that kernel has completed and its
 // writes are visible. What overlaps is the launch itself and the placement of CTAs on SMs that
 // the previous kernel has already left.
+// `cluster` > 1 launches 1-D thread-block clusters of that many CTAs (the grid is a multiple).
 template <typename... KArgs, typename... Args>
-cudaError_t launch(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream, Args &&...args)
+cudaError_t launch_clustered(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, int cluster,
+                             cudaStream_t stream, Args &&...args)
 {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = grid;
     cfg.blockDim = block;
     cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
+    if (cluster > 1) {
+        attr[1].id = cudaLaunchAttributeClusterDimension;
+        attr[1].val.clusterDim.x = (unsigned)cluster;
+        attr[1].val.clusterDim.y = 1;
+        attr[1].val.clusterDim.z = 1;
+        cfg.numAttrs = 2;
+    }
     return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream, Args &&...args)
+{
+    return launch_clustered(kernel, grid, block, smem, 1, stream, std::forward<Args>(args)...);
 }
 
 // Dynamic shared memory attribute, set once per (kernel, device): `done` is the calling
@@ -92,6 +107,43 @@ cudaError_t ensure_smem(K kernel, uint32_t bytes, int dev, std::atomic<uint8_t> 
     cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
     if (e == cudaSuccess && dev >= 0 && dev < kMaxDev) done[dev].store(1, std::memory_order_release);
     return e;
+}
+
+// CTAs per cluster for a backward kernel: the larger of 4 and 2 (at most clmax) that divides the
+// grid and lets all of the grid's clusters be resident at once (the kernel is persistent, one
+// CTA per SM); otherwise 1. The number of co-resident clusters is asked once per (kernel,
+// device, cluster size); `fit` is the calling launcher's own cache (count + 1; 0: not asked). Needs
+// the kernel's dynamic shared memory attribute set first.
+template <typename... KArgs>
+int pick_cluster(void (*kernel)(KArgs...), int grid, int threads, uint32_t smem, int clmax, int dev,
+                 std::atomic<int> (&fit)[kMaxDev][2])
+{
+    for (int i = 0; i < 2; ++i) {
+        const int cl = i == 0 ? 4 : 2;
+        if (cl > clmax || grid % cl != 0) continue;
+        const bool cached = dev >= 0 && dev < kMaxDev;
+        int n = cached ? fit[dev][i].load(std::memory_order_acquire) - 1 : -1;
+        if (n < 0) {
+            cudaLaunchConfig_t cfg = {};
+            cfg.gridDim = dim3((unsigned)cl);
+            cfg.blockDim = dim3((unsigned)threads);
+            cfg.dynamicSmemBytes = smem;
+            cudaLaunchAttribute attr[1];
+            attr[0].id = cudaLaunchAttributeClusterDimension;
+            attr[0].val.clusterDim.x = (unsigned)cl;
+            attr[0].val.clusterDim.y = 1;
+            attr[0].val.clusterDim.z = 1;
+            cfg.attrs = attr;
+            cfg.numAttrs = 1;
+            if (cudaOccupancyMaxActiveClusters(&n, kernel, &cfg) != cudaSuccess) {
+                (void)cudaGetLastError();   // not an error of the caller's stream: fall back
+                n = 0;
+            }
+            if (cached) fit[dev][i].store(n + 1, std::memory_order_release);
+        }
+        if ((int64_t)n * cl >= grid) return cl;
+    }
+    return 1;
 }
 
 bool tc_width_ok(int64_t m) { return m == 16 || m == 32 || m == 64 || m == 128; }
@@ -147,8 +199,9 @@ cudaError_t launch_enc_fwd(const resbm_desc &d, const void *X, const void *F, co
     return e;
 }
 
-// Scratch layout of the backward kernels: the d x m weight gradient has one fp32 slot per CTA
-// (tc_wgrad.cuh); the small one has one slot per (CTA, tile group).
+// Scratch layout of the backward kernels: the d x m weight gradient has one fp32 slot per
+// cluster (sized for clusters of one CTA; tc_wgrad.cuh); the small one has one slot per (CTA,
+// tile group). Every CTA has max_groups tile groups.
 struct BwdPlan {
     int grid = 1, max_groups = 1, nch = 1;
     int64_t slots = 1;              // small partial slots
@@ -219,13 +272,16 @@ cudaError_t launch_dec_bwd(const resbm_desc &d, const void *dY, const void *B, c
                      static_cast<__nv_bfloat16 *>(dB),
                      tc::WgradArgs{p.part_big, p.nch},
                      p.part_small, d.T, d.d, d.act, d.merge_identity, p.max_groups};
-    e = launch(tc::k_dec_bwd<M>, p.grid, Cfg::THREADS, Cfg::SMEM_BYTES, c.stream, m_dy128, m_dy16, m_wd2, m_b, m_yr, a);
+    static std::atomic<int> fit[kMaxDev][2];
+    const int cl = pick_cluster(tc::k_dec_bwd<M>, p.grid, Cfg::THREADS, Cfg::SMEM_BYTES, Cfg::CLMAX, c.device, fit);
+    e = launch_clustered(tc::k_dec_bwd<M>, p.grid, Cfg::THREADS, Cfg::SMEM_BYTES, cl, c.stream, m_dy128, m_dy16, m_wd2,
+                         m_b, m_yr, a);
     count_launches(1);
     if (e != cudaSuccess) return e;
-    // dWd2 (m x d) = sum of the per-CTA slots (d x m), transposed; dWd1 (r x m) = sum of the slices
+    // dWd2 (m x d) = sum of the per-cluster slots (d x m), transposed; dWd1 (r x m) = sum of the slices
     const int64_t cap = (int64_t)c.sm_count * 8;
     return launch_reduce(reduce_job(p.part_small, p.slots, d.r, d.m, dWd1, 0, al16(dWd1), cap),
-                         reduce_job(p.part_big, p.grid, d.d, d.m, dWd2, 1, 0, cap), c);
+                         reduce_job(p.part_big, p.grid / cl, d.d, d.m, dWd2, 1, 0, cap), c);
 }
 
 int dec_bwd_nt(int64_t m)
@@ -278,13 +334,15 @@ cudaError_t launch_enc_bwd(const resbm_desc &d, const void *dB, const void *F, c
     if (e != cudaSuccess) return e;
     tc::EncBwdArgs a{P, static_cast<const __nv_bfloat16 *>(We2), static_cast<__nv_bfloat16 *>(dX),
                      tc::WgradArgs{p.part_big, p.nch}, p.part_small, d.T, d.d, d.act, p.max_groups};
-    e = launch(tc::k_enc_bwd<M>, p.grid, Cfg::THREADS, Cfg::SMEM_BYTES, c.stream, m_f128, m_f16, m_we1, m_df128,
-               m_df16, m_db, a);
+    static std::atomic<int> fit[kMaxDev][2];
+    const int cl = pick_cluster(tc::k_enc_bwd<M>, p.grid, Cfg::THREADS, Cfg::SMEM_BYTES, Cfg::CLMAX, c.device, fit);
+    e = launch_clustered(tc::k_enc_bwd<M>, p.grid, Cfg::THREADS, Cfg::SMEM_BYTES, cl, c.stream, m_f128, m_f16, m_we1,
+                         m_df128, m_df16, m_db, a);
     count_launches(1);
     if (e != cudaSuccess) return e;
     const int64_t cap = (int64_t)c.sm_count * 8;
     return launch_reduce(reduce_job(p.part_small, p.slots, d.m, d.r, dWe2, 0, al16(dWe2), cap),
-                         reduce_job(p.part_big, p.grid, d.d, d.m, dWe1, 0, al16(dWe1), cap), c);
+                         reduce_job(p.part_big, p.grid / cl, d.d, d.m, dWe1, 0, al16(dWe1), cap), c);
 }
 
 }  // namespace

@@ -21,6 +21,7 @@ static __device__ unsigned int g_resbm_device_error = 0;
 enum : unsigned {
     kErrWaitTimeout = 1u,   // an mbarrier wait exceeded kWaitNs
     kErrStoreTimeout = 2u,  // reserved
+    kErrPlan = 4u,          // a CTA's token share does not fit the launch's tile-group plan
 };
 
 constexpr unsigned long long kWaitNs = 2000000000ull;  // 2 s
@@ -63,6 +64,19 @@ __device__ __forceinline__ void token_range(int64_t T, int b, int G, int64_t &st
     end = 16 * ((U * (b + 1)) / G);
     if (end > T) end = T;
     if (start > T) start = T;
+}
+
+// Tiles [tb, te) of tile group g when a CTA's ntiles tiles are cut into ngroups groups as evenly
+// as possible, the larger groups first: the kernels' per-tile barriers (one per position in a
+// group, waited with the group's parity) need every position used by a group to have been used
+// by all earlier groups. Every CTA of a launch has the same ngroups (so that the CTAs of a
+// cluster make the same sequence of weight-gradient exchanges); the host picks it so that every
+// group has between 1 and the kernel's group capacity of tiles.
+__device__ __forceinline__ void group_tiles(int g, int ngroups, int ntiles, int &tb, int &te)
+{
+    const int q = ntiles / ngroups, rem = ntiles - q * ngroups;
+    tb = g * q + (g < rem ? g : rem);
+    te = tb + q + (g < rem ? 1 : 0);
 }
 
 // ---- small per-token products on CUDA cores (fp32 accumulate) ---------------------------------
@@ -163,6 +177,61 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity)
             return false;
         }
     }
+}
+
+// ---- thread-block clusters --------------------------------------------------------------------
+__device__ __forceinline__ uint32_t cluster_rank()
+{
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+__device__ __forceinline__ uint32_t cluster_size()
+{
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
+    return r;
+}
+
+__device__ __forceinline__ uint32_t cluster_index()
+{
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%clusterid.x;" : "=r"(r));
+    return r;
+}
+
+// The address of the same shared-memory location in cluster CTA `rank` (distributed shared memory).
+__device__ __forceinline__ uint32_t map_shared(uint32_t addr, uint32_t rank)
+{
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+    return r;
+}
+
+// All threads of all CTAs of the cluster (release / acquire at cluster scope).
+__device__ __forceinline__ void cluster_sync()
+{
+    asm volatile("barrier.cluster.arrive;\n\tbarrier.cluster.wait;" ::: "memory");
+}
+
+// Arrive on an mbarrier of another CTA of the cluster (address from map_shared). Default
+// semantics (release at CTA scope): used only to hand a shared-memory buffer back to its writer
+// after the values read from it have been consumed, which needs no cluster-scope fence.
+__device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_bar)
+{
+    asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(cluster_bar) : "memory");
+}
+
+// 16-byte store into another CTA's shared memory that counts its bytes on that CTA's mbarrier
+// (both addresses from map_shared). The bytes are visible to the threads that see the barrier's
+// phase complete, as with a TMA load.
+__device__ __forceinline__ void st_async_f4(uint32_t cluster_dst, float4 v, uint32_t cluster_bar)
+{
+    asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.f32 [%0], {%1, %2, %3, %4}, [%5];" ::"r"(
+                     cluster_dst),
+                 "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "r"(cluster_bar)
+                 : "memory");
 }
 
 // ---- proxies and fences -------------------------------------------------------------------------

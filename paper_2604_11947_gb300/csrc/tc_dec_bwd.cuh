@@ -3,8 +3,9 @@
 //   Q = B . Wd1, G = phi(Q);  dG = dY . Wd2^T;  dQ = dG * phi'(Q);
 //   dB = [merge] dY[:, :r] + dQ . Wd1^T;  dWd2 = G^T . dY;  dWd1 = B^T . dQ.
 //
-// Persistent CTAs over contiguous 16-token-aligned token ranges, processed in groups of up to
-// NT tiles of 128 tokens. Every product runs on tcgen05; the CUDA cores only apply phi and phi'
+// Persistent CTAs (in clusters of 1, 2 or 4) over contiguous 16-token-aligned token ranges,
+// processed in groups of up to NT tiles of 128 tokens (every CTA has the same number of groups,
+// its tiles split evenly). Every product runs on tcgen05; the CUDA cores only apply phi and phi'
 // and convert. For each group:
 //   phase 0: the group's B tiles (TMA) -> Q_tile = B . Wd1 in TMEM (kept for phase 2) -> the
 //            epilogue writes G = phi(Q) as bf16 rows [token][m] to shared memory.
@@ -13,7 +14,8 @@
 //              dG_tile   (128 tokens x m, TMEM, kept over all chunks) += dY . Wd2_chunk^T
 //              dWd2T_chk (128 columns x m, TMEM, double-buffered)     += dY^T . G_tile
 //            (the same dY stage read K-major and MN-major; G read MN-major). The epilogue
-//            drains each finished dWd2T chunk to the CTA's fp32 partial slot.
+//            drains each finished dWd2T chunk into the cluster's fp32 partial slot (summed over
+//            the cluster's CTAs through distributed shared memory, tc_wgrad.cuh).
 //   phase 2: the epilogue writes dQ = dG * phi'(Q) as two bf16 tiles hi + lo (rows [token][m],
 //            in the idle dY ring; hi = dQ rounded to bf16, lo = the rounded remainder, so the
 //            products see dQ to about 16 significant bits: dB crosses the boundary and is
@@ -23,7 +25,7 @@
 //            dY[:, :r] (a TMA tile) and stores dB as bf16; the group's dWd1 goes to its slot.
 // A second kernel sums the partial slots in a fixed order (deterministic).
 // HBM traffic per token: read dY (2d), B (2r), dY[:, :r] again (2r, mostly L2), write dB (2r);
-// per slot: d x m + r x m fp32 partials.
+// per cluster: d x m fp32 partials; per CTA and group: r x m.
 #pragma once
 
 #include "common.cuh"
@@ -39,7 +41,9 @@ template <int M_> struct DecBwdCfg {
     static constexpr int MS = M_ < 32 ? 32 : M_;              // TMEM columns per accumulator
     static constexpr int NT = M_ <= 32 ? 4 : 2;               // tiles per group
     static constexpr int NSY = M_ <= 32 ? 4 : 3;              // dY ring depth
-    static constexpr int NW = M_ <= 16 ? 4 : 3;               // Wd2 slice ring depth
+    static constexpr int NW = M_ <= 16 ? 4 : M_ <= 32 ? 2 : 3;  // Wd2 slice ring depth
+    static constexpr int CLMAX = M_ <= 32 ? 2 : 1;            // CTAs per cluster (weight-gradient exchange)
+    static constexpr int NWB = CLMAX > 1 ? 3 : 2;             // dWd2T accumulators in TMEM
     static constexpr uint32_t RB = M_ * 2;                    // row bytes (= swizzle) of the r / m wide tiles
     static constexpr uint32_t Y_STAGE = 128 * 128 * 2;        // 128 tokens x 128 columns
     static constexpr uint32_t W_STAGE = M_ * 128 * 2;         // m rows x 128 columns
@@ -51,7 +55,8 @@ template <int M_> struct DecBwdCfg {
     static constexpr uint32_t OFF_B = OFF_G + NT * TILE;      // B tiles [token][r] (TMA)
     static constexpr uint32_t OFF_WD1 = OFF_B + NT * TILE;    // Wd1 [r][m]: K-major B operand of dQ . Wd1^T
     static constexpr uint32_t OFF_WD1T = OFF_WD1 + WD1_BYTES; // Wd1^T [m][r]: K-major B operand of B . Wd1
-    static constexpr uint32_t SMEM_BYTES = OFF_WD1T + WD1_BYTES + 1024;
+    static constexpr uint32_t OFF_RX = OFF_WD1T + WD1_BYTES;  // weight-gradient receive buffer
+    static constexpr uint32_t SMEM_BYTES = OFF_RX + wgrad_rx_bytes<M_>(CLMAX) + 1024;
     // phase-2 scratch in the idle dY ring: dQ hi tiles (slot 0), dY[:, :r] tiles (slot 1),
     // dQ lo tiles (slot 2)
     static constexpr uint32_t OFF_DQ = OFF_Y;
@@ -59,8 +64,8 @@ template <int M_> struct DecBwdCfg {
     static constexpr uint32_t OFF_DQLO = OFF_Y + 2 * Y_STAGE;
     static_assert(NT * TILE <= Y_STAGE && NSY >= 3, "phase-2 scratch must fit in three ring slots");
     static_assert(SMEM_BYTES <= 232448 - 512, "shared memory budget");
-    // TMEM columns: dG (later dB) NT x MS | Q NT x MS | dWd2T 2 x MS | dWd1 MS
-    static constexpr uint32_t TM_DG = 0, TM_Q = NT * MS, TM_WT = 2 * NT * MS, TM_W1 = TM_WT + 2 * MS;
+    // TMEM columns: dG (later dB) NT x MS | Q NT x MS | dWd2T NWB x MS | dWd1 MS
+    static constexpr uint32_t TM_DG = 0, TM_Q = NT * MS, TM_WT = 2 * NT * MS, TM_W1 = TM_WT + NWB * MS;
     static constexpr uint32_t TMEM_NEED = TM_W1 + MS;
     static_assert(TMEM_NEED <= 512, "TMEM budget");
     static constexpr uint32_t TMEM_COLS = TMEM_NEED <= 128 ? 128 : TMEM_NEED <= 256 ? 256 : 512;
@@ -88,19 +93,28 @@ __global__ void __launch_bounds__(192, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     __shared__ uint64_t y_full[C::NSY], y_empty[C::NSY], w_full[C::NW], w_empty[C::NW];
-    __shared__ uint64_t b_full, q_full, g_full[C::NT], g_empty, wt_full[2], wt_empty[2], dg_full, dg_empty;
+    __shared__ uint64_t b_full, q_full, g_full[C::NT], g_empty, wt_full[C::NWB], wt_empty[C::NWB], dg_full, dg_empty;
     __shared__ uint64_t yr_full, dq_full[C::NT], db_full[C::NT], w1_full, p2_done, done_bar;
+    __shared__ uint64_t rx_full, rx_free[4];
     __shared__ uint32_t tmem_base_sh;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nch = (int)(a.d / 128);
     // every CTA walks the d chunks in the same cyclic order but from its own starting chunk,
     // so that at any moment the CTAs read different column ranges of their rows
-    const int c_first = (int)(blockIdx.x % (unsigned)nch);
+    // (per cluster: the CTAs of a cluster exchange the same chunk at the same time)
+    const int c_first = (int)(cluster_index() % (unsigned)nch);
     int64_t start, end;
     token_range(a.T, blockIdx.x, gridDim.x, start, end);
     const int ntiles = (int)((end - start + 127) / 128);
-    const int ngroups = (ntiles + C::NT - 1) / C::NT;
+    // the same number of tile groups in every CTA (1 .. NT tiles each, checked)
+    int ngroups = a.max_groups;
+    if (ntiles < ngroups || ntiles > C::NT * ngroups) {
+        if (threadIdx.x == 0) flag_error(kErrPlan);
+        ngroups = 0;
+    }
+    WgradXchg<C::M, C::CLMAX> xg{C::CLMAX > 1 ? cluster_size() : 1u, cluster_rank(), cluster_index(),
+                                 smem_u32(smem + C::OFF_RX), smem_u32(&rx_full), smem_u32(&rx_free[0]), 0};
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < C::NSY; ++s) {
@@ -111,7 +125,7 @@ __global__ void __launch_bounds__(192, 1)
             mbar_init(smem_u32(&w_full[i]), 1);
             mbar_init(smem_u32(&w_empty[i]), 1);
         }
-        for (int i = 0; i < 2; ++i) {
+        for (int i = 0; i < C::NWB; ++i) {
             mbar_init(smem_u32(&wt_full[i]), 1);
             mbar_init(smem_u32(&wt_empty[i]), 128);
         }
@@ -129,7 +143,9 @@ __global__ void __launch_bounds__(192, 1)
         mbar_init(smem_u32(&w1_full), 1);
         mbar_init(smem_u32(&p2_done), 1);
         mbar_init(smem_u32(&done_bar), 1);
+        xg.init_barriers();
         fence_mbar_init();
+        xg.arm_first();
     }
     if (warp == 1) tmem_alloc(smem_u32(&tmem_base_sh), C::TMEM_COLS);
     if (warp >= 2) {  // Wd1 (r x m) and Wd1^T (m x r) as swizzled K-major operands
@@ -144,6 +160,7 @@ __global__ void __launch_bounds__(192, 1)
     }
     tc_fence_before();
     __syncthreads();
+    if (C::CLMAX > 1 && xg.cl > 1) cluster_sync();   // every CTA's barriers are initialized before any exchange
     tc_fence_after();
     const uint32_t tmem = tmem_base_sh;
 
@@ -163,7 +180,8 @@ __global__ void __launch_bounds__(192, 1)
                 // the ring, the B tiles and the phase-2 scratch of the previous group are free
                 if (g > 0) ok = mbar_wait(smem_u32(&p2_done), (g - 1) & 1);
                 if (!ok) break;
-                const int tb = g * C::NT, te = min(ntiles, tb + C::NT);
+                int tb, te;
+                group_tiles(g, ngroups, ntiles, tb, te);
                 // the group's B tiles (128-row boxes: rows past T read as zeros, rows past this
                 // CTA's range are loaded but never used)
                 mbar_expect_tx(smem_u32(&b_full), (uint32_t)(te - tb) * C::TILE);
@@ -268,7 +286,8 @@ __global__ void __launch_bounds__(192, 1)
             uint32_t yit = 0, wit = 0, cit = 0;
             bool ok = true;
             for (int g = 0; g < ngroups && ok; ++g) {
-                const int tb = g * C::NT, te = min(ntiles, tb + C::NT);
+                int tb, te;
+                group_tiles(g, ngroups, ntiles, tb, te);
                 // TMEM of the previous group (dG / dB, Q, dWd1) has been read out
                 if (g > 0) ok = mbar_wait(smem_u32(&dg_empty), (g - 1) & 1);
                 ok = ok && mbar_wait(smem_u32(&b_full), g & 1);
@@ -284,9 +303,9 @@ __global__ void __launch_bounds__(192, 1)
                 // ---- phase 1: the dY stream ----
                 for (int c = 0; c < nch && ok; ++c, ++cit) {
                     const uint32_t sw = wit % C::NW;
-                    const uint32_t ab = cit & 1;
+                    const uint32_t ab = cit % C::NWB;
                     ok = mbar_wait(smem_u32(&w_full[sw]), (wit / C::NW) & 1) &&
-                         mbar_wait(smem_u32(&wt_empty[ab]), ((cit >> 1) & 1) ^ 1);
+                         mbar_wait(smem_u32(&wt_empty[ab]), ((cit / C::NWB) & 1) ^ 1);
                     tc_fence_after();
                     const uint64_t wk = wk0 + ((sw * C::W_STAGE) >> 4);
                     const uint32_t d_wt = tmem + C::TM_WT + ab * C::MS;
@@ -365,7 +384,8 @@ __global__ void __launch_bounds__(192, 1)
         uint32_t cit = 0;
         bool ok = true;
         for (int g = 0; g < ngroups && ok; ++g) {
-            const int tb = g * C::NT, te = min(ntiles, tb + C::NT);
+            int tb, te;
+            group_tiles(g, ngroups, ntiles, tb, te);
             const int64_t slot = (int64_t)blockIdx.x * a.max_groups + g;
             // ---- phase 0: G = phi(Q) of every tile of the group ----
             ok = mbar_wait(smem_u32(&g_empty), (g & 1) ^ 1) && mbar_wait(smem_u32(&q_full), g & 1);
@@ -386,17 +406,43 @@ __global__ void __launch_bounds__(192, 1)
             }
 
             // ---- phase 1: drain each chunk's dWd2^T partial ----
+            // With a cluster exchange, the rows this CTA sends go out as soon as their chunk is
+            // complete, and the rows it owns are read out at the start of the next chunk's turn
+            // (the peers' rows of that chunk have arrived by then; the accumulator waits in TMEM).
+            const bool defer = xg.exchanging() && xg.owns(row);
+            int pend = -1, pend_cc = 0;
+            auto drain_owned = [&](int buf, int chunk) {
+                float v[C::M];
+                tmem_ld_row<C::M>(tmem + lane_base + C::TM_WT + buf * C::MS, v);
+                tc_fence_before();
+                mbar_arrive(smem_u32(&wt_empty[buf]));   // the accumulator is free again
+                return xg.receive(a.wg, v, chunk, row, g == 0);
+            };
             for (int c = 0; c < nch && ok; ++c, ++cit) {
                 const int cc = c + c_first < nch ? c + c_first : c + c_first - nch;
-                const uint32_t ab = cit & 1;
-                ok = mbar_wait(smem_u32(&wt_full[ab]), (cit >> 1) & 1);
+                const uint32_t ab = cit % C::NWB;
+                if (pend >= 0) {
+                    ok = drain_owned(pend, pend_cc);
+                    pend = -1;
+                }
+                ok = ok && mbar_wait(smem_u32(&wt_full[ab]), (cit / C::NWB) & 1);
                 tc_fence_after();
+                if (defer) {
+                    pend = (int)ab;
+                    pend_cc = cc;
+                    continue;
+                }
                 float v[C::M];
                 tmem_ld_row<C::M>(tmem + lane_base + C::TM_WT + ab * C::MS, v);
                 tc_fence_before();
                 mbar_arrive(smem_u32(&wt_empty[ab]));   // the accumulator is free again
-                wgrad_chunk<C::M>(a.wg, v, cc, row, g == 0);
+                if (xg.exchanging()) {
+                    ok = ok && xg.send(v, row);
+                } else {
+                    xg.store_own(a.wg, v, cc, row, g == 0);
+                }
             }
+            if (ok && pend >= 0) ok = drain_owned(pend, pend_cc);   // the group's last chunk
 
             // ---- phase 2: dQ (hi + lo), then dB and the dWd1 partial ----
             ok = ok && mbar_wait(smem_u32(&dg_full), g & 1);
@@ -468,11 +514,6 @@ __global__ void __launch_bounds__(192, 1)
             named_barrier(1, 128);   // phase-2 scratch reads done before the ring is reused
             if (et == 0) mbar_arrive(smem_u32(&p2_done));
         }
-        // slots of groups this CTA does not have: zeros
-        for (int g = ngroups; g < a.max_groups; ++g) {
-            const int64_t slot = (int64_t)blockIdx.x * a.max_groups + g;
-            for (int e = et; e < C::R * C::M; e += 128) a.part1[slot * (C::R * C::M) + e] = 0.0f;
-        }
     }
     tc_fence_before();
     __syncthreads();
@@ -480,6 +521,7 @@ __global__ void __launch_bounds__(192, 1)
         tc_fence_after();
         tmem_dealloc(tmem, C::TMEM_COLS);
     }
+    if (C::CLMAX > 1 && xg.cl > 1) cluster_sync();   // no peer addresses this CTA's shared memory any more
 }
 
 // out = sum over slots s = 0, 1, ... of part[s] (rows x cols each, rows * cols % 4 == 0), each

@@ -3,9 +3,9 @@
 //   dA = dB . We2^T;  dP = dA * phi'(P);  dF = dP . We1^T;  dX[:, :r] += dB;
 //   dWe1 = F^T . dP;  dWe2 = phi(P)^T . dB.
 //
-// Persistent CTAs over contiguous 16-token-aligned token ranges, in groups of up to NT tiles of
-// 128 tokens. Every product runs on tcgen05; the CUDA cores apply phi and phi', convert, and
-// do the identity-path update. For each group:
+// Persistent CTAs (in clusters of 1, 2 or 4) over contiguous 16-token-aligned token ranges, in
+// groups of up to NT tiles of 128 tokens. Every product runs on tcgen05; the CUDA cores apply
+// phi and phi', convert, and do the identity-path update. For each group:
 //   phase 0: the group's dB tiles (TMA) -> dA_tile = dB . We2^T in TMEM -> the epilogue reads P
 //            (fp32, from the forward pass) and writes dP = dA * phi'(P) and A = phi(P) as bf16
 //            rows [token][m] to shared memory (for m <= 32 dP also as hi + lo, hi = dP rounded
@@ -19,10 +19,12 @@
 //              dF_tile_chunk (128 x 128 fp32, TMEM, double-buffered) = dP . We1_chunk^T
 //              dWe1_chunk    (128 columns x m, TMEM, double-buffered) += F^T . dP
 //            (F read MN-major, dP read K-major and MN-major). The epilogue converts dF to bf16
-//            and stores it by TMA, and drains each finished dWe1 chunk to the CTA's fp32
-//            partial slot; the group's dWe2 goes to its own partial slot.
+//            and stores it by TMA, and drains each finished dWe1 chunk into the cluster's fp32
+//            partial slot (summed over the cluster's CTAs through distributed shared memory,
+//            tc_wgrad.cuh); the group's dWe2 goes to its own per-CTA partial slot.
+// Every CTA has the same number of tile groups (its tiles split evenly).
 // HBM traffic per token: read F (2d), P (4m), dB (2r), dX[:, :r] (2r); write dF (2d),
-// dX[:, :r] (2r). Per slot: d x m + m x r fp32 partials.
+// dX[:, :r] (2r). Per cluster: d x m fp32 partials; per CTA and group: m x r.
 #pragma once
 
 #include "common.cuh"
@@ -38,7 +40,9 @@ template <int M_> struct EncBwdCfg {
     static constexpr int MS = M_ < 32 ? 32 : M_;                 // TMEM columns per m-wide accumulator
     static constexpr int NT = M_ <= 32 ? 4 : 2;                  // tiles per group
     static constexpr int NSF = 3;                                // F ring depth
-    static constexpr int NW = M_ <= 16 ? 4 : 3;                  // We1 slice ring depth
+    static constexpr int NW = M_ <= 16 ? 4 : M_ <= 32 ? 2 : 3;   // We1 slice ring depth
+    static constexpr int CLMAX = M_ <= 32 ? 2 : 1;               // CTAs per cluster (weight-gradient exchange)
+    static constexpr int NWB = CLMAX > 1 ? 3 : 2;                // dWe1 accumulators in TMEM
     static constexpr int NDA = M_ <= 32 ? NT : 1;                // dA TMEM regions (a ring)
     static constexpr bool DPLO = M_ <= 32;                       // dP kept as bf16 hi + lo for dF
     static constexpr uint32_t RB = M_ * 2;                       // row bytes (= swizzle) of r / m wide tiles
@@ -53,14 +57,15 @@ template <int M_> struct EncBwdCfg {
     static constexpr uint32_t OFF_DP = OFF_W + NW * W_STAGE;     // dP (hi) tiles [token][m]
     static constexpr uint32_t OFF_DPLO = OFF_DP + NT * TILE;     // dP lo tiles (if DPLO)
     static constexpr uint32_t OFF_WE2 = OFF_DPLO + (DPLO ? NT * TILE : 0);  // We2 [m][r], K-major
-    static constexpr uint32_t SMEM_BYTES = OFF_WE2 + WE2_BYTES + 1024;
+    static constexpr uint32_t OFF_RX = OFF_WE2 + WE2_BYTES;      // weight-gradient receive buffer
+    static constexpr uint32_t SMEM_BYTES = OFF_RX + wgrad_rx_bytes<M_>(CLMAX) + 1024;
     // phase-0 scratch in F-ring slots 1 and 2
     static constexpr uint32_t OFF_DB = OFF_F + (NSF - 2) * F_STAGE;   // dB tiles [token][r] (TMA)
     static constexpr uint32_t OFF_A = OFF_F + (NSF - 1) * F_STAGE;    // A = phi(P) tiles [token][m]
     static_assert(NT * TILE <= F_STAGE && NSF >= 3, "phase-0 scratch must fit in two ring slots");
     static_assert(SMEM_BYTES <= 232448 - 512, "shared memory budget");
-    // TMEM columns: dF 2 x 128 | dWe1 2 x MS | dA NDA x MS | dWe2 MS
-    static constexpr uint32_t TM_DF = 0, TM_WE = 256, TM_DA = 256 + 2 * MS, TM_W2 = TM_DA + NDA * MS;
+    // TMEM columns: dF 2 x 128 | dWe1 NWB x MS | dA NDA x MS | dWe2 MS
+    static constexpr uint32_t TM_DF = 0, TM_WE = 256, TM_DA = 256 + NWB * MS, TM_W2 = TM_DA + NDA * MS;
     static_assert(TM_W2 + MS <= 512, "TMEM budget");
     static constexpr uint32_t TMEM_COLS = 512;
     static constexpr int THREADS = 192;
@@ -89,19 +94,28 @@ __global__ void __launch_bounds__(192, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     __shared__ uint64_t f_full[C::NSF], f_empty[C::NSF], w_full[C::NW], w_empty[C::NW];
-    __shared__ uint64_t df_full[2], df_empty[2], we_full[2], we_empty[2];
+    __shared__ uint64_t df_full[2], df_empty[2], we_full[C::NWB], we_empty[C::NWB];
     __shared__ uint64_t db_full, da_full[C::NDA], da_empty[C::NDA], dp_full[C::NT], p0_done, w2_full, st_done, done_bar;
+    __shared__ uint64_t rx_full, rx_free[4];
     __shared__ uint32_t tmem_base_sh;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nch = (int)(a.d / 128);
     // every CTA walks the d chunks in the same cyclic order but from its own starting chunk,
     // so that at any moment the CTAs read different column ranges of their rows
-    const int c_first = (int)(blockIdx.x % (unsigned)nch);
+    // (per cluster: the CTAs of a cluster exchange the same chunk at the same time)
+    const int c_first = (int)(cluster_index() % (unsigned)nch);
     int64_t start, end;
     token_range(a.T, blockIdx.x, gridDim.x, start, end);
     const int ntiles = (int)((end - start + 127) / 128);
-    const int ngroups = (ntiles + C::NT - 1) / C::NT;
+    // the same number of tile groups in every CTA (1 .. NT tiles each, checked)
+    int ngroups = a.max_groups;
+    if (ntiles < ngroups || ntiles > C::NT * ngroups) {
+        if (threadIdx.x == 0) flag_error(kErrPlan);
+        ngroups = 0;
+    }
+    WgradXchg<C::M, C::CLMAX> xg{C::CLMAX > 1 ? cluster_size() : 1u, cluster_rank(), cluster_index(),
+                                 smem_u32(smem + C::OFF_RX), smem_u32(&rx_full), smem_u32(&rx_free[0]), 0};
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < C::NSF; ++s) {
@@ -115,6 +129,8 @@ __global__ void __launch_bounds__(192, 1)
         for (int i = 0; i < 2; ++i) {
             mbar_init(smem_u32(&df_full[i]), 1);
             mbar_init(smem_u32(&df_empty[i]), 128);
+        }
+        for (int i = 0; i < C::NWB; ++i) {
             mbar_init(smem_u32(&we_full[i]), 1);
             mbar_init(smem_u32(&we_empty[i]), 128);
         }
@@ -128,7 +144,9 @@ __global__ void __launch_bounds__(192, 1)
         mbar_init(smem_u32(&w2_full), 1);
         mbar_init(smem_u32(&st_done), 1);
         mbar_init(smem_u32(&done_bar), 1);
+        xg.init_barriers();
         fence_mbar_init();
+        xg.arm_first();
     }
     if (warp == 1) tmem_alloc(smem_u32(&tmem_base_sh), C::TMEM_COLS);
     if (warp >= 2) {  // We2 (m x r) as a swizzled K-major operand
@@ -138,6 +156,7 @@ __global__ void __launch_bounds__(192, 1)
     }
     tc_fence_before();
     __syncthreads();
+    if (C::CLMAX > 1 && xg.cl > 1) cluster_sync();   // every CTA's barriers are initialized before any exchange
     tc_fence_after();
     const uint32_t tmem = tmem_base_sh;
 
@@ -158,7 +177,8 @@ __global__ void __launch_bounds__(192, 1)
                 // the previous group's MMAs are done with the whole ring
                 if (g > 0) ok = mbar_wait(smem_u32(&st_done), (g - 1) & 1);
                 if (!ok) break;
-                const int tb = g * C::NT, te = min(ntiles, tb + C::NT);
+                int tb, te;
+                group_tiles(g, ngroups, ntiles, tb, te);
                 mbar_expect_tx(smem_u32(&db_full), (uint32_t)(te - tb) * C::TILE);
                 for (int i = tb; i < te; ++i)
                     tma_load_2d(smem_u32(smem + C::OFF_DB + (i - tb) * C::TILE), &tm_db, 0,
@@ -252,7 +272,8 @@ __global__ void __launch_bounds__(192, 1)
             uint32_t fpar = 0, wit = 0, cit = 0, dfit = 0, u = 0;
             bool ok = true;
             for (int g = 0; g < ngroups && ok; ++g) {
-                const int tb = g * C::NT, te = min(ntiles, tb + C::NT);
+                int tb, te;
+                group_tiles(g, ngroups, ntiles, tb, te);
                 ok = mbar_wait(smem_u32(&db_full), g & 1);
                 tc_fence_after();
                 // ---- phase 0: dA_tile = dB_tile . We2^T (K = r), a ring of NDA TMEM regions ----
@@ -285,9 +306,9 @@ __global__ void __launch_bounds__(192, 1)
                 // ---- phase 1: the F stream ----
                 uint32_t j = 0;
                 for (int c = 0; c < nch && ok; ++c, ++cit, ++wit) {
-                    const uint32_t sw = wit % C::NW, ae = cit & 1;
+                    const uint32_t sw = wit % C::NW, ae = cit % C::NWB;
                     ok = mbar_wait(smem_u32(&w_full[sw]), (wit / C::NW) & 1) &&
-                         mbar_wait(smem_u32(&we_empty[ae]), ((cit >> 1) & 1) ^ 1);
+                         mbar_wait(smem_u32(&we_empty[ae]), ((cit / C::NWB) & 1) ^ 1);
                     tc_fence_after();
                     const uint64_t wd = wd0 + ((sw * C::W_STAGE) >> 4);
                     const uint32_t d_we = tmem + C::TM_WE + ae * C::MS;
@@ -340,7 +361,8 @@ __global__ void __launch_bounds__(192, 1)
         uint32_t cit = 0, dfit = 0, sit = 0, u = 0;
         bool ok = true;
         for (int g = 0; g < ngroups && ok; ++g) {
-            const int tb = g * C::NT, te = min(ntiles, tb + C::NT);
+            int tb, te;
+            group_tiles(g, ngroups, ntiles, tb, te);
             const int64_t slot = (int64_t)blockIdx.x * a.max_groups + g;
             // ---- phase 0: dP and A = phi(P) of every tile, dX[:, :r] += dB ----
             // the group's P rows and dX[:, :r] rows towards L2 first, so that the per-tile loads
@@ -421,6 +443,18 @@ __global__ void __launch_bounds__(192, 1)
             }
 
             // ---- phase 1: dF tiles out by TMA; dWe1 chunks to the partial slot ----
+            // With a cluster exchange, the rows this CTA sends go out as soon as their chunk is
+            // complete, and the rows it owns are read out after the next chunk's first dF tile
+            // (the peers' rows of that chunk have arrived by then; the accumulator waits in TMEM).
+            const bool defer = xg.exchanging() && xg.owns(row);
+            int pend = -1, pend_cc = 0;
+            auto drain_owned = [&](int buf, int chunk) {
+                float v[C::M];
+                tmem_ld_row<C::M>(tmem + lane_base + C::TM_WE + buf * C::MS, v);
+                tc_fence_before();
+                mbar_arrive(smem_u32(&we_empty[buf]));   // the accumulator is free again
+                return xg.receive(a.wg, v, chunk, row, g == 0);
+            };
             for (int c = 0; c < nch && ok; ++c, ++cit) {
                 const int cc = c + c_first < nch ? c + c_first : c + c_first - nch;
                 for (int i = tb; i < te && ok; ++i, ++dfit) {
@@ -471,17 +505,31 @@ __global__ void __launch_bounds__(192, 1)
                             bulk_commit();
                         }
                     }
+                    if (i == tb && pend >= 0) {
+                        ok = ok && drain_owned(pend, pend_cc);
+                        pend = -1;
+                    }
                 }
-                // the chunk's dWe1 rows (lane = d column) -> the CTA's partial slot
-                const uint32_t ae = cit & 1;
-                ok = ok && mbar_wait(smem_u32(&we_full[ae]), (cit >> 1) & 1);
+                // the chunk's dWe1 rows (lane = d column) -> the cluster's partial slot
+                const uint32_t ae = cit % C::NWB;
+                ok = ok && mbar_wait(smem_u32(&we_full[ae]), (cit / C::NWB) & 1);
                 tc_fence_after();
+                if (defer) {
+                    pend = (int)ae;
+                    pend_cc = cc;
+                    continue;
+                }
                 float v[C::M];
                 tmem_ld_row<C::M>(tmem + lane_base + C::TM_WE + ae * C::MS, v);
                 tc_fence_before();
                 mbar_arrive(smem_u32(&we_empty[ae]));   // the accumulator is free again
-                wgrad_chunk<C::M>(a.wg, v, cc, row, g == 0);
+                if (xg.exchanging()) {
+                    ok = ok && xg.send(v, row);
+                } else {
+                    xg.store_own(a.wg, v, cc, row, g == 0);
+                }
             }
+            if (ok && pend >= 0) ok = drain_owned(pend, pend_cc);   // the group's last chunk
 
             // ---- the group's dWe2 (rows = m, lanes 0 .. m-1) to its partial slot ----
             ok = ok && mbar_wait(smem_u32(&w2_full), g & 1);
@@ -497,10 +545,6 @@ __global__ void __launch_bounds__(192, 1)
             }
             tc_fence_before();
         }
-        for (int g = ngroups; g < a.max_groups; ++g) {
-            const int64_t slot = (int64_t)blockIdx.x * a.max_groups + g;
-            for (int e = et; e < C::M * C::R; e += 128) a.part2[slot * (C::M * C::R) + e] = 0.0f;
-        }
         if (et == 0) bulk_wait<0>();
     }
 
@@ -510,6 +554,7 @@ __global__ void __launch_bounds__(192, 1)
         tc_fence_after();
         tmem_dealloc(tmem, C::TMEM_COLS);
     }
+    if (C::CLMAX > 1 && xg.cl > 1) cluster_sync();   // no peer addresses this CTA's shared memory any more
 }
 
 }  // namespace tc
