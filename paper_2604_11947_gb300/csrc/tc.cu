@@ -109,41 +109,69 @@ cudaError_t ensure_smem(K kernel, uint32_t bytes, int dev, std::atomic<uint8_t> 
     return e;
 }
 
-// CTAs per cluster for a backward kernel: the larger of 4 and 2 (at most clmax) that divides the
-// grid and lets all of the grid's clusters be resident at once (the kernel is persistent, one
-// CTA per SM); otherwise 1. The number of co-resident clusters is asked once per (kernel,
-// device, cluster size); `fit` is the calling launcher's own cache (count + 1; 0: not asked). Needs
-// the kernel's dynamic shared memory attribute set first.
+// Number of clusters of `cl` CTAs of `kernel` (1-D, dynamic shared memory `smem`) that can be
+// resident at once, asked once per (kernel, device, cluster size); `fit` is the calling
+// launcher's own cache (count + 1; 0: not asked; index 0: 4 CTAs, 1: 2 CTAs). Needs the kernel's
+// dynamic shared memory attribute set first. 0 if the query fails.
 template <typename... KArgs>
-int pick_cluster(void (*kernel)(KArgs...), int grid, int threads, uint32_t smem, int clmax, int dev,
-                 std::atomic<int> (&fit)[kMaxDev][2])
+int coresident_clusters(void (*kernel)(KArgs...), int cl, int threads, uint32_t smem, int dev,
+                        std::atomic<int> (&fit)[kMaxDev][2])
 {
-    for (int i = 0; i < 2; ++i) {
-        const int cl = i == 0 ? 4 : 2;
-        if (cl > clmax || grid % cl != 0) continue;
-        const bool cached = dev >= 0 && dev < kMaxDev;
-        int n = cached ? fit[dev][i].load(std::memory_order_acquire) - 1 : -1;
-        if (n < 0) {
-            cudaLaunchConfig_t cfg = {};
-            cfg.gridDim = dim3((unsigned)cl);
-            cfg.blockDim = dim3((unsigned)threads);
-            cfg.dynamicSmemBytes = smem;
-            cudaLaunchAttribute attr[1];
-            attr[0].id = cudaLaunchAttributeClusterDimension;
-            attr[0].val.clusterDim.x = (unsigned)cl;
-            attr[0].val.clusterDim.y = 1;
-            attr[0].val.clusterDim.z = 1;
-            cfg.attrs = attr;
-            cfg.numAttrs = 1;
-            if (cudaOccupancyMaxActiveClusters(&n, kernel, &cfg) != cudaSuccess) {
-                (void)cudaGetLastError();   // not an error of the caller's stream: fall back
-                n = 0;
-            }
-            if (cached) fit[dev][i].store(n + 1, std::memory_order_release);
-        }
-        if ((int64_t)n * cl >= grid) return cl;
+    const int i = cl == 4 ? 0 : 1;
+    const bool cached = dev >= 0 && dev < kMaxDev;
+    int n = cached ? fit[dev][i].load(std::memory_order_acquire) - 1 : -1;
+    if (n >= 0) return n;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)cl);
+    cfg.blockDim = dim3((unsigned)threads);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = (unsigned)cl;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (cudaOccupancyMaxActiveClusters(&n, kernel, &cfg) != cudaSuccess) {
+        (void)cudaGetLastError();   // not an error of the caller's stream: no clusters
+        n = 0;
     }
-    return 1;
+    if (cached) fit[dev][i].store(n + 1, std::memory_order_release);
+    return n;
+}
+
+// Grid and cluster size of a backward launch. The persistent grid would be g_full =
+// min(16-token units, SMs) single CTAs; clusters of 4 are taken when at least 15/16 of g_full
+// CTAs fit as co-resident clusters of 4 (the grid is then that many, a multiple of 4), else
+// clusters of 2 on the same terms, else single CTAs. Fewer, larger weight-gradient partials
+// cost less than the few idle SMs: these kernels are bound by HBM, not by SM count.
+struct BwdShape {
+    int grid, cl;
+};
+int bwd_full_grid(int64_t T, int sms)
+{
+    int64_t g = (T + 15) / 16;
+    if (g > sms) g = sms;
+    return (int)(g < 1 ? 1 : g);
+}
+int bwd_min_grid(int64_t T, int sms)
+{
+    const int gf = bwd_full_grid(T, sms);
+    return (15 * gf + 15) / 16;
+}
+template <typename... KArgs>
+BwdShape bwd_shape(void (*kernel)(KArgs...), int64_t T, int sms, int threads, uint32_t smem, int clmax, int dev,
+                   std::atomic<int> (&fit)[kMaxDev][2])
+{
+    const int gf = bwd_full_grid(T, sms);
+    for (int cl = 4; cl >= 2; cl /= 2) {
+        if (cl > clmax) continue;
+        int64_t g = (int64_t)cl * coresident_clusters(kernel, cl, threads, smem, dev, fit);
+        if (g > gf) g = gf;
+        g -= g % cl;
+        if (g >= cl && 16 * g >= 15 * (int64_t)gf) return BwdShape{(int)g, cl};
+    }
+    return BwdShape{gf, 1};
 }
 
 bool tc_width_ok(int64_t m) { return m == 16 || m == 32 || m == 64 || m == 128; }
@@ -200,32 +228,47 @@ cudaError_t launch_enc_fwd(const resbm_desc &d, const void *X, const void *F, co
 }
 
 // Scratch layout of the backward kernels: the d x m weight gradient has one fp32 slot per
-// cluster (sized for clusters of one CTA; tc_wgrad.cuh); the small one has one slot per (CTA,
-// tile group). Every CTA has max_groups tile groups.
+// cluster (room for g_full single CTAs; tc_wgrad.cuh); the small one has one slot per (CTA, tile
+// group). Every CTA has max_groups tile groups. The scratch size covers every grid the launch
+// may pick (bwd_min_grid .. bwd_full_grid), so it does not depend on the device's occupancy.
 struct BwdPlan {
     int grid = 1, max_groups = 1, nch = 1;
     int64_t slots = 1;              // small partial slots
-    float *part_big = nullptr;      // grid x d x m
+    float *part_big = nullptr;      // g_full x d x m
     float *part_small = nullptr;    // slots x small_elems
     size_t bytes = 0;
 };
 
-BwdPlan bwd_plan(const resbm_desc &d, int sms, int nt, int64_t small_elems, void *ws)
+int bwd_max_groups(int64_t T, int grid, int nt)
+{
+    const int64_t U = (T + 15) / 16;
+    const int64_t max_tokens = 16 * ((U + grid - 1) / grid);
+    const int64_t max_tiles = (max_tokens + 127) / 128;
+    const int64_t g = (max_tiles + nt - 1) / nt;
+    return (int)(g < 1 ? 1 : g);
+}
+
+// grid > 0: the plan of that grid; grid == 0: the scratch size only (the largest over all grids).
+BwdPlan bwd_plan(const resbm_desc &d, int sms, int grid, int nt, int64_t small_elems, void *ws)
 {
     BwdPlan p;
-    int64_t g = (d.T + 15) / 16;
-    if (g > sms) g = sms;
-    p.grid = (int)(g < 1 ? 1 : g);
-    const int64_t U = (d.T + 15) / 16;
-    const int64_t max_tokens = 16 * ((U + p.grid - 1) / p.grid);
-    const int64_t max_tiles = (max_tokens + 127) / 128;
-    p.max_groups = (int)((max_tiles + nt - 1) / nt);
-    if (p.max_groups < 1) p.max_groups = 1;
-    p.slots = (int64_t)p.grid * p.max_groups;
+    const int gf = bwd_full_grid(d.T, sms);
+    int64_t small_slots = 0;
+    if (grid > 0) {
+        p.grid = grid;
+        p.max_groups = bwd_max_groups(d.T, grid, nt);
+        p.slots = (int64_t)grid * p.max_groups;
+        small_slots = p.slots;
+    } else {
+        for (int g = bwd_min_grid(d.T, sms); g <= gf; ++g) {
+            const int64_t s = (int64_t)g * bwd_max_groups(d.T, g, nt);
+            if (s > small_slots) small_slots = s;
+        }
+    }
     p.nch = (int)(d.d / 128);
     WsCarver w(ws);
-    p.part_big = w.take<float>((int64_t)p.grid * d.d * d.m);
-    p.part_small = w.take<float>(p.slots * small_elems);
+    p.part_big = w.take<float>((int64_t)gf * d.d * d.m);
+    p.part_small = w.take<float>(small_slots * small_elems);
     p.bytes = w.used;
     return p;
 }
@@ -257,7 +300,13 @@ cudaError_t launch_dec_bwd(const resbm_desc &d, const void *dY, const void *B, c
                            void *dB, float *dWd1, float *dWd2, void *ws, const Ctx &c)
 {
     using Cfg = tc::DecBwdCfg<M>;
-    const BwdPlan p = bwd_plan(d, c.sm_count, Cfg::NT, d.r * d.m, ws);
+    static std::atomic<uint8_t> smem_set[kMaxDev];
+    cudaError_t e = ensure_smem(tc::k_dec_bwd<M>, Cfg::SMEM_BYTES, c.device, smem_set);
+    if (e != cudaSuccess) return e;
+    static std::atomic<int> fit[kMaxDev][2];
+    const BwdShape sh = bwd_shape(tc::k_dec_bwd<M>, d.T, c.sm_count, Cfg::THREADS, Cfg::SMEM_BYTES, Cfg::CLMAX,
+                                  c.device, fit);
+    const BwdPlan p = bwd_plan(d, c.sm_count, sh.grid, Cfg::NT, d.r * d.m, ws);
     CUtensorMap m_dy128, m_dy16, m_wd2, m_b, m_yr;
     if (!make_map(&m_dy128, dY, d.d, d.T, d.d * 2, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B) ||
         !make_map(&m_dy16, dY, d.d, d.T, d.d * 2, 64, 16, CU_TENSOR_MAP_SWIZZLE_128B) ||
@@ -265,23 +314,18 @@ cudaError_t launch_dec_bwd(const resbm_desc &d, const void *dY, const void *B, c
         !make_map(&m_b, B, d.r, d.T, d.r * 2, M, 128, swizzle_for(Cfg::RB)) ||
         !make_map(&m_yr, dY, d.d, d.T, d.d * 2, M, 128, swizzle_for(Cfg::RB)))
         return cudaErrorInvalidValue;
-    static std::atomic<uint8_t> smem_set[kMaxDev];
-    cudaError_t e = ensure_smem(tc::k_dec_bwd<M>, Cfg::SMEM_BYTES, c.device, smem_set);
-    if (e != cudaSuccess) return e;
     tc::DecBwdArgs a{static_cast<const __nv_bfloat16 *>(Wd1),
                      static_cast<__nv_bfloat16 *>(dB),
                      tc::WgradArgs{p.part_big, p.nch},
                      p.part_small, d.T, d.d, d.act, d.merge_identity, p.max_groups};
-    static std::atomic<int> fit[kMaxDev][2];
-    const int cl = pick_cluster(tc::k_dec_bwd<M>, p.grid, Cfg::THREADS, Cfg::SMEM_BYTES, Cfg::CLMAX, c.device, fit);
-    e = launch_clustered(tc::k_dec_bwd<M>, p.grid, Cfg::THREADS, Cfg::SMEM_BYTES, cl, c.stream, m_dy128, m_dy16, m_wd2,
-                         m_b, m_yr, a);
+    e = launch_clustered(tc::k_dec_bwd<M>, p.grid, Cfg::THREADS, Cfg::SMEM_BYTES, sh.cl, c.stream, m_dy128, m_dy16,
+                         m_wd2, m_b, m_yr, a);
     count_launches(1);
     if (e != cudaSuccess) return e;
     // dWd2 (m x d) = sum of the per-cluster slots (d x m), transposed; dWd1 (r x m) = sum of the slices
     const int64_t cap = (int64_t)c.sm_count * 8;
     return launch_reduce(reduce_job(p.part_small, p.slots, d.r, d.m, dWd1, 0, al16(dWd1), cap),
-                         reduce_job(p.part_big, p.grid / cl, d.d, d.m, dWd2, 1, 0, cap), c);
+                         reduce_job(p.part_big, p.grid / sh.cl, d.d, d.m, dWd2, 1, 0, cap), c);
 }
 
 int dec_bwd_nt(int64_t m)
@@ -296,14 +340,15 @@ struct EncBwdWs {
     size_t bytes;
 };
 
-EncBwdWs enc_bwd_ws(const resbm_desc &d, int sms, void *ws)
+// grid > 0: the plan of that grid; grid == 0: the scratch size only (bwd_plan).
+EncBwdWs enc_bwd_ws(const resbm_desc &d, int sms, int grid, void *ws)
 {
     EncBwdWs w{};
     WsCarver c(ws);
     w.P = c.take<float>(d.T * d.m);
     char *rest = c.take<char>(0);
     const int nt = d.m <= 16 ? tc::EncBwdCfg<16>::NT : d.m <= 32 ? tc::EncBwdCfg<32>::NT : tc::EncBwdCfg<64>::NT;
-    w.plan = bwd_plan(d, sms, nt, d.m * d.r, ws ? rest : nullptr);
+    w.plan = bwd_plan(d, sms, grid, nt, d.m * d.r, ws ? rest : nullptr);
     w.bytes = c.used + w.plan.bytes;
     return w;
 }
@@ -313,7 +358,13 @@ cudaError_t launch_enc_bwd(const resbm_desc &d, const void *dB, const void *F, c
                            const void *We2, void *dF, void *dX, float *dWe1, float *dWe2, void *ws, const Ctx &c)
 {
     using Cfg = tc::EncBwdCfg<M>;
-    const EncBwdWs w = enc_bwd_ws(d, c.sm_count, ws);
+    static std::atomic<uint8_t> smem_set[kMaxDev];
+    cudaError_t e = ensure_smem(tc::k_enc_bwd<M>, Cfg::SMEM_BYTES, c.device, smem_set);
+    if (e != cudaSuccess) return e;
+    static std::atomic<int> fit[kMaxDev][2];
+    const BwdShape sh = bwd_shape(tc::k_enc_bwd<M>, d.T, c.sm_count, Cfg::THREADS, Cfg::SMEM_BYTES, Cfg::CLMAX,
+                                  c.device, fit);
+    const EncBwdWs w = enc_bwd_ws(d, c.sm_count, sh.grid, ws);
     const BwdPlan &p = w.plan;
     CUtensorMap m_f128, m_f16, m_we1, m_df128, m_df16, m_db;
     if (!make_map(&m_f128, F, d.d, d.T, d.d * 2, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B) ||
@@ -323,26 +374,20 @@ cudaError_t launch_enc_bwd(const resbm_desc &d, const void *dB, const void *F, c
         !make_map(&m_df16, dF, d.d, d.T, d.d * 2, 64, 16, CU_TENSOR_MAP_SWIZZLE_128B) ||
         !make_map(&m_db, dB, d.r, d.T, d.r * 2, M, 128, swizzle_for(Cfg::RB)))
         return cudaErrorInvalidValue;
-    cudaError_t e;
     if (!P) {  // P = F . We1 with the forward kernel (no B), so it matches a saved P bit for bit
         e = launch_enc_fwd<M>(d, nullptr, F, We1, We2, nullptr, w.P, c);
         if (e != cudaSuccess) return e;
         P = w.P;
     }
-    static std::atomic<uint8_t> smem_set[kMaxDev];
-    e = ensure_smem(tc::k_enc_bwd<M>, Cfg::SMEM_BYTES, c.device, smem_set);
-    if (e != cudaSuccess) return e;
     tc::EncBwdArgs a{P, static_cast<const __nv_bfloat16 *>(We2), static_cast<__nv_bfloat16 *>(dX),
                      tc::WgradArgs{p.part_big, p.nch}, p.part_small, d.T, d.d, d.act, p.max_groups};
-    static std::atomic<int> fit[kMaxDev][2];
-    const int cl = pick_cluster(tc::k_enc_bwd<M>, p.grid, Cfg::THREADS, Cfg::SMEM_BYTES, Cfg::CLMAX, c.device, fit);
-    e = launch_clustered(tc::k_enc_bwd<M>, p.grid, Cfg::THREADS, Cfg::SMEM_BYTES, cl, c.stream, m_f128, m_f16, m_we1,
-                         m_df128, m_df16, m_db, a);
+    e = launch_clustered(tc::k_enc_bwd<M>, p.grid, Cfg::THREADS, Cfg::SMEM_BYTES, sh.cl, c.stream, m_f128, m_f16,
+                         m_we1, m_df128, m_df16, m_db, a);
     count_launches(1);
     if (e != cudaSuccess) return e;
     const int64_t cap = (int64_t)c.sm_count * 8;
     return launch_reduce(reduce_job(p.part_small, p.slots, d.m, d.r, dWe2, 0, al16(dWe2), cap),
-                         reduce_job(p.part_big, p.grid / cl, d.d, d.m, dWe1, 0, al16(dWe1), cap), c);
+                         reduce_job(p.part_big, p.grid / sh.cl, d.d, d.m, dWe1, 0, al16(dWe1), cap), c);
 }
 
 }  // namespace
@@ -362,8 +407,8 @@ bool tc_supported(const resbm_desc &d, int op)
 
 size_t tc_ws_bytes(const resbm_desc &d, int op, int sms)
 {
-    if (op == RESBM_OP_DECODE_BWD) return bwd_plan(d, sms, dec_bwd_nt(d.m), d.r * d.m, nullptr).bytes;
-    if (op == RESBM_OP_ENCODE_BWD) return enc_bwd_ws(d, sms, nullptr).bytes;
+    if (op == RESBM_OP_DECODE_BWD) return bwd_plan(d, sms, 0, dec_bwd_nt(d.m), d.r * d.m, nullptr).bytes;
+    if (op == RESBM_OP_ENCODE_BWD) return enc_bwd_ws(d, sms, 0, nullptr).bytes;
     return 0;
 }
 

@@ -41,7 +41,7 @@ template <int M_> struct EncBwdCfg {
     static constexpr int NT = M_ <= 32 ? 4 : 2;                  // tiles per group
     static constexpr int NSF = 3;                                // F ring depth
     static constexpr int NW = M_ <= 16 ? 4 : M_ <= 32 ? 2 : 3;   // We1 slice ring depth
-    static constexpr int CLMAX = M_ <= 32 ? 2 : 1;               // CTAs per cluster (weight-gradient exchange)
+    static constexpr int CLMAX = M_ <= 32 ? 4 : 1;               // CTAs per cluster (weight-gradient exchange)
     static constexpr int NWB = CLMAX > 1 ? 3 : 2;                // dWe1 accumulators in TMEM
     static constexpr int NDA = M_ <= 32 ? NT : 1;                // dA TMEM regions (a ring)
     static constexpr bool DPLO = M_ <= 32;                       // dP kept as bf16 hi + lo for dF

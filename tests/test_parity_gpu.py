@@ -27,15 +27,20 @@ SMALL = {
     "bf16_odd_d": synth.BoundaryConfig("bf16_odd_d", T=129, d=100, r=3, m=7),
     "bf16_no_compression": synth.BoundaryConfig("bf16_no_compression", T=200, d=64, r=64, m=16),
     "bf16_r1": synth.BoundaryConfig("bf16_r1", T=64, d=128, r=1, m=1),
-    # ~1000 tokens per CTA on 152 SMs: several groups of tiles per CTA in the backward kernels
-    # (clusters of 4 CTAs when they fit)
+    # ~1000 tokens per CTA: several groups of tiles per CTA in the backward kernels (whose
+    # grids on a 152-SM GB300 are 144 CTAs in clusters of 4)
     "bf16_multi_group": synth.BoundaryConfig("bf16_multi_group", T=150001, d=128, r=32, m=32),
-    # 32 or 33 16-token units per CTA on 152 SMs: 4 or 5 tiles, cut into 2 + 2 or 2 + 3, so the
-    # CTAs of a cluster have different group sizes but the same number of groups
+    # 32 or 33 16-token units per CTA on 152 (or 144) CTAs: 4 or 5 tiles, cut into 2 + 2 or
+    # 3 + 2, so the CTAs of a cluster have different group sizes but the same number of groups
     "bf16_uneven_groups": synth.BoundaryConfig("bf16_uneven_groups", T=79031, d=256, r=32, m=32),
-    # 102 CTAs (a multiple of 2, not of 4): clusters of 2 in the backward kernels
-    "bf16_cluster2": synth.BoundaryConfig("bf16_cluster2", T=1630, d=384, r=32, m=32),
-    "bf16_cluster2_r16": synth.BoundaryConfig("bf16_cluster2_r16", T=1625, d=256, r=16, m=16),
+    "bf16_uneven_groups_144": synth.BoundaryConfig("bf16_uneven_groups_144", T=74871, d=256, r=32, m=32),
+    # 102 units: the backward grid is 100 CTAs in clusters of 4
+    "bf16_cluster4_g100": synth.BoundaryConfig("bf16_cluster4_g100", T=1630, d=384, r=32, m=32),
+    "bf16_cluster4_g100_r16": synth.BoundaryConfig("bf16_cluster4_g100_r16", T=1625, d=256, r=16, m=16),
+    # 18 units: clusters of 4 would leave too many idle (16 < 15/16 x 18), clusters of 2 do not
+    "bf16_cluster2_g18": synth.BoundaryConfig("bf16_cluster2_g18", T=280, d=256, r=32, m=32),
+    # 3 units: single CTAs
+    "bf16_single_ctas": synth.BoundaryConfig("bf16_single_ctas", T=40, d=256, r=32, m=32),
 }
 
 
