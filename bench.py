@@ -4,9 +4,9 @@ decode bwd -> encode bwd (with the weight-gradient reductions) over one batch of
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--config large_bf16] [--impl resbm|reference]
 
-Prints ONE JSON line (rank 0). value = boundary tokens per second over all ranks (inputs
-resident in HBM); `e2e` = the same through resbm_boundary_step with pinned host buffers and the
-host<->device copies inside the timed region; `roofline` = the dominant op's algorithmic HBM
+Prints ONE JSON line (rank 0). value = boundary tokens per second over all ranks, timed over K
+resbm_boundary_step calls (inputs resident in HBM); `e2e` = the same with pinned host buffers and
+the host<->device copies inside the timed region; `roofline` = the dominant op's algorithmic HBM
 bytes / its CUDA-event time against the measured copy bandwidth; `cpu_baseline` = the fp64
 oracle on the host cores, on a bounded token sample. With N > 1 (torchrun) every rank runs an
 independent replica of the workload on its own GPU (the boundary op has no exchange step when
@@ -323,6 +323,12 @@ def main():
         if ev is not None:
             ev[4].record(stream)
 
+    def fused_step():
+        resbm.resbm_boundary_step(desc, ws, X=dev["X"], F=dev["F"], dY=dev["dY"], We1=dev["We1"],
+                                  We2=dev["We2"], Wd1=dev["Wd1"], Wd2=dev["Wd2"], **out)
+
+    for _ in range(max(args.warmup, 0)):
+        fused_step()
     for _ in range(max(args.warmup, 0)):
         step()
     torch.cuda.synchronize()
@@ -338,13 +344,20 @@ def main():
     torch.cuda.synchronize()
     clocks.start()
     time.sleep(0.15)
+    # timed region: K boundary steps through the library's step call, no events in between
+    # (an event between two kernels ends their programmatic-dependent-launch overlap)
     launches0 = resbm.resbm_kernel_launches()
     start.record(stream)
     for i in range(args.steps):
-        step(evs[i])
+        fused_step()
     end.record(stream)
     torch.cuda.synchronize()
     launches = resbm.resbm_kernel_launches() - launches0
+    # second timed pass, same K steps as four op calls with events between them: the per-op
+    # times of the roofline (these steps are a few percent slower than the ones above)
+    for i in range(args.steps):
+        step(evs[i])
+    torch.cuda.synchronize()
     if dist:
         dist.barrier()
     clk = clocks.stop()
@@ -365,6 +378,8 @@ def main():
                 "traffic": traffic_for(dom, cfg),
                 "peak_source": peaks["source"] + " copy bandwidth (MEASURED_PEAKS.json hbm_gbs)",
                 "algorithmic_bytes_per_launch": bytes_[dom],
+                "timing": "per-op CUDA events on the launching stream in a second timed pass "
+                          "of the same K steps (op calls with events between them)",
                 "per_op": {o: {"ms": op_ms[o], "alg_bytes": bytes_[o],
                                "GBps": bytes_[o] / (op_ms[o] / 1e3) / 1e9,
                                "frac": bytes_[o] / (op_ms[o] / 1e3) / 1e9 / peaks["hbm_gbs"],
