@@ -410,43 +410,28 @@ def main():
 
 
 def run_e2e(args, cfg, desc, dev, out, ws, resbm, torch, dist, world):
-    """Same step through resbm_boundary_step from pinned host buffers: every step copies its
-    inputs host->device and its results device->host inside the timed region. The steps are
-    pipelined as a training loop would run them: H2D, compute and D2H on three streams with two
-    sets of device buffers, so step i+1's inputs travel while step i computes and step i-1's
-    results travel back."""
+    """The same step through the C ABI with HOST buffers (resbm_boundary_step_host): inputs in
+    pinned host memory, results back into pinned host memory, every copy inside the call and
+    inside the timed region. Two calls are kept in flight (two streams, two device workspaces,
+    two sets of host results), so one step's results travel back while the next step's inputs
+    travel in, as a training loop fed from the host would run them."""
     ins = ("X", "F", "dY", "We1", "We2", "Wd1", "Wd2")
     res = ("B", "Y", "dB", "dF", "dWe1", "dWe2", "dWd1", "dWd2")
     host_in = {k: dev[k].cpu().pin_memory() for k in ins}
-    h2d = sum(t.numel() * t.element_size() for t in host_in.values())
-    sets = [(dev, {k: v for k, v in out.items() if k != "dX"})]
-    sets.append(({k: torch.empty_like(v) for k, v in dev.items()},
-                 {k: torch.empty_like(v) for k, v in out.items() if k != "dX"}))
-    host_out = [{k: torch.empty(o[k].shape, dtype=o[k].dtype).pin_memory() for k in res} for _, o in sets]
+    host_out = [{k: torch.empty(out[k].shape, dtype=out[k].dtype).pin_memory() for k in res}
+                for _ in range(2)]
+    wss = [resbm.workspace(desc, resbm.RESBM_OP_BOUNDARY_STEP_HOST) for _ in range(2)]
+    streams = [torch.cuda.Stream() for _ in range(2)]
+    es = host_in["F"].element_size()
+    # what the call copies: X[:, :r] only (the identity path), F, dY and the weights in; the
+    # results out
+    h2d = cfg.T * cfg.r * es + sum(host_in[k].numel() * es for k in ins if k != "X")
     d2h = sum(t.numel() * t.element_size() for t in host_out[0].values())
-    s_in, s_comp, s_out = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
-    ev = {n: [torch.cuda.Event() for _ in range(2)] for n in ("in", "comp", "out")}
     n = max(2, min(args.steps, 20))
 
     def step(i):
         b = i % 2
-        di, do = sets[b]
-        with torch.cuda.stream(s_in):
-            if i >= 2:
-                s_in.wait_event(ev["comp"][b])      # step i-2 no longer reads these inputs
-            for k in ins:
-                di[k].copy_(host_in[k], non_blocking=True)
-            ev["in"][b].record(s_in)
-        s_comp.wait_event(ev["in"][b])
-        if i >= 2:
-            s_comp.wait_event(ev["out"][b])         # step i-2's results have left these buffers
-        resbm.resbm_boundary_step(desc, ws, stream=s_comp, **{k: di[k] for k in ins}, **do)
-        ev["comp"][b].record(s_comp)
-        with torch.cuda.stream(s_out):
-            s_out.wait_event(ev["comp"][b])
-            for k in res:
-                host_out[b][k].copy_(do[k], non_blocking=True)
-            ev["out"][b].record(s_out)
+        resbm.resbm_boundary_step_host(desc, wss[b], stream=streams[b], **host_in, **host_out[b])
 
     for i in range(2):
         step(i)
@@ -461,7 +446,8 @@ def run_e2e(args, cfg, desc, dev, out, ws, resbm, torch, dist, world):
     return {"value": job_throughput(cfg.T, world, n, ms), "unit": "tokens/s",
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": n,
             "ms_per_step": ms / n,
-            "pipelined": "H2D, compute and D2H on three streams, two device buffer sets; "
+            "api": "resbm_boundary_step_host (host buffers; copies inside the call)",
+            "pipelined": "two calls in flight on two streams with two device workspaces; "
                          "host wall clock from the first copy to the last result on the host"}
 
 

@@ -80,7 +80,8 @@ typedef enum {
     RESBM_OP_DECODE_FWD = 1,
     RESBM_OP_DECODE_BWD = 2,
     RESBM_OP_ENCODE_BWD = 3,
-    RESBM_OP_BOUNDARY_STEP = 4
+    RESBM_OP_BOUNDARY_STEP = 4,
+    RESBM_OP_BOUNDARY_STEP_HOST = 5
 } resbm_op;
 
 /* desc.flags bits */
@@ -217,6 +218,28 @@ RESBM_API resbm_status resbm_decode_bwd_noalloc(const resbm_desc *desc, const vo
  * encoder backward reads. */
 RESBM_API resbm_status resbm_boundary_step(const resbm_desc *desc, const resbm_step_args *args,
                                  void *ws, size_t ws_bytes, void *stream);
+
+/* resbm_boundary_step with every tensor of `args` in HOST memory. The paper has no counterpart:
+ * this is the host-memory form of the step, a library convenience for callers whose tensors
+ * live on the host (and the form the end-to-end measurement goes through).
+ *   - Same arguments, rules and results as resbm_boundary_step, except that every pointer in
+ *     `args` is a host pointer. Page-locked memory (cudaHostAlloc, cudaHostRegister) lets the
+ *     copies run asynchronously; with pageable memory they block the calling thread.
+ *   - `ws` is DEVICE memory of resbm_workspace_bytes(desc, RESBM_OP_BOUNDARY_STEP_HOST) bytes
+ *     (256-byte aligned): a device copy of every tensor of the step plus the step's own scratch.
+ *   - Only what the step reads crosses to the device: X[:, :r] (the identity path is the only
+ *     use of X), F, dY, the weights, and dX[:, :r] when dX is given; what comes back is B, Y, dB,
+ *     dF, dX[:, :r] (dX given), P (P given) and the weight gradients. The rest of dX is not
+ *     touched.
+ *   - Everything is enqueued on `stream` (the call returns once it is enqueued; the host
+ *     outputs are complete when `stream` reaches that point). Inside the call dY travels on a
+ *     second stream while the forward stages run, and B and Y travel back on a third while the
+ *     backward stages run; both are forked from and joined back into `stream`. Calls on
+ *     different streams with different workspaces may run at the same time, so a caller can
+ *     overlap one step's results with the next step's inputs.
+ *   - Errors: as resbm_boundary_step; RESBM_ERR_CUDA if a copy or a stream could not be set up. */
+RESBM_API resbm_status resbm_boundary_step_host(const resbm_desc *desc, const resbm_step_args *args,
+                                      void *ws, size_t ws_bytes, void *stream);
 
 #ifdef __cplusplus
 }

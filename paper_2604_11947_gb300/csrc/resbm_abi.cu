@@ -179,9 +179,13 @@ size_t step_ws_bytes(const resbm_desc &d)
     return w.used;
 }
 
+size_t host_stage_bytes(const resbm_desc &d);   // resbm_boundary_step_host's workspace
+
 resbm_status check_ws(const resbm_desc &d, int op, void *ws, size_t ws_bytes)
 {
-    size_t need = op == RESBM_OP_BOUNDARY_STEP ? step_ws_bytes(d) : ws_for(d, op);
+    size_t need = op == RESBM_OP_BOUNDARY_STEP_HOST ? host_stage_bytes(d)
+                  : op == RESBM_OP_BOUNDARY_STEP    ? step_ws_bytes(d)
+                                                    : ws_for(d, op);
     if (need == 0) return RESBM_OK;
     if (!ws || ws_bytes < need) return RESBM_ERR_WORKSPACE;
     if (reinterpret_cast<uintptr_t>(ws) % 256) return RESBM_ERR_INVALID_ARG;
@@ -357,6 +361,102 @@ resbm_status exec_encode_bwd(const resbm_desc &d, const void *dB, const void *F,
                                           l.inner, c);
 }
 
+// ---- the boundary step (device or host buffers) ---------------------------------------------
+// All four stages' checks, and no output overlapping another output or an input.
+resbm_status validate_step(const resbm_desc &d, const resbm_step_args *a)
+{
+    resbm_status s = validate_encode_fwd(d, a->X, a->F, a->We1, a->We2, a->B, a->P);
+    if (s == RESBM_OK) s = validate_decode_fwd(d, a->B, a->Wd1, a->Wd2, a->Y);
+    if (s == RESBM_OK) s = validate_decode_bwd(d, a->dY, a->B, a->Wd1, a->Wd2, a->dB, a->dWd1, a->dWd2);
+    if (s == RESBM_OK)
+        s = validate_encode_bwd(d, a->dB, a->F, a->P, a->We1, a->We2, a->dF, a->dX, a->dWe1, a->dWe2);
+    if (s == RESBM_OK) {
+        const size_t es = elem_size(d);
+        const Range outs[] = {rng(a->B, d.T * d.r, es), rng(a->P, d.T * d.m, 4),
+                              rng(a->Y, d.T * d.d, es), rng(a->dB, d.T * d.r, es),
+                              rng(a->dF, d.T * d.d, es), rng(a->dX, d.T * d.d, es),
+                              rng(a->dWe1, d.d * d.m, 4), rng(a->dWe2, d.m * d.r, 4),
+                              rng(a->dWd1, d.r * d.m, 4), rng(a->dWd2, d.m * d.d, 4)};
+        const Range ins[] = {rng(a->X, d.T * d.d, es), rng(a->F, d.T * d.d, es),
+                             rng(a->dY, d.T * d.d, es)};
+        if (any_overlap(outs, ins, 3)) s = RESBM_ERR_INVALID_ARG;
+    }
+    return s;
+}
+
+// Enqueues the four stages on c.stream (device pointers, validated). With fwd_done, records it
+// after the forward stages; with bwd_ready, the backward stages wait for it.
+resbm_status enqueue_step(const resbm_desc &d, const resbm_step_args &a, void *ws, const Ctx &c,
+                          cudaEvent_t fwd_done, cudaEvent_t bwd_ready)
+{
+    WsCarver w(ws);
+    float *P = a.P ? a.P : w.take<float>(d.T * d.m);
+    void *inner = w.take<char>(0);
+    const void *We2 = a.We2, *Wd1 = a.Wd1;
+    float *dWe2 = a.dWe2, *dWd1 = a.dWd1;
+    const resbm_desc e = two_layer(d);
+    resbm_status s = RESBM_OK;
+    if (is_linear(d)) {
+        const LinearWs l = carve_linear(d, inner);
+        s = finish(fill_identity(d, l.I, c));
+        We2 = Wd1 = l.I;
+        dWe2 = l.dW2;
+        dWd1 = l.dW1;
+        inner = l.inner;
+    }
+    if (s == RESBM_OK) s = run_encode_fwd(e, a.X, a.F, a.We1, We2, a.B, P, inner, c);
+    if (s == RESBM_OK) s = run_decode_fwd(e, a.B, Wd1, a.Wd2, a.Y, inner, c);
+    if (s == RESBM_OK && fwd_done) s = finish(cudaEventRecord(fwd_done, c.stream));
+    if (s == RESBM_OK && bwd_ready) s = finish(cudaStreamWaitEvent(c.stream, bwd_ready, 0));
+    if (s == RESBM_OK) s = run_decode_bwd(e, a.dY, a.B, Wd1, a.Wd2, a.dB, dWd1, a.dWd2, inner, c);
+    if (s == RESBM_OK)
+        s = run_encode_bwd(e, a.dB, a.F, P, a.We1, We2, a.dF, a.dX, a.dWe1, dWe2, inner, c);
+    return s;
+}
+
+// Device staging of resbm_boundary_step_host: a device copy of every tensor of the step (X and
+// dX full T x d, of which only the first r columns are copied), then the step's own scratch.
+struct HostStage {
+    resbm_step_args dev;
+    void *inner;
+    size_t bytes;
+};
+HostStage carve_host_stage(const resbm_desc &d, void *ws, const resbm_step_args &host)
+{
+    const size_t es = elem_size(d);
+    const int64_t T = d.T, D = d.d, r = d.r, m = d.m;
+    WsCarver w(ws);
+    HostStage h{};
+    h.dev.X = w.take<char>((size_t)(T * D) * es);
+    h.dev.F = w.take<char>((size_t)(T * D) * es);
+    h.dev.dY = w.take<char>((size_t)(T * D) * es);
+    h.dev.We1 = w.take<char>((size_t)(D * m) * es);
+    h.dev.We2 = w.take<char>((size_t)(m * r) * es);
+    h.dev.Wd1 = w.take<char>((size_t)(r * m) * es);
+    h.dev.Wd2 = w.take<char>((size_t)(m * D) * es);
+    h.dev.B = w.take<char>((size_t)(T * r) * es);
+    h.dev.P = w.take<float>(T * m);
+    h.dev.Y = w.take<char>((size_t)(T * D) * es);
+    h.dev.dB = w.take<char>((size_t)(T * r) * es);
+    h.dev.dF = w.take<char>((size_t)(T * D) * es);
+    void *dX = w.take<char>((size_t)(T * D) * es);
+    h.dev.dX = host.dX ? dX : nullptr;
+    h.dev.dWe1 = w.take<float>(D * m);
+    h.dev.dWe2 = w.take<float>(m * r);
+    h.dev.dWd1 = w.take<float>(r * m);
+    h.dev.dWd2 = w.take<float>(m * D);
+    if (is_linear(d)) {   // one linear layer: the second-layer weights are not read
+        h.dev.We2 = h.dev.Wd1 = nullptr;
+        h.dev.dWe2 = h.dev.dWd1 = nullptr;
+    }
+    h.inner = w.take<char>(0);
+    w.take<char>(step_ws_bytes(d));
+    h.bytes = w.used;
+    return h;
+}
+
+size_t host_stage_bytes(const resbm_desc &d) { return carve_host_stage(d, nullptr, resbm_step_args{}).bytes; }
+
 // ---- fixed scratch of resbm_decode_bwd_noalloc -----------------------------------------------
 // One array per device, reserved with the library's device code; its address is looked up on
 // the first call on each device and kept (all host threads share the cached value).
@@ -417,9 +517,11 @@ resbm_status resbm_workspace_bytes(const resbm_desc *desc, int op, size_t *bytes
 {
     resbm_status s = check_desc(desc);
     if (s != RESBM_OK) return s;
-    if (!bytes || op < RESBM_OP_ENCODE_FWD || op > RESBM_OP_BOUNDARY_STEP)
+    if (!bytes || op < RESBM_OP_ENCODE_FWD || op > RESBM_OP_BOUNDARY_STEP_HOST)
         return RESBM_ERR_INVALID_ARG;
-    *bytes = op == RESBM_OP_BOUNDARY_STEP ? step_ws_bytes(*desc) : ws_for(*desc, op);
+    *bytes = op == RESBM_OP_BOUNDARY_STEP_HOST ? host_stage_bytes(*desc)
+             : op == RESBM_OP_BOUNDARY_STEP    ? step_ws_bytes(*desc)
+                                               : ws_for(*desc, op);
     return RESBM_OK;
 }
 
@@ -501,49 +603,84 @@ resbm_status resbm_boundary_step(const resbm_desc *desc, const resbm_step_args *
     if (!a) return RESBM_ERR_INVALID_ARG;
     const resbm_desc &d = *desc;
     s = check_ws(d, RESBM_OP_BOUNDARY_STEP, ws, ws_bytes);
-    if (s != RESBM_OK) return s;
-    WsCarver w(ws);
-    float *P = a->P ? a->P : w.take<float>(d.T * d.m);
-    void *inner = w.take<char>(0);
-    // validate all four stages before enqueueing anything
-    s = validate_encode_fwd(d, a->X, a->F, a->We1, a->We2, a->B, a->P);
-    if (s == RESBM_OK) s = validate_decode_fwd(d, a->B, a->Wd1, a->Wd2, a->Y);
-    if (s == RESBM_OK)
-        s = validate_decode_bwd(d, a->dY, a->B, a->Wd1, a->Wd2, a->dB, a->dWd1, a->dWd2);
-    if (s == RESBM_OK)
-        s = validate_encode_bwd(d, a->dB, a->F, a->P, a->We1, a->We2, a->dF, a->dX, a->dWe1,
-                                a->dWe2);
-    if (s == RESBM_OK) {
-        // outputs of different stages must not overlap each other or the step's inputs
-        const size_t es = elem_size(d);
-        const Range outs[] = {rng(a->B, d.T * d.r, es), rng(a->P, d.T * d.m, 4),
-                              rng(a->Y, d.T * d.d, es), rng(a->dB, d.T * d.r, es),
-                              rng(a->dF, d.T * d.d, es), rng(a->dX, d.T * d.d, es),
-                              rng(a->dWe1, d.d * d.m, 4), rng(a->dWe2, d.m * d.r, 4),
-                              rng(a->dWd1, d.r * d.m, 4), rng(a->dWd2, d.m * d.d, 4)};
-        const Range ins[] = {rng(a->X, d.T * d.d, es), rng(a->F, d.T * d.d, es),
-                             rng(a->dY, d.T * d.d, es)};
-        if (any_overlap(outs, ins, 3)) s = RESBM_ERR_INVALID_ARG;
-    }
+    if (s == RESBM_OK) s = validate_step(d, a);
     Ctx c;
     if (s == RESBM_OK) s = make_ctx(stream, &c);
-    const void *We2 = a->We2, *Wd1 = a->Wd1;
-    float *dWe2 = a->dWe2, *dWd1 = a->dWd1;
-    const resbm_desc e = two_layer(d);
-    if (s == RESBM_OK && is_linear(d)) {
-        const LinearWs l = carve_linear(d, inner);
-        s = finish(fill_identity(d, l.I, c));
-        We2 = Wd1 = l.I;
-        dWe2 = l.dW2;
-        dWd1 = l.dW1;
-        inner = l.inner;
+    return s == RESBM_OK ? enqueue_step(d, *a, ws, c, nullptr, nullptr) : s;
+}
+
+resbm_status resbm_boundary_step_host(const resbm_desc *desc, const resbm_step_args *a, void *ws,
+                                      size_t ws_bytes, void *stream)
+{
+    resbm_status s = check_desc(desc);
+    if (s != RESBM_OK) return s;
+    if (!a) return RESBM_ERR_INVALID_ARG;
+    const resbm_desc &d = *desc;
+    s = check_ws(d, RESBM_OP_BOUNDARY_STEP_HOST, ws, ws_bytes);
+    if (s == RESBM_OK) s = validate_step(d, a);
+    Ctx c;
+    if (s == RESBM_OK) s = make_ctx(stream, &c);
+    if (s != RESBM_OK) return s;
+    const HostStage hs = carve_host_stage(d, ws, *a);
+    const resbm_step_args &dv = hs.dev;
+    const size_t es = elem_size(d);
+    const int64_t T = d.T, D = d.d, r = d.r, m = d.m;
+    const bool lin = is_linear(d);
+    // two streams of this call (released once their work is done), forked from and joined
+    // back into the caller's stream
+    cudaStream_t s_in = nullptr, s_out = nullptr;
+    cudaEvent_t ev[4] = {};
+    cudaError_t e = cudaStreamCreateWithFlags(&s_in, cudaStreamNonBlocking);
+    if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&s_out, cudaStreamNonBlocking);
+    for (int i = 0; i < 4 && e == cudaSuccess; ++i) e = cudaEventCreateWithFlags(&ev[i], cudaEventDisableTiming);
+    cudaEvent_t fork = ev[0], dy_in = ev[1], fwd_done = ev[2], out_done = ev[3];
+    auto h2d = [&](void *dst, const void *src, size_t bytes, cudaStream_t st) {
+        if (e == cudaSuccess && bytes) e = cudaMemcpyAsync(dst, src, bytes, cudaMemcpyHostToDevice, st);
+    };
+    auto d2h = [&](void *dst, const void *src, size_t bytes, cudaStream_t st) {
+        if (e == cudaSuccess && bytes && dst) e = cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDeviceToHost, st);
+    };
+    // the first r columns of a T x d matrix (rows d * es bytes apart), either way
+    auto cols = [&](void *dst, const void *src, cudaMemcpyKind k, cudaStream_t st) {
+        if (e == cudaSuccess && T > 0)
+            e = cudaMemcpy2DAsync(dst, (size_t)D * es, src, (size_t)D * es, (size_t)r * es, (size_t)T, k, st);
+    };
+    // inputs: dY on the second stream, the rest on the caller's
+    if (e == cudaSuccess) e = cudaEventRecord(fork, c.stream);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(s_in, fork, 0);
+    h2d(const_cast<void *>(dv.dY), a->dY, (size_t)(T * D) * es, s_in);
+    if (e == cudaSuccess) e = cudaEventRecord(dy_in, s_in);
+    h2d(const_cast<void *>(dv.We1), a->We1, (size_t)(D * m) * es, c.stream);
+    if (!lin) h2d(const_cast<void *>(dv.We2), a->We2, (size_t)(m * r) * es, c.stream);
+    if (!lin) h2d(const_cast<void *>(dv.Wd1), a->Wd1, (size_t)(r * m) * es, c.stream);
+    h2d(const_cast<void *>(dv.Wd2), a->Wd2, (size_t)(m * D) * es, c.stream);
+    cols(const_cast<void *>(dv.X), a->X, cudaMemcpyHostToDevice, c.stream);   // the identity path reads X[:, :r] only
+    h2d(const_cast<void *>(dv.F), a->F, (size_t)(T * D) * es, c.stream);
+    if (a->dX) cols(dv.dX, a->dX, cudaMemcpyHostToDevice, c.stream);          // the step adds dB to dX[:, :r] only
+    if (e != cudaSuccess) s = cuda_fail(e);
+    // the step, the forward results leaving on the third stream while the backward runs
+    if (s == RESBM_OK) s = enqueue_step(d, dv, hs.inner, c, fwd_done, dy_in);
+    if (s == RESBM_OK) {
+        e = cudaStreamWaitEvent(s_out, fwd_done, 0);
+        d2h(a->B, dv.B, (size_t)(T * r) * es, s_out);
+        d2h(a->Y, dv.Y, (size_t)(T * D) * es, s_out);
+        if (e == cudaSuccess) e = cudaEventRecord(out_done, s_out);
+        d2h(a->dB, dv.dB, (size_t)(T * r) * es, c.stream);
+        d2h(a->dF, dv.dF, (size_t)(T * D) * es, c.stream);
+        if (a->dX) cols(a->dX, dv.dX, cudaMemcpyDeviceToHost, c.stream);
+        d2h(a->P, dv.P, (size_t)(T * m) * 4, c.stream);
+        d2h(a->dWe1, dv.dWe1, (size_t)(D * m) * 4, c.stream);
+        if (!lin) d2h(a->dWe2, dv.dWe2, (size_t)(m * r) * 4, c.stream);
+        if (!lin) d2h(a->dWd1, dv.dWd1, (size_t)(r * m) * 4, c.stream);
+        d2h(a->dWd2, dv.dWd2, (size_t)(m * D) * 4, c.stream);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(c.stream, out_done, 0);
+        if (e != cudaSuccess) s = cuda_fail(e);
     }
-    if (s == RESBM_OK) s = run_encode_fwd(e, a->X, a->F, a->We1, We2, a->B, P, inner, c);
-    if (s == RESBM_OK) s = run_decode_fwd(e, a->B, Wd1, a->Wd2, a->Y, inner, c);
-    if (s == RESBM_OK)
-        s = run_decode_bwd(e, a->dY, a->B, Wd1, a->Wd2, a->dB, dWd1, a->dWd2, inner, c);
-    if (s == RESBM_OK)
-        s = run_encode_bwd(e, a->dB, a->F, P, a->We1, We2, a->dF, a->dX, a->dWe1, dWe2, inner, c);
+    // streams and events are released by the runtime once the work queued on them is done
+    for (cudaEvent_t x : ev)
+        if (x) cudaEventDestroy(x);
+    if (s_in) cudaStreamDestroy(s_in);
+    if (s_out) cudaStreamDestroy(s_out);
     return s;
 }
 

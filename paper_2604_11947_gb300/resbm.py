@@ -18,7 +18,7 @@ RESBM_OK, RESBM_ERR_INVALID_ARG, RESBM_ERR_UNSUPPORTED, RESBM_ERR_WORKSPACE, RES
 RESBM_F32, RESBM_BF16 = 0, 1
 RESBM_ACT_SILU, RESBM_ACT_GELU_TANH, RESBM_ACT_IDENTITY = 0, 1, 2
 (RESBM_OP_ENCODE_FWD, RESBM_OP_DECODE_FWD, RESBM_OP_DECODE_BWD, RESBM_OP_ENCODE_BWD,
- RESBM_OP_BOUNDARY_STEP) = range(5)
+ RESBM_OP_BOUNDARY_STEP, RESBM_OP_BOUNDARY_STEP_HOST) = range(6)
 RESBM_FLAG_GENERIC = 1
 RESBM_FLAG_LINEAR = 2
 RESBM_STATIC_SCRATCH_BYTES = 32 << 20
@@ -30,8 +30,8 @@ TORCH_DTYPES = {RESBM_F32: torch.float32, RESBM_BF16: torch.bfloat16}
 EXPORTS = ("resbm_version", "resbm_status_string", "resbm_last_cuda_error", "resbm_kernel_launches",
            "resbm_device_error",
            "resbm_workspace_bytes", "resbm_encode_fwd", "resbm_decode_fwd", "resbm_decode_bwd",
-           "resbm_encode_bwd", "resbm_boundary_step", "resbm_decode_bwd_noalloc",
-           "resbm_selftest_wait_timeout")
+           "resbm_encode_bwd", "resbm_boundary_step", "resbm_boundary_step_host",
+           "resbm_decode_bwd_noalloc", "resbm_selftest_wait_timeout")
 
 
 class resbm_desc(ctypes.Structure):
@@ -97,6 +97,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.resbm_decode_bwd_noalloc.restype = i32
     lib.resbm_decode_bwd_noalloc.argtypes = [D] + [vp] * 7 + [vp]
     lib.resbm_boundary_step.argtypes = [D, ctypes.POINTER(resbm_step_args), vp, sz, vp]
+    lib.resbm_boundary_step_host.restype = i32
+    lib.resbm_boundary_step_host.argtypes = [D, ctypes.POINTER(resbm_step_args), vp, sz, vp]
     if path is None:
         _lib = lib
     return lib
@@ -212,6 +214,15 @@ def resbm_boundary_step(desc, ws, stream=None, **tensors):
     st = load().resbm_boundary_step(ctypes.byref(desc), ctypes.byref(args), _p(ws), _nbytes(ws),
                                     _stream(stream))
     _check("resbm_boundary_step", st)
+
+
+def resbm_boundary_step_host(desc, ws, stream=None, **tensors):
+    """resbm_boundary_step with host tensors (CPU torch tensors, pinned for asynchronous
+    copies); ws is the device workspace of RESBM_OP_BOUNDARY_STEP_HOST."""
+    args = resbm_step_args(**{k: _p(v) for k, v in tensors.items()})
+    st = load().resbm_boundary_step_host(ctypes.byref(desc), ctypes.byref(args), _p(ws), _nbytes(ws),
+                                         _stream(stream))
+    _check("resbm_boundary_step_host", st)
 
 
 # ---- convenience: output buffers of one boundary step (allocated by torch) -------------------

@@ -24,7 +24,7 @@ def declared_functions():
 
 def test_exports_every_declared_symbol(lib):
     names = declared_functions()
-    assert len(names) == 13, names
+    assert len(names) == 14, names
     assert sorted(resbm.EXPORTS) == names
     for n in names:
         assert hasattr(lib, n), n
@@ -44,13 +44,16 @@ def test_struct_layout_matches_header():
     assert ctypes.sizeof(resbm.resbm_step_args) == 17 * ctypes.sizeof(ctypes.c_void_p)
 
 
-@pytest.mark.parametrize("op", range(5))
+@pytest.mark.parametrize("op", range(6))
 def test_workspace_query(lib, op):
     d = resbm.make_desc(65536, 4096, 32, 32)
     n = resbm.resbm_workspace_bytes(d, op)
     assert n >= 0
     if op in (resbm.RESBM_OP_DECODE_BWD, resbm.RESBM_OP_ENCODE_BWD, resbm.RESBM_OP_BOUNDARY_STEP):
         assert n > 0
+    if op == resbm.RESBM_OP_BOUNDARY_STEP_HOST:
+        # device copies of X, F, dY, Y, dF, dX (T x d each) on top of the device step's scratch
+        assert n >= 6 * 65536 * 4096 * 2 + resbm.resbm_workspace_bytes(d, resbm.RESBM_OP_BOUNDARY_STEP)
     d0 = resbm.make_desc(0, 4096, 32, 32)
     assert resbm.resbm_workspace_bytes(d0, op) >= 0
 
@@ -73,7 +76,8 @@ def test_bad_descriptor_rejected(lib, bad):
 def test_bad_op_and_null_desc(lib):
     d = resbm.make_desc(16, 64, 8, 8)
     out = ctypes.c_size_t(0)
-    assert lib.resbm_workspace_bytes(ctypes.byref(d), 5, ctypes.byref(out)) == resbm.RESBM_ERR_INVALID_ARG
+    assert lib.resbm_workspace_bytes(ctypes.byref(d), 6, ctypes.byref(out)) == resbm.RESBM_ERR_INVALID_ARG
+    assert lib.resbm_workspace_bytes(ctypes.byref(d), -1, ctypes.byref(out)) == resbm.RESBM_ERR_INVALID_ARG
     assert lib.resbm_workspace_bytes(None, 0, ctypes.byref(out)) == resbm.RESBM_ERR_INVALID_ARG
     assert lib.resbm_workspace_bytes(ctypes.byref(d), 0, None) == resbm.RESBM_ERR_INVALID_ARG
     assert lib.resbm_encode_fwd(None, 1, 1, 1, 1, 1, None, None, 0, None) == resbm.RESBM_ERR_INVALID_ARG
@@ -135,6 +139,17 @@ def test_step_rejects_output_aliasing_input(lib):
     st = lib.resbm_boundary_step(ctypes.byref(d), ctypes.byref(args), 1 << 40, need, None)
     assert st == resbm.RESBM_ERR_INVALID_ARG
     assert lib.resbm_boundary_step(ctypes.byref(d), None, 1 << 40, need, None) == resbm.RESBM_ERR_INVALID_ARG
+    # the host-buffer form applies the same rules, before any copy or stream is set up
+    need_h = resbm.resbm_workspace_bytes(d, resbm.RESBM_OP_BOUNDARY_STEP_HOST)
+    st = lib.resbm_boundary_step_host(ctypes.byref(d), ctypes.byref(args), 1 << 40, need_h, None)
+    assert st == resbm.RESBM_ERR_INVALID_ARG
+    ptrs["dF"] = A + 11 * big
+    ok_args = resbm.resbm_step_args(**ptrs)
+    st = lib.resbm_boundary_step_host(ctypes.byref(d), ctypes.byref(ok_args), 1 << 40, need_h - 1, None)
+    assert st == resbm.RESBM_ERR_WORKSPACE
+    st = lib.resbm_boundary_step_host(ctypes.byref(d), ctypes.byref(ok_args), None, need_h, None)
+    assert st == resbm.RESBM_ERR_WORKSPACE
+    assert lib.resbm_boundary_step_host(ctypes.byref(d), None, 1 << 40, need_h, None) == resbm.RESBM_ERR_INVALID_ARG
 
 
 def test_linear_flag_rules(lib):
