@@ -8,6 +8,7 @@
 #include <cuda_runtime.h>
 
 #include <atomic>
+#include <cstdlib>
 #include <mutex>
 #include <utility>
 
@@ -142,12 +143,23 @@ int coresident_clusters(void (*kernel)(KArgs...), int cl, int threads, uint32_t 
 
 // Grid and cluster size of a backward launch. The persistent grid would be g_full =
 // min(16-token units, SMs) single CTAs; clusters of 4 are taken when at least 15/16 of g_full
-// CTAs fit as co-resident clusters of 4 (the grid is then that many, a multiple of 4), else
-// clusters of 2 on the same terms, else single CTAs. Fewer, larger weight-gradient partials
-// cost less than the few idle SMs: these kernels are bound by HBM, not by SM count.
+// CTAs fit as co-resident clusters of 4 (the grid is then that many, a multiple of 4) and each
+// CTA still gets at least `min_tokens` tokens, else clusters of 2 on the same terms, else single
+// CTAs. Fewer, larger weight-gradient partials cost less than the few idle SMs (these kernels
+// are bound by HBM, not by SM count), but the exchange has a cost per d chunk that only a long
+// enough token range per CTA hides: min_tokens is the kernel's measured crossover.
 struct BwdShape {
     int grid, cl;
 };
+// RESBM_BWD_CLUSTER=1, 2 or 4 forces that cluster size (within the co-residency rule above,
+// regardless of min_tokens); unset or anything else: automatic. Read at every launch.
+int forced_cluster()
+{
+    const char *v = getenv("RESBM_BWD_CLUSTER");
+    if (!v) return 0;
+    const int n = atoi(v);
+    return n == 1 || n == 2 || n == 4 ? n : 0;
+}
 int bwd_full_grid(int64_t T, int sms)
 {
     int64_t g = (T + 15) / 16;
@@ -160,16 +172,17 @@ int bwd_min_grid(int64_t T, int sms)
     return (15 * gf + 15) / 16;
 }
 template <typename... KArgs>
-BwdShape bwd_shape(void (*kernel)(KArgs...), int64_t T, int sms, int threads, uint32_t smem, int clmax, int dev,
-                   std::atomic<int> (&fit)[kMaxDev][2])
+BwdShape bwd_shape(void (*kernel)(KArgs...), int64_t T, int sms, int threads, uint32_t smem, int clmax,
+                   int64_t min_tokens, int dev, std::atomic<int> (&fit)[kMaxDev][2])
 {
     const int gf = bwd_full_grid(T, sms);
+    const int forced = forced_cluster();
     for (int cl = 4; cl >= 2; cl /= 2) {
-        if (cl > clmax) continue;
+        if (cl > clmax || (forced && cl != forced)) continue;
         int64_t g = (int64_t)cl * coresident_clusters(kernel, cl, threads, smem, dev, fit);
         if (g > gf) g = gf;
         g -= g % cl;
-        if (g >= cl && 16 * g >= 15 * (int64_t)gf) return BwdShape{(int)g, cl};
+        if (g >= cl && 16 * g >= 15 * (int64_t)gf && (forced || T >= min_tokens * g)) return BwdShape{(int)g, cl};
     }
     return BwdShape{gf, 1};
 }
@@ -305,7 +318,7 @@ cudaError_t launch_dec_bwd(const resbm_desc &d, const void *dY, const void *B, c
     if (e != cudaSuccess) return e;
     static std::atomic<int> fit[kMaxDev][2];
     const BwdShape sh = bwd_shape(tc::k_dec_bwd<M>, d.T, c.sm_count, Cfg::THREADS, Cfg::SMEM_BYTES, Cfg::CLMAX,
-                                  c.device, fit);
+                                  Cfg::CL_MIN_TOKENS, c.device, fit);
     const BwdPlan p = bwd_plan(d, c.sm_count, sh.grid, Cfg::NT, d.r * d.m, ws);
     CUtensorMap m_dy128, m_dy16, m_wd2, m_b, m_yr;
     if (!make_map(&m_dy128, dY, d.d, d.T, d.d * 2, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B) ||
@@ -363,7 +376,7 @@ cudaError_t launch_enc_bwd(const resbm_desc &d, const void *dB, const void *F, c
     if (e != cudaSuccess) return e;
     static std::atomic<int> fit[kMaxDev][2];
     const BwdShape sh = bwd_shape(tc::k_enc_bwd<M>, d.T, c.sm_count, Cfg::THREADS, Cfg::SMEM_BYTES, Cfg::CLMAX,
-                                  c.device, fit);
+                                  Cfg::CL_MIN_TOKENS, c.device, fit);
     const EncBwdWs w = enc_bwd_ws(d, c.sm_count, sh.grid, ws);
     const BwdPlan &p = w.plan;
     CUtensorMap m_f128, m_f16, m_we1, m_df128, m_df16, m_db;

@@ -43,6 +43,7 @@ template <int M_> struct DecBwdCfg {
     static constexpr int NSY = M_ <= 32 ? 4 : 3;              // dY ring depth
     static constexpr int NW = M_ <= 16 ? 4 : M_ <= 32 ? 2 : 3;  // Wd2 slice ring depth
     static constexpr int CLMAX = M_ <= 32 ? 4 : 1;            // CTAs per cluster (weight-gradient exchange)
+    static constexpr int CL_MIN_TOKENS = 160;                 // clusters only from this many tokens per CTA
     static constexpr int NWB = CLMAX > 1 ? 3 : 2;             // dWd2T accumulators in TMEM
     static constexpr uint32_t RB = M_ * 2;                    // row bytes (= swizzle) of the r / m wide tiles
     static constexpr uint32_t Y_STAGE = 128 * 128 * 2;        // 128 tokens x 128 columns

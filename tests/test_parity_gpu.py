@@ -34,14 +34,36 @@ SMALL = {
     # 3 + 2, so the CTAs of a cluster have different group sizes but the same number of groups
     "bf16_uneven_groups": synth.BoundaryConfig("bf16_uneven_groups", T=79031, d=256, r=32, m=32),
     "bf16_uneven_groups_144": synth.BoundaryConfig("bf16_uneven_groups_144", T=74871, d=256, r=32, m=32),
-    # 102 units: the backward grid is 100 CTAs in clusters of 4
-    "bf16_cluster4_g100": synth.BoundaryConfig("bf16_cluster4_g100", T=1630, d=384, r=32, m=32),
-    "bf16_cluster4_g100_r16": synth.BoundaryConfig("bf16_cluster4_g100_r16", T=1625, d=256, r=16, m=16),
-    # 18 units: clusters of 4 would leave too many idle (16 < 15/16 x 18), clusters of 2 do not
-    "bf16_cluster2_g18": synth.BoundaryConfig("bf16_cluster2_g18", T=280, d=256, r=32, m=32),
-    # 3 units: single CTAs
+    # 3 units: three single CTAs
     "bf16_single_ctas": synth.BoundaryConfig("bf16_single_ctas", T=40, d=256, r=32, m=32),
 }
+
+# Backward grids under each forced cluster size (RESBM_BWD_CLUSTER): 63 units -> 62 CTAs in
+# pairs or 60 in fours; 102 -> 102 or 100; 18 -> 18 in pairs, no fours (16 < 15/16 x 18);
+# uneven tile groups inside clusters.
+CLUSTER_CASES = {
+    "ragged_r32": synth.BoundaryConfig("cl_ragged_r32", T=1000, d=512, r=32, m=32),
+    "u102_r32": synth.BoundaryConfig("cl_u102_r32", T=1630, d=384, r=32, m=32),
+    "u102_r16": synth.BoundaryConfig("cl_u102_r16", T=1625, d=256, r=16, m=16),
+    "u18_r32": synth.BoundaryConfig("cl_u18_r32", T=280, d=256, r=32, m=32),
+    "uneven_r32": synth.BoundaryConfig("cl_uneven_r32", T=79031, d=256, r=32, m=32),
+}
+_ORACLE_CACHE = {}
+
+
+@pytest.mark.parametrize("cluster", ["1", "2", "4"])
+@pytest.mark.parametrize("name", CLUSTER_CASES)
+def test_forced_cluster_sizes_match_oracle(name, cluster, monkeypatch):
+    """The backward kernels with every cluster size forced (1, 2, 4 CTAs), where it fits."""
+    monkeypatch.setenv("RESBM_BWD_CLUSTER", cluster)
+    cfg = CLUSTER_CASES[name]
+    h = host_inputs(cfg)
+    dev = {k: to_dev(v, cfg) for k, v in h.items()}
+    got = gpu_step(cfg, dev)
+    if name not in _ORACLE_CACHE:
+        _ORACLE_CACHE[name] = oracle_step(cfg, h)
+    _compare_all(cfg, got, _ORACLE_CACHE[name], dev)
+    assert resbm.resbm_device_error() == 0
 
 
 def _compare_all(cfg, got, want, dev, flags=0):
