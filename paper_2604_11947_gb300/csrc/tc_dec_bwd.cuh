@@ -526,8 +526,8 @@ __global__ void __launch_bounds__(192, 1)
 }
 
 // out = sum over slots s = 0, 1, ... of part[s] (rows x cols each, rows * cols % 4 == 0), each
-// element summed in slot order. Four consecutive elements per thread (16-byte loads) and eight
-// slots loaded ahead keep enough reads in flight. With transpose the result is written
+// element summed in slot order. Four consecutive elements per thread (16-byte loads), loaded in
+// batches of eight slots, keep enough reads in flight. With transpose the result is written
 // cols x rows (part slices are d x m, the weight gradient is m x d); out4 says out is 16-byte
 // aligned (untransposed only).
 __device__ __forceinline__ void add4(float4 &a, const float4 &b)
@@ -563,15 +563,16 @@ __device__ __forceinline__ void reduce_job(const ReduceJob &j, int64_t block, in
         const int64_t e4 = base + threadIdx.x;
         float4 acc = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
         if (e4 < n4) {
-            int64_t s = s0;
-            for (; s + 8 <= s1; s += 8) {
+            // batches of eight slots, every load of a batch in flight before the first add
+            for (int64_t s = s0; s < s1; s += 8) {
                 float4 v[8];
 #pragma unroll
-                for (int u = 0; u < 8; ++u) v[u] = __ldcs(&p4[(s + u) * n4 + e4]);
+                for (int u = 0; u < 8; ++u)
+                    if (s + u < s1) v[u] = __ldcs(&p4[(s + u) * n4 + e4]);
 #pragma unroll
-                for (int u = 0; u < 8; ++u) add4(acc, v[u]);
+                for (int u = 0; u < 8; ++u)
+                    if (s + u < s1) add4(acc, v[u]);
             }
-            for (; s < s1; ++s) add4(acc, __ldcs(&p4[s * n4 + e4]));
         }
         grp[threadIdx.y][threadIdx.x] = acc;
         __syncthreads();
