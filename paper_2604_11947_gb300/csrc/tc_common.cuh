@@ -410,6 +410,14 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16])
 
 __device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 
+// After tmem_ld_wait: ties the loaded registers to that point, so that no use of them can be
+// scheduled above the wait (the loads write them asynchronously until it).
+template <int N> __device__ __forceinline__ void tmem_regs_ready(float (&v)[N])
+{
+#pragma unroll
+    for (int i = 0; i < N; ++i) asm volatile("" : "+f"(v[i]));
+}
+
 // ---- descriptors --------------------------------------------------------------------------------
 // Swizzle modes of the shared-memory matrix descriptor (bits 61..63) and their row widths.
 enum Swz : uint32_t { kSwzNone = 0, kSwz128 = 2, kSwz64 = 4, kSwz32 = 6 };

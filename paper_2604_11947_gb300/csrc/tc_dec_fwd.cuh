@@ -8,7 +8,10 @@
 //                    D_chunk (128 x NCH fp32, TMEM, double-buffered) = G . Wd2_chunk
 //   epilogue warps : G = phi(Q) -> bf16 -> shared memory (the A operand, K-major), then per
 //                    chunk TMEM -> registers, + B on the first r columns, -> bf16 -> swizzled
-//                    staging -> TMA store of Y (boxes of 128 rows, or 16 rows for a partial tile)
+//                    staging -> TMA store of Y (boxes of 128 rows, or 16 rows for a partial tile).
+//                    Eight warps, two per TMEM lane quarter, each pair splitting a chunk's
+//                    columns: one warp's TMEM and shared-memory latencies overlap the other's
+//                    work (with one warp per quarter the epilogue, not the stores, set the pace)
 // HBM traffic per token: read B (2r bytes), write Y (2d bytes); Wd2 is re-read from L2.
 #pragma once
 
@@ -39,7 +42,8 @@ template <int M_> struct DecFwdCfg {
     static constexpr uint32_t SMEM_BYTES = OFF_WD1T + WD1T_BYTES + 1024;  // + alignment slack
     static_assert(SMEM_BYTES <= 232448 - 512, "shared memory budget");
     static constexpr uint32_t TMEM_COLS = 2 * NCH;
-    static constexpr int THREADS = 192;
+    static constexpr int EPI = 256;                    // epilogue threads (8 warps)
+    static constexpr int THREADS = 64 + EPI;
 };
 
 struct DecFwdArgs {
@@ -53,7 +57,7 @@ struct DecFwdArgs {
 // sequence); the epilogue turns Q into G = phi(Q) (bf16, shared memory) and then drains the
 // tile's Y chunks (G . Wd2_chunk, + B on the first r columns), storing them by TMA.
 template <int M_>
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(320, 1)
     k_dec_fwd(const __grid_constant__ CUtensorMap tm_wd2, const __grid_constant__ CUtensorMap tm_y128,
               const __grid_constant__ CUtensorMap tm_y16, const __grid_constant__ CUtensorMap tm_b,
               const DecFwdArgs a)
@@ -79,7 +83,7 @@ __global__ void __launch_bounds__(192, 1)
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(smem_u32(&acc_full[i]), 1);
-            mbar_init(smem_u32(&acc_empty[i]), 128);
+            mbar_init(smem_u32(&acc_empty[i]), C::EPI);
         }
         mbar_init(smem_u32(&b_full), 1);
         mbar_init(smem_u32(&b_empty), 1);
@@ -89,7 +93,7 @@ __global__ void __launch_bounds__(192, 1)
     }
     if (warp == 1) tmem_alloc(smem_u32(&tmem_base_sh), C::TMEM_COLS);
     if (warp >= 2) {  // Wd1^T (m x r) as a swizzled K-major operand: NB blocks of GB-byte rows
-        for (int e = threadIdx.x - 64; e < C::R * C::M; e += 128) {
+        for (int e = threadIdx.x - 64; e < C::R * C::M; e += C::EPI) {
             const int k = e / C::M, n = e % C::M;   // Wd1[k][n]
             const int kb = k / (C::GB / 2), kk = k % (C::GB / 2);
             *reinterpret_cast<__nv_bfloat16 *>(smem + C::OFF_WD1T + kb * (C::M * C::GB) + swz_offset(n, 2 * kk, C::GB)) =
@@ -189,10 +193,11 @@ __global__ void __launch_bounds__(192, 1)
             mbar_wait(smem_u32(&done_bar), 0);
         }
     } else {
-        // ---------------- epilogue warps (128 threads, TMEM lane quarter = warp % 4) ----------------
+        // ---------------- epilogue warps (256 threads, TMEM lane quarter = warp % 4) ----------------
         const int q = warp & 3;
+        const int half = (warp - 2) >> 2;   // which half of each chunk's columns this warp takes
         const int row = q * 32 + lane;
-        const int et = threadIdx.x - 64;  // 0..127
+        const int et = threadIdx.x - 64;    // 0..255
         const uint32_t lane_base = (uint32_t)(q * 32) << 16;
         uint32_t acc_it = 0, tile_i = 0, store_it = 0;
         bool ok = true;
@@ -205,21 +210,23 @@ __global__ void __launch_bounds__(192, 1)
                 const uint32_t ab = acc_it & 1;
                 ok = mbar_wait(smem_u32(&acc_full[ab]), (acc_it >> 1) & 1);
                 tc_fence_after();
-                float g[C::M];
-                tmem_ld_row<C::M>(tmem + lane_base + ab * C::NCH, g);
-                tc_fence_before();
+                if (half == 0) {   // the first four warps write G
+                    float g[C::M];
+                    tmem_ld_row<C::M>(tmem + lane_base + ab * C::NCH, g);
+                    tc_fence_before();
+                    act_fast_row<C::M>(a.act, g);
+#pragma unroll
+                    for (int b = 0; b < C::NB; ++b) {
+                        float gb[C::GB / 2];
+#pragma unroll
+                        for (int j = 0; j < C::GB / 2; ++j) gb[j] = active ? g[b * (C::GB / 2) + j] : 0.0f;
+                        store_bf16_swz_row<C::GB / 2>(smem + C::OFF_G + b * (128 * C::GB), row, gb);
+                    }
+                    fence_async_smem();
+                }
                 mbar_arrive(smem_u32(&acc_empty[ab]));
                 ++acc_it;
-                act_fast_row<C::M>(a.act, g);
-#pragma unroll
-                for (int b = 0; b < C::NB; ++b) {
-                    float gb[C::GB / 2];
-#pragma unroll
-                    for (int j = 0; j < C::GB / 2; ++j) gb[j] = active ? g[b * (C::GB / 2) + j] : 0.0f;
-                    store_bf16_swz_row<C::GB / 2>(smem + C::OFF_G + b * (128 * C::GB), row, gb);
-                }
-                fence_async_smem();
-                named_barrier(1, 128);
+                named_barrier(1, C::EPI);
                 if (et == 0) mbar_arrive(smem_u32(&g_full));
             }
 
@@ -229,53 +236,63 @@ __global__ void __launch_bounds__(192, 1)
                 ok = mbar_wait(smem_u32(&acc_full[ab]), (acc_it >> 1) & 1);
                 tc_fence_after();
                 if (et == 0) bulk_wait_read<1>();  // staging buffer sb is free again
-                named_barrier(1, 128);
+                named_barrier(1, C::EPI);
                 uint8_t *stg = smem + C::OFF_STG + sb * C::STG_BYTES;
                 const int64_t left = a.d - (int64_t)c * C::NCH;
                 const int ncols = left < C::NCH ? (int)left : C::NCH;
                 // a warp whose 32 rows all lie past the tile's valid tokens has nothing to store
                 const int gend = (q * 32 < valid) ? ncols : 0;
+                // 64 columns (two TMEM loads in flight) at a time: one staging box
 #pragma unroll
-                for (int g = 0; g < C::NCH / 32; ++g) {
-                    if (g * 32 >= gend) break;
-                    float v[32];
-                    tmem_ld32(tmem + lane_base + ab * C::NCH + g * 32, v);
+                for (int gh = 0; gh < C::NCH / 128; ++gh) {
+                    const int g2 = half * (C::NCH / 128) + gh;   // this warp's boxes of the chunk
+                    if (g2 * 64 >= gend) break;
+                    float v2[2][32];
+                    tmem_ld32(tmem + lane_base + ab * C::NCH + g2 * 64, v2[0]);
+                    tmem_ld32(tmem + lane_base + ab * C::NCH + g2 * 64 + 32, v2[1]);
                     tmem_ld_wait();
-                    // identity path: the first r columns of Y get B (only chunk 0 holds them)
-                    if (g * 32 < C::R && a.merge && c == 0) {
-                        const uint8_t *bblk = smem + C::OFF_B + ((g * 32) / (C::GB / 2)) * (128 * C::GB);
-                        const uint32_t b0 = ((g * 32) % (C::GB / 2)) * 2;
+                    tmem_regs_ready(v2[0]);
+                    tmem_regs_ready(v2[1]);
 #pragma unroll
-                        for (int i = 0; i < 32; i += 8) {
-                            if (g * 32 + i < C::R) {
-                                const uint4 u = *reinterpret_cast<const uint4 *>(bblk + swz_offset(row, b0 + 2 * i, C::GB));
-                                const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+                    for (int h = 0; h < 2; ++h) {
+                        const int g = 2 * g2 + h;   // columns [g*32, g*32+32) of the chunk
+                        float (&v)[32] = v2[h];
+                        // identity path: the first r columns of Y get B (only chunk 0 holds them)
+                        if (g * 32 < C::R && a.merge && c == 0) {
+                            const uint8_t *bblk = smem + C::OFF_B + ((g * 32) / (C::GB / 2)) * (128 * C::GB);
+                            const uint32_t b0 = ((g * 32) % (C::GB / 2)) * 2;
 #pragma unroll
-                                for (int e = 0; e < 4; ++e) {
-                                    v[i + 2 * e] += __uint_as_float(w[e] << 16);
-                                    v[i + 2 * e + 1] += __uint_as_float(w[e] & 0xFFFF0000u);
+                            for (int i = 0; i < 32; i += 8) {
+                                if (g * 32 + i < C::R) {
+                                    const uint4 u = *reinterpret_cast<const uint4 *>(bblk + swz_offset(row, b0 + 2 * i, C::GB));
+                                    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+                                    for (int e = 0; e < 4; ++e) {
+                                        v[i + 2 * e] += __uint_as_float(w[e] << 16);
+                                        v[i + 2 * e + 1] += __uint_as_float(w[e] & 0xFFFF0000u);
+                                    }
                                 }
                             }
                         }
-                    }
-                    uint32_t p[16];
+                        uint32_t p[16];
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) {
-                        __nv_bfloat162 h = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
-                        p[i] = *reinterpret_cast<uint32_t *>(&h);
-                    }
-                    // columns [g*32, g*32+32) of the chunk: box g/2, bytes (g%2)*64 .. +64
-                    uint8_t *box = stg + (g >> 1) * 16384;
-                    const uint32_t b0 = (g & 1) * 64;
+                        for (int i = 0; i < 16; ++i) {
+                            __nv_bfloat162 hh = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+                            p[i] = *reinterpret_cast<uint32_t *>(&hh);
+                        }
+                        // columns [g*32, g*32+32) of the chunk: box g/2, bytes (g%2)*64 .. +64
+                        uint8_t *box = stg + (g >> 1) * 16384;
+                        const uint32_t b0 = (g & 1) * 64;
 #pragma unroll
-                    for (int i = 0; i < 4; ++i)
-                        *reinterpret_cast<uint4 *>(box + swz_offset(row, b0 + 16 * i, 128)) =
-                            make_uint4(p[4 * i], p[4 * i + 1], p[4 * i + 2], p[4 * i + 3]);
+                        for (int i = 0; i < 4; ++i)
+                            *reinterpret_cast<uint4 *>(box + swz_offset(row, b0 + 16 * i, 128)) =
+                                make_uint4(p[4 * i], p[4 * i + 1], p[4 * i + 2], p[4 * i + 3]);
+                    }
                 }
                 tc_fence_before();
                 mbar_arrive(smem_u32(&acc_empty[ab]));
                 fence_async_smem();
-                named_barrier(1, 128);
+                named_barrier(1, C::EPI);
                 if (et == 0) {
                     if (c == 0) mbar_arrive(smem_u32(&b_empty));   // the B tile is no longer read
                     const uint32_t sbase = smem_u32(stg);

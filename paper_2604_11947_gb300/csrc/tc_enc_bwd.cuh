@@ -472,12 +472,18 @@ __global__ void __launch_bounds__(192, 1)
                         uint8_t *stg = smem + C::OFF_STG + sb * C::STG_HALF;
                         // a warp whose rows all lie past the valid tokens has nothing to store
                         const int gqend = (q * 32 < valid) ? 2 : 0;
+                        float v2[2][32];
+                        if (gqend) {   // the half's 64 columns, both TMEM loads in flight
+                            tmem_ld32(tmem + lane_base + C::TM_DF + ad_buf * 128 + h * 64, v2[0]);
+                            tmem_ld32(tmem + lane_base + C::TM_DF + ad_buf * 128 + h * 64 + 32, v2[1]);
+                            tmem_ld_wait();
+                            tmem_regs_ready(v2[0]);
+                            tmem_regs_ready(v2[1]);
+                        }
 #pragma unroll
                         for (int gq = 0; gq < 2; ++gq) {
                             if (gq >= gqend) break;
-                            float v[32];
-                            tmem_ld32(tmem + lane_base + C::TM_DF + ad_buf * 128 + h * 64 + gq * 32, v);
-                            tmem_ld_wait();
+                            float (&v)[32] = v2[gq];
                             uint32_t p[16];
 #pragma unroll
                             for (int e = 0; e < 16; ++e) {
