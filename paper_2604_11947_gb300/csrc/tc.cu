@@ -142,7 +142,7 @@ int coresident_clusters(void (*kernel)(KArgs...), int cl, int threads, uint32_t 
 }
 
 // Grid and cluster size of a backward launch. The persistent grid would be g_full =
-// min(16-token units, SMs) single CTAs; clusters of 4 are taken when at least 15/16 of g_full
+// min(128-token tiles, SMs) single CTAs; clusters of 4 are taken when at least 15/16 of g_full
 // CTAs fit as co-resident clusters of 4 (the grid is then that many, a multiple of 4) and each
 // CTA still gets at least `min_tokens` tokens, else clusters of 2 on the same terms, else single
 // CTAs. Fewer, larger weight-gradient partials cost less than the few idle SMs (these kernels
@@ -162,7 +162,7 @@ int forced_cluster()
 }
 int bwd_full_grid(int64_t T, int sms)
 {
-    int64_t g = (T + 15) / 16;
+    int64_t g = (T + 127) / 128;
     if (g > sms) g = sms;
     return (int)(g < 1 ? 1 : g);
 }
@@ -189,9 +189,10 @@ BwdShape bwd_shape(void (*kernel)(KArgs...), int64_t T, int sms, int threads, ui
 
 bool tc_width_ok(int64_t m) { return m == 16 || m == 32 || m == 64 || m == 128; }
 
+// Persistent grid: one CTA per SM, at most one per 128-token tile (token_range).
 int grid_tokens(const Ctx &c, int64_t T)
 {
-    int64_t g = (T + 15) / 16;
+    int64_t g = (T + 127) / 128;
     if (g > c.sm_count) g = c.sm_count;
     return (int)(g < 1 ? 1 : g);
 }
@@ -254,9 +255,8 @@ struct BwdPlan {
 
 int bwd_max_groups(int64_t T, int grid, int nt)
 {
-    const int64_t U = (T + 15) / 16;
-    const int64_t max_tokens = 16 * ((U + grid - 1) / grid);
-    const int64_t max_tiles = (max_tokens + 127) / 128;
+    const int64_t U = (T + 127) / 128;   // tiles, split as token_range does
+    const int64_t max_tiles = (U + grid - 1) / grid;
     const int64_t g = (max_tiles + nt - 1) / nt;
     return (int)(g < 1 ? 1 : g);
 }

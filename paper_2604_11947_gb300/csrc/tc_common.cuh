@@ -55,13 +55,17 @@ __device__ __forceinline__ void flag_error(unsigned code)
     atomicOr(&g_resbm_device_error, code);
 }
 
-// Token range [start, end) of CTA b out of G over T tokens: T is cut into 16-token units and
-// every CTA gets a contiguous run of floor or ceil(units / G) of them (balanced to 16 tokens).
+// Token range [start, end) of CTA b out of G over T tokens: T is cut into whole 128-token
+// tiles and every CTA gets a contiguous run of floor or ceil(tiles / G) of them; only the
+// tensor's last tile can be partial. (A partial tile streams through as many pipeline stages as
+// a full one and costs about as much time, so balancing to finer units made every CTA pay for
+// one; with whole tiles the CTAs with one tile fewer finish early and leave the bandwidth to the
+// others. The grid is at most the number of tiles.)
 __device__ __forceinline__ void token_range(int64_t T, int b, int G, int64_t &start, int64_t &end)
 {
-    const int64_t U = (T + 15) / 16;
-    start = 16 * ((U * b) / G);
-    end = 16 * ((U * (b + 1)) / G);
+    const int64_t U = (T + 127) / 128;
+    start = 128 * ((U * b) / G);
+    end = 128 * ((U * (b + 1)) / G);
     if (end > T) end = T;
     if (start > T) start = T;
 }

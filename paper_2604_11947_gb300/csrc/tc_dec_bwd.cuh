@@ -3,7 +3,7 @@
 //   Q = B . Wd1, G = phi(Q);  dG = dY . Wd2^T;  dQ = dG * phi'(Q);
 //   dB = [merge] dY[:, :r] + dQ . Wd1^T;  dWd2 = G^T . dY;  dWd1 = B^T . dQ.
 //
-// Persistent CTAs (in clusters of 1, 2 or 4) over contiguous 16-token-aligned token ranges,
+// Persistent CTAs (in clusters of 1, 2 or 4) over contiguous runs of whole 128-token tiles,
 // processed in groups of up to NT tiles of 128 tokens (every CTA has the same number of groups,
 // its tiles split evenly). Every product runs on tcgen05; the CUDA cores only apply phi and phi'
 // and convert. For each group:

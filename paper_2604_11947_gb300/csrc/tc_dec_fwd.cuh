@@ -1,8 +1,8 @@
 // tc_dec_fwd.cuh -- receive side of the boundary on tensor cores (Sec. 3.2 decoder, Eq. Pid
 // zero-padding identity path):  Y = [merge] B . I_{r x d} + phi(B . Wd1) . Wd2.
 //
-// Persistent CTAs; CTA b owns a contiguous token range (16-token aligned, balanced to within
-// 16 tokens) and walks it in tiles of up to 128 tokens. Per tile:
+// Persistent CTAs; CTA b owns a contiguous run of whole 128-token tiles (the tensor's last tile
+// may be partial) and walks it tile by tile. Per tile:
 //   producer warp  : the tile's B rows by TMA; Wd2 column chunks (m x NCH, MN-major) into a ring
 //   MMA warp       : Q = B . Wd1 into the next free accumulator, then per chunk
 //                    D_chunk (128 x NCH fp32, TMEM, double-buffered) = G . Wd2_chunk

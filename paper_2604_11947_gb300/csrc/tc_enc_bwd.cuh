@@ -3,7 +3,7 @@
 //   dA = dB . We2^T;  dP = dA * phi'(P);  dF = dP . We1^T;  dX[:, :r] += dB;
 //   dWe1 = F^T . dP;  dWe2 = phi(P)^T . dB.
 //
-// Persistent CTAs (in clusters of 1, 2 or 4) over contiguous 16-token-aligned token ranges, in
+// Persistent CTAs (in clusters of 1, 2 or 4) over contiguous runs of whole 128-token tiles, in
 // groups of up to NT tiles of 128 tokens. Every product runs on tcgen05; the CUDA cores apply
 // phi and phi', convert, and do the identity-path update. For each group:
 //   phase 0: the group's dB tiles (TMA) -> dA_tile = dB . We2^T in TMEM -> the epilogue reads P

@@ -1,7 +1,8 @@
 // tc_enc_fwd.cuh -- send side of the boundary on tensor cores (Sec. 3.2 encoder, Eq. Pid
 // truncating identity path):  P = F . We1 (saved, fp32),  B = X[:, :r] + phi(P) . We2.
 //
-// Persistent CTAs over contiguous 16-token-aligned token ranges, tiles of up to 128 tokens.
+// Persistent CTAs over contiguous runs of whole 128-token tiles (the tensor's last tile may be
+// partial).
 //   producer warp : for each tile, d in chunks of 64 columns: F tile chunk (128 x 64, K-major,
 //                   128B swizzle; 16-row boxes for a partial tile) + We1 rows (64 x m, MN-major)
 //   MMA warp      : P (128 x m fp32 in TMEM, double-buffered per tile) += F_chunk . We1_chunk

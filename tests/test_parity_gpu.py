@@ -30,22 +30,25 @@ SMALL = {
     # ~1000 tokens per CTA: several groups of tiles per CTA in the backward kernels (whose
     # grids on a 152-SM GB300 are 144 CTAs in clusters of 4)
     "bf16_multi_group": synth.BoundaryConfig("bf16_multi_group", T=150001, d=128, r=32, m=32),
-    # 32 or 33 16-token units per CTA on 152 (or 144) CTAs: 4 or 5 tiles, cut into 2 + 2 or
-    # 3 + 2, so the CTAs of a cluster have different group sizes but the same number of groups
+    # 618 (585) tiles on 144 backward CTAs: 4 or 5 tiles per CTA, cut into 2 + 2 or 3 + 2, so
+    # the CTAs of a cluster have different group sizes but the same number of groups
     "bf16_uneven_groups": synth.BoundaryConfig("bf16_uneven_groups", T=79031, d=256, r=32, m=32),
     "bf16_uneven_groups_144": synth.BoundaryConfig("bf16_uneven_groups_144", T=74871, d=256, r=32, m=32),
-    # 3 units: three single CTAs
+    # one partial tile: a single CTA
     "bf16_single_ctas": synth.BoundaryConfig("bf16_single_ctas", T=40, d=256, r=32, m=32),
 }
 
-# Backward grids under each forced cluster size (RESBM_BWD_CLUSTER): 63 units -> 62 CTAs in
-# pairs or 60 in fours; 102 -> 102 or 100; 18 -> 18 in pairs, no fours (16 < 15/16 x 18);
-# uneven tile groups inside clusters.
+# Backward grids under each forced cluster size (RESBM_BWD_CLUSTER), one CTA per 128-token
+# tile at most: 8 tiles -> 8 CTAs in pairs or fours; 16 -> 16; 17 -> 16 in pairs or fours (one
+# idle SM); 18 -> 18 in pairs, no fours (16 < 15/16 x 18); 3 -> single CTAs (fours do not fit,
+# pairs leave too many idle); uneven tile groups inside clusters.
 CLUSTER_CASES = {
-    "ragged_r32": synth.BoundaryConfig("cl_ragged_r32", T=1000, d=512, r=32, m=32),
-    "u102_r32": synth.BoundaryConfig("cl_u102_r32", T=1630, d=384, r=32, m=32),
-    "u102_r16": synth.BoundaryConfig("cl_u102_r16", T=1625, d=256, r=16, m=16),
-    "u18_r32": synth.BoundaryConfig("cl_u18_r32", T=280, d=256, r=32, m=32),
+    "t8_r32": synth.BoundaryConfig("cl_t8_r32", T=1000, d=512, r=32, m=32),
+    "t16_r32": synth.BoundaryConfig("cl_t16_r32", T=2000, d=384, r=32, m=32),
+    "t16_r16": synth.BoundaryConfig("cl_t16_r16", T=1990, d=256, r=16, m=16),
+    "t17_r32": synth.BoundaryConfig("cl_t17_r32", T=2100, d=256, r=32, m=32),
+    "t18_r32": synth.BoundaryConfig("cl_t18_r32", T=2260, d=256, r=32, m=32),
+    "t3_r32": synth.BoundaryConfig("cl_t3_r32", T=280, d=256, r=32, m=32),
     "uneven_r32": synth.BoundaryConfig("cl_uneven_r32", T=79031, d=256, r=32, m=32),
 }
 _ORACLE_CACHE = {}
