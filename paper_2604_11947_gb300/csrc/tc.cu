@@ -212,7 +212,10 @@ cudaError_t launch_dec_fwd(const resbm_desc &d, const void *B, const void *Wd1, 
     cudaError_t e = ensure_smem(tc::k_dec_fwd<M>, Cfg::SMEM_BYTES, c.device, smem_set);
     if (e != cudaSuccess) return e;
     tc::DecFwdArgs a{static_cast<const __nv_bfloat16 *>(Wd1), d.T, d.d, d.act, d.merge_identity};
-    e = launch(tc::k_dec_fwd<M>, grid_tokens(c, d.T), Cfg::THREADS, Cfg::SMEM_BYTES, c.stream, m_wd2, m_y128, m_y16,
+    // one CTA per SM, at most one per (tile, chunk) unit (the decoder forward splits tiles by columns)
+    int64_t units = ((d.T + 127) / 128) * (d.d / Cfg::NCH);
+    const int grid = (int)(units < c.sm_count ? (units < 1 ? 1 : units) : c.sm_count);
+    e = launch(tc::k_dec_fwd<M>, grid, Cfg::THREADS, Cfg::SMEM_BYTES, c.stream, m_wd2, m_y128, m_y16,
                m_b, a);
     count_launches(1);
     return e;

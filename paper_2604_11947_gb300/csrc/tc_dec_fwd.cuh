@@ -1,18 +1,25 @@
 // tc_dec_fwd.cuh -- receive side of the boundary on tensor cores (Sec. 3.2 decoder, Eq. Pid
 // zero-padding identity path):  Y = [merge] B . I_{r x d} + phi(B . Wd1) . Wd2.
 //
-// Persistent CTAs; CTA b owns a contiguous run of whole 128-token tiles (the tensor's last tile
-// may be partial) and walks it tile by tile. Per tile:
-//   producer warp  : the tile's B rows by TMA; Wd2 column chunks (m x NCH, MN-major) into a ring
-//   MMA warp       : Q = B . Wd1 into the next free accumulator, then per chunk
-//                    D_chunk (128 x NCH fp32, TMEM, double-buffered) = G . Wd2_chunk
+// Persistent CTAs. The work is cut in units of (128-token tile, NCH output columns) and every
+// CTA owns a contiguous run of floor or ceil(units / grid) of them in tile-major order: one
+// segment of consecutive chunks per tile it touches (the tiles at the ends of its run partly).
+// Y's columns are independent given G, so no tile has to be finished by one CTA and the runs
+// balance to within one chunk. Per segment:
+//   producer warp  : the tile's B rows by TMA (double-buffered; the next tile's as soon as its
+//                    buffer is free); Wd2 column chunks (m x NCH, MN-major) into a ring
+//   MMA warp       : Q = B . Wd1 of the NEXT segment's tile one chunk before this segment's
+//                    last, then per chunk D_chunk (128 x NCH fp32, TMEM, double-buffered) =
+//                    G . Wd2_chunk; with G double-buffered the epilogue computes the next tile's
+//                    G while this tile's last chunk is being computed (no bubble between tiles)
 //   epilogue warps : G = phi(Q) -> bf16 -> shared memory (the A operand, K-major), then per
-//                    chunk TMEM -> registers, + B on the first r columns, -> bf16 -> swizzled
-//                    staging -> TMA store of Y (boxes of 128 rows, or 16 rows for a partial tile).
-//                    Eight warps, two per TMEM lane quarter, each pair splitting a chunk's
-//                    columns: one warp's TMEM and shared-memory latencies overlap the other's
-//                    work (with one warp per quarter the epilogue, not the stores, set the pace)
-// HBM traffic per token: read B (2r bytes), write Y (2d bytes); Wd2 is re-read from L2.
+//                    chunk TMEM -> registers, + B on the first r columns (chunk 0 only), -> bf16
+//                    -> swizzled staging -> TMA store of Y (boxes of 128 rows, or 16 rows for a
+//                    partial tile). Eight warps, two per TMEM lane quarter, each pair splitting
+//                    a chunk's columns: one warp's TMEM and shared-memory latencies overlap the
+//                    other's work (with one warp per quarter the epilogue set the pace).
+// HBM traffic per token: read B (2r bytes, once per segment), write Y (2d bytes); Wd2 is
+// re-read from L2.
 #pragma once
 
 #include "common.cuh"
@@ -35,9 +42,13 @@ template <int M_> struct DecFwdCfg {
     static constexpr uint32_t WD1T_BYTES = R * M_ * 2;
     // shared-memory map (offsets from a 1024-aligned base)
     static constexpr uint32_t OFF_W = 0;
-    static constexpr uint32_t OFF_G = OFF_W + NSTAGE * W_STAGE_BYTES;   // G tile [token][m]
-    static constexpr uint32_t OFF_B = OFF_G + TILE_BYTES;                // B tile [token][r] (TMA)
-    static constexpr uint32_t OFF_STG = OFF_B + TILE_BYTES;
+    // G and B tiles double-buffered (the next tile's G is made while this tile's last chunk is
+    // computed) where shared memory allows, i.e. for m <= 64
+    static constexpr int NGB = M_ <= 64 ? 2 : 1;
+    static constexpr bool LOOKAHEAD = NGB == 2;
+    static constexpr uint32_t OFF_G = OFF_W + NSTAGE * W_STAGE_BYTES;   // NGB G tiles [token][m]
+    static constexpr uint32_t OFF_B = OFF_G + NGB * TILE_BYTES;          // NGB B tiles [token][r] (TMA)
+    static constexpr uint32_t OFF_STG = OFF_B + NGB * TILE_BYTES;
     static constexpr uint32_t OFF_WD1T = OFF_STG + 2 * STG_BYTES;       // Wd1^T [m][r], K-major
     static constexpr uint32_t SMEM_BYTES = OFF_WD1T + WD1T_BYTES + 1024;  // + alignment slack
     static_assert(SMEM_BYTES <= 232448 - 512, "shared memory budget");
@@ -68,13 +79,21 @@ __global__ void __launch_bounds__(320, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     __shared__ uint64_t w_full[C::NSTAGE], w_empty[C::NSTAGE];
-    __shared__ uint64_t b_full, b_empty, g_full, acc_full[2], acc_empty[2], done_bar;
+    __shared__ uint64_t b_full[C::NGB], b_empty[C::NGB], g_full[C::NGB], acc_full[2], acc_empty[2], done_bar;
     __shared__ uint32_t tmem_base_sh;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int nchunks = (int)(a.d / C::NCH) + ((a.d % C::NCH) ? 1 : 0);
-    int64_t start, end;
-    token_range(a.T, blockIdx.x, gridDim.x, start, end);
+    const int nchunks = (int)(a.d / C::NCH);   // d % NCH == 0 on this path
+    // this CTA's run of (tile, chunk) units
+    const int64_t units = ((a.T + 127) / 128) * nchunks;
+    const int64_t u_begin = units * blockIdx.x / gridDim.x, u_end = units * (blockIdx.x + 1) / gridDim.x;
+    // segment k of the run: tile, first and one-past-last chunk
+    auto seg_at = [&](int64_t u, int64_t &tile, int &c0, int &c1) {
+        tile = u / nchunks;
+        c0 = (int)(u - tile * nchunks);
+        const int64_t last = u_end - tile * nchunks;
+        c1 = last < nchunks ? (int)last : nchunks;
+    };
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < C::NSTAGE; ++s) {
@@ -85,9 +104,11 @@ __global__ void __launch_bounds__(320, 1)
             mbar_init(smem_u32(&acc_full[i]), 1);
             mbar_init(smem_u32(&acc_empty[i]), C::EPI);
         }
-        mbar_init(smem_u32(&b_full), 1);
-        mbar_init(smem_u32(&b_empty), 1);
-        mbar_init(smem_u32(&g_full), 1);
+        for (int i = 0; i < C::NGB; ++i) {
+            mbar_init(smem_u32(&b_full[i]), 1);
+            mbar_init(smem_u32(&b_empty[i]), 1);
+            mbar_init(smem_u32(&g_full[i]), 1);
+        }
         mbar_init(smem_u32(&done_bar), 1);
         fence_mbar_init();
     }
@@ -111,17 +132,39 @@ __global__ void __launch_bounds__(320, 1)
         if (elect_one()) {
             tma_prefetch_desc(&tm_wd2);
             tma_prefetch_desc(&tm_b);
-            uint32_t it = 0, tile_i = 0;
-            bool ok = true;
-            for (int64_t t0 = start; t0 < end && ok; t0 += 128, ++tile_i) {
-                // the tile's B rows, once the previous tile's are no longer read (128-row boxes:
-                // rows past T read as zeros, rows past this CTA's range are loaded, never used)
-                if (!mbar_wait(smem_u32(&b_empty), (tile_i & 1) ^ 1)) break;
-                mbar_expect_tx(smem_u32(&b_full), C::TILE_BYTES);
+            // B rows of segment k's tile into buffer k % NGB, once that buffer's previous tile is
+            // no longer read (128-row boxes: rows past T read as zeros)
+            auto load_b = [&](uint32_t k, int64_t tile) -> bool {
+                const uint32_t bb = k % C::NGB;
+                if (!mbar_wait(smem_u32(&b_empty[bb]), ((k / C::NGB) & 1) ^ 1)) return false;
+                mbar_expect_tx(smem_u32(&b_full[bb]), C::TILE_BYTES);
                 for (int b = 0; b < C::NB; ++b)
-                    tma_load_2d(smem_u32(smem + C::OFF_B + b * (128 * C::GB)), &tm_b, b * (C::GB / 2), (int32_t)t0,
-                                smem_u32(&b_full));
-                for (int c = 0; c < nchunks; ++c) {
+                    tma_load_2d(smem_u32(smem + C::OFF_B + bb * C::TILE_BYTES + b * (128 * C::GB)), &tm_b,
+                                b * (C::GB / 2), (int32_t)(tile * 128), smem_u32(&b_full[bb]));
+                return true;
+            };
+            uint32_t it = 0, k = 0, b_loaded = 0;
+            bool ok = true;
+            if (u_begin < u_end) {
+                int64_t tile;
+                int c0, c1;
+                seg_at(u_begin, tile, c0, c1);
+                ok = load_b(0, tile);
+                b_loaded = ok ? 1 : 0;
+            }
+            for (int64_t u = u_begin; u < u_end && ok; ++k) {
+                int64_t tile;
+                int c0, c1;
+                seg_at(u, tile, c0, c1);
+                u = tile * nchunks + c1;
+                if (C::LOOKAHEAD && u < u_end) {   // the next segment's B, early: its Q comes before this one's end
+                    int64_t nt;
+                    int n0, n1;
+                    seg_at(u, nt, n0, n1);
+                    if (!(ok = load_b(k + 1, nt))) break;
+                    ++b_loaded;
+                }
+                for (int c = c0; c < c1; ++c) {
                     const uint32_t s = it % C::NSTAGE, ph = (it / C::NSTAGE) & 1;
                     if (!mbar_wait(smem_u32(&w_empty[s]), ph ^ 1)) {
                         ok = false;
@@ -133,14 +176,24 @@ __global__ void __launch_bounds__(320, 1)
                         tma_load_2d(dst + b * (C::M * 128), &tm_wd2, c * C::NCH + 64 * b, 0, smem_u32(&w_full[s]));
                     ++it;
                 }
+                if (!C::LOOKAHEAD && ok && u < u_end) {   // one B buffer: the next tile's after this segment's chunks
+                    int64_t nt;
+                    int n0, n1;
+                    seg_at(u, nt, n0, n1);
+                    if (!(ok = load_b(k + 1, nt))) break;
+                    ++b_loaded;
+                }
             }
             // drain: every issued load has landed before the CTA can exit
             const uint32_t n = it < (uint32_t)C::NSTAGE ? it : (uint32_t)C::NSTAGE;
-            for (uint32_t k = 0; k < n; ++k) {
-                const uint32_t j = it - 1 - k;
+            for (uint32_t j0 = 0; j0 < n; ++j0) {
+                const uint32_t j = it - 1 - j0;
                 mbar_wait(smem_u32(&w_full[j % C::NSTAGE]), (j / C::NSTAGE) & 1);
             }
-            if (tile_i > 0) mbar_wait(smem_u32(&b_full), (tile_i - 1) & 1);
+            for (uint32_t j0 = 0; j0 < (b_loaded < (uint32_t)C::NGB ? b_loaded : (uint32_t)C::NGB); ++j0) {
+                const uint32_t j = b_loaded - 1 - j0;
+                mbar_wait(smem_u32(&b_full[j % C::NGB]), (j / C::NGB) & 1);
+            }
         }
     } else if (warp == 1) {
         // ---------------- MMA issuer ----------------
@@ -148,31 +201,44 @@ __global__ void __launch_bounds__(320, 1)
             constexpr Swz gsw = swz_for(C::GB);
             constexpr uint32_t id_q = idesc_bf16(128, C::M, false, false);    // B (K-major) . Wd1^T rows (K-major)
             constexpr uint32_t id_y = idesc_bf16(128, C::NCH, false, true);   // G (K-major) . Wd2 chunk (MN-major)
+            constexpr uint64_t TILE16 = C::TILE_BYTES >> 4;
             const uint64_t bk0 = smem_desc(smem_u32(smem + C::OFF_B), 16, 8 * C::GB, gsw);
             const uint64_t gk0 = smem_desc(smem_u32(smem + C::OFF_G), 16, 8 * C::GB, gsw);
             const uint64_t wt0 = smem_desc(smem_u32(smem + C::OFF_WD1T), 16, 8 * C::GB, gsw);
-            uint32_t it = 0, acc_it = 0, tile_i = 0;
+            uint32_t it = 0, acc_it = 0;
             bool ok = true;
-            for (int64_t t0 = start; t0 < end && ok; t0 += 128, ++tile_i) {
-                // Q = B . Wd1 into the next accumulator
-                {
-                    const uint32_t ab = acc_it & 1;
-                    ok = mbar_wait(smem_u32(&b_full), tile_i & 1) &&
-                         mbar_wait(smem_u32(&acc_empty[ab]), ((acc_it >> 1) & 1) ^ 1);
-                    tc_fence_after();
-#pragma unroll
-                    for (int k = 0; k < C::R / 16; ++k) {
-                        const uint64_t off = (uint64_t)(((k / C::SPB) * (128 * C::GB) + (k % C::SPB) * 32) >> 4);
-                        const uint64_t woff = (uint64_t)(((k / C::SPB) * (C::M * C::GB) + (k % C::SPB) * 32) >> 4);
-                        mma_bf16(tmem + ab * C::NCH, bk0 + off, wt0 + woff, id_q, k > 0);
-                    }
-                    mma_commit(smem_u32(&acc_full[ab]));
-                    ++acc_it;
-                }
-                // the tile's Y chunks once its G is in shared memory
-                ok = ok && mbar_wait(smem_u32(&g_full), tile_i & 1);
+            // Q = B . Wd1 of segment k's tile (B buffer k % NGB) into the next accumulator
+            auto issue_q = [&](uint32_t k) {
+                const uint32_t ab = acc_it & 1;
+                ok = ok && mbar_wait(smem_u32(&b_full[k % C::NGB]), (k / C::NGB) & 1) &&
+                     mbar_wait(smem_u32(&acc_empty[ab]), ((acc_it >> 1) & 1) ^ 1);
                 tc_fence_after();
-                for (int c = 0; c < nchunks && ok; ++c, ++it, ++acc_it) {
+                if (!ok) return;
+#pragma unroll
+                for (int kk = 0; kk < C::R / 16; ++kk) {
+                    const uint64_t off = (uint64_t)(((kk / C::SPB) * (128 * C::GB) + (kk % C::SPB) * 32) >> 4);
+                    const uint64_t woff = (uint64_t)(((kk / C::SPB) * (C::M * C::GB) + (kk % C::SPB) * 32) >> 4);
+                    mma_bf16(tmem + ab * C::NCH, bk0 + (k % C::NGB) * TILE16 + off, wt0 + woff, id_q, kk > 0);
+                }
+                mma_commit(smem_u32(&acc_full[ab]));
+                ++acc_it;
+            };
+            if (u_begin < u_end) issue_q(0);
+            uint32_t k = 0;
+            for (int64_t u = u_begin; u < u_end && ok; ++k) {
+                int64_t tile;
+                int c0, c1;
+                seg_at(u, tile, c0, c1);
+                u = tile * nchunks + c1;
+                const bool has_next = u < u_end;
+                // the segment's Y chunks once its tile's G is in shared memory
+                ok = ok && mbar_wait(smem_u32(&g_full[k % C::NGB]), (k / C::NGB) & 1);
+                tc_fence_after();
+                for (int c = c0; c < c1 && ok; ++c, ++it, ++acc_it) {
+                    if (C::LOOKAHEAD && c == c1 - 1 && has_next) {   // the next tile's Q, before this segment's last chunk
+                        issue_q(k + 1);
+                        if (!ok) break;
+                    }
                     const uint32_t s = it % C::NSTAGE, ph = (it / C::NSTAGE) & 1;
                     const uint32_t ab = acc_it & 1;
                     ok = mbar_wait(smem_u32(&w_full[s]), ph) &&
@@ -180,14 +246,15 @@ __global__ void __launch_bounds__(320, 1)
                     tc_fence_after();
                     const uint32_t waddr = smem_u32(smem + C::OFF_W + s * C::W_STAGE_BYTES);
 #pragma unroll
-                    for (int k = 0; k < C::M / 16; ++k) {
-                        const uint64_t off = (uint64_t)(((k / C::SPB) * (128 * C::GB) + (k % C::SPB) * 32) >> 4);
-                        const uint64_t bd = smem_desc(waddr + k * 16 * 128, C::M * 128, 1024, kSwz128);
-                        mma_bf16(tmem + ab * C::NCH, gk0 + off, bd, id_y, k > 0);
+                    for (int kk = 0; kk < C::M / 16; ++kk) {
+                        const uint64_t off = (uint64_t)(((kk / C::SPB) * (128 * C::GB) + (kk % C::SPB) * 32) >> 4);
+                        const uint64_t bd = smem_desc(waddr + kk * 16 * 128, C::M * 128, 1024, kSwz128);
+                        mma_bf16(tmem + ab * C::NCH, gk0 + (k % C::NGB) * TILE16 + off, bd, id_y, kk > 0);
                     }
                     mma_commit(smem_u32(&w_empty[s]));
                     mma_commit(smem_u32(&acc_full[ab]));
                 }
+                if (!C::LOOKAHEAD && ok && has_next) issue_q(k + 1);   // one G buffer: after this segment
             }
             mma_commit(smem_u32(&done_bar));
             mbar_wait(smem_u32(&done_bar), 0);
@@ -199,38 +266,62 @@ __global__ void __launch_bounds__(320, 1)
         const int row = q * 32 + lane;
         const int et = threadIdx.x - 64;    // 0..255
         const uint32_t lane_base = (uint32_t)(q * 32) << 16;
-        uint32_t acc_it = 0, tile_i = 0, store_it = 0;
+        uint32_t acc_it = 0, store_it = 0;
         bool ok = true;
-        for (int64_t t0 = start; t0 < end && ok; t0 += 128, ++tile_i) {
-            const int64_t t1 = (end - t0) < 128 ? end : t0 + 128;
-            const int valid = (int)(t1 - t0);
-            const bool active = row < valid;
-            // ---- G = phi(Q) -> bf16 -> the G tile (K-major, NB blocks of GB-byte rows) ----
-            {
-                const uint32_t ab = acc_it & 1;
-                ok = mbar_wait(smem_u32(&acc_full[ab]), (acc_it >> 1) & 1);
-                tc_fence_after();
-                if (half == 0) {   // the first four warps write G
-                    float g[C::M];
-                    tmem_ld_row<C::M>(tmem + lane_base + ab * C::NCH, g);
-                    tc_fence_before();
-                    act_fast_row<C::M>(a.act, g);
+        // G = phi(Q) -> bf16 -> G buffer k % NGB (K-major, NB blocks of GB-byte rows), for segment
+        // k's tile whose first `valid` rows are tokens
+        auto make_g = [&](uint32_t k, int valid) {
+            const uint32_t ab = acc_it & 1;
+            ok = ok && mbar_wait(smem_u32(&acc_full[ab]), (acc_it >> 1) & 1);
+            tc_fence_after();
+            if (half == 0 && ok) {   // the first four warps write G
+                const bool active = row < valid;
+                float g[C::M];
+                tmem_ld_row<C::M>(tmem + lane_base + ab * C::NCH, g);
+                tc_fence_before();
+                act_fast_row<C::M>(a.act, g);
 #pragma unroll
-                    for (int b = 0; b < C::NB; ++b) {
-                        float gb[C::GB / 2];
+                for (int b = 0; b < C::NB; ++b) {
+                    float gb[C::GB / 2];
 #pragma unroll
-                        for (int j = 0; j < C::GB / 2; ++j) gb[j] = active ? g[b * (C::GB / 2) + j] : 0.0f;
-                        store_bf16_swz_row<C::GB / 2>(smem + C::OFF_G + b * (128 * C::GB), row, gb);
-                    }
-                    fence_async_smem();
+                    for (int j = 0; j < C::GB / 2; ++j) gb[j] = active ? g[b * (C::GB / 2) + j] : 0.0f;
+                    store_bf16_swz_row<C::GB / 2>(smem + C::OFF_G + (k % C::NGB) * C::TILE_BYTES + b * (128 * C::GB), row, gb);
                 }
-                mbar_arrive(smem_u32(&acc_empty[ab]));
-                ++acc_it;
-                named_barrier(1, C::EPI);
-                if (et == 0) mbar_arrive(smem_u32(&g_full));
+                fence_async_smem();
             }
-
-            for (int c = 0; c < nchunks && ok; ++c, ++acc_it, ++store_it) {
+            mbar_arrive(smem_u32(&acc_empty[ab]));
+            ++acc_it;
+            named_barrier(1, C::EPI);
+            if (et == 0) mbar_arrive(smem_u32(&g_full[k % C::NGB]));
+        };
+        auto valid_of = [&](int64_t tile) -> int {
+            const int64_t left = a.T - tile * 128;
+            return left < 128 ? (int)left : 128;
+        };
+        if (u_begin < u_end) {
+            int64_t tile;
+            int c0, c1;
+            seg_at(u_begin, tile, c0, c1);
+            make_g(0, valid_of(tile));
+        }
+        uint32_t k = 0;
+        for (int64_t u = u_begin; u < u_end && ok; ++k) {
+            int64_t tile;
+            int c0, c1;
+            seg_at(u, tile, c0, c1);
+            u = tile * nchunks + c1;
+            const bool has_next = u < u_end;
+            const int64_t t0 = tile * 128;
+            const int valid = valid_of(tile);
+            const uint8_t *bbuf = smem + C::OFF_B + (k % C::NGB) * C::TILE_BYTES;
+            for (int c = c0; c < c1 && ok; ++c, ++acc_it, ++store_it) {
+                if (C::LOOKAHEAD && c == c1 - 1 && has_next) {   // the next tile's G (its Q was issued before this chunk)
+                    int64_t nt;
+                    int n0, n1;
+                    seg_at(u, nt, n0, n1);
+                    make_g(k + 1, valid_of(nt));
+                    if (!ok) break;
+                }
                 const uint32_t ab = acc_it & 1;
                 const uint32_t sb = store_it & 1;
                 ok = mbar_wait(smem_u32(&acc_full[ab]), (acc_it >> 1) & 1);
@@ -238,10 +329,8 @@ __global__ void __launch_bounds__(320, 1)
                 if (et == 0) bulk_wait_read<1>();  // staging buffer sb is free again
                 named_barrier(1, C::EPI);
                 uint8_t *stg = smem + C::OFF_STG + sb * C::STG_BYTES;
-                const int64_t left = a.d - (int64_t)c * C::NCH;
-                const int ncols = left < C::NCH ? (int)left : C::NCH;
                 // a warp whose 32 rows all lie past the tile's valid tokens has nothing to store
-                const int gend = (q * 32 < valid) ? ncols : 0;
+                const int gend = (q * 32 < valid) ? C::NCH : 0;
                 // 64 columns (two TMEM loads in flight) at a time: one staging box
 #pragma unroll
                 for (int gh = 0; gh < C::NCH / 128; ++gh) {
@@ -259,13 +348,13 @@ __global__ void __launch_bounds__(320, 1)
                         float (&v)[32] = v2[h];
                         // identity path: the first r columns of Y get B (only chunk 0 holds them)
                         if (g * 32 < C::R && a.merge && c == 0) {
-                            const uint8_t *bblk = smem + C::OFF_B + ((g * 32) / (C::GB / 2)) * (128 * C::GB);
+                            const uint8_t *bblk = bbuf + ((g * 32) / (C::GB / 2)) * (128 * C::GB);
                             const uint32_t b0 = ((g * 32) % (C::GB / 2)) * 2;
 #pragma unroll
                             for (int i = 0; i < 32; i += 8) {
                                 if (g * 32 + i < C::R) {
-                                    const uint4 u = *reinterpret_cast<const uint4 *>(bblk + swz_offset(row, b0 + 2 * i, C::GB));
-                                    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+                                    const uint4 u4 = *reinterpret_cast<const uint4 *>(bblk + swz_offset(row, b0 + 2 * i, C::GB));
+                                    const uint32_t w[4] = {u4.x, u4.y, u4.z, u4.w};
 #pragma unroll
                                     for (int e = 0; e < 4; ++e) {
                                         v[i + 2 * e] += __uint_as_float(w[e] << 16);
@@ -294,9 +383,11 @@ __global__ void __launch_bounds__(320, 1)
                 fence_async_smem();
                 named_barrier(1, C::EPI);
                 if (et == 0) {
-                    if (c == 0) mbar_arrive(smem_u32(&b_empty));   // the B tile is no longer read
+                    // the segment's first chunk is drained: its B rows are no longer read (the Q
+                    // product and the identity path of chunk 0 are done)
+                    if (c == c0) mbar_arrive(smem_u32(&b_empty[k % C::NGB]));
                     const uint32_t sbase = smem_u32(stg);
-                    for (int b = 0; b < ncols / 64; ++b) {
+                    for (int b = 0; b < C::NCH / 64; ++b) {
                         const int x = c * C::NCH + 64 * b;
                         if (valid == 128) {
                             tma_store_2d_hint(&tm_y128, x, (int32_t)t0, sbase + b * 16384, l2_evict_first());
@@ -307,6 +398,12 @@ __global__ void __launch_bounds__(320, 1)
                     }
                     bulk_commit();
                 }
+            }
+            if (!C::LOOKAHEAD && ok && has_next) {   // one G buffer: the next tile's G after this segment
+                int64_t nt;
+                int n0, n1;
+                seg_at(u, nt, n0, n1);
+                make_g(k + 1, valid_of(nt));
             }
         }
         if (et == 0) bulk_wait<0>();
