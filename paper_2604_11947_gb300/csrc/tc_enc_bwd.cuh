@@ -42,7 +42,7 @@ template <int M_> struct EncBwdCfg {
     static constexpr int NSF = 3;                                // F ring depth
     static constexpr int NW = M_ <= 16 ? 4 : M_ <= 32 ? 2 : 3;   // We1 slice ring depth
     static constexpr int CLMAX = M_ <= 32 ? 4 : 1;               // CTAs per cluster (weight-gradient exchange)
-    static constexpr int CL_MIN_TOKENS = 320;                 // clusters only from this many tokens per CTA
+    static constexpr int CL_MIN_TOKENS = 256;                 // clusters only from this many tokens per CTA
     static constexpr int NWB = CLMAX > 1 ? 3 : 2;                // dWe1 accumulators in TMEM
     static constexpr int NDA = M_ <= 32 ? NT : 1;                // dA TMEM regions (a ring)
     static constexpr bool DPLO = M_ <= 32;                       // dP kept as bf16 hi + lo for dF
