@@ -41,9 +41,10 @@
  *     RESBM_ERR_CUDA (resbm_last_cuda_error() gives the cudaError_t value).
  *   - Outputs must not overlap inputs (X may alias F: both are only read).
  *   - Results are deterministic: the same inputs, descriptor and device give the same bits.
- *     (The tensor-core backward kernels run in thread-block clusters of 1, 2 or 4 CTAs, chosen
- *     from the device's occupancy and T; the environment variable RESBM_BWD_CLUSTER=1, 2 or 4
- *     forces a size where it fits. Each choice is deterministic; different choices add in
+ *     (The tensor-core backward kernels run in thread-block clusters of 1, 2 or 4 CTAs and the
+ *     encoder forward in pairs, chosen from the device's occupancy and T; the environment
+ *     variable RESBM_CLUSTER=1, 2 or 4 forces the backward size where it fits, and 1 also runs
+ *     the encoder forward as single CTAs. Each choice is deterministic; different choices add in
  *     different fixed orders, so results may differ between them in the last bits.)
  *   - T = 0 is valid: nothing is read, weight gradients are set to zero.
  *   - The scratch memory `ws` (device, >= resbm_workspace_bytes(...) bytes, 256-byte aligned)

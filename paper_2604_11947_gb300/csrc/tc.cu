@@ -151,11 +151,12 @@ int coresident_clusters(void (*kernel)(KArgs...), int cl, int threads, uint32_t 
 struct BwdShape {
     int grid, cl;
 };
-// RESBM_BWD_CLUSTER=1, 2 or 4 forces that cluster size (within the co-residency rule above,
-// regardless of min_tokens); unset or anything else: automatic. Read at every launch.
+// RESBM_CLUSTER=1, 2 or 4 forces that cluster size of the backward kernels (within the
+// co-residency rule above, regardless of min_tokens), and 1 runs the encoder forward as single
+// CTAs instead of pairs; unset or anything else: automatic. Read at every launch.
 int forced_cluster()
 {
-    const char *v = getenv("RESBM_BWD_CLUSTER");
+    const char *v = getenv("RESBM_CLUSTER");
     if (!v) return 0;
     const int n = atoi(v);
     return n == 1 || n == 2 || n == 4 ? n : 0;
@@ -239,7 +240,21 @@ cudaError_t launch_enc_fwd(const resbm_desc &d, const void *X, const void *F, co
     if (e != cudaSuccess) return e;
     tc::EncFwdArgs a{static_cast<const __nv_bfloat16 *>(X), static_cast<const __nv_bfloat16 *>(We2),
                      static_cast<__nv_bfloat16 *>(B), P, d.T, d.d, d.act};
-    e = launch(tc::k_enc_fwd<M>, grid_tokens(c, d.T), Cfg::THREADS, Cfg::SMEM_BYTES, c.stream, m_f128, m_f16, m_we1, a);
+    // pairs of CTAs (clusters of 2), one pair per two SMs and at most one per tile, when all the
+    // pairs fit at once; single CTAs otherwise
+    const int64_t tiles = (d.T + 127) / 128;
+    int cl = 1;
+    int64_t grid = tiles < c.sm_count ? (tiles < 1 ? 1 : tiles) : c.sm_count;
+    if (Cfg::SPLIT && forced_cluster() != 1) {   // RESBM_CLUSTER=1: single CTAs
+        static std::atomic<int> fit[kMaxDev][2];
+        int64_t pairs = tiles < c.sm_count / 2 ? (tiles < 1 ? 1 : tiles) : c.sm_count / 2;
+        if (pairs >= 1 && coresident_clusters(tc::k_enc_fwd<M>, 2, Cfg::THREADS, Cfg::SMEM_BYTES, c.device, fit) >= pairs) {
+            cl = 2;
+            grid = 2 * pairs;
+        }
+    }
+    e = launch_clustered(tc::k_enc_fwd<M>, (unsigned)grid, Cfg::THREADS, Cfg::SMEM_BYTES, cl, c.stream, m_f128, m_f16,
+                         m_we1, a);
     count_launches(1);
     return e;
 }

@@ -38,7 +38,7 @@ SMALL = {
     "bf16_single_ctas": synth.BoundaryConfig("bf16_single_ctas", T=40, d=256, r=32, m=32),
 }
 
-# Backward grids under each forced cluster size (RESBM_BWD_CLUSTER), one CTA per 128-token
+# Backward grids under each forced cluster size (RESBM_CLUSTER), one CTA per 128-token
 # tile at most: 8 tiles -> 8 CTAs in pairs or fours; 16 -> 16; 17 -> 16 in pairs or fours (one
 # idle SM); 18 -> 18 in pairs, no fours (16 < 15/16 x 18); 3 -> single CTAs (fours do not fit,
 # pairs leave too many idle); uneven tile groups inside clusters.
@@ -58,7 +58,7 @@ _ORACLE_CACHE = {}
 @pytest.mark.parametrize("name", CLUSTER_CASES)
 def test_forced_cluster_sizes_match_oracle(name, cluster, monkeypatch):
     """The backward kernels with every cluster size forced (1, 2, 4 CTAs), where it fits."""
-    monkeypatch.setenv("RESBM_BWD_CLUSTER", cluster)
+    monkeypatch.setenv("RESBM_CLUSTER", cluster)
     cfg = CLUSTER_CASES[name]
     h = host_inputs(cfg)
     dev = {k: to_dev(v, cfg) for k, v in h.items()}
