@@ -34,8 +34,13 @@ SMALL = {
     # the CTAs of a cluster have different group sizes but the same number of groups
     "bf16_uneven_groups": synth.BoundaryConfig("bf16_uneven_groups", T=79031, d=256, r=32, m=32),
     "bf16_uneven_groups_144": synth.BoundaryConfig("bf16_uneven_groups_144", T=74871, d=256, r=32, m=32),
-    # one partial tile: a single CTA
+    # one partial tile: a single CTA (the encoder forward: one pair splitting the tile's chunks)
     "bf16_single_ctas": synth.BoundaryConfig("bf16_single_ctas", T=40, d=256, r=32, m=32),
+    # the encoder forward's pairs with one 64-column chunk per tile (the split always falls on
+    # a tile boundary) and with three (a pair's single tile split 1 + 2); the other stages run
+    # on the portable kernels at these widths
+    "bf16_d64": synth.BoundaryConfig("bf16_d64", T=1000, d=64, r=32, m=32),
+    "bf16_d192": synth.BoundaryConfig("bf16_d192", T=300, d=192, r=32, m=32),
 }
 
 # Backward grids under each forced cluster size (RESBM_CLUSTER), one CTA per 128-token
