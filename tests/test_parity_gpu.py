@@ -55,6 +55,11 @@ CLUSTER_CASES = {
     "t18_r32": synth.BoundaryConfig("cl_t18_r32", T=2260, d=256, r=32, m=32),
     "t3_r32": synth.BoundaryConfig("cl_t3_r32", T=280, d=256, r=32, m=32),
     "uneven_r32": synth.BoundaryConfig("cl_uneven_r32", T=79031, d=256, r=32, m=32),
+    # 321 tiles on 152 CTAs (144 in fours): two or three tiles per CTA, the last one partial
+    # (77 tokens)
+    "t321_r32": synth.BoundaryConfig("cl_t321_r32", T=41037, d=256, r=32, m=32),
+    # 235 tiles: one or two per CTA, the last partial (48 tokens); three d chunks
+    "t235_d384_r16": synth.BoundaryConfig("cl_t235_d384_r16", T=30000, d=384, r=16, m=16),
 }
 _ORACLE_CACHE = {}
 
