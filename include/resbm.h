@@ -235,7 +235,9 @@ RESBM_API resbm_status resbm_boundary_step(const resbm_desc *desc, const resbm_s
  *   - Only what the step reads crosses to the device: X[:, :r] (the identity path is the only
  *     use of X), F, dY, the weights, and dX[:, :r] when dX is given; what comes back is B, Y, dB,
  *     dF, dX[:, :r] (dX given), P (P given) and the weight gradients. The rest of dX is not
- *     touched.
+ *     touched. When X or dX is page-locked and mapped into the device's address space (as
+ *     cudaHostAlloc memory is), a small kernel reads or writes those r columns in place through
+ *     the mapping; otherwise a strided copy moves them.
  *   - Everything is enqueued on `stream` (the call returns once it is enqueued; the host
  *     outputs are complete when `stream` reaches that point). Inside the call dY travels on a
  *     second stream while the forward stages run, and B and Y travel back on a third while the

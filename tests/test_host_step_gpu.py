@@ -118,3 +118,21 @@ def test_host_step_empty_batch():
     torch.cuda.synchronize()
     for k in ("dWe1", "dWe2", "dWd1", "dWd2"):
         assert torch.count_nonzero(out[k]) == 0, k
+
+
+def test_pinned_columns_move_through_the_host_mapping():
+    """With page-locked host buffers the r-column copies of X and dX run as a kernel on the host
+    mapping (three launches: X in, dX in, dX out); pageable buffers take strided copies. The
+    results are the same either way (test_host_step_matches_device_step)."""
+    cfg, flags = CASES["bf16_tc"]
+    desc = resbm.desc_from_config(cfg, flags)
+    ws = resbm.workspace(desc, resbm.RESBM_OP_BOUNDARY_STEP_HOST)
+    launches = {}
+    for pinned in (True, False):
+        h, out = _host_args(cfg, desc, flags, pinned)
+        torch.cuda.synchronize()
+        n0 = resbm.resbm_kernel_launches()
+        resbm.resbm_boundary_step_host(desc, ws, **h, **out)
+        torch.cuda.synchronize()
+        launches[pinned] = resbm.resbm_kernel_launches() - n0
+    assert launches[True] == launches[False] + 3, launches
