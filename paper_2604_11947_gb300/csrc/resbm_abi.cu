@@ -5,6 +5,10 @@
 #include <string.h>
 
 #include <atomic>
+#include <map>
+#include <memory>
+#include <mutex>
+#include <utility>
 
 #include "internal.h"
 #include "resbm.h"
@@ -54,6 +58,44 @@ void *mapped_host(const void *p)
 }
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Side streams and events of resbm_boundary_step_host, created on first use for each (device,
+// caller stream) and kept for the life of the process: creating and destroying streams in every
+// call costs host time in the driver. An event re-recorded by the next call on the same caller
+// stream is safe: a wait takes the state the event had when the wait was enqueued, and `mu`
+// keeps two host threads from interleaving their enqueues on one entry.
+struct SideStreams {
+    cudaStream_t in = nullptr, out = nullptr;
+    cudaEvent_t ev[4] = {};
+    std::mutex mu;
+};
+cudaError_t side_streams(cudaStream_t caller, SideStreams **out)
+{
+    static std::mutex mu;
+    static std::map<std::pair<int, cudaStream_t>, std::unique_ptr<SideStreams>> table;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    std::lock_guard<std::mutex> hold(mu);
+    std::unique_ptr<SideStreams> &slot = table[{dev, caller}];
+    if (!slot) {
+        std::unique_ptr<SideStreams> s(new SideStreams);
+        e = cudaStreamCreateWithFlags(&s->in, cudaStreamNonBlocking);
+        if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&s->out, cudaStreamNonBlocking);
+        for (int i = 0; i < 4 && e == cudaSuccess; ++i) e = cudaEventCreateWithFlags(&s->ev[i], cudaEventDisableTiming);
+        if (e != cudaSuccess) {
+            if (s->in) cudaStreamDestroy(s->in);
+            if (s->out) cudaStreamDestroy(s->out);
+            for (cudaEvent_t x : s->ev)
+                if (x) cudaEventDestroy(x);
+            table.erase({dev, caller});
+            return e;
+        }
+        slot = std::move(s);
+    }
+    *out = slot.get();
+    return cudaSuccess;
+}
 
 constexpr int kMaxDevices = 64;
 std::atomic<int> g_sm_count[kMaxDevices];
@@ -654,14 +696,14 @@ resbm_status resbm_boundary_step_host(const resbm_desc *desc, const resbm_step_a
     const size_t es = elem_size(d);
     const int64_t T = d.T, D = d.d, r = d.r, m = d.m;
     const bool lin = is_linear(d);
-    // two streams of this call (released once their work is done), forked from and joined
-    // back into the caller's stream
-    cudaStream_t s_in = nullptr, s_out = nullptr;
-    cudaEvent_t ev[4] = {};
-    cudaError_t e = cudaStreamCreateWithFlags(&s_in, cudaStreamNonBlocking);
-    if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&s_out, cudaStreamNonBlocking);
-    for (int i = 0; i < 4 && e == cudaSuccess; ++i) e = cudaEventCreateWithFlags(&ev[i], cudaEventDisableTiming);
-    cudaEvent_t fork = ev[0], dy_in = ev[1], fwd_done = ev[2], out_done = ev[3];
+    // two side streams, forked from and joined back into the caller's stream; kept per
+    // (device, caller stream) across calls, one call's enqueue at a time
+    SideStreams *side = nullptr;
+    cudaError_t e = side_streams(c.stream, &side);
+    if (e != cudaSuccess) return cuda_fail(e);
+    std::lock_guard<std::mutex> hold(side->mu);
+    cudaStream_t s_in = side->in, s_out = side->out;
+    cudaEvent_t fork = side->ev[0], dy_in = side->ev[1], fwd_done = side->ev[2], out_done = side->ev[3];
     auto h2d = [&](void *dst, const void *src, size_t bytes, cudaStream_t st) {
         if (e == cudaSuccess && bytes) e = cudaMemcpyAsync(dst, src, bytes, cudaMemcpyHostToDevice, st);
     };
@@ -689,17 +731,18 @@ resbm_status resbm_boundary_step_host(const resbm_desc *desc, const resbm_step_a
         count_launches(1);
         e = cudaGetLastError();
     };
-    // inputs: dY on the second stream, the rest on the caller's
-    if (e == cudaSuccess) e = cudaEventRecord(fork, c.stream);
-    if (e == cudaSuccess) e = cudaStreamWaitEvent(s_in, fork, 0);
-    h2d(const_cast<void *>(dv.dY), a->dY, (size_t)(T * D) * es, s_in);
-    if (e == cudaSuccess) e = cudaEventRecord(dy_in, s_in);
+    // inputs: what the forward reads first, on the caller's stream; then dY on the second
+    // stream, travelling in while the forward runs and its results travel out
     h2d(const_cast<void *>(dv.We1), a->We1, (size_t)(D * m) * es, c.stream);
     if (!lin) h2d(const_cast<void *>(dv.We2), a->We2, (size_t)(m * r) * es, c.stream);
     if (!lin) h2d(const_cast<void *>(dv.Wd1), a->Wd1, (size_t)(r * m) * es, c.stream);
     h2d(const_cast<void *>(dv.Wd2), a->Wd2, (size_t)(m * D) * es, c.stream);
     cols(const_cast<void *>(dv.X), a->X, cudaMemcpyHostToDevice, c.stream);   // the identity path reads X[:, :r] only
     h2d(const_cast<void *>(dv.F), a->F, (size_t)(T * D) * es, c.stream);
+    if (e == cudaSuccess) e = cudaEventRecord(fork, c.stream);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(s_in, fork, 0);
+    h2d(const_cast<void *>(dv.dY), a->dY, (size_t)(T * D) * es, s_in);
+    if (e == cudaSuccess) e = cudaEventRecord(dy_in, s_in);
     if (a->dX) cols(dv.dX, a->dX, cudaMemcpyHostToDevice, c.stream);          // the step adds dB to dX[:, :r] only
     if (e != cudaSuccess) s = cuda_fail(e);
     // the step, the forward results leaving on the third stream while the backward runs
@@ -720,11 +763,6 @@ resbm_status resbm_boundary_step_host(const resbm_desc *desc, const resbm_step_a
         if (e == cudaSuccess) e = cudaStreamWaitEvent(c.stream, out_done, 0);
         if (e != cudaSuccess) s = cuda_fail(e);
     }
-    // streams and events are released by the runtime once the work queued on them is done
-    for (cudaEvent_t x : ev)
-        if (x) cudaEventDestroy(x);
-    if (s_in) cudaStreamDestroy(s_in);
-    if (s_out) cudaStreamDestroy(s_out);
     return s;
 }
 
