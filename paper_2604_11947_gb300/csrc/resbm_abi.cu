@@ -348,27 +348,33 @@ resbm_status run_encode_fwd(const resbm_desc &d, const void *X, const void *F, c
     return finish(generic_encode_fwd(d, X, F, We1, We2, B, P, ws, c));
 }
 
+// on_tc (nullable): set when the tensor-core kernel (one launch, no scratch) ran
 resbm_status run_decode_fwd(const resbm_desc &d, const void *B, const void *Wd1, const void *Wd2,
-                            void *Y, void *ws, const Ctx &c)
+                            void *Y, void *ws, const Ctx &c, bool *on_tc = nullptr)
 {
+    if (on_tc) *on_tc = false;
     if (d.T == 0) return RESBM_OK;
     if (use_tc(d, RESBM_OP_DECODE_FWD)) {
         cudaError_t e = tc_decode_fwd(d, B, Wd1, Wd2, Y, ws, c);
-        if (e != cudaErrorNotSupported) return finish(e);
+        if (e != cudaErrorNotSupported) {
+            if (on_tc) *on_tc = e == cudaSuccess;
+            return finish(e);
+        }
     }
     return finish(generic_decode_fwd(d, B, Wd1, Wd2, Y, ws, c));
 }
 
+// after_independent: see tc_decode_bwd (the boundary step, right after its decoder forward)
 resbm_status run_decode_bwd(const resbm_desc &d, const void *dY, const void *B, const void *Wd1,
                             const void *Wd2, void *dB, float *dWd1, float *dWd2, void *ws,
-                            const Ctx &c)
+                            const Ctx &c, bool after_independent = false)
 {
     if (d.T == 0) {
         resbm_status s = zero_f32(dWd1, d.r * d.m, c.stream);
         return s != RESBM_OK ? s : zero_f32(dWd2, d.m * d.d, c.stream);
     }
     if (use_tc(d, RESBM_OP_DECODE_BWD)) {
-        cudaError_t e = tc_decode_bwd(d, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, c);
+        cudaError_t e = tc_decode_bwd(d, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, c, after_independent);
         if (e != cudaErrorNotSupported) return finish(e);
     }
     return finish(generic_decode_bwd(d, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, c));
@@ -475,10 +481,15 @@ resbm_status enqueue_step(const resbm_desc &d, const resbm_step_args &a, void *w
         inner = l.inner;
     }
     if (s == RESBM_OK) s = run_encode_fwd(e, a.X, a.F, a.We1, We2, a.B, P, inner, c);
-    if (s == RESBM_OK) s = run_decode_fwd(e, a.B, Wd1, a.Wd2, a.Y, inner, c);
+    bool dec_fwd_tc = false;
+    if (s == RESBM_OK) s = run_decode_fwd(e, a.B, Wd1, a.Wd2, a.Y, inner, c, &dec_fwd_tc);
     if (s == RESBM_OK && fwd_done) s = finish(cudaEventRecord(fwd_done, c.stream));
     if (s == RESBM_OK && bwd_ready) s = finish(cudaStreamWaitEvent(c.stream, bwd_ready, 0));
-    if (s == RESBM_OK) s = run_decode_bwd(e, a.dY, a.B, Wd1, a.Wd2, a.dB, dWd1, a.dWd2, inner, c);
+    // the decoder backward reads dY and B, not the decoder forward's Y, and the tensor-core
+    // decoder forward uses no scratch: with nothing queued between the two kernels the backward
+    // starts as the forward's CTAs leave (tc_decode_bwd)
+    const bool overlap = dec_fwd_tc && fwd_done == nullptr && bwd_ready == nullptr;
+    if (s == RESBM_OK) s = run_decode_bwd(e, a.dY, a.B, Wd1, a.Wd2, a.dB, dWd1, a.dWd2, inner, c, overlap);
     if (s == RESBM_OK)
         s = run_encode_bwd(e, a.dB, a.F, P, a.We1, We2, a.dF, a.dX, a.dWe1, dWe2, inner, c);
     return s;

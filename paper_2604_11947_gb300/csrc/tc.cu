@@ -328,7 +328,7 @@ cudaError_t launch_reduce(const tc::ReduceJob &small, tc::ReduceJob big, const C
 
 template <int M>
 cudaError_t launch_dec_bwd(const resbm_desc &d, const void *dY, const void *B, const void *Wd1, const void *Wd2,
-                           void *dB, float *dWd1, float *dWd2, void *ws, const Ctx &c)
+                           void *dB, float *dWd1, float *dWd2, void *ws, const Ctx &c, bool after_independent)
 {
     using Cfg = tc::DecBwdCfg<M>;
     static std::atomic<uint8_t> smem_set[kMaxDev];
@@ -348,7 +348,7 @@ cudaError_t launch_dec_bwd(const resbm_desc &d, const void *dY, const void *B, c
     tc::DecBwdArgs a{static_cast<const __nv_bfloat16 *>(Wd1),
                      static_cast<__nv_bfloat16 *>(dB),
                      tc::WgradArgs{p.part_big, p.nch},
-                     p.part_small, d.T, d.d, d.act, d.merge_identity, p.max_groups};
+                     p.part_small, d.T, d.d, d.act, d.merge_identity, p.max_groups, after_independent ? 1 : 0};
     e = launch_clustered(tc::k_dec_bwd<M>, p.grid, Cfg::THREADS, Cfg::SMEM_BYTES, sh.cl, c.stream, m_dy128, m_dy16,
                          m_wd2, m_b, m_yr, a);
     count_launches(1);
@@ -471,13 +471,13 @@ cudaError_t tc_decode_fwd(const resbm_desc &d, const void *B, const void *Wd1, c
 }
 
 cudaError_t tc_decode_bwd(const resbm_desc &d, const void *dY, const void *B, const void *Wd1, const void *Wd2,
-                          void *dB, float *dWd1, float *dWd2, void *ws, const Ctx &c)
+                          void *dB, float *dWd1, float *dWd2, void *ws, const Ctx &c, bool after_independent)
 {
     if (!al16(dY) || !al16(B) || !al16(Wd1) || !al16(Wd2) || !al16(dB)) return cudaErrorNotSupported;
     switch (d.m) {
-    case 16: return launch_dec_bwd<16>(d, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, c);
-    case 32: return launch_dec_bwd<32>(d, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, c);
-    case 64: return launch_dec_bwd<64>(d, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, c);
+    case 16: return launch_dec_bwd<16>(d, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, c, after_independent);
+    case 32: return launch_dec_bwd<32>(d, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, c, after_independent);
+    case 64: return launch_dec_bwd<64>(d, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, c, after_independent);
     }
     return cudaErrorNotSupported;
 }

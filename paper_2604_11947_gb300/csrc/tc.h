@@ -21,9 +21,12 @@ cudaError_t tc_encode_fwd(const resbm_desc &d, const void *X, const void *F, con
                           const void *We2, void *B, float *P_save, void *ws, const Ctx &c);
 cudaError_t tc_decode_fwd(const resbm_desc &d, const void *B, const void *Wd1, const void *Wd2,
                           void *Y, void *ws, const Ctx &c);
+// after_independent: the previous kernel on c.stream is the boundary step's decoder forward of
+// the same B (it reads B and writes Y only, and B was complete before it could let this launch
+// begin), so the kernel starts on SMs as that kernel's CTAs leave, without waiting for its end.
 cudaError_t tc_decode_bwd(const resbm_desc &d, const void *dY, const void *B, const void *Wd1,
                           const void *Wd2, void *dB, float *dWd1, float *dWd2, void *ws,
-                          const Ctx &c);
+                          const Ctx &c, bool after_independent = false);
 cudaError_t tc_encode_bwd(const resbm_desc &d, const void *dB, const void *F, const float *P_save,
                           const void *We1, const void *We2, void *dF, void *dX, float *dWe1,
                           float *dWe2, void *ws, const Ctx &c);

@@ -80,6 +80,10 @@ struct DecBwdArgs {
     float *part1;              // slots x r x m   (dWd1 partials)
     int64_t T, d;
     int act, merge, max_groups;
+    // 1: the previous kernel of the stream neither writes what this one reads nor reads what it
+    // writes (the boundary step's decoder forward), and what this one reads was complete when
+    // that kernel passed its own wait: start without waiting for it to finish
+    int after_independent;
 };
 
 template <int M_>
@@ -89,7 +93,7 @@ __global__ void __launch_bounds__(192, 1)
               const __grid_constant__ CUtensorMap tm_yr, const DecBwdArgs a)
 {
     using C = DecBwdCfg<M_>;
-    griddep_wait();               // the previous kernel of the stream has completed
+    if (!a.after_independent) griddep_wait();   // the previous kernel of the stream has completed
     griddep_launch_dependents();  // the next one may be scheduled on SMs as they free up
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
