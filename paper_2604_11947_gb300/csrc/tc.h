@@ -23,7 +23,9 @@ cudaError_t tc_decode_fwd(const resbm_desc &d, const void *B, const void *Wd1, c
                           void *Y, void *ws, const Ctx &c);
 // after_independent: the previous kernel on c.stream is the boundary step's decoder forward of
 // the same B (it reads B and writes Y only, and B was complete before it could let this launch
-// begin), so the kernel starts on SMs as that kernel's CTAs leave, without waiting for its end.
+// begin), so the kernel starts on SMs as that kernel's CTAs leave, without waiting for its end
+// (it waits for it before it exits, so it never completes first: later kernels of the stream,
+// which wait for their predecessor only, still find the decoder forward complete).
 cudaError_t tc_decode_bwd(const resbm_desc &d, const void *dY, const void *B, const void *Wd1,
                           const void *Wd2, void *dB, float *dWd1, float *dWd2, void *ws,
                           const Ctx &c, bool after_independent = false);

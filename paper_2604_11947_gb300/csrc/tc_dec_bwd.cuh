@@ -82,7 +82,7 @@ struct DecBwdArgs {
     int act, merge, max_groups;
     // 1: the previous kernel of the stream neither writes what this one reads nor reads what it
     // writes (the boundary step's decoder forward), and what this one reads was complete when
-    // that kernel passed its own wait: start without waiting for it to finish
+    // that kernel passed its own wait: start without waiting for it, and wait for it at the end
     int after_independent;
 };
 
@@ -527,6 +527,9 @@ __global__ void __launch_bounds__(192, 1)
         tmem_dealloc(tmem, C::TMEM_COLS);
     }
     if (C::CLMAX > 1 && xg.cl > 1) cluster_sync();   // no peer addresses this CTA's shared memory any more
+    // Started without waiting for the previous kernel: wait for it now, so that this grid does
+    // not complete before it (the kernels after this one wait for this grid only).
+    if (a.after_independent) griddep_wait();
 }
 
 // out = sum over slots s = 0, 1, ... of part[s] (rows x cols each, rows * cols % 4 == 0), each
