@@ -10,7 +10,8 @@
 // paced by its stages, not by bytes, so at T = 65536 the pairs make at most 3.5 tile passes
 // instead of 4 (the tensor's last tile may be partial).
 //   producer warp : for each tile, d in chunks of 64 columns: F tile chunk (128 x 64, K-major,
-//                   128B swizzle; 16-row boxes for a partial tile) + We1 rows (64 x m, MN-major)
+//                   128B swizzle; 16-row boxes for a partial tile) + We1 rows (64 x m, MN-major),
+//                   two consecutive chunks per ring stage for m <= 32
 //   MMA warp      : P (128 x m fp32 in TMEM, double-buffered per tile) += F_chunk . We1_chunk
 //   epilogue warps: TMEM -> registers (one token per thread), store P, A = phi(P) as a bf16
 //                   hi + lo pair in shared memory; the MMA warp then computes E = A . We2 into
@@ -32,7 +33,12 @@ template <int M_> struct EncFwdCfg {
     static constexpr uint32_t F_BYTES = 128 * 128;                      // 128 rows x 64 bf16
     static constexpr uint32_t W_BYTES = 64 * M_ * 2;                    // 64 rows x m bf16
     static constexpr uint32_t STAGE_BYTES = F_BYTES + W_BYTES;
-    static constexpr int NSTAGE = M_ <= 32 ? 8 : (M_ == 64 ? 6 : 3);
+    static constexpr int NSTAGE = M_ <= 32 ? 8 : (M_ == 64 ? 6 : 3);   // chunk slots
+    // chunks per ring stage (one barrier, one wait per stage): two consecutive 64-column chunks
+    // of a tile share a stage for m <= 32 (a tile's odd last chunk fills half a stage); per CTA
+    // the stream is paced by stages in flight, and 32 KB of F per stage streams faster than 16
+    static constexpr int SUB = M_ <= 32 ? 2 : 1;
+    static constexpr int NST = NSTAGE / SUB;                            // ring stages
     static constexpr uint32_t GB = M_ * 2 < 128 ? M_ * 2 : 128;        // row bytes (= swizzle) of an A block
     static constexpr int NB = M_ * 2 / GB;                              // blocks across the m columns
     static constexpr int SPB = GB / 32;                                 // 16-element K steps per block
@@ -104,7 +110,7 @@ __global__ void __launch_bounds__(192, 1)
     griddep_launch_dependents();  // the next one may be scheduled on SMs as they free up
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    __shared__ uint64_t full[C::NSTAGE], empty[C::NSTAGE];
+    __shared__ uint64_t full[C::NST], empty[C::NST];
     __shared__ uint64_t acc_full[2], acc_empty[2], a_full, e_full, done_bar, rx_full;
     __shared__ uint32_t tmem_base_sh;
 
@@ -126,7 +132,7 @@ __global__ void __launch_bounds__(192, 1)
     };
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < C::NSTAGE; ++s) {
+        for (int s = 0; s < C::NST; ++s) {
             mbar_init(smem_u32(&full[s]), 1);
             mbar_init(smem_u32(&empty[s]), 1);
         }
@@ -174,31 +180,35 @@ __global__ void __launch_bounds__(192, 1)
                 const uint32_t fbytes = valid == 128 ? C::F_BYTES : (uint32_t)nbox16 * 2048u;
                 int kc0, kc1;
                 chunks_of(ti, kc0, kc1);
-                for (int kc = kc0; kc < kc1; ++kc) {
-                    const uint32_t s = it % C::NSTAGE, ph = (it / C::NSTAGE) & 1;
+                for (int kc = kc0; kc < kc1; kc += C::SUB) {
+                    const int nsub = kc1 - kc < C::SUB ? kc1 - kc : C::SUB;   // chunks in this stage
+                    const uint32_t s = it % C::NST, ph = (it / C::NST) & 1;
                     if (!mbar_wait(smem_u32(&empty[s]), ph ^ 1)) {
                         ok = false;
                         break;
                     }
-                    const uint32_t fdst = smem_u32(smem + C::OFF_STAGE + s * C::STAGE_BYTES);
-                    const uint32_t wdst = fdst + C::F_BYTES;
                     const uint32_t bar = smem_u32(&full[s]);
-                    mbar_expect_tx(bar, fbytes + C::W_BYTES);
-                    if (valid == 128) {
-                        tma_load_2d_hint(fdst, &tm_f128, kc * 64, (int32_t)t0, bar, stream_pol);
-                    } else {
-                        for (int rg = 0; rg < nbox16; ++rg)
-                            tma_load_2d_hint(fdst + rg * 2048, &tm_f16, kc * 64, (int32_t)(t0 + 16 * rg), bar, stream_pol);
+                    mbar_expect_tx(bar, (uint32_t)nsub * (fbytes + C::W_BYTES));
+                    for (int j = 0; j < nsub; ++j) {
+                        const uint32_t fdst = smem_u32(smem + C::OFF_STAGE + (s * C::SUB + j) * C::STAGE_BYTES);
+                        const uint32_t wdst = fdst + C::F_BYTES;
+                        if (valid == 128) {
+                            tma_load_2d_hint(fdst, &tm_f128, (kc + j) * 64, (int32_t)t0, bar, stream_pol);
+                        } else {
+                            for (int rg = 0; rg < nbox16; ++rg)
+                                tma_load_2d_hint(fdst + rg * 2048, &tm_f16, (kc + j) * 64, (int32_t)(t0 + 16 * rg), bar,
+                                                 stream_pol);
+                        }
+                        for (int wb = 0; wb < C::WBOXES; ++wb)
+                            tma_load_2d(wdst + wb * 64 * C::WSW, &tm_we1, wb * 64, (kc + j) * 64, bar);
                     }
-                    for (int wb = 0; wb < C::WBOXES; ++wb)
-                        tma_load_2d(wdst + wb * 64 * C::WSW, &tm_we1, wb * 64, kc * 64, bar);
                     ++it;
                 }
             }
-            const uint32_t n = it < (uint32_t)C::NSTAGE ? it : (uint32_t)C::NSTAGE;
+            const uint32_t n = it < (uint32_t)C::NST ? it : (uint32_t)C::NST;
             for (uint32_t k = 0; k < n; ++k) {
                 const uint32_t j = it - 1 - k;
-                mbar_wait(smem_u32(&full[j % C::NSTAGE]), (j / C::NSTAGE) & 1);
+                mbar_wait(smem_u32(&full[j % C::NST]), (j / C::NST) & 1);
             }
         }
     } else if (warp == 1) {
@@ -249,17 +259,20 @@ __global__ void __launch_bounds__(192, 1)
                 tc_fence_after();
                 int kc0, kc1;
                 chunks_of(ti, kc0, kc1);
-                for (int kc = kc0; kc < kc1 && ok; ++kc, ++it) {
-                    const uint32_t s = it % C::NSTAGE, ph = (it / C::NSTAGE) & 1;
+                for (int kc = kc0; kc < kc1 && ok; kc += C::SUB, ++it) {
+                    const int nsub = kc1 - kc < C::SUB ? kc1 - kc : C::SUB;
+                    const uint32_t s = it % C::NST, ph = (it / C::NST) & 1;
                     ok = wait_serving_e(smem_u32(&full[s]), ph);
                     tc_fence_after();
-                    const uint32_t faddr = smem_u32(smem + C::OFF_STAGE + s * C::STAGE_BYTES);
-                    const uint32_t waddr = faddr + C::F_BYTES;
+                    for (int j = 0; j < nsub; ++j) {
+                        const uint32_t faddr = smem_u32(smem + C::OFF_STAGE + (s * C::SUB + j) * C::STAGE_BYTES);
+                        const uint32_t waddr = faddr + C::F_BYTES;
 #pragma unroll
-                    for (int k = 0; k < 4; ++k) {
-                        const uint64_t ad = smem_desc(faddr + k * 32, 16, 1024, kSwz128);
-                        const uint64_t bd = smem_desc(waddr + k * 16 * C::WSW, 64 * C::WSW, 8 * C::WSW, wswz);
-                        mma_bf16(tmem + ab * C::ACC_STRIDE, ad, bd, idesc, kc != kc0 || k != 0);
+                        for (int k = 0; k < 4; ++k) {
+                            const uint64_t ad = smem_desc(faddr + k * 32, 16, 1024, kSwz128);
+                            const uint64_t bd = smem_desc(waddr + k * 16 * C::WSW, 64 * C::WSW, 8 * C::WSW, wswz);
+                            mma_bf16(tmem + ab * C::ACC_STRIDE, ad, bd, idesc, kc + j != kc0 || k != 0);
+                        }
                     }
                     mma_commit(smem_u32(&empty[s]));
                 }
