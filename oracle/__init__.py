@@ -11,6 +11,8 @@ Citations (sections and equations of the ResBM paper):
                                across the boundary; identity path) and
                                Eq. generalized_transformer_equation
   decode_bwd / encode_bwd .... the chain rule of the two forward functions
+  effective_rank ............. the appendix's spectral analysis of the bottleneck output
+                               projections: r_eff = sum_i sigma_i^2 / max_i sigma_i^2
 """
 import ctypes
 import os
@@ -264,6 +266,21 @@ class Oracle:
         dF, dX, dWe1, dWe2 = self.encode_bwd(dB, F, We1, We2, act)
         return dict(B=B, P=P, Y=Y, dB=dB, dF=dF, dX=dX, dWe1=dWe1, dWe2=dWe2,
                     dWd1=dWd1, dWd2=dWd2)
+
+
+def effective_rank(W):
+    """r_eff of a matrix as the appendix's spectral analysis defines it: the sum of its squared
+    singular values over the largest squared singular value (1 when one singular value
+    dominates, the smaller dimension when all are equal; 0 for the zero matrix). Singular
+    values from numpy's SVD in float64."""
+    W = np.asarray(W, dtype=np.float64)
+    if W.ndim != 2:
+        raise ValueError("effective_rank takes a matrix")
+    if W.size == 0:
+        return 0.0
+    sig = np.linalg.svd(W, compute_uv=False)
+    top = float(np.max(sig)) ** 2
+    return 0.0 if top == 0.0 else float(np.sum(sig * sig)) / top
 
 
 _default = None
