@@ -57,17 +57,6 @@ def check_output(name, got, want, cfg, dX0=None):
     return check(name, g, want, cfg.dtype)
 
 
-def sample_tokens(T, n, seed=0, tile=128):
-    """Tokens to check at full size: the ends, both sides of tile edges, and random ones."""
-    rng = np.random.default_rng(seed)
-    fixed = {0, 1, T - 1, T - 2}
-    for t in (tile - 1, tile, 2 * tile - 1, T // 2, T // 2 + 1, T - tile, T - tile - 1):
-        if 0 <= t < T:
-            fixed.add(t)
-    rest = rng.choice(T, size=min(T, max(0, n - len(fixed))), replace=False)
-    return np.array(sorted(fixed | set(int(x) for x in rest)))
-
-
 def _ws(desc, op):
     return resbm.workspace(desc, op)
 

@@ -8,8 +8,7 @@ import ctypes
 import pytest
 import torch
 
-from gpu_helpers import host_inputs, to_dev, to_host
-from metrics import check
+from gpu_helpers import host_inputs, to_dev
 from paper_2604_11947_gb300 import build, resbm, synth
 
 CASES = {
@@ -47,8 +46,11 @@ def test_noalloc_matches_decode_bwd_two_calls_in_a_row(case):
         got = _outputs(cfg)
         resbm.resbm_decode_bwd_noalloc(desc, dY, dev["B"], dev["Wd1"], dev["Wd2"], *got)
         torch.cuda.synchronize()
+        # the same kernels on the same inputs with the same launch shapes: only the scratch
+        # address differs, so every output must match bit for bit
         for name, g, w in zip(("dB", "dWd1", "dWd2"), got, want):
-            check(name, to_host(g), to_host(w), cfg.dtype)
+            assert torch.equal(g, w), "%s differs from resbm_decode_bwd (max |diff| %.3e)" % (
+                name, float((g.float() - w.float()).abs().max()))
     assert resbm.resbm_device_error() == 0
 
 
@@ -62,11 +64,16 @@ def test_noalloc_reserves_no_device_memory_per_call():
     out = _outputs(cfg)
     resbm.resbm_decode_bwd_noalloc(desc, dev["dY"], B, dev["Wd1"], dev["Wd2"], *out)
     torch.cuda.synchronize()
+    # torch's caching allocator sees no request (the library never calls into torch), and the
+    # device's free memory does not move (the library calls no cudaMalloc either)
+    alloc0, reserved0 = torch.cuda.memory_allocated(), torch.cuda.memory_reserved()
     free0, _ = torch.cuda.mem_get_info()
     for _ in range(3):
         resbm.resbm_decode_bwd_noalloc(desc, dev["dY"], B, dev["Wd1"], dev["Wd2"], *out)
     torch.cuda.synchronize()
     free1, _ = torch.cuda.mem_get_info()
+    assert torch.cuda.memory_allocated() == alloc0
+    assert torch.cuda.memory_reserved() == reserved0
     assert free1 == free0
 
 
