@@ -45,6 +45,8 @@ def parse():
     p.add_argument("--generic", action="store_true", help="force the CUDA-core kernels")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true", help="skip the oracle CPU baseline")
+    p.add_argument("--no-extra", action="store_true",
+                   help="skip the other workloads (T=16384 d=2048 r=16 and the d=8192 r-sweep)")
     return p.parse_args()
 
 
@@ -72,13 +74,20 @@ def op_flops(cfg):
             "enc_bwd": 2 * T * (r * m + 2 * d * m + m * r)}
 
 
+NOMINAL_HBM_GBS = 8000.0    # the GB300's nominal HBM3e bandwidth (the 70 % target is stated on it)
+TARGET_FRAC = 0.70
+
+
 def measured_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(path):
         with open(path) as f:
             j = json.load(f)
-        return {"hbm_gbs": j["hbm_gbs"], "bf16_tflops": j["bf16_tflops"], "source": "measured"}
-    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "source": "fallback"}
+        return {"hbm_gbs": j["hbm_gbs"], "bf16_tflops": j["bf16_tflops"],
+                "bf16_tflops_sustained": j.get("bf16_tflops_sustained", j["bf16_tflops"]),
+                "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+            "source": "fallback"}
 
 
 def kernel_sources_sha():
@@ -269,6 +278,127 @@ def job_throughput(tokens_per_rank, world, steps, ms_total):
 
 
 # ---- the GPU arm ----------------------------------------------------------------------------
+def device_inputs(cfg, torch, reuse=None):
+    """The workload's seeded inputs in HBM. `reuse`: tensors of another workload with the same
+    (T, d) whose X, F, dY are the same draws (the tensors depend only on their shapes)."""
+    io = torch.bfloat16 if cfg.dtype == "bf16" else torch.float32
+    dev = {}
+    for k in ("X", "F", "dY", "We1", "We2", "Wd1", "Wd2"):
+        if reuse is not None and k in ("X", "F", "dY") and reuse[k].shape == synth.shapes(cfg)[k]:
+            dev[k] = reuse[k]
+        else:
+            dev[k] = torch.from_numpy(synth.tensor(cfg, k)).to("cuda").to(io)
+    return dev
+
+
+class Workload:
+    """One workload's device tensors and its two ways of running a step: the library's step call
+    (timed for `value`) and the four op calls with events between them (per-op times)."""
+
+    def __init__(self, cfg, flags, dev, resbm, torch):
+        self.cfg, self.dev, self.resbm, self.torch = cfg, dev, resbm, torch
+        self.desc = resbm.desc_from_config(cfg, flags)
+        self.out = resbm.step_outputs(self.desc)
+        self.ws = resbm.workspace(self.desc, resbm.RESBM_OP_BOUNDARY_STEP)
+        self.stream = torch.cuda.current_stream()
+
+    def fused_step(self):
+        d, o = self.dev, self.out
+        self.resbm.resbm_boundary_step(self.desc, self.ws, X=d["X"], F=d["F"], dY=d["dY"], We1=d["We1"],
+                                       We2=d["We2"], Wd1=d["Wd1"], Wd2=d["Wd2"], **o)
+
+    def op_step(self, ev=None):
+        r, d, o, desc, ws = self.resbm, self.dev, self.out, self.desc, self.ws
+        if ev is not None:
+            ev[0].record(self.stream)
+        r.resbm_encode_fwd(desc, d["X"], d["F"], d["We1"], d["We2"], o["B"], o["P"], ws)
+        if ev is not None:
+            ev[1].record(self.stream)
+        r.resbm_decode_fwd(desc, o["B"], d["Wd1"], d["Wd2"], o["Y"], ws)
+        if ev is not None:
+            ev[2].record(self.stream)
+        r.resbm_decode_bwd(desc, d["dY"], o["B"], d["Wd1"], d["Wd2"], o["dB"], o["dWd1"], o["dWd2"], ws)
+        if ev is not None:
+            ev[3].record(self.stream)
+        r.resbm_encode_bwd(desc, o["dB"], d["F"], o["P"], d["We1"], d["We2"], o["dF"], o["dX"],
+                           o["dWe1"], o["dWe2"], ws)
+        if ev is not None:
+            ev[4].record(self.stream)
+
+    def warm(self, n):
+        for _ in range(max(n, 0)):
+            self.fused_step()
+        for _ in range(max(n, 0)):
+            self.op_step()
+        self.torch.cuda.synchronize()
+
+    def time_steps(self, steps):
+        """ms of `steps` step calls between two events, no event in between (an event between
+        two kernels ends their programmatic-dependent-launch overlap), and the launches they
+        made."""
+        torch = self.torch
+        start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        l0 = self.resbm.resbm_kernel_launches()
+        start.record(self.stream)
+        for _ in range(steps):
+            self.fused_step()
+        end.record(self.stream)
+        torch.cuda.synchronize()
+        return start.elapsed_time(end), self.resbm.resbm_kernel_launches() - l0
+
+    def time_ops(self, steps):
+        """Mean ms of each op over `steps` op-wise steps (CUDA events on the launching stream)."""
+        torch = self.torch
+        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(steps)]
+        for i in range(steps):
+            self.op_step(evs[i])
+        torch.cuda.synchronize()
+        return {op: statistics.mean(evs[i][j].elapsed_time(evs[i][j + 1]) for i in range(steps))
+                for j, op in enumerate(OPS)}
+
+
+def per_op_table(cfg, op_ms, peaks):
+    """Each op's time, algorithmic GB/s and FLOP rate, and its fractions of the measured copy
+    bandwidth, of the nominal 8 TB/s and of the sustained bf16 tensor rate."""
+    bytes_, flops = op_bytes(cfg), op_flops(cfg)
+    t = {}
+    for o in OPS:
+        gbs = bytes_[o] / (op_ms[o] / 1e3) / 1e9
+        tfs = flops[o] / (op_ms[o] / 1e3) / 1e12
+        t[o] = {"ms": op_ms[o], "alg_bytes": bytes_[o], "GBps": gbs, "frac": gbs / peaks["hbm_gbs"],
+                "frac_of_8TBps": gbs / NOMINAL_HBM_GBS, "TFLOPs": tfs,
+                "frac_of_bf16_sustained": tfs / peaks["bf16_tflops_sustained"]}
+    return t
+
+
+def extra_workload(name, cfg, flags, resbm, torch, steps, warmup, peaks, reuse=None):
+    """The step on another workload (fewer steps): tokens/s, GB/s and per-op fractions."""
+    dev = device_inputs(cfg, torch, reuse)
+    w = Workload(cfg, flags, dev, resbm, torch)
+    w.warm(warmup)
+    ms, launches = w.time_steps(steps)
+    op_ms = w.time_ops(steps)
+    ms_step = ms / steps
+    step_bytes = sum(op_bytes(cfg).values())
+    step_flops = sum(op_flops(cfg).values())
+    per_op = per_op_table(cfg, op_ms, peaks)
+    res = {"workload": describe(cfg)["workload"], "steps": steps, "warmup": warmup,
+           "value": cfg.T / (ms_step / 1e3), "unit": "tokens/s", "ms_per_step": ms_step,
+           "step_GBps": step_bytes / (ms_step / 1e3) / 1e9,
+           "step_frac": step_bytes / (ms_step / 1e3) / 1e9 / peaks["hbm_gbs"],
+           "step_TFLOPs": step_flops / (ms_step / 1e3) / 1e12,
+           "gpu_launches_per_step": launches / steps,
+           "min_op_frac": min(v["frac"] for v in per_op.values()),
+           "per_op": per_op}
+    if cfg.r >= 256:   # compute-bound point: the tensor rate is its roofline
+        res["bound"] = "tensor"
+        res["step_frac_of_bf16_sustained"] = res["step_TFLOPs"] / peaks["bf16_tflops_sustained"]
+    else:
+        res["bound"] = "hbm"
+    del w
+    return res, dev
+
+
 def main():
     args = parse()
     cfg = synth.CONFIGS[args.config]
@@ -293,48 +423,14 @@ def main():
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     build.build()
-    lib = resbm.load()
+    resbm.load()
 
     flags = resbm.RESBM_FLAG_GENERIC if args.generic else 0
-    desc = resbm.desc_from_config(cfg, flags)
-    io = torch.bfloat16 if cfg.dtype == "bf16" else torch.float32
-    dev = {k: torch.from_numpy(synth.tensor(cfg, k)).to("cuda").to(io)
-           for k in ("X", "F", "dY", "We1", "We2", "Wd1", "Wd2")}
-    out = resbm.step_outputs(desc)
-    ws = resbm.workspace(desc, resbm.RESBM_OP_BOUNDARY_STEP)
-    wsz = ws.numel()
-    stream = torch.cuda.current_stream()
+    peaks = measured_peaks()
+    dev = device_inputs(cfg, torch)
+    w = Workload(cfg, flags, dev, resbm, torch)
+    w.warm(args.warmup)
 
-    def step(ev=None):
-        if ev is not None:
-            ev[0].record(stream)
-        resbm.resbm_encode_fwd(desc, dev["X"], dev["F"], dev["We1"], dev["We2"], out["B"], out["P"], ws)
-        if ev is not None:
-            ev[1].record(stream)
-        resbm.resbm_decode_fwd(desc, out["B"], dev["Wd1"], dev["Wd2"], out["Y"], ws)
-        if ev is not None:
-            ev[2].record(stream)
-        resbm.resbm_decode_bwd(desc, dev["dY"], out["B"], dev["Wd1"], dev["Wd2"], out["dB"],
-                               out["dWd1"], out["dWd2"], ws)
-        if ev is not None:
-            ev[3].record(stream)
-        resbm.resbm_encode_bwd(desc, out["dB"], dev["F"], out["P"], dev["We1"], dev["We2"],
-                               out["dF"], out["dX"], out["dWe1"], out["dWe2"], ws)
-        if ev is not None:
-            ev[4].record(stream)
-
-    def fused_step():
-        resbm.resbm_boundary_step(desc, ws, X=dev["X"], F=dev["F"], dY=dev["dY"], We1=dev["We1"],
-                                  We2=dev["We2"], Wd1=dev["Wd1"], Wd2=dev["Wd2"], **out)
-
-    for _ in range(max(args.warmup, 0)):
-        fused_step()
-    for _ in range(max(args.warmup, 0)):
-        step()
-    torch.cuda.synchronize()
-
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(args.steps)]
-    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     props = torch.cuda.get_device_properties(local)
     uuid = getattr(props, "uuid", None)
     uuid = None if uuid is None else (str(uuid) if str(uuid).startswith("GPU-") else "GPU-" + str(uuid))
@@ -344,51 +440,59 @@ def main():
     torch.cuda.synchronize()
     clocks.start()
     time.sleep(0.15)
-    # timed region: K boundary steps through the library's step call, no events in between
-    # (an event between two kernels ends their programmatic-dependent-launch overlap)
-    launches0 = resbm.resbm_kernel_launches()
-    start.record(stream)
-    for i in range(args.steps):
-        fused_step()
-    end.record(stream)
-    torch.cuda.synchronize()
-    launches = resbm.resbm_kernel_launches() - launches0
+    # timed region: K boundary steps through the library's step call
+    ms_total, launches = w.time_steps(args.steps)
     # second timed pass, same K steps as four op calls with events between them: the per-op
     # times of the roofline (these steps are a few percent slower than the ones above)
-    for i in range(args.steps):
-        step(evs[i])
-    torch.cuda.synchronize()
+    op_ms = w.time_ops(args.steps)
     if dist:
         dist.barrier()
     clk = clocks.stop()
-    ms_total = max_over_ranks(start.elapsed_time(end), dist, "cuda")
+    ms_total = max_over_ranks(ms_total, dist, "cuda")
     ms_step = ms_total / max(args.steps, 1)
     value = job_throughput(cfg.T, world, args.steps, ms_total)
 
-    op_ms = {op: statistics.mean(evs[i][j].elapsed_time(evs[i][j + 1]) for i in range(args.steps))
-             for j, op in enumerate(OPS)}
     bytes_ = op_bytes(cfg)
-    flops = op_flops(cfg)
-    peaks = measured_peaks()
+    per_op = per_op_table(cfg, op_ms, peaks)
     dom = max(OPS, key=lambda o: op_ms[o])
-    achieved = bytes_[dom] / (op_ms[dom] / 1e3) / 1e9
+    worst = min(OPS, key=lambda o: per_op[o]["frac"])
+    achieved = per_op[dom]["GBps"]
     step_bytes = sum(bytes_.values())
     roofline = {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peaks["hbm_gbs"],
                 "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"],
+                "frac_of_8TBps": achieved / NOMINAL_HBM_GBS,
                 "traffic": traffic_for(dom, cfg),
                 "peak_source": peaks["source"] + " copy bandwidth (MEASURED_PEAKS.json hbm_gbs)",
                 "algorithmic_bytes_per_launch": bytes_[dom],
                 "timing": "per-op CUDA events on the launching stream in a second timed pass "
                           "of the same K steps (op calls with events between them)",
-                "per_op": {o: {"ms": op_ms[o], "alg_bytes": bytes_[o],
-                               "GBps": bytes_[o] / (op_ms[o] / 1e3) / 1e9,
-                               "frac": bytes_[o] / (op_ms[o] / 1e3) / 1e9 / peaks["hbm_gbs"],
-                               "TFLOPs": flops[o] / (op_ms[o] / 1e3) / 1e12} for o in OPS},
+                "min_op": worst, "min_op_frac": per_op[worst]["frac"],
+                "min_op_frac_of_8TBps": per_op[worst]["frac_of_8TBps"],
+                "target": "every op >= %.2f of peak HBM" % TARGET_FRAC,
+                "target_met_of_measured": all(v["frac"] >= TARGET_FRAC for v in per_op.values()),
+                "target_met_of_8TBps": all(v["frac_of_8TBps"] >= TARGET_FRAC for v in per_op.values()),
+                "per_op": per_op,
                 "step_GBps": step_bytes / (ms_step / 1e3) / 1e9}
 
     e2e = None
     if not args.no_e2e:
-        e2e = run_e2e(args, cfg, desc, dev, out, ws, resbm, torch, dist, world)
+        e2e = run_e2e(args, cfg, w, resbm, torch, dist, world)
+    del w
+
+    extra = None
+    if rank == 0 and world == 1 and not args.no_extra and not args.tokens:
+        del dev
+        torch.cuda.empty_cache()
+        extra = {}
+        k_extra, w_extra = max(3, min(args.steps, 50)), max(3, min(args.warmup, 5))
+        extra["single_bf16"], _ = extra_workload("single_bf16", synth.CONFIGS["single_bf16"], flags, resbm,
+                                                 torch, k_extra, w_extra, peaks)
+        reuse = None
+        for name in ("sweep_r32", "sweep_r64", "sweep_r128", "sweep_r512"):
+            extra[name], reuse = extra_workload(name, synth.CONFIGS[name], flags, resbm, torch,
+                                                k_extra, w_extra, peaks, reuse)
+        del reuse
+        torch.cuda.empty_cache()
 
     line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
@@ -401,6 +505,8 @@ def main():
             "hbm_GBps_step": roofline["step_GBps"],
             "roofline": roofline, "e2e": e2e, "gpu_launches": launches,
             "clocks": clk}
+    if extra is not None:
+        line["workloads"] = extra
     if rank == 0 and world == 1 and not args.no_cpu:
         line["cpu_baseline"] = cpu_baseline(cfg)
     if rank == 0:
@@ -409,24 +515,29 @@ def main():
         dist.destroy_process_group()
 
 
-def run_e2e(args, cfg, desc, dev, out, ws, resbm, torch, dist, world):
+def run_e2e(args, cfg, w, resbm, torch, dist, world):
     """The same step through the C ABI with HOST buffers (resbm_boundary_step_host): inputs in
     pinned host memory, results back into pinned host memory, every copy inside the call and
-    inside the timed region. Two calls are kept in flight (two streams, two device workspaces,
-    two sets of host results), so one step's results travel back while the next step's inputs
-    travel in, as a training loop fed from the host would run them."""
+    inside the timed region. The step is the one `value` times, dX[:, :r] += dB included (a
+    pinned host dX whose first r columns travel in and back). Two calls are kept in flight (two
+    streams, two device workspaces, two sets of host results), so one step's results travel back
+    while the next step's inputs travel in, as a training loop fed from the host would run them."""
+    desc, dev, out = w.desc, w.dev, w.out
     ins = ("X", "F", "dY", "We1", "We2", "Wd1", "Wd2")
     res = ("B", "Y", "dB", "dF", "dWe1", "dWe2", "dWd1", "dWd2")
     host_in = {k: dev[k].cpu().pin_memory() for k in ins}
     host_out = [{k: torch.empty(out[k].shape, dtype=out[k].dtype).pin_memory() for k in res}
                 for _ in range(2)]
+    for h in host_out:   # the residual gradient dX[:, :r] += dB accumulates into
+        h["dX"] = torch.zeros(out["dX"].shape, dtype=out["dX"].dtype).pin_memory()
     wss = [resbm.workspace(desc, resbm.RESBM_OP_BOUNDARY_STEP_HOST) for _ in range(2)]
     streams = [torch.cuda.Stream() for _ in range(2)]
     es = host_in["F"].element_size()
-    # what the call copies: X[:, :r] only (the identity path), F, dY and the weights in; the
-    # results out
-    h2d = cfg.T * cfg.r * es + sum(host_in[k].numel() * es for k in ins if k != "X")
-    d2h = sum(t.numel() * t.element_size() for t in host_out[0].values())
+    cols = cfg.T * cfg.r * es   # X[:, :r] and dX[:, :r]: the only columns of X and dX the step uses
+    # what the call copies: X[:, :r], dX[:, :r], F, dY and the weights in; the results and
+    # dX[:, :r] out
+    h2d = 2 * cols + sum(host_in[k].numel() * es for k in ins if k != "X")
+    d2h = cols + sum(host_out[0][k].numel() * host_out[0][k].element_size() for k in res)
     # up to 100 steps (≈0.65 s): the host link sometimes stalls for ~100 ms (seen as 30-55 ms
     # gaps between consecutive steps whose steady pace is 6.4 ms); a short window would charge
     # one such stall to a handful of steps
@@ -449,7 +560,7 @@ def run_e2e(args, cfg, desc, dev, out, ws, resbm, torch, dist, world):
     return {"value": job_throughput(cfg.T, world, n, ms), "unit": "tokens/s",
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": n,
             "ms_per_step": ms / n,
-            "api": "resbm_boundary_step_host (host buffers; copies inside the call)",
+            "api": "resbm_boundary_step_host (host buffers; copies inside the call; dX[:, :r] += dB)",
             "pipelined": "two calls in flight on two streams with two device workspaces; "
                          "host wall clock from the first copy to the last result on the host"}
 

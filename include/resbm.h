@@ -96,6 +96,12 @@ typedef enum {
  * m == r; act is not used; We2 and Wd1 are not read and dWe2 and dWd1 not written (all may be
  * NULL). Everything else, the identity path included, is as in the two-layer form. */
 #define RESBM_FLAG_LINEAR 2u
+/* Run every op as its chain of tensor-core products with fused element-wise steps (the path
+ * the library takes by itself for bf16 shapes the fused boundary kernels do not cover, e.g.
+ * m = r = 512, or the backward at m = 128, or m != r) even where the fused kernels would run.
+ * bf16 only, d, r and m multiples of 8, 16-byte aligned pointers; otherwise the portable
+ * kernels run. For testing and comparing the two tensor-core paths. */
+#define RESBM_FLAG_GEMM 4u
 
 typedef struct {
     int64_t T;               /* tokens (batch * sequence), >= 0                              */
@@ -244,6 +250,10 @@ RESBM_API resbm_status resbm_boundary_step(const resbm_desc *desc, const resbm_s
  *     backward stages run; both are forked from and joined back into `stream`. Calls on
  *     different streams with different workspaces may run at the same time, so a caller can
  *     overlap one step's results with the next step's inputs.
+ *   - The two side streams and four events are created on the first call for each (device,
+ *     caller stream) pair and kept until the process exits (creating them in every call costs
+ *     driver time). A caller that passes a new stream to every call therefore accumulates two
+ *     streams and four events per distinct stream handle: reuse a small set of streams.
  *   - Errors: as resbm_boundary_step; RESBM_ERR_CUDA if a copy or a stream could not be set up. */
 RESBM_API resbm_status resbm_boundary_step_host(const resbm_desc *desc, const resbm_step_args *args,
                                       void *ws, size_t ws_bytes, void *stream);

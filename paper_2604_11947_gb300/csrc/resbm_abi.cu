@@ -149,7 +149,7 @@ resbm_status check_desc(const resbm_desc *d)
     if (d->act != RESBM_ACT_SILU && d->act != RESBM_ACT_GELU_TANH && d->act != RESBM_ACT_IDENTITY)
         return RESBM_ERR_INVALID_ARG;
     if (d->merge_identity != 0 && d->merge_identity != 1) return RESBM_ERR_INVALID_ARG;
-    if (d->flags & ~(RESBM_FLAG_GENERIC | RESBM_FLAG_LINEAR)) return RESBM_ERR_INVALID_ARG;
+    if (d->flags & ~(RESBM_FLAG_GENERIC | RESBM_FLAG_LINEAR | RESBM_FLAG_GEMM)) return RESBM_ERR_INVALID_ARG;
     if ((d->flags & RESBM_FLAG_LINEAR) && d->m != d->r) return RESBM_ERR_INVALID_ARG;
     // every element count (and the byte counts derived from it) must fit in int64
     const int64_t big = INT64_MAX / 64;
@@ -190,7 +190,13 @@ template <size_t N> bool any_overlap(const Range (&outs)[N], const Range *ins, s
     return false;
 }
 
-bool use_tc(const resbm_desc &d, int op) { return !(d.flags & RESBM_FLAG_GENERIC) && tc_supported(d, op); }
+// Which kernels run an op: the fused tensor-core kernels where they take the shape (unless a
+// flag says otherwise), else the tensor-core GEMM chain, else the portable CUDA-core kernels.
+bool use_tc(const resbm_desc &d, int op)
+{
+    return !(d.flags & (RESBM_FLAG_GENERIC | RESBM_FLAG_GEMM)) && tc_supported(d, op);
+}
+bool use_gemm(const resbm_desc &d, int op) { return !(d.flags & RESBM_FLAG_GENERIC) && gemm_supported(d, op); }
 
 // ---- RESBM_FLAG_LINEAR ---------------------------------------------------------------------
 // One linear layer per side runs as the two-layer path with identity second layers
@@ -232,7 +238,9 @@ size_t ws_for(const resbm_desc &d0, int op)
     const resbm_desc d = two_layer(d0);
     size_t g = generic_ws_bytes(d, op);
     size_t t = tc_supported(d, op) ? tc_ws_bytes(d, op, sizing_sms()) : 0;
-    const size_t inner = g > t ? g : t;
+    size_t k = gemm_supported(d, op) ? gemm_ws_bytes(d, op, sizing_sms()) : 0;
+    size_t inner = g > t ? g : t;
+    if (k > inner) inner = k;
     return is_linear(d0) ? carve_linear(d0, nullptr).bytes + inner : inner;
 }
 
@@ -345,6 +353,10 @@ resbm_status run_encode_fwd(const resbm_desc &d, const void *X, const void *F, c
         cudaError_t e = tc_encode_fwd(d, X, F, We1, We2, B, P, ws, c);
         if (e != cudaErrorNotSupported) return finish(e);
     }
+    if (use_gemm(d, RESBM_OP_ENCODE_FWD)) {
+        cudaError_t e = gemm_encode_fwd(d, X, F, We1, We2, B, P, ws, c);
+        if (e != cudaErrorNotSupported) return finish(e);
+    }
     return finish(generic_encode_fwd(d, X, F, We1, We2, B, P, ws, c));
 }
 
@@ -360,6 +372,10 @@ resbm_status run_decode_fwd(const resbm_desc &d, const void *B, const void *Wd1,
             if (on_tc) *on_tc = e == cudaSuccess;
             return finish(e);
         }
+    }
+    if (use_gemm(d, RESBM_OP_DECODE_FWD)) {
+        cudaError_t e = gemm_decode_fwd(d, B, Wd1, Wd2, Y, ws, c);
+        if (e != cudaErrorNotSupported) return finish(e);
     }
     return finish(generic_decode_fwd(d, B, Wd1, Wd2, Y, ws, c));
 }
@@ -377,6 +393,10 @@ resbm_status run_decode_bwd(const resbm_desc &d, const void *dY, const void *B, 
         cudaError_t e = tc_decode_bwd(d, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, c, after_independent);
         if (e != cudaErrorNotSupported) return finish(e);
     }
+    if (use_gemm(d, RESBM_OP_DECODE_BWD)) {
+        cudaError_t e = gemm_decode_bwd(d, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, c);
+        if (e != cudaErrorNotSupported) return finish(e);
+    }
     return finish(generic_decode_bwd(d, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, c));
 }
 
@@ -390,6 +410,10 @@ resbm_status run_encode_bwd(const resbm_desc &d, const void *dB, const void *F, 
     }
     if (use_tc(d, RESBM_OP_ENCODE_BWD)) {
         cudaError_t e = tc_encode_bwd(d, dB, F, P, We1, We2, dF, dX, dWe1, dWe2, ws, c);
+        if (e != cudaErrorNotSupported) return finish(e);
+    }
+    if (use_gemm(d, RESBM_OP_ENCODE_BWD)) {
+        cudaError_t e = gemm_encode_bwd(d, dB, F, P, We1, We2, dF, dX, dWe1, dWe2, ws, c);
         if (e != cudaErrorNotSupported) return finish(e);
     }
     return finish(generic_encode_bwd(d, dB, F, P, We1, We2, dF, dX, dWe1, dWe2, ws, c));

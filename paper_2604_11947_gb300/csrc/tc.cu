@@ -18,6 +18,7 @@
 #include "tc_enc_fwd.cuh"
 #include "tc_dec_bwd.cuh"
 #include "tc_enc_bwd.cuh"
+#include "tc_gemm.cuh"
 
 namespace resbm {
 
@@ -421,6 +422,177 @@ cudaError_t launch_enc_bwd(const resbm_desc &d, const void *dB, const void *F, c
                          reduce_job(p.part_big, p.grid / sh.cl, d.d, d.m, dWe1, 0, al16(dWe1), cap), c);
 }
 
+// ---- the GEMM chain (tc_gemm.cuh) --------------------------------------------------------
+// C = A . B with A M x K (a_mn: stored K x M row-major, else M x K) and B K x N (b_mn: stored
+// K x N row-major, else N x K), all bf16 with row pitches equal to the stored widths.
+int gemm_bn(int64_t N) { return N > 128 ? 256 : 128; }
+
+// Split-K of a product with few output tiles (the weight gradients, K = tokens): enough splits
+// to give every SM a unit, at most 32 and at least four 64-deep K slices per split.
+int gemm_splits(int64_t M, int64_t N, int64_t K, int sms)
+{
+    const int bn = gemm_bn(N);
+    const int64_t units = ((M + 127) / 128) * ((N + bn - 1) / bn);
+    if (4 * units >= 3 * (int64_t)sms) return 1;
+    int64_t s = sms / units;
+    const int64_t kmax = (K + 255) / 256;
+    if (s > kmax) s = kmax;
+    if (s > 32) s = 32;
+    if (s < 1) s = 1;
+    const int64_t kc = ((K + s - 1) / s + 63) / 64 * 64;
+    return (int)((K + kc - 1) / kc);
+}
+
+template <int BN, bool AMN, bool BMN, bool ALO>
+cudaError_t launch_gemm_t(const CUtensorMap &ma, const CUtensorMap &malo, const CUtensorMap &mb,
+                          const tc::GemmShape &g, const tc::GemmEp &ep, const Ctx &c)
+{
+    using Cfg = tc::GemmCfg<BN, ALO>;
+    static std::atomic<uint8_t> smem_set[kMaxDev];
+    cudaError_t e = ensure_smem(tc::k_gemm<BN, AMN, BMN, ALO>, Cfg::SMEM_BYTES, c.device, smem_set);
+    if (e != cudaSuccess) return e;
+    const int64_t grid = g.units < c.sm_count ? g.units : c.sm_count;
+    e = launch(tc::k_gemm<BN, AMN, BMN, ALO>, (unsigned)grid, Cfg::THREADS, Cfg::SMEM_BYTES, c.stream, ma, malo, mb,
+               g, ep);
+    count_launches(1);
+    return e;
+}
+
+// splits: 1 for every product whose epilogue is not a plain fp32 store; with splits > 1 the
+// epilogue must be GEP_F32 into `splits` slots of M x N (ep.split_stride apart). A_lo (K-major A
+// only): the lo half of A as a bf16 hi + lo pair (same shape as A), or null.
+cudaError_t gemm(const Ctx &c, int64_t M, int64_t N, int64_t K, const void *A, bool a_mn, const void *B, bool b_mn,
+                 const tc::GemmEp &ep, int splits, const void *A_lo = nullptr)
+{
+    if (M <= 0 || N <= 0 || K <= 0) return cudaSuccess;
+    if (A_lo && a_mn) return cudaErrorNotSupported;
+    const int bn = gemm_bn(N);
+    CUtensorMap ma, malo, mbm;
+    const bool okA = a_mn ? make_map(&ma, A, M, K, M * 2, 64, 64, CU_TENSOR_MAP_SWIZZLE_128B)
+                          : make_map(&ma, A, K, M, K * 2, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B);
+    const bool okL = A_lo ? make_map(&malo, A_lo, K, M, K * 2, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B) : true;
+    const bool okB = b_mn ? make_map(&mbm, B, N, K, N * 2, 64, 64, CU_TENSOR_MAP_SWIZZLE_128B)
+                          : make_map(&mbm, B, K, N, K * 2, 64, (uint32_t)bn, CU_TENSOR_MAP_SWIZZLE_128B);
+    if (!okA || !okL || !okB) return cudaErrorInvalidValue;
+    if (!A_lo) malo = ma;   // not read
+    tc::GemmShape g;
+    g.M = M;
+    g.N = N;
+    g.K = K;
+    g.splits = splits < 1 ? 1 : splits;
+    g.kc = ((K + g.splits - 1) / g.splits + 63) / 64 * 64;
+    g.splits = (int)((K + g.kc - 1) / g.kc);
+    g.nm = (int)((M + 127) / 128);
+    g.nn = (int)((N + bn - 1) / bn);
+    g.units = (int64_t)g.nm * g.nn * g.splits;
+    const bool lo = A_lo != nullptr;
+    if (bn == 256) {
+        if (!a_mn && b_mn) return lo ? launch_gemm_t<256, false, true, true>(ma, malo, mbm, g, ep, c)
+                                     : launch_gemm_t<256, false, true, false>(ma, malo, mbm, g, ep, c);
+        if (!a_mn && !b_mn) return lo ? launch_gemm_t<256, false, false, true>(ma, malo, mbm, g, ep, c)
+                                      : launch_gemm_t<256, false, false, false>(ma, malo, mbm, g, ep, c);
+        if (a_mn && b_mn) return launch_gemm_t<256, true, true, false>(ma, malo, mbm, g, ep, c);
+    } else {
+        if (!a_mn && b_mn) return lo ? launch_gemm_t<128, false, true, true>(ma, malo, mbm, g, ep, c)
+                                     : launch_gemm_t<128, false, true, false>(ma, malo, mbm, g, ep, c);
+        if (!a_mn && !b_mn) return lo ? launch_gemm_t<128, false, false, true>(ma, malo, mbm, g, ep, c)
+                                      : launch_gemm_t<128, false, false, false>(ma, malo, mbm, g, ep, c);
+        if (a_mn && b_mn) return launch_gemm_t<128, true, true, false>(ma, malo, mbm, g, ep, c);
+    }
+    return cudaErrorNotSupported;
+}
+
+tc::GemmEp ep_of(int mode, int act, void *out, int64_t ldo)
+{
+    tc::GemmEp e{};
+    e.mode = mode;
+    e.act = act;
+    e.out = out;
+    e.ldo = ldo;
+    return e;
+}
+
+// A weight gradient W (M x N fp32) = A^T . B over K tokens (both operands MN-major), split over
+// the tokens when it has few output tiles: the splits' fp32 slots go to `slots` and the job to
+// sum them (in slot order) is returned in `job` (job->blocks = 0: nothing to reduce).
+cudaError_t wgrad(const Ctx &c, int64_t M, int64_t N, int64_t K, const void *A, const void *B, float *W, float *slots,
+                  tc::ReduceJob *job)
+{
+    const int s = gemm_splits(M, N, K, c.sm_count);
+    *job = tc::ReduceJob{nullptr, 0, 0, 0, nullptr, 0, 0, 0};
+    if (s <= 1) return gemm(c, M, N, K, A, true, B, true, ep_of(tc::GEP_F32, 0, W, N), 1);
+    tc::GemmEp e = ep_of(tc::GEP_F32, 0, slots, N);
+    e.split_stride = M * N;
+    cudaError_t err = gemm(c, M, N, K, A, true, B, true, e, s);
+    if (err != cudaSuccess) return err;
+    // the number of splits the launch took (gemm rounds K per split to 64)
+    const int64_t kc = ((K + s - 1) / s + 63) / 64 * 64;
+    const int64_t ns = (K + kc - 1) / kc;
+    *job = reduce_job(slots, ns, M, N, W, 0, al16(W), (int64_t)c.sm_count * 8);
+    return cudaSuccess;
+}
+
+cudaError_t reduce_jobs(const tc::ReduceJob &a, const tc::ReduceJob &b, const Ctx &c)
+{
+    if (a.blocks == 0 && b.blocks == 0) return cudaSuccess;
+    const tc::ReduceJob none{nullptr, 0, 0, 0, nullptr, 0, 0, 0};
+    const tc::ReduceJob &first = a.blocks ? a : none;
+    const tc::ReduceJob &second = a.blocks ? (b.blocks ? b : none) : b;
+    const int blocks = first.blocks + second.blocks;
+    const cudaError_t e = launch(tc::k_reduce_slots, blocks, kReduceBlock, 0, c.stream, first, second);
+    count_launches(1);
+    return e;
+}
+
+// Scratch of the GEMM chain of each op (grid == the device's SMs): the intermediate T x m
+// tensors and the weight gradients' split slots.
+struct GemmWs {
+    float *P = nullptr, *Q = nullptr;
+    __nv_bfloat16 *A = nullptr, *G = nullptr, *dQ = nullptr, *dP = nullptr;
+    __nv_bfloat16 *A_lo = nullptr, *dQ_lo = nullptr, *dP_lo = nullptr;   // remainders of hi + lo pairs
+    float *slots1 = nullptr, *slots2 = nullptr;
+    size_t bytes = 0;
+};
+
+// dF = dP . We1^T takes dP as a hi + lo pair up to this hidden width (K = m is short there and
+// the product is bound by the dF stream; at larger m it would double the op's largest product)
+constexpr int64_t kDfLoMaxM = 64;
+
+size_t slot_floats(int64_t M, int64_t N, int64_t K, int sms)
+{
+    const int s = gemm_splits(M, N, K, sms);
+    return s > 1 ? (size_t)(s * M * N) : 0;
+}
+
+GemmWs gemm_ws(const resbm_desc &d, int op, int sms, void *ws, bool have_P)
+{
+    GemmWs w;
+    WsCarver cv(ws);
+    const int64_t T = d.T, D = d.d, r = d.r, m = d.m;
+    if (op == RESBM_OP_ENCODE_FWD) {
+        w.A = cv.take<__nv_bfloat16>(T * m);
+        w.A_lo = cv.take<__nv_bfloat16>(T * m);
+    } else if (op == RESBM_OP_DECODE_FWD) {
+        w.G = cv.take<__nv_bfloat16>(T * m);
+    } else if (op == RESBM_OP_DECODE_BWD) {
+        w.Q = cv.take<float>(T * m);
+        w.G = cv.take<__nv_bfloat16>(T * m);
+        w.dQ = cv.take<__nv_bfloat16>(T * m);
+        w.dQ_lo = cv.take<__nv_bfloat16>(T * m);
+        w.slots1 = cv.take<float>(slot_floats(m, D, T, sms));   // dWd2
+        w.slots2 = cv.take<float>(slot_floats(r, m, T, sms));   // dWd1
+    } else if (op == RESBM_OP_ENCODE_BWD) {
+        if (!have_P) w.P = cv.take<float>(T * m);
+        w.A = cv.take<__nv_bfloat16>(T * m);
+        w.dP = cv.take<__nv_bfloat16>(T * m);
+        if (m <= kDfLoMaxM) w.dP_lo = cv.take<__nv_bfloat16>(T * m);
+        w.slots1 = cv.take<float>(slot_floats(D, m, T, sms));   // dWe1
+        w.slots2 = cv.take<float>(slot_floats(m, r, T, sms));   // dWe2
+    }
+    w.bytes = cv.used;
+    return w;
+}
+
 }  // namespace
 
 bool tc_supported(const resbm_desc &d, int op)
@@ -493,6 +665,124 @@ cudaError_t tc_encode_bwd(const resbm_desc &d, const void *dB, const void *F, co
     case 64: return launch_enc_bwd<64>(d, dB, F, P, We1, We2, dF, dX, dWe1, dWe2, ws, c);
     }
     return cudaErrorNotSupported;
+}
+
+// ---- the GEMM chain of each op ------------------------------------------------------------
+bool gemm_supported(const resbm_desc &d, int op)
+{
+    if (d.dtype != RESBM_BF16 || d.T > INT32_MAX || encode_fn() == nullptr) return false;
+    if (d.d % 8 || d.r % 8 || d.m % 8) return false;   // 16-byte row pitches (TMA, vector epilogues)
+    return op >= RESBM_OP_ENCODE_FWD && op <= RESBM_OP_ENCODE_BWD;
+}
+
+size_t gemm_ws_bytes(const resbm_desc &d, int op, int sms) { return gemm_ws(d, op, sms, nullptr, false).bytes; }
+
+cudaError_t gemm_encode_fwd(const resbm_desc &d, const void *X, const void *F, const void *We1, const void *We2,
+                            void *B, float *P, void *ws, const Ctx &c)
+{
+    if (!al16(X) || !al16(F) || !al16(We1) || !al16(We2) || !al16(B) || (P && !al16(P)) || !al16(ws))
+        return cudaErrorNotSupported;
+    const GemmWs w = gemm_ws(d, RESBM_OP_ENCODE_FWD, c.sm_count, ws, true);
+    // P = F . We1 (saved if asked), A = phi(P)
+    tc::GemmEp e1 = ep_of(tc::GEP_P_A, d.act, P, d.m);
+    e1.out2 = w.A;
+    e1.ldo2 = d.m;
+    e1.lo = w.A_lo;
+    cudaError_t e = gemm(c, d.T, d.m, d.d, F, false, We1, true, e1, 1);
+    if (e != cudaSuccess) return e;
+    // B = X[:, :r] + (A_hi + A_lo) . We2 (the truncating identity path added in the epilogue)
+    tc::GemmEp e2 = ep_of(tc::GEP_ADD_AUX, d.act, B, d.r);
+    e2.aux = X;
+    e2.lda = d.d;
+    e2.aux_cols = d.r;
+    return gemm(c, d.T, d.r, d.m, w.A, false, We2, true, e2, 1, w.A_lo);
+}
+
+cudaError_t gemm_decode_fwd(const resbm_desc &d, const void *B, const void *Wd1, const void *Wd2, void *Y, void *ws,
+                            const Ctx &c)
+{
+    if (!al16(B) || !al16(Wd1) || !al16(Wd2) || !al16(Y) || !al16(ws)) return cudaErrorNotSupported;
+    const GemmWs w = gemm_ws(d, RESBM_OP_DECODE_FWD, c.sm_count, ws, true);
+    // G = phi(B . Wd1)
+    cudaError_t e = gemm(c, d.T, d.m, d.r, B, false, Wd1, true, ep_of(tc::GEP_ACT, d.act, w.G, d.m), 1);
+    if (e != cudaSuccess) return e;
+    // Y = G . Wd2 (+ B on the first r columns: the zero-padding identity path)
+    tc::GemmEp e2 = ep_of(tc::GEP_ADD_AUX, d.act, Y, d.d);
+    e2.aux = d.merge_identity ? B : nullptr;
+    e2.lda = d.r;
+    e2.aux_cols = d.merge_identity ? d.r : 0;
+    return gemm(c, d.T, d.d, d.m, w.G, false, Wd2, true, e2, 1);
+}
+
+cudaError_t gemm_decode_bwd(const resbm_desc &d, const void *dY, const void *B, const void *Wd1, const void *Wd2,
+                            void *dB, float *dWd1, float *dWd2, void *ws, const Ctx &c)
+{
+    if (!al16(dY) || !al16(B) || !al16(Wd1) || !al16(Wd2) || !al16(dB) || !al16(dWd1) || !al16(dWd2) || !al16(ws))
+        return cudaErrorNotSupported;
+    const GemmWs w = gemm_ws(d, RESBM_OP_DECODE_BWD, c.sm_count, ws, true);
+    // Q = B . Wd1 (kept), G = phi(Q)
+    tc::GemmEp e1 = ep_of(tc::GEP_ACT, d.act, w.G, d.m);
+    e1.out2 = w.Q;
+    e1.ldo2 = d.m;
+    cudaError_t e = gemm(c, d.T, d.m, d.r, B, false, Wd1, true, e1, 1);
+    // dQ = (dY . Wd2^T) * phi'(Q)
+    tc::GemmEp e2 = ep_of(tc::GEP_DACT, d.act, w.dQ, d.m);
+    e2.aux = w.Q;
+    e2.lda = d.m;
+    e2.lo = w.dQ_lo;
+    if (e == cudaSuccess) e = gemm(c, d.T, d.m, d.d, dY, false, Wd2, false, e2, 1);
+    // dB = [merge] dY[:, :r] + (dQ_hi + dQ_lo) . Wd1^T
+    tc::GemmEp e3 = ep_of(tc::GEP_ADD_AUX, d.act, dB, d.r);
+    e3.aux = d.merge_identity ? dY : nullptr;
+    e3.lda = d.d;
+    e3.aux_cols = d.merge_identity ? d.r : 0;
+    if (e == cudaSuccess) e = gemm(c, d.T, d.r, d.m, w.dQ, false, Wd1, false, e3, 1, w.dQ_lo);
+    // dWd2 = G^T . dY, dWd1 = B^T . dQ (sums over the tokens)
+    tc::ReduceJob j2, j1;
+    if (e == cudaSuccess) e = wgrad(c, d.m, d.d, d.T, w.G, dY, dWd2, w.slots1, &j2);
+    if (e == cudaSuccess) e = wgrad(c, d.r, d.m, d.T, B, w.dQ, dWd1, w.slots2, &j1);
+    if (e == cudaSuccess) e = reduce_jobs(j1, j2, c);
+    return e;
+}
+
+cudaError_t gemm_encode_bwd(const resbm_desc &d, const void *dB, const void *F, const float *P, const void *We1,
+                            const void *We2, void *dF, void *dX, float *dWe1, float *dWe2, void *ws, const Ctx &c)
+{
+    if (!al16(dB) || !al16(F) || (P && !al16(P)) || !al16(We1) || !al16(We2) || !al16(dF) || (dX && !al16(dX)) ||
+        !al16(dWe1) || !al16(dWe2) || !al16(ws))
+        return cudaErrorNotSupported;
+    const GemmWs w = gemm_ws(d, RESBM_OP_ENCODE_BWD, c.sm_count, ws, P != nullptr);
+    cudaError_t e = cudaSuccess;
+    if (!P) {   // P = F . We1, the forward's own product (the same launch shape, so the same bits)
+        tc::GemmEp e0 = ep_of(tc::GEP_P_A, d.act, w.P, d.m);
+        e0.out2 = w.A;   // overwritten below; the forward writes A too
+        e0.ldo2 = d.m;
+        e = gemm(c, d.T, d.m, d.d, F, false, We1, true, e0, 1);
+        P = w.P;
+    }
+    // dP = (dB . We2^T) * phi'(P), and A = phi(P) for dWe2
+    tc::GemmEp e1 = ep_of(tc::GEP_DACT, d.act, w.dP, d.m);
+    e1.aux = P;
+    e1.lda = d.m;
+    e1.out2 = w.A;
+    e1.ldo2 = d.m;
+    e1.lo = w.dP_lo;
+    if (e == cudaSuccess) e = gemm(c, d.T, d.m, d.r, dB, false, We2, false, e1, 1);
+    // dF = dP . We1^T (dP as a hi + lo pair at small m), and dX[:, :r] += dB (the gradient of
+    // the truncating identity path)
+    tc::GemmEp e2 = ep_of(tc::GEP_DF, d.act, dF, d.d);
+    e2.rmw = static_cast<__nv_bfloat16 *>(dX);
+    e2.ldr = d.d;
+    e2.aux = dB;
+    e2.lda = d.r;
+    e2.aux_cols = d.r;
+    if (e == cudaSuccess) e = gemm(c, d.T, d.d, d.m, w.dP, false, We1, false, e2, 1, w.dP_lo);
+    // dWe1 = F^T . dP, dWe2 = A^T . dB
+    tc::ReduceJob j1, j2;
+    if (e == cudaSuccess) e = wgrad(c, d.d, d.m, d.T, F, w.dP, dWe1, w.slots1, &j1);
+    if (e == cudaSuccess) e = wgrad(c, d.m, d.r, d.T, w.A, dB, dWe2, w.slots2, &j2);
+    if (e == cudaSuccess) e = reduce_jobs(j2, j1, c);
+    return e;
 }
 
 namespace tc {

@@ -33,4 +33,21 @@ cudaError_t tc_encode_bwd(const resbm_desc &d, const void *dB, const void *F, co
                           const void *We1, const void *We2, void *dF, void *dX, float *dWe1,
                           float *dWe2, void *ws, const Ctx &c);
 
+// The GEMM chain (tc_gemm.cuh): every op as a sequence of tcgen05 products with fused
+// epilogues, for bf16 shapes the fused kernels do not take (m = r = 512, the r = 128 backward,
+// m != r). Needs d, r, m multiples of 8 and 16-byte aligned pointers (else cudaErrorNotSupported
+// before anything is enqueued).
+bool gemm_supported(const resbm_desc &d, int op);
+size_t gemm_ws_bytes(const resbm_desc &d, int op, int sms);
+cudaError_t gemm_encode_fwd(const resbm_desc &d, const void *X, const void *F, const void *We1,
+                            const void *We2, void *B, float *P_save, void *ws, const Ctx &c);
+cudaError_t gemm_decode_fwd(const resbm_desc &d, const void *B, const void *Wd1, const void *Wd2,
+                            void *Y, void *ws, const Ctx &c);
+cudaError_t gemm_decode_bwd(const resbm_desc &d, const void *dY, const void *B, const void *Wd1,
+                            const void *Wd2, void *dB, float *dWd1, float *dWd2, void *ws,
+                            const Ctx &c);
+cudaError_t gemm_encode_bwd(const resbm_desc &d, const void *dB, const void *F, const float *P_save,
+                            const void *We1, const void *We2, void *dF, void *dX, float *dWe1,
+                            float *dWe2, void *ws, const Ctx &c);
+
 }  // namespace resbm

@@ -320,6 +320,7 @@ __global__ void __launch_bounds__(192, 1)
                         const uint32_t s = yit % C::NSY;
                         ok = mbar_wait(smem_u32(&y_full[s]), (yit / C::NSY) & 1);
                         tc_fence_after();
+                        if (!ok) break;   // a wait gave up: issue nothing more
                         const uint64_t yk = yk0 + ((s * C::Y_STAGE) >> 4);
                         const uint64_t ym = ym0 + ((s * C::Y_STAGE) >> 4);
                         const uint64_t gm = gm0 + (i - tb) * TILE16;
@@ -334,6 +335,7 @@ __global__ void __launch_bounds__(192, 1)
                         if (c == 0) {
                             ok = ok && mbar_wait(smem_u32(&g_full[i - tb]), g & 1);
                             tc_fence_after();
+                            if (!ok) break;
                         }
                         // dWd2T_chunk += dY_tile^T . G_tile: K = the tile's tokens in steps of 16
                         if (valid == 128) {
@@ -360,6 +362,7 @@ __global__ void __launch_bounds__(192, 1)
                     const int valid = (int)((end - t0) < 128 ? (end - t0) : 128);
                     ok = mbar_wait(smem_u32(&dq_full[i - tb]), g & 1);
                     tc_fence_after();
+                    if (!ok) break;
                     const uint64_t qk = qk0 + (i - tb) * TILE16;
                     const uint64_t qm = qm0 + (i - tb) * TILE16;
                     const uint64_t bm = bm0 + (i - tb) * TILE16;

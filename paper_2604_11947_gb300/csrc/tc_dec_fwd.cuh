@@ -244,6 +244,7 @@ __global__ void __launch_bounds__(320, 1)
                     ok = mbar_wait(smem_u32(&w_full[s]), ph) &&
                          mbar_wait(smem_u32(&acc_empty[ab]), ((acc_it >> 1) & 1) ^ 1);
                     tc_fence_after();
+                    if (!ok) break;   // a wait gave up: issue nothing more
                     const uint32_t waddr = smem_u32(smem + C::OFF_W + s * C::W_STAGE_BYTES);
 #pragma unroll
                     for (int kk = 0; kk < C::M / 16; ++kk) {

@@ -296,6 +296,7 @@ __global__ void __launch_bounds__(192, 1)
                     const int valid = (int)((end - t0) < 128 ? (end - t0) : 128);
                     ok = mbar_wait(smem_u32(&dp_full[i - tb]), g & 1);
                     tc_fence_after();
+                    if (!ok) break;   // a wait gave up: issue nothing more
                     const uint64_t am = am0 + (i - tb) * TILE16;
                     const uint64_t dbm = dbm0 + (i - tb) * TILE16;
                     const int nks = (valid + 15) / 16;
@@ -311,6 +312,7 @@ __global__ void __launch_bounds__(192, 1)
                     ok = mbar_wait(smem_u32(&w_full[sw]), (wit / C::NW) & 1) &&
                          mbar_wait(smem_u32(&we_empty[ae]), ((cit / C::NWB) & 1) ^ 1);
                     tc_fence_after();
+                    if (!ok) break;
                     const uint64_t wd = wd0 + ((sw * C::W_STAGE) >> 4);
                     const uint32_t d_we = tmem + C::TM_WE + ae * C::MS;
                     for (int i = tb; i < te && ok; ++i, ++dfit, ++j) {
@@ -321,6 +323,7 @@ __global__ void __launch_bounds__(192, 1)
                              mbar_wait(smem_u32(&df_empty[ad_buf]), ((dfit >> 1) & 1) ^ 1);
                         fpar ^= 1u << s;
                         tc_fence_after();
+                        if (!ok) break;
                         const uint64_t fm = fm0 + ((s * C::F_STAGE) >> 4);
                         const uint64_t pk = pk0 + (i - tb) * TILE16;
                         const uint64_t pm = pm0 + (i - tb) * TILE16;

@@ -257,6 +257,7 @@ __global__ void __launch_bounds__(192, 1)
                 const uint32_t ab = ti & 1;
                 ok = wait_serving_e(smem_u32(&acc_empty[ab]), ((ti >> 1) & 1) ^ 1);
                 tc_fence_after();
+                if (!ok) break;
                 int kc0, kc1;
                 chunks_of(ti, kc0, kc1);
                 for (int kc = kc0; kc < kc1 && ok; kc += C::SUB, ++it) {
@@ -264,6 +265,7 @@ __global__ void __launch_bounds__(192, 1)
                     const uint32_t s = it % C::NST, ph = (it / C::NST) & 1;
                     ok = wait_serving_e(smem_u32(&full[s]), ph);
                     tc_fence_after();
+                    if (!ok) break;   // a wait gave up: issue nothing more
                     for (int j = 0; j < nsub; ++j) {
                         const uint32_t faddr = smem_u32(smem + C::OFF_STAGE + (s * C::SUB + j) * C::STAGE_BYTES);
                         const uint32_t waddr = faddr + C::F_BYTES;

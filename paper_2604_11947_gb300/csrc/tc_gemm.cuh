@@ -1,0 +1,403 @@
+// tc_gemm.cuh -- a persistent tcgen05 GEMM with the boundary's epilogues fused in, for the
+// widths the fused boundary kernels do not take (m = r = 512, the r = 128 backward, m != r):
+// there the two linear layers of Sec. 3.2's encoder and decoder, and their gradients, become a
+// chain of products C = A . B (bf16 operands, fp32 accumulation in TMEM), each with the
+// element-wise step that follows it in the chain (phi, phi', the identity-path merge of Eq. Pid,
+// the residual-gradient update) applied to the accumulator before it leaves the chip.
+//
+//   C[M x N] = sum over k of A[m][k] . B[k][n]
+//   A: K-major (stored M x K row-major) or MN-major (stored K x M row-major, i.e. A^T in memory)
+//   B: K-major (stored N x K row-major) or MN-major (stored K x N row-major)
+//
+// Work units are (128-row block, BN-column block, K split); unit u runs on CTA u mod grid
+// (n fastest, then m, then the split: CTAs running at the same time share their A block and,
+// across a wave, their B rows in L2). Per CTA:
+//   producer warp  : TMA loads of 64-deep K slices of A (128 x 64) and B (BN x 64), 128-byte
+//                    swizzle, into a ring of NST stages
+//   MMA warp       : four 128 x BN x 16 tcgen05.mma per stage into one of two TMEM accumulators
+//                    (double-buffered: the next unit's products overlap this unit's epilogue)
+//   With ALO the A operand is a bf16 pair hi + lo (hi = a value rounded to bf16, lo = the
+//   rounded remainder, two matrices of the same shape): each stage holds both A tiles and the
+//   MMA warp issues hi . B and lo . B into the same accumulator, so the product sees A to about
+//   16 significant bits (used where the result crosses the boundary: B and dB).
+//   epilogue warps : eight warps, two per TMEM lane quarter splitting the columns: TMEM ->
+//                    registers (one output row per thread, 32 columns at a time) -> the
+//                    epilogue's element-wise step -> global memory
+// Out-of-range rows, columns and K are read as zeros by TMA and never written, so any M, N, K
+// with 16-byte row pitches work. Each output element is summed by one CTA in K order (a split-K
+// launch writes per-split fp32 slots that a second kernel adds in slot order), so results are
+// bitwise reproducible.
+#pragma once
+
+#include "common.cuh"
+#include "tc_common.cuh"
+
+namespace resbm {
+namespace tc {
+
+// The element-wise step after the product (acc = the fp32 accumulator of one output element at
+// row `row`, column `col`; phi and phi' as in common.cuh; every bf16 result rounded once to
+// nearest even).
+// `lo` (if set) receives the rounded remainder of the bf16 activation result named below, so that
+// a later product can use it as a hi + lo pair.
+enum GemmEpMode : int {
+    GEP_F32 = 0,   // out f32 = acc (with split-K: slot ks at out + ks * split_stride)
+    GEP_BF16,      // out bf16 = acc
+    GEP_P_A,       // out f32 = acc (if out), out2 bf16 = phi(acc) (lo: its remainder)  (P, A)
+    GEP_ADD_AUX,   // out bf16 = acc + aux[row][col] for col < aux_cols, acc elsewhere  (B, Y, dB)
+    GEP_ACT,       // out bf16 = phi(acc), out2 f32 = acc (if out2)                     (G, Q)
+    GEP_DACT,      // out bf16 = acc * phi'(aux f32) (lo: its remainder), out2 bf16 = phi(aux) if
+                   // out2                                                              (dQ; dP, A)
+    GEP_DF,        // out bf16 = acc; rmw[row][col] += aux[row][col] for col < aux_cols (dF; dX += dB)
+};
+
+struct GemmEp {
+    int mode, act;
+    void *out;           // ldo elements per row
+    int64_t ldo;
+    void *out2;          // ldo2 elements per row
+    int64_t ldo2;
+    const void *aux;     // bf16 (ADD_AUX, DF) or f32 (DACT); lda elements per row
+    int64_t lda, aux_cols;
+    __nv_bfloat16 *rmw;  // DF: ldr elements per row
+    int64_t ldr;
+    int64_t split_stride;
+    __nv_bfloat16 *lo;   // P_A, DACT: the remainder of the bf16 activation result (same pitch)
+};
+
+struct GemmShape {
+    int64_t M, N, K;
+    int64_t kc;          // K per split, a multiple of 64
+    int nm, nn, splits;
+    int64_t units;       // nm * nn * splits
+};
+
+template <int BN_, bool ALO_ = false> struct GemmCfg {
+    static constexpr int BN = BN_;
+    static constexpr uint32_t A_TILE = 128 * 64 * 2;        // 128 rows x 64 K, bf16
+    static constexpr uint32_t A_STAGE = A_TILE * (ALO_ ? 2 : 1);   // hi (+ lo)
+    static constexpr uint32_t B_STAGE = BN_ * 64 * 2;       // BN rows x 64 K, bf16
+    static constexpr uint32_t STAGE = A_STAGE + B_STAGE;
+    static constexpr int NST = (200 * 1024) / STAGE;        // 4 stages at BN = 256, 6 at 128 (3, 4 with lo)
+    static constexpr uint32_t SMEM_BYTES = NST * STAGE + 1024;
+    static_assert(SMEM_BYTES <= 232448 - 512, "shared memory budget");
+    static constexpr uint32_t TMEM_COLS = 2 * BN_;          // two accumulators
+    static_assert(TMEM_COLS <= 512, "TMEM budget");
+    static constexpr int EPI = 256;                         // epilogue threads (8 warps)
+    static constexpr int THREADS = 64 + EPI;
+};
+
+__device__ __forceinline__ void gemm_unit(const GemmShape &g, int64_t u, int &mb, int &nb, int &ks)
+{
+    nb = (int)(u % g.nn);
+    const int64_t rest = u / g.nn;
+    mb = (int)(rest % g.nm);
+    ks = (int)(rest / g.nm);
+}
+
+// ---- the epilogue's element-wise steps on 32 consecutive columns of one row ----------------
+__device__ __forceinline__ void st_bf16x32(__nv_bfloat16 *dst, const float (&v)[32], int nv)
+{
+    if (nv == 32) {
+        uint4 *o = reinterpret_cast<uint4 *>(dst);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            uint32_t pk[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                __nv_bfloat162 h = __floats2bfloat162_rn(v[8 * q + 2 * e], v[8 * q + 2 * e + 1]);
+                pk[e] = *reinterpret_cast<uint32_t *>(&h);
+            }
+            o[q] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+        }
+    } else {   // every index a constant (no dynamic indexing of the register array)
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+            if (j < nv) dst[j] = __float2bfloat16_rn(v[j]);
+    }
+}
+
+// hi = v rounded to bf16 at dst, lo = (v - hi) rounded to bf16 at dst_lo (if set)
+__device__ __forceinline__ void st_bf16x32_split(__nv_bfloat16 *dst, __nv_bfloat16 *dst_lo, float (&v)[32], int nv)
+{
+    st_bf16x32(dst, v, nv);
+    if (dst_lo) {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] -= __bfloat162float(__float2bfloat16_rn(v[j]));
+        st_bf16x32(dst_lo, v, nv);
+    }
+}
+
+__device__ __forceinline__ void st_f32x32(float *dst, const float (&v)[32], int nv)
+{
+    if (nv == 32) {
+        float4 *o = reinterpret_cast<float4 *>(dst);
+#pragma unroll
+        for (int q = 0; q < 8; ++q) o[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+    } else {
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+            if (j < nv) dst[j] = v[j];
+    }
+}
+
+__device__ __forceinline__ void ld_bf16x32(const __nv_bfloat16 *src, float (&x)[32], int nv)
+{
+    if (nv == 32) {
+        load_bf16_row<32>(src, x);
+    } else {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) x[j] = j < nv ? __bfloat162float(src[j]) : 0.0f;
+    }
+}
+
+__device__ __forceinline__ void ld_f32x32(const float *src, float (&x)[32], int nv)
+{
+    if (nv == 32) {
+        const float4 *s = reinterpret_cast<const float4 *>(src);
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+            const float4 t = s[q];
+            x[4 * q] = t.x; x[4 * q + 1] = t.y; x[4 * q + 2] = t.z; x[4 * q + 3] = t.w;
+        }
+    } else {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) x[j] = j < nv ? src[j] : 0.0f;
+    }
+}
+
+// v: the accumulator's columns [col, col + nv) of row `row` (nv <= 32; the vector forms need
+// nv == 32 and 16-byte aligned rows, which the host guarantees for nv == 32)
+__device__ __forceinline__ void gemm_epilogue(const GemmEp &ep, int64_t row, int64_t col, float (&v)[32], int nv,
+                                              int ks)
+{
+    switch (ep.mode) {
+    case GEP_F32:
+        st_f32x32(static_cast<float *>(ep.out) + ks * ep.split_stride + row * ep.ldo + col, v, nv);
+        break;
+    case GEP_BF16:
+        st_bf16x32(static_cast<__nv_bfloat16 *>(ep.out) + row * ep.ldo + col, v, nv);
+        break;
+    case GEP_P_A:
+        if (ep.out) st_f32x32(static_cast<float *>(ep.out) + row * ep.ldo + col, v, nv);
+        act_fast_row<32>(ep.act, v);
+        st_bf16x32_split(static_cast<__nv_bfloat16 *>(ep.out2) + row * ep.ldo2 + col,
+                         ep.lo ? ep.lo + row * ep.ldo2 + col : nullptr, v, nv);
+        break;
+    case GEP_ADD_AUX:
+        if (col < ep.aux_cols) {
+            const int na = ep.aux_cols - col < nv ? (int)(ep.aux_cols - col) : nv;
+            float x[32];
+            ld_bf16x32(static_cast<const __nv_bfloat16 *>(ep.aux) + row * ep.lda + col, x, na);
+#pragma unroll
+            for (int j = 0; j < 32; ++j) v[j] = j < na ? v[j] + x[j] : v[j];
+        }
+        st_bf16x32(static_cast<__nv_bfloat16 *>(ep.out) + row * ep.ldo + col, v, nv);
+        break;
+    case GEP_ACT:
+        if (ep.out2) st_f32x32(static_cast<float *>(ep.out2) + row * ep.ldo2 + col, v, nv);
+        act_fast_row<32>(ep.act, v);
+        st_bf16x32(static_cast<__nv_bfloat16 *>(ep.out) + row * ep.ldo + col, v, nv);
+        break;
+    case GEP_DACT: {
+        float x[32], dx[32];
+        ld_f32x32(static_cast<const float *>(ep.aux) + row * ep.lda + col, x, nv);
+        dact_fast_row<32>(ep.act, x, dx);
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] *= dx[j];
+        st_bf16x32_split(static_cast<__nv_bfloat16 *>(ep.out) + row * ep.ldo + col,
+                         ep.lo ? ep.lo + row * ep.ldo + col : nullptr, v, nv);
+        if (ep.out2) {
+            act_fast_row<32>(ep.act, x);
+            st_bf16x32(static_cast<__nv_bfloat16 *>(ep.out2) + row * ep.ldo2 + col, x, nv);
+        }
+        break;
+    }
+    case GEP_DF:
+        st_bf16x32(static_cast<__nv_bfloat16 *>(ep.out) + row * ep.ldo + col, v, nv);
+        if (ep.rmw && col < ep.aux_cols) {
+            const int na = ep.aux_cols - col < nv ? (int)(ep.aux_cols - col) : nv;
+            float x[32], y[32];
+            __nv_bfloat16 *r = ep.rmw + row * ep.ldr + col;
+            ld_bf16x32(r, y, na);
+            ld_bf16x32(static_cast<const __nv_bfloat16 *>(ep.aux) + row * ep.lda + col, x, na);
+#pragma unroll
+            for (int j = 0; j < 32; ++j) y[j] += x[j];
+            st_bf16x32(r, y, na);
+        }
+        break;
+    }
+}
+
+// tma_lo: the lo matrix of A (same shape and layout as A; read only with ALO)
+template <int BN, bool AMN, bool BMN, bool ALO>
+__global__ void __launch_bounds__(320, 1)
+    k_gemm(const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tma_lo,
+           const __grid_constant__ CUtensorMap tmb, const GemmShape g, const GemmEp ep)
+{
+    using C = GemmCfg<BN, ALO>;
+    static_assert(!(ALO && AMN), "hi + lo pairs only for K-major A");
+    griddep_wait();               // the previous kernel of the stream has completed
+    griddep_launch_dependents();  // the next one may be scheduled on SMs as they free up
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    __shared__ uint64_t full[C::NST], empty[C::NST], acc_full[2], acc_empty[2], done_bar;
+    __shared__ uint32_t tmem_base_sh;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    auto k_steps = [&](int ks, int64_t &k0) -> int {
+        k0 = (int64_t)ks * g.kc;
+        int64_t k1 = k0 + g.kc;
+        if (k1 > g.K) k1 = g.K;
+        return (int)((k1 - k0 + 63) / 64);
+    };
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < C::NST; ++s) {
+            mbar_init(smem_u32(&full[s]), 1);
+            mbar_init(smem_u32(&empty[s]), 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(smem_u32(&acc_full[i]), 1);
+            mbar_init(smem_u32(&acc_empty[i]), C::EPI);
+        }
+        mbar_init(smem_u32(&done_bar), 1);
+        fence_mbar_init();
+    }
+    if (warp == 1) tmem_alloc(smem_u32(&tmem_base_sh), C::TMEM_COLS);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_base_sh;
+
+    if (warp == 0) {
+        // ---------------- producer ----------------
+        if (elect_one()) {
+            tma_prefetch_desc(&tma);
+            if (ALO) tma_prefetch_desc(&tma_lo);
+            tma_prefetch_desc(&tmb);
+            uint32_t it = 0;
+            bool ok = true;
+            for (int64_t u = blockIdx.x; u < g.units && ok; u += gridDim.x) {
+                int mb, nb, ks;
+                gemm_unit(g, u, mb, nb, ks);
+                int64_t k0;
+                const int nk = k_steps(ks, k0);
+                for (int kb = 0; kb < nk; ++kb, ++it) {
+                    const uint32_t s = it % C::NST, ph = (it / C::NST) & 1;
+                    if (!mbar_wait(smem_u32(&empty[s]), ph ^ 1)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t bar = smem_u32(&full[s]);
+                    mbar_expect_tx(bar, C::STAGE);
+                    const uint32_t adst = smem_u32(smem + s * C::STAGE), bdst = adst + C::A_STAGE;
+                    const int32_t kx = (int32_t)(k0 + 64 * kb);
+                    if (!AMN) {
+                        tma_load_2d(adst, &tma, kx, mb * 128, bar);
+                        if (ALO) tma_load_2d(adst + C::A_TILE, &tma_lo, kx, mb * 128, bar);
+                    } else {
+                        tma_load_2d(adst, &tma, mb * 128, kx, bar);
+                        tma_load_2d(adst + 8192, &tma, mb * 128 + 64, kx, bar);
+                    }
+                    if (!BMN) {
+                        tma_load_2d(bdst, &tmb, kx, nb * BN, bar);
+                    } else {
+#pragma unroll
+                        for (int j = 0; j < BN / 64; ++j) tma_load_2d(bdst + j * 8192, &tmb, nb * BN + 64 * j, kx, bar);
+                    }
+                }
+            }
+            // drain the loads still in flight before the CTA may exit
+            const uint32_t n = it < (uint32_t)C::NST ? it : (uint32_t)C::NST;
+            for (uint32_t k = 0; k < n; ++k) {
+                const uint32_t j = it - 1 - k;
+                mbar_wait(smem_u32(&full[j % C::NST]), (j / C::NST) & 1);
+            }
+        }
+    } else if (warp == 1) {
+        // ---------------- MMA issuer ----------------
+        if (elect_one()) {
+            constexpr uint32_t idesc = idesc_bf16(128, BN, AMN, BMN);
+            // stage-0 descriptors, advanced by (byte offset >> 4) in the start-address field.
+            // K-major: rows of 128 bytes (64 K), 8-row groups 1024 bytes apart, a K step of 16 =
+            // 32 bytes. MN-major: 64-wide blocks of 64 K rows (8 KB) 8192 bytes apart along M/N,
+            // 8-row groups along K 1024 bytes apart, a K step of 16 = 16 rows = 2048 bytes.
+            const uint32_t a0 = smem_u32(smem), b0 = a0 + C::A_STAGE;
+            const uint64_t ad0 = AMN ? smem_desc(a0, 8192, 1024, kSwz128) : smem_desc(a0, 16, 1024, kSwz128);
+            const uint64_t bd0 = BMN ? smem_desc(b0, 8192, 1024, kSwz128) : smem_desc(b0, 16, 1024, kSwz128);
+            constexpr uint64_t AK = AMN ? (2048 >> 4) : (32 >> 4);
+            constexpr uint64_t BK = BMN ? (2048 >> 4) : (32 >> 4);
+            uint32_t it = 0, ti = 0;
+            bool ok = true;
+            for (int64_t u = blockIdx.x; u < g.units && ok; u += gridDim.x, ++ti) {
+                int mb, nb, ks;
+                gemm_unit(g, u, mb, nb, ks);
+                int64_t k0;
+                const int nk = k_steps(ks, k0);
+                const uint32_t ab = ti & 1;
+                ok = mbar_wait(smem_u32(&acc_empty[ab]), ((ti >> 1) & 1) ^ 1);
+                tc_fence_after();
+                if (!ok) break;
+                const uint32_t d_tmem = tmem + ab * BN;
+                for (int kb = 0; kb < nk; ++kb, ++it) {
+                    const uint32_t s = it % C::NST, ph = (it / C::NST) & 1;
+                    ok = mbar_wait(smem_u32(&full[s]), ph);
+                    tc_fence_after();
+                    if (!ok) break;
+                    const uint64_t so = (uint64_t)((s * C::STAGE) >> 4);
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk) {
+                        mma_bf16(d_tmem, ad0 + so + kk * AK, bd0 + so + kk * BK, idesc, kb > 0 || kk > 0);
+                        if (ALO) mma_bf16(d_tmem, ad0 + so + (C::A_TILE >> 4) + kk * AK, bd0 + so + kk * BK, idesc, true);
+                    }
+                    mma_commit(smem_u32(&empty[s]));   // the stage is free once these MMAs are done
+                }
+                if (!ok) break;
+                mma_commit(smem_u32(&acc_full[ab]));
+            }
+            mma_commit(smem_u32(&done_bar));
+            mbar_wait(smem_u32(&done_bar), 0);
+        }
+    } else {
+        // ---------------- epilogue warps ----------------
+        const int q = warp & 3;                 // TMEM lane quarter this warp may access
+        const int half = (warp - 2) >> 2;       // which half of the BN columns
+        const int rin = q * 32 + lane;          // row within the 128-row block
+        const uint32_t lane_base = (uint32_t)(q * 32) << 16;
+        uint32_t ti = 0;
+        bool ok = true;
+        for (int64_t u = blockIdx.x; u < g.units && ok; u += gridDim.x, ++ti) {
+            int mb, nb, ks;
+            gemm_unit(g, u, mb, nb, ks);
+            const uint32_t ab = ti & 1;
+            ok = mbar_wait(smem_u32(&acc_full[ab]), (ti >> 1) & 1);
+            tc_fence_after();
+            if (!ok) break;
+            const int64_t row = (int64_t)mb * 128 + rin;
+#pragma unroll 1
+            for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 32) {
+                float v[32];
+                tmem_ld32(tmem + lane_base + ab * BN + c, v);   // warp-collective: every lane
+                tmem_ld_wait();
+                tmem_regs_ready<32>(v);
+                const int64_t col = (int64_t)nb * BN + c;
+                if (col < g.N && row < g.M) {
+                    const int nv = g.N - col < 32 ? (int)(g.N - col) : 32;
+                    gemm_epilogue(ep, row, col, v, nv, ks);
+                }
+            }
+            tc_fence_before();
+            mbar_arrive(smem_u32(&acc_empty[ab]));   // this accumulator may be overwritten
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, C::TMEM_COLS);
+    }
+}
+
+}  // namespace tc
+}  // namespace resbm

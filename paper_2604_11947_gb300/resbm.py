@@ -21,6 +21,7 @@ RESBM_ACT_SILU, RESBM_ACT_GELU_TANH, RESBM_ACT_IDENTITY = 0, 1, 2
  RESBM_OP_BOUNDARY_STEP, RESBM_OP_BOUNDARY_STEP_HOST) = range(6)
 RESBM_FLAG_GENERIC = 1
 RESBM_FLAG_LINEAR = 2
+RESBM_FLAG_GEMM = 4
 RESBM_STATIC_SCRATCH_BYTES = 32 << 20
 
 ACTS = {"silu": RESBM_ACT_SILU, "gelu_tanh": RESBM_ACT_GELU_TANH, "identity": RESBM_ACT_IDENTITY}

@@ -4,7 +4,7 @@ import pytest
 import torch
 
 from gpu_helpers import (INPUTS, assert_step_is_its_stages, check_output, gpu_stages, gpu_step,
-                         host_inputs, oracle_step, sample_tokens, to_dev, to_host)
+                         host_inputs, oracle_step, to_dev, to_host)
 from metrics import TOL, check
 from paper_2604_11947_gb300 import resbm, synth
 
@@ -12,7 +12,10 @@ import oracle
 
 pytestmark = pytest.mark.gpu
 
-PATHS = {"default": 0, "generic": resbm.RESBM_FLAG_GENERIC}
+# default: the fused tensor-core kernels where they take the shape, else the tensor-core GEMM
+# chain, else the portable kernels; gemm: the GEMM chain wherever it takes the shape (bf16, d, r, m
+# multiples of 8); generic: the portable CUDA-core kernels
+PATHS = {"default": 0, "gemm": resbm.RESBM_FLAG_GEMM, "generic": resbm.RESBM_FLAG_GENERIC}
 OUTS = ("B", "Y", "dB", "dF", "dX", "dWe1", "dWe2", "dWd1", "dWd2")
 
 SMALL = {
@@ -41,6 +44,12 @@ SMALL = {
     # on the portable kernels at these widths
     "bf16_d64": synth.BoundaryConfig("bf16_d64", T=1000, d=64, r=32, m=32),
     "bf16_d192": synth.BoundaryConfig("bf16_d192", T=300, d=192, r=32, m=32),
+    # widths the fused kernels do not take run as the tensor-core GEMM chain by default: m = r =
+    # 512 (two 256-column output blocks, split-K weight gradients at this T), and odd multiples
+    # of 8 (d = 776 = 3 x 256 + 8 leaves an 8-column output block and a 8-deep K tail; r = 24 and
+    # m = 40 a partial 32-column epilogue chunk)
+    "bf16_r512": synth.BoundaryConfig("bf16_r512", T=700, d=1024, r=512, m=512),
+    "bf16_r24_m40": synth.BoundaryConfig("bf16_r24_m40", T=999, d=776, r=24, m=40),
 }
 
 # Backward grids under each forced cluster size (RESBM_CLUSTER), one CTA per 128-token
@@ -127,49 +136,32 @@ def test_single_bf16_config_full():
     _compare_all(cfg, got, want, dev)
 
 
-def _sampled_full_size(cfg, n_tokens=96, flags=0):
-    """Full-size launch (the benchmarked shapes) checked on a token sample S:
-    run 1 with the full dY: per-token outputs of S against the oracle on S;
-    run 2 with dY zero outside S: the weight gradients (sums over tokens) are exactly the
-    oracle's over S, and the backward per-token outputs vanish outside S."""
-    S = sample_tokens(cfg.T, n_tokens)
-    dev = {}
-    for k in INPUTS:
-        dev[k] = to_dev(synth.tensor(cfg, k), cfg)
-    hS = {k: synth.rows_at(cfg, k, S) for k in ("X", "F", "dY")}
-    for k in ("We1", "We2", "Wd1", "Wd2"):
-        hS[k] = to_host(dev[k])
-    want = oracle_step(cfg, hS)
-    Sg = torch.from_numpy(S).cuda()
-    got = gpu_step(cfg, dev, flags=flags)
-    for k in ("B", "Y", "dB", "dF", "dX"):
-        check_output(k, got[k][Sg], want[k], cfg)
-    del got
-    dY_masked = torch.zeros_like(dev["dY"])
-    dY_masked[Sg] = dev["dY"][Sg]
-    dev["dY"] = dY_masked
-    got = gpu_step(cfg, dev, flags=flags)
-    for k in ("dWe1", "dWe2", "dWd1", "dWd2"):
-        check(k, to_host(got[k]), want[k], cfg.dtype)
-    for k in ("dB", "dF", "dX"):
-        check_output(k, got[k][Sg], want[k], cfg)
-    outside = torch.ones(cfg.T, dtype=torch.bool, device="cuda")
-    outside[Sg] = False
-    for k in ("dB", "dF", "dX"):
-        assert not torch.any(got[k][outside]), k
+def _full_size_every_element(cfg):
+    """Full-size launch (the benchmarked shapes, the grids and cluster sizes the bench runs)
+    against one oracle step over all T tokens: every element of B, Y, dB, dF, dX[:, :r] and of
+    the four weight gradients, each compared with the stage run on the oracle's transferred
+    tensor as in the small cases, and the step against its own stages bit for bit."""
+    h = host_inputs(cfg)
+    dev = {k: to_dev(v, cfg) for k, v in h.items()}
+    got = gpu_step(cfg, dev)
+    want = oracle_step(cfg, h)
+    del h
+    errs = _compare_all(cfg, got, want, dev)
+    assert resbm.resbm_device_error() == 0
+    return errs
 
 
 @pytest.mark.slow
 def test_large_bf16_full_size():
     """T = 65536, d = 4096, r = 32 (batch 32 x seq 2048, 128x): the headline workload."""
-    _sampled_full_size(synth.CONFIGS["large_bf16"])
+    _full_size_every_element(synth.CONFIGS["large_bf16"])
 
 
 @pytest.mark.slow
 @pytest.mark.parametrize("name", ["sweep_r512", "sweep_r128", "sweep_r64", "sweep_r32"])
 def test_sweep_full_size(name):
     """d = 8192, T = 32768, r in {512, 128, 64, 32} (16x .. 256x compression)."""
-    _sampled_full_size(synth.CONFIGS[name], n_tokens=48)
+    _full_size_every_element(synth.CONFIGS[name])
 
 
 # ---------------------------------------------------------------------------------------------
