@@ -399,6 +399,29 @@ def extra_workload(name, cfg, flags, resbm, torch, steps, warmup, peaks, reuse=N
     return res, dev
 
 
+def pipeline_workload(torch, steps=3, warmup=2):
+    """The simulated 4-stage pipeline: one training step (forward + backward) of the 24-layer
+    transformer with three ResBM boundaries; the boundary kernels' share of the step time."""
+    from paper_2604_11947_gb300 import pipeline
+    cfg = pipeline.PIPELINE
+    model = pipeline.PipelineModel(cfg)
+    tokens = pipeline.synthetic_tokens(cfg)
+    step_ms, bnd_ms, loss = pipeline.time_steps(model, tokens, steps, warmup)
+    del model
+    return {"workload": "%d-layer pre-norm decoder (d=%d, %d heads, SwiGLU %d, vocab %d, bf16) in %d "
+                        "stages with a ResBM boundary (r=%d, m=%d, merge=1) between consecutive stages; "
+                        "batch %d x seq %d uniform random token ids; one training step (forward + "
+                        "backward, no optimizer update)"
+                        % (cfg.layers, cfg.d, cfg.heads, cfg.ffn, cfg.vocab, cfg.stages, cfg.r, cfg.m,
+                           cfg.batch, cfg.seq),
+            "steps": steps, "warmup": warmup, "ms_per_step": step_ms,
+            "value": cfg.tokens / (step_ms / 1e3), "unit": "tokens/s",
+            "boundary_ms_per_step": bnd_ms, "boundary_share": bnd_ms / step_ms,
+            "boundaries": cfg.stages - 1, "loss": loss,
+            "timing": "CUDA events around the K steps and around every boundary C-ABI call "
+                      "(12 per step: encode/decode forward and backward of 3 boundaries)"}
+
+
 def main():
     args = parse()
     cfg = synth.CONFIGS[args.config]
@@ -492,6 +515,8 @@ def main():
             extra[name], reuse = extra_workload(name, synth.CONFIGS[name], flags, resbm, torch,
                                                 k_extra, w_extra, peaks, reuse)
         del reuse
+        torch.cuda.empty_cache()
+        extra["pipeline"] = pipeline_workload(torch)
         torch.cuda.empty_cache()
 
     line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,

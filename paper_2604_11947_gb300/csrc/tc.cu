@@ -459,18 +459,19 @@ cudaError_t launch_gemm_t(const CUtensorMap &ma, const CUtensorMap &malo, const 
 }
 
 // splits: 1 for every product whose epilogue is not a plain fp32 store; with splits > 1 the
-// epilogue must be GEP_F32 into `splits` slots of M x N (ep.split_stride apart). A_lo (K-major A
-// only): the lo half of A as a bf16 hi + lo pair (same shape as A), or null.
+// epilogue must be GEP_F32 into `splits` slots of M x N (ep.split_stride apart). A_lo: the lo
+// half of A as a bf16 hi + lo pair (same shape and layout as A), or null.
 cudaError_t gemm(const Ctx &c, int64_t M, int64_t N, int64_t K, const void *A, bool a_mn, const void *B, bool b_mn,
                  const tc::GemmEp &ep, int splits, const void *A_lo = nullptr)
 {
     if (M <= 0 || N <= 0 || K <= 0) return cudaSuccess;
-    if (A_lo && a_mn) return cudaErrorNotSupported;
     const int bn = gemm_bn(N);
     CUtensorMap ma, malo, mbm;
     const bool okA = a_mn ? make_map(&ma, A, M, K, M * 2, 64, 64, CU_TENSOR_MAP_SWIZZLE_128B)
                           : make_map(&ma, A, K, M, K * 2, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B);
-    const bool okL = A_lo ? make_map(&malo, A_lo, K, M, K * 2, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B) : true;
+    const bool okL = !A_lo ? true
+                     : a_mn ? make_map(&malo, A_lo, M, K, M * 2, 64, 64, CU_TENSOR_MAP_SWIZZLE_128B)
+                            : make_map(&malo, A_lo, K, M, K * 2, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B);
     const bool okB = b_mn ? make_map(&mbm, B, N, K, N * 2, 64, 64, CU_TENSOR_MAP_SWIZZLE_128B)
                           : make_map(&mbm, B, K, N, K * 2, 64, (uint32_t)bn, CU_TENSOR_MAP_SWIZZLE_128B);
     if (!okA || !okL || !okB) return cudaErrorInvalidValue;
@@ -491,13 +492,15 @@ cudaError_t gemm(const Ctx &c, int64_t M, int64_t N, int64_t K, const void *A, b
                                      : launch_gemm_t<256, false, true, false>(ma, malo, mbm, g, ep, c);
         if (!a_mn && !b_mn) return lo ? launch_gemm_t<256, false, false, true>(ma, malo, mbm, g, ep, c)
                                       : launch_gemm_t<256, false, false, false>(ma, malo, mbm, g, ep, c);
-        if (a_mn && b_mn) return launch_gemm_t<256, true, true, false>(ma, malo, mbm, g, ep, c);
+        if (a_mn && b_mn) return lo ? launch_gemm_t<256, true, true, true>(ma, malo, mbm, g, ep, c)
+                                    : launch_gemm_t<256, true, true, false>(ma, malo, mbm, g, ep, c);
     } else {
         if (!a_mn && b_mn) return lo ? launch_gemm_t<128, false, true, true>(ma, malo, mbm, g, ep, c)
                                      : launch_gemm_t<128, false, true, false>(ma, malo, mbm, g, ep, c);
         if (!a_mn && !b_mn) return lo ? launch_gemm_t<128, false, false, true>(ma, malo, mbm, g, ep, c)
                                       : launch_gemm_t<128, false, false, false>(ma, malo, mbm, g, ep, c);
-        if (a_mn && b_mn) return launch_gemm_t<128, true, true, false>(ma, malo, mbm, g, ep, c);
+        if (a_mn && b_mn) return lo ? launch_gemm_t<128, true, true, true>(ma, malo, mbm, g, ep, c)
+                                    : launch_gemm_t<128, true, true, false>(ma, malo, mbm, g, ep, c);
     }
     return cudaErrorNotSupported;
 }
@@ -515,15 +518,16 @@ tc::GemmEp ep_of(int mode, int act, void *out, int64_t ldo)
 // A weight gradient W (M x N fp32) = A^T . B over K tokens (both operands MN-major), split over
 // the tokens when it has few output tiles: the splits' fp32 slots go to `slots` and the job to
 // sum them (in slot order) is returned in `job` (job->blocks = 0: nothing to reduce).
+// A_lo: A as a bf16 hi + lo pair (or null).
 cudaError_t wgrad(const Ctx &c, int64_t M, int64_t N, int64_t K, const void *A, const void *B, float *W, float *slots,
-                  tc::ReduceJob *job)
+                  tc::ReduceJob *job, const void *A_lo = nullptr)
 {
     const int s = gemm_splits(M, N, K, c.sm_count);
     *job = tc::ReduceJob{nullptr, 0, 0, 0, nullptr, 0, 0, 0};
-    if (s <= 1) return gemm(c, M, N, K, A, true, B, true, ep_of(tc::GEP_F32, 0, W, N), 1);
+    if (s <= 1) return gemm(c, M, N, K, A, true, B, true, ep_of(tc::GEP_F32, 0, W, N), 1, A_lo);
     tc::GemmEp e = ep_of(tc::GEP_F32, 0, slots, N);
     e.split_stride = M * N;
-    cudaError_t err = gemm(c, M, N, K, A, true, B, true, e, s);
+    cudaError_t err = gemm(c, M, N, K, A, true, B, true, e, s, A_lo);
     if (err != cudaSuccess) return err;
     // the number of splits the launch took (gemm rounds K per split to 64)
     const int64_t kc = ((K + s - 1) / s + 63) / 64 * 64;
@@ -549,7 +553,7 @@ cudaError_t reduce_jobs(const tc::ReduceJob &a, const tc::ReduceJob &b, const Ct
 struct GemmWs {
     float *P = nullptr, *Q = nullptr;
     __nv_bfloat16 *A = nullptr, *G = nullptr, *dQ = nullptr, *dP = nullptr;
-    __nv_bfloat16 *A_lo = nullptr, *dQ_lo = nullptr, *dP_lo = nullptr;   // remainders of hi + lo pairs
+    __nv_bfloat16 *A_lo = nullptr, *G_lo = nullptr, *dQ_lo = nullptr, *dP_lo = nullptr;   // remainders of hi + lo pairs
     float *slots1 = nullptr, *slots2 = nullptr;
     size_t bytes = 0;
 };
@@ -577,6 +581,7 @@ GemmWs gemm_ws(const resbm_desc &d, int op, int sms, void *ws, bool have_P)
     } else if (op == RESBM_OP_DECODE_BWD) {
         w.Q = cv.take<float>(T * m);
         w.G = cv.take<__nv_bfloat16>(T * m);
+        w.G_lo = cv.take<__nv_bfloat16>(T * m);
         w.dQ = cv.take<__nv_bfloat16>(T * m);
         w.dQ_lo = cv.take<__nv_bfloat16>(T * m);
         w.slots1 = cv.take<float>(slot_floats(m, D, T, sms));   // dWd2
@@ -720,10 +725,11 @@ cudaError_t gemm_decode_bwd(const resbm_desc &d, const void *dY, const void *B, 
     if (!al16(dY) || !al16(B) || !al16(Wd1) || !al16(Wd2) || !al16(dB) || !al16(dWd1) || !al16(dWd2) || !al16(ws))
         return cudaErrorNotSupported;
     const GemmWs w = gemm_ws(d, RESBM_OP_DECODE_BWD, c.sm_count, ws, true);
-    // Q = B . Wd1 (kept), G = phi(Q)
+    // Q = B . Wd1 (kept), G = phi(Q) as a hi + lo pair
     tc::GemmEp e1 = ep_of(tc::GEP_ACT, d.act, w.G, d.m);
     e1.out2 = w.Q;
     e1.ldo2 = d.m;
+    e1.lo = w.G_lo;
     cudaError_t e = gemm(c, d.T, d.m, d.r, B, false, Wd1, true, e1, 1);
     // dQ = (dY . Wd2^T) * phi'(Q)
     tc::GemmEp e2 = ep_of(tc::GEP_DACT, d.act, w.dQ, d.m);
@@ -737,9 +743,9 @@ cudaError_t gemm_decode_bwd(const resbm_desc &d, const void *dY, const void *B, 
     e3.lda = d.d;
     e3.aux_cols = d.merge_identity ? d.r : 0;
     if (e == cudaSuccess) e = gemm(c, d.T, d.r, d.m, w.dQ, false, Wd1, false, e3, 1, w.dQ_lo);
-    // dWd2 = G^T . dY, dWd1 = B^T . dQ (sums over the tokens)
+    // dWd2 = (G_hi + G_lo)^T . dY, dWd1 = B^T . dQ (sums over the tokens)
     tc::ReduceJob j2, j1;
-    if (e == cudaSuccess) e = wgrad(c, d.m, d.d, d.T, w.G, dY, dWd2, w.slots1, &j2);
+    if (e == cudaSuccess) e = wgrad(c, d.m, d.d, d.T, w.G, dY, dWd2, w.slots1, &j2, w.G_lo);
     if (e == cudaSuccess) e = wgrad(c, d.r, d.m, d.T, B, w.dQ, dWd1, w.slots2, &j1);
     if (e == cudaSuccess) e = reduce_jobs(j1, j2, c);
     return e;

@@ -8,12 +8,15 @@
 // its tiles split evenly). Every product runs on tcgen05; the CUDA cores only apply phi and phi'
 // and convert. For each group:
 //   phase 0: the group's B tiles (TMA) -> Q_tile = B . Wd1 in TMEM (kept for phase 2) -> the
-//            epilogue writes G = phi(Q) as bf16 rows [token][m] to shared memory.
+//            epilogue writes G = phi(Q) as a bf16 pair hi + lo, rows [token][m], to shared
+//            memory (hi in the G tiles, lo over the B tiles, which the Q products have read).
 //   phase 1: d in chunks of 128 columns; per chunk one Wd2 slice and, per tile, one dY tile
-//            (128 tokens x 128 columns) feeding two MMAs:
+//            (128 tokens x 128 columns) feeding the MMAs:
 //              dG_tile   (128 tokens x m, TMEM, kept over all chunks) += dY . Wd2_chunk^T
-//              dWd2T_chk (128 columns x m, TMEM, double-buffered)     += dY^T . G_tile
-//            (the same dY stage read K-major and MN-major; G read MN-major). The epilogue
+//              dWd2T_chk (128 columns x m, TMEM, double-buffered)     += dY^T . (G_hi + G_lo)
+//            (the same dY stage read K-major and MN-major; G read MN-major; dWd2 is a sum over
+//            all tokens whose terms cancel strongly for real gradients, so G enters it to about
+//            16 significant bits). The epilogue
 //            drains each finished dWd2T chunk into the cluster's fp32 partial slot (summed over
 //            the cluster's CTAs through distributed shared memory, tc_wgrad.cuh).
 //   phase 2: the epilogue writes dQ = dG * phi'(Q) as two bf16 tiles hi + lo (rows [token][m],
@@ -21,8 +24,9 @@
 //            products see dQ to about 16 significant bits: dB crosses the boundary and is
 //            rounded again there) -> dB_tile = dQ . Wd1^T (into the tile's dG columns) and
 //            dWd1 += B^T . dQ over the group's tokens (the B tile read MN-major as a 128-row
-//            operand whose rows >= r are never read back) -> the epilogue adds [merge]
-//            dY[:, :r] (a TMA tile) and stores dB as bf16; the group's dWd1 goes to its slot.
+//            operand whose rows >= r are never read back; the B tiles are loaded again for this
+//            phase, into a region idle in it) -> the epilogue adds [merge] dY[:, :r] (a TMA
+//            tile) and stores dB as bf16; the group's dWd1 goes to its slot.
 // A second kernel sums the partial slots in a fixed order (deterministic).
 // HBM traffic per token: read dY (2d), B (2r), dY[:, :r] again (2r, mostly L2), write dB (2r);
 // per cluster: d x m fp32 partials; per CTA and group: r x m.
@@ -64,9 +68,19 @@ template <int M_> struct DecBwdCfg {
     static constexpr uint32_t OFF_YR = OFF_Y + Y_STAGE;
     static constexpr uint32_t OFF_DQLO = OFF_Y + 2 * Y_STAGE;
     static_assert(NT * TILE <= Y_STAGE && NSY >= 3, "phase-2 scratch must fit in three ring slots");
+    // G_lo tiles (phase 1) over the B tiles; the B tiles of phase 2 in the fourth ring slot, or in
+    // the Wd2 slice ring (both idle in phase 2)
+    static constexpr uint32_t OFF_GLO = OFF_B;
+    static constexpr uint32_t OFF_B2 = NSY >= 4 ? OFF_Y + 3 * Y_STAGE : OFF_W;
+    static_assert(NSY >= 4 ? NT * TILE <= Y_STAGE : NT * TILE <= NW * W_STAGE, "phase-2 B tiles");
     static_assert(SMEM_BYTES <= 232448 - 512, "shared memory budget");
-    // TMEM columns: dG (later dB) NT x MS | Q NT x MS | dWd2T NWB x MS | dWd1 MS
-    static constexpr uint32_t TM_DG = 0, TM_Q = NT * MS, TM_WT = 2 * NT * MS, TM_W1 = TM_WT + NWB * MS;
+    // dWd2^T products against G_hi and G_lo: for m <= 32 as ONE product with the two tiles as
+    // the two swizzle blocks of an N = 2m operand (the accumulator's columns [0, m) and [m, 2m)
+    // are the hi and lo parts, added by the epilogue), else as two products into one accumulator
+    static constexpr bool WIDE = M_ <= 32;
+    static constexpr int MSW = WIDE ? (2 * M_ < 32 ? 32 : 2 * M_) : MS;   // TMEM columns per dWd2T accumulator
+    // TMEM columns: dG (later dB) NT x MS | Q NT x MS | dWd2T NWB x MSW | dWd1 MS
+    static constexpr uint32_t TM_DG = 0, TM_Q = NT * MS, TM_WT = 2 * NT * MS, TM_W1 = TM_WT + NWB * MSW;
     static constexpr uint32_t TMEM_NEED = TM_W1 + MS;
     static_assert(TMEM_NEED <= 512, "TMEM budget");
     static constexpr uint32_t TMEM_COLS = TMEM_NEED <= 128 ? 128 : TMEM_NEED <= 256 ? 256 : 512;
@@ -244,10 +258,14 @@ __global__ void __launch_bounds__(192, 1)
                 // dY[:, :r] tiles for phase 2, into ring slot 1 once the group's MMAs are done
                 // with the ring
                 if (!mbar_wait(smem_u32(&dg_full), g & 1)) { ok = false; break; }
-                mbar_expect_tx(smem_u32(&yr_full), (uint32_t)(te - tb) * C::TILE);
-                for (int i = tb; i < te; ++i)
+                mbar_expect_tx(smem_u32(&yr_full), 2u * (uint32_t)(te - tb) * C::TILE);
+                for (int i = tb; i < te; ++i) {
                     tma_load_2d(smem_u32(smem + C::OFF_YR + (i - tb) * C::TILE), &tm_yr, 0,
                                 (int32_t)(start + 128 * (int64_t)i), smem_u32(&yr_full));
+                    // the B tiles again (their first copy was overwritten by G_lo)
+                    tma_load_2d(smem_u32(smem + C::OFF_B2 + (i - tb) * C::TILE), &tm_b, 0,
+                                (int32_t)(start + 128 * (int64_t)i), smem_u32(&yr_full));
+                }
                 ++yr_issued;
             }
             // drain the loads still in flight
@@ -268,7 +286,7 @@ __global__ void __launch_bounds__(192, 1)
             constexpr Swz rsw = swz_for(C::RB);
             constexpr uint32_t id_q = idesc_bf16(128, C::M, false, false);   // B (K-major) . Wd1 (Wd1^T rows, K-major)
             constexpr uint32_t id_dg = idesc_bf16(128, C::M, false, false);  // dY (K-major) . Wd2 (K-major)
-            constexpr uint32_t id_wt = idesc_bf16(128, C::M, true, true);    // dY^T (MN-major) . G (MN-major)
+            constexpr uint32_t id_wt = idesc_bf16(128, C::WIDE ? 2 * C::M : C::M, true, true);   // dY^T (MN-major) . G (MN-major)
             constexpr uint32_t id_db = idesc_bf16(128, C::R, false, false);  // dQ (K-major) . Wd1^T (Wd1 rows, K-major)
             constexpr uint32_t id_w1 = idesc_bf16(128, C::M, true, true);    // B^T (MN-major) . dQ (MN-major)
             // shared-memory descriptors of slot / tile 0, advanced by adding the byte offset >> 4
@@ -278,9 +296,11 @@ __global__ void __launch_bounds__(192, 1)
             const uint64_t yk0 = smem_desc(smem_u32(smem + C::OFF_Y), 16, 1024, kSwz128);     // dY, K-major
             const uint64_t ym0 = smem_desc(smem_u32(smem + C::OFF_Y), 16384, 1024, kSwz128);  // dY, MN-major
             const uint64_t wk0 = smem_desc(smem_u32(smem + C::OFF_W), 16, 1024, kSwz128);     // Wd2 slice
-            const uint64_t gm0 = smem_desc(smem_u32(smem + C::OFF_G), 0, 8 * C::RB, rsw);     // G, MN-major
+            // G, MN-major; WIDE: [G_hi | G_lo] as two N blocks (block stride = the hi -> lo distance)
+            const uint64_t gm0 = smem_desc(smem_u32(smem + C::OFF_G), C::WIDE ? C::OFF_GLO - C::OFF_G : 0, 8 * C::RB, rsw);
+            const uint64_t gl0 = smem_desc(smem_u32(smem + C::OFF_GLO), 0, 8 * C::RB, rsw);   // G_lo, MN-major
             const uint64_t bk0 = smem_desc(smem_u32(smem + C::OFF_B), 16, 8 * C::RB, rsw);    // B, K-major
-            const uint64_t bm0 = smem_desc(smem_u32(smem + C::OFF_B), 0, 8 * C::RB, rsw);     // B^T, MN-major
+            const uint64_t bm0 = smem_desc(smem_u32(smem + C::OFF_B2), 0, 8 * C::RB, rsw);    // B^T, MN-major (phase 2)
             const uint64_t qk0 = smem_desc(smem_u32(smem + C::OFF_DQ), 16, 8 * C::RB, rsw);   // dQ, K-major
             const uint64_t qm0 = smem_desc(smem_u32(smem + C::OFF_DQ), 0, 8 * C::RB, rsw);    // dQ, MN-major
             const uint64_t w1k = smem_desc(smem_u32(smem + C::OFF_WD1), 16, 8 * C::RB, rsw);  // Wd1 rows
@@ -313,7 +333,7 @@ __global__ void __launch_bounds__(192, 1)
                          mbar_wait(smem_u32(&wt_empty[ab]), ((cit / C::NWB) & 1) ^ 1);
                     tc_fence_after();
                     const uint64_t wk = wk0 + ((sw * C::W_STAGE) >> 4);
-                    const uint32_t d_wt = tmem + C::TM_WT + ab * C::MS;
+                    const uint32_t d_wt = tmem + C::TM_WT + ab * C::MSW;
                     for (int i = tb; i < te && ok; ++i, ++yit) {
                         const int64_t t0 = start + 128 * (int64_t)i;
                         const int valid = (int)((end - t0) < 128 ? (end - t0) : 128);
@@ -324,6 +344,7 @@ __global__ void __launch_bounds__(192, 1)
                         const uint64_t yk = yk0 + ((s * C::Y_STAGE) >> 4);
                         const uint64_t ym = ym0 + ((s * C::Y_STAGE) >> 4);
                         const uint64_t gm = gm0 + (i - tb) * TILE16;
+                        const uint64_t gl = gl0 + (i - tb) * TILE16;
                         const uint32_t d_dg = tmem + C::TM_DG + (i - tb) * C::MS;
                         // dG_tile += dY_tile . Wd2_chunk^T: K = 128 columns in 8 steps of 16
                         mma_bf16(d_dg, yk, wk, id_dg, c != 0);
@@ -337,15 +358,20 @@ __global__ void __launch_bounds__(192, 1)
                             tc_fence_after();
                             if (!ok) break;
                         }
-                        // dWd2T_chunk += dY_tile^T . G_tile: K = the tile's tokens in steps of 16
+                        // dWd2T_chunk += dY_tile^T . (G_hi + G_lo)_tile: K = the tile's tokens in
+                        // steps of 16
                         if (valid == 128) {
 #pragma unroll
-                            for (int k = 0; k < 8; ++k)
+                            for (int k = 0; k < 8; ++k) {
                                 mma_bf16(d_wt, ym + ((k * 2048) >> 4), gm + k * KROWS16, id_wt, (i > tb) || (k > 0));
+                                if (!C::WIDE) mma_bf16(d_wt, ym + ((k * 2048) >> 4), gl + k * KROWS16, id_wt, true);
+                            }
                         } else {
                             const int nks = (valid + 15) / 16;
-                            for (int k = 0; k < nks; ++k)
+                            for (int k = 0; k < nks; ++k) {
                                 mma_bf16(d_wt, ym + ((k * 2048) >> 4), gm + k * KROWS16, id_wt, (i > tb) || (k > 0));
+                                if (!C::WIDE) mma_bf16(d_wt, ym + ((k * 2048) >> 4), gl + k * KROWS16, id_wt, true);
+                            }
                         }
                         mma_commit(smem_u32(&y_empty[s]));
                     }
@@ -357,6 +383,8 @@ __global__ void __launch_bounds__(192, 1)
                 mma_commit(smem_u32(&dg_full));
                 // ---- phase 2: dB_tile = (dQ_hi + dQ_lo) . Wd1^T (K = m);
                 //      dWd1 += B^T . (dQ_hi + dQ_lo) (K = tokens) ----
+                ok = ok && mbar_wait(smem_u32(&yr_full), g & 1);   // the reloaded B tiles
+                tc_fence_after();
                 for (int i = tb; i < te && ok; ++i) {
                     const int64_t t0 = start + 128 * (int64_t)i;
                     const int valid = (int)((end - t0) < 128 ? (end - t0) : 128);
@@ -407,6 +435,10 @@ __global__ void __launch_bounds__(192, 1)
 #pragma unroll
                 for (int j = 0; j < C::M; ++j) v[j] = active ? v[j] : 0.0f;
                 store_bf16_swz_row<C::M>(smem + C::OFF_G + (i - tb) * C::TILE, row, v);
+                // G_lo = G - bf16(G), over the tile's B rows (the Q products are done: q_full)
+#pragma unroll
+                for (int j = 0; j < C::M; ++j) v[j] -= __bfloat162float(__float2bfloat16_rn(v[j]));
+                store_bf16_swz_row<C::M>(smem + C::OFF_GLO + (i - tb) * C::TILE, row, v);
                 // publish this tile's G so its first dWd2 product can start
                 fence_async_smem();
                 named_barrier(1, 128);
@@ -419,9 +451,19 @@ __global__ void __launch_bounds__(192, 1)
             // (the peers' rows of that chunk have arrived by then; the accumulator waits in TMEM).
             const bool defer = xg.exchanging() && xg.owns(row);
             int pend = -1, pend_cc = 0;
+            // one row of a finished dWd2^T accumulator (WIDE: its hi part + its lo part)
+            auto load_wt = [&](int buf, float (&v)[C::M]) {
+                tmem_ld_row<C::M>(tmem + lane_base + C::TM_WT + buf * C::MSW, v);
+                if (C::WIDE) {
+                    float w[C::M];
+                    tmem_ld_row<C::M>(tmem + lane_base + C::TM_WT + buf * C::MSW + C::M, w);
+#pragma unroll
+                    for (int j = 0; j < C::M; ++j) v[j] += w[j];
+                }
+            };
             auto drain_owned = [&](int buf, int chunk) {
                 float v[C::M];
-                tmem_ld_row<C::M>(tmem + lane_base + C::TM_WT + buf * C::MS, v);
+                load_wt(buf, v);
                 tc_fence_before();
                 mbar_arrive(smem_u32(&wt_empty[buf]));   // the accumulator is free again
                 return xg.receive(a.wg, v, chunk, row, g == 0);
@@ -441,7 +483,7 @@ __global__ void __launch_bounds__(192, 1)
                     continue;
                 }
                 float v[C::M];
-                tmem_ld_row<C::M>(tmem + lane_base + C::TM_WT + ab * C::MS, v);
+                load_wt((int)ab, v);
                 tc_fence_before();
                 mbar_arrive(smem_u32(&wt_empty[ab]));   // the accumulator is free again
                 if (xg.exchanging()) {

@@ -19,7 +19,8 @@
 //   With ALO the A operand is a bf16 pair hi + lo (hi = a value rounded to bf16, lo = the
 //   rounded remainder, two matrices of the same shape): each stage holds both A tiles and the
 //   MMA warp issues hi . B and lo . B into the same accumulator, so the product sees A to about
-//   16 significant bits (used where the result crosses the boundary: B and dB).
+//   16 significant bits (used where the result crosses the boundary, B and dB, and for the
+//   decoder's dWd2 = G^T . dY, a long sum over tokens whose terms cancel for real gradients).
 //   epilogue warps : eight warps, two per TMEM lane quarter splitting the columns: TMEM ->
 //                    registers (one output row per thread, 32 columns at a time) -> the
 //                    epilogue's element-wise step -> global memory
@@ -45,7 +46,7 @@ enum GemmEpMode : int {
     GEP_BF16,      // out bf16 = acc
     GEP_P_A,       // out f32 = acc (if out), out2 bf16 = phi(acc) (lo: its remainder)  (P, A)
     GEP_ADD_AUX,   // out bf16 = acc + aux[row][col] for col < aux_cols, acc elsewhere  (B, Y, dB)
-    GEP_ACT,       // out bf16 = phi(acc), out2 f32 = acc (if out2)                     (G, Q)
+    GEP_ACT,       // out bf16 = phi(acc) (lo: its remainder), out2 f32 = acc if out2   (G, Q)
     GEP_DACT,      // out bf16 = acc * phi'(aux f32) (lo: its remainder), out2 bf16 = phi(aux) if
                    // out2                                                              (dQ; dP, A)
     GEP_DF,        // out bf16 = acc; rmw[row][col] += aux[row][col] for col < aux_cols (dF; dX += dB)
@@ -62,7 +63,7 @@ struct GemmEp {
     __nv_bfloat16 *rmw;  // DF: ldr elements per row
     int64_t ldr;
     int64_t split_stride;
-    __nv_bfloat16 *lo;   // P_A, DACT: the remainder of the bf16 activation result (same pitch)
+    __nv_bfloat16 *lo;   // P_A, ACT, DACT: the remainder of the bf16 activation result (same pitch)
 };
 
 struct GemmShape {
@@ -197,7 +198,8 @@ __device__ __forceinline__ void gemm_epilogue(const GemmEp &ep, int64_t row, int
     case GEP_ACT:
         if (ep.out2) st_f32x32(static_cast<float *>(ep.out2) + row * ep.ldo2 + col, v, nv);
         act_fast_row<32>(ep.act, v);
-        st_bf16x32(static_cast<__nv_bfloat16 *>(ep.out) + row * ep.ldo + col, v, nv);
+        st_bf16x32_split(static_cast<__nv_bfloat16 *>(ep.out) + row * ep.ldo + col,
+                         ep.lo ? ep.lo + row * ep.ldo + col : nullptr, v, nv);
         break;
     case GEP_DACT: {
         float x[32], dx[32];
@@ -236,7 +238,6 @@ __global__ void __launch_bounds__(320, 1)
            const __grid_constant__ CUtensorMap tmb, const GemmShape g, const GemmEp ep)
 {
     using C = GemmCfg<BN, ALO>;
-    static_assert(!(ALO && AMN), "hi + lo pairs only for K-major A");
     griddep_wait();               // the previous kernel of the stream has completed
     griddep_launch_dependents();  // the next one may be scheduled on SMs as they free up
     extern __shared__ uint8_t smem_raw[];
@@ -299,6 +300,10 @@ __global__ void __launch_bounds__(320, 1)
                     } else {
                         tma_load_2d(adst, &tma, mb * 128, kx, bar);
                         tma_load_2d(adst + 8192, &tma, mb * 128 + 64, kx, bar);
+                        if (ALO) {
+                            tma_load_2d(adst + C::A_TILE, &tma_lo, mb * 128, kx, bar);
+                            tma_load_2d(adst + C::A_TILE + 8192, &tma_lo, mb * 128 + 64, kx, bar);
+                        }
                     }
                     if (!BMN) {
                         tma_load_2d(bdst, &tmb, kx, nb * BN, bar);

@@ -31,6 +31,15 @@ def test_bf16_rows_have_their_own_scale():
     assert rel_err(g, o, "bf16", rowwise=False) < 1e-5
 
 
+def test_fp32_weight_gradients_get_no_rounding_allowance():
+    """The weight gradients of a bf16 workload are fp32 outputs: their whole error counts."""
+    o = np.array([[1.0, -1.0, 1.0, -1.0]])
+    g = o.copy()
+    g[0, 0] += 2.0 ** -10             # within half a bf16 spacing of 1.0, but a real fp32 error
+    assert rel_err(g, o, "bf16", rowwise=False) == pytest.approx(2.0 ** -10)
+    assert rel_err(g, o, "bf16", rowwise=True) == 0.0
+
+
 def test_f32_is_relative_with_an_rms_floor():
     o = np.array([[1.0, 1e-9, -2.0, 0.5]])
     g = o.copy()

@@ -1,0 +1,84 @@
+"""The simulated pipeline (a decoder-only transformer in stages with ResBM boundaries, Sec. 3.2
+placement): one training step through the C ABI, and every boundary's tensors of that step
+against the fp64 oracle run on the same inputs."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from gpu_helpers import to_host
+from metrics import check
+from paper_2604_11947_gb300 import pipeline, resbm
+
+pytestmark = pytest.mark.gpu
+
+
+def _check_boundary(cap, bnd, cfg, merge):
+    """Each op of one boundary against the oracle on the inputs the step gave it."""
+    X, F, dY = to_host(cap["X"]), to_host(cap["F"]), to_host(cap["dY"])
+    w = {k: to_host(getattr(bnd, k)) for k in ("We1", "We2", "Wd1", "Wd2")}
+    B, dB = to_host(cap["B"]), to_host(cap["dB"])
+    assert torch.equal(cap["B"], cap["B_dec"])          # the handoff is the tensor itself
+    if merge:
+        # reading A: b has one consumer, so the encoder receives the decoder's dB itself (its
+        # identity-path term included); reading B adds the pad skip's gradient to it
+        assert torch.equal(cap["dB"], cap["dB_in"])
+    dB_in = to_host(cap["dB_in"])
+    wantB, _ = oracle.encode_fwd(X, F, w["We1"], w["We2"], cfg.act)
+    check("B", B, wantB, "bf16")
+    check("Y", to_host(cap["Y"]), oracle.decode_fwd(B, w["Wd1"], w["Wd2"], cfg.act, merge), "bf16")
+    wdB, wdWd1, wdWd2 = oracle.decode_bwd(dY, B, w["Wd1"], w["Wd2"], cfg.act, merge)
+    check("dB", dB, wdB, "bf16")
+    check("dWd1", to_host(cap["dWd1"]), wdWd1, "bf16")
+    check("dWd2", to_host(cap["dWd2"]), wdWd2, "bf16")
+    wdF, wdX, wdWe1, wdWe2 = oracle.encode_bwd(dB_in, F, w["We1"], w["We2"], cfg.act)
+    check("dF", to_host(cap["dF"]), wdF, "bf16")
+    dX = to_host(cap["dX"])
+    assert not np.any(dX[:, cfg.r:]), "the identity path's gradient reaches only the first r columns"
+    check("dX", dX[:, :cfg.r], wdX[:, :cfg.r], "bf16")
+    check("dWe1", to_host(cap["dWe1"]), wdWe1, "bf16")
+    check("dWe2", to_host(cap["dWe2"]), wdWe2, "bf16")
+
+
+def _run(cfg):
+    model = pipeline.PipelineModel(cfg)
+    caps = []
+    for bnd in model.bounds:
+        bnd.capture = {}
+        caps.append(bnd.capture)
+    tokens = pipeline.synthetic_tokens(cfg)
+    loss = pipeline.train_step(model, tokens)
+    torch.cuda.synchronize()
+    assert torch.isfinite(loss)
+    for p in model.parameters():
+        assert p.grad is not None and torch.isfinite(p.grad.float()).all()
+    return model, caps
+
+
+def test_four_stage_pipeline_boundaries_match_oracle():
+    """24 layers, d = 2048, 16 heads, SwiGLU 5632, vocabulary 32000, 4 stages, r = 16, batch 8 x
+    seq 2048: every one of the three boundaries, forward and backward, against the oracle."""
+    cfg = pipeline.PIPELINE
+    model, caps = _run(cfg)
+    assert len(caps) == 3
+    for cap, bnd in zip(caps, model.bounds):
+        assert cap["X"].shape == (cfg.tokens, cfg.d) and cap["B"].shape == (cfg.tokens, cfg.r)
+        _check_boundary(cap, bnd, cfg, merge=1)
+    assert resbm.resbm_device_error() == 0
+
+
+def test_reading_b_wiring_boundaries_match_oracle():
+    """The decoder inside the attention branch (merge_identity = 0; pad(b) is the attention's
+    skip), on a small model."""
+    cfg = pipeline.PipelineConfig(layers=4, d=512, heads=4, ffn=1024, vocab=1000, stages=2, r=16, m=16,
+                                  batch=2, seq=256, wiring="B")
+    model, caps = _run(cfg)
+    _check_boundary(caps[0], model.bounds[0], cfg, merge=0)
+
+
+def test_boundary_share_is_measured():
+    cfg = pipeline.PipelineConfig(layers=4, d=512, heads=4, ffn=1024, vocab=1000, stages=4, r=16, m=16,
+                                  batch=2, seq=256)
+    model = pipeline.PipelineModel(cfg)
+    step_ms, bnd_ms, loss = pipeline.time_steps(model, pipeline.synthetic_tokens(cfg), steps=2, warmup=1)
+    assert 0 < bnd_ms < step_ms and np.isfinite(loss)
