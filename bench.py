@@ -518,6 +518,16 @@ def main():
         torch.cuda.empty_cache()
         extra["pipeline"] = pipeline_workload(torch)
         torch.cuda.empty_cache()
+        from paper_2604_11947_gb300 import pipeline
+        conv = pipeline.convergence()
+        conv["workload"] = ("loss curves (step, mean loss over the previous 25 steps) of a 4-layer "
+                            "decoder (d=512, 8 heads, SwiGLU 1024, vocab 256) in 2 stages with one "
+                            "ResBM boundary (r=16, 32x) wired as reading A (pad(b) + D(b) into the "
+                            "block) and reading B (D(b) into the attention branch, pad(b) its skip), "
+                            "and the same model in 1 stage (no boundary); AdamW lr 1e-3, batch 16 x "
+                            "seq 256 of a seeded random Markov stream (4 successors per token)")
+        extra["convergence"] = conv
+        torch.cuda.empty_cache()
 
     line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,

@@ -86,7 +86,9 @@ typedef enum {
     RESBM_OP_DECODE_BWD = 2,
     RESBM_OP_ENCODE_BWD = 3,
     RESBM_OP_BOUNDARY_STEP = 4,
-    RESBM_OP_BOUNDARY_STEP_HOST = 5
+    RESBM_OP_BOUNDARY_STEP_HOST = 5,
+    RESBM_OP_EFFECTIVE_RANK = 6,     /* resbm_effective_rank (workspace: resbm_matrix_workspace_bytes) */
+    RESBM_OP_NEWTON_SCHULZ = 7       /* resbm_newton_schulz  (workspace: resbm_matrix_workspace_bytes) */
 } resbm_op;
 
 /* desc.flags bits */
@@ -257,6 +259,45 @@ RESBM_API resbm_status resbm_boundary_step(const resbm_desc *desc, const resbm_s
  *   - Errors: as resbm_boundary_step; RESBM_ERR_CUDA if a copy or a stream could not be set up. */
 RESBM_API resbm_status resbm_boundary_step_host(const resbm_desc *desc, const resbm_step_args *args,
                                       void *ws, size_t ws_bytes, void *stream);
+
+/* ---- utilities on the bottleneck weights (outside the boundary op) ----------------------------
+ * Two dense kernels on a bf16 matrix, for training the bottleneck weights with Muon (Sec. 3.4.2:
+ * the bottleneck models are trained with Muon, whose update orthogonalises the gradient momentum
+ * by a Newton-Schulz iteration) and for the appendix's spectral analysis of them (the effective
+ * rank). Shapes: rows and cols multiples of 8; all pointers device memory, 16-byte aligned; `ws`
+ * device memory of resbm_matrix_workspace_bytes(op, rows, cols) bytes, 256-byte aligned; work
+ * enqueued on `stream`, nothing allocated or synchronised. Errors as for the boundary ops. */
+
+/* Muon's Newton-Schulz coefficients: the quintic iteration X <- a X + b (X X^T) X + c (X X^T)^2 X
+ * published with Muon (the paper cites Muon without restating them). */
+#define RESBM_NS_A 3.4445f
+#define RESBM_NS_B (-4.7750f)
+#define RESBM_NS_C 2.0315f
+#define RESBM_NS_EPS 1e-7f
+
+/* Scratch bytes of `op` (RESBM_OP_EFFECTIVE_RANK or RESBM_OP_NEWTON_SCHULZ) for a rows x cols
+ * matrix. INVALID_ARG for another op or a shape the kernels do not take. */
+RESBM_API resbm_status resbm_matrix_workspace_bytes(int op, int64_t rows, int64_t cols, size_t *bytes);
+
+/* Muon's orthogonalisation of a gradient (momentum) matrix G, rows x cols row-major, g_dtype
+ * RESBM_F32 or RESBM_BF16: X_0 = G / (||G||_F + RESBM_NS_EPS), then `steps` (0..100; Muon uses 5)
+ * Newton-Schulz steps X <- a X + (b A + c A A) X with A = X X^T, taken on the wide orientation
+ * (for rows > cols the same iteration on X^T, i.e. X <- a X + X (b A + c A A) with A = X^T X).
+ * X (rows x cols, bf16) receives the result; its singular vectors are G's and its singular values
+ * are driven toward 1 (to about [0.7, 1.2]). The products run on the tensor cores with bf16
+ * operands and fp32 accumulation, every iterate and product rounded to bf16, as Muon does. */
+RESBM_API resbm_status resbm_newton_schulz(int64_t rows, int64_t cols, const void *G, int32_t g_dtype,
+                                 int32_t steps, void *X, void *ws, size_t ws_bytes, void *stream);
+
+/* The effective rank of a bf16 matrix W (rows x cols, row-major) as the appendix's spectral
+ * analysis defines it, r_eff = sum_i sigma_i^2 / max_i sigma_i^2, computed as trace(S) /
+ * lambda_max(S) for the Gram matrix S of W's smaller side (W^T W or W W^T; fp32 sums of the exact
+ * bf16 products), lambda_max by power iteration on one CTA until the residual ||S v - lambda v||
+ * is at most 1e-5 lambda ||v|| (at most 20000 iterations): some eigenvalue of S then lies within
+ * 1e-5 (relative) of lambda (Bauer-Fike; the fp32 products put the residual's floor near 1e-6). `out` (device, 4 doubles): sigma_max^2, ||W||_F^2, r_eff, the iterations
+ * taken. min(rows, cols) <= 4096. */
+RESBM_API resbm_status resbm_effective_rank(int64_t rows, int64_t cols, const void *W, double *out,
+                                  void *ws, size_t ws_bytes, void *stream);
 
 #ifdef __cplusplus
 }

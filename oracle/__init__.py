@@ -13,6 +13,11 @@ Citations (sections and equations of the ResBM paper):
   decode_bwd / encode_bwd .... the chain rule of the two forward functions
   effective_rank ............. the appendix's spectral analysis of the bottleneck output
                                projections: r_eff = sum_i sigma_i^2 / max_i sigma_i^2
+  newton_schulz .............. Muon's orthogonalisation of the gradient momentum (Sec. 3.4.2
+                               trains the bottleneck weights with Muon): X_0 = G / ||G||_F, then
+                               X <- a X + b (X X^T) X + c (X X^T)^2 X on the wide orientation,
+                               with the coefficients published with Muon (the paper cites Muon and
+                               does not restate them)
 """
 import ctypes
 import os
@@ -301,3 +306,26 @@ def __getattr__(name):
                 "linear_boundary_step"):
         return getattr(default(), name)
     raise AttributeError(name)
+
+
+NS_COEFFS = (3.4445, -4.7750, 2.0315)   # Muon's quintic Newton-Schulz coefficients (a, b, c)
+
+
+def newton_schulz(G, steps=5, coeffs=NS_COEFFS, eps=1e-7):
+    """Muon's Newton-Schulz orthogonalisation in float64, step by step as the iteration is
+    stated: X_0 = G / (||G||_F + eps); for a matrix with more rows than columns the iteration runs
+    on its transpose; each step A = X X^T, B = b A + c A A, X <- a X + B X. numpy's matmul is the
+    library step for every product."""
+    G = np.asarray(G, dtype=np.float64)
+    if G.ndim != 2:
+        raise ValueError("newton_schulz takes a matrix")
+    a, b, c = coeffs
+    X = G / (np.linalg.norm(G) + eps)
+    tall = X.shape[0] > X.shape[1]
+    if tall:
+        X = X.T
+    for _ in range(steps):
+        A = X @ X.T
+        B = b * A + c * (A @ A)
+        X = a * X + B @ X
+    return X.T if tall else X

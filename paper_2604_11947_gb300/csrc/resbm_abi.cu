@@ -714,6 +714,48 @@ resbm_status resbm_boundary_step(const resbm_desc *desc, const resbm_step_args *
     return s == RESBM_OK ? enqueue_step(d, *a, ws, c, nullptr, nullptr) : s;
 }
 
+resbm_status resbm_matrix_workspace_bytes(int op, int64_t rows, int64_t cols, size_t *bytes)
+{
+    if (!bytes || (op != RESBM_OP_EFFECTIVE_RANK && op != RESBM_OP_NEWTON_SCHULZ)) return RESBM_ERR_INVALID_ARG;
+    if (!matrix_supported(rows, cols)) return RESBM_ERR_INVALID_ARG;
+    *bytes = matrix_ws_bytes(op, rows, cols, sizing_sms());
+    return RESBM_OK;
+}
+
+resbm_status resbm_newton_schulz(int64_t rows, int64_t cols, const void *G, int32_t g_dtype, int32_t steps, void *X,
+                                 void *ws, size_t ws_bytes, void *stream)
+{
+    if (!matrix_supported(rows, cols) || steps < 0 || steps > 100 || (g_dtype != RESBM_F32 && g_dtype != RESBM_BF16))
+        return RESBM_ERR_INVALID_ARG;
+    const size_t es = g_dtype == RESBM_F32 ? 4 : 2;
+    if (!G || !X || !aligned16(G) || !aligned16(X)) return RESBM_ERR_INVALID_ARG;
+    if (overlaps(rng(G, rows * cols, es), rng(X, rows * cols, 2))) return RESBM_ERR_INVALID_ARG;
+    const size_t need = matrix_ws_bytes(RESBM_OP_NEWTON_SCHULZ, rows, cols, sizing_sms());
+    if (!ws || ws_bytes < need) return RESBM_ERR_WORKSPACE;
+    if (reinterpret_cast<uintptr_t>(ws) % 256) return RESBM_ERR_INVALID_ARG;
+    Ctx c;
+    resbm_status s = make_ctx(stream, &c);
+    if (s != RESBM_OK) return s;
+    const float coef[3] = {RESBM_NS_A, RESBM_NS_B, RESBM_NS_C};
+    const cudaError_t e = tc_newton_schulz(rows, cols, G, g_dtype == RESBM_F32, steps, coef, RESBM_NS_EPS, X, ws, c);
+    return e == cudaErrorNotSupported ? RESBM_ERR_UNSUPPORTED : finish(e);
+}
+
+resbm_status resbm_effective_rank(int64_t rows, int64_t cols, const void *W, double *out, void *ws, size_t ws_bytes,
+                                  void *stream)
+{
+    if (!matrix_supported(rows, cols) || (rows < cols ? rows : cols) > 4096) return RESBM_ERR_INVALID_ARG;
+    if (!W || !out || !aligned16(W) || (reinterpret_cast<uintptr_t>(out) % 8)) return RESBM_ERR_INVALID_ARG;
+    const size_t need = matrix_ws_bytes(RESBM_OP_EFFECTIVE_RANK, rows, cols, sizing_sms());
+    if (!ws || ws_bytes < need) return RESBM_ERR_WORKSPACE;
+    if (reinterpret_cast<uintptr_t>(ws) % 256) return RESBM_ERR_INVALID_ARG;
+    Ctx c;
+    resbm_status s = make_ctx(stream, &c);
+    if (s != RESBM_OK) return s;
+    const cudaError_t e = tc_effective_rank(rows, cols, W, out, ws, c);
+    return e == cudaErrorNotSupported ? RESBM_ERR_UNSUPPORTED : finish(e);
+}
+
 resbm_status resbm_boundary_step_host(const resbm_desc *desc, const resbm_step_args *a, void *ws,
                                       size_t ws_bytes, void *stream)
 {

@@ -19,6 +19,7 @@
 #include "tc_dec_bwd.cuh"
 #include "tc_enc_bwd.cuh"
 #include "tc_gemm.cuh"
+#include "tc_spectral.cuh"
 
 namespace resbm {
 
@@ -518,16 +519,17 @@ tc::GemmEp ep_of(int mode, int act, void *out, int64_t ldo)
 // A weight gradient W (M x N fp32) = A^T . B over K tokens (both operands MN-major), split over
 // the tokens when it has few output tiles: the splits' fp32 slots go to `slots` and the job to
 // sum them (in slot order) is returned in `job` (job->blocks = 0: nothing to reduce).
-// A_lo: A as a bf16 hi + lo pair (or null).
+// A_lo: A as a bf16 hi + lo pair (or null). a_mn / b_mn: the operand majors (both MN-major for the
+// weight gradients, whose K is the tokens).
 cudaError_t wgrad(const Ctx &c, int64_t M, int64_t N, int64_t K, const void *A, const void *B, float *W, float *slots,
-                  tc::ReduceJob *job, const void *A_lo = nullptr)
+                  tc::ReduceJob *job, const void *A_lo = nullptr, bool a_mn = true, bool b_mn = true)
 {
     const int s = gemm_splits(M, N, K, c.sm_count);
     *job = tc::ReduceJob{nullptr, 0, 0, 0, nullptr, 0, 0, 0};
-    if (s <= 1) return gemm(c, M, N, K, A, true, B, true, ep_of(tc::GEP_F32, 0, W, N), 1, A_lo);
+    if (s <= 1) return gemm(c, M, N, K, A, a_mn, B, b_mn, ep_of(tc::GEP_F32, 0, W, N), 1, A_lo);
     tc::GemmEp e = ep_of(tc::GEP_F32, 0, slots, N);
     e.split_stride = M * N;
-    cudaError_t err = gemm(c, M, N, K, A, true, B, true, e, s, A_lo);
+    cudaError_t err = gemm(c, M, N, K, A, a_mn, B, b_mn, e, s, A_lo);
     if (err != cudaSuccess) return err;
     // the number of splits the launch took (gemm rounds K per split to 64)
     const int64_t kc = ((K + s - 1) / s + 63) / 64 * 64;
@@ -788,6 +790,117 @@ cudaError_t gemm_encode_bwd(const resbm_desc &d, const void *dB, const void *F, 
     if (e == cudaSuccess) e = wgrad(c, d.d, d.m, d.T, F, w.dP, dWe1, w.slots1, &j1);
     if (e == cudaSuccess) e = wgrad(c, d.m, d.r, d.T, w.A, dB, dWe2, w.slots2, &j2);
     if (e == cudaSuccess) e = reduce_jobs(j2, j1, c);
+    return e;
+}
+
+// ---- Muon's Newton-Schulz orthogonalisation and the effective rank ----------------------------
+namespace {
+// Scratch: the sum-of-squares partials, the two bf16 iterates (or the Gram matrix and its split
+// slots for the effective rank), and the s x s products (s = min(rows, cols)).
+struct MatrixWs {
+    double *part = nullptr;
+    __nv_bfloat16 *X = nullptr, *A = nullptr, *Bm = nullptr;
+    float *gram = nullptr, *slots = nullptr;
+    double *out = nullptr;
+    size_t bytes = 0;
+};
+MatrixWs matrix_ws(int op, int64_t rows, int64_t cols, int sms, void *ws)
+{
+    MatrixWs w;
+    WsCarver cv(ws);
+    const int64_t sd = rows < cols ? rows : cols, ld = rows < cols ? cols : rows;
+    if (op == RESBM_OP_NEWTON_SCHULZ) {
+        w.part = cv.take<double>(tc::kSqBlocks);
+        w.X = cv.take<__nv_bfloat16>(rows * cols);
+        w.A = cv.take<__nv_bfloat16>(sd * sd);
+        w.Bm = cv.take<__nv_bfloat16>(sd * sd);
+    } else {
+        w.gram = cv.take<float>(sd * sd);
+        w.slots = cv.take<float>(slot_floats(sd, sd, ld, sms));
+    }
+    w.bytes = cv.used;
+    return w;
+}
+}  // namespace
+
+size_t matrix_ws_bytes(int op, int64_t rows, int64_t cols, int sms) { return matrix_ws(op, rows, cols, sms, nullptr).bytes; }
+
+bool matrix_supported(int64_t rows, int64_t cols)
+{
+    return rows >= 1 && cols >= 1 && rows % 8 == 0 && cols % 8 == 0 && rows <= INT32_MAX && cols <= INT32_MAX;
+}
+
+cudaError_t tc_newton_schulz(int64_t rows, int64_t cols, const void *G, bool g_f32, int steps, const float coef[3],
+                             float eps, void *X_out, void *ws, const Ctx &c)
+{
+    if (!al16(G) || !al16(X_out) || !al16(ws) || encode_fn() == nullptr) return cudaErrorNotSupported;
+    const MatrixWs w = matrix_ws(RESBM_OP_NEWTON_SCHULZ, rows, cols, c.sm_count, ws);
+    const int64_t n = rows * cols;
+    __nv_bfloat16 *out = static_cast<__nv_bfloat16 *>(X_out);
+    // the iterates alternate between the output and the scratch copy so that the last one lands in
+    // the output: X0 in the scratch copy for an odd number of steps
+    __nv_bfloat16 *cur = steps % 2 ? w.X : out, *nxt = steps % 2 ? out : w.X;
+    int64_t grid = (n + 255) / 256;
+    if (grid > (int64_t)c.sm_count * 8) grid = (int64_t)c.sm_count * 8;
+    cudaError_t e;
+    if (g_f32) {
+        e = launch(tc::k_sumsq<float>, tc::kSqBlocks, 256, 0, c.stream, static_cast<const float *>(G), n, w.part);
+        if (e == cudaSuccess)
+            e = launch(tc::k_scale_bf16<float>, (unsigned)grid, 256, 0, c.stream, static_cast<const float *>(G), n,
+                       (const double *)w.part, eps, cur);
+    } else {
+        e = launch(tc::k_sumsq<__nv_bfloat16>, tc::kSqBlocks, 256, 0, c.stream, static_cast<const __nv_bfloat16 *>(G),
+                   n, w.part);
+        if (e == cudaSuccess)
+            e = launch(tc::k_scale_bf16<__nv_bfloat16>, (unsigned)grid, 256, 0, c.stream,
+                       static_cast<const __nv_bfloat16 *>(G), n, (const double *)w.part, eps, cur);
+    }
+    count_launches(2);
+    const bool wide = rows <= cols;
+    const int64_t sd = wide ? rows : cols;
+    for (int k = 0; k < steps && e == cudaSuccess; ++k) {
+        // A = X X^T (wide) or X^T X (tall): the s x s Gram matrix of the iterate
+        e = wide ? gemm(c, sd, sd, cols, cur, false, cur, false, ep_of(tc::GEP_BF16, 0, w.A, sd), 1)
+                 : gemm(c, sd, sd, rows, cur, true, cur, true, ep_of(tc::GEP_BF16, 0, w.A, sd), 1);
+        // Bm = b A + c A A
+        tc::GemmEp eb = ep_of(tc::GEP_AXPBY, 0, w.Bm, sd);
+        eb.aux = w.A;
+        eb.lda = sd;
+        eb.alpha = coef[2];
+        eb.beta = coef[1];
+        if (e == cudaSuccess) e = gemm(c, sd, sd, sd, w.A, false, w.A, true, eb, 1);
+        // X <- a X + Bm X (wide) or a X + X Bm (tall; Bm is symmetric)
+        tc::GemmEp ex = ep_of(tc::GEP_AXPBY, 0, nxt, cols);
+        ex.aux = cur;
+        ex.lda = cols;
+        ex.alpha = 1.0f;
+        ex.beta = coef[0];
+        if (e == cudaSuccess)
+            e = wide ? gemm(c, rows, cols, rows, w.Bm, false, cur, true, ex, 1)
+                     : gemm(c, rows, cols, cols, cur, false, w.Bm, true, ex, 1);
+        __nv_bfloat16 *t = cur;
+        cur = nxt;
+        nxt = t;
+    }
+    return e;
+}
+
+cudaError_t tc_effective_rank(int64_t rows, int64_t cols, const void *W, double *out, void *ws, const Ctx &c)
+{
+    if (!al16(W) || !al16(ws) || encode_fn() == nullptr) return cudaErrorNotSupported;
+    const MatrixWs w = matrix_ws(RESBM_OP_EFFECTIVE_RANK, rows, cols, c.sm_count, ws);
+    const bool tall = rows >= cols;
+    const int64_t sd = tall ? cols : rows, ld = tall ? rows : cols;
+    if (sd > tc::kPowMaxN) return cudaErrorNotSupported;
+    // the Gram matrix of the smaller side: W^T W (tall) or W W^T (wide), fp32 sums of bf16 products
+    tc::ReduceJob job;
+    cudaError_t e = tall ? wgrad(c, sd, sd, ld, W, W, w.gram, w.slots, &job)
+                         : wgrad(c, sd, sd, ld, W, W, w.gram, w.slots, &job, nullptr, false, false);
+    if (e == cudaSuccess) e = reduce_jobs(job, tc::ReduceJob{nullptr, 0, 0, 0, nullptr, 0, 0, 0}, c);
+    if (e == cudaSuccess) {
+        e = launch(tc::k_power_iter, 1, 1024, 0, c.stream, (const float *)w.gram, (int)sd, 20000, 1e-5f, out);
+        count_launches(1);
+    }
     return e;
 }
 

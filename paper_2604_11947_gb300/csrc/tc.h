@@ -50,4 +50,14 @@ cudaError_t gemm_encode_bwd(const resbm_desc &d, const void *dB, const void *F, 
                             const void *We1, const void *We2, void *dF, void *dX, float *dWe1,
                             float *dWe2, void *ws, const Ctx &c);
 
+// Muon's Newton-Schulz orthogonalisation and the effective rank of a matrix (tc_spectral.cuh and
+// the GEMM): rows, cols multiples of 8; 16-byte aligned pointers (else cudaErrorNotSupported
+// before anything is enqueued).
+bool matrix_supported(int64_t rows, int64_t cols);
+size_t matrix_ws_bytes(int op, int64_t rows, int64_t cols, int sms);
+cudaError_t tc_newton_schulz(int64_t rows, int64_t cols, const void *G, bool g_f32, int steps,
+                             const float coef[3], float eps, void *X_out, void *ws, const Ctx &c);
+cudaError_t tc_effective_rank(int64_t rows, int64_t cols, const void *W, double *out, void *ws,
+                              const Ctx &c);
+
 }  // namespace resbm

@@ -50,6 +50,7 @@ enum GemmEpMode : int {
     GEP_DACT,      // out bf16 = acc * phi'(aux f32) (lo: its remainder), out2 bf16 = phi(aux) if
                    // out2                                                              (dQ; dP, A)
     GEP_DF,        // out bf16 = acc; rmw[row][col] += aux[row][col] for col < aux_cols (dF; dX += dB)
+    GEP_AXPBY,     // out bf16 = alpha * acc + beta * aux[row][col] (aux bf16; the Newton-Schulz steps)
 };
 
 struct GemmEp {
@@ -64,6 +65,7 @@ struct GemmEp {
     int64_t ldr;
     int64_t split_stride;
     __nv_bfloat16 *lo;   // P_A, ACT, DACT: the remainder of the bf16 activation result (same pitch)
+    float alpha, beta;   // AXPBY
 };
 
 struct GemmShape {
@@ -213,6 +215,14 @@ __device__ __forceinline__ void gemm_epilogue(const GemmEp &ep, int64_t row, int
             act_fast_row<32>(ep.act, x);
             st_bf16x32(static_cast<__nv_bfloat16 *>(ep.out2) + row * ep.ldo2 + col, x, nv);
         }
+        break;
+    }
+    case GEP_AXPBY: {
+        float x[32];
+        ld_bf16x32(static_cast<const __nv_bfloat16 *>(ep.aux) + row * ep.lda + col, x, nv);
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] = fmaf(ep.alpha, v[j], ep.beta * x[j]);
+        st_bf16x32(static_cast<__nv_bfloat16 *>(ep.out) + row * ep.ldo + col, v, nv);
         break;
     }
     case GEP_DF:

@@ -18,7 +18,7 @@ RESBM_OK, RESBM_ERR_INVALID_ARG, RESBM_ERR_UNSUPPORTED, RESBM_ERR_WORKSPACE, RES
 RESBM_F32, RESBM_BF16 = 0, 1
 RESBM_ACT_SILU, RESBM_ACT_GELU_TANH, RESBM_ACT_IDENTITY = 0, 1, 2
 (RESBM_OP_ENCODE_FWD, RESBM_OP_DECODE_FWD, RESBM_OP_DECODE_BWD, RESBM_OP_ENCODE_BWD,
- RESBM_OP_BOUNDARY_STEP, RESBM_OP_BOUNDARY_STEP_HOST) = range(6)
+ RESBM_OP_BOUNDARY_STEP, RESBM_OP_BOUNDARY_STEP_HOST, RESBM_OP_EFFECTIVE_RANK, RESBM_OP_NEWTON_SCHULZ) = range(8)
 RESBM_FLAG_GENERIC = 1
 RESBM_FLAG_LINEAR = 2
 RESBM_FLAG_GEMM = 4
@@ -32,7 +32,8 @@ EXPORTS = ("resbm_version", "resbm_status_string", "resbm_last_cuda_error", "res
            "resbm_device_error",
            "resbm_workspace_bytes", "resbm_encode_fwd", "resbm_decode_fwd", "resbm_decode_bwd",
            "resbm_encode_bwd", "resbm_boundary_step", "resbm_boundary_step_host",
-           "resbm_decode_bwd_noalloc", "resbm_selftest_wait_timeout")
+           "resbm_decode_bwd_noalloc", "resbm_selftest_wait_timeout", "resbm_matrix_workspace_bytes",
+           "resbm_newton_schulz", "resbm_effective_rank")
 
 
 class resbm_desc(ctypes.Structure):
@@ -100,6 +101,13 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.resbm_boundary_step.argtypes = [D, ctypes.POINTER(resbm_step_args), vp, sz, vp]
     lib.resbm_boundary_step_host.restype = i32
     lib.resbm_boundary_step_host.argtypes = [D, ctypes.POINTER(resbm_step_args), vp, sz, vp]
+    i64 = ctypes.c_int64
+    lib.resbm_matrix_workspace_bytes.restype = i32
+    lib.resbm_matrix_workspace_bytes.argtypes = [i32, i64, i64, ctypes.POINTER(sz)]
+    lib.resbm_newton_schulz.restype = i32
+    lib.resbm_newton_schulz.argtypes = [i64, i64, vp, ctypes.c_int32, ctypes.c_int32, vp, vp, sz, vp]
+    lib.resbm_effective_rank.restype = i32
+    lib.resbm_effective_rank.argtypes = [i64, i64, vp, vp, vp, sz, vp]
     if path is None:
         _lib = lib
     return lib
@@ -243,3 +251,30 @@ def step_outputs(desc: resbm_desc, device="cuda", with_dX=True) -> dict:
     if with_dX:
         out["dX"] = torch.zeros(T, d, dtype=io, device=device)
     return out
+
+
+# ---- utilities on the bottleneck weights ------------------------------------------------------
+def resbm_matrix_workspace_bytes(op: int, rows: int, cols: int) -> int:
+    out = ctypes.c_size_t(0)
+    _check("resbm_matrix_workspace_bytes", load().resbm_matrix_workspace_bytes(int(op), int(rows), int(cols),
+                                                                               ctypes.byref(out)))
+    return int(out.value)
+
+
+def matrix_workspace(op: int, rows: int, cols: int, device="cuda") -> torch.Tensor:
+    return torch.empty(max(resbm_matrix_workspace_bytes(op, rows, cols), 1), dtype=torch.uint8, device=device)
+
+
+def resbm_newton_schulz(G, steps, X, ws, stream=None):
+    """X (bf16, G's shape) = Muon's Newton-Schulz orthogonalisation of G (fp32 or bf16)."""
+    rows, cols = G.shape
+    g_dtype = RESBM_F32 if G.dtype == torch.float32 else RESBM_BF16
+    _check("resbm_newton_schulz", load().resbm_newton_schulz(rows, cols, _p(G), g_dtype, int(steps), _p(X), _p(ws),
+                                                             _nbytes(ws), _stream(stream)))
+
+
+def resbm_effective_rank(W, out, ws, stream=None):
+    """out (device float64, 4): sigma_max^2, ||W||_F^2, r_eff, power iterations taken."""
+    rows, cols = W.shape
+    _check("resbm_effective_rank", load().resbm_effective_rank(rows, cols, _p(W), _p(out), _p(ws), _nbytes(ws),
+                                                               _stream(stream)))

@@ -32,7 +32,13 @@ from dataclasses import dataclass, replace
 import numpy as np
 
 TENSOR_IDS = {"X": 1, "F": 2, "dY": 3, "We1": 4, "We2": 5, "Wd1": 6, "Wd2": 7,
-              "scale": 8, "dB": 9, "dX0": 10}
+              "scale": 8, "dB": 9, "dX0": 10, "matrix": 11}
+
+
+def matrix(rows: int, cols: int, seed: int = 0) -> np.ndarray:
+    """A rows x cols matrix of N(0,1) draws (fp64) for the weight-matrix utilities; seed selects
+    the stream."""
+    return normal(seed, TENSOR_IDS["matrix"], 0, rows * cols).reshape(rows, cols)
 
 _G = np.uint64(0x9E3779B97F4A7C15)
 _M1 = np.uint64(0xBF58476D1CE4E5B9)

@@ -24,7 +24,7 @@ def declared_functions():
 
 def test_exports_every_declared_symbol(lib):
     names = declared_functions()
-    assert len(names) == 14, names
+    assert len(names) == 17, names
     assert sorted(resbm.EXPORTS) == names
     for n in names:
         assert hasattr(lib, n), n
@@ -167,3 +167,27 @@ def test_linear_flag_rules(lib):
     assert lib.resbm_decode_fwd(ctypes.byref(ok), A, None, A + big, A + 2 * big, None, 0, None) \
         == resbm.RESBM_ERR_WORKSPACE
     assert resbm.resbm_workspace_bytes(ok, resbm.RESBM_OP_DECODE_FWD) > 0
+
+
+def test_matrix_utilities_reject_bad_arguments(lib):
+    """resbm_newton_schulz / resbm_effective_rank: shapes, dtypes, steps, pointers and workspace are
+    checked on the host before anything is enqueued (fake aligned device addresses)."""
+    sz = ctypes.c_size_t(0)
+    assert lib.resbm_matrix_workspace_bytes(resbm.RESBM_OP_NEWTON_SCHULZ, 32, 4096, ctypes.byref(sz)) == resbm.RESBM_OK
+    assert sz.value > 0
+    assert lib.resbm_matrix_workspace_bytes(resbm.RESBM_OP_EFFECTIVE_RANK, 4096, 32, ctypes.byref(sz)) == resbm.RESBM_OK
+    assert lib.resbm_matrix_workspace_bytes(resbm.RESBM_OP_DECODE_BWD, 32, 32, ctypes.byref(sz)) == resbm.RESBM_ERR_INVALID_ARG
+    assert lib.resbm_matrix_workspace_bytes(resbm.RESBM_OP_NEWTON_SCHULZ, 30, 32, ctypes.byref(sz)) == resbm.RESBM_ERR_INVALID_ARG
+    A, big = 1 << 40, 1 << 30
+    G, X, ws = A, A + big, A + 2 * big
+    ns = lib.resbm_newton_schulz
+    assert ns(30, 64, G, resbm.RESBM_F32, 5, X, ws, 1 << 30, None) == resbm.RESBM_ERR_INVALID_ARG    # rows % 8
+    assert ns(32, 64, G, 7, 5, X, ws, 1 << 30, None) == resbm.RESBM_ERR_INVALID_ARG                  # dtype
+    assert ns(32, 64, G, resbm.RESBM_F32, 101, X, ws, 1 << 30, None) == resbm.RESBM_ERR_INVALID_ARG  # steps
+    assert ns(32, 64, G, resbm.RESBM_F32, 5, G + 8, ws, 1 << 30, None) == resbm.RESBM_ERR_INVALID_ARG  # overlap
+    assert ns(32, 64, G + 4, resbm.RESBM_F32, 5, X, ws, 1 << 30, None) == resbm.RESBM_ERR_INVALID_ARG  # misaligned
+    assert ns(32, 64, G, resbm.RESBM_F32, 5, X, ws, 16, None) == resbm.RESBM_ERR_WORKSPACE
+    er = lib.resbm_effective_rank
+    assert er(4096, 32, G, X, ws, 16, None) == resbm.RESBM_ERR_WORKSPACE
+    assert er(8192, 8192, G, X, ws, 1 << 34, None) == resbm.RESBM_ERR_INVALID_ARG               # min side > 4096
+    assert er(4096, 32, G, X + 4, ws, 1 << 30, None) == resbm.RESBM_ERR_INVALID_ARG              # out not 8-byte aligned
