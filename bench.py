@@ -557,6 +557,41 @@ def main():
         dist.destroy_process_group()
 
 
+def host_link(torch, mib=512, reps=3):
+    """The host link's copy rates with page-locked buffers (GB/s, best of `reps`): host to device
+    and device to host alone on one stream, and both at once on two streams (the floor of the
+    host-buffer step: its bytes each way over these rates)."""
+    n = mib << 20
+    h_in = torch.empty(n, dtype=torch.uint8).pin_memory()
+    h_out = torch.empty(n, dtype=torch.uint8).pin_memory()
+    d_in = torch.empty(n, dtype=torch.uint8, device="cuda")
+    d_out = torch.empty(n, dtype=torch.uint8, device="cuda")
+    s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
+
+    def timed(fn):
+        best = float("inf")
+        for _ in range(reps):
+            torch.cuda.synchronize()
+            t0 = time.perf_counter()
+            fn()
+            torch.cuda.synchronize()
+            best = min(best, time.perf_counter() - t0)
+        return best
+
+    t_h2d = timed(lambda: d_in.copy_(h_in, non_blocking=True))
+    t_d2h = timed(lambda: h_out.copy_(d_out, non_blocking=True))
+
+    def both():
+        with torch.cuda.stream(s1):
+            d_in.copy_(h_in, non_blocking=True)
+        with torch.cuda.stream(s2):
+            h_out.copy_(d_out, non_blocking=True)
+
+    t_both = timed(both)
+    return {"h2d_GBps": n / t_h2d / 1e9, "d2h_GBps": n / t_d2h / 1e9, "bidirectional_each_GBps": n / t_both / 1e9,
+            "bytes": n, "how": "torch copies between page-locked host and device buffers, best of %d" % reps}
+
+
 def run_e2e(args, cfg, w, resbm, torch, dist, world):
     """The same step through the C ABI with HOST buffers (resbm_boundary_step_host): inputs in
     pinned host memory, results back into pinned host memory, every copy inside the call and
@@ -601,7 +636,7 @@ def run_e2e(args, cfg, w, resbm, torch, dist, world):
     ms = max_over_ranks((time.perf_counter() - t0) * 1e3, dist, "cuda")
     return {"value": job_throughput(cfg.T, world, n, ms), "unit": "tokens/s",
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": n,
-            "ms_per_step": ms / n,
+            "ms_per_step": ms / n, "host_link": host_link(torch),
             "api": "resbm_boundary_step_host (host buffers; copies inside the call; dX[:, :r] += dB)",
             "pipelined": "two calls in flight on two streams with two device workspaces; "
                          "host wall clock from the first copy to the last result on the host"}
