@@ -406,6 +406,48 @@ def extra_workload(name, cfg, flags, resbm, torch, steps, warmup, peaks, reuse=N
     return res, dev
 
 
+def ffn_encode_workload(resbm, torch, steps=20, warmup=3):
+    """The encoder fused into the FFN down-projection against the unfused chain, at the fifth
+    workload's boundary (T = 16384, FFN width 5632, d = 2048, r = m = 16): fused (F never stored),
+    fused with F stored (for the backward), and the down-projection by torch.matmul (cuBLAS) with F
+    stored then resbm_encode_fwd reading it back."""
+    T, f, d, r, m = 16384, 5632, 2048, 16, 16
+    cfg = synth.BoundaryConfig("ffn_encode", T=T, d=d, r=r, m=m)
+    g = torch.Generator(device="cuda")
+    g.manual_seed(0)
+    H = (torch.randn(T, f, device="cuda", generator=g) * 0.5).to(torch.bfloat16)
+    W2 = (torch.randn(f, d, device="cuda", generator=g) / f ** 0.5).to(torch.bfloat16)
+    X = torch.randn(T, d, device="cuda", generator=g).to(torch.bfloat16)
+    We1 = (torch.randn(d, m, device="cuda", generator=g) / d ** 0.5).to(torch.bfloat16)
+    We2 = (torch.randn(m, r, device="cuda", generator=g) / m ** 0.5).to(torch.bfloat16)
+    desc = resbm.desc_from_config(cfg)
+    ws = resbm.ffn_down_encode_workspace(desc, f)
+    ws_enc = resbm.workspace(desc, resbm.RESBM_OP_ENCODE_FWD)
+    B = torch.empty(T, r, dtype=torch.bfloat16, device="cuda")
+    P = torch.empty(T, m, dtype=torch.float32, device="cuda")
+    F = torch.empty(T, d, dtype=torch.bfloat16, device="cuda")
+    runs = {"fused": lambda: resbm.resbm_ffn_down_encode_fwd(desc, H, W2, X, We1, We2, B, P, None, ws),
+            "fused_storing_F": lambda: resbm.resbm_ffn_down_encode_fwd(desc, H, W2, X, We1, We2, B, P, F, ws),
+            "unfused_cublas_then_encode": lambda: (torch.matmul(H, W2, out=F),
+                                                   resbm.resbm_encode_fwd(desc, X, F, We1, We2, B, P, ws_enc))}
+    res = {"workload": "FFN down-projection (T=%d, FFN width %d, d=%d) with the ResBM encoder (r=m=%d) "
+                       "after it, bf16" % (T, f, d, r), "steps": steps, "flops": 2 * T * f * d + 2 * T * d * m}
+    for name, fn in runs.items():
+        for _ in range(warmup):
+            fn()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(steps):
+            fn()
+        b.record()
+        torch.cuda.synchronize()
+        ms = a.elapsed_time(b) / steps
+        res[name] = {"ms": ms, "TFLOPs": res["flops"] / (ms / 1e3) / 1e12}
+    res["F_bytes_not_stored"] = 2 * T * d * 2   # written and read back by the unfused chain
+    return res
+
+
 def pipeline_workload(torch, steps=3, warmup=2):
     """The simulated 4-stage pipeline: one training step (forward + backward) of the 24-layer
     transformer with three ResBM boundaries; the boundary kernels' share of the step time."""
@@ -522,6 +564,8 @@ def main():
             extra[name], reuse = extra_workload(name, synth.CONFIGS[name], flags, resbm, torch,
                                                 k_extra, w_extra, peaks, reuse)
         del reuse
+        torch.cuda.empty_cache()
+        extra["ffn_down_encode"] = ffn_encode_workload(resbm, torch)
         torch.cuda.empty_cache()
         extra["pipeline"] = pipeline_workload(torch)
         torch.cuda.empty_cache()

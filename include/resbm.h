@@ -260,6 +260,25 @@ RESBM_API resbm_status resbm_boundary_step(const resbm_desc *desc, const resbm_s
 RESBM_API resbm_status resbm_boundary_step_host(const resbm_desc *desc, const resbm_step_args *args,
                                       void *ws, size_t ws_bytes, void *stream);
 
+/* ---- the encoder fused into the feed-forward down-projection -------------------------------------
+ * Sec. 3.2 places the encoder after the feed-forward layer: z = F = H . W2 (the down-projection of
+ * the FFN hidden state H) is the encoder's input. This entry point computes F on the tensor cores
+ * and feeds each output tile straight into the encoder (P = F . We1 accumulated from the tiles,
+ * then B = X[:, :r] + phi(P) . We2), so F does not travel through memory unless asked for.
+ *   H      T x f bf16 (the FFN hidden state, f = the FFN width), W2 f x d bf16
+ *   X      T x d bf16 (the encoder's skip input; only its first r columns are read)
+ *   We1    d x m, We2 m x r (bf16); B T x r bf16 (output); P_save T x m fp32 or NULL
+ *   F_out  T x d bf16 or NULL: F itself, rounded to bf16 (what the encoder's backward reads)
+ * The encoder sees F rounded to bf16, as it would if F were stored first. Requirements: bf16,
+ * two linear layers (not RESBM_FLAG_LINEAR), m a multiple of 8 with m <= 32, r <= 32, d and f
+ * multiples of 8, 16-byte aligned pointers; otherwise RESBM_ERR_UNSUPPORTED. `ws`: device memory of
+ * resbm_ffn_down_encode_workspace_bytes(desc, f) bytes (the partial P slots), 256-byte aligned. */
+RESBM_API resbm_status resbm_ffn_down_encode_workspace_bytes(const resbm_desc *desc, int64_t f, size_t *bytes);
+RESBM_API resbm_status resbm_ffn_down_encode_fwd(const resbm_desc *desc, int64_t f, const void *H,
+                                       const void *W2, const void *X, const void *We1,
+                                       const void *We2, void *B, float *P_save, void *F_out,
+                                       void *ws, size_t ws_bytes, void *stream);
+
 /* ---- utilities on the bottleneck weights (outside the boundary op) ----------------------------
  * Two dense kernels on a bf16 matrix, for training the bottleneck weights with Muon (Sec. 3.4.2:
  * the bottleneck models are trained with Muon, whose update orthogonalises the gradient momentum

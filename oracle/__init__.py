@@ -13,6 +13,8 @@ Citations (sections and equations of the ResBM paper):
   decode_bwd / encode_bwd .... the chain rule of the two forward functions
   effective_rank ............. the appendix's spectral analysis of the bottleneck output
                                projections: r_eff = sum_i sigma_i^2 / max_i sigma_i^2
+  ffn_down_encode_fwd ........ Sec. 3.2's bottleneck after the feed-forward layer: the encoder on
+                               the FFN's output z = H . W2 (stored in bf16 by the FFN)
   newton_schulz .............. Muon's orthogonalisation of the gradient momentum (Sec. 3.4.2
                                trains the bottleneck weights with Muon): X_0 = G / ||G||_F, then
                                X <- a X + b (X X^T) X + c (X X^T)^2 X on the wide orientation,
@@ -329,3 +331,12 @@ def newton_schulz(G, steps=5, coeffs=NS_COEFFS, eps=1e-7):
         B = b * A + c * (A @ A)
         X = a * X + B @ X
     return X.T if tall else X
+
+
+def ffn_down_encode_fwd(H, W2, X, We1, We2, act="silu"):
+    """The encoder applied after the feed-forward layer (Sec. 3.2: the bottleneck follows the FFN;
+    its input z is the FFN's output): F = H . W2 (numpy's matmul, float64) rounded to bf16 as the
+    FFN's output tensor, then (B, P) = encode_fwd(X, F, We1, We2). Returns (B, P, F)."""
+    F = default().round_to(np.asarray(H, np.float64) @ np.asarray(W2, np.float64), "bf16")
+    B, P = default().encode_fwd(X, F, We1, We2, act)
+    return B, P, F

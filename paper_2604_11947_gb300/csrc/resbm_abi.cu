@@ -714,6 +714,43 @@ resbm_status resbm_boundary_step(const resbm_desc *desc, const resbm_step_args *
     return s == RESBM_OK ? enqueue_step(d, *a, ws, c, nullptr, nullptr) : s;
 }
 
+resbm_status resbm_ffn_down_encode_workspace_bytes(const resbm_desc *desc, int64_t f, size_t *bytes)
+{
+    resbm_status s = check_desc(desc);
+    if (s != RESBM_OK) return s;
+    if (!bytes || f < 1) return RESBM_ERR_INVALID_ARG;
+    if (!ffn_encode_supported(*desc, f)) return RESBM_ERR_UNSUPPORTED;
+    *bytes = ffn_encode_ws_bytes(*desc, f);
+    return RESBM_OK;
+}
+
+resbm_status resbm_ffn_down_encode_fwd(const resbm_desc *desc, int64_t f, const void *H, const void *W2, const void *X,
+                                       const void *We1, const void *We2, void *B, float *P_save, void *F_out,
+                                       void *ws, size_t ws_bytes, void *stream)
+{
+    resbm_status s = check_desc(desc);
+    if (s != RESBM_OK) return s;
+    const resbm_desc &d = *desc;
+    if (f < 1 || !mul_ok(d.T, f) || !mul_ok(f, d.d)) return RESBM_ERR_INVALID_ARG;
+    if (!ffn_encode_supported(d, f)) return RESBM_ERR_UNSUPPORTED;
+    const bool t = d.T > 0;
+    if (!ptr_ok(H, 2, t) || !ptr_ok(W2, 2, true) || !ptr_ok(X, 2, t) || !ptr_ok(We1, 2, true) ||
+        !ptr_ok(We2, 2, true) || !ptr_ok(B, 2, t) || !ptr_ok(P_save, 4, false) || !ptr_ok(F_out, 2, false))
+        return RESBM_ERR_INVALID_ARG;
+    const Range outs[] = {rng(B, d.T * d.r, 2), rng(P_save, d.T * d.m, 4), rng(F_out, d.T * d.d, 2)};
+    const Range ins[] = {rng(H, d.T * f, 2), rng(W2, f * d.d, 2), rng(X, d.T * d.d, 2), rng(We1, d.d * d.m, 2),
+                         rng(We2, d.m * d.r, 2)};
+    if (any_overlap(outs, ins, 5)) return RESBM_ERR_INVALID_ARG;
+    const size_t need = ffn_encode_ws_bytes(d, f);
+    if (!ws || ws_bytes < need) return RESBM_ERR_WORKSPACE;
+    if (reinterpret_cast<uintptr_t>(ws) % 256) return RESBM_ERR_INVALID_ARG;
+    Ctx c;
+    s = make_ctx(stream, &c);
+    if (s != RESBM_OK || d.T == 0) return s;
+    const cudaError_t e = tc_ffn_down_encode(d, f, H, W2, X, We1, We2, B, P_save, F_out, ws, c);
+    return e == cudaErrorNotSupported ? RESBM_ERR_UNSUPPORTED : finish(e);
+}
+
 resbm_status resbm_matrix_workspace_bytes(int op, int64_t rows, int64_t cols, size_t *bytes)
 {
     if (!bytes || (op != RESBM_OP_EFFECTIVE_RANK && op != RESBM_OP_NEWTON_SCHULZ)) return RESBM_ERR_INVALID_ARG;

@@ -444,19 +444,42 @@ int gemm_splits(int64_t M, int64_t N, int64_t K, int sms)
     return (int)((K + kc - 1) / kc);
 }
 
-template <int BN, bool AMN, bool BMN, bool ALO>
+// MC: CTA pairs sharing B by multicast (k_gemm); the grid is then two CTAs per co-resident pair,
+// at most one pair per pair unit (returns cudaErrorNotSupported, before launching, when no pair
+// fits: the caller runs single CTAs).
+template <int BN, bool AMN, bool BMN, bool ALO, bool ENCP = false, bool MC = false>
 cudaError_t launch_gemm_t(const CUtensorMap &ma, const CUtensorMap &malo, const CUtensorMap &mb,
                           const tc::GemmShape &g, const tc::GemmEp &ep, const Ctx &c)
 {
     using Cfg = tc::GemmCfg<BN, ALO>;
     static std::atomic<uint8_t> smem_set[kMaxDev];
-    cudaError_t e = ensure_smem(tc::k_gemm<BN, AMN, BMN, ALO>, Cfg::SMEM_BYTES, c.device, smem_set);
+    cudaError_t e = ensure_smem(tc::k_gemm<BN, AMN, BMN, ALO, ENCP, MC>, Cfg::SMEM_BYTES, c.device, smem_set);
     if (e != cudaSuccess) return e;
-    const int64_t grid = g.units < c.sm_count ? g.units : c.sm_count;
-    e = launch(tc::k_gemm<BN, AMN, BMN, ALO>, (unsigned)grid, Cfg::THREADS, Cfg::SMEM_BYTES, c.stream, ma, malo, mb,
-               g, ep);
+    if (MC) {
+        static std::atomic<int> fit[kMaxDev][2];
+        const int pairs_fit = coresident_clusters(tc::k_gemm<BN, AMN, BMN, ALO, ENCP, MC>, 2, Cfg::THREADS,
+                                                  Cfg::SMEM_BYTES, c.device, fit);
+        const int64_t pair_units = (int64_t)((g.nm + 1) / 2) * g.nn * g.splits;
+        const int64_t pairs = pair_units < pairs_fit ? pair_units : pairs_fit;
+        if (pairs < 1) return cudaErrorNotSupported;
+        e = launch_clustered(tc::k_gemm<BN, AMN, BMN, ALO, ENCP, MC>, (unsigned)(2 * pairs), Cfg::THREADS,
+                             Cfg::SMEM_BYTES, 2, c.stream, ma, malo, mb, g, ep);
+    } else {
+        const int64_t grid = g.units < c.sm_count ? g.units : c.sm_count;
+        e = launch(tc::k_gemm<BN, AMN, BMN, ALO, ENCP, MC>, (unsigned)grid, Cfg::THREADS, Cfg::SMEM_BYTES, c.stream, ma,
+                   malo, mb, g, ep);
+    }
     count_launches(1);
     return e;
+}
+
+// Pairs sharing B by multicast for the 256-column products with at least two row blocks, unless
+// RESBM_GEMM_MC=0 (read at every launch; a tuning and testing knob: both forms compute the same
+// bits, each output element summed in the same order by one CTA).
+bool gemm_pairs(int bn, int64_t M)
+{
+    const char *v = getenv("RESBM_GEMM_MC");
+    return bn == 256 && M > 128 && !(v && v[0] == '0' && v[1] == 0);
 }
 
 // splits: 1 for every product whose epilogue is not a plain fp32 store; with splits > 1 the
@@ -473,8 +496,10 @@ cudaError_t gemm(const Ctx &c, int64_t M, int64_t N, int64_t K, const void *A, b
     const bool okL = !A_lo ? true
                      : a_mn ? make_map(&malo, A_lo, M, K, M * 2, 64, 64, CU_TENSOR_MAP_SWIZZLE_128B)
                             : make_map(&malo, A_lo, K, M, K * 2, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B);
+    const bool pair = gemm_pairs(bn, M);
+    // K-major B: a pair's CTAs each load half of the B tile's rows
     const bool okB = b_mn ? make_map(&mbm, B, N, K, N * 2, 64, 64, CU_TENSOR_MAP_SWIZZLE_128B)
-                          : make_map(&mbm, B, K, N, K * 2, 64, (uint32_t)bn, CU_TENSOR_MAP_SWIZZLE_128B);
+                          : make_map(&mbm, B, K, N, K * 2, 64, (uint32_t)(pair ? bn / 2 : bn), CU_TENSOR_MAP_SWIZZLE_128B);
     if (!okA || !okL || !okB) return cudaErrorInvalidValue;
     if (!A_lo) malo = ma;   // not read
     tc::GemmShape g;
@@ -488,6 +513,19 @@ cudaError_t gemm(const Ctx &c, int64_t M, int64_t N, int64_t K, const void *A, b
     g.nn = (int)((N + bn - 1) / bn);
     g.units = (int64_t)g.nm * g.nn * g.splits;
     const bool lo = A_lo != nullptr;
+    if (pair) {
+        cudaError_t e = cudaErrorNotSupported;
+        if (!a_mn && b_mn) e = lo ? launch_gemm_t<256, false, true, true, false, true>(ma, malo, mbm, g, ep, c)
+                                  : launch_gemm_t<256, false, true, false, false, true>(ma, malo, mbm, g, ep, c);
+        else if (!a_mn && !b_mn) e = lo ? launch_gemm_t<256, false, false, true, false, true>(ma, malo, mbm, g, ep, c)
+                                        : launch_gemm_t<256, false, false, false, false, true>(ma, malo, mbm, g, ep, c);
+        else if (a_mn && b_mn) e = lo ? launch_gemm_t<256, true, true, true, false, true>(ma, malo, mbm, g, ep, c)
+                                      : launch_gemm_t<256, true, true, false, false, true>(ma, malo, mbm, g, ep, c);
+        if (e != cudaErrorNotSupported) return e;
+        // no pair fits: single CTAs need the whole-tile box for K-major B
+        if (!b_mn && !make_map(&mbm, B, K, N, K * 2, 64, (uint32_t)bn, CU_TENSOR_MAP_SWIZZLE_128B))
+            return cudaErrorInvalidValue;
+    }
     if (bn == 256) {
         if (!a_mn && b_mn) return lo ? launch_gemm_t<256, false, true, true>(ma, malo, mbm, g, ep, c)
                                      : launch_gemm_t<256, false, true, false>(ma, malo, mbm, g, ep, c);
@@ -791,6 +829,68 @@ cudaError_t gemm_encode_bwd(const resbm_desc &d, const void *dB, const void *F, 
     if (e == cudaSuccess) e = wgrad(c, d.m, d.r, d.T, w.A, dB, dWe2, w.slots2, &j2);
     if (e == cudaSuccess) e = reduce_jobs(j2, j1, c);
     return e;
+}
+
+// ---- the encoder fused into the FFN down-projection ---------------------------------------------
+namespace {
+int ffn_bn(int64_t d) { return d > 128 ? 256 : 128; }
+int64_t ffn_slots(const resbm_desc &d) { return 2 * ((d.d + ffn_bn(d.d) - 1) / ffn_bn(d.d)); }
+}  // namespace
+
+bool ffn_encode_supported(const resbm_desc &d, int64_t f)
+{
+    return d.dtype == RESBM_BF16 && !(d.flags & RESBM_FLAG_LINEAR) && d.m % 8 == 0 && d.m <= 32 && d.r <= 32 &&
+           d.d % 8 == 0 && f >= 1 && f % 8 == 0 && d.T <= INT32_MAX;
+}
+
+size_t ffn_encode_ws_bytes(const resbm_desc &d, int64_t f)
+{
+    (void)f;
+    WsCarver cv(nullptr);
+    cv.take<float>(ffn_slots(d) * d.T * d.m);
+    return cv.used;
+}
+
+cudaError_t tc_ffn_down_encode(const resbm_desc &d, int64_t f, const void *H, const void *W2, const void *X,
+                               const void *We1, const void *We2, void *B, float *P, void *F_out, void *ws,
+                               const Ctx &c)
+{
+    if (!al16(H) || !al16(W2) || !al16(We1) || !al16(ws) || (F_out && !al16(F_out)) || (P && !al16(P)) ||
+        encode_fn() == nullptr)
+        return cudaErrorNotSupported;
+    const int bn = ffn_bn(d.d);
+    CUtensorMap ma, mb;
+    if (!make_map(&ma, H, f, d.T, f * 2, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&mb, W2, d.d, f, d.d * 2, 64, 64, CU_TENSOR_MAP_SWIZZLE_128B))
+        return cudaErrorInvalidValue;
+    tc::GemmShape g;
+    g.M = d.T;
+    g.N = d.d;
+    g.K = f;
+    g.splits = 1;
+    g.kc = (f + 63) / 64 * 64;
+    g.nm = (int)((d.T + 127) / 128);
+    g.nn = (int)((d.d + bn - 1) / bn);
+    g.units = (int64_t)g.nm * g.nn;
+    tc::GemmEp e{};
+    e.out = F_out;
+    e.ldo = d.d;
+    e.we1 = static_cast<const __nv_bfloat16 *>(We1);
+    e.pslots = static_cast<float *>(ws);
+    e.slot_stride = d.T * d.m;
+    e.pm = (int)d.m;
+    cudaError_t err = cudaErrorNotSupported;
+    if (gemm_pairs(bn, d.T)) err = launch_gemm_t<256, false, true, false, true, true>(ma, ma, mb, g, e, c);
+    if (err == cudaErrorNotSupported)
+        err = bn == 256 ? launch_gemm_t<256, false, true, false, true>(ma, ma, mb, g, e, c)
+                        : launch_gemm_t<128, false, true, false, true>(ma, ma, mb, g, e, c);
+    if (err != cudaSuccess) return err;
+    err = launch(tc::k_enc_finish, (unsigned)((d.T + 127) / 128), 128, 0, c.stream, (const float *)ws,
+                 (int)ffn_slots(d), d.T * d.m, d.T, (int)d.m, (int)d.r, d.act, P,
+                 static_cast<const __nv_bfloat16 *>(We2), static_cast<const __nv_bfloat16 *>(X), d.d,
+                 static_cast<__nv_bfloat16 *>(B));
+    count_launches(1);
+    return err;
 }
 
 // ---- Muon's Newton-Schulz orthogonalisation and the effective rank ----------------------------

@@ -60,4 +60,13 @@ cudaError_t tc_newton_schulz(int64_t rows, int64_t cols, const void *G, bool g_f
 cudaError_t tc_effective_rank(int64_t rows, int64_t cols, const void *W, double *out, void *ws,
                               const Ctx &c);
 
+// The encoder fused into the FFN down-projection (tc_gemm.cuh, ENCP): F = H . W2 on the tensor
+// cores, P = F . We1 accumulated from the F tiles in the epilogue into per-tile partial slots, then
+// B = X[:, :r] + phi(P) . We2; F reaches memory only when F_out is set. bf16, m % 8 == 0, m, r <= 32.
+bool ffn_encode_supported(const resbm_desc &d, int64_t f);
+size_t ffn_encode_ws_bytes(const resbm_desc &d, int64_t f);
+cudaError_t tc_ffn_down_encode(const resbm_desc &d, int64_t f, const void *H, const void *W2, const void *X,
+                               const void *We1, const void *We2, void *B, float *P, void *F_out, void *ws,
+                               const Ctx &c);
+
 }  // namespace resbm

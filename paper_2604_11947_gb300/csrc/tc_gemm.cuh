@@ -36,6 +36,28 @@
 namespace resbm {
 namespace tc {
 
+// tma_load_2d multicast to the CTAs of the cluster in cta_mask: the box lands at the same
+// shared-memory offset in each of them and completes its bytes on the mbarrier at the same
+// offset in each (this GPU's own memory only).
+__device__ __forceinline__ void tma_load_2d_mc(uint32_t dst, const CUtensorMap *m, int32_t x, int32_t y, uint32_t bar,
+                                               uint16_t cta_mask)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster"
+        " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(m)), "r"(x), "r"(y), "r"(bar), "h"(cta_mask)
+        : "memory");
+}
+
+// mma_commit arriving on the mbarrier at the same offset in every CTA of the cluster in cta_mask.
+__device__ __forceinline__ void mma_commit_mc(uint32_t bar, uint16_t cta_mask)
+{
+    asm volatile(
+        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(bar),
+        "h"(cta_mask)
+        : "memory");
+}
+
 // The element-wise step after the product (acc = the fp32 accumulator of one output element at
 // row `row`, column `col`; phi and phi' as in common.cuh; every bf16 result rounded once to
 // nearest even).
@@ -66,7 +88,39 @@ struct GemmEp {
     int64_t split_stride;
     __nv_bfloat16 *lo;   // P_A, ACT, DACT: the remainder of the bf16 activation result (same pitch)
     float alpha, beta;   // AXPBY
+    // ENCP launches (the encoder fused into the FFN down-projection): F = acc rounded to bf16
+    // (stored at out if set), and the partial P_slice = F_tile . We1[cols of the tile] summed over
+    // a thread's BN / 2 columns, written to slot (nb * 2 + half) of pslots (slots T x pm fp32,
+    // slot_stride apart)
+    const __nv_bfloat16 *we1;   // d x pm
+    float *pslots;
+    int64_t slot_stride;
+    int pm;
 };
+
+// P partial of one row over 32 columns: pacc[j] += sum over c of f[c] * We1[col + c][j], j < m
+// (m a multiple of 8, at most 32); We1's rows are read through L1 (every lane of a warp reads the
+// same rows: broadcasts)
+__device__ __forceinline__ void enc_partial32(const __nv_bfloat16 *__restrict__ we1, int m, int64_t col,
+                                              const float (&f)[32], int nv, float (&pacc)[32])
+{
+#pragma unroll
+    for (int c = 0; c < 32; ++c) {   // fully unrolled: f is indexed by constants only
+        if (c >= nv) break;
+        const uint4 *w = reinterpret_cast<const uint4 *>(we1 + (col + c) * m);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            if (8 * q >= m) break;
+            const uint4 u = __ldg(w + q);
+            const uint32_t ww[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                pacc[8 * q + 2 * e] = fmaf(f[c], __uint_as_float(ww[e] << 16), pacc[8 * q + 2 * e]);
+                pacc[8 * q + 2 * e + 1] = fmaf(f[c], __uint_as_float(ww[e] & 0xFFFF0000u), pacc[8 * q + 2 * e + 1]);
+            }
+        }
+    }
+}
 
 struct GemmShape {
     int64_t M, N, K;
@@ -242,7 +296,14 @@ __device__ __forceinline__ void gemm_epilogue(const GemmEp &ep, int64_t row, int
 }
 
 // tma_lo: the lo matrix of A (same shape and layout as A; read only with ALO)
-template <int BN, bool AMN, bool BMN, bool ALO>
+// ENCP: the epilogue of the encoder fused into the FFN down-projection (the GemmEp ENCP fields)
+// instead of gemm_epilogue.
+// MC: CTA pairs (clusters of 2) take the row blocks 2p and 2p + 1 of the same column block and K
+// split; each CTA loads its own A tile and half of the B tile, multicast into both CTAs, so each
+// reads 2/3 of a stage's bytes from L2. A stage's `empty` barrier then takes an arrival from both
+// CTAs' MMA commits (multicast), so neither refills it before both have read it. (For K-major B
+// the tensor map's box is BN / 2 rows.)
+template <int BN, bool AMN, bool BMN, bool ALO, bool ENCP = false, bool MC = false>
 __global__ void __launch_bounds__(320, 1)
     k_gemm(const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tma_lo,
            const __grid_constant__ CUtensorMap tmb, const GemmShape g, const GemmEp ep)
@@ -262,11 +323,25 @@ __global__ void __launch_bounds__(320, 1)
         if (k1 > g.K) k1 = g.K;
         return (int)((k1 - k0 + 63) / 64);
     };
+    // this CTA's units: every gridDim.x-th from blockIdx.x, or for a pair every (gridDim.x / 2)-th
+    // pair unit from the cluster index, the row block 2 * (pair row block) + rank
+    const uint32_t crank = MC ? cluster_rank() : 0u;
+    const int64_t u_first = MC ? (int64_t)cluster_index() : (int64_t)blockIdx.x;
+    const int64_t u_step = MC ? (int64_t)(gridDim.x / 2) : (int64_t)gridDim.x;
+    GemmShape gp = g;
+    if (MC) {
+        gp.nm = (g.nm + 1) / 2;
+        gp.units = (int64_t)gp.nm * gp.nn * gp.splits;
+    }
+    auto unit_of = [&](int64_t u, int &mb, int &nb, int &ks) {
+        gemm_unit(gp, u, mb, nb, ks);
+        if (MC) mb = 2 * mb + (int)crank;   // past the last row block: loads read zeros, nothing is stored
+    };
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < C::NST; ++s) {
             mbar_init(smem_u32(&full[s]), 1);
-            mbar_init(smem_u32(&empty[s]), 1);
+            mbar_init(smem_u32(&empty[s]), MC ? 2 : 1);
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(smem_u32(&acc_full[i]), 1);
@@ -278,6 +353,7 @@ __global__ void __launch_bounds__(320, 1)
     if (warp == 1) tmem_alloc(smem_u32(&tmem_base_sh), C::TMEM_COLS);
     tc_fence_before();
     __syncthreads();
+    if (MC) cluster_sync();   // the peer's barriers exist before anything is multicast to them
     tc_fence_after();
     const uint32_t tmem = tmem_base_sh;
 
@@ -289,9 +365,9 @@ __global__ void __launch_bounds__(320, 1)
             tma_prefetch_desc(&tmb);
             uint32_t it = 0;
             bool ok = true;
-            for (int64_t u = blockIdx.x; u < g.units && ok; u += gridDim.x) {
+            for (int64_t u = u_first; u < gp.units && ok; u += u_step) {
                 int mb, nb, ks;
-                gemm_unit(g, u, mb, nb, ks);
+                unit_of(u, mb, nb, ks);
                 int64_t k0;
                 const int nk = k_steps(ks, k0);
                 for (int kb = 0; kb < nk; ++kb, ++it) {
@@ -315,7 +391,17 @@ __global__ void __launch_bounds__(320, 1)
                             tma_load_2d(adst + C::A_TILE + 8192, &tma_lo, mb * 128 + 64, kx, bar);
                         }
                     }
-                    if (!BMN) {
+                    if (MC) {   // this CTA's half of B, into both CTAs of the pair
+                        if (!BMN) {
+                            tma_load_2d_mc(bdst + crank * (BN / 2) * 128, &tmb, kx, nb * BN + (int)crank * (BN / 2), bar, 3);
+                        } else {
+#pragma unroll
+                            for (int j = 0; j < BN / 128; ++j) {
+                                const int jj = (int)crank * (BN / 128) + j;
+                                tma_load_2d_mc(bdst + jj * 8192, &tmb, nb * BN + 64 * jj, kx, bar, 3);
+                            }
+                        }
+                    } else if (!BMN) {
                         tma_load_2d(bdst, &tmb, kx, nb * BN, bar);
                     } else {
 #pragma unroll
@@ -323,11 +409,14 @@ __global__ void __launch_bounds__(320, 1)
                     }
                 }
             }
-            // drain the loads still in flight before the CTA may exit
+            // drain the loads still in flight before the CTA may exit (for a pair this includes the
+            // peer's multicast halves), and for a pair the last MMA commits of both CTAs on this
+            // CTA's stage barriers
             const uint32_t n = it < (uint32_t)C::NST ? it : (uint32_t)C::NST;
             for (uint32_t k = 0; k < n; ++k) {
                 const uint32_t j = it - 1 - k;
                 mbar_wait(smem_u32(&full[j % C::NST]), (j / C::NST) & 1);
+                if (MC && ok) mbar_wait(smem_u32(&empty[j % C::NST]), (j / C::NST) & 1);
             }
         }
     } else if (warp == 1) {
@@ -345,9 +434,9 @@ __global__ void __launch_bounds__(320, 1)
             constexpr uint64_t BK = BMN ? (2048 >> 4) : (32 >> 4);
             uint32_t it = 0, ti = 0;
             bool ok = true;
-            for (int64_t u = blockIdx.x; u < g.units && ok; u += gridDim.x, ++ti) {
+            for (int64_t u = u_first; u < gp.units && ok; u += u_step, ++ti) {
                 int mb, nb, ks;
-                gemm_unit(g, u, mb, nb, ks);
+                unit_of(u, mb, nb, ks);
                 int64_t k0;
                 const int nk = k_steps(ks, k0);
                 const uint32_t ab = ti & 1;
@@ -366,7 +455,11 @@ __global__ void __launch_bounds__(320, 1)
                         mma_bf16(d_tmem, ad0 + so + kk * AK, bd0 + so + kk * BK, idesc, kb > 0 || kk > 0);
                         if (ALO) mma_bf16(d_tmem, ad0 + so + (C::A_TILE >> 4) + kk * AK, bd0 + so + kk * BK, idesc, true);
                     }
-                    mma_commit(smem_u32(&empty[s]));   // the stage is free once these MMAs are done
+                    // the stage is free once these MMAs are done (for a pair: once both CTAs' are)
+                    if (MC)
+                        mma_commit_mc(smem_u32(&empty[s]), 3);
+                    else
+                        mma_commit(smem_u32(&empty[s]));
                 }
                 if (!ok) break;
                 mma_commit(smem_u32(&acc_full[ab]));
@@ -382,14 +475,19 @@ __global__ void __launch_bounds__(320, 1)
         const uint32_t lane_base = (uint32_t)(q * 32) << 16;
         uint32_t ti = 0;
         bool ok = true;
-        for (int64_t u = blockIdx.x; u < g.units && ok; u += gridDim.x, ++ti) {
+        for (int64_t u = u_first; u < gp.units && ok; u += u_step, ++ti) {
             int mb, nb, ks;
-            gemm_unit(g, u, mb, nb, ks);
+            unit_of(u, mb, nb, ks);
             const uint32_t ab = ti & 1;
             ok = mbar_wait(smem_u32(&acc_full[ab]), (ti >> 1) & 1);
             tc_fence_after();
             if (!ok) break;
             const int64_t row = (int64_t)mb * 128 + rin;
+            float pacc[32];
+            if (ENCP) {
+#pragma unroll
+                for (int j = 0; j < 32; ++j) pacc[j] = 0.0f;
+            }
 #pragma unroll 1
             for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 32) {
                 float v[32];
@@ -399,11 +497,27 @@ __global__ void __launch_bounds__(320, 1)
                 const int64_t col = (int64_t)nb * BN + c;
                 if (col < g.N && row < g.M) {
                     const int nv = g.N - col < 32 ? (int)(g.N - col) : 32;
-                    gemm_epilogue(ep, row, col, v, nv, ks);
+                    if (ENCP) {
+                        // F as the FFN's bf16 output, then its share of P = F . We1
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) v[j] = __bfloat162float(__float2bfloat16_rn(v[j]));
+                        if (ep.out) st_bf16x32(static_cast<__nv_bfloat16 *>(ep.out) + row * ep.ldo + col, v, nv);
+                        enc_partial32(ep.we1, ep.pm, col, v, nv, pacc);
+                    } else {
+                        gemm_epilogue(ep, row, col, v, nv, ks);
+                    }
                 }
             }
             tc_fence_before();
             mbar_arrive(smem_u32(&acc_empty[ab]));   // this accumulator may be overwritten
+            if (ENCP && row < g.M) {
+                float *dst = ep.pslots + (int64_t)(nb * 2 + half) * ep.slot_stride + row * ep.pm;
+#pragma unroll
+                for (int q = 0; q < 8; ++q)
+                    if (4 * q < ep.pm)
+                        reinterpret_cast<float4 *>(dst)[q] =
+                            make_float4(pacc[4 * q], pacc[4 * q + 1], pacc[4 * q + 2], pacc[4 * q + 3]);
+            }
         }
     }
     tc_fence_before();
@@ -412,6 +526,53 @@ __global__ void __launch_bounds__(320, 1)
         tc_fence_after();
         tmem_dealloc(tmem, C::TMEM_COLS);
     }
+    if (MC) cluster_sync();   // neither CTA of a pair leaves while the other may still address it
+}
+
+// The encoder's end after the fused down-projection, one token row per thread: P = the sum of the
+// row's nslots partial slots in slot order (fp32), saved if P is set; A = phi(P) (fp32);
+// E = A . We2 (m x r, fp32); B = X[:, :r] + E rounded to bf16. m, r <= 32.
+__global__ void __launch_bounds__(128) k_enc_finish(const float *__restrict__ pslots, int nslots, int64_t slot_stride,
+                                                    int64_t T, int m, int r, int act, float *__restrict__ P,
+                                                    const __nv_bfloat16 *__restrict__ We2,
+                                                    const __nv_bfloat16 *__restrict__ X, int64_t ldx,
+                                                    __nv_bfloat16 *__restrict__ B)
+{
+    griddep_wait();
+    griddep_launch_dependents();
+    const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+    if (t >= T) return;
+    float p[32];
+#pragma unroll
+    for (int j = 0; j < 32; ++j) p[j] = 0.0f;
+    for (int s = 0; s < nslots; ++s) {
+        const float4 *src = reinterpret_cast<const float4 *>(pslots + s * slot_stride + t * m);
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+            if (4 * q >= m) break;
+            const float4 x = src[q];
+            p[4 * q] += x.x; p[4 * q + 1] += x.y; p[4 * q + 2] += x.z; p[4 * q + 3] += x.w;
+        }
+    }
+    if (P) {
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+            if (j < m) P[t * m + j] = p[j];
+    }
+    act_row<32>(act, p);
+    float e[32];
+#pragma unroll
+    for (int n = 0; n < 32; ++n) e[n] = 0.0f;
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {   // constant indices into the register arrays
+        if (j >= m) break;
+#pragma unroll
+        for (int n = 0; n < 32; ++n)
+            if (n < r) e[n] = fmaf(p[j], __bfloat162float(We2[j * r + n]), e[n]);
+    }
+#pragma unroll
+    for (int n = 0; n < 32; ++n)
+        if (n < r) B[t * r + n] = __float2bfloat16_rn(__bfloat162float(X[t * ldx + n]) + e[n]);
 }
 
 }  // namespace tc

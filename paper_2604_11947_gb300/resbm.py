@@ -33,7 +33,8 @@ EXPORTS = ("resbm_version", "resbm_status_string", "resbm_last_cuda_error", "res
            "resbm_workspace_bytes", "resbm_encode_fwd", "resbm_decode_fwd", "resbm_decode_bwd",
            "resbm_encode_bwd", "resbm_boundary_step", "resbm_boundary_step_host",
            "resbm_decode_bwd_noalloc", "resbm_selftest_wait_timeout", "resbm_matrix_workspace_bytes",
-           "resbm_newton_schulz", "resbm_effective_rank")
+           "resbm_newton_schulz", "resbm_effective_rank", "resbm_ffn_down_encode_workspace_bytes",
+           "resbm_ffn_down_encode_fwd")
 
 
 class resbm_desc(ctypes.Structure):
@@ -108,6 +109,10 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.resbm_newton_schulz.argtypes = [i64, i64, vp, ctypes.c_int32, ctypes.c_int32, vp, vp, sz, vp]
     lib.resbm_effective_rank.restype = i32
     lib.resbm_effective_rank.argtypes = [i64, i64, vp, vp, vp, sz, vp]
+    lib.resbm_ffn_down_encode_workspace_bytes.restype = i32
+    lib.resbm_ffn_down_encode_workspace_bytes.argtypes = [D, i64, ctypes.POINTER(sz)]
+    lib.resbm_ffn_down_encode_fwd.restype = i32
+    lib.resbm_ffn_down_encode_fwd.argtypes = [D, i64] + [vp] * 8 + [vp, sz, vp]
     if path is None:
         _lib = lib
     return lib
@@ -278,3 +283,24 @@ def resbm_effective_rank(W, out, ws, stream=None):
     rows, cols = W.shape
     _check("resbm_effective_rank", load().resbm_effective_rank(rows, cols, _p(W), _p(out), _p(ws), _nbytes(ws),
                                                                _stream(stream)))
+
+
+# ---- the encoder fused into the FFN down-projection ------------------------------------------
+def resbm_ffn_down_encode_workspace_bytes(desc: resbm_desc, f: int) -> int:
+    out = ctypes.c_size_t(0)
+    _check("resbm_ffn_down_encode_workspace_bytes",
+           load().resbm_ffn_down_encode_workspace_bytes(ctypes.byref(desc), int(f), ctypes.byref(out)))
+    return int(out.value)
+
+
+def ffn_down_encode_workspace(desc: resbm_desc, f: int, device="cuda") -> torch.Tensor:
+    return torch.empty(max(resbm_ffn_down_encode_workspace_bytes(desc, f), 1), dtype=torch.uint8, device=device)
+
+
+def resbm_ffn_down_encode_fwd(desc, H, W2, X, We1, We2, B, P_save, F_out, ws, stream=None):
+    """B (and P_save, F_out if given) from the FFN hidden state H (T x f) and the down-projection
+    W2 (f x d): the encoder applied to F = H . W2 without storing F unless F_out is given."""
+    f = H.shape[1]
+    st = load().resbm_ffn_down_encode_fwd(ctypes.byref(desc), int(f), _p(H), _p(W2), _p(X), _p(We1), _p(We2),
+                                          _p(B), _p(P_save), _p(F_out), _p(ws), _nbytes(ws), _stream(stream))
+    _check("resbm_ffn_down_encode_fwd", st)

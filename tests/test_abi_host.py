@@ -24,7 +24,7 @@ def declared_functions():
 
 def test_exports_every_declared_symbol(lib):
     names = declared_functions()
-    assert len(names) == 17, names
+    assert len(names) == 19, names
     assert sorted(resbm.EXPORTS) == names
     for n in names:
         assert hasattr(lib, n), n
@@ -191,3 +191,21 @@ def test_matrix_utilities_reject_bad_arguments(lib):
     assert er(4096, 32, G, X, ws, 16, None) == resbm.RESBM_ERR_WORKSPACE
     assert er(8192, 8192, G, X, ws, 1 << 34, None) == resbm.RESBM_ERR_INVALID_ARG               # min side > 4096
     assert er(4096, 32, G, X + 4, ws, 1 << 30, None) == resbm.RESBM_ERR_INVALID_ARG              # out not 8-byte aligned
+
+
+def test_ffn_down_encode_rejects_bad_arguments(lib):
+    """The fused down-projection encoder's host checks (fake aligned device addresses), through
+    the Python binding's argument list."""
+    A, big = 1 << 40, 1 << 32
+    t = [A + i * big for i in range(9)]
+    d = resbm.make_desc(1024, 512, 32, 32)
+    sz = ctypes.c_size_t(0)
+    assert lib.resbm_ffn_down_encode_workspace_bytes(ctypes.byref(d), 1024, ctypes.byref(sz)) == resbm.RESBM_OK
+    fn = lib.resbm_ffn_down_encode_fwd
+    assert fn(ctypes.byref(d), 1024, *t[:8], t[8], 16, None) == resbm.RESBM_ERR_WORKSPACE
+    assert fn(ctypes.byref(d), 1024, None, *t[1:8], t[8], sz.value, None) == resbm.RESBM_ERR_INVALID_ARG
+    assert fn(ctypes.byref(d), 1024, t[0], t[1], t[2], t[3], t[4], t[2], None, None, t[8], sz.value,
+              None) == resbm.RESBM_ERR_INVALID_ARG                         # B overlaps X
+    wide = resbm.make_desc(1024, 512, 64, 64)                             # m > 32: not this kernel
+    assert lib.resbm_ffn_down_encode_workspace_bytes(ctypes.byref(wide), 1024, ctypes.byref(sz)) == \
+        resbm.RESBM_ERR_UNSUPPORTED
