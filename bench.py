@@ -47,6 +47,9 @@ def parse():
     p.add_argument("--no-cpu", action="store_true", help="skip the oracle CPU baseline")
     p.add_argument("--no-extra", action="store_true",
                    help="skip the other workloads (T=16384 d=2048 r=16 and the d=8192 r-sweep)")
+    p.add_argument("--ffn-only", action="store_true",
+                   help="run only the FFN down-projection + encoder comparison (for profiler captures; "
+                        "--steps / --warmup apply); prints its JSON object, not a bench line")
     return p.parse_args()
 
 
@@ -497,6 +500,10 @@ def main():
     build.build()
     resbm.load()
 
+    if args.ffn_only:
+        print(json.dumps(ffn_encode_workload(resbm, torch, steps=max(args.steps, 1), warmup=max(args.warmup, 0))),
+              flush=True)
+        return
     flags = resbm.RESBM_FLAG_GENERIC if args.generic else 0
     peaks = measured_peaks()
     dev = device_inputs(cfg, torch)

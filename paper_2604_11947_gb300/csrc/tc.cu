@@ -885,7 +885,7 @@ cudaError_t tc_ffn_down_encode(const resbm_desc &d, int64_t f, const void *H, co
         err = bn == 256 ? launch_gemm_t<256, false, true, false, true>(ma, ma, mb, g, e, c)
                         : launch_gemm_t<128, false, true, false, true>(ma, ma, mb, g, e, c);
     if (err != cudaSuccess) return err;
-    err = launch(tc::k_enc_finish, (unsigned)((d.T + 127) / 128), 128, 0, c.stream, (const float *)ws,
+    err = launch(tc::k_enc_finish, (unsigned)((d.T + 7) / 8), 256, 0, c.stream, (const float *)ws,
                  (int)ffn_slots(d), d.T * d.m, d.T, (int)d.m, (int)d.r, d.act, P,
                  static_cast<const __nv_bfloat16 *>(We2), static_cast<const __nv_bfloat16 *>(X), d.d,
                  static_cast<__nv_bfloat16 *>(B));

@@ -529,10 +529,12 @@ __global__ void __launch_bounds__(320, 1)
     if (MC) cluster_sync();   // neither CTA of a pair leaves while the other may still address it
 }
 
-// The encoder's end after the fused down-projection, one token row per thread: P = the sum of the
-// row's nslots partial slots in slot order (fp32), saved if P is set; A = phi(P) (fp32);
-// E = A . We2 (m x r, fp32); B = X[:, :r] + E rounded to bf16. m, r <= 32.
-__global__ void __launch_bounds__(128) k_enc_finish(const float *__restrict__ pslots, int nslots, int64_t slot_stride,
+// The encoder's end after the fused down-projection, one token row per warp: lane j < m sums
+// column j of the row's nslots partial slots in slot order (fp32; the lanes read the slots'
+// rows coalesced), saves P if asked, and takes A_j = phi(P_j); lane n < r then forms
+// E_n = sum over j of A_j . We2[j][n] (the A_j from lane j by shuffles, j in order) and stores
+// B = X[:, :r] + E rounded to bf16. m, r <= 32.
+__global__ void __launch_bounds__(256) k_enc_finish(const float *__restrict__ pslots, int nslots, int64_t slot_stride,
                                                     int64_t T, int m, int r, int act, float *__restrict__ P,
                                                     const __nv_bfloat16 *__restrict__ We2,
                                                     const __nv_bfloat16 *__restrict__ X, int64_t ldx,
@@ -540,39 +542,22 @@ __global__ void __launch_bounds__(128) k_enc_finish(const float *__restrict__ ps
 {
     griddep_wait();
     griddep_launch_dependents();
-    const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-    if (t >= T) return;
-    float p[32];
-#pragma unroll
-    for (int j = 0; j < 32; ++j) p[j] = 0.0f;
-    for (int s = 0; s < nslots; ++s) {
-        const float4 *src = reinterpret_cast<const float4 *>(pslots + s * slot_stride + t * m);
-#pragma unroll
-        for (int q = 0; q < 8; ++q) {
-            if (4 * q >= m) break;
-            const float4 x = src[q];
-            p[4 * q] += x.x; p[4 * q + 1] += x.y; p[4 * q + 2] += x.z; p[4 * q + 3] += x.w;
-        }
+    const int lane = threadIdx.x & 31;
+    const int64_t t = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+    if (t >= T) return;   // whole warps
+    float p = 0.0f;
+    if (lane < m) {
+        const float *src = pslots + t * m + lane;
+        for (int s = 0; s < nslots; ++s) p += src[s * slot_stride];
+        if (P) P[t * m + lane] = p;
     }
-    if (P) {
-#pragma unroll
-        for (int j = 0; j < 32; ++j)
-            if (j < m) P[t * m + j] = p[j];
+    const float a = lane < m ? act_f(act, p) : 0.0f;
+    float e = 0.0f;
+    for (int j = 0; j < m; ++j) {
+        const float aj = __shfl_sync(0xffffffffu, a, j);
+        if (lane < r) e = fmaf(aj, __bfloat162float(We2[j * r + lane]), e);
     }
-    act_row<32>(act, p);
-    float e[32];
-#pragma unroll
-    for (int n = 0; n < 32; ++n) e[n] = 0.0f;
-#pragma unroll
-    for (int j = 0; j < 32; ++j) {   // constant indices into the register arrays
-        if (j >= m) break;
-#pragma unroll
-        for (int n = 0; n < 32; ++n)
-            if (n < r) e[n] = fmaf(p[j], __bfloat162float(We2[j * r + n]), e[n]);
-    }
-#pragma unroll
-    for (int n = 0; n < 32; ++n)
-        if (n < r) B[t * r + n] = __float2bfloat16_rn(__bfloat162float(X[t * ldx + n]) + e[n]);
+    if (lane < r) B[t * r + lane] = __float2bfloat16_rn(__bfloat162float(X[t * ldx + lane]) + e);
 }
 
 }  // namespace tc
