@@ -49,6 +49,9 @@ SMALL = {
     # of 8 (d = 776 = 3 x 256 + 8 leaves an 8-column output block and a 8-deep K tail; r = 24 and
     # m = 40 a partial 32-column epilogue chunk)
     "bf16_r512": synth.BoundaryConfig("bf16_r512", T=700, d=1024, r=512, m=512),
+    # nine 128-row blocks: the GEMM's CTA pairs (B shared by multicast) end with a partner whose
+    # row block lies past T (it loads zeros and stores nothing)
+    "bf16_r512_odd_blocks": synth.BoundaryConfig("bf16_r512_odd_blocks", T=1100, d=1024, r=512, m=512),
     "bf16_r24_m40": synth.BoundaryConfig("bf16_r24_m40", T=999, d=776, r=24, m=40),
 }
 
