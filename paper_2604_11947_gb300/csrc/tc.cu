@@ -428,15 +428,36 @@ cudaError_t launch_enc_bwd(const resbm_desc &d, const void *dB, const void *F, c
 // K x N row-major, else N x K), all bf16 with row pitches equal to the stored widths.
 int gemm_bn(int64_t N) { return N > 128 ? 256 : 128; }
 
+// 256-row units (two 128-row MMAs sharing each B tile, GemmCfg's BM2) for 256-column products
+// without a lo half, where A is K-major (measured on GB300 at d = 8192, T = 32768, m = 512:
+// P = F . We1 and dQ = dY . Wd2^T 6 % and 3 % faster; the MN-major weight gradient dWe1 = F^T dP
+// 6 % slower), K (per split, for a weight gradient that may split it: wg) is long enough that a
+// unit's epilogue, no longer overlapped with the next unit's products, is short next to them,
+// and the 256-row units still give every SM one. RESBM_GEMM_BM2 (read at every call; a tuning
+// and testing knob): 0 never, 1 wherever the shape allows (either major). Both forms sum each
+// output element over K in the same order; a weight gradient's split count can differ.
+bool gemm_bm2(int64_t M, int64_t N, int64_t K, bool lo, bool a_mn, int sms, bool wg)
+{
+    if (gemm_bn(N) != 256 || lo) return false;
+    const char *v = getenv("RESBM_GEMM_BM2");
+    if (v && (v[0] == '0' || v[0] == '1') && v[1] == 0) return v[0] == '1';
+    if (a_mn || M <= 256 || K < 2048) return false;
+    int64_t units = ((M + 255) / 256) * ((N + 255) / 256);
+    if (wg) units *= K / 2048 < 32 ? K / 2048 : 32;
+    return units >= sms;
+}
+
 // Split-K of a product with few output tiles (the weight gradients, K = tokens): enough splits
-// to give every SM a unit, at most 32 and at least four 64-deep K slices per split.
-int gemm_splits(int64_t M, int64_t N, int64_t K, int sms)
+// to give every SM a unit, at most 32 and at least four 64-deep K slices per split. rows: the
+// unit's rows (256 where gemm_bm2 holds).
+int gemm_splits(int64_t M, int64_t N, int64_t K, int sms, int rows = 128)
 {
     const int bn = gemm_bn(N);
-    const int64_t units = ((M + 127) / 128) * ((N + bn - 1) / bn);
+    const int64_t units = ((M + rows - 1) / rows) * ((N + bn - 1) / bn);
     if (4 * units >= 3 * (int64_t)sms) return 1;
     int64_t s = sms / units;
-    const int64_t kmax = (K + 255) / 256;
+    // 256-row units keep 2048 K per split (their epilogue is not overlapped with the next unit)
+    const int64_t kmax = rows == 256 ? (K / 2048 > 1 ? K / 2048 : 1) : (K + 255) / 256;
     if (s > kmax) s = kmax;
     if (s > 32) s = 32;
     if (s < 1) s = 1;
@@ -447,28 +468,30 @@ int gemm_splits(int64_t M, int64_t N, int64_t K, int sms)
 // MC: CTA pairs sharing B by multicast (k_gemm); the grid is then two CTAs per co-resident pair,
 // at most one pair per pair unit (returns cudaErrorNotSupported, before launching, when no pair
 // fits: the caller runs single CTAs).
-template <int BN, bool AMN, bool BMN, bool ALO, bool ENCP = false, bool MC = false>
+template <int BN, bool AMN, bool BMN, bool ALO, bool ENCP = false, bool MC = false, bool BM2 = false>
 cudaError_t launch_gemm_t(const CUtensorMap &ma, const CUtensorMap &malo, const CUtensorMap &mb,
                           const tc::GemmShape &g, const tc::GemmEp &ep, const Ctx &c)
 {
-    using Cfg = tc::GemmCfg<BN, ALO>;
+    using Cfg = tc::GemmCfg<BN, ALO, BM2>;
+#define RESBM_KGEMM tc::k_gemm<BN, AMN, BMN, ALO, ENCP, MC, BM2>
     static std::atomic<uint8_t> smem_set[kMaxDev];
-    cudaError_t e = ensure_smem(tc::k_gemm<BN, AMN, BMN, ALO, ENCP, MC>, Cfg::SMEM_BYTES, c.device, smem_set);
+    cudaError_t e = ensure_smem(RESBM_KGEMM, Cfg::SMEM_BYTES, c.device, smem_set);
     if (e != cudaSuccess) return e;
     if (MC) {
         static std::atomic<int> fit[kMaxDev][2];
-        const int pairs_fit = coresident_clusters(tc::k_gemm<BN, AMN, BMN, ALO, ENCP, MC>, 2, Cfg::THREADS,
+        const int pairs_fit = coresident_clusters(RESBM_KGEMM, 2, Cfg::THREADS,
                                                   Cfg::SMEM_BYTES, c.device, fit);
         const int64_t pair_units = (int64_t)((g.nm + 1) / 2) * g.nn * g.splits;
         const int64_t pairs = pair_units < pairs_fit ? pair_units : pairs_fit;
         if (pairs < 1) return cudaErrorNotSupported;
-        e = launch_clustered(tc::k_gemm<BN, AMN, BMN, ALO, ENCP, MC>, (unsigned)(2 * pairs), Cfg::THREADS,
+        e = launch_clustered(RESBM_KGEMM, (unsigned)(2 * pairs), Cfg::THREADS,
                              Cfg::SMEM_BYTES, 2, c.stream, ma, malo, mb, g, ep);
     } else {
         const int64_t grid = g.units < c.sm_count ? g.units : c.sm_count;
-        e = launch(tc::k_gemm<BN, AMN, BMN, ALO, ENCP, MC>, (unsigned)grid, Cfg::THREADS, Cfg::SMEM_BYTES, c.stream, ma,
+        e = launch(RESBM_KGEMM, (unsigned)grid, Cfg::THREADS, Cfg::SMEM_BYTES, c.stream, ma,
                    malo, mb, g, ep);
     }
+#undef RESBM_KGEMM
     count_launches(1);
     return e;
 }
@@ -484,9 +507,10 @@ bool gemm_pairs(int bn, int64_t M)
 
 // splits: 1 for every product whose epilogue is not a plain fp32 store; with splits > 1 the
 // epilogue must be GEP_F32 into `splits` slots of M x N (ep.split_stride apart). A_lo: the lo
-// half of A as a bf16 hi + lo pair (same shape and layout as A), or null.
+// half of A as a bf16 hi + lo pair (same shape and layout as A), or null. rows: the unit's rows
+// as the caller chose them (128 or 256), or 0 to choose here.
 cudaError_t gemm(const Ctx &c, int64_t M, int64_t N, int64_t K, const void *A, bool a_mn, const void *B, bool b_mn,
-                 const tc::GemmEp &ep, int splits, const void *A_lo = nullptr)
+                 const tc::GemmEp &ep, int splits, const void *A_lo = nullptr, int rows = 0)
 {
     if (M <= 0 || N <= 0 || K <= 0) return cudaSuccess;
     const int bn = gemm_bn(N);
@@ -496,7 +520,9 @@ cudaError_t gemm(const Ctx &c, int64_t M, int64_t N, int64_t K, const void *A, b
     const bool okL = !A_lo ? true
                      : a_mn ? make_map(&malo, A_lo, M, K, M * 2, 64, 64, CU_TENSOR_MAP_SWIZZLE_128B)
                             : make_map(&malo, A_lo, K, M, K * 2, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B);
-    const bool pair = gemm_pairs(bn, M);
+    const bool lo = A_lo != nullptr;
+    const bool bm2 = !lo && bn == 256 && (rows ? rows == 256 : gemm_bm2(M, N, K, lo, a_mn, c.sm_count, false));
+    const bool pair = !bm2 && gemm_pairs(bn, M);
     // K-major B: a pair's CTAs each load half of the B tile's rows
     const bool okB = b_mn ? make_map(&mbm, B, N, K, N * 2, 64, 64, CU_TENSOR_MAP_SWIZZLE_128B)
                           : make_map(&mbm, B, K, N, K * 2, 64, (uint32_t)(pair ? bn / 2 : bn), CU_TENSOR_MAP_SWIZZLE_128B);
@@ -509,10 +535,15 @@ cudaError_t gemm(const Ctx &c, int64_t M, int64_t N, int64_t K, const void *A, b
     g.splits = splits < 1 ? 1 : splits;
     g.kc = ((K + g.splits - 1) / g.splits + 63) / 64 * 64;
     g.splits = (int)((K + g.kc - 1) / g.kc);
-    g.nm = (int)((M + 127) / 128);
+    g.nm = (int)(bm2 ? (M + 255) / 256 : (M + 127) / 128);
     g.nn = (int)((N + bn - 1) / bn);
     g.units = (int64_t)g.nm * g.nn * g.splits;
-    const bool lo = A_lo != nullptr;
+    if (bm2) {
+        if (!a_mn && b_mn) return launch_gemm_t<256, false, true, false, false, false, true>(ma, malo, mbm, g, ep, c);
+        if (!a_mn && !b_mn) return launch_gemm_t<256, false, false, false, false, false, true>(ma, malo, mbm, g, ep, c);
+        if (a_mn && b_mn) return launch_gemm_t<256, true, true, false, false, false, true>(ma, malo, mbm, g, ep, c);
+        return cudaErrorNotSupported;
+    }
     if (pair) {
         cudaError_t e = cudaErrorNotSupported;
         if (!a_mn && b_mn) e = lo ? launch_gemm_t<256, false, true, true, false, true>(ma, malo, mbm, g, ep, c)
@@ -562,12 +593,13 @@ tc::GemmEp ep_of(int mode, int act, void *out, int64_t ldo)
 cudaError_t wgrad(const Ctx &c, int64_t M, int64_t N, int64_t K, const void *A, const void *B, float *W, float *slots,
                   tc::ReduceJob *job, const void *A_lo = nullptr, bool a_mn = true, bool b_mn = true)
 {
-    const int s = gemm_splits(M, N, K, c.sm_count);
+    const int rows = gemm_bm2(M, N, K, A_lo != nullptr, a_mn, c.sm_count, true) ? 256 : 128;
+    const int s = gemm_splits(M, N, K, c.sm_count, rows);
     *job = tc::ReduceJob{nullptr, 0, 0, 0, nullptr, 0, 0, 0};
-    if (s <= 1) return gemm(c, M, N, K, A, a_mn, B, b_mn, ep_of(tc::GEP_F32, 0, W, N), 1, A_lo);
+    if (s <= 1) return gemm(c, M, N, K, A, a_mn, B, b_mn, ep_of(tc::GEP_F32, 0, W, N), 1, A_lo, rows);
     tc::GemmEp e = ep_of(tc::GEP_F32, 0, slots, N);
     e.split_stride = M * N;
-    cudaError_t err = gemm(c, M, N, K, A, a_mn, B, b_mn, e, s, A_lo);
+    cudaError_t err = gemm(c, M, N, K, A, a_mn, B, b_mn, e, s, A_lo, rows);
     if (err != cudaSuccess) return err;
     // the number of splits the launch took (gemm rounds K per split to 64)
     const int64_t kc = ((K + s - 1) / s + 63) / 64 * 64;
@@ -604,7 +636,9 @@ constexpr int64_t kDfLoMaxM = 64;
 
 size_t slot_floats(int64_t M, int64_t N, int64_t K, int sms)
 {
-    const int s = gemm_splits(M, N, K, sms);
+    // room for either unit size (which one a launch takes can depend on RESBM_GEMM_BM2)
+    const int s1 = gemm_splits(M, N, K, sms, 128), s2 = gemm_splits(M, N, K, sms, 256);
+    const int s = s1 > s2 ? s1 : s2;
     return s > 1 ? (size_t)(s * M * N) : 0;
 }
 
@@ -880,6 +914,8 @@ cudaError_t tc_ffn_down_encode(const resbm_desc &d, int64_t f, const void *H, co
     e.slot_stride = d.T * d.m;
     e.pm = (int)d.m;
     cudaError_t err = cudaErrorNotSupported;
+    // (not in 256-row units: measured 0.31 -> 0.47 ms at T = 16384, f = 5632, d = 2048, the P
+    // partials' epilogue no longer hidden behind the next unit's products)
     if (gemm_pairs(bn, d.T)) err = launch_gemm_t<256, false, true, false, true, true>(ma, ma, mb, g, e, c);
     if (err == cudaErrorNotSupported)
         err = bn == 256 ? launch_gemm_t<256, false, true, false, true>(ma, ma, mb, g, e, c)

@@ -129,13 +129,15 @@ struct GemmShape {
     int64_t units;       // nm * nn * splits
 };
 
-template <int BN_, bool ALO_ = false> struct GemmCfg {
+// BM2: 256-row units, two 128-row A sub-tiles per stage against one B tile, the two halves'
+// accumulators side by side in TMEM (one unit at a time: no accumulator double buffering).
+template <int BN_, bool ALO_ = false, bool BM2_ = false> struct GemmCfg {
     static constexpr int BN = BN_;
     static constexpr uint32_t A_TILE = 128 * 64 * 2;        // 128 rows x 64 K, bf16
-    static constexpr uint32_t A_STAGE = A_TILE * (ALO_ ? 2 : 1);   // hi (+ lo)
+    static constexpr uint32_t A_STAGE = A_TILE * (ALO_ ? 2 : 1) * (BM2_ ? 2 : 1);   // hi (+ lo), per half
     static constexpr uint32_t B_STAGE = BN_ * 64 * 2;       // BN rows x 64 K, bf16
     static constexpr uint32_t STAGE = A_STAGE + B_STAGE;
-    static constexpr int NST = (200 * 1024) / STAGE;        // 4 stages at BN = 256, 6 at 128 (3, 4 with lo)
+    static constexpr int NST = (200 * 1024) / STAGE;        // 4 stages at BN = 256, 6 at 128 (3, 4 with lo; 3 for BM2)
     static constexpr uint32_t SMEM_BYTES = NST * STAGE + 1024;
     static_assert(SMEM_BYTES <= 232448 - 512, "shared memory budget");
     static constexpr uint32_t TMEM_COLS = 2 * BN_;          // two accumulators
@@ -298,17 +300,22 @@ __device__ __forceinline__ void gemm_epilogue(const GemmEp &ep, int64_t row, int
 // tma_lo: the lo matrix of A (same shape and layout as A; read only with ALO)
 // ENCP: the epilogue of the encoder fused into the FFN down-projection (the GemmEp ENCP fields)
 // instead of gemm_epilogue.
+// BM2 (GemmCfg): units of 256 rows (two 128-row MMAs per K step sharing the B tile, ~128 flop per
+// shared-memory byte against ~85), for long K where a unit's epilogue is short next to its
+// products; not with ALO or MC.
 // MC: CTA pairs (clusters of 2) take the row blocks 2p and 2p + 1 of the same column block and K
 // split; each CTA loads its own A tile and half of the B tile, multicast into both CTAs, so each
 // reads 2/3 of a stage's bytes from L2. A stage's `empty` barrier then takes an arrival from both
 // CTAs' MMA commits (multicast), so neither refills it before both have read it. (For K-major B
 // the tensor map's box is BN / 2 rows.)
-template <int BN, bool AMN, bool BMN, bool ALO, bool ENCP = false, bool MC = false>
+template <int BN, bool AMN, bool BMN, bool ALO, bool ENCP = false, bool MC = false, bool BM2 = false>
 __global__ void __launch_bounds__(320, 1)
     k_gemm(const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tma_lo,
            const __grid_constant__ CUtensorMap tmb, const GemmShape g, const GemmEp ep)
 {
-    using C = GemmCfg<BN, ALO>;
+    using C = GemmCfg<BN, ALO, BM2>;
+    static_assert(!(BM2 && (ALO || MC)), "256-row units without hi + lo A or pairs");
+    constexpr int MH = BM2 ? 2 : 1;   // 128-row halves per unit (g.nm counts units of 128 * MH rows)
     griddep_wait();               // the previous kernel of the stream has completed
     griddep_launch_dependents();  // the next one may be scheduled on SMs as they free up
     extern __shared__ uint8_t smem_raw[];
@@ -380,7 +387,18 @@ __global__ void __launch_bounds__(320, 1)
                     mbar_expect_tx(bar, C::STAGE);
                     const uint32_t adst = smem_u32(smem + s * C::STAGE), bdst = adst + C::A_STAGE;
                     const int32_t kx = (int32_t)(k0 + 64 * kb);
-                    if (!AMN) {
+                    if (BM2) {   // the unit's two 128-row A sub-tiles
+#pragma unroll
+                        for (int h = 0; h < 2; ++h) {
+                            const int32_t y = mb * 256 + 128 * h;
+                            if (!AMN) {
+                                tma_load_2d(adst + h * C::A_TILE, &tma, kx, y, bar);
+                            } else {
+                                tma_load_2d(adst + h * C::A_TILE, &tma, y, kx, bar);
+                                tma_load_2d(adst + h * C::A_TILE + 8192, &tma, y + 64, kx, bar);
+                            }
+                        }
+                    } else if (!AMN) {
                         tma_load_2d(adst, &tma, kx, mb * 128, bar);
                         if (ALO) tma_load_2d(adst + C::A_TILE, &tma_lo, kx, mb * 128, bar);
                     } else {
@@ -439,8 +457,10 @@ __global__ void __launch_bounds__(320, 1)
                 unit_of(u, mb, nb, ks);
                 int64_t k0;
                 const int nk = k_steps(ks, k0);
-                const uint32_t ab = ti & 1;
-                ok = mbar_wait(smem_u32(&acc_empty[ab]), ((ti >> 1) & 1) ^ 1);
+                // double-buffered accumulators; BM2: one pair of half accumulators, every unit
+                const uint32_t ab = BM2 ? 0u : (ti & 1);
+                const uint32_t eph = BM2 ? ((ti & 1) ^ 1) : (((ti >> 1) & 1) ^ 1);
+                ok = mbar_wait(smem_u32(&acc_empty[ab]), eph);
                 tc_fence_after();
                 if (!ok) break;
                 const uint32_t d_tmem = tmem + ab * BN;
@@ -454,6 +474,9 @@ __global__ void __launch_bounds__(320, 1)
                     for (int kk = 0; kk < 4; ++kk) {
                         mma_bf16(d_tmem, ad0 + so + kk * AK, bd0 + so + kk * BK, idesc, kb > 0 || kk > 0);
                         if (ALO) mma_bf16(d_tmem, ad0 + so + (C::A_TILE >> 4) + kk * AK, bd0 + so + kk * BK, idesc, true);
+                        if (BM2)   // the second 128-row half into the next BN columns
+                            mma_bf16(d_tmem + BN, ad0 + so + (C::A_TILE >> 4) + kk * AK, bd0 + so + kk * BK, idesc,
+                                     kb > 0 || kk > 0);
                     }
                     // the stage is free once these MMAs are done (for a pair: once both CTAs' are)
                     if (MC)
@@ -478,45 +501,51 @@ __global__ void __launch_bounds__(320, 1)
         for (int64_t u = u_first; u < gp.units && ok; u += u_step, ++ti) {
             int mb, nb, ks;
             unit_of(u, mb, nb, ks);
-            const uint32_t ab = ti & 1;
-            ok = mbar_wait(smem_u32(&acc_full[ab]), (ti >> 1) & 1);
+            const uint32_t ab = BM2 ? 0u : (ti & 1);
+            ok = mbar_wait(smem_u32(&acc_full[ab]), BM2 ? (ti & 1) : ((ti >> 1) & 1));
             tc_fence_after();
             if (!ok) break;
-            const int64_t row = (int64_t)mb * 128 + rin;
-            float pacc[32];
-            if (ENCP) {
-#pragma unroll
-                for (int j = 0; j < 32; ++j) pacc[j] = 0.0f;
-            }
 #pragma unroll 1
-            for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 32) {
-                float v[32];
-                tmem_ld32(tmem + lane_base + ab * BN + c, v);   // warp-collective: every lane
-                tmem_ld_wait();
-                tmem_regs_ready<32>(v);
-                const int64_t col = (int64_t)nb * BN + c;
-                if (col < g.N && row < g.M) {
-                    const int nv = g.N - col < 32 ? (int)(g.N - col) : 32;
-                    if (ENCP) {
-                        // F as the FFN's bf16 output, then its share of P = F . We1
+            for (int h = 0; h < MH; ++h) {   // the unit's 128-row halves (one unless BM2)
+                const int64_t row = (int64_t)mb * (128 * MH) + 128 * h + rin;
+                const uint32_t acc_col = (ab + (uint32_t)h) * BN;
+                float pacc[32];
+                if (ENCP) {
 #pragma unroll
-                        for (int j = 0; j < 32; ++j) v[j] = __bfloat162float(__float2bfloat16_rn(v[j]));
-                        if (ep.out) st_bf16x32(static_cast<__nv_bfloat16 *>(ep.out) + row * ep.ldo + col, v, nv);
-                        enc_partial32(ep.we1, ep.pm, col, v, nv, pacc);
-                    } else {
-                        gemm_epilogue(ep, row, col, v, nv, ks);
+                    for (int j = 0; j < 32; ++j) pacc[j] = 0.0f;
+                }
+#pragma unroll 1
+                for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 32) {
+                    float v[32];
+                    tmem_ld32(tmem + lane_base + acc_col + c, v);   // warp-collective: every lane
+                    tmem_ld_wait();
+                    tmem_regs_ready<32>(v);
+                    const int64_t col = (int64_t)nb * BN + c;
+                    if (col < g.N && row < g.M) {
+                        const int nv = g.N - col < 32 ? (int)(g.N - col) : 32;
+                        if (ENCP) {
+                            // F as the FFN's bf16 output, then its share of P = F . We1
+#pragma unroll
+                            for (int j = 0; j < 32; ++j) v[j] = __bfloat162float(__float2bfloat16_rn(v[j]));
+                            if (ep.out) st_bf16x32(static_cast<__nv_bfloat16 *>(ep.out) + row * ep.ldo + col, v, nv);
+                            enc_partial32(ep.we1, ep.pm, col, v, nv, pacc);
+                        } else {
+                            gemm_epilogue(ep, row, col, v, nv, ks);
+                        }
                     }
                 }
-            }
-            tc_fence_before();
-            mbar_arrive(smem_u32(&acc_empty[ab]));   // this accumulator may be overwritten
-            if (ENCP && row < g.M) {
-                float *dst = ep.pslots + (int64_t)(nb * 2 + half) * ep.slot_stride + row * ep.pm;
+                if (h == MH - 1) {
+                    tc_fence_before();
+                    mbar_arrive(smem_u32(&acc_empty[ab]));   // this accumulator may be overwritten
+                }
+                if (ENCP && row < g.M) {
+                    float *dst = ep.pslots + (int64_t)(nb * 2 + half) * ep.slot_stride + row * ep.pm;
 #pragma unroll
-                for (int q = 0; q < 8; ++q)
-                    if (4 * q < ep.pm)
-                        reinterpret_cast<float4 *>(dst)[q] =
-                            make_float4(pacc[4 * q], pacc[4 * q + 1], pacc[4 * q + 2], pacc[4 * q + 3]);
+                    for (int q = 0; q < 8; ++q)
+                        if (4 * q < ep.pm)
+                            reinterpret_cast<float4 *>(dst)[q] =
+                                make_float4(pacc[4 * q], pacc[4 * q + 1], pacc[4 * q + 2], pacc[4 * q + 3]);
+                }
             }
         }
     }

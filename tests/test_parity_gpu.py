@@ -53,6 +53,10 @@ SMALL = {
     # row block lies past T (it loads zeros and stores nothing)
     "bf16_r512_odd_blocks": synth.BoundaryConfig("bf16_r512_odd_blocks", T=1100, d=1024, r=512, m=512),
     "bf16_r24_m40": synth.BoundaryConfig("bf16_r24_m40", T=999, d=776, r=24, m=40),
+    # K = d = 2304 and K = T = 2300: the long-K products (P = F . We1, dQ = dY . Wd2^T and the
+    # weight gradients) where the GEMM may take 256-row units; m = 384 leaves a 128-column output
+    # block, T a 252-row last unit (its second half partly past T)
+    "bf16_r384_long_k": synth.BoundaryConfig("bf16_r384_long_k", T=2300, d=2304, r=384, m=384),
 }
 
 # Backward grids under each forced cluster size (RESBM_CLUSTER), one CTA per 128-token
@@ -115,6 +119,28 @@ def test_small_configs_match_oracle(name, path):
     _compare_all(cfg, got, want, dev, PATHS[path])
     # the saved pre-activation P = F . We1 is an fp32 output: fp32 accumulation error only
     check("P", to_host(got["P"]), want["P"], "f32", tol=1e-4)
+
+
+@pytest.mark.parametrize("bm2", ["0", "1"])
+@pytest.mark.parametrize("name", ["bf16_r384_long_k", "bf16_r512_odd_blocks", "bf16_r24_m40"])
+def test_gemm_row_units_match_oracle(name, bm2, monkeypatch):
+    """The GEMM chain with 256-row units forced wherever the shape allows them (RESBM_GEMM_BM2=1)
+    and with 128-row units only (=0): both against the oracle, and the forward outputs (single
+    products, no split over K) the same bits either way."""
+    cfg = SMALL[name]
+    h = host_inputs(cfg)
+    dev = {k: to_dev(v, cfg) for k, v in h.items()}
+    monkeypatch.setenv("RESBM_GEMM_BM2", bm2)
+    got = gpu_step(cfg, dev)
+    if name not in _ORACLE_CACHE:
+        _ORACLE_CACHE[name] = oracle_step(cfg, h)
+    _compare_all(cfg, got, _ORACLE_CACHE[name], dev)
+    check("P", to_host(got["P"]), _ORACLE_CACHE[name]["P"], "f32", tol=1e-4)
+    monkeypatch.setenv("RESBM_GEMM_BM2", "1" if bm2 == "0" else "0")
+    other = gpu_step(cfg, dev)
+    for k in ("B", "Y", "P"):
+        assert torch.equal(got[k], other[k]), k
+    assert resbm.resbm_device_error() == 0
 
 
 @pytest.mark.parametrize("act", ["gelu_tanh", "identity"])
