@@ -15,6 +15,10 @@ Citations (sections and equations of the ResBM paper):
                                projections: r_eff = sum_i sigma_i^2 / max_i sigma_i^2
   ffn_down_encode_fwd ........ Sec. 3.2's bottleneck after the feed-forward layer: the encoder on
                                the FFN's output z = H . W2 (stored in bf16 by the FFN)
+  rmsnorm / decode_fwd_rmsnorm  the pre-attention RMSNorm of the block the decoder starts (Sec. 3.2
+                               places the decoder at the start of block l+1; Sec. 4.1's model is a
+                               pre-norm transformer with RMSNorm): N = Y / sqrt(mean_j Y_j^2 + eps)
+                               * gamma over each row, on the decoder's output as stored
   newton_schulz .............. Muon's orthogonalisation of the gradient momentum (Sec. 3.4.2
                                trains the bottleneck weights with Muon): X_0 = G / ||G||_F, then
                                X <- a X + b (X X^T) X + c (X X^T)^2 X on the wide orientation,
@@ -340,3 +344,25 @@ def ffn_down_encode_fwd(H, W2, X, We1, We2, act="silu"):
     F = default().round_to(np.asarray(H, np.float64) @ np.asarray(W2, np.float64), "bf16")
     B, P = default().encode_fwd(X, F, We1, We2, act)
     return B, P, F
+
+
+def rmsnorm(Y, gamma, eps):
+    """RMSNorm of every row of Y in float64: the row's root mean square over its d columns,
+    with eps added under the square root, divides the row, and gamma (d) scales each column:
+    N[t, j] = Y[t, j] / sqrt(mean_j Y[t, j]^2 + eps) * gamma[j]."""
+    Y = np.asarray(Y, dtype=np.float64)
+    gamma = np.asarray(gamma, dtype=np.float64)
+    if Y.ndim != 2 or gamma.shape != (Y.shape[1],):
+        raise ValueError("rmsnorm takes a T x d matrix and d weights")
+    mean_sq = np.mean(Y * Y, axis=1, keepdims=True)
+    return Y / np.sqrt(mean_sq + eps) * gamma[None, :]
+
+
+def decode_fwd_rmsnorm(B, Wd1, Wd2, gamma, eps, act="silu", merge=1, store=None):
+    """The decoder forward and the next block's pre-attention RMSNorm: Y = decode_fwd(B, Wd1, Wd2),
+    then N = rmsnorm(Y as stored, gamma, eps). store = "bf16" / "f32" rounds Y to that dtype first
+    (the residual stream is a tensor of that dtype, and the norm reads it); None keeps it exact.
+    Returns (Y, N) with Y unrounded."""
+    Y = default().decode_fwd(B, Wd1, Wd2, act, merge)
+    Ys = default().round_to(Y, store) if store else Y
+    return Y, rmsnorm(Ys, gamma, eps)

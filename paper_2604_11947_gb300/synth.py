@@ -32,7 +32,7 @@ from dataclasses import dataclass, replace
 import numpy as np
 
 TENSOR_IDS = {"X": 1, "F": 2, "dY": 3, "We1": 4, "We2": 5, "Wd1": 6, "Wd2": 7,
-              "scale": 8, "dB": 9, "dX0": 10, "matrix": 11}
+              "scale": 8, "dB": 9, "dX0": 10, "matrix": 11, "gamma": 12}
 
 
 def matrix(rows: int, cols: int, seed: int = 0) -> np.ndarray:
@@ -151,7 +151,7 @@ CONFIGS = {
 def shapes(cfg: BoundaryConfig) -> dict:
     T, d, r, m = cfg.T, cfg.d, cfg.r, cfg.m
     return {"X": (T, d), "F": (T, d), "dY": (T, d), "dB": (T, r), "dX0": (T, d),
-            "We1": (d, m), "We2": (m, r), "Wd1": (r, m), "Wd2": (m, d)}
+            "We1": (d, m), "We2": (m, r), "Wd1": (r, m), "Wd2": (m, d), "gamma": (1, d)}
 
 
 def _std(cfg: BoundaryConfig, name: str) -> float:
@@ -177,6 +177,8 @@ def rows(cfg: BoundaryConfig, name: str, t0: int, t1: int) -> np.ndarray:
     v = normal(cfg.seed, TENSOR_IDS[name], t0 * ncols, (t1 - t0) * ncols).reshape(t1 - t0, ncols)
     if name in ("X", "F"):
         v *= token_scales(cfg, t0, t1)[:, None]
+    elif name == "gamma":   # an RMSNorm weight: near 1, as trained norm weights sit
+        v = 1.0 + 0.1 * v
     else:
         v *= _std(cfg, name)
     return _finish(cfg, v)

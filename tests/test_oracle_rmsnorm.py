@@ -1,0 +1,107 @@
+"""Pins of the oracle's RMSNorm (the pre-attention norm of the block the decoder starts) and of
+its composition with the decoder, to values the definition fixes by hand and to invariants; and
+planted mistakes in a copy of the oracle's rmsnorm, each of which some pin must catch (no GPU)."""
+import inspect
+import textwrap
+
+import numpy as np
+import pytest
+
+import oracle
+
+
+def pin_worked_example(rms):
+    """Y = [1, 2, 2]: mean of squares 3, + eps 1 = 4, root 2; gamma = [1, 2, 0.5]."""
+    N = rms(np.array([[1.0, 2.0, 2.0]]), np.array([1.0, 2.0, 0.5]), 1.0)
+    assert np.array_equal(N, np.array([[0.5, 2.0, 0.5]]))
+
+
+def pin_constant_row(rms):
+    """A constant row c: N_j = c / sqrt(c^2 + eps) gamma_j (c = 3, eps = 7: 3/4 gamma)."""
+    g = np.array([1.0, -2.0, 4.0, 0.25])
+    N = rms(np.full((2, 4), 3.0), g, 7.0)
+    assert np.allclose(N, np.tile(0.75 * g, (2, 1)), rtol=0, atol=1e-15)
+
+
+def pin_rows_are_independent_and_unit_rms(rms):
+    """Each row is normalised on its own; with eps = 0 and gamma = 1 every row has RMS 1 and the
+    direction of Y; rows permute with the input."""
+    rng = np.random.default_rng(5)
+    Y = rng.standard_normal((6, 40)) * np.array([1e-3, 1, 10, 1e3, 0.5, 7])[:, None]
+    N = rms(Y, np.ones(40), 0.0)
+    assert np.allclose(np.sqrt(np.mean(N * N, axis=1)), 1.0, rtol=1e-14)
+    assert np.allclose(N * np.linalg.norm(Y, axis=1)[:, None] / np.sqrt(40), Y, rtol=1e-13)
+    perm = rng.permutation(6)
+    assert np.array_equal(rms(Y[perm], np.ones(40), 0.0), N[perm])
+
+
+def pin_scale_invariance_and_eps(rms):
+    """With eps = 0, scaling a row by alpha scales N by sign(alpha); eps pulls small rows
+    toward zero: a row of RMS s keeps the factor s / sqrt(s^2 + eps)."""
+    rng = np.random.default_rng(6)
+    Y = rng.standard_normal((3, 16))
+    g = rng.standard_normal(16)
+    N = rms(Y, g, 0.0)
+    assert np.allclose(rms(5.0 * Y, g, 0.0), N, rtol=1e-13)
+    assert np.allclose(rms(-0.25 * Y, g, 0.0), -N, rtol=1e-13)
+    s = np.sqrt(np.mean(Y * Y, axis=1, keepdims=True))
+    assert np.allclose(rms(Y, g, 0.3), N * s / np.sqrt(s * s + 0.3), rtol=1e-13)
+
+
+PINS = [pin_worked_example, pin_constant_row, pin_rows_are_independent_and_unit_rms,
+        pin_scale_invariance_and_eps]
+
+
+@pytest.mark.parametrize("pin", PINS, ids=lambda p: p.__name__)
+def test_oracle_rmsnorm_pins(pin):
+    pin(oracle.rmsnorm)
+
+
+def test_decoder_with_zero_second_layer_normalises_the_padded_identity_path():
+    """Wd2 = 0, merge = 1: Y = pad(B) exactly, so N's first r columns are B / sqrt(sum_j B_j^2 / d
+    + eps) * gamma (the mean runs over all d columns, d - r of them zero) and the rest zero."""
+    rng = np.random.default_rng(7)
+    T, d, r, m = 5, 24, 4, 6
+    B = rng.standard_normal((T, r))
+    g = rng.standard_normal(d)
+    Y, N = oracle.decode_fwd_rmsnorm(B, rng.standard_normal((r, m)), np.zeros((m, d)), g, 0.5)
+    assert np.array_equal(Y[:, :r], B) and not np.any(Y[:, r:])
+    want = B / np.sqrt(np.sum(B * B, axis=1, keepdims=True) / d + 0.5) * g[:r]
+    assert np.allclose(N[:, :r], want, rtol=1e-14) and not np.any(N[:, r:])
+
+
+def test_store_rounding_is_applied_before_the_norm():
+    rng = np.random.default_rng(8)
+    T, d, r, m = 7, 32, 8, 8
+    args = (rng.standard_normal((T, r)), rng.standard_normal((r, m)), rng.standard_normal((m, d)) / 3)
+    g = rng.standard_normal(d)
+    Y, N = oracle.decode_fwd_rmsnorm(*args, g, 1e-5, store="bf16")
+    Yb = oracle.round_to(Y, "bf16")
+    assert np.array_equal(N, oracle.rmsnorm(Yb, g, 1e-5))
+    assert not np.array_equal(N, oracle.rmsnorm(Y, g, 1e-5))
+
+
+MUTANTS = {
+    "mean_over_tokens": ("np.mean(Y * Y, axis=1, keepdims=True)", "np.mean(Y * Y, axis=0, keepdims=True)"),
+    "sum_not_mean": ("np.mean(Y * Y, axis=1, keepdims=True)", "np.sum(Y * Y, axis=1, keepdims=True)"),
+    "eps_outside_root": ("np.sqrt(mean_sq + eps)", "(np.sqrt(mean_sq) + eps)"),
+    "no_root": ("np.sqrt(mean_sq + eps)", "(mean_sq + eps)"),
+    "gamma_by_row": ("gamma[None, :]", "gamma[:Y.shape[0], None]"),
+    "mean_of_abs": ("np.mean(Y * Y, axis=1, keepdims=True)", "np.mean(np.abs(Y), axis=1, keepdims=True) ** 2"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_planted_mistake_in_rmsnorm_is_caught(name):
+    find, repl = MUTANTS[name]
+    src = textwrap.dedent(inspect.getsource(oracle.rmsnorm))
+    assert src.count(find) == 1, name
+    ns = {"np": np}
+    exec(compile(src.replace(find, repl), "<mutant %s>" % name, "exec"), ns)
+    caught = []
+    for pin in PINS:
+        try:
+            pin(ns["rmsnorm"])
+        except (AssertionError, ValueError, IndexError):
+            caught.append(pin.__name__)
+    assert caught, "no pin caught the planted mistake %s" % name
