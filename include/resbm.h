@@ -88,7 +88,8 @@ typedef enum {
     RESBM_OP_BOUNDARY_STEP = 4,
     RESBM_OP_BOUNDARY_STEP_HOST = 5,
     RESBM_OP_EFFECTIVE_RANK = 6,     /* resbm_effective_rank (workspace: resbm_matrix_workspace_bytes) */
-    RESBM_OP_NEWTON_SCHULZ = 7       /* resbm_newton_schulz  (workspace: resbm_matrix_workspace_bytes) */
+    RESBM_OP_NEWTON_SCHULZ = 7,      /* resbm_newton_schulz  (workspace: resbm_matrix_workspace_bytes) */
+    RESBM_OP_DECODE_FWD_RMSNORM = 8  /* resbm_decode_fwd_rmsnorm */
 } resbm_op;
 
 /* desc.flags bits */
@@ -177,6 +178,24 @@ RESBM_API resbm_status resbm_encode_fwd(const resbm_desc *desc, const void *X, c
 RESBM_API resbm_status resbm_decode_fwd(const resbm_desc *desc, const void *B, const void *Wd1,
                               const void *Wd2, void *Y, void *ws, size_t ws_bytes,
                               void *stream);
+
+/* The receive side with the next block's pre-attention RMSNorm fused in. Sec. 3.2 places the
+ * decoder at the start of block l+1, whose first step in a pre-norm transformer normalises the
+ * residual stream before attention (the paper's 1B model, Sec. 4.1: RMSNorm). Returns both
+ *   Y = [merge] B . I_{r x d} + phi(B . Wd1) . Wd2          (as resbm_decode_fwd; the residual stream)
+ *   N[t, j] = Y[t, j] / sqrt(mean_j Y[t, j]^2 + eps) * gamma[j]   (the attention's input)
+ * with the norm taken over Y as stored (rounded to the descriptor's dtype) and N rounded once.
+ *   gamma : d elements, the descriptor's dtype (the norm's weight); eps >= 0
+ *   Y, N  : T x d out (distinct buffers)
+ * On the fused tensor-core path Y is not read back from memory: the decoder runs twice, the
+ * first pass storing Y and each row's partial sums of squares (fixed slots in `ws`), the second
+ * recomputing the same Y bits and storing N; elsewhere the norm reads the stored Y. The row sums
+ * have a fixed order, so N is bitwise reproducible. `ws`: resbm_workspace_bytes(desc,
+ * RESBM_OP_DECODE_FWD_RMSNORM). Errors: as resbm_decode_fwd, and RESBM_ERR_INVALID_ARG for a null
+ * gamma or N, a negative or non-finite eps, or Y and N overlapping. */
+RESBM_API resbm_status resbm_decode_fwd_rmsnorm(const resbm_desc *desc, const void *B, const void *Wd1,
+                                                const void *Wd2, const void *gamma, float eps, void *Y,
+                                                void *N, void *ws, size_t ws_bytes, void *stream);
 
 /* Backward of resbm_decode_fwd for the upstream gradient dY (the compressed gradient dB is
  * what crosses the boundary backwards, Appendix A.3).

@@ -6,6 +6,8 @@
 // to the I/O dtype are folded into loads and stores. It handles every shape and both dtypes
 // and is the fp32 path (fp32 products at full fp32 precision). Weight gradients are split
 // over tokens into fp32 partials that a second kernel sums in a fixed order (deterministic).
+#include <type_traits>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -324,7 +326,48 @@ cudaError_t enc_bwd_t(const resbm_desc &d, const T *dB, const T *F, const float 
     return e;
 }
 
+// RMSNorm of every row of Y (the next block's pre-attention norm, after the decoder on the paths
+// without the fused form): N = Y / sqrt(mean_j Y_j^2 + eps) * gamma. One warp per row; the squares
+// of the stored values summed per lane over a fixed column stride, then by a fixed shuffle tree
+// (deterministic). fp32 rows sum in double (their tolerance is fp32's), bf16 rows in float.
+template <typename E>
+__global__ void __launch_bounds__(256) k_rmsnorm(const E *__restrict__ Y, const E *__restrict__ gamma, float eps,
+                                                 int64_t rows, int64_t d, E *__restrict__ N)
+{
+    using Acc = typename std::conditional<std::is_same<E, float>::value, double, float>::type;
+    const int lane = threadIdx.x & 31;
+    for (int64_t t = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5); t < rows; t += (int64_t)gridDim.x * 8) {
+        const E *y = Y + t * d;
+        Acc s = 0;
+        for (int64_t j = lane; j < d; j += 32) {
+            const Acc v = (Acc)to_f32(y[j]);
+            s += v * v;
+        }
+        for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+        const Acc rstd = (Acc)1 / sqrt(s / (Acc)d + (Acc)eps);
+        for (int64_t j = lane; j < d; j += 32)
+            N[t * d + j] = from_f32<E>((float)((Acc)to_f32(y[j]) * rstd * (Acc)to_f32(gamma[j])));
+    }
+}
+
 }  // namespace
+
+cudaError_t generic_rmsnorm(const resbm_desc &d, const void *Y, const void *gamma, float eps, void *N,
+                            const Ctx &c)
+{
+    if (d.T == 0) return cudaSuccess;
+    int64_t blocks = (d.T + 7) / 8;
+    const int64_t cap = (int64_t)c.sm_count * 16;
+    if (blocks > cap) blocks = cap;
+    if (d.dtype == RESBM_F32)
+        k_rmsnorm<float><<<(unsigned)blocks, 256, 0, c.stream>>>((const float *)Y, (const float *)gamma, eps, d.T, d.d,
+                                                                 (float *)N);
+    else
+        k_rmsnorm<__nv_bfloat16><<<(unsigned)blocks, 256, 0, c.stream>>>(
+            (const __nv_bfloat16 *)Y, (const __nv_bfloat16 *)gamma, eps, d.T, d.d, (__nv_bfloat16 *)N);
+    count_launches(1);
+    return cudaGetLastError();
+}
 
 size_t generic_ws_bytes(const resbm_desc &d, int op)
 {

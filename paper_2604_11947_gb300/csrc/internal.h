@@ -47,5 +47,8 @@ cudaError_t generic_decode_bwd(const resbm_desc &d, const void *dY, const void *
 cudaError_t generic_encode_bwd(const resbm_desc &d, const void *dB, const void *F,
                                const float *P_save, const void *We1, const void *We2, void *dF,
                                void *dX, float *dWe1, float *dWe2, void *ws, const Ctx &c);
+// N = RMSNorm(Y) * gamma over rows of d (the descriptor's dtype), reading a stored Y
+cudaError_t generic_rmsnorm(const resbm_desc &d, const void *Y, const void *gamma, float eps, void *N,
+                            const Ctx &c);
 
 }  // namespace resbm

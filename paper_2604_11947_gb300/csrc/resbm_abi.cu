@@ -2,6 +2,7 @@
 // choice between the tensor-core kernels and the portable CUDA-core kernels.
 #include <cuda_runtime.h>
 #include <stdint.h>
+#include <math.h>
 #include <string.h>
 
 #include <atomic>
@@ -235,6 +236,16 @@ LinearWs carve_linear(const resbm_desc &d, void *ws)
 
 size_t ws_for(const resbm_desc &d0, int op)
 {
+    if (op == RESBM_OP_DECODE_FWD_RMSNORM) {
+        // the decoder forward's own scratch, or the fused form's row sums of squares
+        const resbm_desc d = two_layer(d0);
+        size_t b = ws_for(d0, RESBM_OP_DECODE_FWD);
+        if (tc_supported(d, RESBM_OP_DECODE_FWD)) {
+            const size_t f = (is_linear(d0) ? carve_linear(d0, nullptr).bytes : 0) + tc_rmsnorm_ws_bytes(d);
+            if (f > b) b = f;
+        }
+        return b;
+    }
     const resbm_desc d = two_layer(d0);
     size_t g = generic_ws_bytes(d, op);
     size_t t = tc_supported(d, op) ? tc_ws_bytes(d, op, sizing_sms()) : 0;
@@ -306,6 +317,20 @@ resbm_status validate_decode_fwd(const resbm_desc &d, const void *B, const void 
     const Range outs[] = {rng(Y, d.T * d.d, es)};
     const Range ins[] = {rng(B, d.T * d.r, es), rng(Wd1, d.r * d.m, es), rng(Wd2, d.m * d.d, es)};
     return any_overlap(outs, ins, 3) ? RESBM_ERR_INVALID_ARG : RESBM_OK;
+}
+
+resbm_status validate_decode_fwd_rmsnorm(const resbm_desc &d, const void *B, const void *Wd1, const void *Wd2,
+                                         const void *gamma, float eps, const void *Y, const void *N)
+{
+    const size_t es = elem_size(d);
+    const bool t = d.T > 0;
+    if (!ptr_ok(B, es, t) || !ptr_ok(Wd1, es, !is_linear(d)) || !ptr_ok(Wd2, es, true) || !ptr_ok(Y, es, t) ||
+        !ptr_ok(N, es, t) || !ptr_ok(gamma, es, true) || !(eps >= 0.0f) || !(eps < INFINITY))
+        return RESBM_ERR_INVALID_ARG;
+    const Range outs[] = {rng(Y, d.T * d.d, es), rng(N, d.T * d.d, es)};
+    const Range ins[] = {rng(B, d.T * d.r, es), rng(Wd1, d.r * d.m, es), rng(Wd2, d.m * d.d, es),
+                         rng(gamma, d.d, es)};
+    return any_overlap(outs, ins, 4) ? RESBM_ERR_INVALID_ARG : RESBM_OK;
 }
 
 resbm_status validate_decode_bwd(const resbm_desc &d, const void *dY, const void *B,
@@ -436,6 +461,29 @@ resbm_status exec_decode_fwd(const resbm_desc &d, const void *B, const void *Wd1
     const LinearWs l = carve_linear(d, ws);
     resbm_status s = finish(fill_identity(d, l.I, c));
     return s != RESBM_OK ? s : run_decode_fwd(two_layer(d), B, l.I, Wd2, Y, l.inner, c);
+}
+
+// the fused tensor-core form where the decoder forward runs on the fused kernels, else the
+// decoder forward followed by the norm over the stored Y
+resbm_status run_decode_fwd_rmsnorm(const resbm_desc &d, const void *B, const void *Wd1, const void *Wd2,
+                                    const void *gamma, float eps, void *Y, void *N, void *ws, const Ctx &c)
+{
+    if (d.T == 0) return RESBM_OK;
+    if (use_tc(d, RESBM_OP_DECODE_FWD)) {
+        cudaError_t e = tc_decode_fwd_rmsnorm(d, B, Wd1, Wd2, gamma, eps, Y, N, ws, c);
+        if (e != cudaErrorNotSupported) return finish(e);
+    }
+    resbm_status s = run_decode_fwd(d, B, Wd1, Wd2, Y, ws, c);
+    return s != RESBM_OK ? s : finish(generic_rmsnorm(d, Y, gamma, eps, N, c));
+}
+
+resbm_status exec_decode_fwd_rmsnorm(const resbm_desc &d, const void *B, const void *Wd1, const void *Wd2,
+                                     const void *gamma, float eps, void *Y, void *N, void *ws, const Ctx &c)
+{
+    if (!is_linear(d)) return run_decode_fwd_rmsnorm(d, B, Wd1, Wd2, gamma, eps, Y, N, ws, c);
+    const LinearWs l = carve_linear(d, ws);
+    resbm_status s = finish(fill_identity(d, l.I, c));
+    return s != RESBM_OK ? s : run_decode_fwd_rmsnorm(two_layer(d), B, l.I, Wd2, gamma, eps, Y, N, l.inner, c);
 }
 
 resbm_status exec_decode_bwd(const resbm_desc &d, const void *dY, const void *B, const void *Wd1,
@@ -622,7 +670,8 @@ resbm_status resbm_workspace_bytes(const resbm_desc *desc, int op, size_t *bytes
 {
     resbm_status s = check_desc(desc);
     if (s != RESBM_OK) return s;
-    if (!bytes || op < RESBM_OP_ENCODE_FWD || op > RESBM_OP_BOUNDARY_STEP_HOST)
+    if (!bytes || op < RESBM_OP_ENCODE_FWD ||
+        (op > RESBM_OP_BOUNDARY_STEP_HOST && op != RESBM_OP_DECODE_FWD_RMSNORM))
         return RESBM_ERR_INVALID_ARG;
     *bytes = op == RESBM_OP_BOUNDARY_STEP_HOST ? host_stage_bytes(*desc)
              : op == RESBM_OP_BOUNDARY_STEP    ? step_ws_bytes(*desc)
@@ -652,6 +701,19 @@ resbm_status resbm_decode_fwd(const resbm_desc *desc, const void *B, const void 
     Ctx c;
     if (s == RESBM_OK) s = make_ctx(stream, &c);
     if (s == RESBM_OK) s = exec_decode_fwd(*desc, B, Wd1, Wd2, Y, ws, c);
+    return s;
+}
+
+resbm_status resbm_decode_fwd_rmsnorm(const resbm_desc *desc, const void *B, const void *Wd1, const void *Wd2,
+                                      const void *gamma, float eps, void *Y, void *N, void *ws, size_t ws_bytes,
+                                      void *stream)
+{
+    resbm_status s = check_desc(desc);
+    if (s == RESBM_OK) s = validate_decode_fwd_rmsnorm(*desc, B, Wd1, Wd2, gamma, eps, Y, N);
+    if (s == RESBM_OK) s = check_ws(*desc, RESBM_OP_DECODE_FWD_RMSNORM, ws, ws_bytes);
+    Ctx c;
+    if (s == RESBM_OK) s = make_ctx(stream, &c);
+    if (s == RESBM_OK) s = exec_decode_fwd_rmsnorm(*desc, B, Wd1, Wd2, gamma, eps, Y, N, ws, c);
     return s;
 }
 

@@ -200,9 +200,10 @@ int grid_tokens(const Ctx &c, int64_t T)
     return (int)(g < 1 ? 1 : g);
 }
 
-template <int M>
+// NORM (k_dec_fwd): 0 Y; 1 Y and the row sums of squares into ss; 2 N = RMSNorm(Y) * gamma into Y
+template <int M, int NORM = 0>
 cudaError_t launch_dec_fwd(const resbm_desc &d, const void *B, const void *Wd1, const void *Wd2, void *Y,
-                           const Ctx &c)
+                           const Ctx &c, float *ss = nullptr, const void *gamma = nullptr, float eps = 0.0f)
 {
     using Cfg = tc::DecFwdCfg<M>;
     CUtensorMap m_wd2, m_y128, m_y16, m_b;
@@ -212,13 +213,14 @@ cudaError_t launch_dec_fwd(const resbm_desc &d, const void *B, const void *Wd1, 
         !make_map(&m_b, B, d.r, d.T, d.r * 2, Cfg::GB / 2, 128, swizzle_for(Cfg::GB)))
         return cudaErrorInvalidValue;
     static std::atomic<uint8_t> smem_set[kMaxDev];
-    cudaError_t e = ensure_smem(tc::k_dec_fwd<M>, Cfg::SMEM_BYTES, c.device, smem_set);
+    cudaError_t e = ensure_smem(tc::k_dec_fwd<M, NORM>, Cfg::SMEM_BYTES, c.device, smem_set);
     if (e != cudaSuccess) return e;
-    tc::DecFwdArgs a{static_cast<const __nv_bfloat16 *>(Wd1), d.T, d.d, d.act, d.merge_identity};
+    tc::DecFwdArgs a{static_cast<const __nv_bfloat16 *>(Wd1), d.T, d.d, d.act, d.merge_identity,
+                     ss, static_cast<const __nv_bfloat16 *>(gamma), eps};
     // one CTA per SM, at most one per (tile, chunk) unit (the decoder forward splits tiles by columns)
     int64_t units = ((d.T + 127) / 128) * (d.d / Cfg::NCH);
     const int grid = (int)(units < c.sm_count ? (units < 1 ? 1 : units) : c.sm_count);
-    e = launch(tc::k_dec_fwd<M>, grid, Cfg::THREADS, Cfg::SMEM_BYTES, c.stream, m_wd2, m_y128, m_y16,
+    e = launch(tc::k_dec_fwd<M, NORM>, grid, Cfg::THREADS, Cfg::SMEM_BYTES, c.stream, m_wd2, m_y128, m_y16,
                m_b, a);
     count_launches(1);
     return e;
@@ -717,6 +719,35 @@ cudaError_t tc_decode_fwd(const resbm_desc &d, const void *B, const void *Wd1, c
     case 32: return launch_dec_fwd<32>(d, B, Wd1, Wd2, Y, c);
     case 64: return launch_dec_fwd<64>(d, B, Wd1, Wd2, Y, c);
     case 128: return launch_dec_fwd<128>(d, B, Wd1, Wd2, Y, c);
+    }
+    return cudaErrorNotSupported;
+}
+
+size_t tc_rmsnorm_ws_bytes(const resbm_desc &d)
+{
+    const int nch = d.m <= 32 ? 256 : 128;   // DecFwdCfg<m>::NCH
+    return (size_t)(2 * (d.d / nch)) * (size_t)d.T * sizeof(float);
+}
+
+template <int M>
+cudaError_t dec_fwd_rmsnorm_t(const resbm_desc &d, const void *B, const void *Wd1, const void *Wd2,
+                              const void *gamma, float eps, void *Y, void *N, float *ss, const Ctx &c)
+{
+    cudaError_t e = launch_dec_fwd<M, 1>(d, B, Wd1, Wd2, Y, c, ss);
+    return e != cudaSuccess ? e : launch_dec_fwd<M, 2>(d, B, Wd1, Wd2, N, c, ss, gamma, eps);
+}
+
+cudaError_t tc_decode_fwd_rmsnorm(const resbm_desc &d, const void *B, const void *Wd1, const void *Wd2,
+                                  const void *gamma, float eps, void *Y, void *N, void *ws, const Ctx &c)
+{
+    if (!al16(B) || !al16(Wd1) || !al16(Wd2) || !al16(Y) || !al16(N) || !al16(gamma) || !al16(ws))
+        return cudaErrorNotSupported;
+    float *ss = static_cast<float *>(ws);
+    switch (d.m) {
+    case 16: return dec_fwd_rmsnorm_t<16>(d, B, Wd1, Wd2, gamma, eps, Y, N, ss, c);
+    case 32: return dec_fwd_rmsnorm_t<32>(d, B, Wd1, Wd2, gamma, eps, Y, N, ss, c);
+    case 64: return dec_fwd_rmsnorm_t<64>(d, B, Wd1, Wd2, gamma, eps, Y, N, ss, c);
+    case 128: return dec_fwd_rmsnorm_t<128>(d, B, Wd1, Wd2, gamma, eps, Y, N, ss, c);
     }
     return cudaErrorNotSupported;
 }

@@ -21,6 +21,12 @@ cudaError_t tc_encode_fwd(const resbm_desc &d, const void *X, const void *F, con
                           const void *We2, void *B, float *P_save, void *ws, const Ctx &c);
 cudaError_t tc_decode_fwd(const resbm_desc &d, const void *B, const void *Wd1, const void *Wd2,
                           void *Y, void *ws, const Ctx &c);
+// The decoder forward with the next block's pre-attention RMSNorm fused in (k_dec_fwd's NORM
+// passes): Y and N = Y / sqrt(mean_j Y_j^2 + eps) * gamma. ws: tc_rmsnorm_ws_bytes(d) bytes (the
+// row sums of squares), 16-byte aligned.
+size_t tc_rmsnorm_ws_bytes(const resbm_desc &d);
+cudaError_t tc_decode_fwd_rmsnorm(const resbm_desc &d, const void *B, const void *Wd1, const void *Wd2,
+                                  const void *gamma, float eps, void *Y, void *N, void *ws, const Ctx &c);
 // after_independent: the previous kernel on c.stream is the boundary step's decoder forward of
 // the same B (it reads B and writes Y only, and B was complete before it could let this launch
 // begin), so the kernel starts on SMs as that kernel's CTAs leave, without waiting for its end

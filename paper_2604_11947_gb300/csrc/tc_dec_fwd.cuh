@@ -20,6 +20,16 @@
 //                    other's work (with one warp per quarter the epilogue set the pace).
 // HBM traffic per token: read B (2r bytes, once per segment), write Y (2d bytes); Wd2 is
 // re-read from L2.
+//
+// The next block's pre-attention RMSNorm fused in (NORM): N = Y / sqrt(mean_j Y_j^2 + eps) * gamma
+// with Y as stored (bf16) needs a row's sum of squares over all d columns before any of its N
+// values, and a row's chunks may lie in several CTAs. So the kernel runs twice on the same B:
+//   NORM = 1 stores Y and, per row, chunk and column half, the sum of squares of the stored
+//            (rounded) Y values into the slot ss[2 c + half][token] (fp32);
+//   NORM = 2 recomputes the same Y bits (same products, same order), sums the row's 2 d / NCH
+//            slots in slot order, and stores N = bf16(Y * rstd * gamma) instead of Y.
+// Y never travels back from memory: per token the pair reads 2 x 2r bytes of B and 8 d / NCH
+// bytes of slots and writes Y and N (4d bytes), against 6d for a separate norm over a stored Y.
 #pragma once
 
 #include "common.cuh"
@@ -61,19 +71,23 @@ struct DecFwdArgs {
     const __nv_bfloat16 *Wd1;   // r x m
     int64_t T, d;
     int act, merge;
+    float *ss;                    // NORM: 2 d / NCH slots x T row sums of squares
+    const __nv_bfloat16 *gamma;   // NORM = 2: the norm's weight (d)
+    float eps;                    // NORM = 2
 };
 
 // Receive side. Per tile of 128 tokens: the producer loads the tile's B rows by TMA; the MMA
 // computes Q = B . Wd1 into the next free accumulator (a "chunk" of its own in the accumulator
 // sequence); the epilogue turns Q into G = phi(Q) (bf16, shared memory) and then drains the
 // tile's Y chunks (G . Wd2_chunk, + B on the first r columns), storing them by TMA.
-template <int M_>
+template <int M_, int NORM = 0>
 __global__ void __launch_bounds__(320, 1)
     k_dec_fwd(const __grid_constant__ CUtensorMap tm_wd2, const __grid_constant__ CUtensorMap tm_y128,
               const __grid_constant__ CUtensorMap tm_y16, const __grid_constant__ CUtensorMap tm_b,
               const DecFwdArgs a)
 {
     using C = DecFwdCfg<M_>;
+    static_assert(NORM >= 0 && NORM <= 2, "0: Y; 1: Y and row sums of squares; 2: the normalised rows");
     griddep_wait();               // the previous kernel of the stream has completed
     griddep_launch_dependents();  // the next one may be scheduled on SMs as they free up
     extern __shared__ uint8_t smem_raw[];
@@ -315,6 +329,13 @@ __global__ void __launch_bounds__(320, 1)
             const int64_t t0 = tile * 128;
             const int valid = valid_of(tile);
             const uint8_t *bbuf = smem + C::OFF_B + (k % C::NGB) * C::TILE_BYTES;
+            float rstd = 0.0f;   // NORM = 2: this row's 1 / RMS (slots summed in slot order)
+            if (NORM == 2 && row < valid) {
+                const float *sp = a.ss + t0 + row;
+                float sq = 0.0f;
+                for (int sl = 0; sl < 2 * nchunks; ++sl) sq += sp[(int64_t)sl * a.T];
+                rstd = 1.0f / sqrtf(sq / (float)a.d + a.eps);
+            }
             for (int c = c0; c < c1 && ok; ++c, ++acc_it, ++store_it) {
                 if (C::LOOKAHEAD && c == c1 - 1 && has_next) {   // the next tile's G (its Q was issued before this chunk)
                     int64_t nt;
@@ -332,6 +353,7 @@ __global__ void __launch_bounds__(320, 1)
                 uint8_t *stg = smem + C::OFF_STG + sb * C::STG_BYTES;
                 // a warp whose 32 rows all lie past the tile's valid tokens has nothing to store
                 const int gend = (q * 32 < valid) ? C::NCH : 0;
+                float ssq = 0.0f;   // NORM = 1: sum of squares of this row's stored values in the chunk half
                 // 64 columns (two TMEM loads in flight) at a time: one staging box
 #pragma unroll
                 for (int gh = 0; gh < C::NCH / 128; ++gh) {
@@ -365,10 +387,33 @@ __global__ void __launch_bounds__(320, 1)
                             }
                         }
                         uint32_t p[16];
+                        if (NORM == 2) {   // gamma of these 32 columns (the same for every row)
+                            const uint4 *gp = reinterpret_cast<const uint4 *>(a.gamma + (int64_t)c * C::NCH + g * 32);
+                            uint32_t gw[16];
 #pragma unroll
-                        for (int i = 0; i < 16; ++i) {
-                            __nv_bfloat162 hh = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
-                            p[i] = *reinterpret_cast<uint32_t *>(&hh);
+                            for (int i = 0; i < 4; ++i) {
+                                const uint4 u4 = __ldg(gp + i);
+                                gw[4 * i] = u4.x; gw[4 * i + 1] = u4.y; gw[4 * i + 2] = u4.z; gw[4 * i + 3] = u4.w;
+                            }
+#pragma unroll
+                            for (int i = 0; i < 16; ++i) {
+                                const __nv_bfloat162 yy = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+                                const float y0 = __low2float(yy), y1 = __high2float(yy);
+                                const float g0 = __uint_as_float(gw[i] << 16), g1 = __uint_as_float(gw[i] & 0xFFFF0000u);
+                                __nv_bfloat162 hh = __floats2bfloat162_rn(y0 * rstd * g0, y1 * rstd * g1);
+                                p[i] = *reinterpret_cast<uint32_t *>(&hh);
+                            }
+                        } else {
+#pragma unroll
+                            for (int i = 0; i < 16; ++i) {
+                                __nv_bfloat162 hh = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+                                p[i] = *reinterpret_cast<uint32_t *>(&hh);
+                                if (NORM == 1) {
+                                    const float y0 = __low2float(hh), y1 = __high2float(hh);
+                                    ssq = fmaf(y0, y0, ssq);
+                                    ssq = fmaf(y1, y1, ssq);
+                                }
+                            }
                         }
                         // columns [g*32, g*32+32) of the chunk: box g/2, bytes (g%2)*64 .. +64
                         uint8_t *box = stg + (g >> 1) * 16384;
@@ -379,6 +424,7 @@ __global__ void __launch_bounds__(320, 1)
                                 make_uint4(p[4 * i], p[4 * i + 1], p[4 * i + 2], p[4 * i + 3]);
                     }
                 }
+                if (NORM == 1 && row < valid) a.ss[(int64_t)(2 * c + half) * a.T + t0 + row] = ssq;
                 tc_fence_before();
                 mbar_arrive(smem_u32(&acc_empty[ab]));
                 fence_async_smem();

@@ -18,7 +18,8 @@ RESBM_OK, RESBM_ERR_INVALID_ARG, RESBM_ERR_UNSUPPORTED, RESBM_ERR_WORKSPACE, RES
 RESBM_F32, RESBM_BF16 = 0, 1
 RESBM_ACT_SILU, RESBM_ACT_GELU_TANH, RESBM_ACT_IDENTITY = 0, 1, 2
 (RESBM_OP_ENCODE_FWD, RESBM_OP_DECODE_FWD, RESBM_OP_DECODE_BWD, RESBM_OP_ENCODE_BWD,
- RESBM_OP_BOUNDARY_STEP, RESBM_OP_BOUNDARY_STEP_HOST, RESBM_OP_EFFECTIVE_RANK, RESBM_OP_NEWTON_SCHULZ) = range(8)
+ RESBM_OP_BOUNDARY_STEP, RESBM_OP_BOUNDARY_STEP_HOST, RESBM_OP_EFFECTIVE_RANK, RESBM_OP_NEWTON_SCHULZ,
+ RESBM_OP_DECODE_FWD_RMSNORM) = range(9)
 RESBM_FLAG_GENERIC = 1
 RESBM_FLAG_LINEAR = 2
 RESBM_FLAG_GEMM = 4
@@ -34,7 +35,7 @@ EXPORTS = ("resbm_version", "resbm_status_string", "resbm_last_cuda_error", "res
            "resbm_encode_bwd", "resbm_boundary_step", "resbm_boundary_step_host",
            "resbm_decode_bwd_noalloc", "resbm_selftest_wait_timeout", "resbm_matrix_workspace_bytes",
            "resbm_newton_schulz", "resbm_effective_rank", "resbm_ffn_down_encode_workspace_bytes",
-           "resbm_ffn_down_encode_fwd")
+           "resbm_ffn_down_encode_fwd", "resbm_decode_fwd_rmsnorm")
 
 
 class resbm_desc(ctypes.Structure):
@@ -90,6 +91,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.resbm_encode_fwd.argtypes = [D] + [vp] * 6 + [vp, sz, vp]
     lib.resbm_decode_fwd.restype = i32
     lib.resbm_decode_fwd.argtypes = [D] + [vp] * 4 + [vp, sz, vp]
+    lib.resbm_decode_fwd_rmsnorm.restype = i32
+    lib.resbm_decode_fwd_rmsnorm.argtypes = [D] + [vp] * 4 + [ctypes.c_float] + [vp] * 2 + [vp, sz, vp]
     lib.resbm_decode_bwd.restype = i32
     lib.resbm_decode_bwd.argtypes = [D] + [vp] * 7 + [vp, sz, vp]
     lib.resbm_encode_bwd.restype = i32
@@ -199,6 +202,12 @@ def resbm_decode_fwd(desc, B, Wd1, Wd2, Y, ws, stream=None):
     st = load().resbm_decode_fwd(ctypes.byref(desc), _p(B), _p(Wd1), _p(Wd2), _p(Y), _p(ws),
                                  _nbytes(ws), _stream(stream))
     _check("resbm_decode_fwd", st)
+
+
+def resbm_decode_fwd_rmsnorm(desc, B, Wd1, Wd2, gamma, eps, Y, N, ws, stream=None):
+    st = load().resbm_decode_fwd_rmsnorm(ctypes.byref(desc), _p(B), _p(Wd1), _p(Wd2), _p(gamma), float(eps),
+                                         _p(Y), _p(N), _p(ws), _nbytes(ws), _stream(stream))
+    _check("resbm_decode_fwd_rmsnorm", st)
 
 
 def resbm_decode_bwd(desc, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, stream=None):

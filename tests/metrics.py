@@ -21,7 +21,7 @@ token norms log-normally (a factor exp(0.5 n), n ~ N(0,1)).
 import numpy as np
 
 TOL = {"f32": 1e-5, "bf16": 2e-2}
-ROWWISE = {"B", "Y", "dB", "dF", "dX", "F"}
+ROWWISE = {"B", "Y", "dB", "dF", "dX", "F", "N"}
 
 
 def bf16_half_spacing(x):

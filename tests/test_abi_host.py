@@ -24,7 +24,7 @@ def declared_functions():
 
 def test_exports_every_declared_symbol(lib):
     names = declared_functions()
-    assert len(names) == 19, names
+    assert len(names) == 20, names
     assert sorted(resbm.EXPORTS) == names
     for n in names:
         assert hasattr(lib, n), n
@@ -209,3 +209,26 @@ def test_ffn_down_encode_rejects_bad_arguments(lib):
     wide = resbm.make_desc(1024, 512, 64, 64)                             # m > 32: not this kernel
     assert lib.resbm_ffn_down_encode_workspace_bytes(ctypes.byref(wide), 1024, ctypes.byref(sz)) == \
         resbm.RESBM_ERR_UNSUPPORTED
+
+
+def test_decode_fwd_rmsnorm_rejects_bad_arguments(lib):
+    """The fused decoder + RMSNorm's host checks (fake aligned device addresses): gamma, N, eps,
+    Y overlapping N, and the workspace (the row sums of squares on the fused path)."""
+    A, big = 1 << 40, 1 << 34
+    B, W1, W2, g, Y, N, ws = (A + i * big for i in range(7))
+    d = resbm.make_desc(65536, 4096, 32, 32)
+    need = resbm.resbm_workspace_bytes(d, resbm.RESBM_OP_DECODE_FWD_RMSNORM)
+    assert need >= 2 * (4096 // 256) * 65536 * 4   # the fused form's slots
+    fn = lib.resbm_decode_fwd_rmsnorm
+    dp = ctypes.byref(d)
+    assert fn(dp, B, W1, W2, g, 1e-5, Y, N, ws, 16, None) == resbm.RESBM_ERR_WORKSPACE
+    assert fn(dp, B, W1, W2, None, 1e-5, Y, N, ws, need, None) == resbm.RESBM_ERR_INVALID_ARG
+    assert fn(dp, B, W1, W2, g, 1e-5, Y, None, ws, need, None) == resbm.RESBM_ERR_INVALID_ARG
+    assert fn(dp, B, W1, W2, g, -1.0, Y, N, ws, need, None) == resbm.RESBM_ERR_INVALID_ARG
+    assert fn(dp, B, W1, W2, g, float("nan"), Y, N, ws, need, None) == resbm.RESBM_ERR_INVALID_ARG
+    assert fn(dp, B, W1, W2, g, float("inf"), Y, N, ws, need, None) == resbm.RESBM_ERR_INVALID_ARG
+    assert fn(dp, B, W1, W2, g, 1e-5, Y, Y + 1024, ws, need, None) == resbm.RESBM_ERR_INVALID_ARG  # Y and N overlap
+    # f32 descriptors and widths the fused kernels do not take need no slots beyond the decoder's
+    f = resbm.make_desc(333, 200, 8, 5, dtype="f32")
+    assert resbm.resbm_workspace_bytes(f, resbm.RESBM_OP_DECODE_FWD_RMSNORM) == \
+        resbm.resbm_workspace_bytes(f, resbm.RESBM_OP_DECODE_FWD)

@@ -1,0 +1,124 @@
+"""resbm_decode_fwd_rmsnorm (the decoder forward with the next block's pre-attention RMSNorm fused
+in) through the C ABI against the oracle: Y = decode_fwd(B) and N = rmsnorm(Y as stored, gamma,
+eps), on every path, with Y the same bits as resbm_decode_fwd's."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from gpu_helpers import to_dev, to_host
+from metrics import check
+from paper_2604_11947_gb300 import resbm, synth
+
+pytestmark = pytest.mark.gpu
+
+PATHS = {"default": 0, "gemm": resbm.RESBM_FLAG_GEMM, "generic": resbm.RESBM_FLAG_GENERIC}
+EPS = 1e-5
+
+CASES = {
+    # the fused kernels' widths (m = r in {16, 32, 64, 128}: NCH = 256 for m <= 32, else 128),
+    # ragged token counts (a partial last tile), several tiles per CTA
+    "r32": synth.BoundaryConfig("rn_r32", T=1000, d=512, r=32, m=32),
+    "r16": synth.BoundaryConfig("rn_r16", T=777, d=768, r=16, m=16),
+    "r64": synth.BoundaryConfig("rn_r64", T=300, d=256, r=64, m=64),
+    "r128": synth.BoundaryConfig("rn_r128", T=260, d=512, r=128, m=128),
+    "r32_gelu_merge0": synth.BoundaryConfig("rn_r32_g", T=515, d=1024, r=32, m=32, act="gelu_tanh", merge=0),
+    # widths the fused kernels do not take: the GEMM chain / portable decoder, then the norm
+    "r24_m40": synth.BoundaryConfig("rn_r24_m40", T=999, d=776, r=24, m=40),
+    "odd": synth.BoundaryConfig("rn_odd", T=129, d=100, r=3, m=7),
+    "f32": synth.BoundaryConfig("rn_f32", T=333, d=200, r=8, m=5, dtype="f32"),
+    # one token, and a single partial tile
+    "one_token": synth.BoundaryConfig("rn_one", T=1, d=512, r=32, m=32),
+}
+
+
+def _inputs(cfg):
+    B = synth.tensor(cfg, "dB")          # a T x r boundary tensor (the dB stream's draws)
+    h = {"B": B, "Wd1": synth.tensor(cfg, "Wd1"), "Wd2": synth.tensor(cfg, "Wd2"),
+         "gamma": synth.tensor(cfg, "gamma")[0]}
+    dev = {k: to_dev(v, cfg) for k, v in h.items()}
+    return h, dev
+
+
+def _run(cfg, dev, flags=0, eps=EPS):
+    desc = resbm.desc_from_config(cfg, flags)
+    dt = torch.bfloat16 if cfg.dtype == "bf16" else torch.float32
+    Y = torch.empty(cfg.T, cfg.d, dtype=dt, device="cuda")
+    N = torch.empty(cfg.T, cfg.d, dtype=dt, device="cuda")
+    ws = resbm.workspace(desc, resbm.RESBM_OP_DECODE_FWD_RMSNORM)
+    resbm.resbm_decode_fwd_rmsnorm(desc, dev["B"], dev["Wd1"], dev["Wd2"], dev["gamma"], eps, Y, N, ws)
+    torch.cuda.synchronize()
+    return Y, N
+
+
+@pytest.mark.parametrize("path", PATHS)
+@pytest.mark.parametrize("name", CASES)
+def test_decode_fwd_rmsnorm_matches_oracle(name, path):
+    cfg = CASES[name]
+    h, dev = _inputs(cfg)
+    Y, N = _run(cfg, dev, PATHS[path])
+    wY, wN = oracle.decode_fwd_rmsnorm(h["B"], h["Wd1"], h["Wd2"], h["gamma"], EPS, cfg.act, cfg.merge,
+                                       store=cfg.dtype)
+    check("Y", to_host(Y), wY, cfg.dtype)
+    check("N", to_host(N), wN, cfg.dtype)
+    # Y is the decoder forward's own output, bit for bit
+    desc = resbm.desc_from_config(cfg, PATHS[path])
+    Y2 = torch.empty_like(Y)
+    resbm.resbm_decode_fwd(desc, dev["B"], dev["Wd1"], dev["Wd2"], Y2, resbm.workspace(desc, resbm.RESBM_OP_DECODE_FWD))
+    torch.cuda.synchronize()
+    assert torch.equal(Y, Y2)
+    # and N is reproducible bit for bit (fixed-order row sums)
+    _, N2 = _run(cfg, dev, PATHS[path])
+    assert torch.equal(N, N2)
+    assert resbm.resbm_device_error() == 0
+
+
+def test_fused_and_unfused_norms_agree():
+    """The fused form (row sums of squares of the recomputed Y, in fixed slots) against the GEMM
+    chain's decoder followed by the norm over its stored Y: the same N to within bf16 rounding."""
+    cfg = CASES["r32"]
+    h, dev = _inputs(cfg)
+    _, Nf = _run(cfg, dev, 0)
+    _, Ng = _run(cfg, dev, resbm.RESBM_FLAG_GEMM)
+    check("N", to_host(Nf), to_host(Ng), "bf16")
+
+
+def test_zero_second_layer_gives_normalised_identity_path():
+    """Wd2 = 0 and merge = 1: Y = pad(B) exactly, N's first r columns B * rstd * gamma, the rest
+    exactly zero."""
+    cfg = CASES["r32"]
+    h, dev = _inputs(cfg)
+    dev["Wd2"] = torch.zeros_like(dev["Wd2"])
+    Y, N = _run(cfg, dev, 0)
+    r = cfg.r
+    assert torch.equal(Y[:, :r], dev["B"]) and not torch.any(Y[:, r:])
+    assert not torch.any(N[:, r:])
+    _, wN = oracle.decode_fwd_rmsnorm(h["B"], h["Wd1"], np.zeros_like(h["Wd2"]), h["gamma"], EPS, cfg.act, 1,
+                                      store="bf16")
+    check("N", to_host(N), wN, "bf16")
+
+
+def test_empty_token_count_is_a_no_op():
+    cfg = synth.BoundaryConfig("rn_empty", T=0, d=512, r=32, m=32)
+    desc = resbm.desc_from_config(cfg)
+    w = {k: to_dev(synth.tensor(cfg, k), cfg) for k in ("Wd1", "Wd2")}
+    g = to_dev(synth.tensor(cfg, "gamma")[0], cfg)
+    e = torch.empty(0, device="cuda", dtype=torch.bfloat16)
+    ws = resbm.workspace(desc, resbm.RESBM_OP_DECODE_FWD_RMSNORM)
+    resbm.resbm_decode_fwd_rmsnorm(desc, e, w["Wd1"], w["Wd2"], g, EPS, e, e, ws)
+    torch.cuda.synchronize()
+
+
+@pytest.mark.slow
+def test_headline_shape_every_element():
+    """T = 65536, d = 4096, r = 32 (the bench's workload), in the launch configuration the bench
+    times: every element of Y and N against the oracle."""
+    cfg = synth.CONFIGS["large_bf16"]
+    h, dev = _inputs(cfg)
+    Y, N = _run(cfg, dev, 0)
+    wY, wN = oracle.decode_fwd_rmsnorm(h["B"], h["Wd1"], h["Wd2"], h["gamma"], EPS, cfg.act, cfg.merge,
+                                       store="bf16")
+    check("Y", to_host(Y), wY, "bf16")
+    del wY
+    check("N", to_host(N), wN, "bf16")
+    assert resbm.resbm_device_error() == 0
