@@ -47,6 +47,9 @@ def parse():
     p.add_argument("--no-cpu", action="store_true", help="skip the oracle CPU baseline")
     p.add_argument("--no-extra", action="store_true",
                    help="skip the other workloads (T=16384 d=2048 r=16 and the d=8192 r-sweep)")
+    p.add_argument("--rmsnorm-only", action="store_true",
+                   help="run only the decoder forward + RMSNorm comparison (for profiler captures; "
+                        "--steps / --warmup apply); prints its JSON object, not a bench line")
     p.add_argument("--ffn-only", action="store_true",
                    help="run only the FFN down-projection + encoder comparison (for profiler captures; "
                         "--steps / --warmup apply); prints its JSON object, not a bench line")
@@ -451,6 +454,54 @@ def ffn_encode_workload(resbm, torch, steps=20, warmup=3):
     return res
 
 
+def decode_rmsnorm_workload(resbm, torch, peaks, steps=50, warmup=5):
+    """The decoder forward with the next block's pre-attention RMSNorm fused in, at the headline
+    shape (T = 65536, d = 4096, r = m = 32, bf16): resbm_decode_fwd_rmsnorm (Y and N, Y never read
+    back) against resbm_decode_fwd followed by torch's rms_norm over the stored Y, and the decoder
+    forward alone. Algorithmic bytes: the fused pair reads B twice and the row sums of squares
+    once, writes them, Y and N; the unfused chain reads B, writes Y, reads Y, writes N."""
+    cfg = synth.CONFIGS["large_bf16"]
+    T, d, r, m = cfg.T, cfg.d, cfg.r, cfg.m
+    desc = resbm.desc_from_config(cfg)
+    g = torch.Generator(device="cuda")
+    g.manual_seed(0)
+    B = torch.randn(T, r, device="cuda", generator=g).to(torch.bfloat16)
+    Wd1 = (torch.randn(r, m, device="cuda", generator=g) / r ** 0.5).to(torch.bfloat16)
+    Wd2 = (torch.randn(m, d, device="cuda", generator=g) / m ** 0.5).to(torch.bfloat16)
+    gamma = (1 + 0.1 * torch.randn(d, device="cuda", generator=g)).to(torch.bfloat16)
+    Y = torch.empty(T, d, dtype=torch.bfloat16, device="cuda")
+    N = torch.empty(T, d, dtype=torch.bfloat16, device="cuda")
+    ws = resbm.workspace(desc, resbm.RESBM_OP_DECODE_FWD_RMSNORM)
+    ws_dec = resbm.workspace(desc, resbm.RESBM_OP_DECODE_FWD)
+    eps = 1e-5
+    runs = {"fused": lambda: resbm.resbm_decode_fwd_rmsnorm(desc, B, Wd1, Wd2, gamma, eps, Y, N, ws),
+            "unfused_decode_then_torch_rms_norm": lambda: (
+                resbm.resbm_decode_fwd(desc, B, Wd1, Wd2, Y, ws_dec),
+                torch.nn.functional.rms_norm(Y, (d,), gamma, eps)),
+            "decode_fwd_alone": lambda: resbm.resbm_decode_fwd(desc, B, Wd1, Wd2, Y, ws_dec)}
+    nch = d // 256
+    alg = {"fused": T * (2 * 2 * r + 2 * 2 * d + 2 * 4 * 2 * nch) + 2 * (2 * (r * m + m * d)) + 2 * d,
+           "unfused_decode_then_torch_rms_norm": T * (2 * r + 3 * 2 * d) + 2 * (r * m + m * d) + 2 * d,
+           "decode_fwd_alone": T * (2 * r + 2 * d) + 2 * (r * m + m * d)}
+    res = {"workload": "decoder forward + the next block's RMSNorm (T=%d, d=%d, r=m=%d, bf16)" % (T, d, r),
+           "steps": steps, "inputs_exceed_l2": True}
+    for name, fn in runs.items():
+        for _ in range(warmup):
+            fn()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(steps):
+            fn()
+        b.record()
+        torch.cuda.synchronize()
+        ms = a.elapsed_time(b) / steps
+        gbs = alg[name] / (ms / 1e3) / 1e9
+        res[name] = {"ms": ms, "alg_bytes": alg[name], "GBps": gbs, "frac": gbs / peaks["hbm_gbs"]}
+    res["bytes_saved_by_fusion"] = alg["unfused_decode_then_torch_rms_norm"] - alg["fused"]
+    return res
+
+
 def pipeline_workload(torch, steps=3, warmup=2):
     """The simulated 4-stage pipeline: one training step (forward + backward) of the 24-layer
     transformer with three ResBM boundaries; the boundary kernels' share of the step time."""
@@ -500,6 +551,10 @@ def main():
     build.build()
     resbm.load()
 
+    if args.rmsnorm_only:
+        print(json.dumps(decode_rmsnorm_workload(resbm, torch, measured_peaks(), steps=max(args.steps, 1),
+                                                 warmup=max(args.warmup, 0))), flush=True)
+        return
     if args.ffn_only:
         print(json.dumps(ffn_encode_workload(resbm, torch, steps=max(args.steps, 1), warmup=max(args.warmup, 0))),
               flush=True)
@@ -573,6 +628,8 @@ def main():
         del reuse
         torch.cuda.empty_cache()
         extra["ffn_down_encode"] = ffn_encode_workload(resbm, torch)
+        torch.cuda.empty_cache()
+        extra["decode_fwd_rmsnorm"] = decode_rmsnorm_workload(resbm, torch, peaks)
         torch.cuda.empty_cache()
         extra["pipeline"] = pipeline_workload(torch)
         torch.cuda.empty_cache()

@@ -184,7 +184,10 @@ RESBM_API resbm_status resbm_decode_fwd(const resbm_desc *desc, const void *B, c
  * residual stream before attention (the paper's 1B model, Sec. 4.1: RMSNorm). Returns both
  *   Y = [merge] B . I_{r x d} + phi(B . Wd1) . Wd2          (as resbm_decode_fwd; the residual stream)
  *   N[t, j] = Y[t, j] / sqrt(mean_j Y[t, j]^2 + eps) * gamma[j]   (the attention's input)
- * with the norm taken over Y as stored (rounded to the descriptor's dtype) and N rounded once.
+ * with the row's RMS taken over Y as stored (rounded to the descriptor's dtype). On the fused
+ * tensor-core path N = round(y * rstd * gamma) with y the unrounded value of Y[t, j] (one rounding
+ * fewer than normalising the stored Y: the two differ by less than half Y's spacing times
+ * rstd * gamma[j] before N's rounding); elsewhere the norm reads the stored Y.
  *   gamma : d elements, the descriptor's dtype (the norm's weight); eps >= 0
  *   Y, N  : T x d out (distinct buffers)
  * On the fused tensor-core path Y is not read back from memory: the decoder runs twice, the

@@ -203,7 +203,7 @@ int grid_tokens(const Ctx &c, int64_t T)
 // NORM (k_dec_fwd): 0 Y; 1 Y and the row sums of squares into ss; 2 N = RMSNorm(Y) * gamma into Y
 template <int M, int NORM = 0>
 cudaError_t launch_dec_fwd(const resbm_desc &d, const void *B, const void *Wd1, const void *Wd2, void *Y,
-                           const Ctx &c, float *ss = nullptr, const void *gamma = nullptr, float eps = 0.0f)
+                           const Ctx &c, float *ss = nullptr, const float *rstd = nullptr, const float *gamma32 = nullptr)
 {
     using Cfg = tc::DecFwdCfg<M>;
     CUtensorMap m_wd2, m_y128, m_y16, m_b;
@@ -216,7 +216,7 @@ cudaError_t launch_dec_fwd(const resbm_desc &d, const void *B, const void *Wd1, 
     cudaError_t e = ensure_smem(tc::k_dec_fwd<M, NORM>, Cfg::SMEM_BYTES, c.device, smem_set);
     if (e != cudaSuccess) return e;
     tc::DecFwdArgs a{static_cast<const __nv_bfloat16 *>(Wd1), d.T, d.d, d.act, d.merge_identity,
-                     ss, static_cast<const __nv_bfloat16 *>(gamma), eps};
+                     ss, rstd, gamma32};
     // one CTA per SM, at most one per (tile, chunk) unit (the decoder forward splits tiles by columns)
     int64_t units = ((d.T + 127) / 128) * (d.d / Cfg::NCH);
     const int grid = (int)(units < c.sm_count ? (units < 1 ? 1 : units) : c.sm_count);
@@ -723,24 +723,37 @@ cudaError_t tc_decode_fwd(const resbm_desc &d, const void *B, const void *Wd1, c
     return cudaErrorNotSupported;
 }
 
+// gamma as fp32 (d), the row sums of squares (2 d / NCH slots of T), the T reciprocal RMS values
+int rmsnorm_slots(const resbm_desc &d) { return (int)(2 * (d.d / (d.m <= 32 ? 256 : 128))); }   // NCH
 size_t tc_rmsnorm_ws_bytes(const resbm_desc &d)
 {
-    const int nch = d.m <= 32 ? 256 : 128;   // DecFwdCfg<m>::NCH
-    return (size_t)(2 * (d.d / nch)) * (size_t)d.T * sizeof(float);
+    return ((size_t)d.d + ((size_t)rmsnorm_slots(d) + 1) * (size_t)d.T) * sizeof(float);
 }
 
 template <int M>
 cudaError_t dec_fwd_rmsnorm_t(const resbm_desc &d, const void *B, const void *Wd1, const void *Wd2,
                               const void *gamma, float eps, void *Y, void *N, float *ss, const Ctx &c)
 {
+    static_assert(tc::DecFwdCfg<M>::NCH == (M <= 32 ? 256 : 128), "rmsnorm_slots");
+    const int ns = rmsnorm_slots(d);
+    float *gamma32 = ss;   // first: d floats, a multiple of NCH, so the slots stay 16-byte aligned too
+    ss += d.d;
+    float *rstd = ss + (int64_t)ns * d.T;
     cudaError_t e = launch_dec_fwd<M, 1>(d, B, Wd1, Wd2, Y, c, ss);
-    return e != cudaSuccess ? e : launch_dec_fwd<M, 2>(d, B, Wd1, Wd2, N, c, ss, gamma, eps);
+    if (e != cudaSuccess) return e;
+    const int64_t n = d.T > d.d ? d.T : d.d;
+    int64_t blocks = (n + 255) / 256;
+    if (blocks > (int64_t)c.sm_count * 8) blocks = (int64_t)c.sm_count * 8;
+    e = launch(tc::k_row_rstd, (unsigned)blocks, 256, 0, c.stream, (const float *)ss, ns, d.T, d.d, eps, rstd,
+               static_cast<const __nv_bfloat16 *>(gamma), gamma32);
+    count_launches(1);
+    return e != cudaSuccess ? e : launch_dec_fwd<M, 2>(d, B, Wd1, Wd2, N, c, nullptr, rstd, gamma32);
 }
 
 cudaError_t tc_decode_fwd_rmsnorm(const resbm_desc &d, const void *B, const void *Wd1, const void *Wd2,
                                   const void *gamma, float eps, void *Y, void *N, void *ws, const Ctx &c)
 {
-    if (!al16(B) || !al16(Wd1) || !al16(Wd2) || !al16(Y) || !al16(N) || !al16(gamma) || !al16(ws))
+    if (!al16(B) || !al16(Wd1) || !al16(Wd2) || !al16(Y) || !al16(N) || !al16(ws))
         return cudaErrorNotSupported;
     float *ss = static_cast<float *>(ws);
     switch (d.m) {

@@ -25,11 +25,18 @@
 // with Y as stored (bf16) needs a row's sum of squares over all d columns before any of its N
 // values, and a row's chunks may lie in several CTAs. So the kernel runs twice on the same B:
 //   NORM = 1 stores Y and, per row, chunk and column half, the sum of squares of the stored
-//            (rounded) Y values into the slot ss[2 c + half][token] (fp32);
-//   NORM = 2 recomputes the same Y bits (same products, same order), sums the row's 2 d / NCH
-//            slots in slot order, and stores N = bf16(Y * rstd * gamma) instead of Y.
-// Y never travels back from memory: per token the pair reads 2 x 2r bytes of B and 8 d / NCH
-// bytes of slots and writes Y and N (4d bytes), against 6d for a separate norm over a stored Y.
+//            (rounded) Y values into the slot ss[2 c + half][token] (fp32; the even and the odd
+//            columns summed separately in column order, then added);
+//   k_row_rstd sums each row's 2 d / NCH slots in slot order: rstd = 1 / sqrt(sum / d + eps),
+//            and writes gamma as fp32;
+//   NORM = 2 recomputes the same fp32 values (same products, same order) and stores
+//            N = bf16((y * rstd) * gamma) instead of Y, y the fp32 value that rounds to the stored
+//            Y (paired fp32 multiplies, each rounded as a single one). Against the norm of the
+//            stored Y this skips one rounding of y: N differs from it by less than half Y's
+//            spacing times rstd * gamma before N's own rounding (and is closer to the exact norm).
+// Y never travels back from memory: per token the three launches read 2 x 2r bytes of B and
+// 8 d / NCH + 4 bytes of sums and write Y and N (4d bytes), against 6d for a separate norm over a
+// stored Y.
 #pragma once
 
 #include "common.cuh"
@@ -71,10 +78,38 @@ struct DecFwdArgs {
     const __nv_bfloat16 *Wd1;   // r x m
     int64_t T, d;
     int act, merge;
-    float *ss;                    // NORM: 2 d / NCH slots x T row sums of squares
-    const __nv_bfloat16 *gamma;   // NORM = 2: the norm's weight (d)
-    float eps;                    // NORM = 2
+    float *ss;                    // NORM = 1: 2 d / NCH slots x T row sums of squares
+    const float *rstd;            // NORM = 2: T reciprocal row RMS (k_row_rstd)
+    const float *gamma;           // NORM = 2: the norm's weight (d, fp32, 16-byte aligned)
 };
+
+// rstd[t] = 1 / sqrt(sum of the row's nslots partial sums of squares, in slot order, / d + eps);
+// gamma32 = gamma as fp32
+__global__ void __launch_bounds__(256) k_row_rstd(const float *__restrict__ ss, int nslots, int64_t T, int64_t d,
+                                                  float eps, float *__restrict__ rstd,
+                                                  const __nv_bfloat16 *__restrict__ gamma, float *__restrict__ gamma32)
+{
+    griddep_wait();
+    griddep_launch_dependents();
+    const int64_t n = T > d ? T : d;
+    for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < n; t += (int64_t)gridDim.x * blockDim.x) {
+        if (t < d) gamma32[t] = __bfloat162float(gamma[t]);
+        if (t < T) {
+            // eight slots' loads in flight at a time, added in slot order
+            float sq = 0.0f;
+            int sl = 0;
+            for (; sl + 8 <= nslots; sl += 8) {
+                float x[8];
+#pragma unroll
+                for (int u = 0; u < 8; ++u) x[u] = ss[(int64_t)(sl + u) * T + t];
+#pragma unroll
+                for (int u = 0; u < 8; ++u) sq += x[u];
+            }
+            for (; sl < nslots; ++sl) sq += ss[(int64_t)sl * T + t];
+            rstd[t] = 1.0f / sqrtf(sq / (float)d + eps);
+        }
+    }
+}
 
 // Receive side. Per tile of 128 tokens: the producer loads the tile's B rows by TMA; the MMA
 // computes Q = B . Wd1 into the next free accumulator (a "chunk" of its own in the accumulator
@@ -329,13 +364,7 @@ __global__ void __launch_bounds__(320, 1)
             const int64_t t0 = tile * 128;
             const int valid = valid_of(tile);
             const uint8_t *bbuf = smem + C::OFF_B + (k % C::NGB) * C::TILE_BYTES;
-            float rstd = 0.0f;   // NORM = 2: this row's 1 / RMS (slots summed in slot order)
-            if (NORM == 2 && row < valid) {
-                const float *sp = a.ss + t0 + row;
-                float sq = 0.0f;
-                for (int sl = 0; sl < 2 * nchunks; ++sl) sq += sp[(int64_t)sl * a.T];
-                rstd = 1.0f / sqrtf(sq / (float)a.d + a.eps);
-            }
+            const float rstd = (NORM == 2 && row < valid) ? a.rstd[t0 + row] : 0.0f;   // this row's 1 / RMS
             for (int c = c0; c < c1 && ok; ++c, ++acc_it, ++store_it) {
                 if (C::LOOKAHEAD && c == c1 - 1 && has_next) {   // the next tile's G (its Q was issued before this chunk)
                     int64_t nt;
@@ -353,7 +382,7 @@ __global__ void __launch_bounds__(320, 1)
                 uint8_t *stg = smem + C::OFF_STG + sb * C::STG_BYTES;
                 // a warp whose 32 rows all lie past the tile's valid tokens has nothing to store
                 const int gend = (q * 32 < valid) ? C::NCH : 0;
-                float ssq = 0.0f;   // NORM = 1: sum of squares of this row's stored values in the chunk half
+                float2 ssq = make_float2(0.0f, 0.0f);   // NORM = 1: this row's sums of squares (even, odd columns)
                 // 64 columns (two TMEM loads in flight) at a time: one staging box
 #pragma unroll
                 for (int gh = 0; gh < C::NCH / 128; ++gh) {
@@ -388,20 +417,19 @@ __global__ void __launch_bounds__(320, 1)
                         }
                         uint32_t p[16];
                         if (NORM == 2) {   // gamma of these 32 columns (the same for every row)
-                            const uint4 *gp = reinterpret_cast<const uint4 *>(a.gamma + (int64_t)c * C::NCH + g * 32);
-                            uint32_t gw[16];
+                            const float4 *gp = reinterpret_cast<const float4 *>(a.gamma + (int64_t)c * C::NCH + g * 32);
+                            const float2 r2 = make_float2(rstd, rstd);
 #pragma unroll
-                            for (int i = 0; i < 4; ++i) {
-                                const uint4 u4 = __ldg(gp + i);
-                                gw[4 * i] = u4.x; gw[4 * i + 1] = u4.y; gw[4 * i + 2] = u4.z; gw[4 * i + 3] = u4.w;
-                            }
+                            for (int i = 0; i < 8; ++i) {
+                                const float4 g4 = __ldg(gp + i);
 #pragma unroll
-                            for (int i = 0; i < 16; ++i) {
-                                const __nv_bfloat162 yy = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
-                                const float y0 = __low2float(yy), y1 = __high2float(yy);
-                                const float g0 = __uint_as_float(gw[i] << 16), g1 = __uint_as_float(gw[i] & 0xFFFF0000u);
-                                __nv_bfloat162 hh = __floats2bfloat162_rn(y0 * rstd * g0, y1 * rstd * g1);
-                                p[i] = *reinterpret_cast<uint32_t *>(&hh);
+                                for (int e = 0; e < 2; ++e) {
+                                    const int k2 = 2 * i + e;   // the pair of columns 2 k2, 2 k2 + 1
+                                    const float2 yn = __fmul2_rn(__fmul2_rn(make_float2(v[2 * k2], v[2 * k2 + 1]), r2),
+                                                                 e ? make_float2(g4.z, g4.w) : make_float2(g4.x, g4.y));
+                                    __nv_bfloat162 hh = __float22bfloat162_rn(yn);
+                                    p[k2] = *reinterpret_cast<uint32_t *>(&hh);
+                                }
                             }
                         } else {
 #pragma unroll
@@ -409,9 +437,8 @@ __global__ void __launch_bounds__(320, 1)
                                 __nv_bfloat162 hh = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
                                 p[i] = *reinterpret_cast<uint32_t *>(&hh);
                                 if (NORM == 1) {
-                                    const float y0 = __low2float(hh), y1 = __high2float(hh);
-                                    ssq = fmaf(y0, y0, ssq);
-                                    ssq = fmaf(y1, y1, ssq);
+                                    const float2 y2 = __bfloat1622float2(hh);
+                                    ssq = __ffma2_rn(y2, y2, ssq);
                                 }
                             }
                         }
@@ -424,7 +451,7 @@ __global__ void __launch_bounds__(320, 1)
                                 make_uint4(p[4 * i], p[4 * i + 1], p[4 * i + 2], p[4 * i + 3]);
                     }
                 }
-                if (NORM == 1 && row < valid) a.ss[(int64_t)(2 * c + half) * a.T + t0 + row] = ssq;
+                if (NORM == 1 && row < valid) a.ss[(int64_t)(2 * c + half) * a.T + t0 + row] = ssq.x + ssq.y;
                 tc_fence_before();
                 mbar_arrive(smem_u32(&acc_empty[ab]));
                 fence_async_smem();

@@ -73,3 +73,21 @@ def test_bf16_correctly_rounded_outlier_passes_one_spacing_off_fails():
     g[0, 0] = 2.03125 + 2.0 ** -6       # the next bf16 value
     with pytest.raises(AssertionError):
         check("Y", g, o, "bf16")
+
+
+def test_carried_rounding_allowance():
+    """An output computed from another rounded output (N from the stored Y) gets `allow` per
+    element on top of its own half spacing, and nothing more."""
+    o = np.ones((1, 100))
+    o[0, ::2] = -1.0
+    o[0, 0] = 4.98                                     # row RMS ~1.1
+    carried = np.zeros_like(o)
+    carried[0, 0] = 2.0 ** -6                          # half of Y's spacing at ~5, times rstd * gamma ~ 1
+    g = o.copy()
+    g[0, 0] = 5.03125                                  # the neighbouring value past both roundings
+    with pytest.raises(AssertionError):
+        check("N", g, o, "bf16")
+    assert check("N", g, o, "bf16", allow=carried) <= 2e-2
+    g[0, 1] += 0.05                                    # an element without a carried rounding
+    with pytest.raises(AssertionError):
+        check("N", g, o, "bf16", allow=carried)
