@@ -15,6 +15,8 @@ Citations (sections and equations of the ResBM paper):
                                projections: r_eff = sum_i sigma_i^2 / max_i sigma_i^2
   ffn_down_encode_fwd ........ Sec. 3.2's bottleneck after the feed-forward layer: the encoder on
                                the FFN's output z = H . W2 (stored in bf16 by the FFN)
+  rmsnorm_bwd ................ the chain rule of rmsnorm (for the upstream dN), plus an incoming
+                               dY added to the input gradient
   rmsnorm / decode_fwd_rmsnorm  the pre-attention RMSNorm of the block the decoder starts (Sec. 3.2
                                places the decoder at the start of block l+1; Sec. 4.1's model is a
                                pre-norm transformer with RMSNorm): N = Y / sqrt(mean_j Y_j^2 + eps)
@@ -366,3 +368,27 @@ def decode_fwd_rmsnorm(B, Wd1, Wd2, gamma, eps, act="silu", merge=1, store=None)
     Y = default().decode_fwd(B, Wd1, Wd2, act, merge)
     Ys = default().round_to(Y, store) if store else Y
     return Y, rmsnorm(Ys, gamma, eps)
+
+
+def rmsnorm_bwd(Y, gamma, eps, dN, dY=None):
+    """Gradients of N = rmsnorm(Y, gamma, eps) for the upstream dN, in float64, by the chain rule
+    of its three steps (s = 1 / sqrt(mean_j Y_j^2 + eps), xhat = Y s, N = xhat gamma):
+      dxhat = dN gamma
+      ds    = sum_j dxhat_j Y_j                    (per row)
+      dY_j  = dxhat_j s + ds * (-s^3 / d) Y_j       (d s / d Y_j = -s^3 Y_j / d)
+      dgamma = sum over rows of dN xhat.
+    An incoming dY (the residual stream's own gradient) is added to the input gradient.
+    Returns (dY_total, dgamma)."""
+    Y = np.asarray(Y, dtype=np.float64)
+    gamma = np.asarray(gamma, dtype=np.float64)
+    dN = np.asarray(dN, dtype=np.float64)
+    d = Y.shape[1]
+    s = 1.0 / np.sqrt(np.mean(Y * Y, axis=1, keepdims=True) + eps)
+    xhat = Y * s
+    dxhat = dN * gamma[None, :]
+    ds = np.sum(dxhat * Y, axis=1, keepdims=True)
+    dY_norm = dxhat * s + ds * (-(s ** 3) / d) * Y
+    dgamma = np.sum(dN * xhat, axis=0)
+    if dY is not None:
+        dY_norm = dY_norm + np.asarray(dY, dtype=np.float64)
+    return dY_norm, dgamma

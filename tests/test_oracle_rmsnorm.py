@@ -105,3 +105,83 @@ def test_planted_mistake_in_rmsnorm_is_caught(name):
         except (AssertionError, ValueError, IndexError):
             caught.append(pin.__name__)
     assert caught, "no pin caught the planted mistake %s" % name
+
+
+# ---- the backward --------------------------------------------------------------------------
+
+def _fd_grads(Y, g, eps, dN, h=1e-6):
+    """Central differences of sum(dN * rmsnorm(Y, g, eps)) in every element of Y and g."""
+    f = lambda Y_, g_: float(np.sum(dN * oracle.rmsnorm(Y_, g_, eps)))
+    dY = np.zeros_like(Y)
+    for idx in np.ndindex(Y.shape):
+        e = np.zeros_like(Y); e[idx] = h
+        dY[idx] = (f(Y + e, g) - f(Y - e, g)) / (2 * h)
+    dg = np.zeros_like(g)
+    for j in range(g.size):
+        e = np.zeros_like(g); e[j] = h
+        dg[j] = (f(Y, g + e) - f(Y, g - e)) / (2 * h)
+    return dY, dg
+
+
+def bpin_finite_differences(bwd):
+    rng = np.random.default_rng(11)
+    Y = rng.standard_normal((3, 7)) * np.array([0.3, 1.0, 4.0])[:, None]
+    g = 1 + 0.2 * rng.standard_normal(7)
+    dN = rng.standard_normal((3, 7))
+    dY, dg = bwd(Y, g, 0.05, dN)
+    fY, fg = _fd_grads(Y, g, 0.05, dN)
+    assert np.allclose(dY, fY, rtol=1e-7, atol=1e-8) and np.allclose(dg, fg, rtol=1e-7, atol=1e-8)
+
+
+def bpin_scale_invariance_makes_dy_orthogonal_to_y(bwd):
+    """With eps = 0, N does not change when a row is scaled, so each row's gradient is orthogonal
+    to the row itself; and dgamma = sum_t dN * N / gamma."""
+    rng = np.random.default_rng(12)
+    Y = rng.standard_normal((4, 9))
+    g = 1 + 0.1 * rng.standard_normal(9)
+    dN = rng.standard_normal((4, 9))
+    dY, dg = bwd(Y, g, 0.0, dN)
+    assert np.allclose(np.sum(dY * Y, axis=1), 0.0, atol=1e-12)
+    assert np.allclose(dg, np.sum(dN * oracle.rmsnorm(Y, g, 0.0) / g, axis=0), rtol=1e-13)
+
+
+def bpin_incoming_gradient_is_added(bwd):
+    rng = np.random.default_rng(13)
+    Y, dN, dY0 = (rng.standard_normal((2, 5)) for _ in range(3))
+    g = np.ones(5)
+    a, ga = bwd(Y, g, 0.1, dN)
+    b, gb = bwd(Y, g, 0.1, dN, dY0)
+    assert np.allclose(b, a + dY0, rtol=0, atol=1e-15) and np.array_equal(ga, gb)
+
+
+BPINS = [bpin_finite_differences, bpin_scale_invariance_makes_dy_orthogonal_to_y, bpin_incoming_gradient_is_added]
+
+
+@pytest.mark.parametrize("pin", BPINS, ids=lambda p: p.__name__)
+def test_oracle_rmsnorm_bwd_pins(pin):
+    pin(oracle.rmsnorm_bwd)
+
+
+BMUTANTS = {
+    "wrong_power_of_s": ("ds * (-(s ** 3) / d) * Y", "ds * (-(s ** 2) / d) * Y"),
+    "missing_1_over_d": ("ds * (-(s ** 3) / d) * Y", "ds * (-(s ** 3)) * Y"),
+    "dgamma_from_Y": ("dgamma = np.sum(dN * xhat, axis=0)", "dgamma = np.sum(dN * Y, axis=0)"),
+    "ds_without_gamma": ("ds = np.sum(dxhat * Y, axis=1, keepdims=True)", "ds = np.sum(dN * Y, axis=1, keepdims=True)"),
+    "sign_of_second_term": ("dxhat * s + ds", "dxhat * s - ds"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(BMUTANTS))
+def test_planted_mistake_in_rmsnorm_bwd_is_caught(name):
+    find, repl = BMUTANTS[name]
+    src = textwrap.dedent(inspect.getsource(oracle.rmsnorm_bwd))
+    assert src.count(find) == 1, name
+    ns = {"np": np}
+    exec(compile(src.replace(find, repl), "<mutant %s>" % name, "exec"), ns)
+    caught = []
+    for pin in BPINS:
+        try:
+            pin(ns["rmsnorm_bwd"])
+        except (AssertionError, ValueError, IndexError):
+            caught.append(pin.__name__)
+    assert caught, "no pin caught the planted mistake %s" % name
