@@ -507,12 +507,17 @@ def pipeline_workload(torch, steps=3, warmup=2):
     transformer with three ResBM boundaries; the boundary kernels' share of the step time."""
     from paper_2604_11947_gb300 import pipeline
     cfg = pipeline.PIPELINE
-    model = pipeline.PipelineModel(cfg)
     tokens = pipeline.synthetic_tokens(cfg)
+    model = pipeline.PipelineModel(cfg)
     step_ms, bnd_ms, loss = pipeline.time_steps(model, tokens, steps, warmup)
     del model
+    # the same model with the receiving blocks' RMSNorm run by torch after the decoder
+    model = pipeline.PipelineModel(cfg.with_(fuse_norm=False))
+    step_u, bnd_u, loss_u = pipeline.time_steps(model, tokens, steps, warmup)
+    del model
     return {"workload": "%d-layer pre-norm decoder (d=%d, %d heads, SwiGLU %d, vocab %d, bf16) in %d "
-                        "stages with a ResBM boundary (r=%d, m=%d, merge=1) between consecutive stages; "
+                        "stages with a ResBM boundary (r=%d, m=%d, merge=1) between consecutive stages, "
+                        "each receiving block's pre-attention RMSNorm fused into the decoder; "
                         "batch %d x seq %d uniform random token ids; one training step (forward + "
                         "backward, no optimizer update)"
                         % (cfg.layers, cfg.d, cfg.heads, cfg.ffn, cfg.vocab, cfg.stages, cfg.r, cfg.m,
@@ -521,8 +526,10 @@ def pipeline_workload(torch, steps=3, warmup=2):
             "value": cfg.tokens / (step_ms / 1e3), "unit": "tokens/s",
             "boundary_ms_per_step": bnd_ms, "boundary_share": bnd_ms / step_ms,
             "boundaries": cfg.stages - 1, "loss": loss,
+            "unfused_norm": {"ms_per_step": step_u, "boundary_ms_per_step": bnd_u, "loss": loss_u},
             "timing": "CUDA events around the K steps and around every boundary C-ABI call "
-                      "(12 per step: encode/decode forward and backward of 3 boundaries)"}
+                      "(12 per step: encode/decode forward and backward of 3 boundaries; with the fused "
+                      "norm the decoder forward's call includes the norm)"}
 
 
 def main():

@@ -89,7 +89,8 @@ typedef enum {
     RESBM_OP_BOUNDARY_STEP_HOST = 5,
     RESBM_OP_EFFECTIVE_RANK = 6,     /* resbm_effective_rank (workspace: resbm_matrix_workspace_bytes) */
     RESBM_OP_NEWTON_SCHULZ = 7,      /* resbm_newton_schulz  (workspace: resbm_matrix_workspace_bytes) */
-    RESBM_OP_DECODE_FWD_RMSNORM = 8  /* resbm_decode_fwd_rmsnorm */
+    RESBM_OP_DECODE_FWD_RMSNORM = 8, /* resbm_decode_fwd_rmsnorm */
+    RESBM_OP_RMSNORM_BWD = 9         /* resbm_rmsnorm_bwd */
 } resbm_op;
 
 /* desc.flags bits */
@@ -199,6 +200,20 @@ RESBM_API resbm_status resbm_decode_fwd(const resbm_desc *desc, const void *B, c
 RESBM_API resbm_status resbm_decode_fwd_rmsnorm(const resbm_desc *desc, const void *B, const void *Wd1,
                                                 const void *Wd2, const void *gamma, float eps, void *Y,
                                                 void *N, void *ws, size_t ws_bytes, void *stream);
+
+/* Backward of the receiving block's RMSNorm (N of resbm_decode_fwd_rmsnorm) with the residual
+ * stream's own gradient added, so that resbm_decode_bwd can take the sum:
+ *   dY_out = dY + dN . dN/dY,  i.e. per row  dY + s (dN * gamma) - Y (s^3 / d) sum_j dN_j gamma_j Y_j
+ *   dgamma = sum_t dN[t, :] * Y[t, :] * s_t            (fp32, d)
+ * with s = 1 / sqrt(mean_j Y_j^2 + eps) from Y as stored (the chain rule of the norm's three steps).
+ *   Y, dN : T x d in (the descriptor's dtype); gamma: d; dY: T x d in, or NULL for zero; dY_out:
+ *   T x d out, may be the same buffer as dY (in place) but not overlap Y, dN or gamma; dgamma: d
+ *   fp32 out. Requires d <= 16384 (RESBM_ERR_UNSUPPORTED otherwise). Bitwise reproducible on any
+ *   device (fixed row ranges and summation orders). `ws`: resbm_workspace_bytes(desc,
+ *   RESBM_OP_RMSNORM_BWD) (the dgamma partials). Errors: as resbm_decode_fwd_rmsnorm. */
+RESBM_API resbm_status resbm_rmsnorm_bwd(const resbm_desc *desc, const void *Y, const void *gamma, float eps,
+                                         const void *dN, const void *dY, void *dY_out, float *dgamma, void *ws,
+                                         size_t ws_bytes, void *stream);
 
 /* Backward of resbm_decode_fwd for the upstream gradient dY (the compressed gradient dB is
  * what crosses the boundary backwards, Appendix A.3).

@@ -350,7 +350,215 @@ __global__ void __launch_bounds__(256) k_rmsnorm(const E *__restrict__ Y, const 
     }
 }
 
+// Backward of N = RMSNorm(Y) * gamma with the residual stream's own gradient added:
+//   dY_out = dY + s g - Y (s^3 / d) sum_j g_j Y_j,  g = dN * gamma,  s = 1 / sqrt(mean_j Y_j^2 + eps)
+//   dgamma partial of this block = sum over its rows of dN * Y * s
+// A block takes a fixed contiguous range of rows, one row at a time: its threads cover the row's
+// columns (vectors of V elements, thread q owning vectors q, q + 256, ...), the two row sums go
+// through a fixed shuffle tree and the eight warps' partials in warp order, and each thread keeps
+// the dgamma sums of the columns it owns in shared memory (no two threads touch a column), so the
+// result does not depend on timing or on the device. The second pass over the row re-reads it
+// (from L1 / L2). dY may equal dY_out (read before written by the same thread) or be null.
+constexpr int kNormBwdBlocks = 1024;   // ~7 resident per SM on 152 SMs: rows in flight hide the load latency
+constexpr int kNormBwdMaxD = 16384;
+
+template <typename E, int V> struct VecOf;
+template <> struct VecOf<__nv_bfloat16, 8> {
+    static __device__ void load(const __nv_bfloat16 *p, float *f)
+    {
+        const uint4 u = *reinterpret_cast<const uint4 *>(p);
+        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            f[2 * i] = __uint_as_float(w[i] << 16);
+            f[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+        }
+    }
+    static __device__ void store(__nv_bfloat16 *p, const float *f)
+    {
+        uint32_t w[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            __nv_bfloat162 h = __floats2bfloat162_rn(f[2 * i], f[2 * i + 1]);
+            w[i] = *reinterpret_cast<uint32_t *>(&h);
+        }
+        *reinterpret_cast<uint4 *>(p) = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+};
+template <> struct VecOf<float, 4> {
+    static __device__ void load(const float *p, float *f)
+    {
+        const float4 u = *reinterpret_cast<const float4 *>(p);
+        f[0] = u.x; f[1] = u.y; f[2] = u.z; f[3] = u.w;
+    }
+    static __device__ void store(float *p, const float *f) { *reinterpret_cast<float4 *>(p) = make_float4(f[0], f[1], f[2], f[3]); }
+};
+template <typename E> struct VecOf<E, 1> {
+    static __device__ void load(const E *p, float *f) { f[0] = to_f32(*p); }
+    static __device__ void store(E *p, const float *f) { *p = from_f32<E>(f[0]); }
+};
+
+template <typename E, int V>
+__global__ void __launch_bounds__(256) k_rmsnorm_bwd(const E *__restrict__ Y, const E *__restrict__ gamma, float eps,
+                                                     const E *__restrict__ dN, const E *dY, E *dYo,
+                                                     float *__restrict__ dg_part, int64_t rows, int64_t d)
+{
+    extern __shared__ float dgs[];   // d: this block's dgamma sums, column j owned by thread (j / V) % 256
+    __shared__ float2 part[2][8];
+    using L = VecOf<E, V>;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int64_t nv = d / V;
+    for (int64_t q = tid; q < nv; q += 256)
+#pragma unroll
+        for (int i = 0; i < V; ++i) dgs[q * V + i] = 0.0f;
+    const int64_t r0 = rows * blockIdx.x / gridDim.x, r1 = rows * (blockIdx.x + 1) / gridDim.x;
+    for (int64_t t = r0; t < r1; ++t) {
+        const E *y = Y + t * d, *dn = dN + t * d;
+        float sy = 0.0f, sg = 0.0f;   // sum Y^2, sum g Y over this thread's columns
+        for (int64_t q = tid; q < nv; q += 256) {
+            float a[V], b[V], gm[V];
+            L::load(y + q * V, a);
+            L::load(dn + q * V, b);
+            L::load(gamma + q * V, gm);
+#pragma unroll
+            for (int i = 0; i < V; ++i) {
+                sy = fmaf(a[i], a[i], sy);
+                sg = fmaf(b[i] * gm[i], a[i], sg);
+            }
+        }
+        for (int o = 16; o > 0; o >>= 1) {
+            sy += __shfl_xor_sync(0xffffffffu, sy, o);
+            sg += __shfl_xor_sync(0xffffffffu, sg, o);
+        }
+        const int pb = (int)((t - r0) & 1);
+        if (lane == 0) part[pb][warp] = make_float2(sy, sg);
+        __syncthreads();
+        float Sy = 0.0f, Sg = 0.0f;
+#pragma unroll
+        for (int w = 0; w < 8; ++w) {
+            Sy += part[pb][w].x;
+            Sg += part[pb][w].y;
+        }
+        const float s = 1.0f / sqrtf(Sy / (float)d + eps);
+        const float k = s * s * s * Sg / (float)d;
+        for (int64_t q = tid; q < nv; q += 256) {
+            float a[V], b[V], gm[V], o[V];
+            L::load(y + q * V, a);
+            L::load(dn + q * V, b);
+            L::load(gamma + q * V, gm);
+            if (dY) L::load(dY + t * d + q * V, o);
+            else
+#pragma unroll
+                for (int i = 0; i < V; ++i) o[i] = 0.0f;
+            float acc[V];
+            if (V % 4 == 0) {   // 16-byte shared accesses: consecutive threads, consecutive chunks
+#pragma unroll
+                for (int i = 0; i < V; i += 4) {
+                    const float4 u = *reinterpret_cast<const float4 *>(dgs + q * V + i);
+                    acc[i] = u.x; acc[i + 1] = u.y; acc[i + 2] = u.z; acc[i + 3] = u.w;
+                }
+            } else {
+#pragma unroll
+                for (int i = 0; i < V; ++i) acc[i] = dgs[q * V + i];
+            }
+#pragma unroll
+            for (int i = 0; i < V; ++i) {
+                o[i] += s * (b[i] * gm[i]) - a[i] * k;
+                acc[i] = fmaf(b[i], a[i] * s, acc[i]);
+            }
+            if (V % 4 == 0) {
+#pragma unroll
+                for (int i = 0; i < V; i += 4)
+                    *reinterpret_cast<float4 *>(dgs + q * V + i) = make_float4(acc[i], acc[i + 1], acc[i + 2], acc[i + 3]);
+            } else {
+#pragma unroll
+                for (int i = 0; i < V; ++i) dgs[q * V + i] = acc[i];
+            }
+            L::store(dYo + t * d + q * V, o);
+        }
+    }
+    __syncthreads();
+    for (int64_t j = tid; j < d; j += 256) dg_part[(int64_t)blockIdx.x * d + j] = dgs[j];
+}
+
+// dgamma[j] = the blocks' partials summed by a fixed two-level tree: warp w of a CTA sums the
+// partials of blocks [w G, (w + 1) G) in block order (eight loads in flight) for the CTA's 32
+// columns, then the eight group sums are added in group order. CTA x covers columns 32 x .. + 31.
+__global__ void __launch_bounds__(256) k_rmsnorm_dgamma(const float *__restrict__ dg_part, int nblocks, int64_t d,
+                                                        float *__restrict__ dgamma)
+{
+    __shared__ float gs[8][32];
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    const int64_t j = (int64_t)blockIdx.x * 32 + lane;
+    const int G = (nblocks + 7) / 8;
+    const int b0 = w * G, b1 = b0 + G < nblocks ? b0 + G : nblocks;
+    float a = 0.0f;
+    if (j < d) {
+        int b = b0;
+        for (; b + 8 <= b1; b += 8) {
+            float x[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) x[u] = dg_part[(int64_t)(b + u) * d + j];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) a += x[u];
+        }
+        for (; b < b1; ++b) a += dg_part[(int64_t)b * d + j];
+    }
+    gs[w][lane] = a;
+    __syncthreads();
+    if (w == 0 && j < d) {
+        float t = 0.0f;
+#pragma unroll
+        for (int g = 0; g < 8; ++g) t += gs[g][lane];
+        dgamma[j] = t;
+    }
+}
+
 }  // namespace
+
+int rmsnorm_bwd_blocks(int64_t rows) { return (int)(rows < kNormBwdBlocks ? (rows < 1 ? 1 : rows) : kNormBwdBlocks); }
+bool rmsnorm_bwd_supported(const resbm_desc &d) { return d.d >= 1 && d.d <= kNormBwdMaxD; }
+size_t rmsnorm_bwd_ws_bytes(const resbm_desc &d) { return (size_t)rmsnorm_bwd_blocks(d.T) * (size_t)d.d * sizeof(float); }
+
+cudaError_t generic_rmsnorm_bwd(const resbm_desc &d, const void *Y, const void *gamma, float eps, const void *dN,
+                                const void *dY, void *dY_out, float *dgamma, void *ws, const Ctx &c)
+{
+    const int nb = rmsnorm_bwd_blocks(d.T);
+    float *part = static_cast<float *>(ws);
+    const size_t smem = (size_t)d.d * sizeof(float);
+    auto al = [](const void *p) { return p == nullptr || (reinterpret_cast<uintptr_t>(p) & 15u) == 0; };
+    const bool vec = al(Y) && al(gamma) && al(dN) && al(dY) && al(dY_out) &&
+                     d.d % (d.dtype == RESBM_F32 ? 4 : 8) == 0;
+    cudaError_t e = cudaSuccess;
+    if (d.T > 0) {
+        if (d.dtype == RESBM_F32) {
+            auto k = vec ? k_rmsnorm_bwd<float, 4> : k_rmsnorm_bwd<float, 1>;
+            e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+            if (e == cudaSuccess)
+                k<<<nb, 256, smem, c.stream>>>((const float *)Y, (const float *)gamma, eps, (const float *)dN,
+                                              (const float *)dY, (float *)dY_out, part, d.T, d.d);
+        } else {
+            using bf = __nv_bfloat16;
+            auto k = vec ? k_rmsnorm_bwd<bf, 8> : k_rmsnorm_bwd<bf, 1>;
+            e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+            if (e == cudaSuccess)
+                k<<<nb, 256, smem, c.stream>>>((const bf *)Y, (const bf *)gamma, eps, (const bf *)dN, (const bf *)dY,
+                                              (bf *)dY_out, part, d.T, d.d);
+        }
+        count_launches(1);
+        if (e == cudaSuccess) e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    const int64_t gb = (d.d + 31) / 32;
+    if (d.T > 0) {
+        k_rmsnorm_dgamma<<<(unsigned)gb, 256, 0, c.stream>>>(part, nb, d.d, dgamma);
+    } else {
+        e = cudaMemsetAsync(dgamma, 0, (size_t)d.d * sizeof(float), c.stream);
+        if (e != cudaSuccess) return e;
+    }
+    count_launches(d.T > 0 ? 1 : 0);
+    return cudaGetLastError();
+}
 
 cudaError_t generic_rmsnorm(const resbm_desc &d, const void *Y, const void *gamma, float eps, void *N,
                             const Ctx &c)

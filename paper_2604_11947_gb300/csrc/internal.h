@@ -47,6 +47,12 @@ cudaError_t generic_decode_bwd(const resbm_desc &d, const void *dY, const void *
 cudaError_t generic_encode_bwd(const resbm_desc &d, const void *dB, const void *F,
                                const float *P_save, const void *We1, const void *We2, void *dF,
                                void *dX, float *dWe1, float *dWe2, void *ws, const Ctx &c);
+// Backward of N = RMSNorm(Y) * gamma with an incoming dY added (dY may be null or equal dY_out):
+// dY_out (T x d, the descriptor's dtype) and dgamma (d, fp32). ws: rmsnorm_bwd_ws_bytes(d).
+bool rmsnorm_bwd_supported(const resbm_desc &d);
+size_t rmsnorm_bwd_ws_bytes(const resbm_desc &d);
+cudaError_t generic_rmsnorm_bwd(const resbm_desc &d, const void *Y, const void *gamma, float eps, const void *dN,
+                                const void *dY, void *dY_out, float *dgamma, void *ws, const Ctx &c);
 // N = RMSNorm(Y) * gamma over rows of d (the descriptor's dtype), reading a stored Y
 cudaError_t generic_rmsnorm(const resbm_desc &d, const void *Y, const void *gamma, float eps, void *N,
                             const Ctx &c);

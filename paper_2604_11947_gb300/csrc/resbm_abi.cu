@@ -236,6 +236,7 @@ LinearWs carve_linear(const resbm_desc &d, void *ws)
 
 size_t ws_for(const resbm_desc &d0, int op)
 {
+    if (op == RESBM_OP_RMSNORM_BWD) return rmsnorm_bwd_supported(d0) ? rmsnorm_bwd_ws_bytes(d0) : 0;
     if (op == RESBM_OP_DECODE_FWD_RMSNORM) {
         // the decoder forward's own scratch, or the fused form's row sums of squares
         const resbm_desc d = two_layer(d0);
@@ -671,7 +672,7 @@ resbm_status resbm_workspace_bytes(const resbm_desc *desc, int op, size_t *bytes
     resbm_status s = check_desc(desc);
     if (s != RESBM_OK) return s;
     if (!bytes || op < RESBM_OP_ENCODE_FWD ||
-        (op > RESBM_OP_BOUNDARY_STEP_HOST && op != RESBM_OP_DECODE_FWD_RMSNORM))
+        (op > RESBM_OP_BOUNDARY_STEP_HOST && op != RESBM_OP_DECODE_FWD_RMSNORM && op != RESBM_OP_RMSNORM_BWD))
         return RESBM_ERR_INVALID_ARG;
     *bytes = op == RESBM_OP_BOUNDARY_STEP_HOST ? host_stage_bytes(*desc)
              : op == RESBM_OP_BOUNDARY_STEP    ? step_ws_bytes(*desc)
@@ -714,6 +715,32 @@ resbm_status resbm_decode_fwd_rmsnorm(const resbm_desc *desc, const void *B, con
     Ctx c;
     if (s == RESBM_OK) s = make_ctx(stream, &c);
     if (s == RESBM_OK) s = exec_decode_fwd_rmsnorm(*desc, B, Wd1, Wd2, gamma, eps, Y, N, ws, c);
+    return s;
+}
+
+resbm_status resbm_rmsnorm_bwd(const resbm_desc *desc, const void *Y, const void *gamma, float eps, const void *dN,
+                               const void *dY, void *dY_out, float *dgamma, void *ws, size_t ws_bytes, void *stream)
+{
+    resbm_status s = check_desc(desc);
+    if (s != RESBM_OK) return s;
+    const resbm_desc &d = *desc;
+    if (!rmsnorm_bwd_supported(d)) return RESBM_ERR_UNSUPPORTED;
+    const size_t es = elem_size(d);
+    const bool t = d.T > 0;
+    if (!ptr_ok(Y, es, t) || !ptr_ok(gamma, es, true) || !ptr_ok(dN, es, t) || !ptr_ok(dY, es, false) ||
+        !ptr_ok(dY_out, es, t) || !ptr_ok(dgamma, 4, true) || !(eps >= 0.0f) || !(eps < INFINITY))
+        return RESBM_ERR_INVALID_ARG;
+    // dY_out may be dY itself (in place); otherwise no output overlaps an input or the other output
+    const Range outs[] = {rng(dY_out, d.T * d.d, es), rng(dgamma, d.d, 4)};
+    const Range ins[] = {rng(Y, d.T * d.d, es), rng(gamma, d.d, es), rng(dN, d.T * d.d, es),
+                         rng(dY == dY_out ? nullptr : dY, d.T * d.d, es)};
+    if (any_overlap(outs, ins, 4)) return RESBM_ERR_INVALID_ARG;
+    if (dY && dY != dY_out && overlaps(rng(dY, d.T * d.d, es), rng(dY_out, d.T * d.d, es)))
+        return RESBM_ERR_INVALID_ARG;
+    s = check_ws(d, RESBM_OP_RMSNORM_BWD, ws, ws_bytes);
+    Ctx c;
+    if (s == RESBM_OK) s = make_ctx(stream, &c);
+    if (s == RESBM_OK) s = finish(generic_rmsnorm_bwd(d, Y, gamma, eps, dN, dY, dY_out, dgamma, ws, c));
     return s;
 }
 

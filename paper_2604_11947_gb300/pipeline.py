@@ -47,6 +47,7 @@ class PipelineConfig:
                              # "B": D(b) feeds the attention branch, pad(b) its skip
     seed: int = 0
     flags: int = 0           # resbm descriptor flags of the boundaries (RESBM_FLAG_*)
+    fuse_norm: bool = True   # the receiving block's pre-attention RMSNorm fused into the decoder
 
     def with_(self, **kw) -> "PipelineConfig":
         return replace(self, **kw)
@@ -160,6 +161,53 @@ class _Decode(torch.autograd.Function):
         return dB, dWd1.to(Wd1.dtype), dWd2.to(Wd2.dtype), None
 
 
+NORM_EPS = 1e-5
+
+
+class _DecodeNorm(torch.autograd.Function):
+    """(y, n) = (D(b) [+ pad(b)], RMSNorm(y) * gamma): resbm_decode_fwd_rmsnorm forward (the
+    receiving block's pre-attention norm fused into the decoder). Backward: resbm_rmsnorm_bwd adds
+    the norm's gradient to dy (and gives dgamma), then resbm_decode_bwd on the sum."""
+
+    @staticmethod
+    def forward(ctx, B, Wd1, Wd2, gamma, bnd):
+        T = B.shape[0]
+        Y = torch.empty(T, bnd.d, dtype=B.dtype, device=B.device)
+        N = torch.empty_like(Y)
+        ev = bnd.timer.start()
+        resbm.resbm_decode_fwd_rmsnorm(bnd.desc(T), B, Wd1, Wd2, gamma, NORM_EPS, Y, N, bnd.workspace(T))
+        bnd.timer.stop(ev)
+        ctx.save_for_backward(B, Wd1, Wd2, gamma, Y)
+        ctx.bnd = bnd
+        if bnd.capture is not None:
+            bnd.capture.update(B_dec=B.detach(), Y=Y.detach(), N=N.detach(), gamma=gamma.detach())
+        return Y, N
+
+    @staticmethod
+    def backward(ctx, dY, dN):
+        B, Wd1, Wd2, gamma, Y = ctx.saved_tensors
+        bnd = ctx.bnd
+        T = B.shape[0]
+        dgamma = None
+        dB = torch.empty_like(B)
+        dWd1 = torch.empty(bnd.r, bnd.m, dtype=torch.float32, device=B.device)
+        dWd2 = torch.empty(bnd.m, bnd.d, dtype=torch.float32, device=B.device)
+        ev = bnd.timer.start()
+        if dN is not None:
+            dy = torch.empty_like(Y)
+            dg = torch.empty(bnd.d, dtype=torch.float32, device=B.device)
+            resbm.resbm_rmsnorm_bwd(bnd.desc(T), Y, gamma, NORM_EPS, dN.contiguous(),
+                                    None if dY is None else dY.contiguous(), dy, dg, bnd.workspace(T))
+            dgamma = dg.to(gamma.dtype)
+        else:
+            dy = torch.zeros_like(Y) if dY is None else dY.contiguous()
+        resbm.resbm_decode_bwd(bnd.desc(T), dy, B, Wd1, Wd2, dB, dWd1, dWd2, bnd.workspace(T))
+        bnd.timer.stop(ev)
+        if bnd.capture is not None:
+            bnd.capture.update(dY=dy.detach(), dB=dB, dWd1=dWd1, dWd2=dWd2)
+        return dB, dWd1.to(Wd1.dtype), dWd2.to(Wd2.dtype), dgamma, None
+
+
 class Boundary(torch.nn.Module):
     """One ResBM boundary: the encoder on the sending stage, the decoder on the receiving one.
     Weights N(0, 1/fan_in), bf16."""
@@ -187,7 +235,7 @@ class Boundary(torch.nn.Module):
             desc = self.desc(T)
             n = max(resbm.resbm_workspace_bytes(desc, op) for op in
                     (resbm.RESBM_OP_ENCODE_FWD, resbm.RESBM_OP_DECODE_FWD, resbm.RESBM_OP_DECODE_BWD,
-                     resbm.RESBM_OP_ENCODE_BWD))
+                     resbm.RESBM_OP_ENCODE_BWD, resbm.RESBM_OP_DECODE_FWD_RMSNORM, resbm.RESBM_OP_RMSNORM_BWD))
             ws = torch.empty(max(n, 1), dtype=torch.uint8, device=self.We1.device)
             self._ws = {T: ws}
         return ws
@@ -197,6 +245,10 @@ class Boundary(torch.nn.Module):
 
     def decode(self, b):
         return _Decode.apply(b, self.Wd1, self.Wd2, self)
+
+    def decode_norm(self, b, gamma):
+        """(y, RMSNorm(y) * gamma) in one call: the receiving block's attention input with it."""
+        return _DecodeNorm.apply(b, self.Wd1, self.Wd2, gamma, self)
 
 
 def _rope_tables(seq, hd, device):
@@ -228,16 +280,18 @@ class Block(torch.nn.Module):
         self.wqkv, self.wo = w(3 * d, d), w(d, d)
         self.w1, self.w3, self.w2 = w(f, d), w(f, d), w(d, f)
 
-    def attn(self, x, rope):
+    def attn(self, x, rope, normed=None):
+        """Attention of the pre-norm block; normed: RMSNorm(x) * n1 when the caller has it."""
         bsz, seq, d = x.shape
-        qkv = Fn.linear(Fn.rms_norm(x, (d,), self.n1, 1e-5), self.wqkv)
+        u = Fn.rms_norm(x, (d,), self.n1, NORM_EPS) if normed is None else normed
+        qkv = Fn.linear(u, self.wqkv)
         q, k, v = qkv.view(bsz, seq, 3, self.heads, self.hd).permute(2, 0, 3, 1, 4)
         q, k = _rope(q, *rope), _rope(k, *rope)
         o = Fn.scaled_dot_product_attention(q, k, v, is_causal=True)
         return Fn.linear(o.transpose(1, 2).reshape(bsz, seq, d), self.wo)
 
     def ffn(self, h):
-        u = Fn.rms_norm(h, (h.shape[-1],), self.n2, 1e-5)
+        u = Fn.rms_norm(h, (h.shape[-1],), self.n2, NORM_EPS)
         return Fn.linear(Fn.silu(Fn.linear(u, self.w1)) * Fn.linear(u, self.w3), self.w2)
 
 
@@ -281,12 +335,16 @@ class PipelineModel(torch.nn.Module):
                 blk = self.blocks[s * per_stage + j]
                 if j == 0 and s > 0:   # receive: decode the boundary tensor of the previous stage
                     bnd = self.bounds[s - 1]
-                    y = bnd.decode(b).view(bsz, seq, d)
+                    if cfg.fuse_norm:   # the block's attention norm comes out of the decoder
+                        y, n = bnd.decode_norm(b, blk.n1)
+                        y, n = y.view(bsz, seq, d), n.view(bsz, seq, d)
+                    else:
+                        y, n = bnd.decode(b).view(bsz, seq, d), None
                     if cfg.wiring == "A":
                         x = y                                       # pad(b) + D(b)
-                        h = x + blk.attn(x, rope)
+                        h = x + blk.attn(x, rope, n)
                     else:
-                        h = Fn.pad(b, (0, d - r)).view(bsz, seq, d) + blk.attn(y, rope)   # pad(b) + Attn(D(b))
+                        h = Fn.pad(b, (0, d - r)).view(bsz, seq, d) + blk.attn(y, rope, n)   # pad(b) + Attn(D(b))
                 else:
                     h = x + blk.attn(x, rope)
                 z = blk.ffn(h)
@@ -294,7 +352,7 @@ class PipelineModel(torch.nn.Module):
                     b = self.bounds[s].encode(h.reshape(T, d), z.reshape(T, d))
                 else:
                     x = h + z
-        logits = Fn.linear(Fn.rms_norm(x, (d,), self.norm, 1e-5), self.head)
+        logits = Fn.linear(Fn.rms_norm(x, (d,), self.norm, NORM_EPS), self.head)
         return Fn.cross_entropy(logits[:, :-1].reshape(-1, cfg.vocab).float(), tokens[:, 1:].reshape(-1))
 
 

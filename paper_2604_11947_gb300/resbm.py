@@ -19,7 +19,7 @@ RESBM_F32, RESBM_BF16 = 0, 1
 RESBM_ACT_SILU, RESBM_ACT_GELU_TANH, RESBM_ACT_IDENTITY = 0, 1, 2
 (RESBM_OP_ENCODE_FWD, RESBM_OP_DECODE_FWD, RESBM_OP_DECODE_BWD, RESBM_OP_ENCODE_BWD,
  RESBM_OP_BOUNDARY_STEP, RESBM_OP_BOUNDARY_STEP_HOST, RESBM_OP_EFFECTIVE_RANK, RESBM_OP_NEWTON_SCHULZ,
- RESBM_OP_DECODE_FWD_RMSNORM) = range(9)
+ RESBM_OP_DECODE_FWD_RMSNORM, RESBM_OP_RMSNORM_BWD) = range(10)
 RESBM_FLAG_GENERIC = 1
 RESBM_FLAG_LINEAR = 2
 RESBM_FLAG_GEMM = 4
@@ -35,7 +35,7 @@ EXPORTS = ("resbm_version", "resbm_status_string", "resbm_last_cuda_error", "res
            "resbm_encode_bwd", "resbm_boundary_step", "resbm_boundary_step_host",
            "resbm_decode_bwd_noalloc", "resbm_selftest_wait_timeout", "resbm_matrix_workspace_bytes",
            "resbm_newton_schulz", "resbm_effective_rank", "resbm_ffn_down_encode_workspace_bytes",
-           "resbm_ffn_down_encode_fwd", "resbm_decode_fwd_rmsnorm")
+           "resbm_ffn_down_encode_fwd", "resbm_decode_fwd_rmsnorm", "resbm_rmsnorm_bwd")
 
 
 class resbm_desc(ctypes.Structure):
@@ -91,6 +91,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.resbm_encode_fwd.argtypes = [D] + [vp] * 6 + [vp, sz, vp]
     lib.resbm_decode_fwd.restype = i32
     lib.resbm_decode_fwd.argtypes = [D] + [vp] * 4 + [vp, sz, vp]
+    lib.resbm_rmsnorm_bwd.restype = i32
+    lib.resbm_rmsnorm_bwd.argtypes = [D, vp, vp, ctypes.c_float] + [vp] * 4 + [vp, sz, vp]
     lib.resbm_decode_fwd_rmsnorm.restype = i32
     lib.resbm_decode_fwd_rmsnorm.argtypes = [D] + [vp] * 4 + [ctypes.c_float] + [vp] * 2 + [vp, sz, vp]
     lib.resbm_decode_bwd.restype = i32
@@ -208,6 +210,12 @@ def resbm_decode_fwd_rmsnorm(desc, B, Wd1, Wd2, gamma, eps, Y, N, ws, stream=Non
     st = load().resbm_decode_fwd_rmsnorm(ctypes.byref(desc), _p(B), _p(Wd1), _p(Wd2), _p(gamma), float(eps),
                                          _p(Y), _p(N), _p(ws), _nbytes(ws), _stream(stream))
     _check("resbm_decode_fwd_rmsnorm", st)
+
+
+def resbm_rmsnorm_bwd(desc, Y, gamma, eps, dN, dY, dY_out, dgamma, ws, stream=None):
+    st = load().resbm_rmsnorm_bwd(ctypes.byref(desc), _p(Y), _p(gamma), float(eps), _p(dN), _p(dY), _p(dY_out),
+                                  _p(dgamma), _p(ws), _nbytes(ws), _stream(stream))
+    _check("resbm_rmsnorm_bwd", st)
 
 
 def resbm_decode_bwd(desc, dY, B, Wd1, Wd2, dB, dWd1, dWd2, ws, stream=None):

@@ -24,7 +24,7 @@ passes `allow`: per element, the earlier rounding carried into it (half Y's spac
 import numpy as np
 
 TOL = {"f32": 1e-5, "bf16": 2e-2}
-ROWWISE = {"B", "Y", "dB", "dF", "dX", "F", "N"}
+ROWWISE = {"B", "Y", "dB", "dF", "dX", "F", "N", "dY_out"}
 
 
 def bf16_half_spacing(x):

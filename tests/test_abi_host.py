@@ -24,7 +24,7 @@ def declared_functions():
 
 def test_exports_every_declared_symbol(lib):
     names = declared_functions()
-    assert len(names) == 20, names
+    assert len(names) == 21, names
     assert sorted(resbm.EXPORTS) == names
     for n in names:
         assert hasattr(lib, n), n
@@ -232,3 +232,24 @@ def test_decode_fwd_rmsnorm_rejects_bad_arguments(lib):
     f = resbm.make_desc(333, 200, 8, 5, dtype="f32")
     assert resbm.resbm_workspace_bytes(f, resbm.RESBM_OP_DECODE_FWD_RMSNORM) == \
         resbm.resbm_workspace_bytes(f, resbm.RESBM_OP_DECODE_FWD)
+
+
+def test_rmsnorm_bwd_rejects_bad_arguments(lib):
+    A, big = 1 << 40, 1 << 34
+    Y, g, dN, dY, out, dg, ws = (A + i * big for i in range(7))
+    d = resbm.make_desc(16384, 2048, 16, 16)
+    need = resbm.resbm_workspace_bytes(d, resbm.RESBM_OP_RMSNORM_BWD)
+    assert need == 1024 * 2048 * 4
+    fn = lib.resbm_rmsnorm_bwd
+    dp = ctypes.byref(d)
+    assert fn(dp, Y, g, 1e-5, dN, dY, out, dg, ws, 16, None) == resbm.RESBM_ERR_WORKSPACE
+    assert fn(dp, Y, g, -1.0, dN, dY, out, dg, ws, need, None) == resbm.RESBM_ERR_INVALID_ARG
+    assert fn(dp, Y, None, 1e-5, dN, dY, out, dg, ws, need, None) == resbm.RESBM_ERR_INVALID_ARG
+    assert fn(dp, Y, g, 1e-5, dN, dY, out, None, ws, need, None) == resbm.RESBM_ERR_INVALID_ARG
+    assert fn(dp, Y, g, 1e-5, dN, dY, Y + 64, dg, ws, need, None) == resbm.RESBM_ERR_INVALID_ARG     # out overlaps Y
+    assert fn(dp, Y, g, 1e-5, dN, dY, dY + 64, dg, ws, need, None) == resbm.RESBM_ERR_INVALID_ARG    # partial overlap with dY
+    assert fn(dp, Y, g, 1e-5, dN, dY, out, out + 64, ws, need, None) == resbm.RESBM_ERR_INVALID_ARG  # dgamma inside dY_out
+    wide = resbm.make_desc(16, 16392, 16, 16)
+    sz = ctypes.c_size_t(0)
+    assert lib.resbm_rmsnorm_bwd(ctypes.byref(wide), Y, g, 1e-5, dN, None, out, dg, ws, 1 << 30, None) == \
+        resbm.RESBM_ERR_UNSUPPORTED

@@ -7,7 +7,7 @@ import torch
 
 import oracle
 from gpu_helpers import to_host
-from metrics import check
+from metrics import bf16_half_spacing, check
 from paper_2604_11947_gb300 import pipeline, resbm
 
 pytestmark = pytest.mark.gpu
@@ -29,6 +29,11 @@ def _check_boundary(cap, bnd, cfg, merge):
     check("Y", to_host(cap["Y"]), oracle.decode_fwd(B, w["Wd1"], w["Wd2"], cfg.act, merge), "bf16")
     wdB, wdWd1, wdWd2 = oracle.decode_bwd(dY, B, w["Wd1"], w["Wd2"], cfg.act, merge)
     check("dB", dB, wdB, "bf16")
+    if "N" in cap:   # the receiving block's attention input, from the fused decoder + RMSNorm
+        gamma = to_host(cap["gamma"])
+        wY2, wN = oracle.decode_fwd_rmsnorm(B, w["Wd1"], w["Wd2"], gamma, pipeline.NORM_EPS, cfg.act, merge)
+        rstd = 1.0 / np.sqrt(np.mean(wY2 * wY2, axis=1, keepdims=True) + pipeline.NORM_EPS)
+        check("N", to_host(cap["N"]), wN, "bf16", allow=bf16_half_spacing(wY2) * np.abs(rstd * gamma[None, :]))
     check("dWd1", to_host(cap["dWd1"]), wdWd1, "bf16")
     check("dWd2", to_host(cap["dWd2"]), wdWd2, "bf16")
     wdF, wdX, wdWe1, wdWe2 = oracle.encode_bwd(dB_in, F, w["We1"], w["We2"], cfg.act)
@@ -93,4 +98,24 @@ def test_both_wirings_learn_the_markov_stream():
         curve = res[name]
         first, last = curve[0][1], curve[-1][1]
         assert np.isfinite(last) and last < 0.6 * first, (name, curve)
+    assert resbm.resbm_device_error() == 0
+
+
+@pytest.mark.parametrize("wiring", ["A", "B"])
+def test_fused_norm_matches_the_unfused_model(wiring):
+    """The same model with the receiving block's RMSNorm fused into the decoder and without: the
+    loss and every gradient agree to bf16 noise (the fused N skips one rounding of y)."""
+    cfg = pipeline.PipelineConfig(layers=4, d=512, heads=4, ffn=1024, vocab=1000, stages=2, r=16, m=16,
+                                  batch=2, seq=256, wiring=wiring)
+    tokens = pipeline.synthetic_tokens(cfg)
+    grads, losses = [], []
+    for fuse in (True, False):
+        model = pipeline.PipelineModel(cfg.with_(fuse_norm=fuse))
+        losses.append(float(pipeline.train_step(model, tokens)))
+        grads.append({k: p.grad.float().clone() for k, p in model.named_parameters()})
+    assert abs(losses[0] - losses[1]) < 1e-3 * abs(losses[1])
+    for k in grads[1]:
+        a, b = grads[0][k], grads[1][k]
+        rel = float((a - b).norm() / b.norm().clamp_min(1e-30))
+        assert rel < 3e-2, (k, rel)
     assert resbm.resbm_device_error() == 0
