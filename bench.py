@@ -499,6 +499,39 @@ def decode_rmsnorm_workload(resbm, torch, peaks, steps=50, warmup=5):
         gbs = alg[name] / (ms / 1e3) / 1e9
         res[name] = {"ms": ms, "alg_bytes": alg[name], "GBps": gbs, "frac": gbs / peaks["hbm_gbs"]}
     res["bytes_saved_by_fusion"] = alg["unfused_decode_then_torch_rms_norm"] - alg["fused"]
+    # the backward: resbm_rmsnorm_bwd (dY + the norm's input gradient, dgamma) against torch's
+    # rms_norm backward (autograd of a recomputed forward) followed by the residual add
+    dN = torch.randn(T, d, device="cuda", generator=g).to(torch.bfloat16)
+    dYr = torch.randn(T, d, device="cuda", generator=g).to(torch.bfloat16)
+    dYo = torch.empty_like(dYr)
+    dgam = torch.empty(d, dtype=torch.float32, device="cuda")
+    ws_b = resbm.workspace(desc, resbm.RESBM_OP_RMSNORM_BWD)
+    Yl = Y.detach().clone().requires_grad_(True)
+    gl = gamma.detach().clone().requires_grad_(True)
+
+    def torch_bwd():
+        n = torch.nn.functional.rms_norm(Yl, (d,), gl, eps)
+        gy, gg = torch.autograd.grad(n, (Yl, gl), dN)
+        return gy + dYr, gg
+
+    bruns = {"norm_bwd_resbm": lambda: resbm.resbm_rmsnorm_bwd(desc, Y, gamma, eps, dN, dYr, dYo, dgam, ws_b),
+             "norm_bwd_torch_then_add": torch_bwd}
+    balg = {"norm_bwd_resbm": 4 * T * d * 2 + 2 * d + 4 * d, "norm_bwd_torch_then_add": None}
+    for name, fn in bruns.items():
+        for _ in range(warmup):
+            fn()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(steps):
+            fn()
+        b.record()
+        torch.cuda.synchronize()
+        ms = a.elapsed_time(b) / steps
+        res[name] = {"ms": ms}
+        if balg[name]:
+            gbs = balg[name] / (ms / 1e3) / 1e9
+            res[name].update(alg_bytes=balg[name], GBps=gbs, frac=gbs / peaks["hbm_gbs"])
     return res
 
 
