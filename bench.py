@@ -757,6 +757,11 @@ def run_e2e(args, cfg, w, resbm, torch, dist, world):
         h["dX"] = torch.zeros(out["dX"].shape, dtype=out["dX"].dtype).pin_memory()
     wss = [resbm.workspace(desc, resbm.RESBM_OP_BOUNDARY_STEP_HOST) for _ in range(2)]
     streams = [torch.cuda.Stream() for _ in range(2)]
+    # call k+1's copies in wait for call k's (resbm_step_args.wait_before_inputs / inputs_done):
+    # one call's inputs travel in while the previous call's results travel out
+    in_done = [torch.cuda.Event() for _ in range(2)]
+    for ev, st in zip(in_done, streams):
+        ev.record(st)
     es = host_in["F"].element_size()
     cols = cfg.T * cfg.r * es   # X[:, :r] and dX[:, :r]: the only columns of X and dX the step uses
     # what the call copies: X[:, :r], dX[:, :r], F, dY and the weights in; the results and
@@ -770,7 +775,8 @@ def run_e2e(args, cfg, w, resbm, torch, dist, world):
 
     def step(i):
         b = i % 2
-        resbm.resbm_boundary_step_host(desc, wss[b], stream=streams[b], **host_in, **host_out[b])
+        resbm.resbm_boundary_step_host(desc, wss[b], stream=streams[b], wait_before_inputs=in_done[1 - b],
+                                       inputs_done=in_done[b], **host_in, **host_out[b])
 
     for i in range(2):
         step(i)
@@ -786,8 +792,9 @@ def run_e2e(args, cfg, w, resbm, torch, dist, world):
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": n,
             "ms_per_step": ms / n, "host_link": host_link(torch),
             "api": "resbm_boundary_step_host (host buffers; copies inside the call; dX[:, :r] += dB)",
-            "pipelined": "two calls in flight on two streams with two device workspaces; "
-                         "host wall clock from the first copy to the last result on the host"}
+            "pipelined": "two calls in flight on two streams with two device workspaces, each call's "
+                         "copies in chained after the previous call's (events); host wall clock from the "
+                         "first copy to the last result on the host"}
 
 
 if __name__ == "__main__":

@@ -130,6 +130,10 @@ typedef struct {
     void *dF;                               /* out: T x d                                     */
     void *dX;                               /* in/out: T x d, first r columns += dB; or NULL  */
     float *dWe1, *dWe2, *dWd1, *dWd2;       /* out: fp32 weight gradients                     */
+    /* resbm_boundary_step_host only (ignored by resbm_boundary_step; NULL for none): CUDA event
+     * handles (cudaEvent_t) that chain the host-link phases of consecutive calls */
+    void *wait_before_inputs;               /* the call's host-to-device copies wait for it   */
+    void *inputs_done;                      /* recorded when all its host-to-device copies are done */
 } resbm_step_args;
 
 /* Library version string, e.g. "resbm 0.1.0 sm_103a". */
@@ -289,10 +293,16 @@ RESBM_API resbm_status resbm_boundary_step(const resbm_desc *desc, const resbm_s
  *     backward stages run; both are forked from and joined back into `stream`. Calls on
  *     different streams with different workspaces may run at the same time, so a caller can
  *     overlap one step's results with the next step's inputs.
- *   - The two side streams and four events are created on the first call for each (device,
+ *   - Pipelining calls: with two calls in flight on two streams, nothing orders their copies, so
+ *     both calls' inputs share the host-to-device direction at once and both results the other
+ *     way. Passing call k's `inputs_done` event as call k+1's `wait_before_inputs` makes call k+1's
+ *     inputs travel in while call k computes and sends its results back, one transfer per
+ *     direction on the host link. Both events are optional; each call waits only on an event a
+ *     call enqueued before it recorded, so the chain cannot deadlock.
+ *   - The two side streams and five events are created on the first call for each (device,
  *     caller stream) pair and kept until the process exits (creating them in every call costs
  *     driver time). A caller that passes a new stream to every call therefore accumulates two
- *     streams and four events per distinct stream handle: reuse a small set of streams.
+ *     streams and five events per distinct stream handle: reuse a small set of streams.
  *   - Errors: as resbm_boundary_step; RESBM_ERR_CUDA if a copy or a stream could not be set up. */
 RESBM_API resbm_status resbm_boundary_step_host(const resbm_desc *desc, const resbm_step_args *args,
                                       void *ws, size_t ws_bytes, void *stream);

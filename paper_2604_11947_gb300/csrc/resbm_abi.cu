@@ -67,7 +67,7 @@ bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 // keeps two host threads from interleaving their enqueues on one entry.
 struct SideStreams {
     cudaStream_t in = nullptr, out = nullptr;
-    cudaEvent_t ev[4] = {};
+    cudaEvent_t ev[5] = {};
     std::mutex mu;
 };
 cudaError_t side_streams(cudaStream_t caller, SideStreams **out)
@@ -83,7 +83,7 @@ cudaError_t side_streams(cudaStream_t caller, SideStreams **out)
         std::unique_ptr<SideStreams> s(new SideStreams);
         e = cudaStreamCreateWithFlags(&s->in, cudaStreamNonBlocking);
         if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&s->out, cudaStreamNonBlocking);
-        for (int i = 0; i < 4 && e == cudaSuccess; ++i) e = cudaEventCreateWithFlags(&s->ev[i], cudaEventDisableTiming);
+        for (int i = 0; i < 5 && e == cudaSuccess; ++i) e = cudaEventCreateWithFlags(&s->ev[i], cudaEventDisableTiming);
         if (e != cudaSuccess) {
             if (s->in) cudaStreamDestroy(s->in);
             if (s->out) cudaStreamDestroy(s->out);
@@ -907,6 +907,7 @@ resbm_status resbm_boundary_step_host(const resbm_desc *desc, const resbm_step_a
     std::lock_guard<std::mutex> hold(side->mu);
     cudaStream_t s_in = side->in, s_out = side->out;
     cudaEvent_t fork = side->ev[0], dy_in = side->ev[1], fwd_done = side->ev[2], out_done = side->ev[3];
+    cudaEvent_t main_in = side->ev[4];
     auto h2d = [&](void *dst, const void *src, size_t bytes, cudaStream_t st) {
         if (e == cudaSuccess && bytes) e = cudaMemcpyAsync(dst, src, bytes, cudaMemcpyHostToDevice, st);
     };
@@ -936,6 +937,8 @@ resbm_status resbm_boundary_step_host(const resbm_desc *desc, const resbm_step_a
     };
     // inputs: what the forward reads first, on the caller's stream; then dY on the second
     // stream, travelling in while the forward runs and its results travel out
+    if (a->wait_before_inputs)   // after the copies of the call that recorded it (a caller's chain)
+        e = cudaStreamWaitEvent(c.stream, static_cast<cudaEvent_t>(a->wait_before_inputs), 0);
     h2d(const_cast<void *>(dv.We1), a->We1, (size_t)(D * m) * es, c.stream);
     if (!lin) h2d(const_cast<void *>(dv.We2), a->We2, (size_t)(m * r) * es, c.stream);
     if (!lin) h2d(const_cast<void *>(dv.Wd1), a->Wd1, (size_t)(r * m) * es, c.stream);
@@ -947,6 +950,11 @@ resbm_status resbm_boundary_step_host(const resbm_desc *desc, const resbm_step_a
     h2d(const_cast<void *>(dv.dY), a->dY, (size_t)(T * D) * es, s_in);
     if (e == cudaSuccess) e = cudaEventRecord(dy_in, s_in);
     if (a->dX) cols(dv.dX, a->dX, cudaMemcpyHostToDevice, c.stream);          // the step adds dB to dX[:, :r] only
+    if (a->inputs_done && e == cudaSuccess) {   // once both streams' copies in are done
+        e = cudaEventRecord(main_in, c.stream);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(s_in, main_in, 0);
+        if (e == cudaSuccess) e = cudaEventRecord(static_cast<cudaEvent_t>(a->inputs_done), s_in);
+    }
     if (e != cudaSuccess) s = cuda_fail(e);
     // the step, the forward results leaving on the third stream while the backward runs
     if (s == RESBM_OK) s = enqueue_step(d, dv, hs.inner, c, fwd_done, dy_in);

@@ -47,7 +47,7 @@ class resbm_desc(ctypes.Structure):
 class resbm_step_args(ctypes.Structure):
     _fields_ = [(n, ctypes.c_void_p) for n in
                 ("X", "F", "dY", "We1", "We2", "Wd1", "Wd2", "B", "P", "Y", "dB", "dF", "dX",
-                 "dWe1", "dWe2", "dWd1", "dWd2")]
+                 "dWe1", "dWe2", "dWd1", "dWd2", "wait_before_inputs", "inputs_done")]
 
 
 class ResbmError(RuntimeError):
@@ -247,10 +247,22 @@ def resbm_boundary_step(desc, ws, stream=None, **tensors):
     _check("resbm_boundary_step", st)
 
 
-def resbm_boundary_step_host(desc, ws, stream=None, **tensors):
+def _event(ev):
+    """The cudaEvent_t handle of a torch.cuda.Event (recorded once already, so that it exists)."""
+    if ev is None:
+        return None
+    h = ev.cuda_event if hasattr(ev, "cuda_event") else int(ev)
+    if not h:
+        raise ValueError("the event has no CUDA handle yet: record it once first")
+    return h
+
+
+def resbm_boundary_step_host(desc, ws, stream=None, wait_before_inputs=None, inputs_done=None, **tensors):
     """resbm_boundary_step with host tensors (CPU torch tensors, pinned for asynchronous
-    copies); ws is the device workspace of RESBM_OP_BOUNDARY_STEP_HOST."""
-    args = resbm_step_args(**{k: _p(v) for k, v in tensors.items()})
+    copies); ws is the device workspace of RESBM_OP_BOUNDARY_STEP_HOST. wait_before_inputs /
+    inputs_done: torch.cuda.Event objects chaining consecutive calls' host-to-device copies."""
+    args = resbm_step_args(**{k: _p(v) for k, v in tensors.items()},
+                           wait_before_inputs=_event(wait_before_inputs), inputs_done=_event(inputs_done))
     st = load().resbm_boundary_step_host(ctypes.byref(desc), ctypes.byref(args), _p(ws), _nbytes(ws),
                                          _stream(stream))
     _check("resbm_boundary_step_host", st)

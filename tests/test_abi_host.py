@@ -41,7 +41,7 @@ def test_version_and_status_strings(lib):
 
 def test_struct_layout_matches_header():
     assert ctypes.sizeof(resbm.resbm_desc) == 4 * 8 + 4 * 4
-    assert ctypes.sizeof(resbm.resbm_step_args) == 17 * ctypes.sizeof(ctypes.c_void_p)
+    assert ctypes.sizeof(resbm.resbm_step_args) == 19 * ctypes.sizeof(ctypes.c_void_p)
 
 
 @pytest.mark.parametrize("op", range(6))

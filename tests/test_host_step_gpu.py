@@ -106,6 +106,35 @@ def test_host_steps_on_two_streams_at_once():
             _same(out, want, x0, cfg.r)
 
 
+def test_host_steps_chained_by_events():
+    """Calls on two streams whose host-to-device phases are chained (call k+1 waits for call k's
+    inputs_done): every call still gives the device step's results bit for bit."""
+    cfg, flags = CASES["bf16_tc"]
+    desc = resbm.desc_from_config(cfg, flags)
+    runs = [_host_args(cfg, desc, flags, True, seed=s) for s in (3, 4)]
+    wants = [_device_reference(desc, h, out) for h, out in runs]
+    streams = [torch.cuda.Stream() for _ in runs]
+    wss = [resbm.workspace(desc, resbm.RESBM_OP_BOUNDARY_STEP_HOST) for _ in runs]
+    evs = [torch.cuda.Event() for _ in runs]
+    for e, st in zip(evs, streams):
+        e.record(st)          # gives each event its CUDA handle
+    dX0 = [out["dX"].clone() for _, out in runs]
+    prev = None
+    for i in range(6):
+        b = i % 2
+        h, out = runs[b]
+        streams[b].synchronize()   # the previous call on this stream has finished with out["dX"]
+        out["dX"].copy_(dX0[b])
+        resbm.resbm_boundary_step_host(desc, wss[b], stream=streams[b], wait_before_inputs=prev, inputs_done=evs[b],
+                                       **h, **out)
+        prev = evs[b]
+    for st in streams:
+        st.synchronize()
+    for (h, out), want, x0 in zip(runs, wants, dX0):
+        _same(out, want, x0, cfg.r)
+    assert resbm.resbm_device_error() == 0
+
+
 def test_host_step_empty_batch():
     """T = 0: nothing to copy in; the weight gradients come back as zeros."""
     cfg = synth.BoundaryConfig("hs_empty", T=0, d=256, r=16, m=16)
