@@ -38,8 +38,9 @@ class PipelineConfig:
     ffn: int = 5632
     vocab: int = 32000
     stages: int = 4
-    r: int = 16              # bottleneck width of every boundary (d / r compression)
-    m: int = 16              # hidden width of the boundary's encoder / decoder
+    r: object = 16           # bottleneck width (d / r compression): one int for every boundary, or a
+                             # tuple of stages - 1 widths (a non-uniform r per boundary)
+    m: object = 16           # hidden width of the encoder / decoder: an int, or one per boundary
     batch: int = 8
     seq: int = 2048
     act: str = "silu"
@@ -55,6 +56,11 @@ class PipelineConfig:
     @property
     def tokens(self) -> int:
         return self.batch * self.seq
+
+    def boundary_widths(self, k: int):
+        """(r, m) of boundary k (between stage k and stage k + 1)."""
+        pick = lambda v: int(v[k]) if isinstance(v, (tuple, list)) else int(v)
+        return pick(self.r), pick(self.m)
 
 
 # The workload the boundary's share of a training step is measured on: 24 layers, d = 2048,
@@ -309,8 +315,10 @@ class PipelineModel(torch.nn.Module):
             torch.randn(cfg.vocab, cfg.d, generator=gen, device=device, dtype=torch.float32).to(torch.bfloat16))
         self.blocks = torch.nn.ModuleList(Block(cfg, gen, device) for _ in range(cfg.layers))
         merge = 1 if cfg.wiring == "A" else 0
-        self.bounds = torch.nn.ModuleList(Boundary(cfg.d, cfg.r, cfg.m, cfg.act, merge, self.timer, gen, device,
-                                                   cfg.flags) for _ in range(cfg.stages - 1))
+        for v in (cfg.r, cfg.m):
+            assert not isinstance(v, (tuple, list)) or len(v) == cfg.stages - 1, "one width per boundary"
+        self.bounds = torch.nn.ModuleList(Boundary(cfg.d, *cfg.boundary_widths(k), cfg.act, merge, self.timer, gen,
+                                                   device, cfg.flags) for k in range(cfg.stages - 1))
         self.norm = torch.nn.Parameter(torch.ones(cfg.d, device=device, dtype=torch.bfloat16))
         self.head = torch.nn.Parameter(
             (torch.randn(cfg.vocab, cfg.d, generator=gen, device=device, dtype=torch.float32) * 0.02).to(torch.bfloat16))
@@ -325,7 +333,7 @@ class PipelineModel(torch.nn.Module):
         """Mean next-token cross-entropy of a (batch, seq) tensor of token ids."""
         cfg = self.cfg
         bsz, seq = tokens.shape
-        T, d, r = bsz * seq, cfg.d, cfg.r
+        T, d = bsz * seq, cfg.d
         rope = self.rope(seq, tokens.device)
         per_stage = cfg.layers // cfg.stages
         x = Fn.embedding(tokens, self.embed)
@@ -344,7 +352,7 @@ class PipelineModel(torch.nn.Module):
                         x = y                                       # pad(b) + D(b)
                         h = x + blk.attn(x, rope, n)
                     else:
-                        h = Fn.pad(b, (0, d - r)).view(bsz, seq, d) + blk.attn(y, rope, n)   # pad(b) + Attn(D(b))
+                        h = Fn.pad(b, (0, d - bnd.r)).view(bsz, seq, d) + blk.attn(y, rope, n)   # pad(b) + Attn(D(b))
                 else:
                     h = x + blk.attn(x, rope)
                 z = blk.ffn(h)

@@ -39,8 +39,9 @@ def _check_boundary(cap, bnd, cfg, merge):
     wdF, wdX, wdWe1, wdWe2 = oracle.encode_bwd(dB_in, F, w["We1"], w["We2"], cfg.act)
     check("dF", to_host(cap["dF"]), wdF, "bf16")
     dX = to_host(cap["dX"])
-    assert not np.any(dX[:, cfg.r:]), "the identity path's gradient reaches only the first r columns"
-    check("dX", dX[:, :cfg.r], wdX[:, :cfg.r], "bf16")
+    r = bnd.r
+    assert not np.any(dX[:, r:]), "the identity path's gradient reaches only the first r columns"
+    check("dX", dX[:, :r], wdX[:, :r], "bf16")
     check("dWe1", to_host(cap["dWe1"]), wdWe1, "bf16")
     check("dWe2", to_host(cap["dWe2"]), wdWe2, "bf16")
 
@@ -67,7 +68,7 @@ def test_four_stage_pipeline_boundaries_match_oracle():
     model, caps = _run(cfg)
     assert len(caps) == 3
     for cap, bnd in zip(caps, model.bounds):
-        assert cap["X"].shape == (cfg.tokens, cfg.d) and cap["B"].shape == (cfg.tokens, cfg.r)
+        assert cap["X"].shape == (cfg.tokens, cfg.d) and cap["B"].shape == (cfg.tokens, bnd.r)
         _check_boundary(cap, bnd, cfg, merge=1)
     assert resbm.resbm_device_error() == 0
 
@@ -79,6 +80,19 @@ def test_reading_b_wiring_boundaries_match_oracle():
                                   batch=2, seq=256, wiring="B")
     model, caps = _run(cfg)
     _check_boundary(caps[0], model.bounds[0], cfg, merge=0)
+
+
+def test_non_uniform_bottleneck_widths():
+    """A different r (and m) at each boundary (the paper allows the compression to vary per
+    boundary): r = 16, 32, 64 over three boundaries, every boundary against the oracle."""
+    cfg = pipeline.PipelineConfig(layers=4, d=512, heads=4, ffn=1024, vocab=1000, stages=4, r=(16, 32, 64),
+                                  m=(16, 32, 64), batch=2, seq=256)
+    model, caps = _run(cfg)
+    assert [b.r for b in model.bounds] == [16, 32, 64]
+    for cap, bnd in zip(caps, model.bounds):
+        assert cap["B"].shape == (cfg.tokens, bnd.r)
+        _check_boundary(cap, bnd, cfg, merge=1)
+    assert resbm.resbm_device_error() == 0
 
 
 def test_boundary_share_is_measured():

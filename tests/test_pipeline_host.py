@@ -35,3 +35,13 @@ def test_model_structure():
     # the full workload: 24 layers in 4 stages, three boundaries of 128x compression
     full = pipeline.PIPELINE
     assert full.layers // full.stages == 6 and full.d // full.r == 128 and full.tokens == 16384
+
+
+def test_per_boundary_widths():
+    cfg = pipeline.PipelineConfig(layers=4, d=64, heads=4, ffn=128, vocab=50, stages=4, r=(8, 16, 32), m=(8, 16, 32),
+                                  batch=2, seq=16)
+    assert [cfg.boundary_widths(k) for k in range(3)] == [(8, 8), (16, 16), (32, 32)]
+    m = pipeline.PipelineModel(cfg, device="cpu")
+    assert [(b.r, b.m) for b in m.bounds] == [(8, 8), (16, 16), (32, 32)]
+    assert m.bounds[2].We2.shape == (32, 32) and m.bounds[0].Wd2.shape == (8, 64)
+    assert pipeline.PIPELINE.boundary_widths(2) == (16, 16)
