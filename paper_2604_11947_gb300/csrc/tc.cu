@@ -470,12 +470,14 @@ int gemm_splits(int64_t M, int64_t N, int64_t K, int sms, int rows = 128)
 // MC: CTA pairs sharing B by multicast (k_gemm); the grid is then two CTAs per co-resident pair,
 // at most one pair per pair unit (returns cudaErrorNotSupported, before launching, when no pair
 // fits: the caller runs single CTAs).
-template <int BN, bool AMN, bool BMN, bool ALO, bool ENCP = false, bool MC = false, bool BM2 = false>
+// TS: the output leaves by TMA stores through `mo` (k_gemm's TS form); otherwise `mo` is not read.
+template <int BN, bool AMN, bool BMN, bool ALO, bool ENCP = false, bool MC = false, bool BM2 = false, bool TS = false>
 cudaError_t launch_gemm_t(const CUtensorMap &ma, const CUtensorMap &malo, const CUtensorMap &mb,
-                          const tc::GemmShape &g, const tc::GemmEp &ep, const Ctx &c)
+                          const tc::GemmShape &g, const tc::GemmEp &ep, const Ctx &c, const CUtensorMap *mo = nullptr)
 {
-    using Cfg = tc::GemmCfg<BN, ALO, BM2>;
-#define RESBM_KGEMM tc::k_gemm<BN, AMN, BMN, ALO, ENCP, MC, BM2>
+    using Cfg = tc::GemmCfg<BN, ALO, BM2, TS>;
+    const CUtensorMap &mout = mo ? *mo : ma;
+#define RESBM_KGEMM tc::k_gemm<BN, AMN, BMN, ALO, ENCP, MC, BM2, TS>
     static std::atomic<uint8_t> smem_set[kMaxDev];
     cudaError_t e = ensure_smem(RESBM_KGEMM, Cfg::SMEM_BYTES, c.device, smem_set);
     if (e != cudaSuccess) return e;
@@ -487,15 +489,23 @@ cudaError_t launch_gemm_t(const CUtensorMap &ma, const CUtensorMap &malo, const 
         const int64_t pairs = pair_units < pairs_fit ? pair_units : pairs_fit;
         if (pairs < 1) return cudaErrorNotSupported;
         e = launch_clustered(RESBM_KGEMM, (unsigned)(2 * pairs), Cfg::THREADS,
-                             Cfg::SMEM_BYTES, 2, c.stream, ma, malo, mb, g, ep);
+                             Cfg::SMEM_BYTES, 2, c.stream, ma, malo, mb, mout, g, ep);
     } else {
         const int64_t grid = g.units < c.sm_count ? g.units : c.sm_count;
         e = launch(RESBM_KGEMM, (unsigned)grid, Cfg::THREADS, Cfg::SMEM_BYTES, c.stream, ma,
-                   malo, mb, g, ep);
+                   malo, mb, mout, g, ep);
     }
 #undef RESBM_KGEMM
     count_launches(1);
     return e;
+}
+
+// The TMA-store epilogue (k_gemm's TS form) unless RESBM_GEMM_TS=0 (read at every launch; a tuning
+// and testing knob: both forms store the same bits).
+bool ts_enabled()
+{
+    const char *v = getenv("RESBM_GEMM_TS");
+    return !(v && v[0] == '0' && v[1] == 0);
 }
 
 // Pairs sharing B by multicast for the 256-column products with at least two row blocks, unless
@@ -545,6 +555,18 @@ cudaError_t gemm(const Ctx &c, int64_t M, int64_t N, int64_t K, const void *A, b
         if (!a_mn && !b_mn) return launch_gemm_t<256, false, false, false, false, false, true>(ma, malo, mbm, g, ep, c);
         if (a_mn && b_mn) return launch_gemm_t<256, true, true, false, false, false, true>(ma, malo, mbm, g, ep, c);
         return cudaErrorNotSupported;
+    }
+    // TMA-store epilogue for the pairs' plain bf16 outputs (Y = G . Wd2 + pad(B), dF = dP . We1^T)
+    CUtensorMap mo;
+    const bool ts = pair && !a_mn && !(b_mn && lo) && g.splits == 1 &&
+                    (ep.mode == tc::GEP_BF16 || ep.mode == tc::GEP_ADD_AUX || ep.mode == tc::GEP_DF) &&
+                    al16(ep.out) && (ep.ldo * 2) % 16 == 0 && ts_enabled() &&
+                    make_map(&mo, ep.out, N, M, ep.ldo * 2, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B);
+    if (ts) {
+        cudaError_t e = b_mn ? launch_gemm_t<256, false, true, false, false, true, false, true>(ma, malo, mbm, g, ep, c, &mo)
+                        : lo ? launch_gemm_t<256, false, false, true, false, true, false, true>(ma, malo, mbm, g, ep, c, &mo)
+                             : launch_gemm_t<256, false, false, false, false, true, false, true>(ma, malo, mbm, g, ep, c, &mo);
+        if (e != cudaErrorNotSupported) return e;
     }
     if (pair) {
         cudaError_t e = cudaErrorNotSupported;

@@ -131,14 +131,22 @@ struct GemmShape {
 
 // BM2: 256-row units, two 128-row A sub-tiles per stage against one B tile, the two halves'
 // accumulators side by side in TMEM (one unit at a time: no accumulator double buffering).
-template <int BN_, bool ALO_ = false, bool BM2_ = false> struct GemmCfg {
+// TS: the output tile leaves by TMA stores from a shared-memory staging box per half of the
+// epilogue warps (128 rows x 64 columns of bf16, 128-byte swizzle), for the products that write
+// T x d bf16 tensors: per-thread 16-byte stores of 32 different rows per warp instruction made
+// the epilogue, not the products, set such a product's pace.
+template <int BN_, bool ALO_ = false, bool BM2_ = false, bool TS_ = false> struct GemmCfg {
     static constexpr int BN = BN_;
     static constexpr uint32_t A_TILE = 128 * 64 * 2;        // 128 rows x 64 K, bf16
     static constexpr uint32_t A_STAGE = A_TILE * (ALO_ ? 2 : 1) * (BM2_ ? 2 : 1);   // hi (+ lo), per half
     static constexpr uint32_t B_STAGE = BN_ * 64 * 2;       // BN rows x 64 K, bf16
     static constexpr uint32_t STAGE = A_STAGE + B_STAGE;
-    static constexpr int NST = (200 * 1024) / STAGE;        // 4 stages at BN = 256, 6 at 128 (3, 4 with lo; 3 for BM2)
-    static constexpr uint32_t SMEM_BYTES = NST * STAGE + 1024;
+    static constexpr uint32_t STG_HALF = 128 * 64 * 2;      // TS: one half's staging box
+    static constexpr uint32_t STG_BYTES = TS_ ? 2 * STG_HALF : 0;
+    // 4 stages at BN = 256, 6 at 128 (3, 4 with lo; 3 for BM2; one fewer with TS)
+    static constexpr int NST = (200 * 1024 - (int)STG_BYTES) / (int)STAGE;
+    static constexpr uint32_t OFF_STG = NST * STAGE;        // 1024-aligned (STAGE is)
+    static constexpr uint32_t SMEM_BYTES = NST * STAGE + STG_BYTES + 1024;
     static_assert(SMEM_BYTES <= 232448 - 512, "shared memory budget");
     static constexpr uint32_t TMEM_COLS = 2 * BN_;          // two accumulators
     static_assert(TMEM_COLS <= 512, "TMEM budget");
@@ -297,7 +305,33 @@ __device__ __forceinline__ void gemm_epilogue(const GemmEp &ep, int64_t row, int
     }
 }
 
-// tma_lo: the lo matrix of A (same shape and layout as A; read only with ALO)
+// TS: the values of an output tile's 32 columns as gemm_epilogue computes them, without its bf16
+// store (the caller stages them for a TMA store). Only GEP_BF16, GEP_ADD_AUX and GEP_DF; GEP_DF's
+// dX[:, :r] read-modify-write still goes to global memory. in_rows: row < M and col < N.
+__device__ __forceinline__ void gemm_epilogue_ts(const GemmEp &ep, int64_t row, int64_t col, float (&v)[32], int nv,
+                                                 bool in_rows)
+{
+    if (!in_rows) return;
+    if (ep.mode == GEP_ADD_AUX && col < ep.aux_cols) {
+        const int na = ep.aux_cols - col < nv ? (int)(ep.aux_cols - col) : nv;
+        float x[32];
+        ld_bf16x32(static_cast<const __nv_bfloat16 *>(ep.aux) + row * ep.lda + col, x, na);
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] = j < na ? v[j] + x[j] : v[j];
+    } else if (ep.mode == GEP_DF && ep.rmw && col < ep.aux_cols) {
+        const int na = ep.aux_cols - col < nv ? (int)(ep.aux_cols - col) : nv;
+        float x[32], y[32];
+        __nv_bfloat16 *r = ep.rmw + row * ep.ldr + col;
+        ld_bf16x32(r, y, na);
+        ld_bf16x32(static_cast<const __nv_bfloat16 *>(ep.aux) + row * ep.lda + col, x, na);
+#pragma unroll
+        for (int j = 0; j < 32; ++j) y[j] += x[j];
+        st_bf16x32(r, y, na);
+    }
+}
+
+// tma_lo: the lo matrix of A (same shape and layout as A; read only with ALO); tmo: the output
+// (bf16, N x M, boxes of 64 columns x 128 rows, 128-byte swizzle; read only with TS)
 // ENCP: the epilogue of the encoder fused into the FFN down-projection (the GemmEp ENCP fields)
 // instead of gemm_epilogue.
 // BM2 (GemmCfg): units of 256 rows (two 128-row MMAs per K step sharing the B tile, ~128 flop per
@@ -308,13 +342,16 @@ __device__ __forceinline__ void gemm_epilogue(const GemmEp &ep, int64_t row, int
 // reads 2/3 of a stage's bytes from L2. A stage's `empty` barrier then takes an arrival from both
 // CTAs' MMA commits (multicast), so neither refills it before both have read it. (For K-major B
 // the tensor map's box is BN / 2 rows.)
-template <int BN, bool AMN, bool BMN, bool ALO, bool ENCP = false, bool MC = false, bool BM2 = false>
+template <int BN, bool AMN, bool BMN, bool ALO, bool ENCP = false, bool MC = false, bool BM2 = false,
+          bool TS = false>
 __global__ void __launch_bounds__(320, 1)
     k_gemm(const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tma_lo,
-           const __grid_constant__ CUtensorMap tmb, const GemmShape g, const GemmEp ep)
+           const __grid_constant__ CUtensorMap tmb, const __grid_constant__ CUtensorMap tmo, const GemmShape g,
+           const GemmEp ep)
 {
-    using C = GemmCfg<BN, ALO, BM2>;
+    using C = GemmCfg<BN, ALO, BM2, TS>;
     static_assert(!(BM2 && (ALO || MC)), "256-row units without hi + lo A or pairs");
+    static_assert(!(TS && (ENCP || BM2)), "TMA-store epilogue: plain 128-row units");
     constexpr int MH = BM2 ? 2 : 1;   // 128-row halves per unit (g.nm counts units of 128 * MH rows)
     griddep_wait();               // the previous kernel of the stream has completed
     griddep_launch_dependents();  // the next one may be scheduled on SMs as they free up
@@ -514,8 +551,47 @@ __global__ void __launch_bounds__(320, 1)
 #pragma unroll
                     for (int j = 0; j < 32; ++j) pacc[j] = 0.0f;
                 }
+                if (TS) {
+                    // 64 columns at a time through this half's staging box, stored by one thread
+                    const bool issuer = q == 0 && lane == 0;
+                    uint8_t *stg = smem + C::OFF_STG + half * C::STG_HALF;
 #pragma unroll 1
-                for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 32) {
+                    for (int c0 = half * (BN / 2); c0 < (half + 1) * (BN / 2); c0 += 64) {
+                        if (issuer) bulk_wait_read<0>();   // the box's previous store has read it
+                        named_barrier(1 + half, 128);
+                        float v2[2][32];
+                        tmem_ld32(tmem + lane_base + acc_col + c0, v2[0]);   // warp-collective: every lane
+                        tmem_ld32(tmem + lane_base + acc_col + c0 + 32, v2[1]);
+                        tmem_ld_wait();
+                        tmem_regs_ready(v2[0]);
+                        tmem_regs_ready(v2[1]);
+#pragma unroll
+                        for (int hh = 0; hh < 2; ++hh) {
+                            const int64_t col = (int64_t)nb * BN + c0 + 32 * hh;
+                            const int nv = g.N - col < 32 ? (int)(g.N - col) : 32;
+                            gemm_epilogue_ts(ep, row, col, v2[hh], nv, row < g.M && col < g.N);
+                            uint32_t pk[16];
+#pragma unroll
+                            for (int e = 0; e < 16; ++e) {
+                                __nv_bfloat162 b2 = __floats2bfloat162_rn(v2[hh][2 * e], v2[hh][2 * e + 1]);
+                                pk[e] = *reinterpret_cast<uint32_t *>(&b2);
+                            }
+#pragma unroll
+                            for (int e = 0; e < 4; ++e)
+                                *reinterpret_cast<uint4 *>(stg + swz_offset((uint32_t)rin, 64 * hh + 16 * e, 128)) =
+                                    make_uint4(pk[4 * e], pk[4 * e + 1], pk[4 * e + 2], pk[4 * e + 3]);
+                        }
+                        fence_async_smem();
+                        named_barrier(1 + half, 128);
+                        const int64_t row0 = (int64_t)mb * (128 * MH) + 128 * h, col0 = (int64_t)nb * BN + c0;
+                        if (issuer && row0 < g.M && col0 < g.N) {   // boxes past the tensor: nothing to store
+                            tma_store_2d(&tmo, (int32_t)col0, (int32_t)row0, smem_u32(stg));
+                            bulk_commit();
+                        }
+                    }
+                }
+#pragma unroll 1
+                for (int c = half * (BN / 2); c < (TS ? half * (BN / 2) : (half + 1) * (BN / 2)); c += 32) {
                     float v[32];
                     tmem_ld32(tmem + lane_base + acc_col + c, v);   // warp-collective: every lane
                     tmem_ld_wait();
@@ -549,6 +625,7 @@ __global__ void __launch_bounds__(320, 1)
             }
         }
     }
+    if (TS && warp >= 2 && (warp & 3) == 0 && lane == 0) bulk_wait<0>();   // the output tiles' stores are done
     tc_fence_before();
     __syncthreads();
     if (warp == 1) {

@@ -143,6 +143,23 @@ def test_gemm_row_units_match_oracle(name, bm2, monkeypatch):
     assert resbm.resbm_device_error() == 0
 
 
+@pytest.mark.parametrize("name", ["bf16_r512_odd_blocks", "bf16_r24_m40", "bf16_r384_long_k"])
+def test_gemm_tma_store_epilogue_same_bits(name, monkeypatch):
+    """The GEMM chain's TMA-store epilogue for Y and dF (on by default) against per-thread stores
+    (RESBM_GEMM_TS=0): every output of the step the same bits (d = 776 leaves an 8-column last
+    box, T = 999 and 1100 partial row blocks and a pair partner past T; m = 40 takes dF from a
+    hi + lo dP)."""
+    cfg = SMALL[name]
+    h = host_inputs(cfg)
+    dev = {k: to_dev(v, cfg) for k, v in h.items()}
+    got = gpu_step(cfg, dev, flags=resbm.RESBM_FLAG_GEMM)
+    monkeypatch.setenv("RESBM_GEMM_TS", "0")
+    ref = gpu_step(cfg, dev, flags=resbm.RESBM_FLAG_GEMM)
+    for k in OUTS:
+        assert torch.equal(got[k], ref[k]), k
+    assert resbm.resbm_device_error() == 0
+
+
 @pytest.mark.parametrize("act", ["gelu_tanh", "identity"])
 @pytest.mark.parametrize("merge", [0, 1])
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
