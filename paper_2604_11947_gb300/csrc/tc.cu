@@ -244,12 +244,17 @@ cudaError_t launch_enc_fwd(const resbm_desc &d, const void *X, const void *F, co
     if (e != cudaSuccess) return e;
     tc::EncFwdArgs a{static_cast<const __nv_bfloat16 *>(X), static_cast<const __nv_bfloat16 *>(We2),
                      static_cast<__nv_bfloat16 *>(B), P, d.T, d.d, d.act};
-    // pairs of CTAs (clusters of 2), one pair per two SMs and at most one per tile, when all the
-    // pairs fit at once; single CTAs otherwise
+    // pairs of CTAs (clusters of 2), one pair per two SMs and at most one per tile, when there are
+    // more tiles than SMs (single CTAs would make a second pass: the pairs split the tiles evenly)
+    // and all the pairs fit at once; single CTAs otherwise (with at most one tile each they finish
+    // together, and a pair's exchange of partial P costs more than its share of a tile saves:
+    // T = 16384, d = 2048, 128 tiles: 22.3 us in pairs, 21.0 us single). RESBM_CLUSTER=1 forces
+    // single CTAs, 2 or 4 pairs.
     const int64_t tiles = (d.T + 127) / 128;
     int cl = 1;
     int64_t grid = tiles < c.sm_count ? (tiles < 1 ? 1 : tiles) : c.sm_count;
-    if (Cfg::SPLIT && forced_cluster() != 1) {   // RESBM_CLUSTER=1: single CTAs
+    const int forced = forced_cluster();
+    if (Cfg::SPLIT && forced != 1 && (forced != 0 || tiles > c.sm_count)) {
         static std::atomic<int> fit[kMaxDev][2];
         int64_t pairs = tiles < c.sm_count / 2 ? (tiles < 1 ? 1 : tiles) : c.sm_count / 2;
         if (pairs >= 1 && coresident_clusters(tc::k_enc_fwd<M>, 2, Cfg::THREADS, Cfg::SMEM_BYTES, c.device, fit) >= pairs) {

@@ -37,11 +37,10 @@ SMALL = {
     # the CTAs of a cluster have different group sizes but the same number of groups
     "bf16_uneven_groups": synth.BoundaryConfig("bf16_uneven_groups", T=79031, d=256, r=32, m=32),
     "bf16_uneven_groups_144": synth.BoundaryConfig("bf16_uneven_groups_144", T=74871, d=256, r=32, m=32),
-    # one partial tile: a single CTA (the encoder forward: one pair splitting the tile's chunks)
+    # one partial tile: a single CTA (pairs of the encoder forward: the forced-cluster cases)
     "bf16_single_ctas": synth.BoundaryConfig("bf16_single_ctas", T=40, d=256, r=32, m=32),
-    # the encoder forward's pairs with one 64-column chunk per tile (the split always falls on
-    # a tile boundary) and with three (a pair's single tile split 1 + 2); the other stages run
-    # on the portable kernels at these widths
+    # one 64-column chunk per tile and three; the other stages run on the portable kernels at
+    # these widths
     "bf16_d64": synth.BoundaryConfig("bf16_d64", T=1000, d=64, r=32, m=32),
     "bf16_d192": synth.BoundaryConfig("bf16_d192", T=300, d=192, r=32, m=32),
     # widths the fused kernels do not take run as the tensor-core GEMM chain by default: m = r =
@@ -76,6 +75,12 @@ CLUSTER_CASES = {
     "t321_r32": synth.BoundaryConfig("cl_t321_r32", T=41037, d=256, r=32, m=32),
     # 235 tiles: one or two per CTA, the last partial (48 tokens); three d chunks
     "t235_d384_r16": synth.BoundaryConfig("cl_t235_d384_r16", T=30000, d=384, r=16, m=16),
+    # the encoder forward's pairs where it has no more tiles than SMs (single CTAs by default):
+    # one partial tile split by a pair; one 64-column chunk per tile (the split always falls on a
+    # tile boundary) and three (a pair's single tile split 1 + 2)
+    "t1_partial": synth.BoundaryConfig("cl_t1_partial", T=40, d=256, r=32, m=32),
+    "d64": synth.BoundaryConfig("cl_d64", T=1000, d=64, r=32, m=32),
+    "d192": synth.BoundaryConfig("cl_d192", T=300, d=192, r=32, m=32),
 }
 _ORACLE_CACHE = {}
 
