@@ -131,20 +131,22 @@ struct GemmShape {
 
 // BM2: 256-row units, two 128-row A sub-tiles per stage against one B tile, the two halves'
 // accumulators side by side in TMEM (one unit at a time: no accumulator double buffering).
-// TS: the output tile leaves by TMA stores from a shared-memory staging box per half of the
-// epilogue warps (128 rows x 64 columns of bf16, 128-byte swizzle), for the products that write
-// T x d bf16 tensors: per-thread 16-byte stores of 32 different rows per warp instruction made
-// the epilogue, not the products, set such a product's pace.
+// TS: the output tile leaves by TMA stores from shared-memory staging boxes, two per half of the
+// epilogue warps (128 rows x 64 columns of bf16, 128-byte swizzle; one fills while the other's
+// store reads it), for the products that write T x d bf16 tensors: per-thread 16-byte stores of
+// 32 different rows per warp instruction made the epilogue, not the products, set such a
+// product's pace.
 template <int BN_, bool ALO_ = false, bool BM2_ = false, bool TS_ = false> struct GemmCfg {
     static constexpr int BN = BN_;
     static constexpr uint32_t A_TILE = 128 * 64 * 2;        // 128 rows x 64 K, bf16
     static constexpr uint32_t A_STAGE = A_TILE * (ALO_ ? 2 : 1) * (BM2_ ? 2 : 1);   // hi (+ lo), per half
     static constexpr uint32_t B_STAGE = BN_ * 64 * 2;       // BN rows x 64 K, bf16
     static constexpr uint32_t STAGE = A_STAGE + B_STAGE;
-    static constexpr uint32_t STG_HALF = 128 * 64 * 2;      // TS: one half's staging box
-    static constexpr uint32_t STG_BYTES = TS_ ? 2 * STG_HALF : 0;
-    // 4 stages at BN = 256, 6 at 128 (3, 4 with lo; 3 for BM2; one fewer with TS)
-    static constexpr int NST = (200 * 1024 - (int)STG_BYTES) / (int)STAGE;
+    static constexpr uint32_t STG_HALF = 128 * 64 * 2;      // TS: one staging box
+    static constexpr uint32_t STG_BYTES = TS_ ? 4 * STG_HALF : 0;   // two per half
+    // 4 stages at BN = 256, 6 at 128 (3, 4 with lo; 3 for BM2); TS: 3 at BN = 256 (2 with lo)
+    // beside its four boxes, from a larger share of the 227 KB
+    static constexpr int NST = ((TS_ ? 224 : 200) * 1024 - (int)STG_BYTES) / (int)STAGE;
     static constexpr uint32_t OFF_STG = NST * STAGE;        // 1024-aligned (STAGE is)
     static constexpr uint32_t SMEM_BYTES = NST * STAGE + STG_BYTES + 1024;
     static_assert(SMEM_BYTES <= 232448 - 512, "shared memory budget");
@@ -533,7 +535,7 @@ __global__ void __launch_bounds__(320, 1)
         const int half = (warp - 2) >> 2;       // which half of the BN columns
         const int rin = q * 32 + lane;          // row within the 128-row block
         const uint32_t lane_base = (uint32_t)(q * 32) << 16;
-        uint32_t ti = 0;
+        uint32_t ti = 0, stg_it = 0;   // units; TS staging boxes filled
         bool ok = true;
         for (int64_t u = u_first; u < gp.units && ok; u += u_step, ++ti) {
             int mb, nb, ks;
@@ -552,12 +554,13 @@ __global__ void __launch_bounds__(320, 1)
                     for (int j = 0; j < 32; ++j) pacc[j] = 0.0f;
                 }
                 if (TS) {
-                    // 64 columns at a time through this half's staging box, stored by one thread
+                    // 64 columns at a time through this half's two staging boxes in turn, each
+                    // stored by one thread
                     const bool issuer = q == 0 && lane == 0;
-                    uint8_t *stg = smem + C::OFF_STG + half * C::STG_HALF;
 #pragma unroll 1
-                    for (int c0 = half * (BN / 2); c0 < (half + 1) * (BN / 2); c0 += 64) {
-                        if (issuer) bulk_wait_read<0>();   // the box's previous store has read it
+                    for (int c0 = half * (BN / 2); c0 < (half + 1) * (BN / 2); c0 += 64, ++stg_it) {
+                        uint8_t *stg = smem + C::OFF_STG + (2 * half + (stg_it & 1)) * C::STG_HALF;
+                        if (issuer) bulk_wait_read<1>();   // the box's previous store has read it
                         named_barrier(1 + half, 128);
                         float v2[2][32];
                         tmem_ld32(tmem + lane_base + acc_col + c0, v2[0]);   // warp-collective: every lane
