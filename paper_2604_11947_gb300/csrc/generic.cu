@@ -364,6 +364,15 @@ constexpr int kNormBwdMaxD = 16384;
 
 template <typename E, int V> struct VecOf;
 template <> struct VecOf<__nv_bfloat16, 8> {
+    static __device__ void unpack(const uint4 u, float *f)
+    {
+        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            f[2 * i] = __uint_as_float(w[i] << 16);
+            f[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+        }
+    }
     static __device__ void load(const __nv_bfloat16 *p, float *f)
     {
         const uint4 u = *reinterpret_cast<const uint4 *>(p);
@@ -386,6 +395,10 @@ template <> struct VecOf<__nv_bfloat16, 8> {
     }
 };
 template <> struct VecOf<float, 4> {
+    static __device__ void unpack(const uint4 u, float *f)
+    {
+        f[0] = __uint_as_float(u.x); f[1] = __uint_as_float(u.y); f[2] = __uint_as_float(u.z); f[3] = __uint_as_float(u.w);
+    }
     static __device__ void load(const float *p, float *f)
     {
         const float4 u = *reinterpret_cast<const float4 *>(p);
@@ -481,6 +494,100 @@ __global__ void __launch_bounds__(256) k_rmsnorm_bwd(const E *__restrict__ Y, co
     for (int64_t j = tid; j < d; j += 256) dg_part[(int64_t)blockIdx.x * d + j] = dgs[j];
 }
 
+// The vector path for rows of at most 256 * KV vectors: each thread keeps its vectors of Y, dN and
+// dY (as loaded, 16 bytes each) in registers from the first pass to the second, so a row costs one
+// trip to memory, and loads dY with Y and dN. The same sums in the same order as k_rmsnorm_bwd, so
+// the same bits.
+template <typename E, int V, int KV>
+__global__ void __launch_bounds__(256) k_rmsnorm_bwd_reg(const E *__restrict__ Y, const E *__restrict__ gamma, float eps,
+                                                         const E *__restrict__ dN, const E *dY, E *dYo,
+                                                         float *__restrict__ dg_part, int64_t rows, int64_t d)
+{
+    extern __shared__ float dgs[];
+    __shared__ float2 part[2][8];
+    using L = VecOf<E, V>;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int64_t nv = d / V;
+#pragma unroll
+    for (int k = 0; k < KV; ++k) {
+        const int64_t q = tid + 256 * k;
+        if (q < nv)
+#pragma unroll
+            for (int i = 0; i < V; ++i) dgs[q * V + i] = 0.0f;
+    }
+    const int64_t r0 = rows * blockIdx.x / gridDim.x, r1 = rows * (blockIdx.x + 1) / gridDim.x;
+    for (int64_t t = r0; t < r1; ++t) {
+        uint4 ry[KV], rn[KV], ro[KV];
+#pragma unroll
+        for (int k = 0; k < KV; ++k) {   // every load of the row in flight before the first use
+            const int64_t q = tid + 256 * k;
+            if (q < nv) {
+                ry[k] = *reinterpret_cast<const uint4 *>(Y + t * d + q * V);
+                rn[k] = *reinterpret_cast<const uint4 *>(dN + t * d + q * V);
+                ro[k] = dY ? *reinterpret_cast<const uint4 *>(dY + t * d + q * V) : make_uint4(0u, 0u, 0u, 0u);
+            }
+        }
+        float sy = 0.0f, sg = 0.0f;
+#pragma unroll
+        for (int k = 0; k < KV; ++k) {
+            const int64_t q = tid + 256 * k;
+            if (q < nv) {
+                float a[V], b[V], gm[V];
+                L::unpack(ry[k], a);
+                L::unpack(rn[k], b);
+                L::load(gamma + q * V, gm);
+#pragma unroll
+                for (int i = 0; i < V; ++i) {
+                    sy = fmaf(a[i], a[i], sy);
+                    sg = fmaf(b[i] * gm[i], a[i], sg);
+                }
+            }
+        }
+        for (int o = 16; o > 0; o >>= 1) {
+            sy += __shfl_xor_sync(0xffffffffu, sy, o);
+            sg += __shfl_xor_sync(0xffffffffu, sg, o);
+        }
+        const int pb = (int)((t - r0) & 1);
+        if (lane == 0) part[pb][warp] = make_float2(sy, sg);
+        __syncthreads();
+        float Sy = 0.0f, Sg = 0.0f;
+#pragma unroll
+        for (int w = 0; w < 8; ++w) {
+            Sy += part[pb][w].x;
+            Sg += part[pb][w].y;
+        }
+        const float s = 1.0f / sqrtf(Sy / (float)d + eps);
+        const float kk = s * s * s * Sg / (float)d;
+#pragma unroll
+        for (int k = 0; k < KV; ++k) {
+            const int64_t q = tid + 256 * k;
+            if (q < nv) {
+                float a[V], b[V], gm[V], o[V], acc[V];
+                L::unpack(ry[k], a);
+                L::unpack(rn[k], b);
+                L::unpack(ro[k], o);
+                L::load(gamma + q * V, gm);
+#pragma unroll
+                for (int i = 0; i < V; i += 4) {
+                    const float4 u = *reinterpret_cast<const float4 *>(dgs + q * V + i);
+                    acc[i] = u.x; acc[i + 1] = u.y; acc[i + 2] = u.z; acc[i + 3] = u.w;
+                }
+#pragma unroll
+                for (int i = 0; i < V; ++i) {
+                    o[i] += s * (b[i] * gm[i]) - a[i] * kk;
+                    acc[i] = fmaf(b[i], a[i] * s, acc[i]);
+                }
+#pragma unroll
+                for (int i = 0; i < V; i += 4)
+                    *reinterpret_cast<float4 *>(dgs + q * V + i) = make_float4(acc[i], acc[i + 1], acc[i + 2], acc[i + 3]);
+                L::store(dYo + t * d + q * V, o);
+            }
+        }
+    }
+    __syncthreads();
+    for (int64_t j = tid; j < d; j += 256) dg_part[(int64_t)blockIdx.x * d + j] = dgs[j];
+}
+
 // dgamma[j] = the blocks' partials summed by a fixed two-level tree: warp w of a CTA sums the
 // partials of blocks [w G, (w + 1) G) in block order (eight loads in flight) for the CTA's 32
 // columns, then the eight group sums are added in group order. CTA x covers columns 32 x .. + 31.
@@ -531,15 +638,20 @@ cudaError_t generic_rmsnorm_bwd(const resbm_desc &d, const void *Y, const void *
                      d.d % (d.dtype == RESBM_F32 ? 4 : 8) == 0;
     cudaError_t e = cudaSuccess;
     if (d.T > 0) {
+        // the register-cached vector path up to 4 vectors a thread (bf16 d <= 8192, fp32 d <= 4096)
+        const int64_t nv = d.d / (d.dtype == RESBM_F32 ? 4 : 8);
+        const int kv = !vec ? 0 : nv <= 256 ? 1 : nv <= 512 ? 2 : nv <= 1024 ? 4 : 0;
         if (d.dtype == RESBM_F32) {
-            auto k = vec ? k_rmsnorm_bwd<float, 4> : k_rmsnorm_bwd<float, 1>;
+            auto k = kv == 1 ? k_rmsnorm_bwd_reg<float, 4, 1> : kv == 2 ? k_rmsnorm_bwd_reg<float, 4, 2>
+                   : kv == 4 ? k_rmsnorm_bwd_reg<float, 4, 4> : vec ? k_rmsnorm_bwd<float, 4> : k_rmsnorm_bwd<float, 1>;
             e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
             if (e == cudaSuccess)
                 k<<<nb, 256, smem, c.stream>>>((const float *)Y, (const float *)gamma, eps, (const float *)dN,
                                               (const float *)dY, (float *)dY_out, part, d.T, d.d);
         } else {
             using bf = __nv_bfloat16;
-            auto k = vec ? k_rmsnorm_bwd<bf, 8> : k_rmsnorm_bwd<bf, 1>;
+            auto k = kv == 1 ? k_rmsnorm_bwd_reg<bf, 8, 1> : kv == 2 ? k_rmsnorm_bwd_reg<bf, 8, 2>
+                   : kv == 4 ? k_rmsnorm_bwd_reg<bf, 8, 4> : vec ? k_rmsnorm_bwd<bf, 8> : k_rmsnorm_bwd<bf, 1>;
             e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
             if (e == cudaSuccess)
                 k<<<nb, 256, smem, c.stream>>>((const bf *)Y, (const bf *)gamma, eps, (const bf *)dN, (const bf *)dY,

@@ -21,6 +21,9 @@ CASES = {
     "d16384_max": synth.BoundaryConfig("nb_d16384", T=5, d=16384, r=32, m=32),
     "one_row": synth.BoundaryConfig("nb_one", T=1, d=64, r=32, m=32),
     "rows_lt_blocks": synth.BoundaryConfig("nb_300", T=300, d=768, r=16, m=16),   # fewer rows than blocks
+    # rows held in registers with 1, 2 and 4 vectors a thread (d = 2048 above: 1), the last one partial
+    "d3000_two_vectors": synth.BoundaryConfig("nb_d3000", T=777, d=3000, r=8, m=8),
+    "d6144_four_vectors": synth.BoundaryConfig("nb_d6144", T=77, d=6144, r=32, m=32),
 }
 
 
