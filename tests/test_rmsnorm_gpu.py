@@ -130,3 +130,27 @@ def test_headline_shape_every_element():
     Y, N = _run(cfg, dev, 0)
     _check_yn(cfg, Y, N, h)
     assert resbm.resbm_device_error() == 0
+
+
+@pytest.mark.parametrize("path", ["default", "generic"])
+def test_linear_decoder_with_rmsnorm(path):
+    """One linear layer per side (RESBM_FLAG_LINEAR: Y = pad(B) + B . Wd, Wd r x d; Wd1 absent):
+    Y and N against the oracle's one-layer decoder followed by its norm."""
+    cfg = synth.BoundaryConfig("rn_lin", T=700, d=512, r=32, m=32)
+    flags = resbm.RESBM_FLAG_LINEAR | PATHS[path]
+    B = synth.tensor(cfg, "dB")
+    Wd = synth.tensor(cfg, "Wd2")[: cfg.r]          # r x d
+    gamma = synth.tensor(cfg, "gamma")[0]
+    desc = resbm.desc_from_config(cfg, flags)
+    dB, dWd, dg = to_dev(B, cfg), to_dev(Wd, cfg), to_dev(gamma, cfg)
+    Y = torch.empty(cfg.T, cfg.d, dtype=torch.bfloat16, device="cuda")
+    N = torch.empty_like(Y)
+    ws = resbm.workspace(desc, resbm.RESBM_OP_DECODE_FWD_RMSNORM)
+    resbm.resbm_decode_fwd_rmsnorm(desc, dB, None, dWd, dg, EPS, Y, N, ws)
+    torch.cuda.synchronize()
+    wY = oracle.linear_decode_fwd(B, Wd, cfg.merge)
+    check("Y", to_host(Y), wY, "bf16")
+    rstd = 1.0 / np.sqrt(np.mean(wY * wY, axis=1, keepdims=True) + EPS)
+    check("N", to_host(N), oracle.rmsnorm(wY, gamma, EPS), "bf16",
+          allow=bf16_half_spacing(wY) * np.abs(rstd * np.asarray(gamma, np.float64)[None, :]))
+    assert resbm.resbm_device_error() == 0
