@@ -768,10 +768,10 @@ def run_e2e(args, cfg, w, resbm, torch, dist, world):
     # dX[:, :r] out
     h2d = 2 * cols + sum(host_in[k].numel() * es for k in ins if k != "X")
     d2h = cols + sum(host_out[0][k].numel() * host_out[0][k].element_size() for k in res)
-    # up to 100 steps (≈0.65 s): the host link sometimes stalls for ~100 ms (seen as 30-55 ms
-    # gaps between consecutive steps whose steady pace is 6.4 ms); a short window would charge
-    # one such stall to a handful of steps
-    n = max(2, min(args.steps, 100))
+    # 300 steps (≈2.3 s) whatever --steps is: the host link sometimes stalls for ~100 ms (seen as
+    # 30-55 ms gaps between consecutive steps whose steady pace is 6.5 ms); a short window would
+    # charge one such burst to a handful of steps, so the window is long enough to average them
+    n = 300
 
     def step(i):
         b = i % 2
