@@ -454,6 +454,18 @@ def ffn_encode_workload(resbm, torch, steps=20, warmup=3):
     return res
 
 
+def rmsnorm_alg_bytes(T, d, r, m):
+    """Algorithmic HBM bytes (bf16) of the decoder forward + RMSNorm forms at T tokens: the fused
+    pair reads B twice, the weights twice and gamma, writes Y and N, and writes then reads each
+    row's 2 d / 256 fp32 partial sums (d / 256 column chunks of two halves, m <= 32); the unfused
+    chain reads B and the weights once, writes Y, reads it back and writes N."""
+    nch = d // 256
+    w = 2 * (r * m + m * d)
+    return {"fused": T * (2 * 2 * r + 2 * 2 * d + 2 * 4 * 2 * nch) + 2 * w + 2 * d,
+            "unfused_decode_then_torch_rms_norm": T * (2 * r + 3 * 2 * d) + w + 2 * d,
+            "decode_fwd_alone": T * (2 * r + 2 * d) + w}
+
+
 def decode_rmsnorm_workload(resbm, torch, peaks, steps=50, warmup=5):
     """The decoder forward with the next block's pre-attention RMSNorm fused in, at the headline
     shape (T = 65536, d = 4096, r = m = 32, bf16): resbm_decode_fwd_rmsnorm (Y and N, Y never read
@@ -479,10 +491,7 @@ def decode_rmsnorm_workload(resbm, torch, peaks, steps=50, warmup=5):
                 resbm.resbm_decode_fwd(desc, B, Wd1, Wd2, Y, ws_dec),
                 torch.nn.functional.rms_norm(Y, (d,), gamma, eps)),
             "decode_fwd_alone": lambda: resbm.resbm_decode_fwd(desc, B, Wd1, Wd2, Y, ws_dec)}
-    nch = d // 256
-    alg = {"fused": T * (2 * 2 * r + 2 * 2 * d + 2 * 4 * 2 * nch) + 2 * (2 * (r * m + m * d)) + 2 * d,
-           "unfused_decode_then_torch_rms_norm": T * (2 * r + 3 * 2 * d) + 2 * (r * m + m * d) + 2 * d,
-           "decode_fwd_alone": T * (2 * r + 2 * d) + 2 * (r * m + m * d)}
+    alg = rmsnorm_alg_bytes(T, d, r, m)
     res = {"workload": "decoder forward + the next block's RMSNorm (T=%d, d=%d, r=m=%d, bf16)" % (T, d, r),
            "steps": steps, "inputs_exceed_l2": True}
     for name, fn in runs.items():

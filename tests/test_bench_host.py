@@ -40,3 +40,15 @@ def test_captured_traffic_is_close_to_the_algorithmic_bytes(op):
     got = j["ops"][cfg.name][op]["dram_bytes_per_launch"]
     alg = bench.op_bytes(cfg)[op]
     assert alg - 129e6 <= got <= 1.1 * alg, (op, got, alg)
+
+
+def test_rmsnorm_byte_model():
+    """The decoder + RMSNorm byte model at T = 65536, d = 4096, r = m = 32: the fused form saves
+    the read-back of Y (T d 2 bytes) less its second read of B and its row sums
+    (T (2r + 2 * 8 d / 256) bytes); the bench's figure of 515.6 MB."""
+    T, d, r, m = 65536, 4096, 32, 32
+    a = bench.rmsnorm_alg_bytes(T, d, r, m)
+    saved = a["unfused_decode_then_torch_rms_norm"] - a["fused"]
+    assert saved == T * 2 * d - T * (2 * r + 16 * (d // 256)) - 2 * (r * m + m * d)
+    assert saved == 515635200
+    assert a["decode_fwd_alone"] == T * (2 * r + 2 * d) + 2 * (r * m + m * d)
