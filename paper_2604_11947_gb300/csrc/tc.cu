@@ -563,15 +563,23 @@ cudaError_t gemm(const Ctx &c, int64_t M, int64_t N, int64_t K, const void *A, b
     }
     // TMA-store epilogue for the pairs' plain bf16 outputs (Y = G . Wd2 + pad(B), dF = dP . We1^T)
     CUtensorMap mo;
-    const bool ts = pair && !a_mn && !(b_mn && lo) && g.splits == 1 &&
+    const bool ts = bn == 256 && !bm2 && !a_mn && !(b_mn && lo) && g.splits == 1 &&
                     (ep.mode == tc::GEP_BF16 || ep.mode == tc::GEP_ADD_AUX || ep.mode == tc::GEP_DF) &&
                     al16(ep.out) && (ep.ldo * 2) % 16 == 0 && ts_enabled() &&
                     make_map(&mo, ep.out, N, M, ep.ldo * 2, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B);
-    if (ts) {
+    if (ts && pair) {
         cudaError_t e = b_mn ? launch_gemm_t<256, false, true, false, false, true, false, true>(ma, malo, mbm, g, ep, c, &mo)
                         : lo ? launch_gemm_t<256, false, false, true, false, true, false, true>(ma, malo, mbm, g, ep, c, &mo)
                              : launch_gemm_t<256, false, false, false, false, true, false, true>(ma, malo, mbm, g, ep, c, &mo);
         if (e != cudaErrorNotSupported) return e;
+        // no pair fits: single CTAs need the whole-tile box for K-major B
+        if (!b_mn && !make_map(&mbm, B, K, N, K * 2, 64, (uint32_t)bn, CU_TENSOR_MAP_SWIZZLE_128B))
+            return cudaErrorInvalidValue;
+    }
+    if (ts) {   // single CTAs
+        return b_mn ? launch_gemm_t<256, false, true, false, false, false, false, true>(ma, malo, mbm, g, ep, c, &mo)
+               : lo ? launch_gemm_t<256, false, false, true, false, false, false, true>(ma, malo, mbm, g, ep, c, &mo)
+                    : launch_gemm_t<256, false, false, false, false, false, false, true>(ma, malo, mbm, g, ep, c, &mo);
     }
     if (pair) {
         cudaError_t e = cudaErrorNotSupported;
