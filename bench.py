@@ -50,6 +50,8 @@ def parse():
     p.add_argument("--rmsnorm-only", action="store_true",
                    help="run only the decoder forward + RMSNorm comparison (for profiler captures; "
                         "--steps / --warmup apply); prints its JSON object, not a bench line")
+    p.add_argument("--hbm-forms-only", action="store_true",
+                   help="only the HBM rate of each access form (resbm_measure_hbm_form), 1 GiB buffers")
     p.add_argument("--ffn-only", action="store_true",
                    help="run only the FFN down-projection + encoder comparison (for profiler captures; "
                         "--steps / --warmup apply); prints its JSON object, not a bench line")
@@ -604,6 +606,10 @@ def main():
         print(json.dumps(decode_rmsnorm_workload(resbm, torch, measured_peaks(), steps=max(args.steps, 1),
                                                  warmup=max(args.warmup, 0))), flush=True)
         return
+    if args.hbm_forms_only:
+        print(json.dumps(hbm_forms(resbm, torch, reps=max(args.steps, 1), warmup=max(args.warmup, 0),
+                                   sampler=ClockSampler())), flush=True)
+        return
     if args.ffn_only:
         print(json.dumps(ffn_encode_workload(resbm, torch, steps=max(args.steps, 1), warmup=max(args.warmup, 0))),
               flush=True)
@@ -682,6 +688,7 @@ def main():
         torch.cuda.empty_cache()
         extra["pipeline"] = pipeline_workload(torch)
         torch.cuda.empty_cache()
+        extra["hbm_forms"] = hbm_forms(resbm, torch)
         from paper_2604_11947_gb300 import pipeline
         conv = pipeline.convergence()
         conv["workload"] = ("loss curves (step, mean loss over the previous 25 steps) of a 4-layer "
@@ -712,6 +719,45 @@ def main():
         print(json.dumps(line), flush=True)
     if dist:
         dist.destroy_process_group()
+
+
+def hbm_forms(resbm, torch, gib=1, reps=10, warmup=3, sampler=None):
+    """The HBM rate each access form of resbm_measure_hbm_form attains on this device: every form
+    over `gib` GiB buffers (above the 129 MB L2, so no flush), `warmup` untimed launches, then
+    `reps` launches each timed with CUDA events on the launching stream; GB/s of the bytes the
+    form moves (reads + writes), median and best. `sampler`: a ClockSampler to run around it."""
+    n = gib << 30
+    a = torch.full((n,), 0x3C, dtype=torch.uint8, device="cuda")
+    b = torch.zeros(n, dtype=torch.uint8, device="cuda")
+    s = torch.cuda.current_stream()
+    if sampler is not None:
+        torch.cuda.synchronize()
+        sampler.start()
+        time.sleep(0.15)
+    out = {}
+    for name in resbm.HBM_FORMS:
+        for _ in range(warmup):
+            resbm.resbm_measure_hbm_form(name, a, b)
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
+        for e0, e1 in ev:
+            e0.record(s)
+            resbm.resbm_measure_hbm_form(name, a, b)
+            e1.record(s)
+        torch.cuda.synchronize()
+        ms = sorted(e0.elapsed_time(e1) for e0, e1 in ev)
+        moved = 2 * n if name.startswith("copy") else n
+        out[name] = {"GBps_median": moved / (statistics.median(ms) / 1e3) / 1e9,
+                     "GBps_best": moved / (ms[0] / 1e3) / 1e9, "ms_median": statistics.median(ms),
+                     "moved_bytes": moved}
+    res = {"forms": out, "buffer_bytes": n, "reps": reps, "warmup": warmup,
+           "device_error": resbm.resbm_device_error(),
+           "how": "one launch per timed rep, CUDA events on the launching stream; the forms are those of "
+                  "include/resbm.h resbm_hbm_form"}
+    if sampler is not None:
+        res["clocks"] = sampler.stop()
+    del a, b
+    torch.cuda.empty_cache()
+    return res
 
 
 def host_link(torch, mib=512, reps=3):

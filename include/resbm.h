@@ -164,6 +164,46 @@ RESBM_API resbm_status resbm_device_error(unsigned int *code, int clear);
  * that a stuck wait is reported instead of hanging the device. */
 RESBM_API resbm_status resbm_selftest_wait_timeout(void *stream);
 
+/* Memory-system probe (no counterpart in the paper): the access forms whose HBM rates the
+ * kernels' choice of load and store forms rests on. One call enqueues on `stream` one launch of
+ * `form` over `bytes` bytes:
+ *   RESBM_HBM_READ_V4         reads a: 16-byte loads by every thread (four 512-thread CTAs per SM)
+ *   RESBM_HBM_WRITE_V4        writes b the same way (every byte 0xA5)
+ *   RESBM_HBM_COPY_V4         copies a to b the same way (moves 2 * bytes)
+ *   RESBM_HBM_READ_TMA_2D     reads a with one CTA per SM: 2-D tensor loads of 64-column x
+ *                             128-row bf16 boxes (16 KB, 128-byte swizzle), 8 stages in flight
+ *   RESBM_HBM_READ_TMA_2D_PAIR two such boxes per 32 KB stage on one barrier, 4 stages
+ *   RESBM_HBM_READ_TMA_3D     one 3-D box of two neighbouring 64-column blocks per 32 KB stage
+ *   RESBM_HBM_READ_BULK       1-D bulk copies of 16 KB, 8 stages
+ *   RESBM_HBM_WRITE_TMA_2D    writes b with 2-D tensor stores of the 64 x 128 boxes (0xA5)
+ *   RESBM_HBM_WRITE_BULK      writes b with 1-D bulk stores of 16 KB (0xA5)
+ *   RESBM_HBM_READ_TMA_2D_TILES  as RESBM_HBM_READ_TMA_2D_PAIR in the backward kernels' walk:
+ *                             each CTA's run of 128-row tiles in groups of up to four, per group
+ *                             the 128-column chunks in cyclic order from a chunk that depends on
+ *                             the CTA, each chunk's tiles one after the other
+ *   RESBM_HBM_WRITE_TMA_2D_TILES  as RESBM_HBM_WRITE_TMA_2D in that walk (0xA5)
+ * The TMA forms view a buffer as a row-major bf16 matrix of 4096 columns (8 KB rows); each
+ * CTA streams a contiguous run of its boxes (row-tile-major unless a form says otherwise). a and b: device memory of `bytes` bytes each,
+ * 16-byte aligned, not overlapping, both required for every form (RESBM_HBM_READ_V4 writes at
+ * most 4 bytes of b, and only for an input it does not expect). bytes: a positive multiple of
+ * 1 MiB. Errors: RESBM_ERR_INVALID_ARG for a bad form, size or pointer (nothing enqueued);
+ * RESBM_ERR_CUDA if a launch (or the tensor-map encoding) failed. Waits are bounded as in the
+ * other tensor-core kernels (resbm_device_error reports a timeout). */
+typedef enum {
+    RESBM_HBM_READ_V4 = 0,
+    RESBM_HBM_WRITE_V4 = 1,
+    RESBM_HBM_COPY_V4 = 2,
+    RESBM_HBM_READ_TMA_2D = 3,
+    RESBM_HBM_READ_TMA_2D_PAIR = 4,
+    RESBM_HBM_READ_TMA_3D = 5,
+    RESBM_HBM_READ_BULK = 6,
+    RESBM_HBM_WRITE_TMA_2D = 7,
+    RESBM_HBM_WRITE_BULK = 8,
+    RESBM_HBM_READ_TMA_2D_TILES = 9,
+    RESBM_HBM_WRITE_TMA_2D_TILES = 10
+} resbm_hbm_form;
+RESBM_API resbm_status resbm_measure_hbm_form(int form, const void *a, void *b, int64_t bytes, void *stream);
+
 /* Scratch bytes that `op` (a resbm_op) needs for `desc`, written to *bytes.
  * Returns RESBM_ERR_INVALID_ARG for a bad descriptor or op. Does not touch the GPU. */
 RESBM_API resbm_status resbm_workspace_bytes(const resbm_desc *desc, int op, size_t *bytes);

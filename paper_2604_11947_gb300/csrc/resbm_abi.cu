@@ -667,6 +667,18 @@ resbm_status resbm_selftest_wait_timeout(void *stream)
     return s != RESBM_OK ? s : finish(tc_wait_selftest(c));
 }
 
+resbm_status resbm_measure_hbm_form(int form, const void *a, void *b, int64_t bytes, void *stream)
+{
+    constexpr int64_t kMiB = int64_t(1) << 20;
+    if (form < RESBM_HBM_READ_V4 || form > RESBM_HBM_WRITE_TMA_2D_TILES || bytes < kMiB || bytes % kMiB != 0 ||
+        bytes / 8192 > INT32_MAX || !a || !b || !aligned16(a) || !aligned16(b) ||
+        overlaps(rng(a, bytes, 1), rng(b, bytes, 1)))
+        return RESBM_ERR_INVALID_ARG;
+    Ctx c;
+    resbm_status s = make_ctx(stream, &c);
+    return s != RESBM_OK ? s : finish(tc_hbm_form(form, a, b, bytes, c));
+}
+
 resbm_status resbm_workspace_bytes(const resbm_desc *desc, int op, size_t *bytes)
 {
     resbm_status s = check_desc(desc);

@@ -9,6 +9,7 @@
 
 #include <atomic>
 #include <cstdlib>
+#include <cstring>
 #include <mutex>
 #include <utility>
 
@@ -20,6 +21,7 @@
 #include "tc_enc_bwd.cuh"
 #include "tc_gemm.cuh"
 #include "tc_spectral.cuh"
+#include "tc_hbm_forms.cuh"
 
 namespace resbm {
 
@@ -174,20 +176,44 @@ int bwd_min_grid(int64_t T, int sms)
     const int gf = bwd_full_grid(T, sms);
     return (15 * gf + 15) / 16;
 }
+// RESBM_BWD_BALANCE=0 keeps the decoder backward's grid at the cluster rule's size; unset or
+// anything else: balanced (bwd_balanced). Read at every launch.
+bool bwd_balance_enabled()
+{
+    const char *v = getenv("RESBM_BWD_BALANCE");
+    return !(v && v[0] == '0' && v[1] == 0);
+}
+// The fewest CTAs (a multiple of cl, at most g) that leave no CTA more whole tiles than g CTAs
+// do: every CTA then has the same number of tiles or one fewer, as few as possible having
+// fewer. At T = 65536 (512 tiles) on 144 CTAs, 80 CTAs make a fourth tile pass while 64 are
+// done after three; 128 CTAs make the same four passes each, with fewer weight-gradient
+// partial slots (32 clusters instead of 36). Measured at that size (bench, two A/B pairs): the
+// decoder backward 116.5 -> 115.3 us; the encoder backward 211.0 -> 214.5 us (its epilogue's
+// per-tile work gains from more SMs), so only the decoder backward takes it.
+int bwd_balanced(int64_t T, int g, int cl)
+{
+    const int64_t U = (T + 127) / 128;
+    const int64_t mt = (U + g - 1) / g;                    // the most tiles a CTA gets on g CTAs
+    int64_t gb = (U + mt - 1) / mt;                        // the fewest CTAs with at most mt each
+    gb = (gb + cl - 1) / cl * cl;
+    return gb < g ? (int)gb : g;
+}
 template <typename... KArgs>
 BwdShape bwd_shape(void (*kernel)(KArgs...), int64_t T, int sms, int threads, uint32_t smem, int clmax,
-                   int64_t min_tokens, int dev, std::atomic<int> (&fit)[kMaxDev][2])
+                   int64_t min_tokens, int dev, std::atomic<int> (&fit)[kMaxDev][2], bool balance)
 {
     const int gf = bwd_full_grid(T, sms);
     const int forced = forced_cluster();
+    const bool bal = balance && bwd_balance_enabled();
     for (int cl = 4; cl >= 2; cl /= 2) {
         if (cl > clmax || (forced && cl != forced)) continue;
         int64_t g = (int64_t)cl * coresident_clusters(kernel, cl, threads, smem, dev, fit);
         if (g > gf) g = gf;
         g -= g % cl;
-        if (g >= cl && 16 * g >= 15 * (int64_t)gf && (forced || T >= min_tokens * g)) return BwdShape{(int)g, cl};
+        if (g >= cl && 16 * g >= 15 * (int64_t)gf && (forced || T >= min_tokens * g))
+            return BwdShape{bal ? bwd_balanced(T, (int)g, cl) : (int)g, cl};
     }
-    return BwdShape{gf, 1};
+    return BwdShape{bal ? bwd_balanced(T, gf, 1) : gf, 1};
 }
 
 bool tc_width_ok(int64_t m) { return m == 16 || m == 32 || m == 64 || m == 128; }
@@ -271,7 +297,8 @@ cudaError_t launch_enc_fwd(const resbm_desc &d, const void *X, const void *F, co
 // Scratch layout of the backward kernels: the d x m weight gradient has one fp32 slot per
 // cluster (room for g_full single CTAs; tc_wgrad.cuh); the small one has one slot per (CTA, tile
 // group). Every CTA has max_groups tile groups. The scratch size covers every grid the launch
-// may pick (bwd_min_grid .. bwd_full_grid), so it does not depend on the device's occupancy.
+// may pick (bwd_min_grid .. bwd_full_grid, and the balanced grids below them, which have no
+// more tile groups per CTA and fewer CTAs), so it does not depend on the device's occupancy.
 struct BwdPlan {
     int grid = 1, max_groups = 1, nch = 1;
     int64_t slots = 1;              // small partial slots
@@ -345,7 +372,7 @@ cudaError_t launch_dec_bwd(const resbm_desc &d, const void *dY, const void *B, c
     if (e != cudaSuccess) return e;
     static std::atomic<int> fit[kMaxDev][2];
     const BwdShape sh = bwd_shape(tc::k_dec_bwd<M>, d.T, c.sm_count, Cfg::THREADS, Cfg::SMEM_BYTES, Cfg::CLMAX,
-                                  Cfg::CL_MIN_TOKENS, c.device, fit);
+                                  Cfg::CL_MIN_TOKENS, c.device, fit, true);
     const BwdPlan p = bwd_plan(d, c.sm_count, sh.grid, Cfg::NT, d.r * d.m, ws);
     CUtensorMap m_dy128, m_dy16, m_wd2, m_b, m_yr;
     if (!make_map(&m_dy128, dY, d.d, d.T, d.d * 2, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B) ||
@@ -403,7 +430,7 @@ cudaError_t launch_enc_bwd(const resbm_desc &d, const void *dB, const void *F, c
     if (e != cudaSuccess) return e;
     static std::atomic<int> fit[kMaxDev][2];
     const BwdShape sh = bwd_shape(tc::k_enc_bwd<M>, d.T, c.sm_count, Cfg::THREADS, Cfg::SMEM_BYTES, Cfg::CLMAX,
-                                  Cfg::CL_MIN_TOKENS, c.device, fit);
+                                  Cfg::CL_MIN_TOKENS, c.device, fit, false);
     const EncBwdWs w = enc_bwd_ws(d, c.sm_count, sh.grid, ws);
     const BwdPlan &p = w.plan;
     CUtensorMap m_f128, m_f16, m_we1, m_df128, m_df16, m_db;
@@ -1133,6 +1160,85 @@ __global__ void k_wait_selftest()
     if (threadIdx.x == 0) mbar_wait(smem_u32(&bar), 0);
 }
 }  // namespace tc
+
+namespace {
+// The 3-D view of the 3-D load form: {64 columns, rows, 64 column blocks} with the blocks 128
+// bytes apart, so that one box {64, 128, 2} holds two neighbouring 64-column blocks of 128 rows
+// and lands as two 64 x 128 swizzled boxes.
+bool make_map_form3d(CUtensorMap *m, const void *ptr, uint64_t rows)
+{
+    auto fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[3] = {64, rows, (cuuint64_t)tc::kFormBlocks};
+    cuuint64_t strides[2] = {(cuuint64_t)tc::kFormBlocks * 128, 128};
+    cuuint32_t box[3] = {64, 128, 2};
+    cuuint32_t es[3] = {1, 1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(ptr), dims, strides, box, es,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int FORM>
+cudaError_t launch_form_load(const CUtensorMap &m, const void *a, int64_t boxes, const Ctx &c)
+{
+    static std::atomic<uint8_t> smem_set[kMaxDev];
+    cudaError_t e = ensure_smem(tc::k_form_load<FORM>, tc::kFormSmem, c.device, smem_set);
+    if (e != cudaSuccess) return e;
+    tc::k_form_load<FORM><<<c.sm_count, 128, tc::kFormSmem, c.stream>>>(m, static_cast<const uint8_t *>(a), boxes);
+    return cudaGetLastError();
+}
+
+template <int FORM>
+cudaError_t launch_form_store(const CUtensorMap &m, void *b, int64_t boxes, const Ctx &c)
+{
+    static std::atomic<uint8_t> smem_set[kMaxDev];
+    cudaError_t e = ensure_smem(tc::k_form_store<FORM>, tc::kFormSmem, c.device, smem_set);
+    if (e != cudaSuccess) return e;
+    tc::k_form_store<FORM><<<c.sm_count, 128, tc::kFormSmem, c.stream>>>(m, static_cast<uint8_t *>(b), boxes);
+    return cudaGetLastError();
+}
+}  // namespace
+
+cudaError_t tc_hbm_form(int form, const void *a, void *b, int64_t bytes, const Ctx &c)
+{
+    const int64_t boxes = bytes / tc::kFormBox, rows = bytes / (tc::kFormBlocks * 128), n16 = bytes / 16;
+    const int vgrid = c.sm_count * 4;
+    CUtensorMap m;
+    std::memset(&m, 0, sizeof(m));
+    const bool reads = form == RESBM_HBM_READ_TMA_2D || form == RESBM_HBM_READ_TMA_2D_PAIR ||
+                       form == RESBM_HBM_READ_TMA_2D_TILES;
+    const bool writes = form == RESBM_HBM_WRITE_TMA_2D || form == RESBM_HBM_WRITE_TMA_2D_TILES;
+    if ((reads || writes) && !make_map(&m, reads ? a : b, tc::kFormBlocks * 64, (uint64_t)rows,
+                                       tc::kFormBlocks * 128, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B))
+        return cudaErrorInvalidValue;
+    if (form == RESBM_HBM_READ_TMA_3D && !make_map_form3d(&m, a, (uint64_t)rows)) return cudaErrorInvalidValue;
+    cudaError_t e = cudaSuccess;
+    switch (form) {
+    case RESBM_HBM_READ_V4:
+        tc::k_form_read_v4<<<vgrid, 512, 0, c.stream>>>(static_cast<const uint4 *>(a), n16, static_cast<unsigned *>(b));
+        e = cudaGetLastError();
+        break;
+    case RESBM_HBM_WRITE_V4:
+        tc::k_form_write_v4<<<vgrid, 512, 0, c.stream>>>(static_cast<uint4 *>(b), n16);
+        e = cudaGetLastError();
+        break;
+    case RESBM_HBM_COPY_V4:
+        tc::k_form_copy_v4<<<vgrid, 512, 0, c.stream>>>(static_cast<const uint4 *>(a), static_cast<uint4 *>(b), n16);
+        e = cudaGetLastError();
+        break;
+    case RESBM_HBM_READ_TMA_2D: e = launch_form_load<tc::kLoad2d>(m, a, boxes, c); break;
+    case RESBM_HBM_READ_TMA_2D_PAIR: e = launch_form_load<tc::kLoad2dPair>(m, a, boxes, c); break;
+    case RESBM_HBM_READ_TMA_3D: e = launch_form_load<tc::kLoad3d>(m, a, boxes, c); break;
+    case RESBM_HBM_READ_BULK: e = launch_form_load<tc::kLoadBulk>(m, a, boxes, c); break;
+    case RESBM_HBM_WRITE_TMA_2D: e = launch_form_store<tc::kStore2d>(m, b, boxes, c); break;
+    case RESBM_HBM_WRITE_BULK: e = launch_form_store<tc::kStoreBulk>(m, b, boxes, c); break;
+    case RESBM_HBM_READ_TMA_2D_TILES: e = launch_form_load<tc::kLoadTiles>(m, a, boxes, c); break;
+    case RESBM_HBM_WRITE_TMA_2D_TILES: e = launch_form_store<tc::kStoreTiles>(m, b, boxes, c); break;
+    default: return cudaErrorInvalidValue;
+    }
+    count_launches(1);
+    return e;
+}
 
 cudaError_t tc_wait_selftest(const Ctx &c)
 {

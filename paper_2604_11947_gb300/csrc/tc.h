@@ -14,6 +14,9 @@ cudaError_t tc_device_error(unsigned int *code, bool clear);
 // Enqueues a one-CTA kernel whose only wait can never complete: it gives up after the bounded
 // wait time and records the timeout in the error word (a test of that path; nothing faults).
 cudaError_t tc_wait_selftest(const Ctx &c);
+// One launch of the HBM access-form probe `form` (resbm_hbm_form, tc_hbm_forms.cuh) over `bytes`
+// bytes: a is read, b written (arguments checked by the caller).
+cudaError_t tc_hbm_form(int form, const void *a, void *b, int64_t bytes, const Ctx &c);
 // Scratch bytes of the tensor-core kernels for `op` on a device with `sms` SMs.
 size_t tc_ws_bytes(const resbm_desc &d, int op, int sms);
 

@@ -20,6 +20,14 @@ RESBM_ACT_SILU, RESBM_ACT_GELU_TANH, RESBM_ACT_IDENTITY = 0, 1, 2
 (RESBM_OP_ENCODE_FWD, RESBM_OP_DECODE_FWD, RESBM_OP_DECODE_BWD, RESBM_OP_ENCODE_BWD,
  RESBM_OP_BOUNDARY_STEP, RESBM_OP_BOUNDARY_STEP_HOST, RESBM_OP_EFFECTIVE_RANK, RESBM_OP_NEWTON_SCHULZ,
  RESBM_OP_DECODE_FWD_RMSNORM, RESBM_OP_RMSNORM_BWD) = range(10)
+(RESBM_HBM_READ_V4, RESBM_HBM_WRITE_V4, RESBM_HBM_COPY_V4, RESBM_HBM_READ_TMA_2D, RESBM_HBM_READ_TMA_2D_PAIR,
+ RESBM_HBM_READ_TMA_3D, RESBM_HBM_READ_BULK, RESBM_HBM_WRITE_TMA_2D, RESBM_HBM_WRITE_BULK,
+ RESBM_HBM_READ_TMA_2D_TILES, RESBM_HBM_WRITE_TMA_2D_TILES) = range(11)
+HBM_FORMS = {"read_v4": RESBM_HBM_READ_V4, "write_v4": RESBM_HBM_WRITE_V4, "copy_v4": RESBM_HBM_COPY_V4,
+             "read_tma_2d": RESBM_HBM_READ_TMA_2D, "read_tma_2d_pair": RESBM_HBM_READ_TMA_2D_PAIR,
+             "read_tma_3d": RESBM_HBM_READ_TMA_3D, "read_bulk": RESBM_HBM_READ_BULK,
+             "write_tma_2d": RESBM_HBM_WRITE_TMA_2D, "write_bulk": RESBM_HBM_WRITE_BULK,
+             "read_tma_2d_tiles": RESBM_HBM_READ_TMA_2D_TILES, "write_tma_2d_tiles": RESBM_HBM_WRITE_TMA_2D_TILES}
 RESBM_FLAG_GENERIC = 1
 RESBM_FLAG_LINEAR = 2
 RESBM_FLAG_GEMM = 4
@@ -35,7 +43,8 @@ EXPORTS = ("resbm_version", "resbm_status_string", "resbm_last_cuda_error", "res
            "resbm_encode_bwd", "resbm_boundary_step", "resbm_boundary_step_host",
            "resbm_decode_bwd_noalloc", "resbm_selftest_wait_timeout", "resbm_matrix_workspace_bytes",
            "resbm_newton_schulz", "resbm_effective_rank", "resbm_ffn_down_encode_workspace_bytes",
-           "resbm_ffn_down_encode_fwd", "resbm_decode_fwd_rmsnorm", "resbm_rmsnorm_bwd")
+           "resbm_ffn_down_encode_fwd", "resbm_decode_fwd_rmsnorm", "resbm_rmsnorm_bwd",
+           "resbm_measure_hbm_form")
 
 
 class resbm_desc(ctypes.Structure):
@@ -118,6 +127,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.resbm_ffn_down_encode_workspace_bytes.argtypes = [D, i64, ctypes.POINTER(sz)]
     lib.resbm_ffn_down_encode_fwd.restype = i32
     lib.resbm_ffn_down_encode_fwd.argtypes = [D, i64] + [vp] * 8 + [vp, sz, vp]
+    lib.resbm_measure_hbm_form.restype = i32
+    lib.resbm_measure_hbm_form.argtypes = [i32, vp, vp, i64, vp]
     if path is None:
         _lib = lib
     return lib
@@ -145,6 +156,16 @@ def resbm_device_error(clear=False) -> int:
 def resbm_selftest_wait_timeout(stream=None):
     """Enqueue the failure-path self-test kernel (a wait that gives up after ~2 s)."""
     _check("resbm_selftest_wait_timeout", load().resbm_selftest_wait_timeout(_stream(stream)))
+
+
+def resbm_measure_hbm_form(form, a, b, stream=None):
+    """One launch of an HBM access-form probe (resbm_hbm_form; a name of HBM_FORMS or its value)
+    over a's bytes: a read, b written; both device tensors of the same byte size."""
+    f = HBM_FORMS[form] if isinstance(form, str) else int(form)
+    n = _nbytes(a)
+    if _nbytes(b) != n:
+        raise ValueError("a and b must have the same byte size")
+    _check("resbm_measure_hbm_form", load().resbm_measure_hbm_form(f, _p(a), _p(b), n, _stream(stream)))
 
 
 def make_desc(T, d, r, m, dtype="bf16", act="silu", merge_identity=1, flags=0) -> resbm_desc:

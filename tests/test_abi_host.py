@@ -24,7 +24,7 @@ def declared_functions():
 
 def test_exports_every_declared_symbol(lib):
     names = declared_functions()
-    assert len(names) == 21, names
+    assert len(names) == 22, names
     assert sorted(resbm.EXPORTS) == names
     for n in names:
         assert hasattr(lib, n), n
@@ -253,3 +253,18 @@ def test_rmsnorm_bwd_rejects_bad_arguments(lib):
     sz = ctypes.c_size_t(0)
     assert lib.resbm_rmsnorm_bwd(ctypes.byref(wide), Y, g, 1e-5, dN, None, out, dg, ws, 1 << 30, None) == \
         resbm.RESBM_ERR_UNSUPPORTED
+
+
+def test_hbm_form_probe_rejects_bad_arguments(lib):
+    A, B = 1 << 40, (1 << 40) + (1 << 34)
+    mib = 1 << 20
+    fn = lib.resbm_measure_hbm_form
+    assert fn(-1, A, B, mib, None) == resbm.RESBM_ERR_INVALID_ARG
+    assert fn(len(resbm.HBM_FORMS), A, B, mib, None) == resbm.RESBM_ERR_INVALID_ARG
+    for bad in (0, mib - 16, mib + 16, -mib):
+        assert fn(resbm.RESBM_HBM_READ_TMA_2D, A, B, bad, None) == resbm.RESBM_ERR_INVALID_ARG
+    assert fn(resbm.RESBM_HBM_READ_V4, None, B, mib, None) == resbm.RESBM_ERR_INVALID_ARG
+    assert fn(resbm.RESBM_HBM_WRITE_V4, A, None, mib, None) == resbm.RESBM_ERR_INVALID_ARG
+    assert fn(resbm.RESBM_HBM_COPY_V4, A + 8, B, mib, None) == resbm.RESBM_ERR_INVALID_ARG   # misaligned
+    assert fn(resbm.RESBM_HBM_COPY_V4, A, A + mib // 2, mib, None) == resbm.RESBM_ERR_INVALID_ARG   # overlap
+    assert sorted(resbm.HBM_FORMS.values()) == list(range(11))

@@ -31,7 +31,8 @@ SMALL = {
     "bf16_no_compression": synth.BoundaryConfig("bf16_no_compression", T=200, d=64, r=64, m=16),
     "bf16_r1": synth.BoundaryConfig("bf16_r1", T=64, d=128, r=1, m=1),
     # ~1000 tokens per CTA: several groups of tiles per CTA in the backward kernels (whose
-    # grids on a 152-SM GB300 are 144 CTAs in clusters of 4)
+    # grids on a 152-SM GB300 are 144 CTAs in clusters of 4; the decoder backward's balanced grid
+    # keeps the most tiles per CTA on fewer clusters: 132 CTAs here)
     "bf16_multi_group": synth.BoundaryConfig("bf16_multi_group", T=150001, d=128, r=32, m=32),
     # 618 (585) tiles on 144 backward CTAs: 4 or 5 tiles per CTA, cut into 2 + 2 or 3 + 2, so
     # the CTAs of a cluster have different group sizes but the same number of groups
@@ -61,7 +62,9 @@ SMALL = {
 # Backward grids under each forced cluster size (RESBM_CLUSTER), one CTA per 128-token
 # tile at most: 8 tiles -> 8 CTAs in pairs or fours; 16 -> 16; 17 -> 16 in pairs or fours (one
 # idle SM); 18 -> 18 in pairs, no fours (16 < 15/16 x 18); 3 -> single CTAs (fours do not fit,
-# pairs leave too many idle); uneven tile groups inside clusters.
+# pairs leave too many idle); uneven tile groups inside clusters. The decoder backward then
+# shrinks that grid to the fewest clusters that keep its most tiles per CTA (17 tiles: 12 CTAs in
+# fours, two tiles each but one; test_decoder_backward_grid_rules_match_oracle runs both rules).
 CLUSTER_CASES = {
     "t8_r32": synth.BoundaryConfig("cl_t8_r32", T=1000, d=512, r=32, m=32),
     "t16_r32": synth.BoundaryConfig("cl_t16_r32", T=2000, d=384, r=32, m=32),
@@ -90,6 +93,23 @@ _ORACLE_CACHE = {}
 def test_forced_cluster_sizes_match_oracle(name, cluster, monkeypatch):
     """The backward kernels with every cluster size forced (1, 2, 4 CTAs), where it fits."""
     monkeypatch.setenv("RESBM_CLUSTER", cluster)
+    cfg = CLUSTER_CASES[name]
+    h = host_inputs(cfg)
+    dev = {k: to_dev(v, cfg) for k, v in h.items()}
+    got = gpu_step(cfg, dev)
+    if name not in _ORACLE_CACHE:
+        _ORACLE_CACHE[name] = oracle_step(cfg, h)
+    _compare_all(cfg, got, _ORACLE_CACHE[name], dev)
+    assert resbm.resbm_device_error() == 0
+
+
+@pytest.mark.parametrize("balance", ["0", "1"])
+@pytest.mark.parametrize("name", ["t321_r32", "uneven_r32"])
+def test_decoder_backward_grid_rules_match_oracle(name, balance, monkeypatch):
+    """The decoder backward on its balanced grid (the fewest clusters that keep the most tiles a
+    CTA gets: 321 tiles on 108 CTAs instead of 144, 618 on 124) and on the cluster rule's full
+    grid (RESBM_BWD_BALANCE=0): both against the oracle."""
+    monkeypatch.setenv("RESBM_BWD_BALANCE", balance)
     cfg = CLUSTER_CASES[name]
     h = host_inputs(cfg)
     dev = {k: to_dev(v, cfg) for k, v in h.items()}
