@@ -268,3 +268,12 @@ def test_hbm_form_probe_rejects_bad_arguments(lib):
     assert fn(resbm.RESBM_HBM_COPY_V4, A + 8, B, mib, None) == resbm.RESBM_ERR_INVALID_ARG   # misaligned
     assert fn(resbm.RESBM_HBM_COPY_V4, A, A + mib // 2, mib, None) == resbm.RESBM_ERR_INVALID_ARG   # overlap
     assert sorted(resbm.HBM_FORMS.values()) == list(range(11))
+
+
+def test_hbm_form_enum_matches_header():
+    src = open(os.path.join(ROOT, "include", "resbm.h")).read()
+    declared = {name: int(v) for name, v in re.findall(r"\bRESBM_HBM_(\w+)\s*=\s*(\d+)", src)}
+    assert len(declared) == len(resbm.HBM_FORMS) == 11
+    for name, v in declared.items():
+        assert getattr(resbm, "RESBM_HBM_" + name) == v, name
+        assert resbm.HBM_FORMS[name.lower()] == v, name
