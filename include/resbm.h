@@ -69,7 +69,7 @@ extern "C" {
 typedef enum {
     RESBM_OK = 0,
     RESBM_ERR_INVALID_ARG = 1,   /* null/misaligned pointer, bad size or enum, overlap */
-    RESBM_ERR_UNSUPPORTED = 2,   /* valid request this build cannot run */
+    RESBM_ERR_UNSUPPORTED = 2,   /* valid request the library does not run */
     RESBM_ERR_WORKSPACE = 3,     /* ws is NULL or smaller than resbm_workspace_bytes() */
     RESBM_ERR_CUDA = 4           /* a CUDA runtime call or launch failed */
 } resbm_status;
