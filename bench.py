@@ -606,9 +606,12 @@ def main():
         print(json.dumps(decode_rmsnorm_workload(resbm, torch, measured_peaks(), steps=max(args.steps, 1),
                                                  warmup=max(args.warmup, 0))), flush=True)
         return
-    if args.hbm_forms_only:
-        print(json.dumps(hbm_forms(resbm, torch, reps=max(args.steps, 1), warmup=max(args.warmup, 0),
-                                   sampler=ClockSampler())), flush=True)
+    if args.hbm_forms_only:   # one GPU's memory system: rank 0 alone measures and prints
+        if rank == 0:
+            print(json.dumps(hbm_forms(resbm, torch, reps=max(args.steps, 1), warmup=max(args.warmup, 0),
+                                       sampler=ClockSampler())), flush=True)
+        if dist:
+            dist.destroy_process_group()
         return
     if args.ffn_only:
         print(json.dumps(ffn_encode_workload(resbm, torch, steps=max(args.steps, 1), warmup=max(args.warmup, 0))),
