@@ -51,10 +51,6 @@ def _load(path=None):
     lib.oracle_dact.restype = ctypes.c_double
     lib.oracle_dact.argtypes = [ctypes.c_int, ctypes.c_double]
     lib.oracle_rect_identity.argtypes = [_i64, _i64, _dp]
-    lib.oracle_round_bf16.restype = ctypes.c_double
-    lib.oracle_round_bf16.argtypes = [ctypes.c_double]
-    lib.oracle_round_f32.restype = ctypes.c_double
-    lib.oracle_round_f32.argtypes = [ctypes.c_double]
     lib.oracle_round_array.argtypes = [ctypes.c_int, _i64, _dp]
     lib.oracle_pid.restype = ctypes.c_int
     lib.oracle_pid.argtypes = [_i64, _i64, _i64, _dp, _dp]

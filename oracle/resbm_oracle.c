@@ -171,9 +171,6 @@ static double round_significand(double x, int bits)
     return ldexp(r, e - bits);
 }
 
-double oracle_round_bf16(double x) { return round_significand(x, 8); }
-double oracle_round_f32(double x) { return round_significand(x, 24); }
-
 void oracle_round_array(int dtype_bits, int64_t n, double *x)
 {
     for (int64_t i = 0; i < n; ++i) x[i] = round_significand(x[i], dtype_bits);

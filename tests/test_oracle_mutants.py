@@ -37,6 +37,11 @@ MUTANTS = {
     "linear_decoder_bwd_transposed": ("mm_nt(T, r, d, dY, Wd, dB);              /* dB  = dY . Wd^T         */",
                                       "mm_nn(T, r, d, dY, Wd, dB);              /* dB  = dY . Wd^T         */"),
     "linear_encoder_bwd_drops_dX": ("return dX ? pid_backward(T, d, r, dB, dX) : 0;", "return 0;"),
+    "gelu_derivative_drops_factor_3": ("double du = kSqrt2OverPi * (1.0 + 3.0 * kGeluC * x * x);",
+                                       "double du = kSqrt2OverPi * (1.0 + kGeluC * x * x);"),
+    "gelu_derivative_tanh_sign": ("0.5 * x * (1.0 - th * th) * du", "0.5 * x * (1.0 + th * th) * du"),
+    "identity_derivative_zero": ("    return 1.0;\n}", "    return 0.0;\n}"),
+    "linear_decoder_drops_padded_skip": ("Y[i] = merge ? Pad[i] + L[i] : L[i];", "Y[i] = L[i];"),
 }
 
 
