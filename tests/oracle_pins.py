@@ -367,4 +367,18 @@ def pin_boundary_bytes(o):
     assert per_step * (B.size + dB.size) // 2 * e == g["compressed_step_bytes"]
 
 
+def pin_encoder_saves_the_preactivation(o):
+    """The saved P is F . We1 before phi (Sec. 3.2's encoder; the backward needs phi'(P)), by
+    brute-force loops on a tiny case with nonlinear phi, where P and phi(P) differ."""
+    T, d, r, m = 3, 5, 2, 4
+    X, F = _rand((T, d), 71), _rand((T, d), 72)
+    w = _weights(d, r, m, 73)
+    for act in ("silu", "gelu_tanh"):
+        _, P = o.encode_fwd(X, F, w["We1"], w["We2"], act)
+        for t in range(T):
+            for i in range(m):
+                want = sum(F[t, j] * w["We1"][j, i] for j in range(d))
+                assert abs(P[t, i] - want) <= 1e-13 * (1.0 + abs(want)), (act, t, i)
+
+
 PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_")]

@@ -42,6 +42,12 @@ MUTANTS = {
     "gelu_derivative_tanh_sign": ("0.5 * x * (1.0 - th * th) * du", "0.5 * x * (1.0 + th * th) * du"),
     "identity_derivative_zero": ("    return 1.0;\n}", "    return 0.0;\n}"),
     "linear_decoder_drops_padded_skip": ("Y[i] = merge ? Pad[i] + L[i] : L[i];", "Y[i] = L[i];"),
+    "encoder_saves_activation_for_P": ("if (P_out) memcpy(P_out, P,", "if (P_out) memcpy(P_out, A,"),
+    "decoder_gradient_from_Q_for_G": ("mm_tn(m, d, T, G, dY, dWd2);", "mm_tn(m, d, T, Q, dY, dWd2);"),
+    "encoder_gradient_from_P_for_A": ("mm_tn(m, r, T, A, dB, dWe2);", "mm_tn(m, r, T, P, dB, dWe2);"),
+    "decoder_skips_activation": ("apply_act(act, T * m, Q, G);\n        mm_nn(T, d, m, G, Wd2, D);",
+                                 "apply_act(act, T * m, Q, G);\n        mm_nn(T, d, m, Q, Wd2, D);"),
+    "rounding_ties_down": ("double r = nearbyint(scaled);", "double r = floor(scaled);"),
 }
 
 
