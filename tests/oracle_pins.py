@@ -345,6 +345,22 @@ def pin_step_hands_over_rounded_tensors(o):
     np.testing.assert_array_equal(s["dF"], o.encode_bwd(o.round_to(dB, "bf16"), F, w["We1"], w["We2"])[0])
 
 
+
+def pin_linear_step_hands_over_rounded_tensors(o):
+    """The one-linear-layer step with bf16 transfer: the decoder sees the bf16 value of B and the
+    encoder backward the bf16 value of dB, as in the two-layer step."""
+    T, d, r = 5, 16, 4
+    X, F, dY = _rand((T, d), 121), _rand((T, d), 122), _rand((T, d), 123)
+    We, Wd = _rand((d, r), 124, 0.25), _rand((r, d), 125, 0.5)
+    s = o.linear_boundary_step(X, F, dY, We, Wd, transfer="bf16")
+    Bq = o.round_to(o.linear_encode_fwd(X, F, We), "bf16")
+    assert np.array_equal(s["B"], Bq)
+    np.testing.assert_array_equal(s["Y"], o.linear_decode_fwd(Bq, Wd))
+    dB, _ = o.linear_decode_bwd(dY, Bq, Wd)
+    dBq = o.round_to(dB, "bf16")
+    assert np.array_equal(s["dB"], dBq) and not np.array_equal(dBq, dB)
+    np.testing.assert_array_equal(s["dF"], o.linear_encode_bwd(dBq, F, We)[0])
+
 # ---------------------------------------------------------------------------------------------
 # Appendix A.3 / Sec. 4.1: what crosses the boundary.
 # ---------------------------------------------------------------------------------------------

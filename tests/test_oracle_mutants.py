@@ -69,3 +69,53 @@ def test_planted_mistake_is_caught(name):
             except AssertionError:
                 caught.append(pin.__name__)
         assert caught, "no pin caught the planted mistake %s" % name
+
+
+# Planted mistakes in the Python side of the oracle (the methods that chain the C functions and
+# round what crosses the boundary): a copy of one method, changed, on a subclass.
+PY_MUTANTS = {
+    "step_B_not_rounded": ("boundary_step", "B = self.round_to(B, transfer)", "B = B"),
+    "step_dB_not_rounded": ("boundary_step", "dB = self.round_to(dB, transfer)", "dB = dB"),
+    "step_decoder_reads_unrounded_B": ("boundary_step", "B = self.round_to(B, transfer)\n",
+                                       "Bq = self.round_to(B, transfer)\n"),
+    "step_forward_merge_flipped": ("boundary_step", "Y = self.decode_fwd(B, Wd1, Wd2, act, merge)",
+                                   "Y = self.decode_fwd(B, Wd1, Wd2, act, 1 - merge)"),
+    "step_backward_merge_flipped": ("boundary_step", "dB, dWd1, dWd2 = self.decode_bwd(dY, B, Wd1, Wd2, act, merge)",
+                                    "dB, dWd1, dWd2 = self.decode_bwd(dY, B, Wd1, Wd2, act, 1 - merge)"),
+    "linear_step_B_not_rounded": ("linear_boundary_step", "B = self.round_to(B, transfer)", "B = B"),
+    "linear_step_dB_not_rounded": ("linear_boundary_step", "dB = self.round_to(dB, transfer)", "dB = dB"),
+    "linear_step_merge_flipped": ("linear_boundary_step", "Y = self.linear_decode_fwd(B, Wd, merge)",
+                                  "Y = self.linear_decode_fwd(B, Wd, 1 - merge)"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(PY_MUTANTS))
+def test_planted_mistake_in_python_oracle_is_caught(name):
+    import inspect
+    import textwrap
+    method, find, repl = PY_MUTANTS[name]
+    src = textwrap.dedent(inspect.getsource(getattr(oracle.Oracle, method)))
+    assert src.count(find) == 1, "mutation anchor not unique: %s" % name
+    ns = dict(vars(oracle))
+    exec(compile(src.replace(find, repl), "<mutant %s>" % name, "exec"), ns)
+    o = type("MutantOracle", (oracle.Oracle,), {method: ns[method]})()
+    caught = []
+    for pin in PINS:
+        try:
+            pin(o)
+        except AssertionError:
+            caught.append(pin.__name__)
+    assert caught, "no pin caught the planted mistake %s" % name
+
+
+def test_transfer_width_mistake_is_caught():
+    """fp32 transfer rounding to 23 significant bits instead of 24."""
+    o = type("MutantOracle", (oracle.Oracle,), {"_BITS": {"bf16": 8, "f32": 23}})()
+    caught = []
+    for pin in PINS:
+        try:
+            pin(o)
+        except AssertionError:
+            caught.append(pin.__name__)
+    assert caught
+
