@@ -57,28 +57,66 @@ def test_oracle_rmsnorm_pins(pin):
     pin(oracle.rmsnorm)
 
 
-def test_decoder_with_zero_second_layer_normalises_the_padded_identity_path():
+def dpin_zero_second_layer_normalises_the_padded_identity_path(fn):
     """Wd2 = 0, merge = 1: Y = pad(B) exactly, so N's first r columns are B / sqrt(sum_j B_j^2 / d
-    + eps) * gamma (the mean runs over all d columns, d - r of them zero) and the rest zero."""
+    + eps) * gamma (the mean runs over all d columns, d - r of them zero) and the rest zero;
+    merge = 0: Y = 0 and N = 0."""
     rng = np.random.default_rng(7)
     T, d, r, m = 5, 24, 4, 6
     B = rng.standard_normal((T, r))
+    Wd1 = rng.standard_normal((r, m))
     g = rng.standard_normal(d)
-    Y, N = oracle.decode_fwd_rmsnorm(B, rng.standard_normal((r, m)), np.zeros((m, d)), g, 0.5)
+    Y, N = fn(B, Wd1, np.zeros((m, d)), g, 0.5)
     assert np.array_equal(Y[:, :r], B) and not np.any(Y[:, r:])
     want = B / np.sqrt(np.sum(B * B, axis=1, keepdims=True) / d + 0.5) * g[:r]
     assert np.allclose(N[:, :r], want, rtol=1e-14) and not np.any(N[:, r:])
+    Y0, N0 = fn(B, Wd1, np.zeros((m, d)), g, 0.5, merge=0)
+    assert not np.any(Y0) and not np.any(N0)
 
 
-def test_store_rounding_is_applied_before_the_norm():
+def dpin_store_rounding_is_applied_before_the_norm(fn):
+    """store = "bf16": N is the norm of the bf16 value of Y, and the Y returned is the exact one."""
     rng = np.random.default_rng(8)
     T, d, r, m = 7, 32, 8, 8
     args = (rng.standard_normal((T, r)), rng.standard_normal((r, m)), rng.standard_normal((m, d)) / 3)
     g = rng.standard_normal(d)
-    Y, N = oracle.decode_fwd_rmsnorm(*args, g, 1e-5, store="bf16")
+    Y, N = fn(*args, g, 1e-5, store="bf16")
+    assert np.array_equal(Y, oracle.decode_fwd(*args, "silu", 1))
     Yb = oracle.round_to(Y, "bf16")
     assert np.array_equal(N, oracle.rmsnorm(Yb, g, 1e-5))
     assert not np.array_equal(N, oracle.rmsnorm(Y, g, 1e-5))
+
+
+DPINS = [dpin_zero_second_layer_normalises_the_padded_identity_path, dpin_store_rounding_is_applied_before_the_norm]
+
+
+@pytest.mark.parametrize("pin", DPINS, ids=lambda p: p.__name__)
+def test_oracle_decode_fwd_rmsnorm_pins(pin):
+    pin(oracle.decode_fwd_rmsnorm)
+
+
+DMUTANTS = {
+    "store_ignored": ("Ys = default().round_to(Y, store) if store else Y", "Ys = Y"),
+    "returns_the_stored_Y": ("return Y, rmsnorm(Ys, gamma, eps)", "return Ys, rmsnorm(Ys, gamma, eps)"),
+    "merge_ignored": ("default().decode_fwd(B, Wd1, Wd2, act, merge)", "default().decode_fwd(B, Wd1, Wd2, act, 1)"),
+    "norm_of_the_exact_Y": ("return Y, rmsnorm(Ys, gamma, eps)", "return Y, rmsnorm(Y, gamma, eps)"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(DMUTANTS))
+def test_planted_mistake_in_decode_fwd_rmsnorm_is_caught(name):
+    find, repl = DMUTANTS[name]
+    src = textwrap.dedent(inspect.getsource(oracle.decode_fwd_rmsnorm))
+    assert src.count(find) == 1, name
+    ns = {"np": np, "default": oracle.default, "rmsnorm": oracle.rmsnorm}
+    exec(compile(src.replace(find, repl), "<mutant %s>" % name, "exec"), ns)
+    caught = []
+    for pin in DPINS:
+        try:
+            pin(ns["decode_fwd_rmsnorm"])
+        except (AssertionError, ValueError, IndexError):
+            caught.append(pin.__name__)
+    assert caught, "no pin caught the planted mistake %s" % name
 
 
 MUTANTS = {
