@@ -48,6 +48,11 @@ MUTANTS = {
     "decoder_skips_activation": ("apply_act(act, T * m, Q, G);\n        mm_nn(T, d, m, G, Wd2, D);",
                                  "apply_act(act, T * m, Q, G);\n        mm_nn(T, d, m, Q, Wd2, D);"),
     "rounding_ties_down": ("double r = nearbyint(scaled);", "double r = floor(scaled);"),
+    "rounding_skips_small_magnitudes": ("if (x == 0.0 || !isfinite(x)) return x;",
+                                        "if (x == 0.0 || !isfinite(x) || fabs(x) < 1.0) return x;"),
+    "nn_product_drops_last_k": ("        for (int64_t k = 0; k < K; ++k) {\n            const double a = A[i * K + k];",
+                                "        for (int64_t k = 0; k < K - 1; ++k) {\n            const double a = A[i * K + k];"),
+    "identity_backward_not_transposed": ("mm_nt(L, c, C, dy, I, dx);", "mm_nn(L, c, C, dy, I, dx);"),
 }
 
 
